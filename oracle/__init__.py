@@ -1,0 +1,211 @@
+"""fp64 CPU oracle for RLA / RDN (arXiv 2509.25223), Section 3.4.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+the CPU-baseline / reference leg of ``bench.py`` may import this package.
+The product library (``paper_2509_25223_gb300``) never imports it and shares
+no code with it; the two meet only in the seeded input generator
+(``rdn_synthetic``), which holds none of the method's arithmetic.
+
+The arithmetic lives in ``rdn_oracle.c``: the paper's token recurrence
+(Section 3.4, "Final Formulations"; clipping Section 3.3) written out one token
+at a time in double precision, plus hand-written back-propagation through
+time.  This module compiles it with gcc (``build()``) and wraps it with ctypes.
+All arrays are numpy float64, C-contiguous, in the layouts
+
+    q, k [B,T,H,Dk]   v, o [B,T,H,Dv]   g, beta, gamma [B,T,H]
+    S0, R0, ST, RT [B,H,Dk,Dv]
+
+where g = log(alpha) is the per-token log-decay and the states are stored
+[d_k][d_v] (the paper's d_v x d_k matrices, transposed).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "rdn_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+RLA, RDN = 0, 1
+
+
+def build(force: bool = False) -> str:
+    """Compile rdn_oracle.c into oracle/_build/liboracle.so (gcc, OpenMP).
+
+    -ffp-contract=off keeps x86_64 and aarch64 results bit-identical."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < os.path.getmtime(_SRC):
+        tmp = _SO + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O3", "-ffp-contract=off", "-fopenmp", "-fPIC", "-shared",
+               "-std=c11", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _SO)
+    return _SO
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I = ctypes.c_int
+            D = ctypes.c_double
+            fwd_sig = [I, I, I, I, I, P, P, P, P, P, P, D, D, P, P, P, P, P]
+            for name in ("orc_rla_fwd", "orc_rdn_fwd"):
+                getattr(lib, name).argtypes = fwd_sig
+                getattr(lib, name).restype = None
+            lib.orc_fwd_with_residual.argtypes = [I] + fwd_sig + [P]
+            lib.orc_fwd_with_residual.restype = None
+            bwd_sig = [I, I, I, I, I, P, P, P, P, P, P, D, D, P, P, P, P, P,
+                       P, P, P, P, P, P, P, P]
+            for name in ("orc_rla_bwd", "orc_rdn_bwd"):
+                getattr(lib, name).argtypes = bwd_sig
+                getattr(lib, name).restype = None
+            lib.orc_decode_step.argtypes = [I, I, I, I, I, P, P, P, P, P, P, D, D, P, P, P]
+            lib.orc_decode_step.restype = None
+            lib.orc_clip_margin_condition.argtypes = [I, I, I, I, I, I, P, P, P, P, P, P,
+                                                      D, D, P, P, D, I]
+            lib.orc_clip_margin_condition.restype = ctypes.c_long
+            lib.orc_max_threads.restype = I
+            lib.orc_set_threads.argtypes = [I]
+            _lib = lib
+    return _lib
+
+
+def _f64(x):
+    if x is None:
+        return None
+    if hasattr(x, "detach"):  # torch tensor
+        x = x.detach().cpu().double().numpy()
+    return np.ascontiguousarray(x, dtype=np.float64)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def max_threads() -> int:
+    return _load().orc_max_threads()
+
+
+def set_threads(n: int) -> None:
+    _load().orc_set_threads(int(n))
+
+
+def _dims(q, v):
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    return B, T, H, Dk, Dv
+
+
+def fwd(variant, q, k, v, g, beta, gamma, c=1.0, S0=None, R0=None, scale=1.0,
+        return_residual=False):
+    """Forward of RLA (variant=RLA) or RDN (variant=RDN).
+
+    Returns (o, ST, RT) as float64 arrays, plus r (the clipped residuals,
+    [B,T,H,Dv]) when return_residual is set."""
+    lib = _load()
+    q, k, v, g, beta, gamma = map(_f64, (q, k, v, g, beta, gamma))
+    S0, R0 = _f64(S0), _f64(R0)
+    B, T, H, Dk, Dv = _dims(q, v)
+    o = np.zeros((B, T, H, Dv))
+    ST = np.zeros((B, H, Dk, Dv))
+    RT = np.zeros((B, H, Dk, Dv))
+    args = (B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta),
+            _ptr(gamma), float(c), float(scale), _ptr(S0), _ptr(R0), _ptr(o),
+            _ptr(ST), _ptr(RT))
+    if return_residual:
+        r = np.zeros((B, T, H, Dv))
+        lib.orc_fwd_with_residual(int(variant), *args, _ptr(r))
+        return o, ST, RT, r
+    (lib.orc_rdn_fwd if variant == RDN else lib.orc_rla_fwd)(*args)
+    return o, ST, RT
+
+
+def rdn_fwd(*a, **kw):
+    """RDN forward (Section 3.4, right formulation)."""
+    return fwd(RDN, *a, **kw)
+
+
+def rla_fwd(*a, **kw):
+    """RLA forward (Section 3.4, left formulation)."""
+    return fwd(RLA, *a, **kw)
+
+
+def bwd(variant, q, k, v, g, beta, gamma, c, S0, R0, dO, dST=None, dRT=None,
+        scale=1.0):
+    """Back-propagation through time of the forward above.
+
+    Returns a dict with dq, dk, dv, dg (w.r.t. the log-decay g), dbeta,
+    dgamma, dS0, dR0 (float64)."""
+    lib = _load()
+    q, k, v, g, beta, gamma, dO = map(_f64, (q, k, v, g, beta, gamma, dO))
+    S0, R0, dST, dRT = map(_f64, (S0, R0, dST, dRT))
+    B, T, H, Dk, Dv = _dims(q, v)
+    out = dict(dq=np.zeros((B, T, H, Dk)), dk=np.zeros((B, T, H, Dk)),
+               dv=np.zeros((B, T, H, Dv)), dg=np.zeros((B, T, H)),
+               dbeta=np.zeros((B, T, H)), dgamma=np.zeros((B, T, H)),
+               dS0=np.zeros((B, H, Dk, Dv)), dR0=np.zeros((B, H, Dk, Dv)))
+    fn = lib.orc_rdn_bwd if variant == RDN else lib.orc_rla_bwd
+    fn(B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta),
+       _ptr(gamma), float(c), float(scale), _ptr(S0), _ptr(R0), _ptr(dO),
+       _ptr(dST), _ptr(dRT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]),
+       _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"]),
+       _ptr(out["dS0"]), _ptr(out["dR0"]))
+    return out
+
+
+def rdn_bwd(*a, **kw):
+    return bwd(RDN, *a, **kw)
+
+
+def rla_bwd(*a, **kw):
+    return bwd(RLA, *a, **kw)
+
+
+def decode_step(variant, q, k, v, g, beta, gamma, c, S, R, scale=1.0):
+    """One recurrent step for N independent sequences.
+
+    q, k [N,H,Dk]; v [N,H,Dv]; gates [N,H]; S, R [N,H,Dk,Dv].
+    Returns (o [N,H,Dv], S_new, R_new); the inputs are not modified."""
+    lib = _load()
+    q, k, v, g, beta, gamma = map(_f64, (q, k, v, g, beta, gamma))
+    S = _f64(S).copy()
+    R = _f64(R).copy()
+    N, H, Dk = q.shape
+    Dv = v.shape[-1]
+    o = np.zeros((N, H, Dv))
+    lib.orc_decode_step(int(variant), N, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v),
+                        _ptr(g), _ptr(beta), _ptr(gamma), float(c), float(scale),
+                        _ptr(S), _ptr(R), _ptr(o))
+    return o, S, R
+
+
+QUANT = {"f64": 0, "f32": 1, "bf16": 2}
+
+
+def clip_margin_condition(variant, q, k, v, g, beta, gamma, c, S0=None, R0=None,
+                          scale=1.0, margin=4e-3, quant="bf16"):
+    """Return (v_conditioned, n_moved): v moved, in token order and in steps
+    representable in `quant`, so that every |v - S_{t-1}k| of the fp64
+    forward is at least `margin` away from the clip threshold c.  Makes the
+    clip mask, and so the backward, unique at tolerance level."""
+    lib = _load()
+    q, k, g, beta, gamma = map(_f64, (q, k, g, beta, gamma))
+    v = _f64(v).copy()
+    S0, R0 = _f64(S0), _f64(R0)
+    B, T, H, Dk, Dv = _dims(q, v)
+    n = lib.orc_clip_margin_condition(int(variant), B, T, H, Dk, Dv, _ptr(q), _ptr(k),
+                                      _ptr(v), _ptr(g), _ptr(beta), _ptr(gamma),
+                                      float(c), float(scale), _ptr(S0), _ptr(R0),
+                                      float(margin), QUANT[quant])
+    return v, int(n)

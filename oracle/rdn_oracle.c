@@ -1,0 +1,548 @@
+/*
+ * rdn_oracle.c -- fp64 CPU oracle for Residual Linear Attention (RLA) and
+ * Residual Delta Net (RDN), arXiv 2509.25223.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path links, loads or
+ * calls this file: only tests/, __graft_entry__.smoke() and bench.py's CPU
+ * baseline leg use it.  It shares no code, header or constant with the CUDA
+ * library.
+ *
+ * What it computes is the paper's token recurrence written out directly, one
+ * token at a time, in double precision (Section 3.4, "Final Formulations",
+ * RLA left and RDN right; clipping from Section 3.3; gates from Section 3.2):
+ *
+ *   r_t = Clip_[-c,c](v_t - S_{t-1} k_t)                        (elementwise)
+ *   RLA: R_t = a_t R_{t-1} + g_t r_t k_t^T
+ *        S_t = a_t S_{t-1} + b_t v_t k_t^T
+ *   RDN: R_t = a_t R_{t-1} (I - g_t k_t k_t^T) + g_t r_t k_t^T
+ *        S_t = a_t S_{t-1} (I - b_t k_t k_t^T) + b_t v_t k_t^T
+ *   o_t = a_t S_{t-1} q_t + g_t R_t q_t
+ *
+ * (a = alpha = exp(log-decay), b = beta, g = gamma.)  The paper writes the
+ * states as d_v x d_k matrices; this file stores them transposed, as
+ * [d_k][d_v] row-major, so "S k" is sum_i k_i S[i][j].  That is a transpose
+ * of storage only.
+ *
+ * Readings taken where the paper leaves room (each listed in the design doc):
+ *  - the residual uses the undecayed S_{t-1} k_t (Section 3.3 and 3.4),
+ *    not a_t S_{t-1} k_t;
+ *  - the output uses S_{t-1} (before the update) and R_t (after it);
+ *  - the Appendix B recurrence's minus signs and fixed +-1 bound are read as
+ *    "+" and a general threshold c;
+ *  - clamp(x,-c,c) = min(max(x,-c),c); its derivative is 1 on |x| <= c
+ *    (the tie |x| == c passes the gradient through);
+ *  - q is multiplied by `scale` (the paper uses 1, i.e. no 1/sqrt(d)).
+ *
+ * The backward is hand-written reverse-mode through the same token loop
+ * (back-propagation through time), with the states re-computed from
+ * checkpoints taken every ORC_CKPT tokens.  The paper has no backward; it is
+ * pinned by finite differences and by fp64 autograd in the tests.
+ *
+ * Layouts (all contiguous, row-major):
+ *   q,k [B,T,H,Dk]   v,o [B,T,H,Dv]   g,beta,gamma [B,T,H]
+ *   S0,R0,ST,RT [B,H,Dk,Dv]          (S0/R0 may be NULL = zeros;
+ *                                      ST/RT may be NULL = not returned)
+ * One (b,h) pair is an independent problem; OpenMP runs them in parallel.
+ */
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORC_CKPT 64
+
+enum { ORC_RLA = 0, ORC_RDN = 1 };
+
+static double clampd(double x, double c) {
+  if (x < -c) return -c;
+  if (x > c) return c;
+  return x;
+}
+
+int orc_max_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+void orc_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+#else
+  (void)n;
+#endif
+}
+
+/* One token of the recurrence for one (b,h).  S,R [Dk][Dv] are updated in
+ * place; o[Dv] receives the output.  p, rk are scratch of length Dv.
+ * Returns nothing; r (length Dv, may be NULL) receives the clipped residual. */
+static void token_step(int variant, int Dk, int Dv, const double *q,
+                       const double *k, const double *v, double alpha,
+                       double beta, double gamma, double c, double scale,
+                       double *S, double *R, double *o, double *p, double *rk,
+                       double *r_out) {
+  /* base read-outs against the state before the update: p = S_{t-1} k and
+     sq = S_{t-1} q (kept in o until the end) */
+  for (int j = 0; j < Dv; ++j) {
+    double pj = 0.0, sqj = 0.0, rkj = 0.0;
+    for (int i = 0; i < Dk; ++i) {
+      pj += k[i] * S[i * Dv + j];
+      sqj += scale * q[i] * S[i * Dv + j];
+      rkj += k[i] * R[i * Dv + j];
+    }
+    p[j] = pj;
+    o[j] = alpha * sqj; /* base prediction a_t S_{t-1} q_t */
+    rk[j] = rkj;
+  }
+  for (int j = 0; j < Dv; ++j) {
+    double rj = clampd(v[j] - p[j], c); /* Section 3.3 */
+    if (r_out) r_out[j] = rj;
+    /* auxiliary state update */
+    for (int i = 0; i < Dk; ++i) {
+      double Rij = R[i * Dv + j];
+      if (variant == ORC_RDN)
+        R[i * Dv + j] = alpha * Rij - alpha * gamma * k[i] * rk[j] + gamma * k[i] * rj;
+      else
+        R[i * Dv + j] = alpha * Rij + gamma * k[i] * rj;
+    }
+    /* base state update */
+    for (int i = 0; i < Dk; ++i) {
+      double Sij = S[i * Dv + j];
+      if (variant == ORC_RDN)
+        S[i * Dv + j] = alpha * Sij - alpha * beta * k[i] * p[j] + beta * k[i] * v[j];
+      else
+        S[i * Dv + j] = alpha * Sij + beta * k[i] * v[j];
+    }
+  }
+  /* correction read-out against the updated auxiliary state R_t */
+  for (int j = 0; j < Dv; ++j) {
+    double aq = 0.0;
+    for (int i = 0; i < Dk; ++i) aq += scale * q[i] * R[i * Dv + j];
+    o[j] += gamma * aq;
+  }
+}
+
+static void fwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
+                     const double *q, const double *k, const double *v,
+                     const double *g, const double *beta, const double *gamma,
+                     double c, double scale, const double *S0, const double *R0,
+                     double *o, double *ST, double *RT, double *r_all) {
+  const long SD = (long)Dk * Dv;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long bh = 0; bh < (long)B * H; ++bh) {
+    const long b = bh / H, h = bh % H;
+    double *S = (double *)malloc(sizeof(double) * SD);
+    double *R = (double *)malloc(sizeof(double) * SD);
+    double *p = (double *)malloc(sizeof(double) * Dv);
+    double *rk = (double *)malloc(sizeof(double) * Dv);
+    if (S0) memcpy(S, S0 + bh * SD, sizeof(double) * SD); else memset(S, 0, sizeof(double) * SD);
+    if (R0) memcpy(R, R0 + bh * SD, sizeof(double) * SD); else memset(R, 0, sizeof(double) * SD);
+    for (long t = 0; t < T; ++t) {
+      const long tok = (b * T + t) * H + h; /* index into [B,T,H] */
+      token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+                 exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R,
+                 o + tok * Dv, p, rk, r_all ? r_all + tok * Dv : NULL);
+    }
+    if (ST) memcpy(ST + bh * SD, S, sizeof(double) * SD);
+    if (RT) memcpy(RT + bh * SD, R, sizeof(double) * SD);
+    free(S); free(R); free(p); free(rk);
+  }
+}
+
+/* RLA forward (Section 3.4, left formulation). */
+void orc_rla_fwd(int B, int T, int H, int Dk, int Dv, const double *q,
+                 const double *k, const double *v, const double *g,
+                 const double *beta, const double *gamma, double c,
+                 double scale, const double *S0, const double *R0, double *o,
+                 double *ST, double *RT) {
+  fwd_impl(ORC_RLA, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           o, ST, RT, NULL);
+}
+
+/* RDN forward (Section 3.4, right formulation). */
+void orc_rdn_fwd(int B, int T, int H, int Dk, int Dv, const double *q,
+                 const double *k, const double *v, const double *g,
+                 const double *beta, const double *gamma, double c,
+                 double scale, const double *S0, const double *R0, double *o,
+                 double *ST, double *RT) {
+  fwd_impl(ORC_RDN, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           o, ST, RT, NULL);
+}
+
+/* Forward that also returns the clipped residuals r [B,T,H,Dv]
+ * (variant 0 = RLA, 1 = RDN).  Used by tests of the residual itself. */
+void orc_fwd_with_residual(int variant, int B, int T, int H, int Dk, int Dv,
+                           const double *q, const double *k, const double *v,
+                           const double *g, const double *beta,
+                           const double *gamma, double c, double scale,
+                           const double *S0, const double *R0, double *o,
+                           double *ST, double *RT, double *r) {
+  fwd_impl(variant, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           o, ST, RT, r);
+}
+
+/* One decode step: the same token recurrence applied to N independent
+ * sequences, states [N,H,Dk,Dv] updated in place; q,k [N,H,Dk], v,o [N,H,Dv],
+ * gates [N,H].  variant 0 = RLA, 1 = RDN. */
+void orc_decode_step(int variant, int N, int H, int Dk, int Dv, const double *q,
+                     const double *k, const double *v, const double *g,
+                     const double *beta, const double *gamma, double c,
+                     double scale, double *S, double *R, double *o) {
+  const long SD = (long)Dk * Dv;
+#pragma omp parallel for schedule(static)
+  for (long nh = 0; nh < (long)N * H; ++nh) {
+    double *p = (double *)malloc(sizeof(double) * Dv);
+    double *rk = (double *)malloc(sizeof(double) * Dv);
+    token_step(variant, Dk, Dv, q + nh * Dk, k + nh * Dk, v + nh * Dv,
+               exp(g[nh]), beta[nh], gamma[nh], c, scale, S + nh * SD,
+               R + nh * SD, o + nh * Dv, p, rk, NULL);
+    free(p); free(rk);
+  }
+}
+
+/* ------------------------------------------------------------------------ *
+ * Backward (reverse-mode through the token loop).
+ *
+ * Given dO [B,T,H,Dv] and optional dST, dRT (NULL = 0), produce
+ * dq, dk [B,T,H,Dk], dv [B,T,H,Dv], dg, dbeta, dgamma [B,T,H] and
+ * (optional) dS0, dR0 [B,H,Dk,Dv].  dg is the gradient with respect to the
+ * log-decay g = log(alpha); d/dalpha = dg / alpha.
+ *
+ * Per token, with a = alpha, p = S_{t-1}k, x = v - p, r = clip(x),
+ * e = v - a p (delta error of S), rk = R_{t-1}k, e2 = r - a rk (RDN), and
+ * carried dS' = dL/dS_t, dR' = dL/dR_t:
+ *   output:  da += dO.(S_{t-1}q);  dgam += dO.(R_t q);
+ *            dq += a S_{t-1}^T dO + gam R_t^T dO;
+ *            dS += a q dO^T;  dR' += gam q dO^T
+ *   R-step:  u = dR'^T k;  RDN: R_t = a R + gam k e2^T
+ *            da += <dR',R> - gam u.rk;  dgam += u.e2;  dr = gam u;
+ *            dk += gam dR' e2 - a gam R u;  dR = a dR' - a gam k u^T
+ *            RLA: R_t = a R + gam k r^T: da += <dR',R>; dgam += u.r;
+ *            dr = gam u; dk += gam dR' r; dR = a dR'
+ *   clip:    dx = dr * [|x| <= c];  dv += dx;  dp = -dx
+ *   S-step:  w = dS'^T k;  RDN: S_t = a S + b k e^T
+ *            da += <dS',S> - b w.p;  db += w.e;  dv += b w;  dp -= a b w;
+ *            dk += b dS' e;  dS += a dS'
+ *            RLA: S_t = a S + b k v^T: da += <dS',S>; db += w.v;
+ *            dv += b w; dk += b dS' v; dS += a dS'
+ *   p = S^T k: dk += S dp;  dS += k dp^T
+ *   dg = a * da.
+ * ------------------------------------------------------------------------ */
+static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
+                     const double *q, const double *k, const double *v,
+                     const double *g, const double *beta, const double *gamma,
+                     double c, double scale, const double *S0,
+                     const double *R0, const double *dO, const double *dST,
+                     const double *dRT, double *dq, double *dk, double *dv,
+                     double *dg, double *dbeta, double *dgamma, double *dS0,
+                     double *dR0) {
+  const long SD = (long)Dk * Dv;
+  const int nck = (T + ORC_CKPT - 1) / ORC_CKPT;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (long bh = 0; bh < (long)B * H; ++bh) {
+    const long b = bh / H, h = bh % H;
+    /* checkpoints of (S,R) at the start of every segment */
+    double *ckS = (double *)malloc(sizeof(double) * SD * nck);
+    double *ckR = (double *)malloc(sizeof(double) * SD * nck);
+    /* states before every token of the current segment */
+    double *segS = (double *)malloc(sizeof(double) * SD * ORC_CKPT);
+    double *segR = (double *)malloc(sizeof(double) * SD * ORC_CKPT);
+    double *S = (double *)malloc(sizeof(double) * SD);
+    double *R = (double *)malloc(sizeof(double) * SD);
+    double *dS = (double *)malloc(sizeof(double) * SD);
+    double *dR = (double *)malloc(sizeof(double) * SD);
+    double *dSp = (double *)malloc(sizeof(double) * SD);
+    double *dRp = (double *)malloc(sizeof(double) * SD);
+    double *p = (double *)malloc(sizeof(double) * Dv);
+    double *rk = (double *)malloc(sizeof(double) * Dv);
+    double *ob = (double *)malloc(sizeof(double) * Dv);
+    double *Rt = (double *)malloc(sizeof(double) * SD);
+    double *u = (double *)malloc(sizeof(double) * Dv);
+    double *w = (double *)malloc(sizeof(double) * Dv);
+    double *dp = (double *)malloc(sizeof(double) * Dv);
+    double *r = (double *)malloc(sizeof(double) * Dv);
+
+    if (S0) memcpy(S, S0 + bh * SD, sizeof(double) * SD); else memset(S, 0, sizeof(double) * SD);
+    if (R0) memcpy(R, R0 + bh * SD, sizeof(double) * SD); else memset(R, 0, sizeof(double) * SD);
+    /* forward pass storing segment checkpoints */
+    for (int sgi = 0; sgi < nck; ++sgi) {
+      memcpy(ckS + sgi * SD, S, sizeof(double) * SD);
+      memcpy(ckR + sgi * SD, R, sizeof(double) * SD);
+      const int t0 = sgi * ORC_CKPT, t1 = t0 + ORC_CKPT < T ? t0 + ORC_CKPT : T;
+      for (int t = t0; t < t1; ++t) {
+        const long tok = (b * T + t) * H + h;
+        token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+                   exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R, ob, p,
+                   rk, NULL);
+      }
+    }
+    if (dST) memcpy(dS, dST + bh * SD, sizeof(double) * SD); else memset(dS, 0, sizeof(double) * SD);
+    if (dRT) memcpy(dR, dRT + bh * SD, sizeof(double) * SD); else memset(dR, 0, sizeof(double) * SD);
+
+    for (int sgi = nck - 1; sgi >= 0; --sgi) {
+      const int t0 = sgi * ORC_CKPT, t1 = t0 + ORC_CKPT < T ? t0 + ORC_CKPT : T;
+      /* recompute the states before each token of the segment */
+      memcpy(S, ckS + sgi * SD, sizeof(double) * SD);
+      memcpy(R, ckR + sgi * SD, sizeof(double) * SD);
+      for (int t = t0; t < t1; ++t) {
+        const long tok = (b * T + t) * H + h;
+        memcpy(segS + (t - t0) * SD, S, sizeof(double) * SD);
+        memcpy(segR + (t - t0) * SD, R, sizeof(double) * SD);
+        token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+                   exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R, ob, p,
+                   rk, NULL);
+      }
+      for (int t = t1 - 1; t >= t0; --t) {
+        const long tok = (b * T + t) * H + h;
+        const double *Sp = segS + (t - t0) * SD; /* S_{t-1} */
+        const double *Rp = segR + (t - t0) * SD; /* R_{t-1} */
+        const double *qt = q + tok * Dk, *kt = k + tok * Dk, *vt = v + tok * Dv;
+        const double *dOt = dO + tok * Dv;
+        const double a = exp(g[tok]), bb = beta[tok], gm = gamma[tok];
+        double da = 0.0, db = 0.0, dgm = 0.0;
+        double *dqt = dq + tok * Dk, *dkt = dk + tok * Dk, *dvt = dv + tok * Dv;
+        for (int i = 0; i < Dk; ++i) { dqt[i] = 0.0; dkt[i] = 0.0; }
+        for (int j = 0; j < Dv; ++j) dvt[j] = 0.0;
+
+        /* recompute p, rk, r and R_t for this token */
+        for (int j = 0; j < Dv; ++j) {
+          double pj = 0.0, rkj = 0.0;
+          for (int i = 0; i < Dk; ++i) {
+            pj += kt[i] * Sp[i * Dv + j];
+            rkj += kt[i] * Rp[i * Dv + j];
+          }
+          p[j] = pj; rk[j] = rkj;
+          r[j] = clampd(vt[j] - pj, c);
+        }
+        for (int i = 0; i < Dk; ++i)
+          for (int j = 0; j < Dv; ++j) {
+            const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
+            Rt[i * Dv + j] = a * Rp[i * Dv + j] + gm * kt[i] * e2;
+          }
+
+        /* output o = a S_{t-1} q + gam R_t q (q scaled) */
+        for (int j = 0; j < Dv; ++j) {
+          double sq = 0.0, rq = 0.0;
+          for (int i = 0; i < Dk; ++i) {
+            sq += scale * qt[i] * Sp[i * Dv + j];
+            rq += scale * qt[i] * Rt[i * Dv + j];
+          }
+          da += dOt[j] * sq;
+          dgm += dOt[j] * rq;
+        }
+        for (int i = 0; i < Dk; ++i) {
+          double acc = 0.0;
+          for (int j = 0; j < Dv; ++j)
+            acc += (a * Sp[i * Dv + j] + gm * Rt[i * Dv + j]) * dOt[j];
+          dqt[i] = scale * acc;
+        }
+        /* dR' += gam (scale q) dO^T ; dS_{t-1} starts at a (scale q) dO^T */
+        for (int i = 0; i < Dk; ++i)
+          for (int j = 0; j < Dv; ++j) {
+            dR[i * Dv + j] += gm * scale * qt[i] * dOt[j];
+            dSp[i * Dv + j] = a * scale * qt[i] * dOt[j];
+          }
+
+        /* R step */
+        for (int j = 0; j < Dv; ++j) {
+          double uj = 0.0;
+          for (int i = 0; i < Dk; ++i) uj += kt[i] * dR[i * Dv + j];
+          u[j] = uj;
+        }
+        {
+          double dRR = 0.0;
+          for (long e = 0; e < SD; ++e) dRR += dR[e] * Rp[e];
+          da += dRR;
+        }
+        for (int j = 0; j < Dv; ++j) {
+          const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
+          if (variant == ORC_RDN) da -= gm * u[j] * rk[j];
+          dgm += u[j] * e2;
+        }
+        for (int i = 0; i < Dk; ++i) {
+          double acc = 0.0, acc2 = 0.0;
+          for (int j = 0; j < Dv; ++j) {
+            const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
+            acc += dR[i * Dv + j] * e2;
+            acc2 += Rp[i * Dv + j] * u[j];
+          }
+          dkt[i] += gm * acc;
+          if (variant == ORC_RDN) dkt[i] -= a * gm * acc2;
+        }
+        for (int i = 0; i < Dk; ++i)
+          for (int j = 0; j < Dv; ++j) {
+            double nv = a * dR[i * Dv + j];
+            if (variant == ORC_RDN) nv -= a * gm * kt[i] * u[j];
+            dRp[i * Dv + j] = nv;
+          }
+
+        /* clip */
+        for (int j = 0; j < Dv; ++j) {
+          const double x = vt[j] - p[j];
+          const double dr = gm * u[j];
+          const double dx = fabs(x) <= c ? dr : 0.0;
+          dvt[j] += dx;
+          dp[j] = -dx;
+        }
+
+        /* S step */
+        for (int j = 0; j < Dv; ++j) {
+          double wj = 0.0;
+          for (int i = 0; i < Dk; ++i) wj += kt[i] * dS[i * Dv + j];
+          w[j] = wj;
+        }
+        {
+          double dSS = 0.0;
+          for (long e = 0; e < SD; ++e) dSS += dS[e] * Sp[e];
+          da += dSS;
+        }
+        for (int j = 0; j < Dv; ++j) {
+          if (variant == ORC_RDN) {
+            const double ej = vt[j] - a * p[j];
+            da -= bb * w[j] * p[j];
+            db += w[j] * ej;
+            dp[j] -= a * bb * w[j];
+          } else {
+            db += w[j] * vt[j];
+          }
+          dvt[j] += bb * w[j];
+        }
+        for (int i = 0; i < Dk; ++i) {
+          double acc = 0.0, acc2 = 0.0;
+          for (int j = 0; j < Dv; ++j) {
+            const double ej = variant == ORC_RDN ? vt[j] - a * p[j] : vt[j];
+            acc += dS[i * Dv + j] * ej;
+            acc2 += Sp[i * Dv + j] * dp[j];
+          }
+          dkt[i] += bb * acc + acc2;
+        }
+        for (int i = 0; i < Dk; ++i)
+          for (int j = 0; j < Dv; ++j)
+            dSp[i * Dv + j] += a * dS[i * Dv + j] + kt[i] * dp[j];
+
+        dg[tok] = a * da;
+        dbeta[tok] = db;
+        dgamma[tok] = dgm;
+        memcpy(dS, dSp, sizeof(double) * SD);
+        memcpy(dR, dRp, sizeof(double) * SD);
+      }
+    }
+    if (dS0) memcpy(dS0 + bh * SD, dS, sizeof(double) * SD);
+    if (dR0) memcpy(dR0 + bh * SD, dR, sizeof(double) * SD);
+    free(ckS); free(ckR); free(segS); free(segR); free(S); free(R);
+    free(dS); free(dR); free(dSp); free(dRp); free(p); free(rk); free(ob);
+    free(Rt); free(u); free(w); free(dp); free(r);
+  }
+}
+
+void orc_rdn_bwd(int B, int T, int H, int Dk, int Dv, const double *q,
+                 const double *k, const double *v, const double *g,
+                 const double *beta, const double *gamma, double c,
+                 double scale, const double *S0, const double *R0,
+                 const double *dO, const double *dST, const double *dRT,
+                 double *dq, double *dk, double *dv, double *dg, double *dbeta,
+                 double *dgamma, double *dS0, double *dR0) {
+  bwd_impl(ORC_RDN, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           dO, dST, dRT, dq, dk, dv, dg, dbeta, dgamma, dS0, dR0);
+}
+
+void orc_rla_bwd(int B, int T, int H, int Dk, int Dv, const double *q,
+                 const double *k, const double *v, const double *g,
+                 const double *beta, const double *gamma, double c,
+                 double scale, const double *S0, const double *R0,
+                 const double *dO, const double *dST, const double *dRT,
+                 double *dq, double *dk, double *dv, double *dg, double *dbeta,
+                 double *dgamma, double *dS0, double *dR0) {
+  bwd_impl(ORC_RLA, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           dO, dST, dRT, dq, dk, dv, dg, dbeta, dgamma, dS0, dR0);
+}
+
+/* ------------------------------------------------------------------------ *
+ * Clip-margin input conditioning (test infrastructure for the backward).
+ *
+ * The derivative of Clip jumps at |x| = c, so two correct implementations
+ * whose forward residual x = v - S_{t-1}k differs by rounding can take
+ * different clip-mask decisions at elements that sit within rounding of the
+ * threshold.  To make the gradient unique at the tolerance the tests use,
+ * this routine runs the fp64 forward token by token and, wherever
+ * | |x| - c | < margin, moves v away from the threshold (keeping the side of
+ * the threshold that x is on; a push towards zero that would cross zero goes
+ * outward instead) until | |x| - c | >= margin, stepping through values
+ * representable in the input dtype (quant: 0 = double, 1 = fp32, 2 = bf16).
+ * Because p_t depends only on tokens before t, fixing v in token order leaves
+ * every later decision well defined.  v [B,T,H,Dv] is modified in place;
+ * returns the number of moved elements.  variant 0 = RLA, 1 = RDN.
+ * ------------------------------------------------------------------------ */
+static double quantize(double x, int quant) {
+  if (quant == 1) return (double)(float)x;
+  if (quant == 2) {
+    float f = (float)x;
+    unsigned int u;
+    memcpy(&u, &f, sizeof u);
+    u += 0x7FFFu + ((u >> 16) & 1u); /* round to nearest even on 16 bits */
+    u &= 0xFFFF0000u;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+  }
+  return x;
+}
+
+/* smallest representable step away from x in direction dir (+1/-1) */
+static double step_away(double x, double dir, int quant) {
+  double y = x + dir * (fabs(x) > 1e-30 ? fabs(x) : 1e-30) * 1e-3;
+  double q = quantize(y, quant);
+  /* widen until the quantised value actually moves */
+  double s = (fabs(x) > 1e-30 ? fabs(x) : 1e-30) * 1e-3;
+  while (q == x) { s *= 2.0; q = quantize(x + dir * s, quant); }
+  return q;
+}
+
+long orc_clip_margin_condition(int variant, int B, int T, int H, int Dk,
+                               int Dv, const double *q, const double *k,
+                               double *v, const double *g, const double *beta,
+                               const double *gamma, double c, double scale,
+                               const double *S0, const double *R0,
+                               double margin, int quant) {
+  const long SD = (long)Dk * Dv;
+  long moved = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(+ : moved)
+  for (long bh = 0; bh < (long)B * H; ++bh) {
+    const long b = bh / H, h = bh % H;
+    double *S = (double *)malloc(sizeof(double) * SD);
+    double *R = (double *)malloc(sizeof(double) * SD);
+    double *p = (double *)malloc(sizeof(double) * Dv);
+    double *rk = (double *)malloc(sizeof(double) * Dv);
+    double *o = (double *)malloc(sizeof(double) * Dv);
+    if (S0) memcpy(S, S0 + bh * SD, sizeof(double) * SD); else memset(S, 0, sizeof(double) * SD);
+    if (R0) memcpy(R, R0 + bh * SD, sizeof(double) * SD); else memset(R, 0, sizeof(double) * SD);
+    for (long t = 0; t < T; ++t) {
+      const long tok = (b * T + t) * H + h;
+      double *vt = v + tok * Dv;
+      const double *kt = k + tok * Dk;
+      for (int j = 0; j < Dv; ++j) {
+        double pj = 0.0;
+        for (int i = 0; i < Dk; ++i) pj += kt[i] * S[i * Dv + j];
+        double x = vt[j] - pj;
+        if (fabs(fabs(x) - c) < margin) {
+          const double sgn_x = x >= 0.0 ? 1.0 : -1.0;
+          /* outside (|x| >= c): grow |x|; inside: shrink |x| unless that
+             would cross zero before leaving the band */
+          double dir = fabs(x) >= c ? sgn_x : -sgn_x;
+          if (fabs(x) < c && fabs(x) < 2.0 * margin) dir = sgn_x;
+          int guard = 0;
+          while (fabs(fabs(vt[j] - pj) - c) < margin && guard++ < 100000)
+            vt[j] = step_away(vt[j], dir, quant);
+          ++moved;
+        }
+      }
+      token_step(variant, Dk, Dv, q + tok * Dk, kt, vt, exp(g[tok]), beta[tok],
+                 gamma[tok], c, scale, S, R, o, p, rk, NULL);
+    }
+    free(S); free(R); free(p); free(rk); free(o);
+  }
+  return moved;
+}
