@@ -1,0 +1,183 @@
+/*
+ * rdn.h -- C ABI of the GB300 (sm_103a) library for the layer hot path of
+ * Residual Linear Attention (RLA) and Residual Delta Net (RDN),
+ * "Enhancing Linear Attention with Residual Learning", arXiv 2509.25223.
+ *
+ * The operation (Section 3.4, "Final Formulations"; residual clipping
+ * Section 3.3; gates Section 3.2), per batch element b and head h, token t:
+ *
+ *   r_t = Clip_[-c,c](v_t - S_{t-1} k_t)                (elementwise in d_v)
+ *   RLA: R_t = a_t R_{t-1} + gam_t r_t k_t^T
+ *        S_t = a_t S_{t-1} + beta_t v_t k_t^T
+ *   RDN: R_t = a_t R_{t-1} (I - gam_t k_t k_t^T) + gam_t r_t k_t^T
+ *        S_t = a_t S_{t-1} (I - beta_t k_t k_t^T) + beta_t v_t k_t^T
+ *   o_t = a_t S_{t-1} (scale q_t) + gam_t R_t (scale q_t)
+ *
+ * with a_t = exp(g_t).  The gates are passed as the log-decay g = log(a) <= 0
+ * and the rates beta, gam in [0,1]; the model-side gate projections, the SiLU
+ * and the L2 normalisation of q and k (Section 3.4, paragraph after the
+ * formulations) happen before these calls.
+ *
+ * Conventions shared by every entry point:
+ *  - Pointers are DEVICE pointers owned by the caller.  The library never
+ *    frees them and keeps none of them after the call returns.
+ *  - Layouts are contiguous row-major:
+ *      q, k          [B,T,H,Dk]        v, o, dO      [B,T,H,Dv]
+ *      g, beta, gam  [B,T,H]  fp32
+ *      S0,R0,ST,RT   [B,H,Dk,Dv] fp32  (the paper's d_v x d_k state,
+ *                                        stored transposed: row i is key dim i)
+ *      S_chunks, R_chunks [B,H,NC,Dk,Dv] fp32, NC = ceil(T/64): the states at
+ *                    the start of each 64-token chunk.
+ *  - Every pointer must be 16-byte aligned.
+ *  - All work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream) and is asynchronous.  Argument errors are reported before
+ *    anything is enqueued; launch errors are checked right after the launch;
+ *    faults inside a kernel surface at the caller's next synchronisation.
+ *  - Scratch memory is the caller's: each entry point that needs it states
+ *    the size through its *_workspace_size function, and the caller passes a
+ *    device buffer of at least that size (16-byte aligned).  The library
+ *    makes no allocation of its own on these paths.
+ *  - No C++ exception or abort crosses this boundary.  Every function
+ *    returns an rdn_status_t; rdn_last_error() gives a message for the last
+ *    failure on the calling thread.
+ *  - Calls are reentrant: the library keeps no per-call state outside the
+ *    caller's buffers.
+ */
+#ifndef RDN_H_
+#define RDN_H_
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *rdn_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+  RDN_OK = 0,
+  RDN_ERR_INVALID_ARG = 1, /* bad shape, NULL where required, c < 0 or NaN */
+  RDN_ERR_UNSUPPORTED = 2, /* valid but not implemented (dtype, Dk/Dv, flags) */
+  RDN_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed */
+  RDN_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up */
+  RDN_ERR_WORKSPACE = 5,   /* workspace missing, too small or misaligned */
+  RDN_ERR_MISALIGNED = 6   /* a pointer is not 16-byte aligned */
+} rdn_status_t;
+
+typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
+
+/* Arguments of rla_fwd / rdn_fwd.
+ *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
+ *                     S0/R0 to ST/RT).
+ *   Dk, Dv            head dimensions.  RDN_BF16 supports Dk = Dv = 128 and
+ *                     Dk = Dv = 64; RDN_F32 supports Dk, Dv in {64, 128}.
+ *   dtype             element type of q, k, v and o.  Gates and states are
+ *                     always fp32 and every accumulation is fp32.
+ *   q, k, v           inputs (q, k expected L2-normalised; not checked).
+ *   g, beta, gamma    per-token, per-head log-decay g = log(alpha) and rates.
+ *   clip              the threshold c of Section 3.3; INFINITY = no clip;
+ *                     c < 0 or NaN -> RDN_ERR_INVALID_ARG.
+ *   S0, R0            initial states or NULL (= zero).
+ *   o                 output [B,T,H,Dv] in `dtype`.
+ *   ST, RT            final states or NULL (= not returned).
+ *   S_chunks,R_chunks optional chunk-start states (outputs; NULL = not
+ *                     stored).  rdn_bwd can consume them instead of
+ *                     recomputing.
+ *   scale             multiplies q (the paper uses 1).
+ *   flags             must be 0 (paper variants are reserved bits).
+ *   workspace         device scratch of *_fwd_workspace_size() bytes.     */
+typedef struct {
+  int B, T, H, Dk, Dv;
+  int dtype; /* rdn_dtype_t */
+  const void *q, *k, *v;
+  const float *g, *beta, *gamma;
+  float clip;
+  const float *S0, *R0;
+  void *o;
+  float *ST, *RT;
+  float *S_chunks, *R_chunks;
+  float scale;
+  unsigned flags;
+  void *workspace;
+  size_t workspace_bytes;
+} rdn_fwd_args;
+
+/* Arguments of rdn_bwd.  `fwd` holds the forward's inputs (its o, ST, RT,
+ * S_chunks and R_chunks outputs are ignored except as noted).
+ *   fwd.S_chunks/R_chunks  if both non-NULL they are READ as the forward's
+ *                     chunk-start states (as written by rdn_fwd on the same
+ *                     inputs); if NULL the backward recomputes them into its
+ *                     workspace.
+ *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
+ *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
+ *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype.
+ *   dg, dbeta, dgamma [B,T,H] fp32.  dg is the gradient w.r.t. the
+ *                     log-decay g; the gradient w.r.t. alpha is dg / alpha.
+ *   dS0, dR0          [B,H,Dk,Dv] fp32, or NULL (= not returned).
+ * At |v - S_{t-1}k| == c the clip passes the gradient (inclusive mask).    */
+typedef struct {
+  rdn_fwd_args fwd;
+  const void *dO;
+  const float *dST, *dRT;
+  void *dq, *dk, *dv;
+  float *dg, *dbeta, *dgamma;
+  float *dS0, *dR0;
+  void *workspace;
+  size_t workspace_bytes;
+} rdn_bwd_args;
+
+/* Arguments of rdn_decode_step: one token for N independent sequences.
+ *   N, H, Dk, Dv      Dk = Dv = 128 or 64.
+ *   dtype             element type of q, k, v, o (RDN_BF16 or RDN_F32).
+ *   q, k [N,H,Dk]; v, o [N,H,Dv]; g, beta, gamma [N,H] fp32.
+ *   S, R [N,H,Dk,Dv] fp32, read and updated IN PLACE (must not alias any
+ *   other argument).
+ *   variant           0 = RLA, 1 = RDN.                                   */
+typedef struct {
+  int N, H, Dk, Dv;
+  int dtype;
+  int variant;
+  const void *q, *k, *v;
+  const float *g, *beta, *gamma;
+  float clip;
+  float scale;
+  float *S, *R;
+  void *o;
+} rdn_decode_args;
+
+/* RLA forward, Section 3.4 (left formulation).  Chunkwise-parallel form:
+ * additive base state, no triangular solves. */
+rdn_status_t rla_fwd(const rdn_fwd_args *args, rdn_stream_t stream);
+
+/* RDN forward, Section 3.4 (right formulation).  Gated delta rule on S and
+ * on R, chunkwise (64 tokens) with the UT/WY triangular form of the delta
+ * rule; the clipped residual is formed and consumed on chip. */
+rdn_status_t rdn_fwd(const rdn_fwd_args *args, rdn_stream_t stream);
+
+/* Backward of rdn_fwd (reverse-mode of the same chunkwise computation).
+ * Supports RDN_BF16 with Dk = Dv in {64, 128} and RDN_F32 likewise. */
+rdn_status_t rdn_bwd(const rdn_bwd_args *args, rdn_stream_t stream);
+
+/* One recurrent step (Section 3.4 recurrence at a single t), states in
+ * place; memory-bound: reads and writes S and R once. */
+rdn_status_t rdn_decode_step(const rdn_decode_args *args, rdn_stream_t stream);
+
+/* Workspace sizes in bytes for the arguments' shapes (pointers ignored).
+ * Return RDN_OK and set *bytes, or an error for invalid shapes. */
+rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
+rdn_status_t rdn_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
+rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *args, size_t *bytes);
+
+/* Message describing the last non-OK status returned on this thread
+ * ("" if none).  The pointer stays valid until the next call on the
+ * thread. */
+const char *rdn_last_error(void);
+
+/* Library version string. */
+const char *rdn_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RDN_H_ */

@@ -1,0 +1,203 @@
+"""GB300 (sm_103a) layer hot path of Residual Linear Attention (RLA) and
+Residual Delta Net (RDN), arXiv 2509.25223, Section 3.4.
+
+A thin binding over the C ABI in include/rdn.h (librdn.so): it marshals torch
+tensor pointers, sizes and the current CUDA stream, allocates the workspace
+the library asks for, and raises on a non-OK status.  Every step of the
+computation runs in the library's CUDA kernels; there is no CPU or PyTorch
+fallback, and a missing or unloadable library is an error.
+
+Tensors (contiguous, on one CUDA device):
+    q, k [B,T,H,Dk]; v [B,T,H,Dv]            bf16 or fp32 (same dtype)
+    g (log-decay = log alpha), beta, gamma [B,T,H]   fp32
+    S0, R0 [B,H,Dk,Dv] fp32 or None
+Results: o [B,T,H,Dv] in the input dtype; ST, RT [B,H,Dk,Dv] fp32.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+
+import torch
+
+from . import _abi
+from ._abi import BwdArgs, DecodeArgs, FwdArgs
+
+__all__ = ["rla_fwd", "rdn_fwd", "rdn_bwd", "rdn_decode_step", "RdnError", "library",
+           "CHUNK"]
+
+CHUNK = 64
+
+
+class RdnError(RuntimeError):
+    def __init__(self, fn, status, msg):
+        super().__init__(f"{fn} -> {_abi.STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def library():
+    """The loaded librdn.so (ctypes.CDLL)."""
+    return _abi.load()
+
+
+def _check(fn, st):
+    if st != 0:
+        raise RdnError(fn, st, _abi.load().rdn_last_error().decode())
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("rdn: tensors must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("rdn: tensors must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype_code(t):
+    if t.dtype == torch.bfloat16:
+        return _abi.RDN_BF16
+    if t.dtype == torch.float32:
+        return _abi.RDN_F32
+    raise ValueError(f"rdn: unsupported dtype {t.dtype}")
+
+
+def _stream(t):
+    return ctypes.c_void_p(torch.cuda.current_stream(t.device).cuda_stream)
+
+
+def _alloc_ws(nbytes, device):
+    if nbytes == 0:
+        return None
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale):
+    B, T, H, Dk = q.shape
+    a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, Dk, v.shape[-1]
+    a.dtype = _dtype_code(q)
+    a.q, a.k, a.v = _ptr(q), _ptr(k), _ptr(v)
+    a.g, a.beta, a.gamma = _ptr(g), _ptr(beta), _ptr(gamma)
+    a.clip = float(clip)
+    a.S0, a.R0 = _ptr(S0), _ptr(R0)
+    a.o = _ptr(o)
+    a.ST, a.RT = _ptr(ST), _ptr(RT)
+    a.S_chunks, a.R_chunks = _ptr(Sc), _ptr(Rc)
+    a.scale = float(scale)
+    a.flags = 0
+
+
+def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
+         return_final_state=True, return_chunk_states=False, out=None, workspace=None):
+    lib = _abi.load()
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    dev = q.device
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    ST = RT = Sc = Rc = None
+    if return_final_state:
+        ST = torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev)
+        RT = torch.empty_like(ST)
+    if return_chunk_states:
+        NC = (T + CHUNK - 1) // CHUNK
+        Sc = torch.empty(B, H, NC, Dk, Dv, dtype=torch.float32, device=dev)
+        Rc = torch.empty_like(Sc)
+    a = FwdArgs()
+    _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale)
+    nbytes = ctypes.c_size_t(0)
+    _check(name + "_workspace_size",
+           getattr(lib, name + "_workspace_size")(ctypes.byref(a), ctypes.byref(nbytes)))
+    ws = workspace
+    if ws is None or ws.numel() < nbytes.value:
+        ws = _alloc_ws(nbytes.value, dev)
+    a.workspace = _ptr(ws)
+    a.workspace_bytes = nbytes.value if ws is not None else 0
+    _check(name, getattr(lib, name)(ctypes.byref(a), _stream(q)))
+    res = [o]
+    if return_final_state:
+        res += [ST, RT]
+    if return_chunk_states:
+        res += [Sc, Rc]
+    return tuple(res) if len(res) > 1 else o
+
+
+def rla_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw):
+    """RLA forward (Section 3.4, left).  Returns (o, ST, RT)."""
+    return _fwd("rla_fwd", q, k, v, g, beta, gamma, clip, S0, R0, scale, **kw)
+
+
+def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw):
+    """RDN forward (Section 3.4, right).  Returns (o, ST, RT) and, with
+    return_chunk_states=True, also the chunk-start states (Sc, Rc) that
+    rdn_bwd can reuse."""
+    return _fwd("rdn_fwd", q, k, v, g, beta, gamma, clip, S0, R0, scale, **kw)
+
+
+def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
+            scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None):
+    """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
+    dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32)."""
+    lib = _abi.load()
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    dev = q.device
+    if out is None:
+        out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
+                   dg=torch.empty(B, T, H, dtype=torch.float32, device=dev),
+                   dbeta=torch.empty(B, T, H, dtype=torch.float32, device=dev),
+                   dgamma=torch.empty(B, T, H, dtype=torch.float32, device=dev),
+                   dS0=torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev),
+                   dR0=torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev))
+    a = BwdArgs()
+    _fill_fwd(a.fwd, q, k, v, g, beta, gamma, clip, S0, R0, None, None, None, S_chunks,
+              R_chunks, scale)
+    a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
+    a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
+    a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"])
+    a.dS0, a.dR0 = _ptr(out.get("dS0")), _ptr(out.get("dR0"))
+    nbytes = ctypes.c_size_t(0)
+    _check("rdn_bwd_workspace_size", lib.rdn_bwd_workspace_size(ctypes.byref(a), ctypes.byref(nbytes)))
+    ws = workspace
+    if ws is None or ws.numel() < nbytes.value:
+        ws = _alloc_ws(nbytes.value, dev)
+    a.workspace = _ptr(ws)
+    a.workspace_bytes = nbytes.value if ws is not None else 0
+    _check("rdn_bwd", lib.rdn_bwd(ctypes.byref(a), _stream(q)))
+    return out
+
+
+def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant="rdn", out=None):
+    """One recurrent step for N sequences; S, R [N,H,Dk,Dv] fp32 are updated
+    in place.  q, k [N,H,Dk]; v [N,H,Dv]; gates [N,H].  Returns o [N,H,Dv]."""
+    lib = _abi.load()
+    N, H, Dk = q.shape
+    Dv = v.shape[-1]
+    o = out if out is not None else torch.empty(N, H, Dv, dtype=q.dtype, device=q.device)
+    a = DecodeArgs()
+    a.N, a.H, a.Dk, a.Dv = N, H, Dk, Dv
+    a.dtype = _dtype_code(q)
+    a.variant = 1 if variant == "rdn" else 0
+    a.q, a.k, a.v = _ptr(q), _ptr(k), _ptr(v)
+    a.g, a.beta, a.gamma = _ptr(g), _ptr(beta), _ptr(gamma)
+    a.clip, a.scale = float(clip), float(scale)
+    a.S, a.R, a.o = _ptr(S), _ptr(R), _ptr(o)
+    _check("rdn_decode_step", lib.rdn_decode_step(ctypes.byref(a), _stream(q)))
+    return o
+
+
+def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16):
+    """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rdn_bwd)."""
+    lib = _abi.load()
+    a = FwdArgs()
+    a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
+    a.dtype = _abi.RDN_BF16 if dtype == torch.bfloat16 else _abi.RDN_F32
+    a.clip, a.scale = 1.0, 1.0
+    n = ctypes.c_size_t(0)
+    if op == "rdn_bwd":
+        b = BwdArgs()
+        b.fwd = a
+        _check(op, lib.rdn_bwd_workspace_size(ctypes.byref(b), ctypes.byref(n)))
+    else:
+        _check(op, getattr(lib, op + "_workspace_size")(ctypes.byref(a), ctypes.byref(n)))
+    return n.value

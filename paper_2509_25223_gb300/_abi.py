@@ -1,0 +1,80 @@
+"""ctypes declarations mirroring include/rdn.h (structs and entry points)."""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from . import build as _build
+
+P = ctypes.c_void_p
+F = ctypes.POINTER(ctypes.c_float)
+
+RDN_F32, RDN_BF16 = 0, 1
+
+STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "RDN_ERR_CUDA",
+          4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}
+
+# every function the header declares (checked by the CPU tests)
+EXPORTS = ["rla_fwd", "rdn_fwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
+           "rdn_fwd_workspace_size", "rdn_bwd_workspace_size", "rdn_last_error", "rdn_version"]
+
+
+class FwdArgs(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("Dk", ctypes.c_int), ("Dv", ctypes.c_int), ("dtype", ctypes.c_int),
+                ("q", P), ("k", P), ("v", P), ("g", P), ("beta", P), ("gamma", P),
+                ("clip", ctypes.c_float), ("S0", P), ("R0", P), ("o", P),
+                ("ST", P), ("RT", P), ("S_chunks", P), ("R_chunks", P),
+                ("scale", ctypes.c_float), ("flags", ctypes.c_uint),
+                ("workspace", P), ("workspace_bytes", ctypes.c_size_t)]
+
+
+class BwdArgs(ctypes.Structure):
+    _fields_ = [("fwd", FwdArgs), ("dO", P), ("dST", P), ("dRT", P),
+                ("dq", P), ("dk", P), ("dv", P), ("dg", P), ("dbeta", P), ("dgamma", P),
+                ("dS0", P), ("dR0", P), ("workspace", P), ("workspace_bytes", ctypes.c_size_t)]
+
+
+class DecodeArgs(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int), ("H", ctypes.c_int), ("Dk", ctypes.c_int),
+                ("Dv", ctypes.c_int), ("dtype", ctypes.c_int), ("variant", ctypes.c_int),
+                ("q", P), ("k", P), ("v", P), ("g", P), ("beta", P), ("gamma", P),
+                ("clip", ctypes.c_float), ("scale", ctypes.c_float),
+                ("S", P), ("R", P), ("o", P)]
+
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Load librdn.so (building it first if needed and allowed)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path) or (build_if_missing and not _build.up_to_date()):
+        if not build_if_missing:
+            raise RuntimeError(f"librdn.so not built ({path}); run paper_2509_25223_gb300.build")
+        _build.build()
+    lib = ctypes.CDLL(path)
+    S = ctypes.c_int
+    for name, argt in [("rla_fwd", [ctypes.POINTER(FwdArgs), P]),
+                       ("rdn_fwd", [ctypes.POINTER(FwdArgs), P]),
+                       ("rdn_bwd", [ctypes.POINTER(BwdArgs), P]),
+                       ("rdn_decode_step", [ctypes.POINTER(DecodeArgs), P]),
+                       ("rla_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
+                       ("rdn_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
+                       ("rdn_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)])]:
+        fn = getattr(lib, name)
+        fn.argtypes = argt
+        fn.restype = S
+    lib.rdn_last_error.restype = ctypes.c_char_p
+    lib.rdn_last_error.argtypes = []
+    lib.rdn_version.restype = ctypes.c_char_p
+    lib.rdn_version.argtypes = []
+    _lib = lib
+    return lib

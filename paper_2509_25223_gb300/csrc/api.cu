@@ -1,0 +1,220 @@
+// api.cu -- the C ABI declared in include/rdn.h: argument validation, error
+// reporting and dispatch to the kernel launchers.  No exception or abort
+// crosses this boundary; every entry point returns an rdn_status_t.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "common.cuh"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+rdn_status_t fail(rdn_status_t st, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof g_err, fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+rdn_status_t ok() {
+  g_err[0] = '\0';
+  return RDN_OK;
+}
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+#define REQUIRE_PTR(p)                                                        \
+  do {                                                                        \
+    if (!(p)) return fail(RDN_ERR_INVALID_ARG, "%s: " #p " is NULL", fn);     \
+    if (!aligned16(p))                                                        \
+      return fail(RDN_ERR_MISALIGNED, "%s: " #p " is not 16-byte aligned", fn); \
+  } while (0)
+#define OPTIONAL_PTR(p)                                                       \
+  do {                                                                        \
+    if ((p) && !aligned16(p))                                                 \
+      return fail(RDN_ERR_MISALIGNED, "%s: " #p " is not 16-byte aligned", fn); \
+  } while (0)
+
+rdn_status_t check_clip(const char *fn, float c) {
+  if (isnan(c) || c < 0.f) return fail(RDN_ERR_INVALID_ARG, "%s: clip must be >= 0 (got %g)", fn, c);
+  return RDN_OK;
+}
+
+rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
+  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  if (a->B < 1 || a->H < 1 || a->T < 0)
+    return fail(RDN_ERR_INVALID_ARG, "%s: need B >= 1, H >= 1, T >= 0 (got B=%d T=%d H=%d)", fn,
+                a->B, a->T, a->H);
+  if (a->dtype != RDN_F32 && a->dtype != RDN_BF16)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: dtype %d unsupported", fn, a->dtype);
+  if (!((a->Dk == 64 || a->Dk == 128) && a->Dv == a->Dk))
+    return fail(RDN_ERR_UNSUPPORTED, "%s: supported head dims are Dk = Dv in {64, 128} (got %d, %d)",
+                fn, a->Dk, a->Dv);
+  if ((long long)a->B * a->T * a->H > (1ll << 31) / 128)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: B*T*H = %lld too large", fn,
+                (long long)a->B * a->T * a->H);
+  if (a->flags != 0) return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
+  if (isnan(a->scale) || isinf(a->scale))
+    return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
+  return check_clip(fn, a->clip);
+}
+
+rdn_status_t check_fwd_ptrs(const char *fn, const rdn_fwd_args *a) {
+  if (a->T > 0) {
+    REQUIRE_PTR(a->q);
+    REQUIRE_PTR(a->k);
+    REQUIRE_PTR(a->v);
+    REQUIRE_PTR(a->g);
+    REQUIRE_PTR(a->beta);
+    REQUIRE_PTR(a->gamma);
+    REQUIRE_PTR(a->o);
+  }
+  OPTIONAL_PTR(a->S0);
+  OPTIONAL_PTR(a->R0);
+  OPTIONAL_PTR(a->ST);
+  OPTIONAL_PTR(a->RT);
+  OPTIONAL_PTR(a->S_chunks);
+  OPTIONAL_PTR(a->R_chunks);
+  if ((a->S_chunks == nullptr) != (a->R_chunks == nullptr))
+    return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  return RDN_OK;
+}
+
+rdn_status_t cuda_status(const char *fn, cudaError_t e) {
+  if (e == cudaSuccess) return ok();
+  return fail(RDN_ERR_CUDA, "%s: CUDA error %d (%s)", fn, (int)e, cudaGetErrorString(e));
+}
+
+rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a, int variant, cudaStream_t s) {
+  rdn_status_t st = check_fwd_shapes(fn, a);
+  if (st != RDN_OK) return st;
+  if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
+  const rdn::FwdPlan plan = rdn::plan_fwd(*a, variant);
+  if (plan.total_bytes > 0) {
+    if (!a->workspace || a->workspace_bytes < plan.total_bytes)
+      return fail(RDN_ERR_WORKSPACE, "%s: workspace of %zu bytes required (got %zu)", fn,
+                  plan.total_bytes, a->workspace ? a->workspace_bytes : (size_t)0);
+    if (!aligned16(a->workspace))
+      return fail(RDN_ERR_WORKSPACE, "%s: workspace is not 16-byte aligned", fn);
+  }
+  return cuda_status(fn, rdn::launch_fwd(*a, variant, s));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *rdn_last_error(void) { return g_err; }
+
+const char *rdn_version(void) { return "rdn-gb300 0.1 (sm_103a)"; }
+
+rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *a, size_t *bytes) {
+  rdn_status_t st = check_fwd_shapes("rla_fwd_workspace_size", a);
+  if (st != RDN_OK) return st;
+  if (!bytes) return fail(RDN_ERR_INVALID_ARG, "rla_fwd_workspace_size: bytes is NULL");
+  *bytes = rdn::plan_fwd(*a, 0).total_bytes;
+  return ok();
+}
+
+rdn_status_t rdn_fwd_workspace_size(const rdn_fwd_args *a, size_t *bytes) {
+  rdn_status_t st = check_fwd_shapes("rdn_fwd_workspace_size", a);
+  if (st != RDN_OK) return st;
+  if (!bytes) return fail(RDN_ERR_INVALID_ARG, "rdn_fwd_workspace_size: bytes is NULL");
+  *bytes = rdn::plan_fwd(*a, 1).total_bytes;
+  return ok();
+}
+
+rdn_status_t rla_fwd(const rdn_fwd_args *a, rdn_stream_t stream) {
+  return fwd_common("rla_fwd", a, 0, (cudaStream_t)stream);
+}
+
+rdn_status_t rdn_fwd(const rdn_fwd_args *a, rdn_stream_t stream) {
+  return fwd_common("rdn_fwd", a, 1, (cudaStream_t)stream);
+}
+
+rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *a, size_t *bytes) {
+  const char *fn = "rdn_bwd_workspace_size";
+  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  rdn_status_t st = check_fwd_shapes(fn, &a->fwd);
+  if (st != RDN_OK) return st;
+  if (!bytes) return fail(RDN_ERR_INVALID_ARG, "%s: bytes is NULL", fn);
+  *bytes = rdn::plan_bwd(*a).total_bytes;
+  return ok();
+}
+
+rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
+  const char *fn = "rdn_bwd";
+  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  rdn_status_t st = check_fwd_shapes(fn, &a->fwd);
+  if (st != RDN_OK) return st;
+  const rdn_fwd_args *f = &a->fwd;
+  if (f->T > 0) {
+    REQUIRE_PTR(f->q);
+    REQUIRE_PTR(f->k);
+    REQUIRE_PTR(f->v);
+    REQUIRE_PTR(f->g);
+    REQUIRE_PTR(f->beta);
+    REQUIRE_PTR(f->gamma);
+    REQUIRE_PTR(a->dO);
+    REQUIRE_PTR(a->dq);
+    REQUIRE_PTR(a->dk);
+    REQUIRE_PTR(a->dv);
+    REQUIRE_PTR(a->dg);
+    REQUIRE_PTR(a->dbeta);
+    REQUIRE_PTR(a->dgamma);
+  }
+  OPTIONAL_PTR(f->S0);
+  OPTIONAL_PTR(f->R0);
+  OPTIONAL_PTR(f->S_chunks);
+  OPTIONAL_PTR(f->R_chunks);
+  if ((f->S_chunks == nullptr) != (f->R_chunks == nullptr))
+    return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  OPTIONAL_PTR(a->dST);
+  OPTIONAL_PTR(a->dRT);
+  OPTIONAL_PTR(a->dS0);
+  OPTIONAL_PTR(a->dR0);
+  const rdn::BwdPlan plan = rdn::plan_bwd(*a);
+  if (plan.total_bytes > 0) {
+    if (!a->workspace || a->workspace_bytes < plan.total_bytes)
+      return fail(RDN_ERR_WORKSPACE, "%s: workspace of %zu bytes required (got %zu)", fn,
+                  plan.total_bytes, a->workspace ? a->workspace_bytes : (size_t)0);
+    if (!aligned16(a->workspace))
+      return fail(RDN_ERR_WORKSPACE, "%s: workspace is not 16-byte aligned", fn);
+  }
+  return cuda_status(fn, rdn::launch_bwd(*a, (cudaStream_t)stream));
+}
+
+rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {
+  const char *fn = "rdn_decode_step";
+  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  if (a->N < 1 || a->H < 1)
+    return fail(RDN_ERR_INVALID_ARG, "%s: need N >= 1, H >= 1 (got N=%d H=%d)", fn, a->N, a->H);
+  if (!((a->Dk == 64 || a->Dk == 128) && a->Dv == a->Dk))
+    return fail(RDN_ERR_UNSUPPORTED, "%s: supported head dims are Dk = Dv in {64, 128}", fn);
+  if (a->dtype != RDN_F32 && a->dtype != RDN_BF16)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: dtype %d unsupported", fn, a->dtype);
+  if (a->variant != 0 && a->variant != 1)
+    return fail(RDN_ERR_INVALID_ARG, "%s: variant must be 0 (RLA) or 1 (RDN)", fn);
+  if ((long long)a->N * a->H > (1ll << 31) / 4)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: N*H too large", fn);
+  rdn_status_t st = check_clip(fn, a->clip);
+  if (st != RDN_OK) return st;
+  if (isnan(a->scale) || isinf(a->scale)) return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
+  REQUIRE_PTR(a->q);
+  REQUIRE_PTR(a->k);
+  REQUIRE_PTR(a->v);
+  REQUIRE_PTR(a->g);
+  REQUIRE_PTR(a->beta);
+  REQUIRE_PTR(a->gamma);
+  REQUIRE_PTR(a->S);
+  REQUIRE_PTR(a->R);
+  REQUIRE_PTR(a->o);
+  if (a->S == a->R) return fail(RDN_ERR_INVALID_ARG, "%s: S and R alias", fn);
+  return cuda_status(fn, rdn::launch_decode(*a, (cudaStream_t)stream));
+}
+
+}  // extern "C"

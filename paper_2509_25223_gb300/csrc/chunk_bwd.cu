@@ -1,0 +1,755 @@
+// chunk_bwd.cu -- backward of the chunkwise RLA / RDN forward (fp32 SIMT).
+//
+// Reverse mode of the chunk algebra in chunk_fwd.cu (the paper gives no
+// backward; this is the adjoint of the forward as computed).  Per chunk,
+// given the carried dS, dR (gradients w.r.t. the chunk-end states) and dO:
+//
+//   auxiliary pass  dOa = diag(gam) dO;  dgam += rowsum(dO * Oa)
+//                   dM2 = incl(dOa E2^T);  dE2 = M2^T dOa + diag(wR) K dR
+//                   RDN: dX2 = Tg^T dE2, dAg = -strict(dX2 E2^T), dRv = dX2,
+//                        dKR = -diag(Gam) dX2;   RLA: dRv = dE2
+//                   dR0 = Gam_C dR + K^T dKR + Q^T diag(Gam) dOa
+//   clip            dV = dRv * [|v - P| <= c],  dP = -dV
+//   base pass       dMq = strict(dO E^T);  dAp = strict(dP E^T)
+//                   dE = Mq^T dO + Ap^T dP + diag(wS) K dS
+//                   RDN: dX = Tb^T dE, dAb = -strict(dX E^T), dV += dX,
+//                        dKS = diag(Gprev) dP - diag(Gam) dX;   RLA: dV += dE
+//                   dS0 = Gam_C dS + K^T dKS + Q^T diag(Gam) dO
+//   dK, dQ collect the state products (E dS^T, dKS S0^T, ...); the C x C
+//   gradients dAp, dMq, dM2, dAb, dAg and the per-row factors then give
+//   d(KK^T), d(QK^T), dbeta, dgamma and the gradient of the in-chunk
+//   cumulative log-decay, whose reverse cumulative sum is dg.
+//
+// Kernel bwd_scan: one CTA per (b, h, 16-column slice of d_v), chunks in
+// reverse, recomputing the chunk's forward pieces from the chunk-start
+// states.  Value columns are independent in the forward, so each slice owns
+// its dv, dS, dR columns; its contributions to dK, dQ and to the C x C and
+// per-row gradients (sums over d_v) are added into a per-chunk accumulator.
+// Kernel bwd_finish: one CTA per chunk, folds the accumulator into dq, dk,
+// dg, dbeta, dgamma.
+#include "chunk_common.cuh"
+
+namespace rdn {
+namespace {
+
+constexpr int kBDVS = 16;       // value columns per backward scan CTA
+constexpr int LDV = kBDVS + 1;  // padded row stride of the [C][kBDVS] tiles
+
+template <int DK>
+struct Acc {  // per-chunk accumulator record (floats)
+  static constexpr int DKo = 0, DQo = C * DK;
+  static constexpr int DAP = 2 * C * DK, DMQ = DAP + kCC, DM2 = DMQ + kCC, DAB = DM2 + kCC,
+                       DAG = DAB + kCC, VEC = DAG + kCC;
+  // per-row vectors: d(gamma) from the read-out, dGam, dGprev, dwS, dwR; then dGamC
+  static constexpr int V_DGAM_OUT = 0, V_DGAM = C, V_DGPREV = 2 * C, V_DWS = 3 * C, V_DWR = 4 * C,
+                       V_DGAMC = 5 * C;
+  static constexpr int FLOATS = VEC + 6 * C;
+};
+
+struct BwdParams {
+  FwdParams f;  // forward inputs; f.ws = prep records
+  const void *dO;
+  const float *dST, *dRT;
+  const float *Sc, *Rc;  // chunk-start states [B,H,NC,DK,DV]
+  void *dq, *dk, *dv;
+  float *dg, *dbeta, *dgamma, *dS0, *dR0;
+  float *acc;  // [B*H*NC] accumulator records
+};
+
+// ---------------------------------------------------------------- kernel 1
+template <int DK, bool RDNV, typename InT>
+__global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
+  constexpr int DV = DK;
+  constexpr int LDK = DK + 1;
+  using L = Acc<DK>;
+  extern __shared__ float sm[];
+  float *Ks = sm;                // [C][LDK]
+  float *Qs = Ks + C * LDK;      // [C][LDK] (scaled q)
+  float *S0 = Qs + C * LDK;      // [DK][LDV] chunk-start states (slice)
+  float *R0 = S0 + DK * LDV;
+  float *dS = R0 + DK * LDV;     // carried gradients w.r.t. the chunk-end states
+  float *dR = dS + DK * LDV;
+  float *CC = dR + DK * LDV;     // [C][C] staging of one chunk matrix
+  float *Vs = CC + C * C;        // [C][LDV] tiles
+  float *dOs = Vs + C * LDV;
+  float *KS = dOs + C * LDV;
+  float *QS = KS + C * LDV;
+  float *KR = QS + C * LDV;
+  float *QR = KR + C * LDV;
+  float *Es = QR + C * LDV;
+  float *E2 = Es + C * LDV;
+  float *XR = E2 + C * LDV;      // v - P, the residual before the clip
+  float *T1 = XR + C * LDV;
+  float *T2 = T1 + C * LDV;
+  float *T3 = T2 + C * LDV;
+  float *vec = T3 + C * LDV;     // [6*C] Gam, Gprev, alpha, wS, wR, GamC
+  float *gmv = vec + 6 * C;      // [C] gamma per token
+  float *red = gmv + C;          // [6*C] per-row sums of this slice
+
+  const int bh = blockIdx.x;
+  const int b = bh / p.f.H, h = bh % p.f.H;
+  const int j0 = blockIdx.y * kBDVS;
+  const int tid = threadIdx.x;
+  const int NC = p.f.NC, T = p.f.T, H = p.f.H;
+  const InT *q = (const InT *)p.f.q;
+  const InT *k = (const InT *)p.f.k;
+  const InT *v = (const InT *)p.f.v;
+  const InT *dO = (const InT *)p.dO;
+  InT *dv = (InT *)p.dv;
+  const float clip = p.f.clip;
+  const size_t sbase = (size_t)bh * DK * DV;
+
+  using MMk = BlockMM<C, kBDVS, DK>;   // [C x DK] @ [DK x DVS]
+  using MMc = BlockMM<C, kBDVS, C>;    // [C x C] @ [C x DVS]
+  using MMg = BlockMM<C, C, kBDVS>;    // [C x DVS] @ [DVS x C]
+  using MMd = BlockMM<C, DK, kBDVS>;   // [C x DVS] @ [DVS x DK]
+  using MMu = BlockMM<DK, kBDVS, C>;   // [DK x C] @ [C x DVS]
+  const int col = MMk::col();
+
+  for (int e = tid; e < DK * kBDVS; e += kThreads) {
+    const int i = e / kBDVS, jj = e % kBDVS;
+    dS[i * LDV + jj] = p.dST ? p.dST[sbase + (size_t)i * DV + j0 + jj] : 0.f;
+    dR[i * LDV + jj] = p.dRT ? p.dRT[sbase + (size_t)i * DV + j0 + jj] : 0.f;
+  }
+
+  for (int c = NC - 1; c >= 0; --c) {
+    const int t0 = c * C;
+    const int n = min(C, T - t0);
+    const size_t chunk = (size_t)bh * NC + c;
+    const float *rec = p.f.ws + chunk * kRecFloats;
+    float *acc = p.acc + chunk * L::FLOATS;
+    __syncthreads();
+    for (int e = tid; e < C * DK; e += kThreads) {
+      const int t = e / DK, d = e % DK;
+      float kv = 0.f, qv = 0.f;
+      if (t < n) {
+        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+        kv = to_f32(k[off]);
+        qv = p.f.scale * to_f32(q[off]);
+      }
+      Ks[t * LDK + d] = kv;
+      Qs[t * LDK + d] = qv;
+    }
+    for (int e = tid; e < C * kBDVS; e += kThreads) {
+      const int t = e / kBDVS, jj = e % kBDVS;
+      float vv = 0.f, dd = 0.f;
+      if (t < n) {
+        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DV + j0 + jj;
+        vv = to_f32(v[off]);
+        dd = to_f32(dO[off]);
+      }
+      Vs[t * LDV + jj] = vv;
+      dOs[t * LDV + jj] = dd;
+    }
+    for (int e = tid; e < DK * kBDVS; e += kThreads) {
+      const int i = e / kBDVS, jj = e % kBDVS;
+      const size_t off = chunk * DK * DV + (size_t)i * DV + j0 + jj;
+      S0[i * LDV + jj] = p.Sc[off];
+      R0[i * LDV + jj] = p.Rc[off];
+    }
+    for (int e = tid; e < 6 * C; e += kThreads) {
+      vec[e] = rec[OFF_VEC + e];
+      red[e] = 0.f;
+    }
+    if (tid < C) gmv[tid] = tid < n ? p.f.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    __syncthreads();
+    const float *Gam = vec + V_GAM, *Gprev = vec + V_GPREV, *wS = vec + V_WS, *wR = vec + V_WR;
+    const float GamC = vec[V_GAMC];
+
+    // ---- recompute the chunk's forward pieces
+    {
+      float a1[MMk::RPT], a2[MMk::RPT], a3[MMk::RPT], a4[MMk::RPT];
+      MMk::run(Ks, LDK, 1, S0, LDV, 1, a1);
+      MMk::run(Qs, LDK, 1, S0, LDV, 1, a2);
+      MMk::run(Ks, LDK, 1, R0, LDV, 1, a3);
+      MMk::run(Qs, LDK, 1, R0, LDV, 1, a4);
+#pragma unroll
+      for (int i = 0; i < MMk::RPT; ++i) {
+        const int t = MMk::row(i);
+        KS[t * LDV + col] = a1[i];
+        QS[t * LDV + col] = a2[i];
+        KR[t * LDV + col] = a3[i];
+        QR[t * LDV + col] = a4[i];
+        if (RDNV) T1[t * LDV + col] = Vs[t * LDV + col] - Gam[t] * a1[i];
+      }
+    }
+    const float *E = Vs;
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, T1, LDV, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) Es[MMc::row(i) * LDV + col] = a1[i];
+      E = Es;
+    }
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    __syncthreads();
+    {
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, E, LDV, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        const float x = Vs[t * LDV + col] - (Gprev[t] * KS[t * LDV + col] + a1[i]);
+        XR[t * LDV + col] = x;
+        if (RDNV) T1[t * LDV + col] = clampf(x, clip) - Gam[t] * KR[t * LDV + col];
+        else E2[t * LDV + col] = clampf(x, clip);
+      }
+    }
+    __syncthreads();
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, T1, LDV, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) E2[MMc::row(i) * LDV + col] = a1[i];
+      __syncthreads();
+    }
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_M2 + e];
+    __syncthreads();
+    {  // Oa -> T2, dOa -> T3, row sums d(gamma)_out and dGam
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, E2, LDV, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        const float oa = Gam[t] * QR[t * LDV + col] + a1[i];
+        const float dOv = dOs[t * LDV + col];
+        const float doa = gmv[t] * dOv;
+        T3[t * LDV + col] = doa;
+        atomicAdd(&red[L::V_DGAM_OUT + t], dOv * oa);
+        atomicAdd(&red[L::V_DGAM + t], doa * QR[t * LDV + col]);
+      }
+    }
+    __syncthreads();
+
+    // ---- adjoint of the auxiliary pass
+    {
+      float kd[MMk::RPT], a1[MMc::RPT];
+      MMk::run(Ks, LDK, 1, dR, LDV, 1, kd);
+      MMc::run(CC, 1, C, T3, LDV, 1, a1);  // M2^T dOa
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        T1[t * LDV + col] = a1[i] + wR[t] * kd[i];  // dE2
+        atomicAdd(&red[L::V_DWR + t], kd[i] * E2[t * LDV + col]);
+        QR[t * LDV + col] = Gam[t] * T3[t * LDV + col];  // dQR
+      }
+      float g1[MMg::RPT];
+      MMg::run(T3, LDV, 1, E2, 1, LDV, g1);  // dM2 = dOa E2^T (inclusive)
+#pragma unroll
+      for (int i = 0; i < MMg::RPT; ++i) {
+        const int t = MMg::row(i), ii = MMg::col();
+        if (ii <= t) atomicAdd(&acc[L::DM2 + t * C + ii], g1[i]);
+      }
+    }
+    __syncthreads();
+    const float *dRv = T1;
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, 1, C, T1, LDV, 1, a1);  // dX2 = Tg^T dE2
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) T2[MMc::row(i) * LDV + col] = a1[i];
+      __syncthreads();
+      float g1[MMg::RPT];
+      MMg::run(T2, LDV, 1, E2, 1, LDV, g1);  // dAg = -strict(dX2 E2^T)
+#pragma unroll
+      for (int i = 0; i < MMg::RPT; ++i) {
+        const int t = MMg::row(i), ii = MMg::col();
+        if (ii < t) atomicAdd(&acc[L::DAG + t * C + ii], -g1[i]);
+      }
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        T1[t * LDV + col] = -Gam[t] * a1[i];  // dKR
+        atomicAdd(&red[L::V_DGAM + t], -a1[i] * KR[t * LDV + col]);
+      }
+      dRv = T2;
+    }
+    // T3 <- diag(wR) E2 for dK += diag(wR) E2 dR^T
+    for (int e = tid; e < C * kBDVS; e += kThreads) {
+      const int t = e / kBDVS, jj = e % kBDVS;
+      T3[t * LDV + jj] = wR[t] * E2[t * LDV + jj];
+    }
+    __syncthreads();
+    float dKacc[MMd::RPT], dQacc[MMd::RPT];
+    {
+      float g1[MMd::RPT];
+      MMd::run(T3, LDV, 1, dR, 1, LDV, dKacc);
+      if (RDNV) {
+        MMd::run(T1, LDV, 1, R0, 1, LDV, g1);
+#pragma unroll
+        for (int i = 0; i < MMd::RPT; ++i) dKacc[i] += g1[i];
+      }
+      MMd::run(QR, LDV, 1, R0, 1, LDV, dQacc);
+      float s = 0.f;
+      for (int e = tid; e < DK * kBDVS; e += kThreads) {
+        const int i = e / kBDVS, jj = e % kBDVS;
+        s += dR[i * LDV + jj] * R0[i * LDV + jj];
+      }
+      atomicAdd(&red[L::V_DGAMC], s);
+    }
+    __syncthreads();
+    {  // dR0 = Gam_C dR + K^T dKR + Q^T dQR
+      float u1[MMu::RPT], u2[MMu::RPT];
+      MMu::run(Qs, 1, LDK, QR, LDV, 1, u2);
+      if (RDNV) MMu::run(Ks, 1, LDK, T1, LDV, 1, u1);
+#pragma unroll
+      for (int i = 0; i < MMu::RPT; ++i) {
+        const int r = MMu::row(i);
+        dR[r * LDV + col] = GamC * dR[r * LDV + col] + u2[i] + (RDNV ? u1[i] : 0.f);
+      }
+    }
+    // clip: dV = dRv * [|x| <= c] into T3 (dP = -dV)
+    for (int e = tid; e < C * kBDVS; e += kThreads) {
+      const int t = e / kBDVS, jj = e % kBDVS;
+      T3[t * LDV + jj] = fabsf(XR[t * LDV + jj]) <= clip ? dRv[t * LDV + jj] : 0.f;
+    }
+    __syncthreads();
+
+    // ---- adjoint of the base pass
+    {
+      float g1[MMg::RPT], g2[MMg::RPT];
+      MMg::run(dOs, LDV, 1, E, 1, LDV, g1);  // dMq = strict(dO E^T)
+      MMg::run(T3, LDV, 1, E, 1, LDV, g2);   // dAp = strict(dP E^T) = -strict(dV E^T)
+#pragma unroll
+      for (int i = 0; i < MMg::RPT; ++i) {
+        const int t = MMg::row(i), ii = MMg::col();
+        if (ii < t) {
+          atomicAdd(&acc[L::DMQ + t * C + ii], g1[i]);
+          atomicAdd(&acc[L::DAP + t * C + ii], -g2[i]);
+        }
+      }
+    }
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_MQ + e];
+    __syncthreads();
+    float de[MMc::RPT];
+    MMc::run(CC, 1, C, dOs, LDV, 1, de);  // Mq^T dO
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    __syncthreads();
+    {
+      float a1[MMc::RPT], kd[MMk::RPT];
+      MMc::run(CC, 1, C, T3, LDV, 1, a1);  // Ap^T dV  (= -Ap^T dP)
+      MMk::run(Ks, LDK, 1, dS, LDV, 1, kd);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        const float dv_ = T3[t * LDV + col];
+        T1[t * LDV + col] = de[i] - a1[i] + wS[t] * kd[i];  // dE
+        atomicAdd(&red[L::V_DWS + t], kd[i] * E[t * LDV + col]);
+        atomicAdd(&red[L::V_DGPREV + t], -dv_ * KS[t * LDV + col]);
+        T2[t * LDV + col] = -Gprev[t] * dv_;  // dKS (base part)
+        const float dOv = dOs[t * LDV + col];
+        atomicAdd(&red[L::V_DGAM + t], dOv * QS[t * LDV + col]);
+        QS[t * LDV + col] = Gam[t] * dOv;  // dQS
+      }
+    }
+    __syncthreads();
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, 1, C, T1, LDV, 1, a1);  // dX = Tb^T dE
+      __syncthreads();
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        T1[t * LDV + col] = a1[i];
+        T3[t * LDV + col] += a1[i];                  // dV += dX
+        T2[t * LDV + col] -= Gam[t] * a1[i];         // dKS -= Gam dX
+        atomicAdd(&red[L::V_DGAM + t], -a1[i] * KS[t * LDV + col]);
+      }
+      __syncthreads();
+      float g1[MMg::RPT];
+      MMg::run(T1, LDV, 1, E, 1, LDV, g1);  // dAb = -strict(dX E^T)
+#pragma unroll
+      for (int i = 0; i < MMg::RPT; ++i) {
+        const int t = MMg::row(i), ii = MMg::col();
+        if (ii < t) atomicAdd(&acc[L::DAB + t * C + ii], -g1[i]);
+      }
+    } else {
+      for (int e = tid; e < C * kBDVS; e += kThreads) {
+        const int t = e / kBDVS, jj = e % kBDVS;
+        T3[t * LDV + jj] += T1[t * LDV + jj];  // dV += dE
+      }
+    }
+    // XR <- diag(wS) E for dK += diag(wS) E dS^T
+    for (int e = tid; e < C * kBDVS; e += kThreads) {
+      const int t = e / kBDVS, jj = e % kBDVS;
+      XR[t * LDV + jj] = wS[t] * E[t * LDV + jj];
+    }
+    __syncthreads();
+    {
+      float g1[MMd::RPT];
+      MMd::run(XR, LDV, 1, dS, 1, LDV, g1);
+#pragma unroll
+      for (int i = 0; i < MMd::RPT; ++i) dKacc[i] += g1[i];
+      MMd::run(T2, LDV, 1, S0, 1, LDV, g1);
+#pragma unroll
+      for (int i = 0; i < MMd::RPT; ++i) dKacc[i] += g1[i];
+      MMd::run(QS, LDV, 1, S0, 1, LDV, g1);
+#pragma unroll
+      for (int i = 0; i < MMd::RPT; ++i) dQacc[i] += g1[i];
+      float s = 0.f;
+      for (int e = tid; e < DK * kBDVS; e += kThreads) {
+        const int i = e / kBDVS, jj = e % kBDVS;
+        s += dS[i * LDV + jj] * S0[i * LDV + jj];
+      }
+      atomicAdd(&red[L::V_DGAMC], s);
+    }
+    __syncthreads();
+    {  // dS0 = Gam_C dS + K^T dKS + Q^T dQS
+      float u1[MMu::RPT], u2[MMu::RPT];
+      MMu::run(Ks, 1, LDK, T2, LDV, 1, u1);
+      MMu::run(Qs, 1, LDK, QS, LDV, 1, u2);
+#pragma unroll
+      for (int i = 0; i < MMu::RPT; ++i) {
+        const int r = MMu::row(i);
+        dS[r * LDV + col] = GamC * dS[r * LDV + col] + u1[i] + u2[i];
+      }
+    }
+    // ---- outputs of this slice
+#pragma unroll
+    for (int i = 0; i < MMd::RPT; ++i) {
+      const int t = MMd::row(i), d = MMd::col();
+      atomicAdd(&acc[L::DKo + t * DK + d], dKacc[i]);
+      atomicAdd(&acc[L::DQo + t * DK + d], dQacc[i]);
+    }
+    for (int e = tid; e < C * kBDVS; e += kThreads) {
+      const int t = e / kBDVS, jj = e % kBDVS;
+      if (t < n) dv[((size_t)(b * T + t0 + t) * H + h) * DV + j0 + jj] = from_f32<InT>(T3[t * LDV + jj]);
+    }
+    __syncthreads();
+    for (int e = tid; e < 5 * C + 1; e += kThreads) atomicAdd(&acc[L::VEC + e], red[e]);
+  }
+  __syncthreads();
+  for (int e = tid; e < DK * kBDVS; e += kThreads) {
+    const int i = e / kBDVS, jj = e % kBDVS;
+    if (p.dS0) p.dS0[sbase + (size_t)i * DV + j0 + jj] = dS[i * LDV + jj];
+    if (p.dR0) p.dR0[sbase + (size_t)i * DV + j0 + jj] = dR[i * LDV + jj];
+  }
+}
+
+// ---------------------------------------------------------------- kernel 2
+template <int DK, bool RDNV, typename InT>
+__global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
+  constexpr int LDK = DK + 1;
+  constexpr int LDC = C + 1;
+  using L = Acc<DK>;
+  extern __shared__ float sm[];
+  float *Ks = sm;               // [C][LDK]
+  float *Qs = Ks + C * LDK;     // [C][LDK]
+  float *KK = Qs + C * LDK;     // [C][LDC]
+  float *QK = KK + C * LDC;     // [C][LDC]
+  float *dKK = QK + C * LDC;    // [C][LDC] symmetrised at the end
+  float *dQK = dKK + C * LDC;   // [C][LDC]
+  float *cum = dQK + C * LDC;   // [C]
+  float *cprev = cum + C;
+  float *bet = cprev + C;
+  float *gam = bet + C;
+  float *gg = gam + C;
+  float *dcum = gg + C;
+  float *dcprev = dcum + C;
+  float *dbet = dcprev + C;
+  float *dgam = dbet + C;
+
+  const int chunk = blockIdx.x;
+  const int NC = p.f.NC, T = p.f.T, H = p.f.H;
+  const int bh = chunk / NC, c = chunk % NC;
+  const int b = bh / H, h = bh % H;
+  const int t0 = c * C;
+  const int n = min(C, T - t0);
+  const int tid = threadIdx.x;
+  const InT *q = (const InT *)p.f.q;
+  const InT *k = (const InT *)p.f.k;
+  const float *acc = p.acc + (size_t)chunk * L::FLOATS;
+
+  for (int e = tid; e < C * DK; e += kThreads) {
+    const int t = e / DK, d = e % DK;
+    float kv = 0.f, qv = 0.f;
+    if (t < n) {
+      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+      kv = to_f32(k[off]);
+      qv = p.f.scale * to_f32(q[off]);
+    }
+    Ks[t * LDK + d] = kv;
+    Qs[t * LDK + d] = qv;
+  }
+  if (tid < C) {
+    const int t = tid;
+    float gv = 0.f, bv = 0.f, mv = 0.f;
+    if (t < n) {
+      const size_t off = (size_t)(b * T + t0 + t) * H + h;
+      gv = p.f.g[off];
+      bv = p.f.beta[off];
+      mv = p.f.gamma[off];
+    }
+    gg[t] = gv;
+    bet[t] = bv;
+    gam[t] = mv;
+    dcprev[t] = 0.f;
+    dbet[t] = 0.f;
+    dgam[t] = acc[L::VEC + L::V_DGAM_OUT + t];
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float s = 0.f;
+    for (int t = 0; t < C; ++t) {
+      cprev[t] = s;
+      s += gg[t];
+      cum[t] = s;
+    }
+  }
+  {
+    using MM = BlockMM<C, C, DK>;
+    float a[MM::RPT];
+    MM::run(Ks, LDK, 1, Ks, 1, LDK, a);
+#pragma unroll
+    for (int i = 0; i < MM::RPT; ++i) KK[MM::row(i) * LDC + MM::col()] = a[i];
+    MM::run(Qs, LDK, 1, Ks, 1, LDK, a);
+#pragma unroll
+    for (int i = 0; i < MM::RPT; ++i) QK[MM::row(i) * LDC + MM::col()] = a[i];
+  }
+  __syncthreads();
+  // per-row factors: Gam_t = e^{cum_t}, Gprev_t = e^{cprev_t}, w_t = rate_t e^{cum_C - cum_t}
+  if (tid < C) {
+    const int t = tid;
+    const float cC = cum[C - 1];
+    const float eC = expf(cC - cum[t]);
+    const float dwS = acc[L::VEC + L::V_DWS + t], dwR = acc[L::VEC + L::V_DWR + t];
+    dbet[t] += dwS * eC;
+    dgam[t] += dwR * eC;
+    dcum[t] = acc[L::VEC + L::V_DGAM + t] * expf(cum[t]) - (dwS * bet[t] + dwR * gam[t]) * eC;
+    dcprev[t] = acc[L::VEC + L::V_DGPREV + t] * expf(cprev[t]);
+  }
+  __syncthreads();
+  if (tid < C) {  // the chunk-end terms land on cum_C (= cum[C-1]; padding has g = 0)
+    float s = 0.f;
+    const float cC = cum[C - 1];
+    for (int t = 0; t < C; ++t) {
+      const float eC = expf(cC - cum[t]);
+      s += (acc[L::VEC + L::V_DWS + t] * bet[t] + acc[L::VEC + L::V_DWR + t] * gam[t]) * eC;
+    }
+    if (tid == C - 1) dcum[C - 1] += s + acc[L::VEC + L::V_DGAMC] * expf(cC);
+  }
+  __syncthreads();
+  // C x C gradients -> d(KK), d(QK), rates and cumulative log-decay
+  for (int e = tid; e < C * C; e += kThreads) {
+    const int t = e / C, i = e % C;
+    float dkk = 0.f, dqk = 0.f;
+    if (i <= t) {
+      const float dec = expf(cum[t] - cum[i]);
+      const float kk = KK[t * LDC + i], qk = QK[t * LDC + i];
+      float rowc = 0.f, rowp = 0.f, colc = 0.f;
+      // M2 (inclusive, gamma, QK)
+      {
+        const float dm = acc[L::DM2 + e];
+        const float m = dec * gam[i] * qk;
+        rowc += dm * m;
+        colc += dm * m;
+        atomicAdd(&dgam[i], dm * dec * qk);
+        dqk += dm * dec * gam[i];
+      }
+      if (i < t) {
+        const float decp = expf(cprev[t] - cum[i]);
+        {  // Ap (strict, beta, KK, previous-token decay)
+          const float dm = acc[L::DAP + e];
+          const float m = decp * bet[i] * kk;
+          rowp += dm * m;
+          colc += dm * m;
+          atomicAdd(&dbet[i], dm * decp * kk);
+          dkk += dm * decp * bet[i];
+        }
+        {  // Mq (strict, beta, QK)
+          const float dm = acc[L::DMQ + e];
+          const float m = dec * bet[i] * qk;
+          rowc += dm * m;
+          colc += dm * m;
+          atomicAdd(&dbet[i], dm * dec * qk);
+          dqk += dm * dec * bet[i];
+        }
+        if (RDNV) {
+          {  // Ab (strict, beta, KK)
+            const float dm = acc[L::DAB + e];
+            const float m = dec * bet[i] * kk;
+            rowc += dm * m;
+            colc += dm * m;
+            atomicAdd(&dbet[i], dm * dec * kk);
+            dkk += dm * dec * bet[i];
+          }
+          {  // Ag (strict, gamma, KK)
+            const float dm = acc[L::DAG + e];
+            const float m = dec * gam[i] * kk;
+            rowc += dm * m;
+            colc += dm * m;
+            atomicAdd(&dgam[i], dm * dec * kk);
+            dkk += dm * dec * gam[i];
+          }
+        }
+      }
+      atomicAdd(&dcum[t], rowc);
+      atomicAdd(&dcprev[t], rowp);
+      atomicAdd(&dcum[i], -colc);
+    }
+    dKK[t * LDC + i] = dkk;
+    dQK[t * LDC + i] = dqk;
+  }
+  __syncthreads();
+  // symmetrise: dK gets (dKK + dKK^T) K
+  for (int e = tid; e < C * C; e += kThreads) {
+    const int t = e / C, i = e % C;
+    if (i < t) {
+      const float s = dKK[t * LDC + i] + dKK[i * LDC + t];
+      dKK[t * LDC + i] = s;
+      dKK[i * LDC + t] = s;
+    } else if (i == t) {
+      dKK[t * LDC + i] *= 2.f;
+    }
+  }
+  __syncthreads();
+  {
+    using MM = BlockMM<C, DK, C>;
+    float a1[MM::RPT], a2[MM::RPT], a3[MM::RPT];
+    MM::run(dKK, LDC, 1, Ks, LDK, 1, a1);   // (dKK + dKK^T) K
+    MM::run(dQK, 1, LDC, Qs, LDK, 1, a2);   // dQK^T Q
+    MM::run(dQK, LDC, 1, Ks, LDK, 1, a3);   // dQK K
+    InT *dk = (InT *)p.dk;
+    InT *dq = (InT *)p.dq;
+#pragma unroll
+    for (int i = 0; i < MM::RPT; ++i) {
+      const int t = MM::row(i), d = MM::col();
+      if (t < n) {
+        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+        dk[off] = from_f32<InT>(acc[L::DKo + t * DK + d] + a1[i] + a2[i]);
+        dq[off] = from_f32<InT>(p.f.scale * (acc[L::DQo + t * DK + d] + a3[i]));
+      }
+    }
+  }
+  if (tid == 0) {  // dg_s = sum_{t>=s} dcum_t + sum_{t>s} dcprev_t
+    float s1 = 0.f, s2 = 0.f;
+    for (int t = C - 1; t >= 0; --t) {
+      s1 += dcum[t];
+      const float dgt = s1 + s2;
+      s2 += dcprev[t];
+      gg[t] = dgt;
+    }
+  }
+  __syncthreads();
+  if (tid < n) {
+    const size_t off = (size_t)(b * T + t0 + tid) * H + h;
+    p.dg[off] = gg[tid];
+    p.dbeta[off] = dbet[tid];
+    p.dgamma[off] = dgam[tid];
+  }
+}
+
+template <int DK>
+constexpr size_t scan_smem() {
+  return sizeof(float) * (2 * C * (DK + 1) + 4 * DK * LDV + C * C + 13 * C * LDV + 6 * C + C + 6 * C);
+}
+template <int DK>
+constexpr size_t finish_smem() {
+  return sizeof(float) * (2 * C * (DK + 1) + 4 * C * (C + 1) + 9 * C);
+}
+
+template <int DK, bool RDNV, typename InT>
+cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
+  auto scan = bwd_scan_kernel<DK, RDNV, InT>;
+  auto fin = bwd_finish_kernel<DK, RDNV, InT>;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(scan, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)scan_smem<DK>())) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)finish_smem<DK>())) != cudaSuccess)
+    return e;
+  scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p);
+  return cudaGetLastError();
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+struct BwdLayout {
+  size_t prep, acc, states, o, total;
+};
+
+BwdLayout layout(const rdn_bwd_args &a) {
+  const rdn_fwd_args &f = a.fwd;
+  const size_t nct = (size_t)f.B * f.H * ((f.T + C - 1) / C);
+  const size_t accf = f.Dk == 128 ? Acc<128>::FLOATS : Acc<64>::FLOATS;
+  BwdLayout l;
+  l.prep = align256(sizeof(float) * nct * kRecFloats);
+  l.acc = align256(sizeof(float) * nct * accf);
+  const bool need_states = f.S_chunks == nullptr;
+  l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
+  const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
+  l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
+  l.total = l.prep + l.acc + 2 * l.states + l.o;
+  return l;
+}
+
+}  // namespace
+
+BwdPlan plan_bwd(const rdn_bwd_args &a) {
+  if (a.fwd.T == 0) return BwdPlan{0};
+  return BwdPlan{layout(a).total};
+}
+
+cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
+  const rdn_fwd_args &f = a.fwd;
+  const size_t sbytes = sizeof(float) * (size_t)f.B * f.H * f.Dk * f.Dv;
+  if (f.T == 0) {  // no tokens: the initial-state gradients are the upstream ones
+    cudaError_t e = cudaSuccess;
+    if (a.dS0) e = a.dST ? cudaMemcpyAsync(a.dS0, a.dST, sbytes, cudaMemcpyDeviceToDevice, s)
+                         : cudaMemsetAsync(a.dS0, 0, sbytes, s);
+    if (e == cudaSuccess && a.dR0)
+      e = a.dRT ? cudaMemcpyAsync(a.dR0, a.dRT, sbytes, cudaMemcpyDeviceToDevice, s)
+                : cudaMemsetAsync(a.dR0, 0, sbytes, s);
+    return e;
+  }
+  const BwdLayout l = layout(a);
+  char *ws = (char *)a.workspace;
+  BwdParams p;
+  p.f = make_fwd_params(f);
+  p.f.ws = (float *)ws;
+  p.f.ST = p.f.RT = nullptr;
+  const bool bf = f.dtype == RDN_BF16;
+  const bool rdnv = true;
+  cudaError_t e;
+  if (f.S_chunks == nullptr) {  // recompute the chunk-start states
+    p.f.S_chunks = (float *)(ws + l.prep + l.acc);
+    p.f.R_chunks = (float *)(ws + l.prep + l.acc + l.states);
+    p.f.o = ws + l.prep + l.acc + 2 * l.states;
+    e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
+  } else {
+    e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, false, s);
+  }
+  if (e != cudaSuccess) return e;
+  p.Sc = p.f.S_chunks;
+  p.Rc = p.f.R_chunks;
+  p.acc = (float *)(ws + l.prep);
+  if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
+  p.dO = a.dO;
+  p.dST = a.dST;
+  p.dRT = a.dRT;
+  p.dq = a.dq;
+  p.dk = a.dk;
+  p.dv = a.dv;
+  p.dg = a.dg;
+  p.dbeta = a.dbeta;
+  p.dgamma = a.dgamma;
+  p.dS0 = a.dS0;
+  p.dR0 = a.dR0;
+  if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
+  return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
+}
+
+}  // namespace rdn

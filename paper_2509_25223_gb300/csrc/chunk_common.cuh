@@ -1,0 +1,76 @@
+// chunk_common.cuh -- layout of the per-chunk records shared by the
+// chunkwise forward and backward, and a block-level fp32 product helper.
+#pragma once
+#include "common.cuh"
+
+namespace rdn {
+
+constexpr int C = kChunk;
+constexpr int kThreads = 256;
+constexpr int kDVS = 32;  // value columns per scan CTA
+
+// Per-chunk workspace record written by chunk_prep (floats).
+constexpr int kCC = C * C;
+constexpr int OFF_TB = 0, OFF_TG = kCC, OFF_AP = 2 * kCC, OFF_MQ = 3 * kCC, OFF_M2 = 4 * kCC;
+constexpr int OFF_VEC = 5 * kCC;
+// vectors: Gam, Gprev, alpha, wS, wR, then GamC at [5*C]
+constexpr int V_GAM = 0, V_GPREV = C, V_ALPHA = 2 * C, V_WS = 3 * C, V_WR = 4 * C, V_GAMC = 5 * C;
+constexpr int kRecFloats = OFF_VEC + 6 * C;
+
+// Block-level fp32 product over shared memory: the calling thread gets
+// acc[i] = sum_k A(m_i, k) B(k, n) for n = tid % N and m_i = tid / N + i * (256 / N).
+// A(m,k) = A[m*a_m + k*a_k], B(k,n) = B[k*b_k + n*b_n].  With N >= 32 the lanes
+// of a warp share m, so A reads are broadcasts.
+template <int M, int N, int K>
+struct BlockMM {
+  static constexpr int RG = kThreads / N;
+  static constexpr int RPT = M / RG;
+  static_assert(kThreads % N == 0 && M % RG == 0, "tile");
+  __device__ static __forceinline__ void run(const float *A, int a_m, int a_k, const float *B,
+                                             int b_k, int b_n, float (&acc)[RPT]) {
+    const int n = threadIdx.x % N, rg = threadIdx.x / N;
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) acc[i] = 0.f;
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+      const float bv = B[k * b_k + n * b_n];
+#pragma unroll
+      for (int i = 0; i < RPT; ++i) acc[i] = fmaf(A[(rg + i * RG) * a_m + k * a_k], bv, acc[i]);
+    }
+  }
+  __device__ static __forceinline__ int row(int i) { return threadIdx.x / N + i * RG; }
+  __device__ static __forceinline__ int col() { return threadIdx.x % N; }
+};
+
+struct FwdParams {
+  int B, T, H, NC;
+  const void *q, *k, *v;
+  const float *g, *beta, *gamma;
+  float clip, scale;
+  const float *S0, *R0;
+  void *o;
+  float *ST, *RT, *S_chunks, *R_chunks;
+  float *ws;  // NC*B*H records of kRecFloats
+};
+
+
+inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
+  FwdParams p;
+  p.B = a.B; p.T = a.T; p.H = a.H;
+  p.NC = (a.T + C - 1) / C;
+  p.q = a.q; p.k = a.k; p.v = a.v;
+  p.g = a.g; p.beta = a.beta; p.gamma = a.gamma;
+  p.clip = a.clip; p.scale = a.scale;
+  p.S0 = a.S0; p.R0 = a.R0;
+  p.o = a.o;
+  p.ST = a.ST; p.RT = a.RT; p.S_chunks = a.S_chunks; p.R_chunks = a.R_chunks;
+  p.ws = nullptr;
+  return p;
+}
+
+// Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
+// scan kernel (outputs, optional chunk-start states).
+cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, bool do_prep,
+                             bool do_scan, cudaStream_t s);
+
+}  // namespace rdn

@@ -1,0 +1,428 @@
+// chunk_fwd.cu -- chunkwise-parallel forward of RLA / RDN (Section 3.4),
+// fp32 SIMT path.
+//
+// Chunk algebra (C = 64 tokens; b_t = in-chunk cumulative log-decay,
+// Gam_t = exp(b_t), Gprev_t = exp(b_{t-1}), b_0 = 0; states stored [d_k][d_v]):
+//
+//   RDN writes the delta rule as S_t = a_t S_{t-1} + beta_t k_t e_t^T with the
+//   delta error e_t = v_t - a_t S_{t-1}^T k_t (Section 2.2).  Unrolling the
+//   chunk gives (I + A) E = V - diag(Gam) K S0 with the strictly lower
+//   A[t,i] = exp(b_t - b_i) beta_i (k_t.k_i), so E = T (V - diag(Gam) K S0),
+//   T = (I + A)^-1 (the UT form of the WY representation).  RLA: E = V.
+//
+//   P   = diag(Gprev) K S0 + Ap E,   Ap[t,i] = exp(b_{t-1}-b_i) beta_i (k_t.k_i), i<t
+//         (P_t = S_{t-1}^T k_t, the undecayed prediction of Section 3.3)
+//   Ob  = diag(Gam) Q S0 + Mq E,     Mq[t,i] = exp(b_t-b_i) beta_i (q_t.k_i), i<t
+//         (Ob_t = a_t S_{t-1}^T q_t, the base prediction)
+//   S_C = Gam_C S0 + K^T diag(beta_i exp(b_C - b_i)) E
+//   r   = clip(V - P, -c, c)                                   (Section 3.3)
+//   the auxiliary pass repeats this with values r, rate gamma, state R; its
+//   read-out includes token t:  Oa = diag(Gam) Q R0 + M2 E2,
+//         M2[t,i] = exp(b_t-b_i) gamma_i (q_t.k_i), i<=t
+//   o   = Ob + diag(gamma) Oa.
+//
+// Kernel 1 (chunk_prep): one CTA per chunk -- everything that does not depend
+// on the state: the Gram matrices, the masked/decayed matrices Ap, Mq, M2 and
+// (RDN) the two unit-lower inverses T_beta, T_gamma by forward substitution.
+// Kernel 2 (chunk_scan): one CTA per (b, h, 32-column slice of d_v) -- the
+// sequential pass over chunks carrying S and R slices in shared memory.  Each
+// value column is independent (the clip is elementwise), so slicing d_v is
+// exact; only the prep work is shared between slices.
+#include "chunk_common.cuh"
+
+namespace rdn {
+namespace {
+
+// ---------------------------------------------------------------- kernel 1
+template <int DK, bool RDNV, typename InT>
+__global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
+  constexpr int LDK = DK + 1;
+  constexpr int LDC = C + 1;
+  extern __shared__ float sm[];
+  float *Ks = sm;                 // [C][LDK]
+  float *Qs = Ks + C * LDK;       // [C][LDK]
+  float *KK = Qs + C * LDK;       // [C][LDC]
+  float *QK = KK + C * LDC;       // [C][LDC]
+  float *Ab = QK + C * LDC;       // [C][LDC]
+  float *Ag = Ab + C * LDC;       // [C][LDC]
+  float *Tb = Ag + C * LDC;       // [C][LDC]
+  float *Tg = Tb + C * LDC;       // [C][LDC]
+  float *cum = Tg + C * LDC;      // [C]
+  float *cprev = cum + C;         // [C]
+  float *bet = cprev + C;         // [C]
+  float *gam = bet + C;           // [C]
+  float *gg = gam + C;            // [C]
+
+  const int chunk = blockIdx.x;
+  const int bh = chunk / p.NC, c = chunk % p.NC;
+  const int b = bh / p.H, h = bh % p.H;
+  const int t0 = c * C;
+  const int n = min(C, p.T - t0);
+  const int tid = threadIdx.x;
+  const InT *q = (const InT *)p.q;
+  const InT *k = (const InT *)p.k;
+
+  for (int e = tid; e < C * DK; e += kThreads) {
+    const int t = e / DK, d = e % DK;
+    float kv = 0.f, qv = 0.f;
+    if (t < n) {
+      const size_t off = ((size_t)(b * p.T + t0 + t) * p.H + h) * DK + d;
+      kv = to_f32(k[off]);
+      qv = p.scale * to_f32(q[off]);
+    }
+    Ks[t * LDK + d] = kv;
+    Qs[t * LDK + d] = qv;
+  }
+  if (tid < C) {
+    const int t = tid;
+    float gv = 0.f, bv = 0.f, mv = 0.f;
+    if (t < n) {
+      const size_t off = (size_t)(b * p.T + t0 + t) * p.H + h;
+      gv = p.g[off];
+      bv = p.beta[off];
+      mv = p.gamma[off];
+    }
+    gg[t] = gv;
+    bet[t] = bv;
+    gam[t] = mv;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float s = 0.f;
+    for (int t = 0; t < C; ++t) {
+      cprev[t] = s;
+      s += gg[t];
+      cum[t] = s;
+    }
+  }
+  // Gram matrices K K^T and Q K^T
+  {
+    using MM = BlockMM<C, C, DK>;
+    float acc[MM::RPT];
+    MM::run(Ks, LDK, 1, Ks, 1, LDK, acc);
+#pragma unroll
+    for (int i = 0; i < MM::RPT; ++i) KK[MM::row(i) * LDC + MM::col()] = acc[i];
+    MM::run(Qs, LDK, 1, Ks, 1, LDK, acc);
+#pragma unroll
+    for (int i = 0; i < MM::RPT; ++i) QK[MM::row(i) * LDC + MM::col()] = acc[i];
+  }
+  __syncthreads();
+  float *rec = p.ws + (size_t)chunk * kRecFloats;
+  for (int e = tid; e < C * C; e += kThreads) {
+    const int t = e / C, i = e % C;
+    float ap = 0.f, mq = 0.f, m2 = 0.f, ab = 0.f, ag = 0.f;
+    if (i <= t) {
+      const float dec = expf(cum[t] - cum[i]);
+      m2 = dec * gam[i] * QK[t * LDC + i];
+      if (i < t) {
+        ap = expf(cprev[t] - cum[i]) * bet[i] * KK[t * LDC + i];
+        mq = dec * bet[i] * QK[t * LDC + i];
+        ab = dec * bet[i] * KK[t * LDC + i];
+        ag = dec * gam[i] * KK[t * LDC + i];
+      }
+    }
+    rec[OFF_AP + e] = ap;
+    rec[OFF_MQ + e] = mq;
+    rec[OFF_M2 + e] = m2;
+    if (RDNV) {
+      Ab[t * LDC + i] = ab;
+      Ag[t * LDC + i] = ag;
+    }
+  }
+  if (tid < C) {
+    const int t = tid;
+    const float cC = cum[C - 1];
+    rec[OFF_VEC + V_GAM + t] = expf(cum[t]);
+    rec[OFF_VEC + V_GPREV + t] = expf(cprev[t]);
+    rec[OFF_VEC + V_ALPHA + t] = expf(gg[t]);
+    rec[OFF_VEC + V_WS + t] = bet[t] * expf(cC - cum[t]);
+    rec[OFF_VEC + V_WR + t] = gam[t] * expf(cC - cum[t]);
+    if (t == 0) rec[OFF_VEC + V_GAMC] = expf(cC);
+  }
+  if (RDNV) {
+    __syncthreads();
+    // (I + A)^-1 by forward substitution, one column per thread:
+    // threads 0..63 invert I + A_beta, threads 64..127 invert I + A_gamma.
+    if (tid < 2 * C) {
+      const int j = tid % C;
+      const float *A = tid < C ? Ab : Ag;
+      float *Tm = tid < C ? Tb : Tg;
+      for (int t = 0; t < C; ++t) {
+        float s = (t == j) ? 1.f : 0.f;
+        for (int i = j; i < t; ++i) s = fmaf(-A[t * LDC + i], Tm[i * LDC + j], s);
+        Tm[t * LDC + j] = (t < j) ? 0.f : s;
+      }
+    }
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) {
+      const int t = e / C, i = e % C;
+      rec[OFF_TB + e] = Tb[t * LDC + i];
+      rec[OFF_TG + e] = Tg[t * LDC + i];
+    }
+  }
+}
+
+// ---------------------------------------------------------------- kernel 2
+template <int DK, bool RDNV, typename InT>
+__global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
+  constexpr int DV = DK;
+  extern __shared__ float sm[];
+  float *Ks = sm;                 // [C][DK]
+  float *Qs = Ks + C * DK;        // [C][DK]
+  float *Ss = Qs + C * DK;        // [DK][kDVS]
+  float *Rs = Ss + DK * kDVS;     // [DK][kDVS]
+  float *Vs = Rs + DK * kDVS;     // [C][kDVS]
+  float *CC = Vs + C * kDVS;      // [C][C]
+  float *KS = CC + C * C;         // [C][kDVS]
+  float *QS = KS + C * kDVS;
+  float *Es = QS + C * kDVS;
+  float *Ps = Es + C * kDVS;
+  float *Ob = Ps + C * kDVS;
+  float *Ws = Ob + C * kDVS;
+  float *vec = Ws + C * kDVS;     // [6*C]
+
+  const int bh = blockIdx.x;
+  const int b = bh / p.H, h = bh % p.H;
+  const int j0 = blockIdx.y * kDVS;
+  const int tid = threadIdx.x;
+  const InT *q = (const InT *)p.q;
+  const InT *k = (const InT *)p.k;
+  const InT *v = (const InT *)p.v;
+  InT *o = (InT *)p.o;
+  const float clip = p.clip;
+
+  const size_t sbase = (size_t)bh * DK * DV;
+  for (int e = tid; e < DK * kDVS; e += kThreads) {
+    const int i = e / kDVS, jj = e % kDVS;
+    Ss[e] = p.S0 ? p.S0[sbase + (size_t)i * DV + j0 + jj] : 0.f;
+    Rs[e] = p.R0 ? p.R0[sbase + (size_t)i * DV + j0 + jj] : 0.f;
+  }
+
+  for (int c = 0; c < p.NC; ++c) {
+    const int t0 = c * C;
+    const int n = min(C, p.T - t0);
+    const float *rec = p.ws + ((size_t)bh * p.NC + c) * kRecFloats;
+    __syncthreads();  // previous chunk done with every buffer
+    if (p.S_chunks) {
+      float *sc = p.S_chunks + ((size_t)bh * p.NC + c) * DK * DV;
+      float *rc = p.R_chunks + ((size_t)bh * p.NC + c) * DK * DV;
+      for (int e = tid; e < DK * kDVS; e += kThreads) {
+        const int i = e / kDVS, jj = e % kDVS;
+        sc[(size_t)i * DV + j0 + jj] = Ss[e];
+        rc[(size_t)i * DV + j0 + jj] = Rs[e];
+      }
+    }
+    for (int e = tid; e < C * DK; e += kThreads) {
+      const int t = e / DK, d = e % DK;
+      float kv = 0.f, qv = 0.f;
+      if (t < n) {
+        const size_t off = ((size_t)(b * p.T + t0 + t) * p.H + h) * DK + d;
+        kv = to_f32(k[off]);
+        qv = p.scale * to_f32(q[off]);
+      }
+      Ks[e] = kv;
+      Qs[e] = qv;
+    }
+    for (int e = tid; e < C * kDVS; e += kThreads) {
+      const int t = e / kDVS, jj = e % kDVS;
+      Vs[e] = t < n ? to_f32(v[((size_t)(b * p.T + t0 + t) * p.H + h) * DV + j0 + jj]) : 0.f;
+    }
+    for (int e = tid; e < 6 * C; e += kThreads) vec[e] = rec[OFF_VEC + e];
+    __syncthreads();
+    const float *Gam = vec + V_GAM, *Gprev = vec + V_GPREV;
+    const float *wS = vec + V_WS, *wR = vec + V_WR;
+    const float GamC = vec[V_GAMC];
+
+    using MMk = BlockMM<C, kDVS, DK>;  // [C x DK] @ [DK x DVS]
+    using MMc = BlockMM<C, kDVS, C>;   // [C x C] @ [C x DVS]
+    using MMu = BlockMM<DK, kDVS, C>;  // [DK x C] @ [C x DVS]
+    const int col = MMk::col();
+    {
+      float a1[MMk::RPT], a2[MMk::RPT];
+      MMk::run(Ks, DK, 1, Ss, kDVS, 1, a1);
+      MMk::run(Qs, DK, 1, Ss, kDVS, 1, a2);
+#pragma unroll
+      for (int i = 0; i < MMk::RPT; ++i) {
+        const int t = MMk::row(i);
+        KS[t * kDVS + col] = a1[i];
+        QS[t * kDVS + col] = a2[i];
+        if (RDNV) Ws[t * kDVS + col] = Vs[t * kDVS + col] - Gam[t] * a1[i];
+      }
+    }
+    const float *E = Vs;
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, Ws, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) Es[MMc::row(i) * kDVS + col] = a1[i];
+      E = Es;
+    }
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    __syncthreads();
+    {
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, E, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        const float pt = Gprev[t] * KS[t * kDVS + col] + a1[i];
+        Ps[t * kDVS + col] = clampf(Vs[t * kDVS + col] - pt, clip);  // r, Section 3.3
+      }
+    }
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_MQ + e];
+    __syncthreads();
+    {
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, E, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        Ob[t * kDVS + col] = Gam[t] * QS[t * kDVS + col] + a1[i];
+      }
+    }
+    // S_C = Gam_C S0 + K^T diag(wS) E   (W = wS * E)
+    for (int e = tid; e < C * kDVS; e += kThreads) Ws[e] = wS[e / kDVS] * E[e];
+    __syncthreads();
+    {
+      float a1[MMu::RPT];
+      MMu::run(Ks, 1, DK, Ws, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMu::RPT; ++i) {
+        const int r = MMu::row(i);
+        Ss[r * kDVS + col] = GamC * Ss[r * kDVS + col] + a1[i];
+      }
+    }
+    // auxiliary pass: values r (in Ps), rate gamma, state R
+    {
+      float a1[MMk::RPT], a2[MMk::RPT];
+      MMk::run(Ks, DK, 1, Rs, kDVS, 1, a1);
+      MMk::run(Qs, DK, 1, Rs, kDVS, 1, a2);
+      __syncthreads();  // every thread done reading Ws / CC of the S pass
+#pragma unroll
+      for (int i = 0; i < MMk::RPT; ++i) {
+        const int t = MMk::row(i);
+        QS[t * kDVS + col] = a2[i];  // Q R0
+        if (RDNV) Ws[t * kDVS + col] = Ps[t * kDVS + col] - Gam[t] * a1[i];
+      }
+    }
+    const float *E2 = Ps;
+    if (RDNV) {
+      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      __syncthreads();
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, Ws, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) Es[MMc::row(i) * kDVS + col] = a1[i];
+      E2 = Es;
+    }
+    __syncthreads();
+    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_M2 + e];
+    __syncthreads();
+    {
+      float a1[MMc::RPT];
+      MMc::run(CC, C, 1, E2, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMc::RPT; ++i) {
+        const int t = MMc::row(i);
+        if (t < n) {
+          const float gm = p.gamma[(size_t)(b * p.T + t0 + t) * p.H + h];
+          const float oa = Gam[t] * QS[t * kDVS + col] + a1[i];
+          o[((size_t)(b * p.T + t0 + t) * p.H + h) * DV + j0 + col] =
+              from_f32<InT>(Ob[t * kDVS + col] + gm * oa);
+        }
+      }
+    }
+    // R_C = Gam_C R0 + K^T diag(wR) E2
+    for (int e = tid; e < C * kDVS; e += kThreads) Ws[e] = wR[e / kDVS] * E2[e];
+    __syncthreads();
+    {
+      float a1[MMu::RPT];
+      MMu::run(Ks, 1, DK, Ws, kDVS, 1, a1);
+#pragma unroll
+      for (int i = 0; i < MMu::RPT; ++i) {
+        const int r = MMu::row(i);
+        Rs[r * kDVS + col] = GamC * Rs[r * kDVS + col] + a1[i];
+      }
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < DK * kDVS; e += kThreads) {
+    const int i = e / kDVS, jj = e % kDVS;
+    if (p.ST) p.ST[sbase + (size_t)i * DV + j0 + jj] = Ss[e];
+    if (p.RT) p.RT[sbase + (size_t)i * DV + j0 + jj] = Rs[e];
+  }
+}
+
+template <int DK>
+constexpr size_t prep_smem() {
+  return sizeof(float) * (2 * C * (DK + 1) + 6 * C * (C + 1) + 5 * C);
+}
+template <int DK>
+constexpr size_t scan_smem() {
+  return sizeof(float) * (2 * C * DK + 2 * DK * kDVS + C * kDVS + C * C + 6 * C * kDVS + 6 * C);
+}
+
+template <int DK, bool RDNV, typename InT>
+cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_scan) {
+  auto prep = chunk_prep_kernel<DK, RDNV, InT>;
+  auto scan = chunk_scan_kernel<DK, RDNV, InT>;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(prep, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)prep_smem<DK>())) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(scan, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)scan_smem<DK>())) != cudaSuccess)
+    return e;
+  if (do_prep) {
+    prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (do_scan) scan<<<dim3(p.B * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, bool do_prep,
+                             bool do_scan, cudaStream_t s) {
+  if (DK == 128) {
+    if (rdnv) return bf16 ? launch_t<128, true, __nv_bfloat16>(p, s, do_prep, do_scan)
+                          : launch_t<128, true, float>(p, s, do_prep, do_scan);
+    return bf16 ? launch_t<128, false, __nv_bfloat16>(p, s, do_prep, do_scan)
+                : launch_t<128, false, float>(p, s, do_prep, do_scan);
+  }
+  if (rdnv) return bf16 ? launch_t<64, true, __nv_bfloat16>(p, s, do_prep, do_scan)
+                        : launch_t<64, true, float>(p, s, do_prep, do_scan);
+  return bf16 ? launch_t<64, false, __nv_bfloat16>(p, s, do_prep, do_scan)
+              : launch_t<64, false, float>(p, s, do_prep, do_scan);
+}
+
+FwdPlan plan_fwd(const rdn_fwd_args &a, int /*variant*/) {
+  FwdPlan pl;
+  pl.NC = (a.T + C - 1) / C;
+  pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
+  pl.total_bytes = pl.prep_bytes * (size_t)a.B * a.H * pl.NC;
+  return pl;
+}
+
+cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
+  const size_t sbytes = sizeof(float) * (size_t)a.B * a.H * a.Dk * a.Dv;
+  if (a.T == 0) {  // no tokens: the final states are the initial ones
+    cudaError_t e = cudaSuccess;
+    if (a.ST) e = a.S0 ? cudaMemcpyAsync(a.ST, a.S0, sbytes, cudaMemcpyDeviceToDevice, s)
+                       : cudaMemsetAsync(a.ST, 0, sbytes, s);
+    if (e == cudaSuccess && a.RT)
+      e = a.R0 ? cudaMemcpyAsync(a.RT, a.R0, sbytes, cudaMemcpyDeviceToDevice, s)
+               : cudaMemsetAsync(a.RT, 0, sbytes, s);
+    return e;
+  }
+  FwdParams p = make_fwd_params(a);
+  p.ws = (float *)a.workspace;
+  return launch_fwd_parts(p, a.Dk, variant == 1, a.dtype == RDN_BF16, true, true, s);
+}
+
+}  // namespace rdn

@@ -1,0 +1,49 @@
+// common.cuh -- small device helpers shared by the RLA/RDN kernels.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "rdn.h"
+
+namespace rdn {
+
+// Chunk length of the chunkwise-parallel forms (tokens per chunk).
+constexpr int kChunk = 64;
+
+template <typename T> __device__ __forceinline__ float to_f32(T x);
+template <> __device__ __forceinline__ float to_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) {
+  return __bfloat162float(x);
+}
+
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+  return __float2bfloat16_rn(x);
+}
+
+__device__ __forceinline__ float clampf(float x, float c) { return fminf(fmaxf(x, -c), c); }
+
+}  // namespace rdn
+
+// Internal launchers (defined in the kernel translation units, called by
+// api.cu after argument validation).  Each returns cudaGetLastError() of its
+// launches.
+namespace rdn {
+cudaError_t launch_decode(const rdn_decode_args &a, cudaStream_t s);
+
+struct FwdPlan {
+  int NC;                // chunks per sequence
+  size_t prep_bytes;     // per-chunk precomputed matrices
+  size_t total_bytes;    // workspace the forward needs
+};
+FwdPlan plan_fwd(const rdn_fwd_args &a, int variant);
+cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s);
+
+struct BwdPlan {
+  size_t total_bytes;
+};
+BwdPlan plan_bwd(const rdn_bwd_args &a);
+cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s);
+}  // namespace rdn

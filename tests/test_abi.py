@@ -1,0 +1,124 @@
+"""The C-ABI library: builds, loads, exports what include/rdn.h declares, and
+rejects bad arguments with a status code before touching the GPU (CPU only)."""
+import ctypes
+import math
+import os
+import re
+import subprocess
+
+import pytest
+
+import paper_2509_25223_gb300 as rdn
+from paper_2509_25223_gb300 import _abi
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _header_functions():
+    src = open(os.path.join(ROOT, "include", "rdn.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(\w+)\s*\(", src, flags=re.M)))
+
+
+def test_header_matches_binding():
+    assert _header_functions() == sorted(_abi.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol():
+    lib = _abi.load()
+    out = subprocess.run(["nm", "-D", "--defined-only", _abi.lib_path()], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {ln.split()[-1] for ln in out.splitlines() if ln.strip()}
+    for name in _header_functions():
+        assert name in exported, name
+        assert getattr(lib, name) is not None
+    assert lib.rdn_version().decode().startswith("rdn-gb300")
+
+
+def _fwd_args(**over):
+    a = _abi.FwdArgs()
+    a.B, a.T, a.H, a.Dk, a.Dv = 2, 128, 4, 128, 128
+    a.dtype = _abi.RDN_BF16
+    a.clip, a.scale = 1.0, 1.0
+    for k, v in over.items():
+        setattr(a, k, v)
+    return a
+
+
+def _status(fn, a):
+    lib = _abi.load()
+    return getattr(lib, fn)(ctypes.byref(a), None)
+
+
+FAKE = ctypes.c_void_p(0x10000)  # aligned, never dereferenced: validation fails first
+
+
+@pytest.mark.parametrize("fn", ["rla_fwd", "rdn_fwd"])
+def test_fwd_validation(fn):
+    lib = _abi.load()
+    assert lib[fn](None, None) == 1
+    assert _status(fn, _fwd_args(B=0)) == 1
+    assert _status(fn, _fwd_args(T=-1)) == 1
+    assert _status(fn, _fwd_args(Dk=96, Dv=96)) == 2
+    assert _status(fn, _fwd_args(Dk=128, Dv=64)) == 2
+    assert _status(fn, _fwd_args(dtype=7)) == 2
+    assert _status(fn, _fwd_args(clip=-1.0)) == 1
+    assert _status(fn, _fwd_args(clip=float("nan"))) == 1
+    assert _status(fn, _fwd_args(flags=1)) == 2
+    assert _status(fn, _fwd_args()) == 1  # q is NULL
+    assert "q is NULL" in lib.rdn_last_error().decode()
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE, o=FAKE)
+    mis = dict(ok)
+    mis["v"] = ctypes.c_void_p(0x10004)
+    assert _status(fn, _fwd_args(**mis)) == 6
+    assert _status(fn, _fwd_args(S_chunks=FAKE, **ok)) == 1  # R_chunks missing
+    assert _status(fn, _fwd_args(**ok)) == 5  # no workspace
+    assert "workspace" in lib.rdn_last_error().decode()
+
+
+def test_workspace_size_queries():
+    lib = _abi.load()
+    n = ctypes.c_size_t(0)
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args()), ctypes.byref(n)) == 0
+    assert n.value > 0
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args(Dk=32, Dv=32)), ctypes.byref(n)) == 2
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args()), None) == 1
+
+
+def test_decode_validation():
+    lib = _abi.load()
+    a = _abi.DecodeArgs()
+    a.N, a.H, a.Dk, a.Dv, a.dtype, a.variant = 4, 2, 128, 128, _abi.RDN_BF16, 1
+    a.clip, a.scale = 1.0, 1.0
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 1  # NULL pointers
+    for f in ("q", "k", "v", "g", "beta", "gamma", "o"):
+        setattr(a, f, FAKE)
+    a.S = ctypes.c_void_p(0x20000)
+    a.R = ctypes.c_void_p(0x20000)
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 1  # S aliases R
+    assert "alias" in lib.rdn_last_error().decode()
+    a.variant = 3
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 1
+    a.variant = 1
+    a.clip = -2.0
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 1
+    a.clip = math.inf
+    a.Dk = a.Dv = 256
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 2
+
+
+def test_bwd_validation():
+    lib = _abi.load()
+    b = _abi.BwdArgs()
+    b.fwd = _fwd_args()
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 1
+    b.fwd = _fwd_args(clip=-0.5)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 1
+
+
+def test_binding_rejects_cpu_tensors():
+    import torch
+    x = torch.zeros(1, 64, 1, 64)
+    g = torch.zeros(1, 64, 1)
+    with pytest.raises(ValueError):
+        rdn.rla_fwd(x, x, x, g, g, g)

@@ -1,0 +1,138 @@
+"""Parity of rdn_bwd with the oracle's back-propagation through time.
+
+The derivative of the clip jumps at |v - S_{t-1}k| = c, so before each
+comparison the inputs are conditioned with the oracle (v moved, in steps
+representable in the input dtype, until every fp64 residual is at least a
+margin away from c).  The clip mask is then unique at tolerance level and so
+is the gradient; see oracle.clip_margin_condition."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2509_25223_gb300 as rdn
+from rdn_synthetic import WORKLOADS, make_inputs, make_workload_inputs
+from tests.parity_util import as64, assert_close
+
+pytestmark = pytest.mark.gpu
+
+NAMES = ("q", "k", "v", "g", "beta", "gamma")
+GRADS = ("dq", "dk", "dv", "dg", "dbeta", "dgamma", "dS0", "dR0")
+MARGIN = 1e-2
+
+
+def _condition(x, clip, dtype, heads=None):
+    """Move v (in place on the device tensor) so the fp64 clip decisions have
+    a margin; only the listed (b, h) heads when given."""
+    sel = heads if heads is not None else [(b, h) for b in range(x["q"].shape[0])
+                                           for h in range(x["q"].shape[2])]
+    for b, h in sel:
+        sl = {n: as64(x[n][b:b + 1, :, h:h + 1]) for n in NAMES}
+        S0 = None if x["S0"] is None else as64(x["S0"][b:b + 1, h:h + 1])
+        R0 = None if x["R0"] is None else as64(x["R0"][b:b + 1, h:h + 1])
+        v2, _ = oracle.clip_margin_condition(oracle.RDN, sl["q"], sl["k"], sl["v"], sl["g"],
+                                             sl["beta"], sl["gamma"], clip, S0, R0,
+                                             margin=MARGIN, quant=dtype)
+        x["v"][b, :, h] = torch.from_numpy(v2[0, :, 0]).to(x["v"].dtype).to(x["v"].device)
+
+
+def _ref(x, clip, dST=None, dRT=None, heads=None):
+    if heads is None:
+        return oracle.rdn_bwd(*(as64(x[n]) for n in NAMES), clip, as64(x["S0"]), as64(x["R0"]),
+                              as64(x["dO"]), as64(dST), as64(dRT))
+    outs = []
+    for b, h in heads:
+        sl = lambda t: None if t is None else as64(t[b:b + 1, :, h:h + 1])
+        st = lambda t: None if t is None else as64(t[b:b + 1, h:h + 1])
+        outs.append(oracle.rdn_bwd(*(sl(x[n]) for n in NAMES), clip, st(x["S0"]), st(x["R0"]),
+                                   sl(x["dO"]), st(dST), st(dRT)))
+    return outs
+
+
+def _gpu(x, clip, dST=None, dRT=None, **kw):
+    d = rdn.rdn_bwd(*(x[n] for n in NAMES), x["dO"], clip=clip, S0=x["S0"], R0=x["R0"],
+                    dST=dST, dRT=dRT, **kw)
+    torch.cuda.synchronize()
+    return d
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("T", [1, 64, 65, 200])
+def test_bwd_small(dtype, D, T):
+    clip = 1.0
+    x = make_inputs(2, T, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    gen = torch.Generator(device="cpu").manual_seed(7)
+    dST = torch.randn(x["S0"].shape, generator=gen).cuda()
+    dRT = torch.randn(x["R0"].shape, generator=gen).cuda()
+    _condition(x, clip, dtype)
+    d = _gpu(x, clip, dST, dRT)
+    ref = _ref(x, clip, dST, dRT)
+    for name in GRADS:
+        assert_close(d[name], ref[name], dtype, name)
+
+
+def test_bwd_zero_upstream_state_grads_and_no_init_state():
+    x = make_inputs(1, 100, 2, 128, dtype="bf16", nonzero_state=False, with_grad_out=True,
+                    device="cuda")
+    _condition(x, 1.0, "bf16")
+    d = _gpu(x, 1.0)
+    ref = _ref(x, 1.0)
+    for name in GRADS:
+        assert_close(d[name], ref[name], "bf16", name)
+
+
+@pytest.mark.parametrize("clip", [0.3, float("inf")])
+def test_bwd_clip_values(clip):
+    x = make_inputs(1, 130, 2, 128, dtype="bf16", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    _condition(x, clip, "bf16")
+    d = _gpu(x, clip)
+    ref = _ref(x, clip)
+    for name in GRADS:
+        assert_close(d[name], ref[name], "bf16", name)
+
+
+def test_bwd_reuses_forward_chunk_states():
+    """Passing the forward's chunk-start states gives the same gradients as
+    letting the backward recompute them."""
+    x = make_inputs(2, 192, 2, 128, dtype="bf16", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                                    return_chunk_states=True)
+    d1 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc)
+    d2 = _gpu(x, 1.0)
+    # the per-chunk accumulators sum d_v slices with fp32 atomics, so two runs
+    # may differ by fp32 rounding, i.e. by one bf16 ulp after the final store
+    for name in GRADS:
+        torch.testing.assert_close(d1[name].float(), d2[name].float(), atol=1e-5, rtol=8e-3)
+
+
+def test_bwd_full_size_sampled():
+    """The bench's fwd+bwd workload (B=8, H=16, T=4096, D=128, bf16) in the
+    bench's launch configuration (chunk states from rdn_fwd); the oracle
+    checks sampled heads."""
+    w = WORKLOADS["rdn_fwd_bwd_bf16_B8H16T4096D128"]
+    x = make_workload_inputs(w, device="cuda")
+    heads = [(0, 0), (5, 9), (7, 15)]
+    _condition(x, 1.0, "bf16", heads=heads)
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, return_chunk_states=True)
+    d = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc)
+    for name in GRADS:
+        assert torch.isfinite(d[name].float()).all(), name
+    for (b, h), ref in zip(heads, _ref(x, 1.0, heads=heads)):
+        for name in GRADS:
+            g = d[name][b:b + 1, h:h + 1] if name in ("dS0", "dR0") else d[name][b:b + 1, :, h:h + 1]
+            assert_close(g, ref[name], "bf16", f"{name} ({b},{h})")
+
+
+def test_dalpha_from_dg():
+    """dL/dalpha = dg / alpha (the library returns the log-decay gradient)."""
+    x = make_inputs(1, 70, 1, 64, dtype="f32", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    _condition(x, 1.0, "f32")
+    d = _gpu(x, 1.0)
+    ref = _ref(x, 1.0)
+    alpha = np.exp(as64(x["g"]))
+    np.testing.assert_allclose(as64(d["dg"]) / alpha, ref["dg"] / alpha, atol=2e-4, rtol=1e-4)

@@ -493,3 +493,23 @@ def test_split_sequence_continuation():
     np.testing.assert_allclose(np.concatenate([oa, ob], 1), o, atol=1e-13)
     np.testing.assert_allclose(Sb, ST, atol=1e-13)
     np.testing.assert_allclose(Rb, RT, atol=1e-13)
+
+
+@pytest.mark.parametrize("variant,name", [(RLA, "rla"), (RDN, "rdn")])
+@pytest.mark.parametrize("C", [1, 16, 64])
+def test_chunkwise_backward_equals_bptt(variant, name, C):
+    """The reverse-mode chunk algebra (test helper) equals the oracle's
+    back-propagation through time (and so, via the autograd pins, the exact
+    gradient)."""
+    from tests.chunk_algebra import chunk_bwd
+    x = _inputs(B=1, T=100, H=2, D=8, Dv=6)
+    x["v"] = x["v"] * 1.5
+    c = 0.8
+    dST = np.random.default_rng(1).standard_normal(x["S0"].shape)
+    dRT = np.random.default_rng(2).standard_normal(x["R0"].shape)
+    ref = oracle.bwd(variant, x["q"], x["k"], x["v"], x["g"], x["beta"], x["gamma"], c,
+                     x["S0"], x["R0"], x["dO"], dST, dRT, scale=0.7)
+    got = chunk_bwd(name, x["q"], x["k"], x["v"], x["g"], x["beta"], x["gamma"], c, x["S0"],
+                    x["R0"], x["dO"], dST, dRT, C=C, scale=0.7)
+    for key in ref:
+        np.testing.assert_allclose(got[key], ref[key], atol=1e-10, err_msg=key)
