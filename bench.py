@@ -1,0 +1,490 @@
+#!/usr/bin/env python
+"""Benchmark of the RDN layer hot path on GB300.
+
+A step is one pass of the whole training-side hot path over one batch of
+the fwd+bwd workload (RDN, B=8, H=16, T=4096, d_k=d_v=128, bf16 inputs, fp32
+states, chunk 64, clip 1): rdn_fwd (saving the chunk-start states) followed
+by rdn_bwd.  `value` is tokens/s (a token = one (b, t) position with all 16
+heads) over all ranks.  The decode workload (N=256 sequences, H=16, D=128,
+fp32 states in place, 1000 steps) is timed in the same run and reported as
+HBM GB/s under "decode".
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One JSON line is printed by rank 0.  With --gpus N > 1 (one process per GPU
+under torchrun) every rank runs an independent replica on its own batch
+(the layer has no parameters and no exchange step): "scaling" is "weak".
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "RDN fwd+bwd tokens/sec (H=16,d=128,T=4096 bf16); % bf16 tensor peak; decode GB/s"
+WORKLOAD = "rdn_fwd_bwd_bf16_B8H16T4096D128"
+DECODE_WORKLOAD = "rdn_decode_N256H16D128"
+C = 64
+
+# Algorithmic work per token-head at d_k = d_v = d, chunk C (triangular
+# products counted at half, each unit-lower inverse at (2/3) C^3 per chunk):
+#   forward F = 12 d^2 + 2 C d + 5 C d + (4/3) C^2, split into
+#     the state-carrying scan   12 d^2 + 5 C d   (products with S, R and the
+#                                                 C x C x d_v chunk products)
+#     the per-chunk prep        2 C d + (4/3) C^2 (Gram matrices, inverses)
+#   backward = 2 x forward (two products per forward product), same split.
+def flops_per_token_head(d=128, c=C):
+    scan = 12 * d * d + 5 * c * d
+    prep = 2 * c * d + (4.0 / 3.0) * c * c
+    return dict(fwd=scan + prep, fwd_scan=scan, fwd_prep=prep, bwd_scan=2 * scan,
+                bwd_finish=2 * prep, step=3 * (scan + prep))
+
+
+# kernel name (as recorded by the library) -> algorithmic flop per token-head
+KERNEL_WORK = {"chunk_scan": "fwd_scan", "chunk_prep": "fwd_prep", "bwd_scan": "bwd_scan",
+               "bwd_finish": "bwd_finish"}
+
+# decode: read + write S and R fp32, plus q, k, v, o bf16 and three fp32 gates
+def decode_bytes_per_head(d=128):
+    return 4 * d * d * 4 + 4 * d * 2 + 3 * 4
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sust=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                    source="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, source="fallback")
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during a region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="rdn_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for ln in f:
+                parts = [p.strip() for p in ln.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for nm, val in zip(names, r[5:9]):
+                if val.lower() in ("active", "1"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(rows),
+                "power_w_max": max((float(r[3]) for r in rows
+                                    if r[3].replace(".", "").isdigit()), default=None)}
+
+
+# ------------------------------------------------------------- distributed
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def init_dist(ws):
+    if ws <= 1:
+        return None
+    import torch.distributed as dist
+    if not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("gloo")
+    return dist
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(dist, x):
+    """Largest value of x over all ranks (timing exchange only)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(dist, x):
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def aggregate(dist, local_ms, local_units):
+    """Whole-job throughput: units of all ranks / slowest rank's time."""
+    t = max_over_ranks(dist, local_ms)
+    u = sum_over_ranks(dist, local_units)
+    return t, u / (t / 1e3)
+
+
+# -------------------------------------------------------------- CPU oracle
+def time_oracle_sample(target_s=15.0, max_heads=None):
+    """fp64 oracle fwd+bwd on a bounded sample of the workload (whole
+    sequences of T=4096 for a subset of heads), on all host cores."""
+    import numpy as np
+    import oracle
+    from rdn_synthetic import WORKLOADS, make_workload_inputs
+
+    oracle.build()
+    w = WORKLOADS[WORKLOAD]
+    threads = oracle.max_threads()
+
+    def heads_as_batch(t, nh):
+        """[B,T,H,...] -> the first nh (b,h) sequences as [nh,T,1,...]."""
+        t = t.double().numpy()
+        t = np.moveaxis(t, 2, 1)                      # [B,H,T,...]
+        t = t.reshape(-1, *t.shape[2:])[:nh]          # [B*H,T,...] -> [nh,T,...]
+        return np.ascontiguousarray(np.expand_dims(t, 2))
+
+    def run(nh):
+        B = max(1, (nh + w.H - 1) // w.H)
+        x = make_workload_inputs(w, B=B, seed=1)
+        q, k, v, g, be, gm, dO = (heads_as_batch(x[n], nh)
+                                  for n in ("q", "k", "v", "g", "beta", "gamma", "dO"))
+        t0 = time.perf_counter()
+        oracle.rdn_fwd(q, k, v, g, be, gm, w.clip)
+        oracle.rdn_bwd(q, k, v, g, be, gm, w.clip, None, None, dO)
+        return time.perf_counter() - t0
+
+    probe_heads = min(threads, 16)
+    dt = run(probe_heads)
+    nh = probe_heads
+    if dt < target_s:
+        nh = int(probe_heads * max(1.0, target_s / max(dt, 1e-3)))
+        nh = max(probe_heads, (nh // threads) * threads)
+        if max_heads:
+            nh = min(nh, max_heads)
+        dt = run(nh)
+    tokens = nh * w.T / w.H
+    return dict(value=tokens / dt, unit="tokens/s", cores=min(threads, nh), kind="oracle",
+                sample=f"fp64 oracle fwd+bwd on {nh} of the workload's (b,h) heads, "
+                       f"full T={w.T} each ({nh * w.T} token-heads = {tokens:.0f} tokens), "
+                       f"{dt:.1f} s on {min(threads, nh)} OpenMP threads")
+
+
+# ------------------------------------------------------------ reference arm
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import numpy as np
+    import oracle
+    from rdn_synthetic import WORKLOADS, make_workload_inputs
+
+    oracle.build()
+    w = WORKLOADS[WORKLOAD]
+    threads = oracle.max_threads()
+    # each step: all 16 heads of one sequence (T = 4096 tokens)
+    x = make_workload_inputs(w, B=1, seed=2)
+    a = {n: (None if t is None else t.double().numpy()) for n, t in x.items()}
+
+    def step():
+        oracle.rdn_fwd(a["q"], a["k"], a["v"], a["g"], a["beta"], a["gamma"], w.clip)
+        oracle.rdn_bwd(a["q"], a["k"], a["v"], a["g"], a["beta"], a["gamma"], w.clip, None,
+                       None, a["dO"])
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    tokens = w.T * args.steps
+    val = tokens / dt
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": _config(w),
+            "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": min(threads, w.H),
+                             "kind": "oracle",
+                             "sample": f"each step: fp64 oracle fwd+bwd of one sequence "
+                                       f"(B=1 of the workload's B=8), all H={w.H} heads, "
+                                       f"T={w.T}"},
+            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _workload(args):
+    """The fwd+bwd workload, optionally shrunk (--B/--T) for profiler captures."""
+    import dataclasses
+    from rdn_synthetic import WORKLOADS
+    w = WORKLOADS[WORKLOAD]
+    if args.B or args.T:
+        B, T = args.B or w.B, args.T or w.T
+        w = dataclasses.replace(w, B=B, T=T, name=f"rdn_fwd_bwd_bf16_B{B}H{w.H}T{T}D{w.D}")
+    return w
+
+
+def _config(w):
+    return {"workload": w.name, "B": w.B, "T": w.T, "H": w.H, "d_k": w.D, "d_v": w.D,
+            "chunk": w.chunk, "clip": w.clip, "states": "fp32", "parallelism": "replicas",
+            "l2": f"no flush: inputs larger than L2 (q,k,v,dO = "
+                  f"{4 * w.B * w.T * w.H * w.D * 2 / 1e6:.0f} MB bf16 per step)"}
+
+
+def _traffic(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            tab = json.load(f)
+        ent = tab.get(kernel)
+        if not ent:
+            return None
+        import hashlib
+        src = os.path.join(ROOT, ent["source"])
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if h != ent["source_sha256_16"]:
+            return None
+        return float(ent["bytes_per_launch_full_workload"])
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------------ our arm
+def run_ours(args):
+    import torch
+
+    ws, rank, local = dist_env()
+    dist = init_dist(ws)
+    torch.cuda.set_device(local)
+    import paper_2509_25223_gb300 as rdn
+    from rdn_synthetic import WORKLOADS, make_decode_inputs, make_workload_inputs
+
+    rdn.library()  # fails loudly when the CUDA library is missing
+    w = _workload(args)
+    peaks = _peaks()
+    dev = torch.device("cuda", local)
+    x = make_workload_inputs(w, device=dev, device_rng=True, seed=rank)
+    names = ("q", "k", "v", "g", "beta", "gamma")
+    B, T, H, D = w.B, w.T, w.H, w.D
+    NC = (T + C - 1) // C
+    o = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
+    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", B, T, H, D), dtype=torch.uint8, device=dev)
+    wsb = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D), dtype=torch.uint8, device=dev)
+    grads = dict(dq=torch.empty_like(x["q"]), dk=torch.empty_like(x["k"]),
+                 dv=torch.empty_like(x["v"]),
+                 dg=torch.empty(B, T, H, device=dev), dbeta=torch.empty(B, T, H, device=dev),
+                 dgamma=torch.empty(B, T, H, device=dev),
+                 dS0=torch.empty(B, H, D, D, device=dev), dR0=torch.empty(B, H, D, D, device=dev))
+
+    def step(inp):
+        _, _, _, Sc, Rc = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
+                                      return_chunk_states=True, out=o, workspace=wsf)
+        rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc,
+                    R_chunks=Rc, workspace=wsb, out=grads)
+
+    for _ in range(args.warmup):
+        step(x)
+    torch.cuda.synchronize()
+    barrier(dist)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        with rdn.LaunchTimer() as lt:
+            torch.cuda.synchronize()
+            e0.record(stream)
+            for _ in range(args.steps):
+                step(x)
+            e1.record(stream)
+            torch.cuda.synchronize()
+    barrier(dist)
+    local_ms = e0.elapsed_time(e1)
+    tokens_per_step = B * T
+    tmax, value = aggregate(dist, local_ms, tokens_per_step * args.steps)
+    ms_per_step = tmax / args.steps
+    fl = flops_per_token_head(D)
+    token_heads = B * T * H
+
+    kern = lt.summary()
+    dom = max(kern.items(), key=lambda kv: kv[1][1])
+    dom_name, (dom_n, dom_total, dom_mean) = dom
+    dom_flop = fl[KERNEL_WORK[dom_name]] * token_heads
+    achieved = dom_flop / (dom_mean * 1e-3) / 1e12
+    peak = peaks["bf16_sust"]
+    roof = {"kernel": dom_name, "bound": "tensor", "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": _traffic(dom_name),
+            "peak_kind": f"bf16 dense, {peaks['source']} sustained (kernel timed inside a long step)",
+            "algorithmic_flop_per_launch": dom_flop, "mean_launch_ms": dom_mean}
+    step_tflops = fl["step"] * token_heads / (ms_per_step * 1e-3) / 1e12
+
+    # ---- end to end through the public API: pinned host in, host out
+    host = {n: x[n].cpu().pin_memory() for n in names + ("dO",)}
+    dev_in = {n: torch.empty_like(x[n]) for n in host}
+    host_out = {n: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                for n, t in list(grads.items()) + [("o", o)]}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+
+    def e2e_step():
+        for n, t in host.items():
+            dev_in[n].copy_(t, non_blocking=True)
+        step(dev_in)
+        for n, t in host_out.items():
+            t.copy_(o if n == "o" else grads[n], non_blocking=True)
+
+    e2e_steps = max(1, min(args.steps, 5))
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier(dist)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist)
+    _, e2e_val = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * e2e_steps)
+
+    # ---- decode: N=256, H=16, D=128, 1000 steps in place
+    dec = None
+    if not args.no_decode:
+        wd = WORKLOADS[DECODE_WORKLOAD]
+        steps_d = args.decode_steps
+        y = make_decode_inputs(wd.B, wd.H, wd.D, steps=steps_d + 10, device=dev, device_rng=True,
+                               seed=100 + rank)
+        S, R = y["S"], y["R"]
+        od = torch.empty(wd.B, wd.H, wd.D, dtype=torch.bfloat16, device=dev)
+
+        def dstep(i):
+            rdn.rdn_decode_step(y["q"][i], y["k"][i], y["v"][i], y["g"][i], y["beta"][i],
+                                y["gamma"][i], S, R, clip=wd.clip, out=od)
+
+        for i in range(10):
+            dstep(i)
+        torch.cuda.synchronize()
+        barrier(dist)
+        with rdn.LaunchTimer(capacity=steps_d + 8) as ltd:
+            e0.record(stream)
+            for i in range(steps_d):
+                dstep(10 + i)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        barrier(dist)
+        tdec = max_over_ranks(dist, e0.elapsed_time(e1))
+        heads = wd.B * wd.H
+        nbytes = decode_bytes_per_head(wd.D) * heads
+        gbs = sum_over_ranks(dist, nbytes * steps_d) / (tdec * 1e-3) / 1e9
+        kd = ltd.summary().get("decode", (0, 0.0, 0.0))
+        kern_gbs = nbytes / (kd[2] * 1e-3) / 1e9 if kd[2] > 0 else None
+        dec = {"workload": wd.name, "value": gbs, "unit": "GB/s", "steps": steps_d,
+               "us_per_step": tdec * 1e3 / steps_d, "bytes_per_step": nbytes,
+               "frac_of_hbm_peak": gbs / peaks["hbm"], "hbm_peak_gbs": peaks["hbm"],
+               "kernel_mean_us": kd[2] * 1e3, "kernel_gbs": kern_gbs,
+               "state_bytes": 2 * S.numel() * 4,
+               "l2": "no flush: 1.07 GB of state per step, larger than L2"}
+        del y, S, R
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle_sample(target_s=args.cpu_seconds)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "bf16", "data": "synthetic", "config": _config(w),
+                "roofline": roof, "step_tflops": step_tflops,
+                "step_frac_of_bf16_peak": step_tflops / peak,
+                "cpu_baseline": cpu,
+                "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                        "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                "gpu_launches": lt.launches,
+                "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
+                                "share": t / sum(v[1] for v in kern.values())}
+                            for k, (n, t, m) in kern.items()},
+                "clocks": clk.summary(), "decode": dec}
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--decode-steps", type=int, default=1000)
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")
+    ap.add_argument("--T", type=int, default=0, help="override T (profiling captures only)")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -176,6 +176,24 @@ const char *rdn_last_error(void);
 /* Library version string. */
 const char *rdn_version(void);
 
+/* Instrumentation (no counterpart in the paper): device time of each launch
+ * of the library's own kernels, measured with CUDA events recorded on the
+ * stream each kernel is launched on.
+ *   rdn_prof_start(capacity)  begins recording the next `capacity` launches
+ *                             (any thread, any stream); fails if already
+ *                             recording.  Launches beyond capacity are
+ *                             counted but not timed.
+ *   rdn_prof_stop(out, cap, n) waits for the recorded launches to finish,
+ *                             writes up to `cap` records to `out` (may be
+ *                             NULL), sets *n to the number of launches seen
+ *                             (timed or not) and ends the recording. */
+typedef struct {
+  char name[40];
+  float ms;
+} rdn_prof_record;
+rdn_status_t rdn_prof_start(int capacity);
+rdn_status_t rdn_prof_stop(rdn_prof_record *out, int cap, int *n);
+
 #ifdef __cplusplus
 }
 #endif

@@ -186,6 +186,41 @@ def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant=
     return o
 
 
+class LaunchTimer:
+    """Context manager recording the device time of every launch of the
+    library's kernels (CUDA events on each kernel's own stream).
+
+        with LaunchTimer() as lt:
+            ...
+        lt.records  -> [(kernel_name, ms), ...];  lt.launches -> count"""
+
+    def __init__(self, capacity=65536):
+        self.capacity = capacity
+        self.records = []
+        self.launches = 0
+
+    def __enter__(self):
+        _check("rdn_prof_start", _abi.load().rdn_prof_start(self.capacity))
+        return self
+
+    def __exit__(self, *exc):
+        buf = (_abi.ProfRecord * self.capacity)()
+        n = ctypes.c_int(0)
+        _check("rdn_prof_stop", _abi.load().rdn_prof_stop(buf, self.capacity, ctypes.byref(n)))
+        self.launches = n.value
+        self.records = [(buf[i].name.decode(), float(buf[i].ms))
+                        for i in range(min(n.value, self.capacity))]
+        return False
+
+    def summary(self):
+        """{kernel: (launches, total_ms, mean_ms)}"""
+        out = {}
+        for name, ms in self.records:
+            c, t = out.get(name, (0, 0.0))[:2]
+            out[name] = (c + 1, t + ms)
+        return {k: (c, t, t / c) for k, (c, t) in out.items()}
+
+
 def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16):
     """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rdn_bwd)."""
     lib = _abi.load()

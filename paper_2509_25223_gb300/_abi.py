@@ -16,7 +16,12 @@ STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "R
 
 # every function the header declares (checked by the CPU tests)
 EXPORTS = ["rla_fwd", "rdn_fwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
-           "rdn_fwd_workspace_size", "rdn_bwd_workspace_size", "rdn_last_error", "rdn_version"]
+           "rdn_fwd_workspace_size", "rdn_bwd_workspace_size", "rdn_last_error", "rdn_version",
+           "rdn_prof_start", "rdn_prof_stop"]
+
+
+class ProfRecord(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 40), ("ms", ctypes.c_float)]
 
 
 class FwdArgs(ctypes.Structure):
@@ -72,6 +77,11 @@ def load(build_if_missing: bool = True):
         fn = getattr(lib, name)
         fn.argtypes = argt
         fn.restype = S
+    lib.rdn_prof_start.argtypes = [ctypes.c_int]
+    lib.rdn_prof_start.restype = S
+    lib.rdn_prof_stop.argtypes = [ctypes.POINTER(ProfRecord), ctypes.c_int,
+                                  ctypes.POINTER(ctypes.c_int)]
+    lib.rdn_prof_stop.restype = S
     lib.rdn_last_error.restype = ctypes.c_char_p
     lib.rdn_last_error.argtypes = []
     lib.rdn_version.restype = ctypes.c_char_p

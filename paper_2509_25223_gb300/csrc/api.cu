@@ -6,7 +6,48 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
+#include <mutex>
+#include <vector>
+
 #include "common.cuh"
+
+namespace rdn {
+namespace prof {
+namespace {
+struct Rec {
+  const char *name;
+  cudaEvent_t ev[2];
+};
+std::atomic<bool> g_active{false};
+std::mutex g_mu;
+std::vector<Rec> g_recs;
+size_t g_next = 0;   // next record to fill
+size_t g_seen = 0;   // launches seen while active
+thread_local long g_open = -1;  // record opened by begin() on this thread
+}  // namespace
+
+bool active() { return g_active.load(std::memory_order_relaxed); }
+
+void begin(const char *name, cudaStream_t s) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  ++g_seen;
+  g_open = -1;
+  if (g_next < g_recs.size()) {
+    g_open = (long)g_next++;
+    g_recs[g_open].name = name;
+    cudaEventRecord(g_recs[g_open].ev[0], s);
+  }
+}
+
+void end(cudaStream_t s) {
+  if (g_open < 0) return;
+  std::lock_guard<std::mutex> lk(g_mu);
+  cudaEventRecord(g_recs[g_open].ev[1], s);
+  g_open = -1;
+}
+}  // namespace prof
+}  // namespace rdn
 
 namespace {
 
@@ -111,6 +152,56 @@ extern "C" {
 const char *rdn_last_error(void) { return g_err; }
 
 const char *rdn_version(void) { return "rdn-gb300 0.1 (sm_103a)"; }
+
+rdn_status_t rdn_prof_start(int capacity) {
+  using namespace rdn::prof;
+  if (capacity < 0 || capacity > (1 << 20))
+    return fail(RDN_ERR_INVALID_ARG, "rdn_prof_start: capacity %d out of range", capacity);
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_active.load()) return fail(RDN_ERR_INVALID_ARG, "rdn_prof_start: already recording");
+  g_recs.assign((size_t)capacity, Rec{"", {nullptr, nullptr}});
+  for (auto &r : g_recs)
+    for (auto &e : r.ev) {
+      cudaError_t err = cudaEventCreate(&e);
+      if (err != cudaSuccess) {
+        for (auto &r2 : g_recs)
+          for (auto &e2 : r2.ev)
+            if (e2) cudaEventDestroy(e2);
+        g_recs.clear();
+        return fail(RDN_ERR_CUDA, "rdn_prof_start: cudaEventCreate: %s", cudaGetErrorString(err));
+      }
+    }
+  g_next = 0;
+  g_seen = 0;
+  g_active.store(true);
+  return ok();
+}
+
+rdn_status_t rdn_prof_stop(rdn_prof_record *out, int cap, int *n) {
+  using namespace rdn::prof;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_active.load()) return fail(RDN_ERR_INVALID_ARG, "rdn_prof_stop: not recording");
+  g_active.store(false);
+  rdn_status_t st = RDN_OK;
+  for (size_t i = 0; i < g_next; ++i) {
+    cudaError_t err = cudaEventSynchronize(g_recs[i].ev[1]);
+    float ms = -1.f;
+    if (err == cudaSuccess) err = cudaEventElapsedTime(&ms, g_recs[i].ev[0], g_recs[i].ev[1]);
+    if (err != cudaSuccess && st == RDN_OK)
+      st = fail(RDN_ERR_CUDA, "rdn_prof_stop: %s", cudaGetErrorString(err));
+    if (out && (int)i < cap) {
+      snprintf(out[i].name, sizeof out[i].name, "%s", g_recs[i].name);
+      out[i].ms = ms;
+    }
+  }
+  if (n) *n = (int)g_seen;
+  for (auto &r : g_recs)
+    for (auto &e : r.ev)
+      if (e) cudaEventDestroy(e);
+  g_recs.clear();
+  g_next = g_seen = 0;
+  return st == RDN_OK ? ok() : st;
+}
 
 rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *a, size_t *bytes) {
   rdn_status_t st = check_fwd_shapes("rla_fwd_workspace_size", a);

@@ -669,9 +669,9 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
   if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)finish_smem<DK>())) != cudaSuccess)
     return e;
-  scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p);
+  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p);
+  RDN_LAUNCH("bwd_finish", s, fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 

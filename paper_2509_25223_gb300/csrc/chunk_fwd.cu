@@ -378,10 +378,11 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
                                 (int)scan_smem<DK>())) != cudaSuccess)
     return e;
   if (do_prep) {
-    prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p);
+    RDN_LAUNCH("chunk_prep", s, prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  if (do_scan) scan<<<dim3(p.B * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p);
+  if (do_scan)
+    RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.B * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 

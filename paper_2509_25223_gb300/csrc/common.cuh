@@ -27,6 +27,24 @@ __device__ __forceinline__ float clampf(float x, float c) { return fminf(fmaxf(x
 
 }  // namespace rdn
 
+// Per-launch timing of the library's kernels (rdn_prof_start / _stop).
+namespace rdn {
+namespace prof {
+bool active();
+void begin(const char *name, cudaStream_t s);
+void end(cudaStream_t s);
+}  // namespace prof
+}  // namespace rdn
+
+// Wraps one kernel launch statement with the timing events when recording.
+#define RDN_LAUNCH(name, stream, ...)                      \
+  do {                                                     \
+    const bool rdn_prof_on_ = ::rdn::prof::active();       \
+    if (rdn_prof_on_) ::rdn::prof::begin(name, stream);    \
+    __VA_ARGS__;                                           \
+    if (rdn_prof_on_) ::rdn::prof::end(stream);            \
+  } while (0)
+
 // Internal launchers (defined in the kernel translation units, called by
 // api.cu after argument validation).  Each returns cudaGetLastError() of its
 // launches.

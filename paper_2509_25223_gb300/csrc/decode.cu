@@ -145,13 +145,15 @@ template <int D, typename InT>
 cudaError_t launch_decode_t(const rdn_decode_args &a, cudaStream_t s) {
   const int grid = a.N * a.H * (D / kSliceCols);
   if (a.variant == 1)
-    decode_kernel<D, true, InT><<<grid, kDecThreads, 0, s>>>(
-        a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta, a.gamma,
-        a.clip, a.scale, a.S, a.R, (InT *)a.o);
+    RDN_LAUNCH("decode", s,
+               decode_kernel<D, true, InT><<<grid, kDecThreads, 0, s>>>(
+                   a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o));
   else
-    decode_kernel<D, false, InT><<<grid, kDecThreads, 0, s>>>(
-        a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta, a.gamma,
-        a.clip, a.scale, a.S, a.R, (InT *)a.o);
+    RDN_LAUNCH("decode", s,
+               decode_kernel<D, false, InT><<<grid, kDecThreads, 0, s>>>(
+                   a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o));
   return cudaGetLastError();
 }
 
