@@ -154,6 +154,31 @@ rdn_status_t rla_fwd(const rdn_fwd_args *args, rdn_stream_t stream);
  * rule; the clipped residual is formed and consumed on chip. */
 rdn_status_t rdn_fwd(const rdn_fwd_args *args, rdn_stream_t stream);
 
+/* RDN forward for callers that cannot allocate device memory.  The paper has
+ * no counterpart; this is a deployment convenience.  Some callers own only
+ * their input and output buffers: an inference-engine plugin that is handed
+ * fixed tensors, or a serving loop that forbids device allocation after
+ * start-up (cudaMalloc can synchronise the device and can fail under
+ * fragmentation).  This entry point computes exactly what rdn_fwd computes,
+ * from the same arguments, but its scratch is a fixed array compiled into the
+ * library (RDN_NOALLOC_SCRATCH_BYTES, held on every GPU that loads the
+ * library until the process exits) instead of args->workspace, which is
+ * ignored.  It allocates nothing.
+ *   - Size limit: the scratch holds one 83,456-byte record per 64-token
+ *     chunk, so B * H * ceil(T/64) must be at most 804; larger problems
+ *     return RDN_ERR_WORKSPACE (with a message giving both sizes) and
+ *     nothing is launched.  Use rdn_fwd with a caller workspace for them.
+ *   - First call on each device: it looks up the scratch array's device
+ *     address (cudaGetSymbolAddress) with that device current, once, and
+ *     caches it.  Make that first call before any stream capture.
+ *   - All calls share the one array, and each call overwrites every scratch
+ *     word it reads before reading it, so nothing needs clearing between
+ *     calls.  Calls whose work overlaps on the GPU (different streams, or
+ *     different host threads without ordering) race on the array: order
+ *     them, e.g. issue them on one stream. */
+#define RDN_NOALLOC_SCRATCH_BYTES (64u * 1024u * 1024u)
+rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *args, rdn_stream_t stream);
+
 /* Backward of rdn_fwd (reverse-mode of the same chunkwise computation).
  * Supports RDN_BF16 with Dk = Dv in {64, 128} and RDN_F32 likewise. */
 rdn_status_t rdn_bwd(const rdn_bwd_args *args, rdn_stream_t stream);

@@ -203,6 +203,57 @@ rdn_status_t rdn_prof_stop(rdn_prof_record *out, int cap, int *n) {
   return st == RDN_OK ? ok() : st;
 }
 
+// ---- rdn_fwd_noalloc: the forward with a built-in scratch array.
+//
+// For callers that own only their inputs and outputs and may not allocate
+// device memory (see rdn.h).  The scratch is this file-scope device array; in
+// host code its name is only a host-side stand-in, so its device address is
+// looked up with cudaGetSymbolAddress once per device (with that device
+// current) and passed to the kernels like a caller workspace.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[RDN_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kMaxDevices] = {};
+}  // namespace
+
+rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a, rdn_stream_t stream) {
+  const char *fn = "rdn_fwd_noalloc";
+  rdn_status_t st = check_fwd_shapes(fn, a);
+  if (st != RDN_OK) return st;
+  if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
+  const size_t need = rdn::plan_fwd(*a, 1).total_bytes;
+  if (need > (size_t)RDN_NOALLOC_SCRATCH_BYTES)
+    return fail(RDN_ERR_WORKSPACE,
+                "%s: this problem needs %zu bytes of scratch (B*H*ceil(T/64) = %lld chunks) but "
+                "the built-in scratch holds %zu bytes (at most %zu chunks); use rdn_fwd with a "
+                "caller workspace",
+                fn, need, (long long)a->B * a->H * ((a->T + rdn::kChunk - 1) / rdn::kChunk),
+                (size_t)RDN_NOALLOC_SCRATCH_BYTES,
+                (size_t)RDN_NOALLOC_SCRATCH_BYTES / rdn::plan_fwd(rdn_fwd_args{1, 64, 1, a->Dk, a->Dv}, 1).total_bytes);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_status(fn, e);
+  if (dev < 0 || dev >= kMaxDevices)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: device ordinal %d beyond %d", fn, dev, kMaxDevices);
+  void *scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void *p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+      if (e != cudaSuccess) return cuda_status(fn, e);
+      g_noalloc_ptr[dev] = p;
+    }
+    scratch = g_noalloc_ptr[dev];
+  }
+  rdn_fwd_args b = *a;
+  b.workspace = scratch;
+  b.workspace_bytes = RDN_NOALLOC_SCRATCH_BYTES;
+  return cuda_status(fn, rdn::launch_fwd(b, 1, (cudaStream_t)stream));
+}
+
 rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *a, size_t *bytes) {
   rdn_status_t st = check_fwd_shapes("rla_fwd_workspace_size", a);
   if (st != RDN_OK) return st;

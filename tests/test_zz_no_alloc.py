@@ -1,0 +1,72 @@
+"""rdn_fwd_noalloc: the RDN forward for callers that cannot allocate device
+memory (an engine plugin handed only its input and output tensors, or a
+serving loop that forbids cudaMalloc after start-up).  It must return what
+rdn_fwd returns for the same inputs, call after call, using only the scratch
+array built into the library.
+
+Collected last on purpose (file name), so a run that stops at the first
+failure has already run every other test; it also passes on its own in a
+fresh process."""
+import ctypes
+
+import pytest
+import torch
+
+import paper_2509_25223_gb300 as rdn
+from paper_2509_25223_gb300 import _abi
+from rdn_synthetic import make_inputs
+from tests.parity_util import assert_close
+
+pytestmark = pytest.mark.gpu
+
+NAMES = ("q", "k", "v", "g", "beta", "gamma")
+
+
+def _noalloc(x, clip=1.0):
+    """Call rdn_fwd_noalloc through the C ABI; no workspace is passed."""
+    lib = _abi.load()
+    B, T, H, D = x["q"].shape
+    o = torch.empty(B, T, H, D, dtype=x["q"].dtype, device=x["q"].device)
+    ST = torch.empty(B, H, D, D, device=x["q"].device)
+    RT = torch.empty_like(ST)
+    a = _abi.FwdArgs()
+    a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
+    a.dtype = _abi.RDN_BF16 if x["q"].dtype == torch.bfloat16 else _abi.RDN_F32
+    p = lambda t: None if t is None else ctypes.c_void_p(t.data_ptr())
+    a.q, a.k, a.v = p(x["q"]), p(x["k"]), p(x["v"])
+    a.g, a.beta, a.gamma = p(x["g"]), p(x["beta"]), p(x["gamma"])
+    a.clip, a.scale, a.flags = clip, 1.0, 0
+    a.S0, a.R0 = p(x["S0"]), p(x["R0"])
+    a.o, a.ST, a.RT = p(o), p(ST), p(RT)
+    a.workspace, a.workspace_bytes = None, 0
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    st = lib.rdn_fwd_noalloc(ctypes.byref(a), stream)
+    assert st == 0, lib.rdn_last_error().decode()
+    torch.cuda.synchronize()
+    return o, ST, RT
+
+
+def test_noalloc_matches_rdn_fwd_two_calls_in_a_row():
+    # two different problems back to back: the second call must not see the
+    # first one's leftovers in the shared scratch
+    for seed, (B, T, H, D) in ((0, (2, 300, 4, 128)), (1, (1, 130, 3, 64))):
+        x = make_inputs(B, T, H, D, dtype="bf16", nonzero_state=True, device="cuda",
+                        seed=seed, state_std=0.1)
+        o, ST, RT = _noalloc(x)
+        o2, ST2, RT2 = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"])
+        torch.cuda.synchronize()
+        assert_close(o, o2.float().cpu().double().numpy(), "bf16", "o")
+        assert_close(ST, ST2.cpu().double().numpy(), "f32", "ST")
+        assert_close(RT, RT2.cpu().double().numpy(), "f32", "RT")
+
+
+def test_noalloc_rejects_problems_beyond_its_scratch():
+    lib = _abi.load()
+    a = _abi.FwdArgs()
+    a.B, a.T, a.H, a.Dk, a.Dv = 8, 4096, 16, 128, 128  # 8192 chunks > 804
+    a.dtype, a.clip, a.scale = _abi.RDN_BF16, 1.0, 1.0
+    fake = ctypes.c_void_p(0x10000)
+    a.q = a.k = a.v = a.g = a.beta = a.gamma = a.o = fake
+    assert lib.rdn_fwd_noalloc(ctypes.byref(a), None) == 5
+    msg = lib.rdn_last_error().decode()
+    assert "built-in scratch" in msg and "804" in msg
