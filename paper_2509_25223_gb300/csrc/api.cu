@@ -224,14 +224,22 @@ rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a, rdn_stream_t stream) {
   if (st != RDN_OK) return st;
   if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
   const size_t need = rdn::plan_fwd(*a, 1).total_bytes;
-  if (need > (size_t)RDN_NOALLOC_SCRATCH_BYTES)
+  if (need > (size_t)RDN_NOALLOC_SCRATCH_BYTES) {
+    // per-chunk record size and fixed overhead, from the workspace plan
+    rdn_fwd_args one = *a, two = *a;
+    one.B = one.H = two.B = two.H = 1;
+    one.T = rdn::kChunk;
+    two.T = 2 * rdn::kChunk;
+    const size_t per_chunk = rdn::plan_fwd(two, 1).total_bytes - rdn::plan_fwd(one, 1).total_bytes;
+    const size_t fixed = rdn::plan_fwd(one, 1).total_bytes - per_chunk;
     return fail(RDN_ERR_WORKSPACE,
                 "%s: this problem needs %zu bytes of scratch (B*H*ceil(T/64) = %lld chunks) but "
                 "the built-in scratch holds %zu bytes (at most %zu chunks); use rdn_fwd with a "
                 "caller workspace",
                 fn, need, (long long)a->B * a->H * ((a->T + rdn::kChunk - 1) / rdn::kChunk),
                 (size_t)RDN_NOALLOC_SCRATCH_BYTES,
-                (size_t)RDN_NOALLOC_SCRATCH_BYTES / rdn::plan_fwd(rdn_fwd_args{1, 64, 1, a->Dk, a->Dv}, 1).total_bytes);
+                ((size_t)RDN_NOALLOC_SCRATCH_BYTES - fixed) / per_chunk);
+  }
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_status(fn, e);

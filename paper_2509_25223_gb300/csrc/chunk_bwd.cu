@@ -692,7 +692,7 @@ BwdLayout layout(const rdn_bwd_args &a) {
   l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
-  l.total = l.prep + l.acc + 2 * l.states + l.o;
+  l.total = l.prep + l.acc + 2 * l.states + l.o + 256;  // + device status word
   return l;
 }
 
@@ -720,6 +720,7 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   BwdParams p;
   p.f = make_fwd_params(f);
   p.f.ws = (float *)ws;
+  p.f.err = (int *)(ws + l.total - 256);
   p.f.ST = p.f.RT = nullptr;
   const bool bf = f.dtype == RDN_BF16;
   const bool rdnv = true;
@@ -729,6 +730,10 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
     p.f.R_chunks = (float *)(ws + l.prep + l.acc + l.states);
     p.f.o = ws + l.prep + l.acc + 2 * l.states;
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
+    // the tensor-core scan reads the records as shared-memory images; the
+    // reverse scan below reads them in fp32: rewrite them
+    if (e == cudaSuccess && bf && f.Dk == 128)
+      e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, false, s);
   } else {
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, false, s);
   }

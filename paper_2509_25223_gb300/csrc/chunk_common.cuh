@@ -17,6 +17,17 @@ constexpr int OFF_VEC = 5 * kCC;
 constexpr int V_GAM = 0, V_GPREV = C, V_ALPHA = 2 * C, V_WS = 3 * C, V_WR = 4 * C, V_GAMC = 5 * C;
 constexpr int kRecFloats = OFF_VEC + 6 * C;
 
+// The tensor-core scan reads the same record in a second format: the chunk
+// matrices as shared-memory images (bf16 hi + lo parts, K-major, 128-byte
+// swizzled), copied to shared memory with bulk copies.  Byte offsets:
+//   T_beta  hi | lo  (64 rows each)      [IMG_TB,   IMG_TB + 16 KB)
+//   [Ap ; Mq] hi | lo (128 rows each)    [IMG_APMQ, IMG_APMQ + 32 KB)
+//   T_gamma hi | lo                      [IMG_TG,   ...)
+//   M2      hi | lo                      [IMG_M2,   ...)
+//   the gate vectors at the same place as in the fp32 record (OFF_VEC).
+constexpr int IMG_TB = 0, IMG_APMQ = 16384, IMG_TG = 49152, IMG_M2 = 65536;
+static_assert(IMG_M2 + 16384 == OFF_VEC * 4, "image fills the matrix part of the record");
+
 // Block-level fp32 product over shared memory: the calling thread gets
 // acc[i] = sum_k A(m_i, k) B(k, n) for n = tid % N and m_i = tid / N + i * (256 / N).
 // A(m,k) = A[m*a_m + k*a_k], B(k,n) = B[k*b_k + n*b_n].  With N >= 32 the lanes
@@ -51,6 +62,7 @@ struct FwdParams {
   void *o;
   float *ST, *RT, *S_chunks, *R_chunks;
   float *ws;  // NC*B*H records of kRecFloats
+  int *err;   // device status word (RDN_ERR_TIMEOUT if a bounded wait gave up) or NULL
 };
 
 
@@ -65,8 +77,13 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.o = a.o;
   p.ST = a.ST; p.RT = a.RT; p.S_chunks = a.S_chunks; p.R_chunks = a.R_chunks;
   p.ws = nullptr;
+  p.err = nullptr;
   return p;
 }
+
+// Tensor-core scan (fwd_tc.cu): bf16 inputs with d_k = d_v = 128.
+bool fwd_tc_supported(const rdn_fwd_args &a);
+cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s);
 
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).

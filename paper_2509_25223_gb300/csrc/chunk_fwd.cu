@@ -34,7 +34,16 @@ namespace rdn {
 namespace {
 
 // ---------------------------------------------------------------- kernel 1
-template <int DK, bool RDNV, typename InT>
+// Image writer: element (r, c) of a 64-column chunk matrix, value x, into a
+// K-major 128B-swizzled bf16 hi / lo pair (lo tile `lo_off` bytes after hi).
+__device__ __forceinline__ void img_put(uint8_t *tile, uint32_t lo_off, int r, int c, float x) {
+  const uint32_t o = (uint32_t)(r * 128 + ((((c >> 3) ^ (r & 7)) & 7) << 4) + (c & 7) * 2);
+  const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+  *reinterpret_cast<__nv_bfloat16 *>(tile + o) = hi;
+  *reinterpret_cast<__nv_bfloat16 *>(tile + lo_off + o) = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
+template <int DK, bool RDNV, typename InT, bool IMG>
 __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   constexpr int LDK = DK + 1;
   constexpr int LDC = C + 1;
@@ -121,9 +130,16 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
         ag = dec * gam[i] * KK[t * LDC + i];
       }
     }
-    rec[OFF_AP + e] = ap;
-    rec[OFF_MQ + e] = mq;
-    rec[OFF_M2 + e] = m2;
+    if (IMG) {
+      uint8_t *img = reinterpret_cast<uint8_t *>(rec);
+      img_put(img + IMG_APMQ, 16384, t, i, ap);
+      img_put(img + IMG_APMQ, 16384, 64 + t, i, mq);
+      img_put(img + IMG_M2, 8192, t, i, m2);
+    } else {
+      rec[OFF_AP + e] = ap;
+      rec[OFF_MQ + e] = mq;
+      rec[OFF_M2 + e] = m2;
+    }
     if (RDNV) {
       Ab[t * LDC + i] = ab;
       Ag[t * LDC + i] = ag;
@@ -156,8 +172,14 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
     __syncthreads();
     for (int e = tid; e < C * C; e += kThreads) {
       const int t = e / C, i = e % C;
-      rec[OFF_TB + e] = Tb[t * LDC + i];
-      rec[OFF_TG + e] = Tg[t * LDC + i];
+      if (IMG) {
+        uint8_t *img = reinterpret_cast<uint8_t *>(rec);
+        img_put(img + IMG_TB, 8192, t, i, Tb[t * LDC + i]);
+        img_put(img + IMG_TG, 8192, t, i, Tg[t * LDC + i]);
+      } else {
+        rec[OFF_TB + e] = Tb[t * LDC + i];
+        rec[OFF_TG + e] = Tg[t * LDC + i];
+      }
     }
   }
 }
@@ -367,8 +389,9 @@ constexpr size_t scan_smem() {
 }
 
 template <int DK, bool RDNV, typename InT>
-cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_scan) {
-  auto prep = chunk_prep_kernel<DK, RDNV, InT>;
+cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_scan,
+                     bool img = false) {
+  auto prep = img ? chunk_prep_kernel<DK, RDNV, InT, true> : chunk_prep_kernel<DK, RDNV, InT, false>;
   auto scan = chunk_scan_kernel<DK, RDNV, InT>;
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(prep, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -390,23 +413,34 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
 
 cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, bool do_prep,
                              bool do_scan, cudaStream_t s) {
+  // RDN with bf16 inputs and d = 128 runs the tensor-core scan; everything
+  // else the fp32 SIMT one.  (RLA's state is not contracted by the delta
+  // term, and its output error with single-bf16 state operands reaches the
+  // 2e-2 RMS bound, so RLA stays on the fp32 path.)
+  const bool tc_scan = do_scan && bf16 && DK == 128 && rdnv;
+  cudaError_t e = cudaSuccess;
+  // (the tensor-core scan reads the records as shared-memory images)
   if (DK == 128) {
-    if (rdnv) return bf16 ? launch_t<128, true, __nv_bfloat16>(p, s, do_prep, do_scan)
-                          : launch_t<128, true, float>(p, s, do_prep, do_scan);
-    return bf16 ? launch_t<128, false, __nv_bfloat16>(p, s, do_prep, do_scan)
-                : launch_t<128, false, float>(p, s, do_prep, do_scan);
+    if (rdnv) e = bf16 ? launch_t<128, true, __nv_bfloat16>(p, s, do_prep, do_scan && !tc_scan, tc_scan)
+                       : launch_t<128, true, float>(p, s, do_prep, do_scan);
+    else e = bf16 ? launch_t<128, false, __nv_bfloat16>(p, s, do_prep, do_scan && !tc_scan, tc_scan)
+                  : launch_t<128, false, float>(p, s, do_prep, do_scan);
+  } else {
+    if (rdnv) e = bf16 ? launch_t<64, true, __nv_bfloat16>(p, s, do_prep, do_scan)
+                       : launch_t<64, true, float>(p, s, do_prep, do_scan);
+    else e = bf16 ? launch_t<64, false, __nv_bfloat16>(p, s, do_prep, do_scan)
+                  : launch_t<64, false, float>(p, s, do_prep, do_scan);
   }
-  if (rdnv) return bf16 ? launch_t<64, true, __nv_bfloat16>(p, s, do_prep, do_scan)
-                        : launch_t<64, true, float>(p, s, do_prep, do_scan);
-  return bf16 ? launch_t<64, false, __nv_bfloat16>(p, s, do_prep, do_scan)
-              : launch_t<64, false, float>(p, s, do_prep, do_scan);
+  if (e != cudaSuccess || !tc_scan) return e;
+  return launch_fwd_tc(p, rdnv, s);
 }
 
 FwdPlan plan_fwd(const rdn_fwd_args &a, int /*variant*/) {
   FwdPlan pl;
   pl.NC = (a.T + C - 1) / C;
   pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
-  pl.total_bytes = pl.prep_bytes * (size_t)a.B * a.H * pl.NC;
+  // per-chunk records, then a 256-byte device status word
+  pl.total_bytes = pl.prep_bytes * (size_t)a.B * a.H * pl.NC + 256;
   return pl;
 }
 
@@ -423,6 +457,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   }
   FwdParams p = make_fwd_params(a);
   p.ws = (float *)a.workspace;
+  p.err = (int *)((char *)a.workspace + plan_fwd(a, variant).total_bytes - 256);
   return launch_fwd_parts(p, a.Dk, variant == 1, a.dtype == RDN_BF16, true, true, s);
 }
 

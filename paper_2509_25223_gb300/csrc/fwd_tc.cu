@@ -1,0 +1,460 @@
+// fwd_tc.cu -- tensor-core (tcgen05 / TMEM) scan of the chunkwise RLA / RDN
+// forward, bf16 inputs, d_k = d_v = 128.
+//
+// Same chunk algebra as chunk_fwd.cu (see its header), computed in the
+// transposed orientation so that every product has the value dimension
+// d_v = 128 as its M dimension: TMEM lane j holds value column j, and thread
+// j of the CTA's 128 threads owns that column end to end.  Per chunk of 64
+// tokens, with B1 = [diag(Gprev) K ; diag(Gam) Q] (128 x d_k, bf16):
+//
+//   MMA1  D1   = S^T  B1^T          -> [Gprev*KS | Gam*QS]        (N=128, K=128)
+//         X    = V - alpha * (Gprev*KS)                  (= V - Gam*KS)
+//   MMA2  E^T  = X^T  T_beta^T                                    (N=64,  K=64)
+//   MMA3  D1  += E^T  [Ap ; Mq]^T   -> [P | Ob]                   (N=128, K=64)
+//   MMA4  U    = (wS E)^T K         -> S_C = Gam_C S + U          (N=128, K=64)
+//         r    = clip(V - P)        (Section 3.3; kept in registers)
+//   MMA5  D3   = R^T  B1^T          -> [Gprev*KR | Gam*QR]
+//         X2   = r - alpha * (Gprev*KR)
+//   MMA6  E2^T = X2^T T_gamma^T
+//   MMA7  D3[:, Q half] += E2^T M2^T -> Oa
+//   MMA8  U2   = (wR E2)^T K        -> R_C = Gam_C R + U2 (two N=64 halves)
+//         o    = Ob + gamma * Oa
+//
+// RLA skips MMA2 and MMA6 (E = V, E2 = r).  X, E, wS E and their auxiliary
+// counterparts (magnitude ~ |v|) enter the MMAs as bf16 hi + lo pairs, which
+// keeps their rounding well below the state's own scale; the other operands
+// (states, scaled K and Q, chunk matrices) are single bf16.  The states S, R live in TMEM in
+// fp32 for the whole sequence; their bf16 copies (the A operands of MMA1 and
+// MMA5) are rewritten in shared memory after each update.  One thread issues
+// the MMAs; every wait is an mbarrier wait with a time limit.  The
+// state-independent chunk matrices (T_beta, T_gamma, Ap, Mq, M2) come from
+// chunk_prep's records as bf16 hi + lo shared-memory images; they are streamed
+// into two slots by bulk copies one phase ahead of their use (slot A: T_beta
+// then T_gamma; slot B: [Ap;Mq] then M2) and enter the MMAs as three products
+// (hi*hi + hi*lo + lo*hi).
+//
+// TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) X
+// (X holds E, then U, then D3; D1 holds P|Ob, then E2 | Ob, then U2a | Ob).
+#include "chunk_common.cuh"
+#include "tc_common.cuh"
+
+namespace rdn {
+namespace {
+
+using namespace tc;
+
+constexpr int D = 128;
+constexpr int kTcThreads = 128;
+
+// shared-memory carve-up (bytes from the 1024-aligned dynamic base)
+constexpr uint32_t SM_SA = 0;          // S^T bf16, 128 x 128, two 64-col blocks
+constexpr uint32_t SM_RA = 32768;      // R^T bf16
+constexpr uint32_t SM_B1 = 65536;      // [Gprev K ; Gam Q], 128 x 128
+constexpr uint32_t SM_KT = 98304;      // K^T, 128 (d_k) x 64 (t)
+constexpr uint32_t SM_SLOTA = 114688;  // T_beta then T_gamma image (hi | lo), 16 KB
+constexpr uint32_t SM_SLOTB = 131072;  // [Ap;Mq] then M2 image (hi | lo), 32 KB
+// value-like operands are split into bf16 hi + lo parts (two MMAs each):
+constexpr uint32_t SM_XE = 163840;     // X^T then E^T (X2^T then E2^T), hi part, 128 x 64
+constexpr uint32_t SM_XE_LO = 180224;  //   lo part
+constexpr uint32_t SM_W = 196608;      // (wS E)^T / (wR E2)^T, hi part
+constexpr uint32_t SM_W_LO = 212992;   //   lo part
+constexpr uint32_t SM_VEC = 229376;    // 7 x 64 fp32: Gam Gprev alpha wS wR gamma, GamC
+constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;  // 3 mbarriers: MMA, slot A, slot B
+constexpr uint32_t SM_SLOT = SM_BAR + 24;
+constexpr uint32_t SM_FLAG = SM_SLOT + 4;
+constexpr uint32_t SM_BYTES = SM_FLAG + 4;
+constexpr size_t kTcSmem = SM_BYTES;
+static_assert(kTcSmem <= 232448, "shared memory");
+
+constexpr uint32_t T_S = 0, T_R = 128, T_D1 = 256, T_X = 384;
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Write 16 consecutive values (columns c0..c0+15 of row r) of a K-major SW128
+// tile whose 64-column blocks are blk_bytes apart.
+__device__ __forceinline__ void st_row16(uint8_t *tile, uint32_t blk_bytes, int r, int c0,
+                                         const float (&v)[16]) {
+  uint8_t *blk = tile + (c0 >> 6) * blk_bytes;
+  const int cc = c0 & 63;
+  uint4 a, b;
+  a.x = pack_bf16(v[0], v[1]);
+  a.y = pack_bf16(v[2], v[3]);
+  a.z = pack_bf16(v[4], v[5]);
+  a.w = pack_bf16(v[6], v[7]);
+  b.x = pack_bf16(v[8], v[9]);
+  b.y = pack_bf16(v[10], v[11]);
+  b.z = pack_bf16(v[12], v[13]);
+  b.w = pack_bf16(v[14], v[15]);
+  *reinterpret_cast<uint4 *>(blk + sw128(r, cc)) = a;
+  *reinterpret_cast<uint4 *>(blk + sw128(r, cc + 8)) = b;
+}
+
+// Same, split: hi = bf16(v), lo = bf16(v - hi) into two tiles, so that
+// hi + lo carries about 16 significant bits.
+__device__ __forceinline__ void st_row16_split(uint8_t *hi, uint8_t *lo, int r, int c0,
+                                               const float (&v)[16]) {
+  float a[16], b[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+    b[i] = v[i] - a[i];
+  }
+  st_row16(hi, 0, r, c0, a);
+  st_row16(lo, 0, r, c0, b);
+}
+
+// D (+)= (A_hi + A_lo)(B_hi + B_lo)^T without the lo*lo term: three MMAs
+// over K = 64 for K-major 128B-swizzled tiles.
+__device__ __forceinline__ void mma_split3(uint32_t d, uint32_t a_hi, uint32_t a_lo,
+                                           uint32_t b_hi, uint32_t b_lo, uint32_t idesc,
+                                           bool accumulate_first) {
+  mma_tile(d, a_hi, 0, b_hi, 0, 4, idesc, accumulate_first);
+  mma_tile(d, a_hi, 0, b_lo, 0, 4, idesc, true);
+  mma_tile(d, a_lo, 0, b_hi, 0, 4, idesc, true);
+}
+
+template <bool RDNV>
+__global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
+  extern __shared__ __align__(1024) uint8_t sm[];
+  const uint32_t sbase = smem_u32(sm);
+  if (sbase & 1023u) {  // the swizzled tiles need a 1024-byte aligned base
+    if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
+    return;
+  }
+  float *vec = reinterpret_cast<float *>(sm + SM_VEC);
+  float *Gam = vec, *Gprev = vec + 64, *alpha = vec + 128, *wS = vec + 192, *wR = vec + 256,
+        *gamv = vec + 320;
+  uint64_t *bar = reinterpret_cast<uint64_t *>(sm + SM_BAR);
+  uint64_t *barA = bar + 1, *barB = bar + 2;  // slot A / slot B bulk copies
+  uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SM_SLOT);
+  volatile int *flag = reinterpret_cast<volatile int *>(sm + SM_FLAG);
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int j = tid;  // value column == TMEM lane
+  const int bh = blockIdx.x;
+  const int b = bh / p.H, h = bh % p.H;
+  const int T = p.T, H = p.H, NC = p.NC;
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q;
+  const __nv_bfloat16 *k = (const __nv_bfloat16 *)p.k;
+  const __nv_bfloat16 *v = (const __nv_bfloat16 *)p.v;
+  __nv_bfloat16 *o = (__nv_bfloat16 *)p.o;
+  const float clip = p.clip;
+  const size_t st_base = (size_t)bh * D * D;
+
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    mbar_init(barA, 1);
+    mbar_init(barB, 1);
+    fence_mbar_init();
+    *flag = 0;
+  }
+  if (warp == 0) tmem_alloc(slot, 512);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  uint32_t phase = 0, phA = 0, phB = 0;  // phA/phB: tracked by thread 0 only
+  auto rec_of = [&](int c) {
+    return reinterpret_cast<const uint8_t *>(p.ws + ((size_t)bh * NC + c) * kRecFloats);
+  };
+  // thread 0: start the bulk copy of a chunk-matrix image into a slot
+  auto load_slot = [&](uint8_t *dst, uint64_t *b, const uint8_t *src, uint32_t bytes) {
+    mbar_expect_tx(b, bytes);
+    bulk_g2s(dst, src, bytes, b);
+  };
+  if (tid == 0) {
+    if (RDNV) load_slot(sm + SM_SLOTA, barA, rec_of(0) + IMG_TB, 16384);
+    load_slot(sm + SM_SLOTB, barB, rec_of(0) + IMG_APMQ, 32768);
+  }
+
+  // initial states -> TMEM (fp32) and bf16 A operands
+  for (int c0 = 0; c0 < D; c0 += 16) {
+    float s[16], r[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      s[i] = p.S0 ? p.S0[st_base + (size_t)(c0 + i) * D + j] : 0.f;
+      r[i] = p.R0 ? p.R0[st_base + (size_t)(c0 + i) * D + j] : 0.f;
+    }
+    tmem_st16(tm + lane + T_S + c0, s);
+    tmem_st16(tm + lane + T_R + c0, r);
+    st_row16(sm + SM_SA, 16384, j, c0, s);
+    st_row16(sm + SM_RA, 16384, j, c0, r);
+  }
+
+  // one MMA phase: make smem writes visible, issue, wait.  Returns false on
+  // timeout (the caller aborts).
+  auto run_phase = [&](auto issue) -> bool {
+    fence_async_smem();
+    fence_before_sync();
+    __syncthreads();
+    if (tid == 0) {
+      fence_after_sync();
+      if (!issue()) *flag = 1;  // a slot's bulk copy did not arrive in time
+      mma_commit(bar);
+    }
+    const bool ok = mbar_wait(bar, phase);
+    phase ^= 1u;
+    if (!ok) *flag = 1;
+    __syncthreads();
+    fence_after_sync();
+    return *flag == 0;
+  };
+
+  float rres[64];  // clipped residual r[t] of column j
+  // v[t, j] of the current chunk (0 beyond the sequence), read from L2/HBM
+  auto vval = [&](int t0, int n, int t) -> float {
+    return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  };
+  bool alive = true;
+  for (int c = 0; c < NC && alive; ++c) {
+    const int t0 = c * 64;
+    const int n = min(64, T - t0);
+    const float *rec = p.ws + ((size_t)bh * NC + c) * kRecFloats;
+    __syncthreads();  // every thread is done with the previous chunk's tiles and vectors
+
+    // ---- (a) chunk inputs -> shared memory
+    if (p.S_chunks) {  // chunk-start states for the backward
+      float *sc = p.S_chunks + ((size_t)bh * NC + c) * D * D;
+      float *rc = p.R_chunks + ((size_t)bh * NC + c) * D * D;
+      for (int c0 = 0; c0 < D; c0 += 16) {
+        float s[16], r[16];
+        tmem_ld16(tm + lane + T_S + c0, s);
+        tmem_ld16(tm + lane + T_R + c0, r);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          sc[(size_t)(c0 + i) * D + j] = s[i];
+          rc[(size_t)(c0 + i) * D + j] = r[i];
+        }
+      }
+    }
+    if (tid < 64) {
+      Gam[tid] = rec[OFF_VEC + V_GAM + tid];
+      Gprev[tid] = rec[OFF_VEC + V_GPREV + tid];
+      alpha[tid] = rec[OFF_VEC + V_ALPHA + tid];
+      wS[tid] = rec[OFF_VEC + V_WS + tid];
+      wR[tid] = rec[OFF_VEC + V_WR + tid];
+      gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    }
+    const float GamC = rec[OFF_VEC + V_GAMC];
+    __syncthreads();
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // K, Q: 64 rows x 16 chunks of 8
+      const int t = e >> 4, ch = e & 15;
+      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+      if (t < n) {
+        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8;
+        kv = *reinterpret_cast<const uint4 *>(k + off);
+        qv = *reinterpret_cast<const uint4 *>(q + off);
+      }
+      const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
+      const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(&qv);
+      const float gk = Gprev[t], gq = Gam[t] * p.scale;
+      uint4 ks, qs;
+      uint32_t *kw = &ks.x, *qw = &qs.x;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        kw[i] = pack_bf16(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
+        qw[i] = pack_bf16(gq * __bfloat162float(qb[2 * i]), gq * __bfloat162float(qb[2 * i + 1]));
+      }
+      const int blk = ch >> 3, cc = (ch & 7) * 8;
+      *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(t, cc)) = ks;
+      *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc)) = qs;
+      __nv_bfloat16 *kt = reinterpret_cast<__nv_bfloat16 *>(sm + SM_KT);
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        kt[sw128(ch * 8 + i, t) / 2] = kb[i];
+    }
+
+    // ---- (b) MMA1: D1 = S^T B1^T
+    alive = run_phase([&] {
+      mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_B1, 16384, 8, idesc_bf16(128, 128),
+               false);
+      return true;
+    });
+    if (!alive) break;
+
+    // ---- (c) X = V - alpha * (Gprev KS)  ->  MMA2: E^T = X^T T_beta^T
+    if (RDNV) {
+      for (int c0 = 0; c0 < 64; c0 += 16) {
+        float x[16];
+        tmem_ld16(tm + lane + T_D1 + c0, x);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) x[i] = vval(t0, n, c0 + i) - alpha[c0 + i] * x[i];
+        st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+      }
+      alive = run_phase([&] {
+        if (!mbar_wait(barA, phA)) return false;
+        phA ^= 1u;
+        mma_split3(tm + T_X, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
+                   sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
+        return true;
+      });
+      if (!alive) break;
+      if (tid == 0) load_slot(sm + SM_SLOTA, barA, rec_of(c) + IMG_TG, 16384);
+    }
+
+    // ---- (d) E -> EA, wS*E -> WA;  MMA3: D1 += E^T [Ap;Mq]^T,  MMA4: U = (wS E)^T K
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float e[16], w[16];
+      if (RDNV) {
+        tmem_ld16(tm + lane + T_X + c0, e);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) e[i] = vval(t0, n, c0 + i);
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) w[i] = wS[c0 + i] * e[i];
+      st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, e);
+      st_row16_split(sm + SM_W, sm + SM_W_LO, j, c0, w);
+    }
+    alive = run_phase([&] {
+      if (!mbar_wait(barB, phB)) return false;
+      phB ^= 1u;
+      mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
+                 sbase + SM_SLOTB + 16384, idesc_bf16(128, 128), true);
+      mma_tile(tm + T_X, sbase + SM_W, 0, sbase + SM_KT, 0, 4, idesc_bf16(128, 128), false);
+      mma_tile(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT, 0, 4, idesc_bf16(128, 128), true);
+      return true;
+    });
+    if (!alive) break;
+    if (tid == 0) load_slot(sm + SM_SLOTB, barB, rec_of(c) + IMG_M2, 16384);
+
+    // ---- (e) r = clip(V - P); S = Gam_C S + U (fp32 in TMEM, bf16 copy in SA)
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float pp[16];
+      tmem_ld16(tm + lane + T_D1 + c0, pp);
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        rres[c0 + i] = clampf(vval(t0, n, c0 + i) - pp[i], clip);
+    }
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], u[16];
+      tmem_ld16(tm + lane + T_S + c0, s);
+      tmem_ld16(tm + lane + T_X + c0, u);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
+      tmem_st16(tm + lane + T_S + c0, s);
+      st_row16(sm + SM_SA, 16384, j, c0, s);
+    }
+    // MMA5: D3 = R^T B1^T (into X)
+    alive = run_phase([&] {
+      mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_B1, 16384, 8, idesc_bf16(128, 128),
+               false);
+      return true;
+    });
+    if (!alive) break;
+
+    // ---- (f) X2 = r - alpha * (Gprev KR);  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
+    if (RDNV) {
+#pragma unroll
+      for (int c0 = 0; c0 < 64; c0 += 16) {
+        float x[16];
+        tmem_ld16(tm + lane + T_X + c0, x);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - alpha[c0 + i] * x[i];
+        st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+      }
+      alive = run_phase([&] {
+        if (!mbar_wait(barA, phA)) return false;
+        phA ^= 1u;
+        mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
+                   sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
+        return true;
+      });
+      if (!alive) break;
+      if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTA, barA, rec_of(c + 1) + IMG_TB, 16384);
+    }
+
+    // ---- (g) E2 -> EA, wR*E2 -> WA;  MMA7: Oa += E2^T M2^T;  MMA8: U2 = (wR E2)^T K
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float e[16], w[16];
+      if (RDNV) {
+        tmem_ld16(tm + lane + T_D1 + c0, e);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) w[i] = wR[c0 + i] * e[i];
+      st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, e);
+      st_row16_split(sm + SM_W, sm + SM_W_LO, j, c0, w);
+    }
+    alive = run_phase([&] {
+      const uint32_t i64 = idesc_bf16(128, 64);
+      if (!mbar_wait(barB, phB)) return false;
+      phB ^= 1u;
+      mma_split3(tm + T_X + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
+                 sbase + SM_SLOTB + 8192, i64, true);
+      mma_tile(tm + T_D1, sbase + SM_W, 0, sbase + SM_KT, 0, 4, i64, false);
+      mma_tile(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KT, 0, 4, i64, true);
+      mma_tile(tm + T_X, sbase + SM_W, 0, sbase + SM_KT + 8192, 0, 4, i64, false);
+      mma_tile(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT + 8192, 0, 4, i64, true);
+      return true;
+    });
+    if (!alive) break;
+    if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTB, barB, rec_of(c + 1) + IMG_APMQ, 32768);
+
+    // ---- (h) o = Ob + gamma * Oa;  R = Gam_C R + U2
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float ob[16], oa[16];
+      tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);
+      tmem_ld16(tm + lane + T_X + 64 + c0, oa);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = c0 + i;
+        if (t < n)
+          o[((size_t)(b * T + t0 + t) * H + h) * D + j] =
+              __float2bfloat16_rn(fmaf(gamv[t], oa[i], ob[i]));
+      }
+    }
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float r[16], u[16];
+      tmem_ld16(tm + lane + T_R + c0, r);
+      tmem_ld16(tm + lane + (c0 < 64 ? T_D1 + c0 : T_X + c0 - 64), u);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
+      tmem_st16(tm + lane + T_R + c0, r);
+      st_row16(sm + SM_RA, 16384, j, c0, r);
+    }
+  }
+
+  if (alive) {  // final states
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], r[16];
+      tmem_ld16(tm + lane + T_S + c0, s);
+      tmem_ld16(tm + lane + T_R + c0, r);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (p.ST) p.ST[st_base + (size_t)(c0 + i) * D + j] = s[i];
+        if (p.RT) p.RT[st_base + (size_t)(c0 + i) * D + j] = r[i];
+      }
+    }
+  } else if (tid == 0 && p.err) {
+    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+}  // namespace
+
+bool fwd_tc_supported(const rdn_fwd_args &a) {
+  return a.dtype == RDN_BF16 && a.Dk == 128 && a.Dv == 128;
+}  // (the dispatcher uses it for RDN only)
+
+cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
+  auto kern = rdnv ? fwd_tc_kernel<true> : fwd_tc_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kTcSmem);
+  if (e != cudaSuccess) return e;
+  RDN_LAUNCH("fwd_tc_scan", s, kern<<<p.B * p.H, kTcThreads, kTcSmem, s>>>(p));
+  return cudaGetLastError();
+}
+
+}  // namespace rdn
