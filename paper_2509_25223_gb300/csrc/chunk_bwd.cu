@@ -437,6 +437,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
 }
 
 // ---------------------------------------------------------------- kernel 2
+// One CTA per chunk.  Each warp owns 8 rows t of the C x C gradients; lane l
+// handles columns l and l + 32.  Row sums (d cum_t, d cprev_t) are reduced
+// with shuffles; column sums (d cum_i, dbeta_i, dgamma_i) go through
+// shared-memory tiles and a column pass, so no shared-memory atomics are
+// contended.
 template <int DK, bool RDNV, typename InT>
 __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   constexpr int LDK = DK + 1;
@@ -447,9 +452,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   float *Qs = Ks + C * LDK;     // [C][LDK]
   float *KK = Qs + C * LDK;     // [C][LDC]
   float *QK = KK + C * LDC;     // [C][LDC]
-  float *dKK = QK + C * LDC;    // [C][LDC] symmetrised at the end
+  float *dKK = QK + C * LDC;    // [C][LDC] symmetrised before use
   float *dQK = dKK + C * LDC;   // [C][LDC]
-  float *cum = dQK + C * LDC;   // [C]
+  float *colG = dQK + C * LDC;  // [C][LDC] column contributions to d cum
+  float *colB = colG + C * LDC; // [C][LDC] ... to dbeta
+  float *colM = colB + C * LDC; // [C][LDC] ... to dgamma
+  float *cum = colM + C * LDC;  // [C]
   float *cprev = cum + C;
   float *bet = cprev + C;
   float *gam = bet + C;
@@ -465,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   const int b = bh / H, h = bh % H;
   const int t0 = c * C;
   const int n = min(C, T - t0);
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const InT *q = (const InT *)p.f.q;
   const InT *k = (const InT *)p.f.k;
   const float *acc = p.acc + (size_t)chunk * L::FLOATS;
@@ -493,18 +501,24 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     gg[t] = gv;
     bet[t] = bv;
     gam[t] = mv;
-    dcprev[t] = 0.f;
-    dbet[t] = 0.f;
-    dgam[t] = acc[L::VEC + L::V_DGAM_OUT + t];
   }
   __syncthreads();
-  if (tid == 0) {
-    float s = 0.f;
-    for (int t = 0; t < C; ++t) {
-      cprev[t] = s;
-      s += gg[t];
-      cum[t] = s;
+  if (warp == 0) {  // in-chunk cumulative log-decay (two 32-wide shuffle scans)
+    float a = gg[lane], b2 = gg[32 + lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float ua = __shfl_up_sync(0xffffffffu, a, off);
+      const float ub = __shfl_up_sync(0xffffffffu, b2, off);
+      if (lane >= off) {
+        a += ua;
+        b2 += ub;
+      }
     }
+    b2 += __shfl_sync(0xffffffffu, a, 31);
+    cum[lane] = a;
+    cum[32 + lane] = b2;
+    cprev[lane] = a - gg[lane];
+    cprev[32 + lane] = b2 - gg[32 + lane];
   }
   {
     using MM = BlockMM<C, C, DK>;
@@ -517,97 +531,109 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     for (int i = 0; i < MM::RPT; ++i) QK[MM::row(i) * LDC + MM::col()] = a[i];
   }
   __syncthreads();
-  // per-row factors: Gam_t = e^{cum_t}, Gprev_t = e^{cprev_t}, w_t = rate_t e^{cum_C - cum_t}
+  // ---- row pass over the C x C gradients
+  for (int rr = 0; rr < C / 8; ++rr) {
+    const int t = warp * (C / 8) + rr;
+    float rowc = 0.f, rowp = 0.f;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int i = lane + 32 * half;
+      const int e = t * C + i;
+      float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
+      if (i <= t) {
+        const float dec = expf(cum[t] - cum[i]);
+        const float kk = KK[t * LDC + i], qk = QK[t * LDC + i];
+        const float bi = bet[i], gi = gam[i];
+        {  // M2: inclusive, gamma, QK
+          const float dm = acc[L::DM2 + e];
+          const float G = dm * dec * gi * qk;
+          rowc += G;
+          cg += G;
+          cm += dm * dec * qk;
+          dqk += dm * dec * gi;
+        }
+        if (i < t) {
+          const float decp = expf(cprev[t] - cum[i]);
+          {  // Ap: strict, beta, KK, previous-token decay
+            const float dm = acc[L::DAP + e];
+            const float G = dm * decp * bi * kk;
+            rowp += G;
+            cg += G;
+            cb += dm * decp * kk;
+            dkk += dm * decp * bi;
+          }
+          {  // Mq: strict, beta, QK
+            const float dm = acc[L::DMQ + e];
+            const float G = dm * dec * bi * qk;
+            rowc += G;
+            cg += G;
+            cb += dm * dec * qk;
+            dqk += dm * dec * bi;
+          }
+          if (RDNV) {
+            const float da = acc[L::DAB + e], dg2 = acc[L::DAG + e];
+            const float Gb = da * dec * bi * kk, Gg = dg2 * dec * gi * kk;
+            rowc += Gb + Gg;
+            cg += Gb + Gg;
+            cb += da * dec * kk;
+            cm += dg2 * dec * kk;
+            dkk += da * dec * bi + dg2 * dec * gi;
+          }
+        }
+      }
+      dKK[t * LDC + i] = dkk;
+      dQK[t * LDC + i] = dqk;
+      colG[t * LDC + i] = cg;
+      colB[t * LDC + i] = cb;
+      colM[t * LDC + i] = cm;
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+      rowc += __shfl_xor_sync(0xffffffffu, rowc, off);
+      rowp += __shfl_xor_sync(0xffffffffu, rowp, off);
+    }
+    if (lane == 0) {
+      dcum[t] = rowc;
+      dcprev[t] = rowp;
+    }
+  }
+  __syncthreads();
+  // ---- column pass and per-row factors
   if (tid < C) {
-    const int t = tid;
+    const int i = tid;
+    float sg = 0.f, sb = 0.f, sm2 = 0.f;
+    for (int t = i; t < C; ++t) {
+      sg += colG[t * LDC + i];
+      sb += colB[t * LDC + i];
+      sm2 += colM[t * LDC + i];
+    }
     const float cC = cum[C - 1];
-    const float eC = expf(cC - cum[t]);
-    const float dwS = acc[L::VEC + L::V_DWS + t], dwR = acc[L::VEC + L::V_DWR + t];
-    dbet[t] += dwS * eC;
-    dgam[t] += dwR * eC;
-    dcum[t] = acc[L::VEC + L::V_DGAM + t] * expf(cum[t]) - (dwS * bet[t] + dwR * gam[t]) * eC;
-    dcprev[t] = acc[L::VEC + L::V_DGPREV + t] * expf(cprev[t]);
+    const float eC = expf(cC - cum[i]);
+    const float dwS = acc[L::VEC + L::V_DWS + i], dwR = acc[L::VEC + L::V_DWR + i];
+    dbet[i] = sb + dwS * eC;
+    dgam[i] = sm2 + acc[L::VEC + L::V_DGAM_OUT + i] + dwR * eC;
+    // d cum_i: - column sums - (dwS wS + dwR wR) + dGam * Gam
+    dcum[i] += -sg - (dwS * bet[i] + dwR * gam[i]) * eC + acc[L::VEC + L::V_DGAM + i] * expf(cum[i]);
+    dcprev[i] += acc[L::VEC + L::V_DGPREV + i] * expf(cprev[i]);
   }
   __syncthreads();
-  if (tid < C) {  // the chunk-end terms land on cum_C (= cum[C-1]; padding has g = 0)
+  if (warp == 0) {  // chunk-end terms land on cum_C = cum[C-1] (padding has g = 0)
+    const float cC = cum[C - 1];
     float s = 0.f;
-    const float cC = cum[C - 1];
-    for (int t = 0; t < C; ++t) {
-      const float eC = expf(cC - cum[t]);
-      s += (acc[L::VEC + L::V_DWS + t] * bet[t] + acc[L::VEC + L::V_DWR + t] * gam[t]) * eC;
-    }
-    if (tid == C - 1) dcum[C - 1] += s + acc[L::VEC + L::V_DGAMC] * expf(cC);
+    for (int t = lane; t < C; t += 32)
+      s += (acc[L::VEC + L::V_DWS + t] * bet[t] + acc[L::VEC + L::V_DWR + t] * gam[t]) *
+           expf(cC - cum[t]);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) dcum[C - 1] += s + acc[L::VEC + L::V_DGAMC] * expf(cC);
   }
-  __syncthreads();
-  // C x C gradients -> d(KK), d(QK), rates and cumulative log-decay
-  for (int e = tid; e < C * C; e += kThreads) {
-    const int t = e / C, i = e % C;
-    float dkk = 0.f, dqk = 0.f;
-    if (i <= t) {
-      const float dec = expf(cum[t] - cum[i]);
-      const float kk = KK[t * LDC + i], qk = QK[t * LDC + i];
-      float rowc = 0.f, rowp = 0.f, colc = 0.f;
-      // M2 (inclusive, gamma, QK)
-      {
-        const float dm = acc[L::DM2 + e];
-        const float m = dec * gam[i] * qk;
-        rowc += dm * m;
-        colc += dm * m;
-        atomicAdd(&dgam[i], dm * dec * qk);
-        dqk += dm * dec * gam[i];
-      }
-      if (i < t) {
-        const float decp = expf(cprev[t] - cum[i]);
-        {  // Ap (strict, beta, KK, previous-token decay)
-          const float dm = acc[L::DAP + e];
-          const float m = decp * bet[i] * kk;
-          rowp += dm * m;
-          colc += dm * m;
-          atomicAdd(&dbet[i], dm * decp * kk);
-          dkk += dm * decp * bet[i];
-        }
-        {  // Mq (strict, beta, QK)
-          const float dm = acc[L::DMQ + e];
-          const float m = dec * bet[i] * qk;
-          rowc += dm * m;
-          colc += dm * m;
-          atomicAdd(&dbet[i], dm * dec * qk);
-          dqk += dm * dec * bet[i];
-        }
-        if (RDNV) {
-          {  // Ab (strict, beta, KK)
-            const float dm = acc[L::DAB + e];
-            const float m = dec * bet[i] * kk;
-            rowc += dm * m;
-            colc += dm * m;
-            atomicAdd(&dbet[i], dm * dec * kk);
-            dkk += dm * dec * bet[i];
-          }
-          {  // Ag (strict, gamma, KK)
-            const float dm = acc[L::DAG + e];
-            const float m = dec * gam[i] * kk;
-            rowc += dm * m;
-            colc += dm * m;
-            atomicAdd(&dgam[i], dm * dec * kk);
-            dkk += dm * dec * gam[i];
-          }
-        }
-      }
-      atomicAdd(&dcum[t], rowc);
-      atomicAdd(&dcprev[t], rowp);
-      atomicAdd(&dcum[i], -colc);
-    }
-    dKK[t * LDC + i] = dkk;
-    dQK[t * LDC + i] = dqk;
-  }
-  __syncthreads();
   // symmetrise: dK gets (dKK + dKK^T) K
   for (int e = tid; e < C * C; e += kThreads) {
     const int t = e / C, i = e % C;
     if (i < t) {
-      const float s = dKK[t * LDC + i] + dKK[i * LDC + t];
-      dKK[t * LDC + i] = s;
-      dKK[i * LDC + t] = s;
+      const float s2 = dKK[t * LDC + i] + dKK[i * LDC + t];
+      dKK[t * LDC + i] = s2;
+      dKK[i * LDC + t] = s2;
     } else if (i == t) {
       dKK[t * LDC + i] *= 2.f;
     }
@@ -631,14 +657,27 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
       }
     }
   }
-  if (tid == 0) {  // dg_s = sum_{t>=s} dcum_t + sum_{t>s} dcprev_t
-    float s1 = 0.f, s2 = 0.f;
-    for (int t = C - 1; t >= 0; --t) {
-      s1 += dcum[t];
-      const float dgt = s1 + s2;
-      s2 += dcprev[t];
-      gg[t] = dgt;
+  if (warp == 0) {  // dg_s = sum_{t>=s} dcum_t + sum_{t>s} dcprev_t (reverse scans)
+    float a = dcum[C - 1 - lane], b2 = dcum[31 - lane];
+    float pa = dcprev[C - 1 - lane], pb = dcprev[31 - lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float ua = __shfl_up_sync(0xffffffffu, a, off), ub = __shfl_up_sync(0xffffffffu, b2, off);
+      const float upa = __shfl_up_sync(0xffffffffu, pa, off), upb = __shfl_up_sync(0xffffffffu, pb, off);
+      if (lane >= off) {
+        a += ua;
+        b2 += ub;
+        pa += upa;
+        pb += upb;
+      }
     }
+    // a: suffix sums over t in [C-1-lane, C) ; b2 over [31-lane, 32) plus the upper half
+    const float topc = __shfl_sync(0xffffffffu, a, 31), topp = __shfl_sync(0xffffffffu, pa, 31);
+    b2 += topc;
+    pb += topp;
+    // sum_{t>s} dcprev_t = (suffix including s) - dcprev_s
+    gg[C - 1 - lane] = a + (pa - dcprev[C - 1 - lane]);
+    gg[31 - lane] = b2 + (pb - dcprev[31 - lane]);
   }
   __syncthreads();
   if (tid < n) {
@@ -655,7 +694,7 @@ constexpr size_t scan_smem() {
 }
 template <int DK>
 constexpr size_t finish_smem() {
-  return sizeof(float) * (2 * C * (DK + 1) + 4 * C * (C + 1) + 9 * C);
+  return sizeof(float) * (2 * C * (DK + 1) + 7 * C * (C + 1) + 9 * C);
 }
 
 template <int DK, bool RDNV, typename InT>

@@ -43,6 +43,55 @@ __device__ __forceinline__ void img_put(uint8_t *tile, uint32_t lo_off, int r, i
   *reinterpret_cast<__nv_bfloat16 *>(tile + lo_off + o) = __float2bfloat16_rn(x - __bfloat162float(hi));
 }
 
+// (I + A)^-1 for a 64 x 64 strictly lower A (row stride ld), by 16 x 16
+// blocks, with 128 threads (g = thread index within the group):
+//   diagonal blocks  T_ii = (I + A_ii)^-1 by forward substitution (one thread
+//                    per block column, the column kept in registers);
+//   block row i      W_j = sum_{k=j}^{i-1} A_ik T_kj,  T_ij = -T_ii W_j.
+// W is scratch of 3 x 256 floats.  The caller synchronises the block between
+// the calls of the 4 stages (stage 0: diagonal; stage i: block row i).
+__device__ __forceinline__ void inv_diag_blocks(const float *A, float *Tm, int ld, int g) {
+  if (g < 64) {
+    const int blk = g >> 4, col = g & 15, b0 = blk * 16;
+    float x[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      float s = (r == col) ? 1.f : 0.f;
+#pragma unroll
+      for (int m = 0; m < r; ++m) s = fmaf(-A[(b0 + r) * ld + b0 + m], x[m], s);
+      x[r] = (r < col) ? 0.f : s;
+    }
+#pragma unroll
+    for (int r = 0; r < 16; ++r) Tm[(b0 + r) * ld + b0 + col] = x[r];
+  }
+  // zero the strictly upper blocks once
+  for (int e = g; e < 64 * 64; e += 128) {
+    const int r = e >> 6, c = e & 63;
+    if ((c >> 4) > (r >> 4)) Tm[r * ld + c] = 0.f;
+  }
+}
+__device__ __forceinline__ void inv_block_row_w(const float *A, const float *Tm, float *W, int ld,
+                                                int i, int g) {
+  for (int e = g; e < i * 256; e += 128) {
+    const int j = e >> 8, r = (e >> 4) & 15, cc = e & 15;
+    float s = 0.f;
+    for (int k = j; k < i; ++k)
+#pragma unroll
+      for (int m = 0; m < 16; ++m)
+        s = fmaf(A[(16 * i + r) * ld + 16 * k + m], Tm[(16 * k + m) * ld + 16 * j + cc], s);
+    W[e] = s;
+  }
+}
+__device__ __forceinline__ void inv_block_row_t(float *Tm, const float *W, int ld, int i, int g) {
+  for (int e = g; e < i * 256; e += 128) {
+    const int j = e >> 8, r = (e >> 4) & 15, cc = e & 15;
+    float s = 0.f;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) s = fmaf(Tm[(16 * i + r) * ld + 16 * i + m], W[j * 256 + m * 16 + cc], s);
+    Tm[(16 * i + r) * ld + 16 * j + cc] = -s;
+  }
+}
+
 template <int DK, bool RDNV, typename InT, bool IMG>
 __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   constexpr int LDK = DK + 1;
@@ -61,6 +110,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   float *bet = cprev + C;         // [C]
   float *gam = bet + C;           // [C]
   float *gg = gam + C;            // [C]
+  float *Wsc = gg + C;            // [2][3*256] scratch of the blocked inverse
 
   const int chunk = blockIdx.x;
   const int bh = chunk / p.NC, c = chunk % p.NC;
@@ -157,16 +207,19 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   }
   if (RDNV) {
     __syncthreads();
-    // (I + A)^-1 by forward substitution, one column per thread:
-    // threads 0..63 invert I + A_beta, threads 64..127 invert I + A_gamma.
-    if (tid < 2 * C) {
-      const int j = tid % C;
-      const float *A = tid < C ? Ab : Ag;
-      float *Tm = tid < C ? Tb : Tg;
-      for (int t = 0; t < C; ++t) {
-        float s = (t == j) ? 1.f : 0.f;
-        for (int i = j; i < t; ++i) s = fmaf(-A[t * LDC + i], Tm[i * LDC + j], s);
-        Tm[t * LDC + j] = (t < j) ? 0.f : s;
+    // (I + A)^-1 by 16 x 16 blocks: threads 0..127 invert I + A_beta,
+    // threads 128..255 invert I + A_gamma.
+    {
+      const int g = tid & 127;
+      const float *A = tid < 128 ? Ab : Ag;
+      float *Tm = tid < 128 ? Tb : Tg;
+      float *W = Wsc + (tid < 128 ? 0 : 768);
+      inv_diag_blocks(A, Tm, LDC, g);
+      for (int i = 1; i < 4; ++i) {
+        __syncthreads();
+        inv_block_row_w(A, Tm, W, LDC, i, g);
+        __syncthreads();
+        inv_block_row_t(Tm, W, LDC, i, g);
       }
     }
     __syncthreads();
@@ -381,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
 
 template <int DK>
 constexpr size_t prep_smem() {
-  return sizeof(float) * (2 * C * (DK + 1) + 6 * C * (C + 1) + 5 * C);
+  return sizeof(float) * (2 * C * (DK + 1) + 6 * C * (C + 1) + 5 * C + 2 * 768);
 }
 template <int DK>
 constexpr size_t scan_smem() {
