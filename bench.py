@@ -40,17 +40,24 @@ C = 64
 #     the state-carrying scan   12 d^2 + 5 C d   (products with S, R and the
 #                                                 C x C x d_v chunk products)
 #     the per-chunk prep        2 C d + (4/3) C^2 (Gram matrices, inverses)
-#   backward = 2 x forward (two products per forward product), same split.
+#   backward = 2 x forward (two products per forward product), same split:
+#     the reverse scan carrying dS, dR            12 d^2 + 5 C d
+#     the products over the value dimension        12 d^2 + 5 C d
+#     (dK, dQ state terms; C x C gradients)
+#     the backward of the prep                     2 (2 C d + (4/3) C^2)
+#   recomputation of forward pieces is not algorithmic work (counted 0).
 def flops_per_token_head(d=128, c=C):
     scan = 12 * d * d + 5 * c * d
     prep = 2 * c * d + (4.0 / 3.0) * c * c
     return dict(fwd=scan + prep, fwd_scan=scan, fwd_prep=prep, bwd_scan=2 * scan,
-                bwd_finish=2 * prep, step=3 * (scan + prep))
+                bwd_chain=scan, bwd_post=scan, bwd_finish=2 * prep, recompute=0.0,
+                step=3 * (scan + prep))
 
 
 # kernel name (as recorded by the library) -> algorithmic flop per token-head
-KERNEL_WORK = {"chunk_scan": "fwd_scan", "chunk_prep": "fwd_prep", "bwd_scan": "bwd_scan",
-               "bwd_finish": "bwd_finish"}
+KERNEL_WORK = {"chunk_scan": "fwd_scan", "fwd_tc_scan": "fwd_scan", "chunk_prep": "fwd_prep",
+               "bwd_scan": "bwd_scan", "bwd_chain": "bwd_chain", "bwd_post": "bwd_post",
+               "bwd_finish": "bwd_finish", "bwd_recompute": "recompute"}
 
 # decode: read + write S and R fp32, plus q, k, v, o bf16 and three fp32 gates
 def decode_bytes_per_head(d=128):

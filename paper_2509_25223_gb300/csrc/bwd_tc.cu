@@ -1,0 +1,1132 @@
+// bwd_tc.cu -- tensor-core (tcgen05 / TMEM) backward of the chunkwise RDN
+// forward, bf16 inputs, d_k = d_v = 128.
+//
+// Reverse mode of the chunk algebra of chunk_fwd.cu (the same steps as
+// chunk_bwd.cu, whose header lists them), split by what depends on the
+// gradients carried between chunks:
+//
+//  1. bwd_recompute (parallel, one CTA per chunk): from the chunk-start
+//     states rebuild E, E2, the clip mask and the read-out term
+//     dgamma_t += dO_t . Oa_t (the forward's pieces for one chunk).
+//  2. bwd_chain (sequential over chunks, one CTA per (b,h)): the carried
+//     gradients.  With dR, dS the gradients w.r.t. a chunk's end states,
+//        dE2 = M2^T dOa + diag(wR) K dR        dX2 = T_gamma^T dE2
+//        dP  = -mask * dX2                     dKR = -diag(Gam) dX2
+//        dR_prev = Gam_C dR + K^T dKR + Q^T diag(Gam gamma) dO
+//        dE  = Mq^T dO + Ap^T dP + diag(wS) K dS     dX = T_beta^T dE
+//        dKS = diag(Gprev) dP - diag(Gam) dX
+//        dS_prev = Gam_C dS + K^T dKS + Q^T diag(Gam) dO
+//        dv  = -dP + dX
+//     No forward quantity other than the clip mask enters this chain.
+//  3. bwd_post (parallel, one CTA per chunk): every product that reduces over
+//     the value dimension -- the state terms of dK, dQ, the five C x C
+//     gradients, the per-row gate terms -- written to the per-chunk record
+//     that bwd_finish (chunk_bwd.cu) turns into dq, dk, dg, dbeta, dgamma.
+//
+// Orientation: thread j of 128 owns value column j = TMEM lane j for every
+// column quantity (X, E, dO, dX2, ...), which is kept as a bf16 hi + lo tile
+// [j][t] (K-major for products over t).  Products over j use the same tiles
+// as MN-major operands.  The chunk matrices come from chunk_prep's images
+// (bf16 hi + lo); products with them are three MMAs (hi*hi + hi*lo + lo*hi).
+// States and carried gradients enter their products as bf16 hi + lo as well.
+#include "chunk_common.cuh"
+#include "tc_common.cuh"
+
+namespace rdn {
+namespace {
+
+using namespace tc;
+
+constexpr int D = 128;
+constexpr int NT = 128;  // threads per CTA
+
+template <int DK>
+struct AccL;  // layout of the per-chunk record, identical to chunk_bwd.cu's
+template <>
+struct AccL<128> {
+  static constexpr int DKo = 0, DQo = C * 128;
+  static constexpr int DAP = 2 * C * 128, DMQ = DAP + kCC, DM2 = DMQ + kCC, DAB = DM2 + kCC,
+                       DAG = DAB + kCC, VEC = DAG + kCC;
+  static constexpr int V_DGAM_OUT = 0, V_DGAM = C, V_DGPREV = 2 * C, V_DWS = 3 * C,
+                       V_DWR = 4 * C, V_DGAMC = 5 * C;
+  static constexpr int FLOATS = VEC + 6 * C;
+};
+using A8 = AccL<128>;
+
+struct TcBwdParams {
+  FwdParams f;          // inputs; f.ws = prep records (shared-memory images)
+  const void *dO;
+  const float *dST, *dRT;
+  const float *Sc, *Rc;  // chunk-start states [B,H,NC,D,D]
+  void *dv;
+  float *dS0, *dR0;
+  float *acc;            // per-chunk records
+  float *Ebuf, *E2buf;   // [B*H*NC][64][128] fp32 (t, j)
+  float *dX2buf, *dXbuf; // [B*H*NC][64][128]
+  float *dSc, *dRc;      // [B*H*NC][128][128] (i, j): gradients w.r.t. chunk-end states
+  unsigned long long *mask;  // [B*H*NC][128]: bit t = clip inactive (|x| <= c)
+  uint8_t *gM2;              // [B*H*NC][16 KB]: image of diag(gamma) M2 (hi | lo)
+};
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Row r, columns c0..c0+15 of a K-major SW128 tile (64-col blocks blk apart).
+__device__ __forceinline__ void put16(uint8_t *tile, uint32_t blk, int r, int c0,
+                                      const float (&v)[16]) {
+  uint8_t *b = tile + (c0 >> 6) * blk;
+  const int cc = c0 & 63;
+  uint4 x, y;
+  x.x = pack2(v[0], v[1]); x.y = pack2(v[2], v[3]); x.z = pack2(v[4], v[5]); x.w = pack2(v[6], v[7]);
+  y.x = pack2(v[8], v[9]); y.y = pack2(v[10], v[11]); y.z = pack2(v[12], v[13]); y.w = pack2(v[14], v[15]);
+  *reinterpret_cast<uint4 *>(b + sw128(r, cc)) = x;
+  *reinterpret_cast<uint4 *>(b + sw128(r, cc + 8)) = y;
+}
+// hi / lo split of 16 values into two single-block tiles
+__device__ __forceinline__ void put16s(uint8_t *hi, uint8_t *lo, int r, int c0,
+                                       const float (&v)[16]) {
+  float a[16], b[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+    b[i] = v[i] - a[i];
+  }
+  put16(hi, 0, r, c0, a);
+  put16(lo, 0, r, c0, b);
+}
+// a whole 64-value row, split
+__device__ __forceinline__ void put64s(uint8_t *hi, uint8_t *lo, int r, const float (&v)[64]) {
+#pragma unroll
+  for (int c0 = 0; c0 < 64; c0 += 16) {
+    float w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
+    put16s(hi, lo, r, c0, w);
+  }
+}
+
+// K-major A (single block, K = 64) times MN-major B, split both: 3 products
+__device__ __forceinline__ void mma_s3_kmn(uint32_t d, uint32_t a_hi, uint32_t a_lo,
+                                           uint32_t b_hi, uint32_t b_lo, uint32_t b_lbo,
+                                           uint32_t idesc, bool acc_first) {
+  mma_tile_kmn(d, a_hi, 0, b_hi, b_lbo, 4, idesc, acc_first);
+  mma_tile_kmn(d, a_hi, 0, b_lo, b_lbo, 4, idesc, true);
+  mma_tile_kmn(d, a_lo, 0, b_hi, b_lbo, 4, idesc, true);
+}
+// K-major A and B (single block, K = 64), split both
+__device__ __forceinline__ void mma_s3_kk(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint32_t b_hi,
+                                          uint32_t b_lo, uint32_t idesc, bool acc_first) {
+  mma_tile(d, a_hi, 0, b_hi, 0, 4, idesc, acc_first);
+  mma_tile(d, a_hi, 0, b_lo, 0, 4, idesc, true);
+  mma_tile(d, a_lo, 0, b_hi, 0, 4, idesc, true);
+}
+
+// Common per-CTA machinery: mbarriers (MMA, slot A, slot B), TMEM, phases.
+struct Ctl {
+  uint64_t *bar, *barA, *barB;
+  volatile int *flag;
+  uint32_t phase, phA, phB;
+};
+
+__device__ __forceinline__ void ctl_init(Ctl &k, uint8_t *base, int tid) {
+  k.bar = reinterpret_cast<uint64_t *>(base);
+  k.barA = k.bar + 1;
+  k.barB = k.bar + 2;
+  k.flag = reinterpret_cast<volatile int *>(base + 28);
+  k.phase = k.phA = k.phB = 0;
+  if (tid == 0) {
+    mbar_init(k.bar, 1);
+    mbar_init(k.barA, 1);
+    mbar_init(k.barB, 1);
+    fence_mbar_init();
+    *k.flag = 0;
+  }
+}
+
+__device__ __forceinline__ void load_slot(uint8_t *dst, uint64_t *bar, const void *src,
+                                          uint32_t bytes) {
+  mbar_expect_tx(bar, bytes);
+  bulk_g2s(dst, src, bytes, bar);
+}
+
+// One MMA phase: publish shared-memory writes, issue (thread 0), wait.
+template <typename F>
+__device__ __forceinline__ bool phase_run(Ctl &k, int tid, F issue) {
+  fence_async_smem();
+  fence_before_sync();
+  __syncthreads();
+  if (tid == 0) {
+    fence_after_sync();
+    if (!issue()) *k.flag = 1;
+    mma_commit(k.bar);
+  }
+  const bool ok = mbar_wait(k.bar, k.phase);
+  k.phase ^= 1u;
+  if (!ok) *k.flag = 1;
+  __syncthreads();
+  fence_after_sync();
+  return *k.flag == 0;
+}
+
+// thread 0: wait for a slot's bulk copy
+__device__ __forceinline__ bool slot_wait(uint64_t *bar, uint32_t &ph) {
+  const bool ok = mbar_wait(bar, ph);
+  ph ^= 1u;
+  return ok;
+}
+
+__device__ __forceinline__ const uint8_t *rec_bytes(const FwdParams &p, size_t chunk) {
+  return reinterpret_cast<const uint8_t *>(p.ws + chunk * kRecFloats);
+}
+
+// Per-row sums over the CTA's 128 columns of a vector v[64] (one value per
+// token t per thread): out[t] in shared memory.  `scratch` holds 4*64 floats.
+__device__ __forceinline__ void cta_row_sum(const float (&v)[64], float *scratch, float *out,
+                                            int tid) {
+  const int warp = tid >> 5, lane = tid & 31;
+  const int tb = transpose_reduce_tbase(lane);
+  float o2[2];
+  warp_transpose_reduce64(v, o2);
+  scratch[warp * 64 + tb] = o2[0];
+  scratch[warp * 64 + tb + 1] = o2[1];
+  __syncthreads();
+  if (tid < 64) out[tid] = scratch[tid] + scratch[64 + tid] + scratch[128 + tid] + scratch[192 + tid];
+  __syncthreads();
+}
+
+// ======================================================================== 1
+// bwd_recompute: the forward pieces of one chunk from its start states.
+namespace rc {
+constexpr uint32_t SA = 0, RA = 32768, B1 = 65536, SLOTA = 98304, SLOTB = 114688;
+constexpr uint32_t XE = 147456, XE_LO = 163840, VEC = 180224;
+constexpr uint32_t RED = VEC + 7 * 64 * 4;       // 4*64 floats
+constexpr uint32_t CTL = RED + 4 * 64 * 4;
+constexpr uint32_t SLOT = CTL + 32;
+constexpr size_t SMEM = SLOT + 16;
+constexpr uint32_t T_D1 = 0, T_D3 = 128, T_X = 256;
+}  // namespace rc
+
+__global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
+  using namespace rc;
+  extern __shared__ __align__(1024) uint8_t sm[];
+  const uint32_t sb = smem_u32(sm);
+  const FwdParams &p = P.f;
+  if (sb & 1023u) {
+    if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
+    return;
+  }
+  float *vec = reinterpret_cast<float *>(sm + VEC);
+  float *Gam = vec, *Gprev = vec + 64, *alpha = vec + 128, *gamv = vec + 320;
+  float *red = reinterpret_cast<float *>(sm + RED);
+  uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
+  const int tid = threadIdx.x, warp = tid >> 5, j = tid;
+  const size_t chunk = blockIdx.x;
+  const int NC = p.NC, T = p.T, H = p.H;
+  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
+  const int b = bh / H, h = bh % H;
+  const int t0 = c * 64, n = min(64, T - t0);
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
+                      *v = (const __nv_bfloat16 *)p.v, *dO = (const __nv_bfloat16 *)P.dO;
+  const uint8_t *rec = rec_bytes(p, chunk);
+  const float clip = p.clip;
+
+  Ctl K;
+  ctl_init(K, sm + CTL, tid);
+  if (warp == 0) tmem_alloc(slot, 512);
+  if (tid == 0) {
+    load_slot(sm + SLOTA, K.barA, rec + IMG_TB, 16384);
+    load_slot(sm + SLOTB, K.barB, rec + IMG_APMQ, 32768);
+  }
+  if (tid < 64) {
+    Gam[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GAM + tid];
+    Gprev[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GPREV + tid];
+    alpha[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_ALPHA + tid];
+    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+  }
+  // chunk-start states -> bf16 A operands (row j = column j of [i][j])
+  {
+    const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], r[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        s[i] = S0[(size_t)(c0 + i) * D + j];
+        r[i] = R0[(size_t)(c0 + i) * D + j];
+      }
+      put16(sm + SA, 16384, j, c0, s);
+      put16(sm + RA, 16384, j, c0, r);
+    }
+  }
+  __syncthreads();
+  // B1 = [Gprev K ; Gam Q]
+  for (int e = tid; e < 64 * 16; e += NT) {
+    const int t = e >> 4, ch = e & 15;
+    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+    if (t < n) {
+      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8;
+      kv = *reinterpret_cast<const uint4 *>(k + off);
+      qv = *reinterpret_cast<const uint4 *>(q + off);
+    }
+    const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
+    const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(&qv);
+    const float gk = Gprev[t], gq = Gam[t] * p.scale;
+    uint4 ks, qs;
+    uint32_t *kw = &ks.x, *qw = &qs.x;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      kw[i] = pack2(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
+      qw[i] = pack2(gq * __bfloat162float(qb[2 * i]), gq * __bfloat162float(qb[2 * i + 1]));
+    }
+    const int blk = ch >> 3, cc = (ch & 7) * 8;
+    *reinterpret_cast<uint4 *>(sm + B1 + blk * 16384 + sw128(t, cc)) = ks;
+    *reinterpret_cast<uint4 *>(sm + B1 + blk * 16384 + sw128(64 + t, cc)) = qs;
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  auto vval = [&](int t) -> float {
+    return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  };
+
+  bool ok = phase_run(K, tid, [&] {
+    mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 128), false);
+    mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 128), false);
+    return true;
+  });
+  float r[64];
+  if (ok) {  // X = V - alpha * (Gprev KS) -> E = T_beta X
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float x[16];
+      tmem_ld16(tm + lane + T_D1 + c0, x);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = vval(c0 + i) - alpha[c0 + i] * x[i];
+      put16s(sm + XE, sm + XE_LO, j, c0, x);
+    }
+    ok = phase_run(K, tid, [&] {
+      if (!slot_wait(K.barA, K.phA)) return false;
+      mma_s3_kk(tm + T_X, sb + XE, sb + XE_LO, sb + SLOTA, sb + SLOTA + 8192, idesc_bf16(128, 64),
+                 false);
+      return true;
+    });
+  }
+  if (ok) {
+    if (tid == 0) load_slot(sm + SLOTA, K.barA, rec + IMG_TG, 16384);
+    float *Eg = P.Ebuf + chunk * 64 * D;
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float e[16];
+      tmem_ld16(tm + lane + T_X + c0, e);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) Eg[(c0 + i) * D + j] = e[i];
+      put16s(sm + XE, sm + XE_LO, j, c0, e);
+    }
+    ok = phase_run(K, tid, [&] {  // D1 += E [Ap ; Mq]^T -> [P | Ob]
+      if (!slot_wait(K.barB, K.phB)) return false;
+      mma_s3_kk(tm + T_D1, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 16384,
+                 idesc_bf16(128, 128), true);
+      return true;
+    });
+  }
+  if (ok) {
+    if (tid == 0) load_slot(sm + SLOTB, K.barB, rec + IMG_M2, 16384);
+    unsigned long long m = 0ull;
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float pp[16], kr[16];
+      tmem_ld16(tm + lane + T_D1 + c0, pp);
+      tmem_ld16(tm + lane + T_D3 + c0, kr);
+      float x2[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = c0 + i;
+        const float x = vval(t) - pp[i];
+        if (fabsf(x) <= clip) m |= 1ull << t;
+        r[t] = clampf(x, clip);
+        x2[i] = r[t] - alpha[t] * kr[i];
+      }
+      put16s(sm + XE, sm + XE_LO, j, c0, x2);
+    }
+    P.mask[chunk * D + j] = m;
+    ok = phase_run(K, tid, [&] {  // E2 = T_gamma X2
+      if (!slot_wait(K.barA, K.phA)) return false;
+      mma_s3_kk(tm + T_X, sb + XE, sb + XE_LO, sb + SLOTA, sb + SLOTA + 8192, idesc_bf16(128, 64),
+                 false);
+      return true;
+    });
+  }
+  if (ok) {
+    float *E2g = P.E2buf + chunk * 64 * D;
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float e[16];
+      tmem_ld16(tm + lane + T_X + c0, e);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) E2g[(c0 + i) * D + j] = e[i];
+      put16s(sm + XE, sm + XE_LO, j, c0, e);
+    }
+    ok = phase_run(K, tid, [&] {  // Oa = Gam QR + M2 E2 (into D3[:, 64:128])
+      if (!slot_wait(K.barB, K.phB)) return false;
+      mma_s3_kk(tm + T_D3 + 64, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 8192,
+                 idesc_bf16(128, 64), true);
+      return true;
+    });
+  }
+  if (ok) {
+    // image of diag(gamma) M2 (rows s scaled by gamma_s) for the chain's
+    // M2^T (gamma dO) product; same swizzled positions as the M2 image
+    uint8_t *dstimg = P.gM2 + chunk * 16384;
+    for (int e = tid; e < 64 * 8; e += NT) {
+      const int r = e >> 3, c8 = (e & 7) * 8;
+      const uint32_t o = sw128(r, c8);
+      const uint4 hv = *reinterpret_cast<const uint4 *>(sm + SLOTB + o);
+      const uint4 lv = *reinterpret_cast<const uint4 *>(sm + SLOTB + 8192 + o);
+      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
+      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
+      float w[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) w[i] = gamv[r] * (__bfloat162float(hb[i]) + __bfloat162float(lb[i]));
+      uint4 ho, lo;
+      uint32_t *hw = &ho.x, *lw = &lo.x;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float a0 = __bfloat162float(__float2bfloat16_rn(w[2 * i]));
+        const float a1 = __bfloat162float(__float2bfloat16_rn(w[2 * i + 1]));
+        hw[i] = pack2(a0, a1);
+        lw[i] = pack2(w[2 * i] - a0, w[2 * i + 1] - a1);
+      }
+      *reinterpret_cast<uint4 *>(dstimg + o) = ho;
+      *reinterpret_cast<uint4 *>(dstimg + 8192 + o) = lo;
+    }
+  }
+  if (ok) {  // d gamma_t (read-out) = sum_j dO[t,j] Oa[t,j]
+    float prod[64];
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float oa[16];
+      tmem_ld16(tm + lane + T_D3 + 64 + c0, oa);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = c0 + i;
+        const float d =
+            t < n ? __bfloat162float(dO[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+        prod[t] = d * oa[i];
+      }
+    }
+    float *out = reinterpret_cast<float *>(sm + XE_LO);
+    cta_row_sum(prod, reinterpret_cast<float *>(sm + XE), out, tid);
+    float *acc = P.acc + chunk * A8::FLOATS;
+    if (tid < 64) acc[A8::VEC + A8::V_DGAM_OUT + tid] = out[tid];
+  } else if (tid == 0 && p.err) {
+    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+// ======================================================================== 2
+// bwd_chain: the gradients carried between chunks, chunks in reverse.
+namespace ch {
+// K, Q | carried gradients dS, dR as bf16 hi + lo A operands (phase A) | slots
+// | dO.  After phase A the 128 KB of gradient tiles serve as scratch for the
+// split column tiles; the gradient tiles are rewritten at the chunk end.
+constexpr uint32_t KQ = 0;
+constexpr uint32_t DSH = 32768, DRH = 65536, DSL = 98304, DRL = 131072;
+constexpr uint32_t SLOTA = 163840;   // diag(gamma) M2 -> T_gamma -> T_beta (16 KB)
+constexpr uint32_t SLOTB = 180224;   // Mq -> Ap (hi 8 KB | lo 8 KB)
+constexpr uint32_t DOT = 196608;     // dO^T, exact bf16
+// scratch column tiles (hi, lo) inside the gradient-tile region
+constexpr uint32_t S0H = 32768, S0L = 49152, S1H = 65536, S1L = 81920;
+constexpr uint32_t S2H = 98304, S2L = 114688, S3H = 131072, S3L = 147456;
+constexpr uint32_t VEC = 212992;                 // Gam Gprev wS wR gamma (5 x 64)
+constexpr uint32_t RED = VEC + 5 * 64 * 4;       // 4 x 64 + 64 floats (row sums)
+constexpr uint32_t CTL = RED + 5 * 64 * 4;
+constexpr uint32_t SLOT = CTL + 32;
+constexpr size_t SMEM = SLOT + 16;
+static_assert(SMEM <= 232448, "shared memory");
+constexpr uint32_t T_DS = 0, T_DR = 128, T_R1 = 256, T_R2 = 320, T_R3 = 384, T_R4 = 448;
+}  // namespace ch
+
+__global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
+  using namespace ch;
+  extern __shared__ __align__(1024) uint8_t sm[];
+  const uint32_t sb = smem_u32(sm);
+  const FwdParams &p = P.f;
+  if (sb & 1023u) {
+    if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
+    return;
+  }
+  float *vec = reinterpret_cast<float *>(sm + VEC);
+  float *Gam = vec, *Gprev = vec + 64, *wS = vec + 128, *wR = vec + 192, *gamv = vec + 256;
+  uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
+  const int tid = threadIdx.x, warp = tid >> 5, j = tid;
+  const int bh = blockIdx.x;
+  const int NC = p.NC, T = p.T, H = p.H;
+  const int b = bh / H, h = bh % H;
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
+                      *dOp = (const __nv_bfloat16 *)P.dO;
+  __nv_bfloat16 *dv = (__nv_bfloat16 *)P.dv;
+  const size_t st_base = (size_t)bh * D * D;
+
+  Ctl K;
+  ctl_init(K, sm + CTL, tid);
+  if (warp == 0) tmem_alloc(slot, 512);
+  // slot loads: A holds diag(gamma) M2, then T_gamma, then T_beta; B holds
+  // Mq (hi | lo), then Ap (hi | lo) -- each 8 KB half copied from the
+  // [Ap ; Mq] image
+  auto load_mq = [&](size_t ck) {
+    const uint8_t *r = rec_bytes(p, ck);
+    mbar_expect_tx(K.barB, 16384);
+    bulk_g2s(sm + SLOTB, r + IMG_APMQ + 8192, 8192, K.barB);
+    bulk_g2s(sm + SLOTB + 8192, r + IMG_APMQ + 16384 + 8192, 8192, K.barB);
+  };
+  auto load_ap = [&](size_t ck) {
+    const uint8_t *r = rec_bytes(p, ck);
+    mbar_expect_tx(K.barB, 16384);
+    bulk_g2s(sm + SLOTB, r + IMG_APMQ, 8192, K.barB);
+    bulk_g2s(sm + SLOTB + 8192, r + IMG_APMQ + 16384, 8192, K.barB);
+  };
+  if (tid == 0) {
+    const size_t last = (size_t)bh * NC + NC - 1;
+    load_slot(sm + SLOTA, K.barA, P.gM2 + last * 16384, 16384);
+    load_mq(last);
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  // carried gradients (bf16 hi + lo tiles, rows j) from their fp32 TMEM copy
+  auto write_grad_tiles = [&]() {
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], r[16], sh[16], sl[16], rh[16], rl[16];
+      tmem_ld16(tm + lane + T_DS + c0, s);
+      tmem_ld16(tm + lane + T_DR + c0, r);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        sh[i] = __bfloat162float(__float2bfloat16_rn(s[i]));
+        sl[i] = s[i] - sh[i];
+        rh[i] = __bfloat162float(__float2bfloat16_rn(r[i]));
+        rl[i] = r[i] - rh[i];
+      }
+      put16(sm + DSH, 16384, j, c0, sh);
+      put16(sm + DSL, 16384, j, c0, sl);
+      put16(sm + DRH, 16384, j, c0, rh);
+      put16(sm + DRL, 16384, j, c0, rl);
+    }
+  };
+  for (int c0 = 0; c0 < D; c0 += 16) {  // upstream gradients of the final states
+    float s[16], r[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      s[i] = P.dST ? P.dST[st_base + (size_t)(c0 + i) * D + j] : 0.f;
+      r[i] = P.dRT ? P.dRT[st_base + (size_t)(c0 + i) * D + j] : 0.f;
+    }
+    tmem_st16(tm + lane + T_DS + c0, s);
+    tmem_st16(tm + lane + T_DR + c0, r);
+  }
+  write_grad_tiles();
+
+  bool ok = true;
+  for (int c = NC - 1; c >= 0 && ok; --c) {
+    const size_t chunk = (size_t)bh * NC + c;
+    const int t0 = c * 64, n = min(64, T - t0);
+    const float *recf = p.ws + chunk * kRecFloats;
+    __syncthreads();
+    {  // gradients w.r.t. this chunk's end states, for bwd_post
+      float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
+      for (int c0 = 0; c0 < D; c0 += 16) {
+        float s[16], r[16];
+        tmem_ld16(tm + lane + T_DS + c0, s);
+        tmem_ld16(tm + lane + T_DR + c0, r);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          gS[(size_t)(c0 + i) * D + j] = s[i];
+          gR[(size_t)(c0 + i) * D + j] = r[i];
+        }
+      }
+    }
+    if (tid < 64) {
+      Gam[tid] = recf[OFF_VEC + V_GAM + tid];
+      Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
+      wS[tid] = recf[OFF_VEC + V_WS + tid];
+      wR[tid] = recf[OFF_VEC + V_WR + tid];
+      gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    }
+    const float GamC = recf[OFF_VEC + V_GAMC];
+    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q (exact bf16) and dO^T
+      const int t = e >> 4, chn = e & 15;
+      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+      if (t < n) {
+        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
+        kv = *reinterpret_cast<const uint4 *>(k + off);
+        qv = *reinterpret_cast<const uint4 *>(q + off);
+        if (p.scale != 1.f) {
+          __nv_bfloat16 *qb = reinterpret_cast<__nv_bfloat16 *>(&qv);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) qb[i] = __float2bfloat16_rn(p.scale * __bfloat162float(qb[i]));
+        }
+      }
+      const int blk = chn >> 3, cc = (chn & 7) * 8;
+      *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
+      *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+    }
+    __syncthreads();
+    float dO[64];
+#pragma unroll
+    for (int t = 0; t < 64; ++t)
+      dO[t] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+    const unsigned long long m = P.mask[chunk * D + j];
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {  // dO^T, exact in bf16
+      float y[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) y[i] = dO[c0 + i];
+      put16(sm + DOT, 0, j, c0, y);
+    }
+    // ---- phase A: K dR, K dS (gradients hi + lo), M2^T (gamma dO), Mq^T dO
+    ok = phase_run(K, tid, [&] {
+      if (!slot_wait(K.barA, K.phA)) return false;
+      if (!slot_wait(K.barB, K.phB)) return false;
+      const uint32_t i64 = idesc_bf16(128, 64);
+      mma_tile(tm + T_R1, sb + DRH, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile(tm + T_R1, sb + DRL, 16384, sb + KQ, 16384, 8, i64, true);
+      mma_tile(tm + T_R2, sb + DSH, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile(tm + T_R2, sb + DSL, 16384, sb + KQ, 16384, 8, i64, true);
+      mma_tile_kmn(tm + T_R3, sb + DOT, 0, sb + SLOTA, 16384, 4, i64, false);
+      mma_tile_kmn(tm + T_R3, sb + DOT, 0, sb + SLOTA + 8192, 16384, 4, i64, true);
+      mma_tile_kmn(tm + T_R4, sb + DOT, 0, sb + SLOTB, 16384, 4, i64, false);
+      mma_tile_kmn(tm + T_R4, sb + DOT, 0, sb + SLOTB + 8192, 16384, 4, i64, true);
+      return true;
+    });
+    if (!ok) break;
+    if (tid == 0) {
+      load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TG, 16384);
+      load_ap(chunk);
+    }
+    // dE2 = M2^T dOa + wR K dR ; dE (partial) = Mq^T dO + wS K dS ; dQR = Gam gamma dO
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float kdr[16], kds[16], m2[16], mq[16], dqr[16];
+      tmem_ld16(tm + lane + T_R1 + c0, kdr);
+      tmem_ld16(tm + lane + T_R2 + c0, kds);
+      tmem_ld16(tm + lane + T_R3 + c0, m2);
+      tmem_ld16(tm + lane + T_R4 + c0, mq);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = c0 + i;
+        m2[i] = m2[i] + wR[t] * kdr[i];
+        mq[i] = mq[i] + wS[t] * kds[i];
+        dqr[i] = Gam[t] * gamv[t] * dO[t];
+      }
+      tmem_st16(tm + lane + T_R4 + c0, mq);
+      put16s(sm + S0H, sm + S0L, j, c0, m2);
+      put16s(sm + S1H, sm + S1L, j, c0, dqr);
+    }
+    {  // dwS_t = sum_j (K dS)[t,j] E[t,j], dwR_t = sum_j (K dR)[t,j] E2[t,j]
+      float *red = reinterpret_cast<float *>(sm + RED);
+      float *acc = P.acc + chunk * A8::FLOATS;
+      const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
+      for (int w = 0; w < 2; ++w) {
+        float pr[64];
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) {
+          float kd[16];
+          tmem_ld16(tm + lane + (w == 0 ? T_R2 : T_R1) + c0, kd);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) pr[c0 + i] = kd[i] * (w == 0 ? Eg : E2g)[(c0 + i) * D + j];
+        }
+        cta_row_sum(pr, red, red + 256, tid);
+        if (tid < 64) acc[A8::VEC + (w == 0 ? A8::V_DWS : A8::V_DWR) + tid] = red[256 + tid];
+      }
+    }
+    // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
+    ok = phase_run(K, tid, [&] {
+      if (!slot_wait(K.barA, K.phA)) return false;
+      mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
+                 idesc_bf16(128, 64), false);
+      const uint32_t i128 = idesc_bf16(128, 128);
+      mma_tile_kmn(tm + T_R1, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, false);
+      mma_tile_kmn(tm + T_R1, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      return true;
+    });
+    if (!ok) break;
+    if (tid == 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TB, 16384);
+    float dP[64];
+    {  // dX2 -> dP = -mask dX2, dKR = -Gam dX2
+      float *gx = P.dX2buf + chunk * 64 * D;
+#pragma unroll
+      for (int c0 = 0; c0 < 64; c0 += 16) {
+        float x[16], dkr[16], dp[16];
+        tmem_ld16(tm + lane + T_R3 + c0, x);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int t = c0 + i;
+          gx[t * D + j] = x[i];
+          dp[i] = ((m >> t) & 1ull) ? -x[i] : 0.f;
+          dP[t] = dp[i];
+          dkr[i] = -Gam[t] * x[i];
+        }
+        put16s(sm + S2H, sm + S2L, j, c0, dkr);
+        put16s(sm + S3H, sm + S3L, j, c0, dp);
+      }
+    }
+    // ---- phase C: U_R += K^T dKR ; Ap^T dP
+    ok = phase_run(K, tid, [&] {
+      if (!slot_wait(K.barB, K.phB)) return false;
+      const uint32_t i128 = idesc_bf16(128, 128);
+      mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
+      mma_s3_kmn(tm + T_R3, sb + S3H, sb + S3L, sb + SLOTB, sb + SLOTB + 8192, 16384,
+                 idesc_bf16(128, 64), false);
+      return true;
+    });
+    if (!ok) break;
+    if (tid == 0 && c > 0) load_mq(chunk - 1);
+    {  // dR update (fp32 in TMEM); dE = dE_partial + Ap^T dP; dQS = Gam dO
+      for (int c0 = 0; c0 < D; c0 += 16) {
+        float r[16], u[16];
+        tmem_ld16(tm + lane + T_DR + c0, r);
+        tmem_ld16(tm + lane + T_R1 + c0, u);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
+        tmem_st16(tm + lane + T_DR + c0, r);
+      }
+#pragma unroll
+      for (int c0 = 0; c0 < 64; c0 += 16) {
+        float a[16], e[16], dqs[16];
+        tmem_ld16(tm + lane + T_R4 + c0, a);
+        tmem_ld16(tm + lane + T_R3 + c0, e);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          a[i] += e[i];
+          dqs[i] = Gam[c0 + i] * dO[c0 + i];
+        }
+        put16s(sm + S0H, sm + S0L, j, c0, a);
+        put16s(sm + S1H, sm + S1L, j, c0, dqs);
+      }
+    }
+    // ---- phase D: dX = T_beta^T dE ; U_S = Q^T dQS
+    ok = phase_run(K, tid, [&] {
+      if (!slot_wait(K.barA, K.phA)) return false;
+      mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
+                 idesc_bf16(128, 64), false);
+      const uint32_t i128 = idesc_bf16(128, 128);
+      mma_tile_kmn(tm + T_R1, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, false);
+      mma_tile_kmn(tm + T_R1, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      return true;
+    });
+    if (!ok) break;
+    if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, P.gM2 + (chunk - 1) * 16384, 16384);
+    {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX
+      float *gx = P.dXbuf + chunk * 64 * D;
+#pragma unroll
+      for (int c0 = 0; c0 < 64; c0 += 16) {
+        float x[16], dks[16];
+        tmem_ld16(tm + lane + T_R3 + c0, x);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int t = c0 + i;
+          gx[t * D + j] = x[i];
+          if (t < n)
+            dv[((size_t)(b * T + t0 + t) * H + h) * D + j] = __float2bfloat16_rn(x[i] - dP[t]);
+          dks[i] = Gprev[t] * dP[t] - Gam[t] * x[i];
+        }
+        put16s(sm + S2H, sm + S2L, j, c0, dks);
+      }
+    }
+    // ---- phase E: U_S += K^T dKS
+    ok = phase_run(K, tid, [&] {
+      const uint32_t i128 = idesc_bf16(128, 128);
+      mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
+      return true;
+    });
+    if (!ok) break;
+    for (int c0 = 0; c0 < D; c0 += 16) {  // dS update
+      float s[16], u[16];
+      tmem_ld16(tm + lane + T_DS + c0, s);
+      tmem_ld16(tm + lane + T_R1 + c0, u);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
+      tmem_st16(tm + lane + T_DS + c0, s);
+    }
+    write_grad_tiles();  // A operands of the next chunk's phase A
+  }
+  if (ok) {
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], r[16];
+      tmem_ld16(tm + lane + T_DS + c0, s);
+      tmem_ld16(tm + lane + T_DR + c0, r);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (P.dS0) P.dS0[st_base + (size_t)(c0 + i) * D + j] = s[i];
+        if (P.dR0) P.dR0[st_base + (size_t)(c0 + i) * D + j] = r[i];
+      }
+    }
+  } else if (tid == 0 && p.err) {
+    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+// ======================================================================== 3
+// bwd_post: the products over the value dimension, one chunk per CTA.
+// States and carried gradients enter as bf16 hi + lo, like the column tiles.
+namespace po {
+// phase 1: chunk-start states (hi | lo, rows j) and K, Q
+constexpr uint32_t S0H = 0, S0L = 32768, R0H = 65536, R0L = 98304, KQ = 131072;
+// later: pair buffer (4 x 16 KB) over the K, Q region, zero tile after it
+constexpr uint32_t C0 = 131072, C1 = 147456, C2 = 163840, C3 = 180224, Z = 196608;
+// phase 4: carried gradients (hi | lo) over the state region
+constexpr uint32_t GRH = 0, GRL = 32768, GSH = 65536, GSL = 98304;
+// phases 5-6: E / E2 (hi, lo) and dX (hi, lo) over the state region
+constexpr uint32_t EH = 0, EL = 16384, XH = 32768, XL = 49152;
+constexpr uint32_t RED = 212992;                 // 4 x 64 + 64 floats
+constexpr uint32_t VEC = RED + 5 * 64 * 4;       // Gam Gprev wS wR gamma (5 x 64)
+constexpr uint32_t CTL = VEC + 5 * 64 * 4;
+constexpr uint32_t SLOT = CTL + 32;
+constexpr size_t SMEM = SLOT + 16;
+static_assert(SMEM <= 232448, "shared memory");
+constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256;
+// after phase 1 the read-out columns hold the C x C gradients
+constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128;
+}  // namespace po
+
+__global__ void __launch_bounds__(NT, 1) bwd_post_kernel(TcBwdParams P) {
+  using namespace po;
+  extern __shared__ __align__(1024) uint8_t sm[];
+  const uint32_t sb = smem_u32(sm);
+  const FwdParams &p = P.f;
+  if (sb & 1023u) {
+    if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
+    return;
+  }
+  float *vec = reinterpret_cast<float *>(sm + VEC);
+  float *Gam = vec, *Gprev = vec + 64, *wS = vec + 128, *wR = vec + 192, *gamv = vec + 256;
+  float *red = reinterpret_cast<float *>(sm + RED);
+  uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
+  const int tid = threadIdx.x, warp = tid >> 5, j = tid;
+  const size_t chunk = blockIdx.x;
+  const int NC = p.NC, T = p.T, H = p.H;
+  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
+  const int b = bh / H, h = bh % H;
+  const int t0 = c * 64, n = min(64, T - t0);
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
+                      *dOp = (const __nv_bfloat16 *)P.dO;
+  const float *recf = p.ws + chunk * kRecFloats;
+  float *acc = P.acc + chunk * A8::FLOATS;
+
+  Ctl K;
+  ctl_init(K, sm + CTL, tid);
+  if (warp == 0) tmem_alloc(slot, 512);
+  if (tid < 64) {
+    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
+    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
+    wS[tid] = recf[OFF_VEC + V_WS + tid];
+    wR[tid] = recf[OFF_VEC + V_WR + tid];
+    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+  }
+  // a [i][j] fp32 matrix -> rows j of a (hi, lo) pair of two-block tiles
+  auto put_state = [&](const float *src, uint32_t hi, uint32_t lo) {
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float v[16], a[16], bb[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        v[i] = src[(size_t)(c0 + i) * D + j];
+        a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+        bb[i] = v[i] - a[i];
+      }
+      put16(sm + hi, 16384, j, c0, a);
+      put16(sm + lo, 16384, j, c0, bb);
+    }
+  };
+  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
+  const float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
+  put_state(S0, S0H, S0L);
+  put_state(R0, R0H, R0L);
+  float gdot = 0.f;  // <dR, R0> + <dS, S0> over this column
+  for (int i = 0; i < D; ++i) {
+    const size_t o = (size_t)i * D + j;
+    gdot += gS[o] * S0[o] + gR[o] * R0[o];
+  }
+  for (int e = tid; e < 64 * 16; e += NT) {  // unscaled K, Q
+    const int t = e >> 4, chn = e & 15;
+    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+    if (t < n) {
+      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
+      kv = *reinterpret_cast<const uint4 *>(k + off);
+      qv = *reinterpret_cast<const uint4 *>(q + off);
+      if (p.scale != 1.f) {
+        __nv_bfloat16 *qb = reinterpret_cast<__nv_bfloat16 *>(&qv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) qb[i] = __float2bfloat16_rn(p.scale * __bfloat162float(qb[i]));
+      }
+    }
+    const int blk = chn >> 3, cc = (chn & 7) * 8;
+    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
+    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
+  const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
+  const unsigned long long m = P.mask[chunk * D + j];
+  auto dov = [&](int t) -> float {
+    return t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  };
+  const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
+
+  // ---- phase 1: read-outs [KS|QS], [KR|QR] with split states
+  bool ok = phase_run(K, tid, [&] {
+    mma_tile(tm + T_KS, sb + S0H, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile(tm + T_KS, sb + S0L, 16384, sb + KQ, 16384, 8, i128, true);
+    mma_tile(tm + T_KR, sb + R0H, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile(tm + T_KR, sb + R0L, 16384, sb + KQ, 16384, 8, i128, true);
+    return true;
+  });
+  if (ok) {  // per-row gate terms dGam, dGprev and <dR,R0> + <dS,S0>
+    for (int w = 0; w < 2; ++w) {
+      float rv[64];
+      if (w == 0) {
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) {
+          float qs[16], qr[16];
+          tmem_ld16(tm + lane + T_KS + 64 + c0, qs);
+          tmem_ld16(tm + lane + T_KR + 64 + c0, qr);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) rv[c0 + i] = dov(c0 + i) * (qs[i] + gamv[c0 + i] * qr[i]);
+        }
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) {
+          float ks[16], kr[16];
+          tmem_ld16(tm + lane + T_KS + c0, ks);
+          tmem_ld16(tm + lane + T_KR + c0, kr);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int t = c0 + i;
+            rv[t] -= X2g[t * D + j] * kr[i] + Xg[t * D + j] * ks[i];
+          }
+        }
+      } else {
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) {
+          float ks[16];
+          tmem_ld16(tm + lane + T_KS + c0, ks);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int t = c0 + i;
+            rv[t] = ((m >> t) & 1ull) ? -X2g[t * D + j] * ks[i] : 0.f;
+          }
+        }
+      }
+      cta_row_sum(rv, red, red + 256, tid);
+      if (tid < 64) acc[A8::VEC + (w == 0 ? A8::V_DGAM : A8::V_DGPREV) + tid] = red[256 + tid];
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
+    if ((tid & 31) == 0) red[warp] = gdot;
+    __syncthreads();
+    if (tid == 0) acc[A8::VEC + A8::V_DGAMC] = red[0] + red[1] + red[2] + red[3];
+    for (int e = tid; e < 16384 / 16; e += NT)  // zero tile for the one-sided pairs
+      reinterpret_cast<uint4 *>(sm + Z)[e] = make_uint4(0, 0, 0, 0);
+  }
+  // write the column pair X (rows t' 0..63) and Y (rows 64..127): hi @C1/C2, lo @C0/C3
+  auto put_pair = [&](int which) {
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float x[16], y[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = c0 + i;
+        const float x2 = X2g[t * D + j];
+        const float dp = ((m >> t) & 1ull) ? -x2 : 0.f;
+        switch (which) {
+          case 0: x[i] = -Gam[t] * x2; y[i] = Gam[t] * gamv[t] * dov(t); break;  // [dKR;dQR]
+          case 1: x[i] = Gprev[t] * dp - Gam[t] * Xg[t * D + j]; y[i] = Gam[t] * dov(t); break;
+          case 2: x[i] = gamv[t] * dov(t); y[i] = x2; break;                  // [dOa ; dX2]
+          default: x[i] = dov(t); y[i] = dp; break;                           // [dO ; dP]
+        }
+      }
+      put16s(sm + C1, sm + C0, j, c0, x);
+      put16s(sm + C2, sm + C3, j, c0, y);
+    }
+  };
+  // D (+)= [X;Y] (hi + lo, MN-major, atoms a_lbo apart) * (B hi + lo)^T, 3 products
+  auto pair_x_state = [&](uint32_t d, uint32_t bh_, uint32_t bl_, bool acc_first) {
+    mma_tile_mnmn(d, sb + C1, C2 - C1, sb + bh_, 16384, 8, i128, acc_first);
+    mma_tile_mnmn(d, sb + C1, C2 - C1, sb + bl_, 16384, 8, i128, true);
+    mma_tile_mnmn(d, sb + C0, C3 - C0, sb + bh_, 16384, 8, i128, true);
+  };
+  // ---- phases 2, 3: [dKR ; dQR] R0^T and [dKS ; dQS] S0^T (lanes t' = dK | dQ rows)
+  if (ok) {
+    put_pair(0);
+    ok = phase_run(K, tid, [&] { pair_x_state(tm + T_DKQ, R0H, R0L, false); return true; });
+  }
+  if (ok) {
+    put_pair(1);
+    ok = phase_run(K, tid, [&] { pair_x_state(tm + T_DKQ, S0H, S0L, true); return true; });
+  }
+  // ---- phase 4: diag(wR) E2 dR^T + diag(wS) E dS^T (dK rows only: Y = zero tile)
+  if (ok) {
+    put_state(gR, GRH, GRL);
+    put_state(gS, GSH, GSL);
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float x[16], y[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        x[i] = wR[c0 + i] * E2g[(c0 + i) * D + j];
+        y[i] = wS[c0 + i] * Eg[(c0 + i) * D + j];
+      }
+      put16s(sm + C1, sm + C0, j, c0, x);   // wE2: hi @C1, lo @C0
+      put16s(sm + C2, sm + C3, j, c0, y);   // wE:  hi @C2, lo @C3
+    }
+    ok = phase_run(K, tid, [&] {
+      const uint32_t d = tm + T_DKQ;
+      mma_tile_mnmn(d, sb + C1, Z - C1, sb + GRH, 16384, 8, i128, true);
+      mma_tile_mnmn(d, sb + C1, Z - C1, sb + GRL, 16384, 8, i128, true);
+      mma_tile_mnmn(d, sb + C0, Z - C0, sb + GRH, 16384, 8, i128, true);
+      mma_tile_mnmn(d, sb + C2, Z - C2, sb + GSH, 16384, 8, i128, true);
+      mma_tile_mnmn(d, sb + C2, Z - C2, sb + GSL, 16384, 8, i128, true);
+      mma_tile_mnmn(d, sb + C3, Z - C3, sb + GSH, 16384, 8, i128, true);
+      return true;
+    });
+  }
+  // ---- phases 5, 6: C x C gradients (lanes t' = stacked rows, columns s)
+  //   [dOa ; dX2] E2^T -> G1,  [dX ; 0] E^T -> G3,  [dO ; dP] E^T -> G2
+  auto put_e = [&](const float *src, uint32_t hi, uint32_t lo) {
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float v[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = src[(c0 + i) * D + j];
+      put16s(sm + hi, sm + lo, j, c0, v);
+    }
+  };
+  auto pair_x_e = [&](uint32_t d, uint32_t ah, uint32_t al, uint32_t ah_lbo, uint32_t al_lbo,
+                      uint32_t eh, uint32_t el) {
+    mma_tile_mnmn(d, sb + ah, ah_lbo, sb + eh, 16384, 8, i64, false);
+    mma_tile_mnmn(d, sb + ah, ah_lbo, sb + el, 16384, 8, i64, true);
+    mma_tile_mnmn(d, sb + al, al_lbo, sb + eh, 16384, 8, i64, true);
+  };
+  if (ok) {
+    put_pair(2);
+    put_e(E2g, EH, EL);
+    put_e(Xg, XH, XL);
+    ok = phase_run(K, tid, [&] {
+      pair_x_e(tm + T_G1, C1, C0, C2 - C1, C3 - C0, EH, EL);
+      return true;
+    });
+  }
+  if (ok) {
+    put_e(Eg, EH, EL);
+    ok = phase_run(K, tid, [&] {
+      pair_x_e(tm + T_G3, XH, XL, Z - XH, Z - XL, EH, EL);  // [dX ; 0] E^T
+      return true;
+    });
+  }
+  if (ok) {
+    put_pair(3);
+    ok = phase_run(K, tid, [&] {
+      pair_x_e(tm + T_G2, C1, C0, C2 - C1, C3 - C0, EH, EL);
+      return true;
+    });
+  }
+  if (ok) {
+    const int tp = tid;  // lanes t' < 64: dK row t', else dQ row t' - 64
+    float *dst = acc + (tp < 64 ? A8::DKo + tp * D : A8::DQo + (tp - 64) * D);
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float vv[16];
+      tmem_ld16(tm + lane + T_DKQ + c0, vv);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) dst[c0 + i] = vv[i];
+    }
+    const int t = tp & 63;
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float g1[16], g2[16], g3[16];
+      tmem_ld16(tm + lane + T_G1 + c0, g1);
+      tmem_ld16(tm + lane + T_G2 + c0, g2);
+      tmem_ld16(tm + lane + T_G3 + c0, g3);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int s = c0 + i;
+        if (tp < 64) {
+          acc[A8::DM2 + t * 64 + s] = g1[i];   // dOa E2^T
+          acc[A8::DMQ + t * 64 + s] = g2[i];   // dO E^T
+          acc[A8::DAB + t * 64 + s] = -g3[i];  // -dX E^T
+        } else {
+          acc[A8::DAG + t * 64 + s] = -g1[i];  // -dX2 E2^T
+          acc[A8::DAP + t * 64 + s] = g2[i];   // dP E^T
+        }
+      }
+    }
+  } else if (tid == 0 && p.err) {
+    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+}  // namespace
+
+size_t bwd_tc_extra_bytes(int B, int H, int NC) {
+  const size_t nct = (size_t)B * H * NC;
+  return nct * (4 * 64 * D * sizeof(float) + 2 * (size_t)D * D * sizeof(float) +
+                D * sizeof(unsigned long long) + 16384);
+}
+
+cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
+                          const float *Sc, const float *Rc, void *dv, float *dS0, float *dR0,
+                          float *acc, char *extra, cudaStream_t s) {
+  TcBwdParams P;
+  P.f = f;
+  P.dO = dO;
+  P.dST = dST;
+  P.dRT = dRT;
+  P.Sc = Sc;
+  P.Rc = Rc;
+  P.dv = dv;
+  P.dS0 = dS0;
+  P.dR0 = dR0;
+  P.acc = acc;
+  const size_t nct = (size_t)f.B * f.H * f.NC;
+  float *x = reinterpret_cast<float *>(extra);
+  P.Ebuf = x;
+  P.E2buf = x + nct * 64 * D;
+  P.dX2buf = x + 2 * nct * 64 * D;
+  P.dXbuf = x + 3 * nct * 64 * D;
+  P.dSc = x + 4 * nct * 64 * D;
+  P.dRc = P.dSc + nct * D * D;
+  P.mask = reinterpret_cast<unsigned long long *>(P.dRc + nct * D * D);
+  P.gM2 = reinterpret_cast<uint8_t *>(P.mask + nct * D);
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(bwd_recompute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)rc::SMEM)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(bwd_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)ch::SMEM)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(bwd_post_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)po::SMEM)) != cudaSuccess)
+    return e;
+  RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NT, ch::SMEM, s>>>(P));
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<(unsigned)nct, NT, po::SMEM, s>>>(P));
+  return cudaGetLastError();
+}
+
+}  // namespace rdn

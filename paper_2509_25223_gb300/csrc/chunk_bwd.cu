@@ -698,7 +698,7 @@ constexpr size_t finish_smem() {
 }
 
 template <int DK, bool RDNV, typename InT>
-cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
+cudaError_t launch_t(const BwdParams &p, cudaStream_t s, bool do_scan = true) {
   auto scan = bwd_scan_kernel<DK, RDNV, InT>;
   auto fin = bwd_finish_kernel<DK, RDNV, InT>;
   cudaError_t e;
@@ -708,8 +708,10 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
   if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)finish_smem<DK>())) != cudaSuccess)
     return e;
-  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (do_scan) {
+    RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   RDN_LAUNCH("bwd_finish", s, fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
@@ -717,8 +719,11 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct BwdLayout {
-  size_t prep, acc, states, o, total;
+  size_t prep, acc, states, o, tc, total;
 };
+
+// bf16 inputs with d = 128 take the tensor-core backward
+bool use_tc_bwd(const rdn_fwd_args &f) { return f.dtype == RDN_BF16 && f.Dk == 128; }
 
 BwdLayout layout(const rdn_bwd_args &a) {
   const rdn_fwd_args &f = a.fwd;
@@ -731,7 +736,8 @@ BwdLayout layout(const rdn_bwd_args &a) {
   l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
-  l.total = l.prep + l.acc + 2 * l.states + l.o + 256;  // + device status word
+  l.tc = use_tc_bwd(f) ? align256(bwd_tc_extra_bytes(f.B, f.H, (f.T + C - 1) / C)) : 0;
+  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + 256;  // + device status word
   return l;
 }
 
@@ -763,24 +769,24 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   p.f.ST = p.f.RT = nullptr;
   const bool bf = f.dtype == RDN_BF16;
   const bool rdnv = true;
+  const bool tc = use_tc_bwd(f);
   cudaError_t e;
   if (f.S_chunks == nullptr) {  // recompute the chunk-start states
     p.f.S_chunks = (float *)(ws + l.prep + l.acc);
     p.f.R_chunks = (float *)(ws + l.prep + l.acc + l.states);
     p.f.o = ws + l.prep + l.acc + 2 * l.states;
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
-    // the tensor-core scan reads the records as shared-memory images; the
-    // reverse scan below reads them in fp32: rewrite them
-    if (e == cudaSuccess && bf && f.Dk == 128)
-      e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, false, s);
+    // the tensor-core forward leaves its records as shared-memory images,
+    // which the tensor-core backward reads too; the SIMT backward needs fp32
+    if (e == cudaSuccess && bf && f.Dk == 128 && !tc)
+      e = launch_prep(p.f, f.Dk, rdnv, bf, false, s);
   } else {
-    e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, false, s);
+    e = launch_prep(p.f, f.Dk, rdnv, bf, tc, s);
   }
   if (e != cudaSuccess) return e;
   p.Sc = p.f.S_chunks;
   p.Rc = p.f.R_chunks;
   p.acc = (float *)(ws + l.prep);
-  if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
   p.dO = a.dO;
   p.dST = a.dST;
   p.dRT = a.dRT;
@@ -792,6 +798,13 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   p.dgamma = a.dgamma;
   p.dS0 = a.dS0;
   p.dR0 = a.dR0;
+  if (tc) {  // every accumulator word is written by the recompute / post kernels
+    e = launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dv, a.dS0, a.dR0, p.acc,
+                      ws + l.prep + l.acc + 2 * l.states + l.o, s);
+    if (e != cudaSuccess) return e;
+    return launch_t<128, true, __nv_bfloat16>(p, s, false);
+  }
+  if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
   if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
   return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
 }

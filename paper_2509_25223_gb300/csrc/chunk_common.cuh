@@ -85,6 +85,16 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
 bool fwd_tc_supported(const rdn_fwd_args &a);
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s);
 
+// Prep kernel alone; img selects the shared-memory-image record format read
+// by the tensor-core kernels (else the fp32 format of the SIMT kernels).
+cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool img, cudaStream_t s);
+
+// Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
+size_t bwd_tc_extra_bytes(int B, int H, int NC);
+cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
+                          const float *Sc, const float *Rc, void *dv, float *dS0, float *dR0,
+                          float *acc, char *extra, cudaStream_t s);
+
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).
 cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, bool do_prep,

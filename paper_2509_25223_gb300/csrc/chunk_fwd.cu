@@ -488,6 +488,19 @@ cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, b
   return launch_fwd_tc(p, rdnv, s);
 }
 
+cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool img, cudaStream_t s) {
+  if (DK == 128) {
+    if (rdnv) return bf16 ? launch_t<128, true, __nv_bfloat16>(p, s, true, false, img)
+                          : launch_t<128, true, float>(p, s, true, false, img);
+    return bf16 ? launch_t<128, false, __nv_bfloat16>(p, s, true, false, img)
+                : launch_t<128, false, float>(p, s, true, false, img);
+  }
+  if (rdnv) return bf16 ? launch_t<64, true, __nv_bfloat16>(p, s, true, false, img)
+                        : launch_t<64, true, float>(p, s, true, false, img);
+  return bf16 ? launch_t<64, false, __nv_bfloat16>(p, s, true, false, img)
+              : launch_t<64, false, float>(p, s, true, false, img);
+}
+
 FwdPlan plan_fwd(const rdn_fwd_args &a, int /*variant*/) {
   FwdPlan pl;
   pl.NC = (a.T + C - 1) / C;

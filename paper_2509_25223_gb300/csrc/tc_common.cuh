@@ -158,6 +158,21 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
   return d;
 }
 
+// Descriptor of an MN-major operand in the 128-byte swizzled layout: rows are
+// the K index (128 bytes = 64 elements of the M or N index each), 8-row
+// groups 1024 bytes apart, and consecutive 64-element M/N atoms `lbo` bytes
+// apart.  Advancing K by 16 rows is +2048 bytes on the start address.
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;  // stride between M/N atoms
+  d |= (uint64_t)(1024 >> 4) << 32;              // stride between 8-row K groups
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+constexpr uint32_t kAMajorMN = 1u << 15, kBMajorMN = 1u << 16;
+
 // D[tmem] (+)= A * B^T for one K = 16 slice, issued by one thread.
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                          uint32_t idesc, uint32_t accumulate) {
@@ -177,6 +192,90 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
       : "memory");
+}
+
+// D (+)= A * B^T over K = 16 * ksteps, A K-major (64-column blocks a_blk
+// apart), B MN-major (K rows, N in 64-wide atoms b_lbo apart).
+__device__ __forceinline__ void mma_tile_kmn(uint32_t d_tmem, uint32_t a_base, uint32_t a_blk,
+                                             uint32_t b_base, uint32_t b_lbo, int ksteps,
+                                             uint32_t idesc, bool accumulate_first) {
+  for (int kk = 0; kk < ksteps; ++kk) {
+    const uint32_t a = a_base + (uint32_t)(kk >> 2) * a_blk + (uint32_t)(kk & 3) * 32u;
+    mma_bf16(d_tmem, sdesc_sw128(a), sdesc_sw128_mn(b_base + (uint32_t)kk * 2048u, b_lbo),
+             idesc | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
+  }
+}
+
+// D (+)= A * B^T over K = 16 * ksteps with both operands MN-major (K rows;
+// M / N atoms a_lbo / b_lbo apart).
+__device__ __forceinline__ void mma_tile_mnmn(uint32_t d_tmem, uint32_t a_base, uint32_t a_lbo,
+                                              uint32_t b_base, uint32_t b_lbo, int ksteps,
+                                              uint32_t idesc, bool accumulate_first) {
+  for (int kk = 0; kk < ksteps; ++kk)
+    mma_bf16(d_tmem, sdesc_sw128_mn(a_base + (uint32_t)kk * 2048u, a_lbo),
+             sdesc_sw128_mn(b_base + (uint32_t)kk * 2048u, b_lbo),
+             idesc | kAMajorMN | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
+}
+
+// Sum a per-thread vector v[64] over the 32 lanes of a warp by halving
+// exchanges: afterwards lane l holds the warp sums for tokens
+// t = tbase(l) and tbase(l) + 1 in out[0..1], with
+// tbase(l) = 32 b4 + 16 b3 + 8 b2 + 4 b1 + 2 b0 for the bits b of l.
+__device__ __forceinline__ void warp_transpose_reduce64(const float (&v)[64], float (&out)[2]) {
+  const int lane = threadIdx.x & 31;
+  float a[32];
+  {
+    const bool hi = lane & 16;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float send = hi ? v[k] : v[32 + k];
+      const float keep = hi ? v[32 + k] : v[k];
+      a[k] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+    }
+  }
+  float b[16];
+  {
+    const bool hi = lane & 8;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float send = hi ? a[k] : a[16 + k];
+      const float keep = hi ? a[16 + k] : a[k];
+      b[k] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+    }
+  }
+  float c[8];
+  {
+    const bool hi = lane & 4;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float send = hi ? b[k] : b[8 + k];
+      const float keep = hi ? b[8 + k] : b[k];
+      c[k] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+    }
+  }
+  float d[4];
+  {
+    const bool hi = lane & 2;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float send = hi ? c[k] : c[4 + k];
+      const float keep = hi ? c[4 + k] : c[k];
+      d[k] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+    }
+  }
+  {
+    const bool hi = lane & 1;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const float send = hi ? d[k] : d[2 + k];
+      const float keep = hi ? d[2 + k] : d[k];
+      out[k] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+    }
+  }
+}
+__device__ __forceinline__ int transpose_reduce_tbase(int lane) {
+  return ((lane >> 4) & 1) * 32 + ((lane >> 3) & 1) * 16 + ((lane >> 2) & 1) * 8 +
+         ((lane >> 1) & 1) * 4 + (lane & 1) * 2;
 }
 
 // Byte offset of element (r, c), c in [0, 64), in a K-major 128B-swizzled tile
