@@ -45,12 +45,14 @@ C = 64
 #     the products over the value dimension        12 d^2 + 5 C d
 #     (dK, dQ state terms; C x C gradients)
 #     the backward of the prep                     2 (2 C d + (4/3) C^2)
-#   recomputation of forward pieces is not algorithmic work (counted 0).
+#   (the tensor-core bwd_post does the last two; the SIMT path splits them
+#   into bwd_scan and bwd_finish).  Recomputation of forward pieces is not
+#   algorithmic work (counted 0).
 def flops_per_token_head(d=128, c=C):
     scan = 12 * d * d + 5 * c * d
     prep = 2 * c * d + (4.0 / 3.0) * c * c
     return dict(fwd=scan + prep, fwd_scan=scan, fwd_prep=prep, bwd_scan=2 * scan,
-                bwd_chain=scan, bwd_post=scan, bwd_finish=2 * prep, recompute=0.0,
+                bwd_chain=scan, bwd_post=scan + 2 * prep, bwd_finish=2 * prep, recompute=0.0,
                 step=3 * (scan + prep))
 
 

@@ -20,8 +20,9 @@
 //     No forward quantity other than the clip mask enters this chain.
 //  3. bwd_post (parallel, one CTA per chunk): every product that reduces over
 //     the value dimension -- the state terms of dK, dQ, the five C x C
-//     gradients, the per-row gate terms -- written to the per-chunk record
-//     that bwd_finish (chunk_bwd.cu) turns into dq, dk, dg, dbeta, dgamma.
+//     gradients, the per-row gate terms -- and then the gradients of the chunk
+//     matrices' entries turned into dq, dk, dg, dbeta, dgamma (the work that
+//     bwd_finish of chunk_bwd.cu does on the SIMT path).
 //
 // Orientation: thread j of 128 owns value column j = TMEM lane j for every
 // column quantity (X, E, dO, dX2, ...), which is kept as a bf16 hi + lo tile
@@ -66,6 +67,8 @@ struct TcBwdParams {
   float *dSc, *dRc;      // [B*H*NC][128][128] (i, j): gradients w.r.t. chunk-end states
   unsigned long long *mask;  // [B*H*NC][128]: bit t = clip inactive (|x| <= c)
   uint8_t *gM2;              // [B*H*NC][16 KB]: image of diag(gamma) M2 (hi | lo)
+  void *dq, *dk;             // outputs of bwd_post
+  float *dg, *dbeta, *dgamma;
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
@@ -96,17 +99,6 @@ __device__ __forceinline__ void put16s(uint8_t *hi, uint8_t *lo, int r, int c0,
   put16(hi, 0, r, c0, a);
   put16(lo, 0, r, c0, b);
 }
-// a whole 64-value row, split
-__device__ __forceinline__ void put64s(uint8_t *hi, uint8_t *lo, int r, const float (&v)[64]) {
-#pragma unroll
-  for (int c0 = 0; c0 < 64; c0 += 16) {
-    float w[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
-    put16s(hi, lo, r, c0, w);
-  }
-}
-
 // K-major A (single block, K = 64) times MN-major B, split both: 3 products
 __device__ __forceinline__ void mma_s3_kmn(uint32_t d, uint32_t a_hi, uint32_t a_lo,
                                            uint32_t b_hi, uint32_t b_lo, uint32_t b_lbo,
@@ -219,7 +211,6 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   }
   float *vec = reinterpret_cast<float *>(sm + VEC);
   float *Gam = vec, *Gprev = vec + 64, *alpha = vec + 128, *gamv = vec + 320;
-  float *red = reinterpret_cast<float *>(sm + RED);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, j = tid;
   const size_t chunk = blockIdx.x;
@@ -778,29 +769,58 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
 }
 
 // ======================================================================== 3
-// bwd_post: the products over the value dimension, one chunk per CTA.
-// States and carried gradients enter as bf16 hi + lo, like the column tiles.
+// bwd_post: everything that reduces over the value dimension, followed by the
+// chunk-matrix part of the gradients (the work bwd_finish of chunk_bwd.cu does
+// for the SIMT path), one chunk per CTA of 256 threads.  Thread (j, hf) owns
+// value column j = TMEM lane j and half hf of the chunk's tokens (or of the
+// key rows of a state).
+//
+// dK and dQ are accumulated transposed in TMEM (lane = key dimension d,
+// column t for dK_t, 64 + t for dQ_t):
+//   P2  R0 [dKR ; dQR]^T        P3  S0 [dKS ; dQS]^T
+//   P4  dR (diag(wR) E2)^T + dS (diag(wS) E)^T        (dK columns only)
+//   P7  K^T [dKK + dKK^T ; dQK]^T, and Q^T dQK kept apart (scaled at read-out)
+// The C x C gradients (P5) and the Gram matrices K K^T, Q K^T go through
+// shared memory for the element-wise pass over (t, i) of Eqs. for T, M2, Mq, Ap.
+// Q enters the tensor-core products unscaled; the scale is applied to the
+// fp32 results.
 namespace po {
-// phase 1: chunk-start states (hi | lo, rows j) and K, Q
-constexpr uint32_t S0H = 0, S0L = 32768, R0H = 65536, R0L = 98304, KQ = 131072;
-// later: pair buffer (4 x 16 KB) over the K, Q region, zero tile after it
-constexpr uint32_t C0 = 131072, C1 = 147456, C2 = 163840, C3 = 180224, Z = 196608;
-// phase 4: carried gradients (hi | lo) over the state region
-constexpr uint32_t GRH = 0, GRL = 32768, GSH = 65536, GSL = 98304;
-// phases 5-6: E / E2 (hi, lo) and dX (hi, lo) over the state region
-constexpr uint32_t EH = 0, EL = 16384, XH = 32768, XL = 49152;
-constexpr uint32_t RED = 212992;                 // 4 x 64 + 64 floats
-constexpr uint32_t VEC = RED + 5 * 64 * 4;       // Gam Gprev wS wR gamma (5 x 64)
-constexpr uint32_t CTL = VEC + 5 * 64 * 4;
+constexpr int NTP = 256;
+constexpr uint32_t SA = 0, SB = 65536;  // state images: hi 2 x 16 KB | lo 2 x 16 KB, rows j
+constexpr uint32_t XH = 131072, XL = 147456, YH = 163840, YL = 180224;  // [j][t] atoms
+constexpr uint32_t KQ = 196608;         // K rows 0..63, Q rows 64..127, 2 x 16 KB
+constexpr uint32_t VEC = 229376;        // Gam Gprev wS wR gamma dGam dGprev (7 x 64), dGamC
+constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // 8 warps x 32 floats
+constexpr uint32_t CTL = RED + 8 * 32 * 4;
 constexpr uint32_t SLOT = CTL + 32;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
-constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256;
-// after phase 1 the read-out columns hold the C x C gradients
-constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128;
+// element-wise pass: fp32 C x C tiles (row stride 65) over the state images
+constexpr int LDC = 65, TILE = 64 * LDC;
+constexpr int F_DM2 = 0, F_DMQ = TILE, F_DAB = 2 * TILE, F_KK = 3 * TILE, F_DAG = 4 * TILE,
+              F_DAP = 5 * TILE, F_QK = 6 * TILE, F_VEC = 7 * TILE;
+static_assert((F_VEC + 9 * 64 + 5 * 4 * 64) * 4 <= (int)XH, "finish scratch");
+// TMEM columns
+constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
+constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
 }  // namespace po
 
-__global__ void __launch_bounds__(NT, 1) bwd_post_kernel(TcBwdParams P) {
+// Sums over the 128 value columns: thread (j, hf) holds v[t - 32 hf] for the
+// tokens t of its half; out[t] for t in [0, 64).
+__device__ __forceinline__ void cta_row_sum256(const float (&v)[32], float *red, float *out,
+                                               int tid) {
+  const float o = warp_transpose_reduce32(v);
+  red[tid] = o;  // red[warp * 32 + lane]
+  __syncthreads();
+  if (tid < 64) {
+    const int hh = tid >> 5, l = tid & 31;
+    out[tid] = red[(4 * hh) * 32 + l] + red[(4 * hh + 1) * 32 + l] + red[(4 * hh + 2) * 32 + l] +
+               red[(4 * hh + 3) * 32 + l];
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   using namespace po;
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sb = smem_u32(sm);
@@ -811,18 +831,21 @@ __global__ void __launch_bounds__(NT, 1) bwd_post_kernel(TcBwdParams P) {
   }
   float *vec = reinterpret_cast<float *>(sm + VEC);
   float *Gam = vec, *Gprev = vec + 64, *wS = vec + 128, *wR = vec + 192, *gamv = vec + 256;
+  float *dGamS = vec + 320, *dGprevS = vec + 384, *dGamC = vec + 448;
   float *red = reinterpret_cast<float *>(sm + RED);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
-  const int tid = threadIdx.x, warp = tid >> 5, j = tid;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int j = tid & 127, hf = tid >> 7, tb = 32 * hf;
   const size_t chunk = blockIdx.x;
   const int NC = p.NC, T = p.T, H = p.H;
   const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
   const int b = bh / H, h = bh % H;
   const int t0 = c * 64, n = min(64, T - t0);
+  const float scale = p.scale;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   const float *recf = p.ws + chunk * kRecFloats;
-  float *acc = P.acc + chunk * A8::FLOATS;
+  const float *acc = P.acc + chunk * A8::FLOATS;
 
   Ctl K;
   ctl_init(K, sm + CTL, tid);
@@ -834,240 +857,442 @@ __global__ void __launch_bounds__(NT, 1) bwd_post_kernel(TcBwdParams P) {
     wR[tid] = recf[OFF_VEC + V_WR + tid];
     gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
   }
-  // a [i][j] fp32 matrix -> rows j of a (hi, lo) pair of two-block tiles
-  auto put_state = [&](const float *src, uint32_t hi, uint32_t lo) {
-    for (int c0 = 0; c0 < D; c0 += 16) {
-      float v[16], a[16], bb[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        v[i] = src[(size_t)(c0 + i) * D + j];
-        a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
-        bb[i] = v[i] - a[i];
-      }
-      put16(sm + hi, 16384, j, c0, a);
-      put16(sm + lo, 16384, j, c0, bb);
-    }
-  };
-  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
-  const float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
-  put_state(S0, S0H, S0L);
-  put_state(R0, R0H, R0L);
-  float gdot = 0.f;  // <dR, R0> + <dS, S0> over this column
-  for (int i = 0; i < D; ++i) {
-    const size_t o = (size_t)i * D + j;
-    gdot += gS[o] * S0[o] + gR[o] * R0[o];
-  }
-  for (int e = tid; e < 64 * 16; e += NT) {  // unscaled K, Q
+  for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16)
     const int t = e >> 4, chn = e & 15;
     uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
     if (t < n) {
       const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
       kv = *reinterpret_cast<const uint4 *>(k + off);
       qv = *reinterpret_cast<const uint4 *>(q + off);
-      if (p.scale != 1.f) {
-        __nv_bfloat16 *qb = reinterpret_cast<__nv_bfloat16 *>(&qv);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) qb[i] = __float2bfloat16_rn(p.scale * __bfloat162float(qb[i]));
-      }
     }
     const int blk = chn >> 3, cc = (chn & 7) * 8;
     *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
     *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
   }
-  fence_before_sync();
-  __syncthreads();
-  fence_after_sync();
-  const uint32_t tm = *slot;
-  const uint32_t lane = (uint32_t)(warp * 32) << 16;
   const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
   const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
-  const unsigned long long m = P.mask[chunk * D + j];
-  auto dov = [&](int t) -> float {
-    return t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
+  const float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
+  const unsigned long long m = P.mask[chunk * D + j] >> tb;
+  // this thread's tokens of dX2, dX, dO
+  float x2v[32], xv[32], dov[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int t = tb + i;
+    x2v[i] = X2g[t * D + j];
+    xv[i] = Xg[t * D + j];
+    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  }
+  // a [i][j] fp32 state -> rows j of its (hi | lo) image, key rows of half hf
+  auto put_state = [&](const float *src, uint32_t img) {
+    float v[64];
+#pragma unroll
+    for (int i = 0; i < 64; ++i) v[i] = src[(size_t)(64 * hf + i) * D + j];
+#pragma unroll
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float w[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
+      put16s(sm + img + hf * 16384, sm + img + 32768 + hf * 16384, j, c0, w);
+    }
   };
+  // <src, g> over this thread's 64 entries
+  auto dot_state = [&](const float *src, const float *g) {
+    float s = 0.f;
+#pragma unroll 16
+    for (int i = 0; i < 64; ++i) {
+      const size_t o = (size_t)(64 * hf + i) * D + j;
+      s += src[o] * g[o];
+    }
+    return s;
+  };
+  // this thread's 32 tokens of a [j][t] atom pair (hi, lo)
+  auto put_tok = [&](const float (&x)[32], uint32_t hi, uint32_t lo) {
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float w[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) w[i] = x[c0 + i];
+      put16s(sm + hi, sm + lo, j, tb + c0, w);
+    }
+  };
+  auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
+  const uint32_t tm_lane = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
 
-  // ---- phase 1: read-outs [KS|QS], [KR|QR] with split states
+  put_state(S0, SA);
+  put_state(R0, SB);
+  float gdot = dot_state(S0, gS) + dot_state(R0, gR);
+  // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
   bool ok = phase_run(K, tid, [&] {
-    mma_tile(tm + T_KS, sb + S0H, 16384, sb + KQ, 16384, 8, i128, false);
-    mma_tile(tm + T_KS, sb + S0L, 16384, sb + KQ, 16384, 8, i128, true);
-    mma_tile(tm + T_KR, sb + R0H, 16384, sb + KQ, 16384, 8, i128, false);
-    mma_tile(tm + T_KR, sb + R0L, 16384, sb + KQ, 16384, 8, i128, true);
+    const uint32_t t_ = *slot;
+    mma_tile(t_ + T_KS, sb + SA, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile(t_ + T_KS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i128, true);
+    mma_tile(t_ + T_KR, sb + SB, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
     return true;
   });
-  if (ok) {  // per-row gate terms dGam, dGprev and <dR,R0> + <dS,S0>
-    for (int w = 0; w < 2; ++w) {
-      float rv[64];
-      if (w == 0) {
+  const uint32_t tm = *slot;
+  if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
+    float rv[32];
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) {
-          float qs[16], qr[16];
-          tmem_ld16(tm + lane + T_KS + 64 + c0, qs);
-          tmem_ld16(tm + lane + T_KR + 64 + c0, qr);
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float qs[16], qr[16];
+      tmem_ld16(tm + tm_lane + T_KS + 64 + tb + c0, qs);
+      tmem_ld16(tm + tm_lane + T_KR + 64 + tb + c0, qr);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) rv[c0 + i] = dov(c0 + i) * (qs[i] + gamv[c0 + i] * qr[i]);
-        }
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) {
-          float ks[16], kr[16];
-          tmem_ld16(tm + lane + T_KS + c0, ks);
-          tmem_ld16(tm + lane + T_KR + c0, kr);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int t = c0 + i;
-            rv[t] -= X2g[t * D + j] * kr[i] + Xg[t * D + j] * ks[i];
-          }
-        }
-      } else {
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) {
-          float ks[16];
-          tmem_ld16(tm + lane + T_KS + c0, ks);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int t = c0 + i;
-            rv[t] = ((m >> t) & 1ull) ? -X2g[t * D + j] * ks[i] : 0.f;
-          }
-        }
-      }
-      cta_row_sum(rv, red, red + 256, tid);
-      if (tid < 64) acc[A8::VEC + (w == 0 ? A8::V_DGAM : A8::V_DGPREV) + tid] = red[256 + tid];
+      for (int i = 0; i < 16; ++i)
+        rv[c0 + i] = scale * dov[c0 + i] * (qs[i] + gamv[tb + c0 + i] * qr[i]);
     }
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float ks[16], kr[16];
+      tmem_ld16(tm + tm_lane + T_KS + tb + c0, ks);
+      tmem_ld16(tm + tm_lane + T_KR + tb + c0, kr);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) rv[c0 + i] -= x2v[c0 + i] * kr[i] + xv[c0 + i] * ks[i];
+    }
+    cta_row_sum256(rv, red, dGamS, tid);
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float ks[16];
+      tmem_ld16(tm + tm_lane + T_KS + tb + c0, ks);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) rv[c0 + i] = dp_of(c0 + i) * ks[i];
+    }
+    cta_row_sum256(rv, red, dGprevS, tid);
 #pragma unroll
     for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
-    if ((tid & 31) == 0) red[warp] = gdot;
+    if (lane == 0) red[warp] = gdot;
     __syncthreads();
-    if (tid == 0) acc[A8::VEC + A8::V_DGAMC] = red[0] + red[1] + red[2] + red[3];
-    for (int e = tid; e < 16384 / 16; e += NT)  // zero tile for the one-sided pairs
-      reinterpret_cast<uint4 *>(sm + Z)[e] = make_uint4(0, 0, 0, 0);
+    if (tid == 0) {
+      float s = 0.f;
+      for (int w = 0; w < NTP / 32; ++w) s += red[w];
+      *dGamC = s;
+    }
+    // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
+    float x[32], y[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int t = tb + i;
+      x[i] = -Gam[t] * x2v[i];
+      y[i] = Gam[t] * gamv[t] * dov[i];
+    }
+    put_tok(x, XH, XL);
+    put_tok(y, YH, YL);
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XH, 32768, 8, i128, false);
+      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 32768, 8, i128, true);
+      return true;
+    });
   }
-  // write the column pair X (rows t' 0..63) and Y (rows 64..127): hi @C1/C2, lo @C0/C3
-  auto put_pair = [&](int which) {
+  if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO
+    float x[32], y[32];
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float x[16], y[16];
+    for (int i = 0; i < 32; ++i) {
+      const int t = tb + i;
+      x[i] = Gprev[t] * dp_of(i) - Gam[t] * xv[i];
+      y[i] = Gam[t] * dov[i];
+    }
+    put_tok(x, XH, XL);
+    put_tok(y, YH, YL);
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + XH, 32768, 8, i128, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SA + 32768, 16384, sb + XH, 32768, 8, i128, true);
+      return true;
+    });
+  }
+  if (ok) {  // ---- P4: dK += dR (diag(wR) E2)^T + dS (diag(wS) E)^T
+    put_state(gR, SB);
+    put_state(gS, SA);
+    float x[32], y[32];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = c0 + i;
-        const float x2 = X2g[t * D + j];
-        const float dp = ((m >> t) & 1ull) ? -x2 : 0.f;
-        switch (which) {
-          case 0: x[i] = -Gam[t] * x2; y[i] = Gam[t] * gamv[t] * dov(t); break;  // [dKR;dQR]
-          case 1: x[i] = Gprev[t] * dp - Gam[t] * Xg[t * D + j]; y[i] = Gam[t] * dov(t); break;
-          case 2: x[i] = gamv[t] * dov(t); y[i] = x2; break;                  // [dOa ; dX2]
-          default: x[i] = dov(t); y[i] = dp; break;                           // [dO ; dP]
+    for (int i = 0; i < 32; ++i) {
+      const int t = tb + i;
+      x[i] = wR[t] * E2g[t * D + j];
+      y[i] = wS[t] * Eg[t * D + j];
+    }
+    put_tok(x, XH, XL);
+    put_tok(y, YH, YL);
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XH, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_DKQ, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
+      return true;
+    });
+  }
+  // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
+  //   G1 = [dOa ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
+  //   and the Gram matrices [K ; Q] K^T
+  // images: E2 at SA (hi | lo), E at SA + 32 KB, dX at SB; the pair at X / Y
+  if (ok) {
+    float x[32], y[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int t = tb + i;
+      x[i] = E2g[t * D + j];
+      y[i] = Eg[t * D + j];
+    }
+    put_tok(x, SA, SA + 16384);
+    put_tok(y, SA + 32768, SA + 49152);
+    put_tok(xv, SB, SB + 16384);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] = gamv[tb + i] * dov[i];
+    put_tok(x, XH, XL);
+    put_tok(x2v, YH, YL);
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnmn(tm + T_G1, sb + XH, 32768, sb + SA, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G1, sb + XH, 32768, sb + SA + 16384, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G1, sb + XL, 32768, sb + SA, 16384, 8, i64, true);
+      // the second M atom of [dX ; -] is any valid tile: lanes 64..127 are unused
+      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + SA + 32768, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + SA + 49152, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G3, sb + SB + 16384, 32768, sb + SA + 32768, 16384, 8, i64, true);
+      mma_tile(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
+      return true;
+    });
+  }
+  if (ok) {
+    float y[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) y[i] = dp_of(i);
+    put_tok(dov, XH, XL);
+    put_tok(y, YH, YL);
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnmn(tm + T_G2, sb + XH, 32768, sb + SA + 32768, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G2, sb + XH, 32768, sb + SA + 49152, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G2, sb + XL, 32768, sb + SA + 32768, 16384, 8, i64, true);
+      return true;
+    });
+  }
+  // ---- element-wise pass over (t, i): the gradients of the chunk matrices'
+  // entries turned into gradients of K K^T, Q K^T and of the gates
+  float *F = reinterpret_cast<float *>(sm);
+  float *cum = F + F_VEC, *cprev = cum + 64, *bet = cum + 128, *gam = cum + 192, *gg = cum + 256,
+        *dcum = cum + 320, *dcprev = cum + 384, *dbet = cum + 448, *dgam = cum + 512;
+  float *prt = cum + 576;  // [5][4][64] partial sums
+  if (ok) {
+    {
+      const int r = j & 63;
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float g1[16], g2[16], g3[16], gr[16];
+        tmem_ld16(tm + tm_lane + T_G1 + tb + c0, g1);
+        tmem_ld16(tm + tm_lane + T_G2 + tb + c0, g2);
+        tmem_ld16(tm + tm_lane + T_G3 + tb + c0, g3);
+        tmem_ld16(tm + tm_lane + T_GR + tb + c0, gr);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int e = r * LDC + tb + c0 + i;
+          if (j < 64) {
+            F[F_DM2 + e] = g1[i];
+            F[F_DMQ + e] = g2[i];
+            F[F_DAB + e] = -g3[i];
+            F[F_KK + e] = gr[i];
+          } else {
+            F[F_DAG + e] = -g1[i];
+            F[F_DAP + e] = g2[i];
+            F[F_QK + e] = scale * gr[i];
+          }
         }
       }
-      put16s(sm + C1, sm + C0, j, c0, x);
-      put16s(sm + C2, sm + C3, j, c0, y);
     }
-  };
-  // D (+)= [X;Y] (hi + lo, MN-major, atoms a_lbo apart) * (B hi + lo)^T, 3 products
-  auto pair_x_state = [&](uint32_t d, uint32_t bh_, uint32_t bl_, bool acc_first) {
-    mma_tile_mnmn(d, sb + C1, C2 - C1, sb + bh_, 16384, 8, i128, acc_first);
-    mma_tile_mnmn(d, sb + C1, C2 - C1, sb + bl_, 16384, 8, i128, true);
-    mma_tile_mnmn(d, sb + C0, C3 - C0, sb + bh_, 16384, 8, i128, true);
-  };
-  // ---- phases 2, 3: [dKR ; dQR] R0^T and [dKS ; dQS] S0^T (lanes t' = dK | dQ rows)
-  if (ok) {
-    put_pair(0);
-    ok = phase_run(K, tid, [&] { pair_x_state(tm + T_DKQ, R0H, R0L, false); return true; });
-  }
-  if (ok) {
-    put_pair(1);
-    ok = phase_run(K, tid, [&] { pair_x_state(tm + T_DKQ, S0H, S0L, true); return true; });
-  }
-  // ---- phase 4: diag(wR) E2 dR^T + diag(wS) E dS^T (dK rows only: Y = zero tile)
-  if (ok) {
-    put_state(gR, GRH, GRL);
-    put_state(gS, GSH, GSL);
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float x[16], y[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        x[i] = wR[c0 + i] * E2g[(c0 + i) * D + j];
-        y[i] = wS[c0 + i] * Eg[(c0 + i) * D + j];
+    if (tid < 64) {
+      const int t = tid;
+      float gv = 0.f, bv = 0.f;
+      if (t < n) {
+        const size_t off = (size_t)(b * T + t0 + t) * H + h;
+        gv = p.g[off];
+        bv = p.beta[off];
       }
-      put16s(sm + C1, sm + C0, j, c0, x);   // wE2: hi @C1, lo @C0
-      put16s(sm + C2, sm + C3, j, c0, y);   // wE:  hi @C2, lo @C3
+      gg[t] = gv;
+      bet[t] = bv;
+      gam[t] = gamv[t];
     }
-    ok = phase_run(K, tid, [&] {
-      const uint32_t d = tm + T_DKQ;
-      mma_tile_mnmn(d, sb + C1, Z - C1, sb + GRH, 16384, 8, i128, true);
-      mma_tile_mnmn(d, sb + C1, Z - C1, sb + GRL, 16384, 8, i128, true);
-      mma_tile_mnmn(d, sb + C0, Z - C0, sb + GRH, 16384, 8, i128, true);
-      mma_tile_mnmn(d, sb + C2, Z - C2, sb + GSH, 16384, 8, i128, true);
-      mma_tile_mnmn(d, sb + C2, Z - C2, sb + GSL, 16384, 8, i128, true);
-      mma_tile_mnmn(d, sb + C3, Z - C3, sb + GSH, 16384, 8, i128, true);
-      return true;
-    });
-  }
-  // ---- phases 5, 6: C x C gradients (lanes t' = stacked rows, columns s)
-  //   [dOa ; dX2] E2^T -> G1,  [dX ; 0] E^T -> G3,  [dO ; dP] E^T -> G2
-  auto put_e = [&](const float *src, uint32_t hi, uint32_t lo) {
+    __syncthreads();
+    if (warp == 0) {  // in-chunk cumulative log-decay
+      float a = gg[lane], a2 = gg[32 + lane];
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float v[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) v[i] = src[(c0 + i) * D + j];
-      put16s(sm + hi, sm + lo, j, c0, v);
+      for (int off = 1; off < 32; off <<= 1) {
+        const float ua = __shfl_up_sync(0xffffffffu, a, off);
+        const float ub = __shfl_up_sync(0xffffffffu, a2, off);
+        if (lane >= off) {
+          a += ua;
+          a2 += ub;
+        }
+      }
+      a2 += __shfl_sync(0xffffffffu, a, 31);
+      cum[lane] = a;
+      cum[32 + lane] = a2;
+      cprev[lane] = a - gg[lane];
+      cprev[32 + lane] = a2 - gg[32 + lane];
     }
-  };
-  auto pair_x_e = [&](uint32_t d, uint32_t ah, uint32_t al, uint32_t ah_lbo, uint32_t al_lbo,
-                      uint32_t eh, uint32_t el) {
-    mma_tile_mnmn(d, sb + ah, ah_lbo, sb + eh, 16384, 8, i64, false);
-    mma_tile_mnmn(d, sb + ah, ah_lbo, sb + el, 16384, 8, i64, true);
-    mma_tile_mnmn(d, sb + al, al_lbo, sb + eh, 16384, 8, i64, true);
-  };
-  if (ok) {
-    put_pair(2);
-    put_e(E2g, EH, EL);
-    put_e(Xg, XH, XL);
-    ok = phase_run(K, tid, [&] {
-      pair_x_e(tm + T_G1, C1, C0, C2 - C1, C3 - C0, EH, EL);
-      return true;
-    });
-  }
-  if (ok) {
-    put_e(Eg, EH, EL);
-    ok = phase_run(K, tid, [&] {
-      pair_x_e(tm + T_G3, XH, XL, Z - XH, Z - XL, EH, EL);  // [dX ; 0] E^T
-      return true;
-    });
-  }
-  if (ok) {
-    put_pair(3);
-    ok = phase_run(K, tid, [&] {
-      pair_x_e(tm + T_G2, C1, C0, C2 - C1, C3 - C0, EH, EL);
-      return true;
-    });
-  }
-  if (ok) {
-    const int tp = tid;  // lanes t' < 64: dK row t', else dQ row t' - 64
-    float *dst = acc + (tp < 64 ? A8::DKo + tp * D : A8::DQo + (tp - 64) * D);
-    for (int c0 = 0; c0 < D; c0 += 16) {
-      float vv[16];
-      tmem_ld16(tm + lane + T_DKQ + c0, vv);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) dst[c0 + i] = vv[i];
+    __syncthreads();
+    {  // row pass: thread (t, quarter) over i in [16 q, 16 q + 16)
+      const int t = tid & 63, q4 = tid >> 6;
+      const float ct = cum[t], cpt = cprev[t];
+      float rowc = 0.f, rowp = 0.f;
+#pragma unroll 4
+      for (int ii = 0; ii < 16; ++ii) {
+        const int i = 16 * q4 + ii, e = t * LDC + i;
+        float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
+        if (i <= t) {
+          const float dec = __expf(ct - cum[i]);
+          const float kk = F[F_KK + e], qk = F[F_QK + e], bi = bet[i], gi = gam[i];
+          {  // M2: inclusive, gamma, Q K^T
+            const float dm = F[F_DM2 + e];
+            const float G = dm * dec * gi * qk;
+            rowc += G;
+            cg += G;
+            cm += dm * dec * qk;
+            dqk += dm * dec * gi;
+          }
+          if (i < t) {
+            const float decp = __expf(cpt - cum[i]);
+            {  // Ap: strict, beta, K K^T, previous-token decay
+              const float dm = F[F_DAP + e];
+              const float G = dm * decp * bi * kk;
+              rowp += G;
+              cg += G;
+              cb += dm * decp * kk;
+              dkk += dm * decp * bi;
+            }
+            {  // Mq: strict, beta, Q K^T
+              const float dm = F[F_DMQ + e];
+              const float G = dm * dec * bi * qk;
+              rowc += G;
+              cg += G;
+              cb += dm * dec * qk;
+              dqk += dm * dec * bi;
+            }
+            {  // A_beta, A_gamma: strict, K K^T
+              const float da = F[F_DAB + e], dg2 = F[F_DAG + e];
+              const float Gb = da * dec * bi * kk, Gg = dg2 * dec * gi * kk;
+              rowc += Gb + Gg;
+              cg += Gb + Gg;
+              cb += da * dec * kk;
+              cm += dg2 * dec * kk;
+              dkk += da * dec * bi + dg2 * dec * gi;
+            }
+          }
+        }
+        F[F_KK + e] = dkk;
+        F[F_QK + e] = dqk;
+        F[F_DM2 + e] = cg;
+        F[F_DMQ + e] = cb;
+        F[F_DAB + e] = cm;
+      }
+      prt[0 * 256 + q4 * 64 + t] = rowc;
+      prt[1 * 256 + q4 * 64 + t] = rowp;
     }
-    const int t = tp & 63;
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float g1[16], g2[16], g3[16];
-      tmem_ld16(tm + lane + T_G1 + c0, g1);
-      tmem_ld16(tm + lane + T_G2 + c0, g2);
-      tmem_ld16(tm + lane + T_G3 + c0, g3);
+    __syncthreads();
+    {  // column pass: thread (i, quarter) over t in [16 q, 16 q + 16)
+      const int i = tid & 63, q4 = tid >> 6;
+      float sg = 0.f, sbv = 0.f, smv = 0.f;
+#pragma unroll 4
+      for (int tt = 0; tt < 16; ++tt) {
+        const int e = (16 * q4 + tt) * LDC + i;
+        sg += F[F_DM2 + e];
+        sbv += F[F_DMQ + e];
+        smv += F[F_DAB + e];
+      }
+      prt[2 * 256 + q4 * 64 + i] = sg;
+      prt[3 * 256 + q4 * 64 + i] = sbv;
+      prt[4 * 256 + q4 * 64 + i] = smv;
+    }
+    __syncthreads();
+    if (tid < 64) {
+      const int i = tid;
+      float s5[5];
+#pragma unroll
+      for (int w = 0; w < 5; ++w)
+        s5[w] = prt[w * 256 + i] + prt[w * 256 + 64 + i] + prt[w * 256 + 128 + i] +
+                prt[w * 256 + 192 + i];
+      const float cC = cum[63];
+      const float eC = __expf(cC - cum[i]);
+      const float dwS = acc[A8::VEC + A8::V_DWS + i], dwR = acc[A8::VEC + A8::V_DWR + i];
+      dbet[i] = s5[3] + dwS * eC;
+      dgam[i] = s5[4] + acc[A8::VEC + A8::V_DGAM_OUT + i] + dwR * eC;
+      dcum[i] = s5[0] - s5[2] - (dwS * bet[i] + dwR * gam[i]) * eC + dGamS[i] * __expf(cum[i]);
+      dcprev[i] = s5[1] + dGprevS[i] * __expf(cprev[i]);
+    }
+    __syncthreads();
+    if (warp == 0) {  // chunk-end terms land on cum_C = cum[63] (padding has g = 0)
+      const float cC = cum[63];
+      float s = 0.f;
+      for (int t = lane; t < 64; t += 32)
+        s += (acc[A8::VEC + A8::V_DWS + t] * bet[t] + acc[A8::VEC + A8::V_DWR + t] * gam[t]) *
+             __expf(cC - cum[t]);
+#pragma unroll
+      for (int off = 16; off; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (lane == 0) dcum[63] += s + *dGamC * __expf(cC);
+      __syncwarp();
+      // dg_s = sum_{t >= s} dcum_t + sum_{t > s} dcprev_t (reverse scans)
+      float a = dcum[63 - lane], a2 = dcum[31 - lane];
+      float pa = dcprev[63 - lane], pb = dcprev[31 - lane];
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const float ua = __shfl_up_sync(0xffffffffu, a, off), ub = __shfl_up_sync(0xffffffffu, a2, off);
+        const float upa = __shfl_up_sync(0xffffffffu, pa, off), upb = __shfl_up_sync(0xffffffffu, pb, off);
+        if (lane >= off) {
+          a += ua;
+          a2 += ub;
+          pa += upa;
+          pb += upb;
+        }
+      }
+      a2 += __shfl_sync(0xffffffffu, a, 31);
+      pb += __shfl_sync(0xffffffffu, pa, 31);
+      gg[63 - lane] = a + (pa - dcprev[63 - lane]);
+      gg[31 - lane] = a2 + (pb - dcprev[31 - lane]);
+    }
+    {  // B operand [dKK + dKK^T ; dQK] (rows t, columns i), hi | lo
+      const int t = tid & 63, q4 = tid >> 6;
+      float v[16], w[16];
+#pragma unroll
+      for (int ii = 0; ii < 16; ++ii) {
+        const int i = 16 * q4 + ii;
+        v[ii] = i == t ? 2.f * F[F_KK + t * LDC + t] : F[F_KK + t * LDC + i] + F[F_KK + i * LDC + t];
+        w[ii] = F[F_QK + t * LDC + i];
+      }
+      put16s(sm + XH, sm + XL, t, 16 * q4, v);
+      put16s(sm + XH, sm + XL, 64 + t, 16 * q4, w);
+    }
+    // ---- P7: dK, dQ += K^T [dKK + dKK^T ; dQK]^T ; D2 = Q^T dQK
+    ok = phase_run(K, tid, [&] {
+      mma_tile_mnk(tm + T_DKQ, sb + KQ, 16384, sb + XH, 4, i128, true);
+      mma_tile_mnk(tm + T_DKQ, sb + KQ, 16384, sb + XL, 4, i128, true);
+      mma_tile_mnmn(tm + T_D2, sb + KQ + 8192, 16384, sb + XH + 8192, 16384, 4, i64, false);
+      mma_tile_mnmn(tm + T_D2, sb + KQ + 8192, 16384, sb + XL + 8192, 16384, 4, i64, true);
+      return true;
+    });
+  }
+  if (ok) {
+    if (tid < n) {
+      const size_t off = (size_t)(b * T + t0 + tid) * H + h;
+      P.dg[off] = gg[tid];
+      P.dbeta[off] = dbet[tid];
+      P.dgamma[off] = dgam[tid];
+    }
+    __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float a[16], d2[16], qv[16];
+      tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);
+      tmem_ld16(tm + tm_lane + T_D2 + tb + c0, d2);
+      tmem_ld16(tm + tm_lane + T_DKQ + 64 + tb + c0, qv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const int s = c0 + i;
-        if (tp < 64) {
-          acc[A8::DM2 + t * 64 + s] = g1[i];   // dOa E2^T
-          acc[A8::DMQ + t * 64 + s] = g2[i];   // dO E^T
-          acc[A8::DAB + t * 64 + s] = -g3[i];  // -dX E^T
-        } else {
-          acc[A8::DAG + t * 64 + s] = -g1[i];  // -dX2 E2^T
-          acc[A8::DAP + t * 64 + s] = g2[i];   // dP E^T
+        const int t = tb + c0 + i;
+        if (t < n) {
+          const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + j;
+          dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
+          dq[off] = __float2bfloat16_rn(scale * qv[i]);
         }
       }
     }
@@ -1088,9 +1313,15 @@ size_t bwd_tc_extra_bytes(int B, int H, int NC) {
 }
 
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
-                          const float *Sc, const float *Rc, void *dv, float *dS0, float *dR0,
-                          float *acc, char *extra, cudaStream_t s) {
+                          const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
+                          float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
+                          char *extra, cudaStream_t s) {
   TcBwdParams P;
+  P.dq = dq;
+  P.dk = dk;
+  P.dg = dg;
+  P.dbeta = dbeta;
+  P.dgamma = dgamma;
   P.f = f;
   P.dO = dO;
   P.dST = dST;
@@ -1125,7 +1356,7 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NT, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<(unsigned)nct, NT, po::SMEM, s>>>(P));
+  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<(unsigned)nct, po::NTP, po::SMEM, s>>>(P));
   return cudaGetLastError();
 }
 

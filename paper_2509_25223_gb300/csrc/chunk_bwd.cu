@@ -698,7 +698,7 @@ constexpr size_t finish_smem() {
 }
 
 template <int DK, bool RDNV, typename InT>
-cudaError_t launch_t(const BwdParams &p, cudaStream_t s, bool do_scan = true) {
+cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
   auto scan = bwd_scan_kernel<DK, RDNV, InT>;
   auto fin = bwd_finish_kernel<DK, RDNV, InT>;
   cudaError_t e;
@@ -708,10 +708,8 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s, bool do_scan = true) {
   if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)finish_smem<DK>())) != cudaSuccess)
     return e;
-  if (do_scan) {
-    RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
+  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   RDN_LAUNCH("bwd_finish", s, fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
@@ -798,12 +796,10 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   p.dgamma = a.dgamma;
   p.dS0 = a.dS0;
   p.dR0 = a.dR0;
-  if (tc) {  // every accumulator word is written by the recompute / post kernels
-    e = launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dv, a.dS0, a.dR0, p.acc,
-                      ws + l.prep + l.acc + 2 * l.states + l.o, s);
-    if (e != cudaSuccess) return e;
-    return launch_t<128, true, __nv_bfloat16>(p, s, false);
-  }
+  if (tc)  // the accumulator words it reads are written by its own kernels
+    return launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dq, a.dk, a.dv, a.dg, a.dbeta,
+                         a.dgamma, a.dS0, a.dR0, p.acc, ws + l.prep + l.acc + 2 * l.states + l.o,
+                         s);
   if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
   if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
   return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);

@@ -206,6 +206,17 @@ __device__ __forceinline__ void mma_tile_kmn(uint32_t d_tmem, uint32_t a_base, u
   }
 }
 
+// D (+)= A * B^T over K = 16 * ksteps (<= 4), A MN-major (K rows, M atoms
+// a_lbo apart), B K-major in one 64-column block.
+__device__ __forceinline__ void mma_tile_mnk(uint32_t d_tmem, uint32_t a_base, uint32_t a_lbo,
+                                             uint32_t b_base, int ksteps, uint32_t idesc,
+                                             bool accumulate_first) {
+  for (int kk = 0; kk < ksteps; ++kk)
+    mma_bf16(d_tmem, sdesc_sw128_mn(a_base + (uint32_t)kk * 2048u, a_lbo),
+             sdesc_sw128(b_base + (uint32_t)kk * 32u), idesc | kAMajorMN,
+             (kk > 0 || accumulate_first) ? 1u : 0u);
+}
+
 // D (+)= A * B^T over K = 16 * ksteps with both operands MN-major (K rows;
 // M / N atoms a_lbo / b_lbo apart).
 __device__ __forceinline__ void mma_tile_mnmn(uint32_t d_tmem, uint32_t a_base, uint32_t a_lbo,
@@ -273,6 +284,35 @@ __device__ __forceinline__ void warp_transpose_reduce64(const float (&v)[64], fl
     }
   }
 }
+// Sum a per-thread vector v[32] over the 32 lanes of a warp by halving
+// exchanges: afterwards lane l holds the warp sum of v[l].
+__device__ __forceinline__ float warp_transpose_reduce32(const float (&v)[32]) {
+  const int lane = threadIdx.x & 31;
+  float a[16], b[8], c[4], d[2];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const bool hi = lane & 16;
+    a[k] = (hi ? v[16 + k] : v[k]) + __shfl_xor_sync(0xffffffffu, hi ? v[k] : v[16 + k], 16);
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const bool hi = lane & 8;
+    b[k] = (hi ? a[8 + k] : a[k]) + __shfl_xor_sync(0xffffffffu, hi ? a[k] : a[8 + k], 8);
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const bool hi = lane & 4;
+    c[k] = (hi ? b[4 + k] : b[k]) + __shfl_xor_sync(0xffffffffu, hi ? b[k] : b[4 + k], 4);
+  }
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const bool hi = lane & 2;
+    d[k] = (hi ? c[2 + k] : c[k]) + __shfl_xor_sync(0xffffffffu, hi ? c[k] : c[2 + k], 2);
+  }
+  const bool hi = lane & 1;
+  return (hi ? d[1] : d[0]) + __shfl_xor_sync(0xffffffffu, hi ? d[0] : d[1], 1);
+}
+
 __device__ __forceinline__ int transpose_reduce_tbase(int lane) {
   return ((lane >> 4) & 1) * 32 + ((lane >> 3) & 1) * 16 + ((lane >> 2) & 1) * 8 +
          ((lane >> 1) & 1) * 4 + (lane & 1) * 2;
