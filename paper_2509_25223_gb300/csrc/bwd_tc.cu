@@ -557,11 +557,6 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
         const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
         kv = *reinterpret_cast<const uint4 *>(k + off);
         qv = *reinterpret_cast<const uint4 *>(q + off);
-        if (p.scale != 1.f) {
-          __nv_bfloat16 *qb = reinterpret_cast<__nv_bfloat16 *>(&qv);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) qb[i] = __float2bfloat16_rn(p.scale * __bfloat162float(qb[i]));
-        }
       }
       const int blk = chn >> 3, cc = (chn & 7) * 8;
       *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
@@ -613,7 +608,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
         const int t = c0 + i;
         m2[i] = m2[i] + wR[t] * kdr[i];
         mq[i] = mq[i] + wS[t] * kds[i];
-        dqr[i] = Gam[t] * gamv[t] * dO[t];
+        dqr[i] = p.scale * Gam[t] * gamv[t] * dO[t];  // Q below is unscaled
       }
       tmem_st16(tm + lane + T_R4 + c0, mq);
       put16s(sm + S0H, sm + S0L, j, c0, m2);
@@ -696,7 +691,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           a[i] += e[i];
-          dqs[i] = Gam[c0 + i] * dO[c0 + i];
+          dqs[i] = p.scale * Gam[c0 + i] * dO[c0 + i];
         }
         put16s(sm + S0H, sm + S0L, j, c0, a);
         put16s(sm + S1H, sm + S1L, j, c0, dqs);

@@ -36,10 +36,10 @@ def _condition(x, clip, dtype, heads=None):
         x["v"][b, :, h] = torch.from_numpy(v2[0, :, 0]).to(x["v"].dtype).to(x["v"].device)
 
 
-def _ref(x, clip, dST=None, dRT=None, heads=None):
+def _ref(x, clip, dST=None, dRT=None, heads=None, scale=1.0):
     if heads is None:
         return oracle.rdn_bwd(*(as64(x[n]) for n in NAMES), clip, as64(x["S0"]), as64(x["R0"]),
-                              as64(x["dO"]), as64(dST), as64(dRT))
+                              as64(x["dO"]), as64(dST), as64(dRT), scale=scale)
     outs = []
     for b, h in heads:
         sl = lambda t: None if t is None else as64(t[b:b + 1, :, h:h + 1])
@@ -81,6 +81,23 @@ def test_bwd_zero_upstream_state_grads_and_no_init_state():
     ref = _ref(x, 1.0)
     for name in GRADS:
         assert_close(d[name], ref[name], "bf16", name)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("D", [64, 128])
+def test_bwd_query_scale(dtype, D):
+    """The query scale (e.g. 1/sqrt(d_k)): dq is w.r.t. the unscaled query."""
+    scale = D ** -0.5
+    x = make_inputs(2, 130, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    gen = torch.Generator(device="cpu").manual_seed(11)
+    dST = torch.randn(x["S0"].shape, generator=gen).cuda()
+    dRT = torch.randn(x["R0"].shape, generator=gen).cuda()
+    _condition(x, 1.0, dtype)
+    d = _gpu(x, 1.0, dST, dRT, scale=scale)
+    ref = _ref(x, 1.0, dST, dRT, scale=scale)
+    for name in GRADS:
+        assert_close(d[name], ref[name], dtype, name)
 
 
 @pytest.mark.parametrize("clip", [0.3, float("inf")])

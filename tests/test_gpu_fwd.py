@@ -24,11 +24,12 @@ def _gpu(variant, x, clip=1.0, **kw):
     return out
 
 
-def _ref(variant, x, clip=1.0, heads=None):
+def _ref(variant, x, clip=1.0, heads=None, scale=1.0):
     """Oracle on all heads, or on the listed (b, h) pairs (returns stacked)."""
     v = oracle.RDN if variant == "rdn" else oracle.RLA
     if heads is None:
-        return oracle.fwd(v, *(as64(x[n]) for n in NAMES), clip, as64(x["S0"]), as64(x["R0"]))
+        return oracle.fwd(v, *(as64(x[n]) for n in NAMES), clip, as64(x["S0"]), as64(x["R0"]),
+                          scale=scale)
     outs = []
     for b, h in heads:
         sl = {n: as64(x[n][b:b + 1, :, h:h + 1]) for n in NAMES}
@@ -58,6 +59,20 @@ def test_fwd_small(variant, dtype, D, T):
     x = make_inputs(2, T, 3, D, dtype=dtype, nonzero_state=True, device="cuda", state_std=0.1)
     o, ST, RT = _gpu(variant, x)
     oref, Sref, Rref = _ref(variant, x)
+    assert_close(o, oref, dtype, "o")
+    assert_close(ST, Sref, dtype, "ST")
+    assert_close(RT, Rref, dtype, "RT")
+
+
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("D", [64, 128])
+def test_fwd_query_scale(variant, dtype, D):
+    """The query scale (e.g. 1/sqrt(d_k)) enters every read-out."""
+    scale = D ** -0.5
+    x = make_inputs(2, 130, 2, D, dtype=dtype, nonzero_state=True, device="cuda", state_std=0.1)
+    o, ST, RT = _gpu(variant, x, scale=scale)
+    oref, Sref, Rref = _ref(variant, x, scale=scale)
     assert_close(o, oref, dtype, "o")
     assert_close(ST, Sref, dtype, "ST")
     assert_close(RT, Rref, dtype, "RT")
