@@ -348,7 +348,7 @@ def run_ours(args):
         _, _, _, Sc, Rc = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
                                       return_chunk_states=True, out=o, workspace=wsf)
         rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc,
-                    R_chunks=Rc, workspace=wsb, out=grads)
+                    R_chunks=Rc, workspace=wsb, out=grads, fwd_workspace=wsf)
 
     for _ in range(args.warmup):
         step(x)

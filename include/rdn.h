@@ -108,6 +108,14 @@ typedef struct {
  *                     chunk-start states (as written by rdn_fwd on the same
  *                     inputs); if NULL the backward recomputes them into its
  *                     workspace.
+ *   fwd.workspace     NULL, or (only together with S_chunks/R_chunks) the
+ *                     workspace of the rdn_fwd call that wrote them, READ
+ *                     as that forward left it: its per-chunk matrices
+ *                     (Section 3.5's T, A and M blocks) are reused instead of
+ *                     recomputed.  fwd.workspace_bytes must be at least
+ *                     rdn_fwd_workspace_size(&fwd); the same q, k, g, beta,
+ *                     gamma, scale and clip as in that call are the caller's
+ *                     responsibility (not checked).  It is only read.
  *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
  *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
  *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype.

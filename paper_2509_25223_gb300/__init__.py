@@ -135,9 +135,14 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
-            scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None):
+            scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
+            fwd_workspace=None):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
-    dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32)."""
+    dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
+
+    S_chunks/R_chunks: the forward's chunk-start states (return_chunk_states).
+    fwd_workspace: with them, the workspace that forward call used, whose
+    per-chunk matrices are then reused instead of recomputed."""
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -152,6 +157,9 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     a = BwdArgs()
     _fill_fwd(a.fwd, q, k, v, g, beta, gamma, clip, S0, R0, None, None, None, S_chunks,
               R_chunks, scale)
+    if fwd_workspace is not None:
+        a.fwd.workspace = _ptr(fwd_workspace)
+        a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"])

@@ -323,6 +323,17 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
   OPTIONAL_PTR(f->R_chunks);
   if ((f->S_chunks == nullptr) != (f->R_chunks == nullptr))
     return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  if (f->workspace && f->T > 0) {  // the forward's records, reused
+    if (!f->S_chunks)
+      return fail(RDN_ERR_INVALID_ARG,
+                  "%s: fwd.workspace is reused only together with fwd.S_chunks/R_chunks", fn);
+    if (!aligned16(f->workspace))
+      return fail(RDN_ERR_WORKSPACE, "%s: fwd.workspace is not 16-byte aligned", fn);
+    const size_t fneed = rdn::plan_fwd(*f, 1).total_bytes;
+    if (f->workspace_bytes < fneed)
+      return fail(RDN_ERR_WORKSPACE, "%s: fwd.workspace of %zu bytes required (got %zu)", fn, fneed,
+                  f->workspace_bytes);
+  }
   OPTIONAL_PTR(a->dST);
   OPTIONAL_PTR(a->dRT);
   OPTIONAL_PTR(a->dS0);

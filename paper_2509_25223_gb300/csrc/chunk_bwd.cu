@@ -723,12 +723,19 @@ struct BwdLayout {
 // bf16 inputs with d = 128 take the tensor-core backward
 bool use_tc_bwd(const rdn_fwd_args &f) { return f.dtype == RDN_BF16 && f.Dk == 128; }
 
+// The forward's per-chunk records are valid input when the caller passes the
+// forward's workspace with its chunk-start states.  Both passes pick the same
+// record format: shared-memory images for bf16, d = 128 (tensor-core forward
+// and backward), fp32 otherwise.
+bool reuse_fwd_records(const rdn_fwd_args &f) { return f.workspace && f.S_chunks; }
+
 BwdLayout layout(const rdn_bwd_args &a) {
   const rdn_fwd_args &f = a.fwd;
   const size_t nct = (size_t)f.B * f.H * ((f.T + C - 1) / C);
   const size_t accf = f.Dk == 128 ? Acc<128>::FLOATS : Acc<64>::FLOATS;
   BwdLayout l;
-  l.prep = align256(sizeof(float) * nct * kRecFloats);
+  // the forward's records are read from its workspace when it is passed
+  l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nct * kRecFloats);
   l.acc = align256(sizeof(float) * nct * accf);
   const bool need_states = f.S_chunks == nullptr;
   l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
@@ -762,7 +769,8 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   char *ws = (char *)a.workspace;
   BwdParams p;
   p.f = make_fwd_params(f);
-  p.f.ws = (float *)ws;
+  const bool reuse = reuse_fwd_records(f);
+  p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
   p.f.err = (int *)(ws + l.total - 256);
   p.f.ST = p.f.RT = nullptr;
   const bool bf = f.dtype == RDN_BF16;
@@ -778,7 +786,7 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
     // which the tensor-core backward reads too; the SIMT backward needs fp32
     if (e == cudaSuccess && bf && f.Dk == 128 && !tc)
       e = launch_prep(p.f, f.Dk, rdnv, bf, false, s);
-  } else {
+  } else if (!reuse) {
     e = launch_prep(p.f, f.Dk, rdnv, bf, tc, s);
   }
   if (e != cudaSuccess) return e;

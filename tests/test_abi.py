@@ -114,6 +114,22 @@ def test_bwd_validation():
     assert lib.rdn_bwd(ctypes.byref(b), None) == 1
     b.fwd = _fwd_args(clip=-0.5)
     assert lib.rdn_bwd(ctypes.byref(b), None) == 1
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE)
+    for f in ("dO", "dq", "dk", "dv", "dg", "dbeta", "dgamma"):
+        setattr(b, f, FAKE)
+    # the forward's workspace is reused only with its chunk states
+    b.fwd = _fwd_args(workspace=FAKE, workspace_bytes=1 << 40, **ok)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 1
+    assert "S_chunks" in lib.rdn_last_error().decode()
+    n = ctypes.c_size_t(0)
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args()), ctypes.byref(n)) == 0
+    b.fwd = _fwd_args(workspace=FAKE, workspace_bytes=n.value - 16, S_chunks=FAKE, R_chunks=FAKE,
+                      **ok)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 5
+    assert "fwd.workspace" in lib.rdn_last_error().decode()
+    b.fwd = _fwd_args(workspace=ctypes.c_void_p(0x10008), workspace_bytes=n.value, S_chunks=FAKE,
+                      R_chunks=FAKE, **ok)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 5
 
 
 def test_binding_rejects_cpu_tensors():
