@@ -336,7 +336,8 @@ def run_ours(args):
     B, T, H, D = w.B, w.T, w.H, w.D
     NC = (T + C - 1) // C
     o = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
-    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", B, T, H, D), dtype=torch.uint8, device=dev)
+    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", B, T, H, D, save_for_bwd=True),
+                      dtype=torch.uint8, device=dev)
     wsb = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D), dtype=torch.uint8, device=dev)
     grads = dict(dq=torch.empty_like(x["q"]), dk=torch.empty_like(x["k"]),
                  dv=torch.empty_like(x["v"]),
@@ -346,9 +347,10 @@ def run_ours(args):
 
     def step(inp):
         _, _, _, Sc, Rc = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
-                                      return_chunk_states=True, out=o, workspace=wsf)
+                                      return_chunk_states=True, out=o, workspace=wsf,
+                                      save_for_bwd=True)
         rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc,
-                    R_chunks=Rc, workspace=wsb, out=grads, fwd_workspace=wsf)
+                    R_chunks=Rc, workspace=wsb, out=grads, fwd_workspace=wsf, fwd_saved=True)
 
     for _ in range(args.warmup):
         step(x)

@@ -66,6 +66,16 @@ typedef enum {
 
 typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
 
+/* rdn_fwd_args.flags.  RDN_FLAG_SAVE_FOR_BWD (rdn_fwd only; needs S_chunks
+ * and R_chunks): the forward also keeps, in its workspace after the per-chunk
+ * matrices, the delta errors E and E2 of both passes and the clip mask of
+ * every chunk (Section 3.5's intermediates of the residual pass); ask
+ * rdn_fwd_workspace_size with the flag set.  rdn_bwd given that workspace
+ * (fwd.workspace) and the same flag in fwd.flags reads them instead of
+ * recomputing them.  On the bf16, Dk = 128 path this removes a pass of the
+ * backward; on the others the flag only reserves the space. */
+#define RDN_FLAG_SAVE_FOR_BWD 0x1u
+
 /* Arguments of rla_fwd / rdn_fwd.
  *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
  *                     S0/R0 to ST/RT).
@@ -84,7 +94,7 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *                     stored).  rdn_bwd can consume them instead of
  *                     recomputing.
  *   scale             multiplies q (the paper uses 1).
- *   flags             must be 0 (paper variants are reserved bits).
+ *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd (above).
  *   workspace         device scratch of *_fwd_workspace_size() bytes.     */
 typedef struct {
   int B, T, H, Dk, Dv;
@@ -116,6 +126,8 @@ typedef struct {
  *                     rdn_fwd_workspace_size(&fwd); the same q, k, g, beta,
  *                     gamma, scale and clip as in that call are the caller's
  *                     responsibility (not checked).  It is only read.
+ *   fwd.flags         RDN_FLAG_SAVE_FOR_BWD if that forward ran with it
+ *                     (then fwd.workspace is required), else 0.
  *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
  *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
  *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype.

@@ -73,7 +73,7 @@ def _alloc_ws(nbytes, device):
     return torch.empty(nbytes, dtype=torch.uint8, device=device)
 
 
-def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale):
+def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale, flags=0):
     B, T, H, Dk = q.shape
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, Dk, v.shape[-1]
     a.dtype = _dtype_code(q)
@@ -85,11 +85,12 @@ def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale
     a.ST, a.RT = _ptr(ST), _ptr(RT)
     a.S_chunks, a.R_chunks = _ptr(Sc), _ptr(Rc)
     a.scale = float(scale)
-    a.flags = 0
+    a.flags = flags
 
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
-         return_final_state=True, return_chunk_states=False, out=None, workspace=None):
+         return_final_state=True, return_chunk_states=False, out=None, workspace=None,
+         save_for_bwd=False):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -104,7 +105,8 @@ def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
         Sc = torch.empty(B, H, NC, Dk, Dv, dtype=torch.float32, device=dev)
         Rc = torch.empty_like(Sc)
     a = FwdArgs()
-    _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale)
+    _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale,
+              _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0)
     nbytes = ctypes.c_size_t(0)
     _check(name + "_workspace_size",
            getattr(lib, name + "_workspace_size")(ctypes.byref(a), ctypes.byref(nbytes)))
@@ -130,19 +132,22 @@ def rla_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw):
     """RDN forward (Section 3.4, right).  Returns (o, ST, RT) and, with
     return_chunk_states=True, also the chunk-start states (Sc, Rc) that
-    rdn_bwd can reuse."""
+    rdn_bwd can reuse.  With save_for_bwd=True (needs return_chunk_states and
+    a caller workspace sized with the same flag) the workspace also keeps the
+    intermediates rdn_bwd(fwd_workspace=..., fwd_saved=True) reads."""
     return _fwd("rdn_fwd", q, k, v, g, beta, gamma, clip, S0, R0, scale, **kw)
 
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None):
+            fwd_workspace=None, fwd_saved=False):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
     S_chunks/R_chunks: the forward's chunk-start states (return_chunk_states).
     fwd_workspace: with them, the workspace that forward call used, whose
-    per-chunk matrices are then reused instead of recomputed."""
+    per-chunk matrices are then reused instead of recomputed.
+    fwd_saved: that forward ran with save_for_bwd=True."""
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -160,6 +165,8 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     if fwd_workspace is not None:
         a.fwd.workspace = _ptr(fwd_workspace)
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
+    if fwd_saved:
+        a.fwd.flags = _abi.RDN_FLAG_SAVE_FOR_BWD
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"])
@@ -229,13 +236,14 @@ class LaunchTimer:
         return {k: (c, t, t / c) for k, (c, t) in out.items()}
 
 
-def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16):
+def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False):
     """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rdn_bwd)."""
     lib = _abi.load()
     a = FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
     a.dtype = _abi.RDN_BF16 if dtype == torch.bfloat16 else _abi.RDN_F32
     a.clip, a.scale = 1.0, 1.0
+    a.flags = _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0
     n = ctypes.c_size_t(0)
     if op == "rdn_bwd":
         b = BwdArgs()

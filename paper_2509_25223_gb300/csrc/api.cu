@@ -98,7 +98,8 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
   if ((long long)a->B * a->T * a->H > (1ll << 31) / 128)
     return fail(RDN_ERR_UNSUPPORTED, "%s: B*T*H = %lld too large", fn,
                 (long long)a->B * a->T * a->H);
-  if (a->flags != 0) return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
+  if (a->flags & ~RDN_FLAG_SAVE_FOR_BWD)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
   if (isnan(a->scale) || isinf(a->scale))
     return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
   return check_clip(fn, a->clip);
@@ -122,6 +123,8 @@ rdn_status_t check_fwd_ptrs(const char *fn, const rdn_fwd_args *a) {
   OPTIONAL_PTR(a->R_chunks);
   if ((a->S_chunks == nullptr) != (a->R_chunks == nullptr))
     return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  if ((a->flags & RDN_FLAG_SAVE_FOR_BWD) && !a->S_chunks && a->T > 0)
+    return fail(RDN_ERR_INVALID_ARG, "%s: RDN_FLAG_SAVE_FOR_BWD needs S_chunks and R_chunks", fn);
   return RDN_OK;
 }
 
@@ -133,6 +136,8 @@ rdn_status_t cuda_status(const char *fn, cudaError_t e) {
 rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a, int variant, cudaStream_t s) {
   rdn_status_t st = check_fwd_shapes(fn, a);
   if (st != RDN_OK) return st;
+  if (variant == 0 && (a->flags & RDN_FLAG_SAVE_FOR_BWD))
+    return fail(RDN_ERR_UNSUPPORTED, "%s: RDN_FLAG_SAVE_FOR_BWD is for rdn_fwd", fn);
   if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
   const rdn::FwdPlan plan = rdn::plan_fwd(*a, variant);
   if (plan.total_bytes > 0) {
@@ -323,6 +328,9 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
   OPTIONAL_PTR(f->R_chunks);
   if ((f->S_chunks == nullptr) != (f->R_chunks == nullptr))
     return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  if ((f->flags & RDN_FLAG_SAVE_FOR_BWD) && !f->workspace && f->T > 0)
+    return fail(RDN_ERR_INVALID_ARG,
+                "%s: RDN_FLAG_SAVE_FOR_BWD in fwd.flags needs the forward's fwd.workspace", fn);
   if (f->workspace && f->T > 0) {  // the forward's records, reused
     if (!f->S_chunks)
       return fail(RDN_ERR_INVALID_ARG,

@@ -6,8 +6,8 @@
 // gradients carried between chunks:
 //
 //  1. bwd_recompute (parallel, one CTA per chunk): from the chunk-start
-//     states rebuild E, E2, the clip mask and the read-out term
-//     dgamma_t += dO_t . Oa_t (the forward's pieces for one chunk).
+//     states rebuild E, E2 and the clip mask (the forward's pieces for one
+//     chunk).  It does not run when the forward saved them.
 //  2. bwd_chain (sequential over chunks, one CTA per (b,h)): the carried
 //     gradients.  With dR, dS the gradients w.r.t. a chunk's end states,
 //        dE2 = M2^T dOa + diag(wR) K dR        dX2 = T_gamma^T dE2
@@ -66,7 +66,6 @@ struct TcBwdParams {
   float *dX2buf, *dXbuf; // [B*H*NC][64][128]
   float *dSc, *dRc;      // [B*H*NC][128][128] (i, j): gradients w.r.t. chunk-end states
   unsigned long long *mask;  // [B*H*NC][128]: bit t = clip inactive (|x| <= c)
-  uint8_t *gM2;              // [B*H*NC][16 KB]: image of diag(gamma) M2 (hi | lo)
   void *dq, *dk;             // outputs of bwd_post
   float *dg, *dbeta, *dgamma;
 };
@@ -218,8 +217,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
   const int b = bh / H, h = bh % H;
   const int t0 = c * 64, n = min(64, T - t0);
-  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
-                      *v = (const __nv_bfloat16 *)p.v, *dO = (const __nv_bfloat16 *)P.dO;
+  const __nv_bfloat16 *k = (const __nv_bfloat16 *)p.k, *v = (const __nv_bfloat16 *)p.v;
   const uint8_t *rec = rec_bytes(p, chunk);
   const float clip = p.clip;
 
@@ -251,28 +249,23 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     }
   }
   __syncthreads();
-  // B1 = [Gprev K ; Gam Q]
+  // B1 = diag(Gprev) K (64 rows)
   for (int e = tid; e < 64 * 16; e += NT) {
     const int t = e >> 4, ch = e & 15;
-    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+    uint4 kv = make_uint4(0, 0, 0, 0);
     if (t < n) {
       const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8;
       kv = *reinterpret_cast<const uint4 *>(k + off);
-      qv = *reinterpret_cast<const uint4 *>(q + off);
     }
     const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
-    const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(&qv);
-    const float gk = Gprev[t], gq = Gam[t] * p.scale;
-    uint4 ks, qs;
-    uint32_t *kw = &ks.x, *qw = &qs.x;
+    const float gk = Gprev[t];
+    uint4 ks;
+    uint32_t *kw = &ks.x;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 4; ++i)
       kw[i] = pack2(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
-      qw[i] = pack2(gq * __bfloat162float(qb[2 * i]), gq * __bfloat162float(qb[2 * i + 1]));
-    }
     const int blk = ch >> 3, cc = (ch & 7) * 8;
     *reinterpret_cast<uint4 *>(sm + B1 + blk * 16384 + sw128(t, cc)) = ks;
-    *reinterpret_cast<uint4 *>(sm + B1 + blk * 16384 + sw128(64 + t, cc)) = qs;
   }
   fence_before_sync();
   __syncthreads();
@@ -283,9 +276,9 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
   };
 
-  bool ok = phase_run(K, tid, [&] {
-    mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 128), false);
-    mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 128), false);
+  bool ok = phase_run(K, tid, [&] {  // Gprev KS, Gprev KR
+    mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
+    mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
     return true;
   });
   float r[64];
@@ -316,15 +309,14 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       for (int i = 0; i < 16; ++i) Eg[(c0 + i) * D + j] = e[i];
       put16s(sm + XE, sm + XE_LO, j, c0, e);
     }
-    ok = phase_run(K, tid, [&] {  // D1 += E [Ap ; Mq]^T -> [P | Ob]
+    ok = phase_run(K, tid, [&] {  // D1 += E Ap^T -> P (the Ap rows of the [Ap ; Mq] image)
       if (!slot_wait(K.barB, K.phB)) return false;
       mma_s3_kk(tm + T_D1, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 16384,
-                 idesc_bf16(128, 128), true);
+                 idesc_bf16(128, 64), true);
       return true;
     });
   }
   if (ok) {
-    if (tid == 0) load_slot(sm + SLOTB, K.barB, rec + IMG_M2, 16384);
     unsigned long long m = 0ull;
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
@@ -358,60 +350,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       tmem_ld16(tm + lane + T_X + c0, e);
 #pragma unroll
       for (int i = 0; i < 16; ++i) E2g[(c0 + i) * D + j] = e[i];
-      put16s(sm + XE, sm + XE_LO, j, c0, e);
     }
-    ok = phase_run(K, tid, [&] {  // Oa = Gam QR + M2 E2 (into D3[:, 64:128])
-      if (!slot_wait(K.barB, K.phB)) return false;
-      mma_s3_kk(tm + T_D3 + 64, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 8192,
-                 idesc_bf16(128, 64), true);
-      return true;
-    });
-  }
-  if (ok) {
-    // image of diag(gamma) M2 (rows s scaled by gamma_s) for the chain's
-    // M2^T (gamma dO) product; same swizzled positions as the M2 image
-    uint8_t *dstimg = P.gM2 + chunk * 16384;
-    for (int e = tid; e < 64 * 8; e += NT) {
-      const int r = e >> 3, c8 = (e & 7) * 8;
-      const uint32_t o = sw128(r, c8);
-      const uint4 hv = *reinterpret_cast<const uint4 *>(sm + SLOTB + o);
-      const uint4 lv = *reinterpret_cast<const uint4 *>(sm + SLOTB + 8192 + o);
-      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
-      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
-      float w[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) w[i] = gamv[r] * (__bfloat162float(hb[i]) + __bfloat162float(lb[i]));
-      uint4 ho, lo;
-      uint32_t *hw = &ho.x, *lw = &lo.x;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float a0 = __bfloat162float(__float2bfloat16_rn(w[2 * i]));
-        const float a1 = __bfloat162float(__float2bfloat16_rn(w[2 * i + 1]));
-        hw[i] = pack2(a0, a1);
-        lw[i] = pack2(w[2 * i] - a0, w[2 * i + 1] - a1);
-      }
-      *reinterpret_cast<uint4 *>(dstimg + o) = ho;
-      *reinterpret_cast<uint4 *>(dstimg + 8192 + o) = lo;
-    }
-  }
-  if (ok) {  // d gamma_t (read-out) = sum_j dO[t,j] Oa[t,j]
-    float prod[64];
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float oa[16];
-      tmem_ld16(tm + lane + T_D3 + 64 + c0, oa);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = c0 + i;
-        const float d =
-            t < n ? __bfloat162float(dO[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
-        prod[t] = d * oa[i];
-      }
-    }
-    float *out = reinterpret_cast<float *>(sm + XE_LO);
-    cta_row_sum(prod, reinterpret_cast<float *>(sm + XE), out, tid);
-    float *acc = P.acc + chunk * A8::FLOATS;
-    if (tid < 64) acc[A8::VEC + A8::V_DGAM_OUT + tid] = out[tid];
   } else if (tid == 0 && p.err) {
     atomicExch(p.err, RDN_ERR_TIMEOUT);
   }
@@ -484,7 +423,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   };
   if (tid == 0) {
     const size_t last = (size_t)bh * NC + NC - 1;
-    load_slot(sm + SLOTA, K.barA, P.gM2 + last * 16384, 16384);
+    load_slot(sm + SLOTA, K.barA, rec_bytes(p, last) + IMG_M2, 16384);
     load_mq(last);
   }
   fence_before_sync();
@@ -708,7 +647,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       return true;
     });
     if (!ok) break;
-    if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, P.gM2 + (chunk - 1) * 16384, 16384);
+    if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
     {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX
       float *gx = P.dXbuf + chunk * 64 * D;
 #pragma unroll
@@ -794,7 +733,7 @@ static_assert(SMEM <= 232448, "shared memory");
 constexpr int LDC = 65, TILE = 64 * LDC;
 constexpr int F_DM2 = 0, F_DMQ = TILE, F_DAB = 2 * TILE, F_KK = 3 * TILE, F_DAG = 4 * TILE,
               F_DAP = 5 * TILE, F_QK = 6 * TILE, F_VEC = 7 * TILE;
-static_assert((F_VEC + 9 * 64 + 5 * 4 * 64) * 4 <= (int)XH, "finish scratch");
+static_assert((F_VEC + 9 * 64 + 6 * 4 * 64) * 4 <= (int)XH, "finish scratch");
 // TMEM columns
 constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
 constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
@@ -840,7 +779,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   const float *recf = p.ws + chunk * kRecFloats;
-  const float *acc = P.acc + chunk * A8::FLOATS;
+  float *acc = P.acc + chunk * A8::FLOATS;
 
   Ctl K;
   ctl_init(K, sm + CTL, tid);
@@ -930,6 +869,19 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const uint32_t tm = *slot;
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
     float rv[32];
+    {  // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float qr[16];
+        tmem_ld16(tm + tm_lane + T_KR + 64 + tb + c0, qr);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rv[c0 + i] = scale * Gam[tb + c0 + i] * dov[c0 + i] * qr[i];
+      }
+      cta_row_sum256(rv, red, dGamS, tid);
+      // parked in the record's slot (shared memory is full); the same thread reads it back
+      if (tid < 64) acc[A8::VEC + A8::V_DGAM_OUT + tid] = dGamS[tid];
+      __syncthreads();
+    }
 #pragma unroll
     for (int c0 = 0; c0 < 32; c0 += 16) {
       float qs[16], qr[16];
@@ -1022,7 +974,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     });
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
-  //   G1 = [dOa ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
+  //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
   //   and the Gram matrices [K ; Q] K^T
   // images: E2 at SA (hi | lo), E at SA + 32 KB, dX at SB; the pair at X / Y
   if (ok) {
@@ -1036,9 +988,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     put_tok(x, SA, SA + 16384);
     put_tok(y, SA + 32768, SA + 49152);
     put_tok(xv, SB, SB + 16384);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) x[i] = gamv[tb + i] * dov[i];
-    put_tok(x, XH, XL);
+    put_tok(dov, XH, XL);  // [dO ; dX2]: gamma_t enters in the element-wise pass
     put_tok(x2v, YH, YL);
     ok = phase_run(K, tid, [&] {
       mma_tile_mnmn(tm + T_G1, sb + XH, 32768, sb + SA, 16384, 8, i64, false);
@@ -1070,7 +1020,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   float *F = reinterpret_cast<float *>(sm);
   float *cum = F + F_VEC, *cprev = cum + 64, *bet = cum + 128, *gam = cum + 192, *gg = cum + 256,
         *dcum = cum + 320, *dcprev = cum + 384, *dbet = cum + 448, *dgam = cum + 512;
-  float *prt = cum + 576;  // [5][4][64] partial sums
+  float *prt = cum + 576;  // [6][4][64] partial sums
   if (ok) {
     {
       const int r = j & 63;
@@ -1131,7 +1081,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {  // row pass: thread (t, quarter) over i in [16 q, 16 q + 16)
       const int t = tid & 63, q4 = tid >> 6;
       const float ct = cum[t], cpt = cprev[t];
-      float rowc = 0.f, rowp = 0.f;
+      const float gt = gam[t];
+      float rowc = 0.f, rowp = 0.f, dgo = 0.f;
 #pragma unroll 4
       for (int ii = 0; ii < 16; ++ii) {
         const int i = 16 * q4 + ii, e = t * LDC + i;
@@ -1139,8 +1090,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         if (i <= t) {
           const float dec = __expf(ct - cum[i]);
           const float kk = F[F_KK + e], qk = F[F_QK + e], bi = bet[i], gi = gam[i];
-          {  // M2: inclusive, gamma, Q K^T
-            const float dm = F[F_DM2 + e];
+          {  // M2: inclusive, gamma, Q K^T; G1 holds dO E2^T, dM2 = gamma_t dO E2^T
+            const float g1 = F[F_DM2 + e];
+            dgo += dec * gi * qk * g1;  // d gamma_t += (M2 E2)_t . dO_t
+            const float dm = gt * g1;
             const float G = dm * dec * gi * qk;
             rowc += G;
             cg += G;
@@ -1184,6 +1137,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       }
       prt[0 * 256 + q4 * 64 + t] = rowc;
       prt[1 * 256 + q4 * 64 + t] = rowp;
+      prt[5 * 256 + q4 * 64 + t] = dgo;
     }
     __syncthreads();
     {  // column pass: thread (i, quarter) over t in [16 q, 16 q + 16)
@@ -1203,16 +1157,16 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     __syncthreads();
     if (tid < 64) {
       const int i = tid;
-      float s5[5];
+      float s5[6];
 #pragma unroll
-      for (int w = 0; w < 5; ++w)
+      for (int w = 0; w < 6; ++w)
         s5[w] = prt[w * 256 + i] + prt[w * 256 + 64 + i] + prt[w * 256 + 128 + i] +
                 prt[w * 256 + 192 + i];
       const float cC = cum[63];
       const float eC = __expf(cC - cum[i]);
       const float dwS = acc[A8::VEC + A8::V_DWS + i], dwR = acc[A8::VEC + A8::V_DWR + i];
       dbet[i] = s5[3] + dwS * eC;
-      dgam[i] = s5[4] + acc[A8::VEC + A8::V_DGAM_OUT + i] + dwR * eC;
+      dgam[i] = s5[4] + s5[5] + acc[A8::VEC + A8::V_DGAM_OUT + i] + dwR * eC;
       dcum[i] = s5[0] - s5[2] - (dwS * bet[i] + dwR * gam[i]) * eC + dGamS[i] * __expf(cum[i]);
       dcprev[i] = s5[1] + dGprevS[i] * __expf(cprev[i]);
     }
@@ -1304,7 +1258,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 size_t bwd_tc_extra_bytes(int B, int H, int NC) {
   const size_t nct = (size_t)B * H * NC;
   return nct * (4 * 64 * D * sizeof(float) + 2 * (size_t)D * D * sizeof(float) +
-                D * sizeof(unsigned long long) + 16384);
+                D * sizeof(unsigned long long));
 }
 
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
@@ -1336,7 +1290,12 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.dSc = x + 4 * nct * 64 * D;
   P.dRc = P.dSc + nct * D * D;
   P.mask = reinterpret_cast<unsigned long long *>(P.dRc + nct * D * D);
-  P.gM2 = reinterpret_cast<uint8_t *>(P.mask + nct * D);
+  const bool saved = f.sv_E && f.sv_E2 && f.sv_mask;  // E, E2, mask kept by the forward
+  if (saved) {
+    P.Ebuf = f.sv_E;
+    P.E2buf = f.sv_E2;
+    P.mask = f.sv_mask;
+  }
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(bwd_recompute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)rc::SMEM)) != cudaSuccess)
@@ -1347,8 +1306,10 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   if ((e = cudaFuncSetAttribute(bwd_post_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)po::SMEM)) != cudaSuccess)
     return e;
-  RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (!saved) {
+    RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NT, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<(unsigned)nct, po::NTP, po::SMEM, s>>>(P));

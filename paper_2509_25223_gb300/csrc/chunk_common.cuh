@@ -23,7 +23,7 @@ constexpr int kRecFloats = OFF_VEC + 6 * C;
 //   T_beta  hi | lo  (64 rows each)      [IMG_TB,   IMG_TB + 16 KB)
 //   [Ap ; Mq] hi | lo (128 rows each)    [IMG_APMQ, IMG_APMQ + 32 KB)
 //   T_gamma hi | lo                      [IMG_TG,   ...)
-//   M2      hi | lo                      [IMG_M2,   ...)
+//   diag(gamma) M2 hi | lo               [IMG_M2,   ...)  (rows t scaled by gamma_t)
 //   the gate vectors at the same place as in the fp32 record (OFF_VEC).
 constexpr int IMG_TB = 0, IMG_APMQ = 16384, IMG_TG = 49152, IMG_M2 = 65536;
 static_assert(IMG_M2 + 16384 == OFF_VEC * 4, "image fills the matrix part of the record");
@@ -63,7 +63,24 @@ struct FwdParams {
   float *ST, *RT, *S_chunks, *R_chunks;
   float *ws;  // NC*B*H records of kRecFloats
   int *err;   // device status word (RDN_ERR_TIMEOUT if a bounded wait gave up) or NULL
+  // forward intermediates kept for the backward (RDN_FLAG_SAVE_FOR_BWD) or NULL:
+  // E, E2 as [chunk][t][j] fp32, the clip mask as [chunk][j] (bit t = |x| <= c)
+  float *sv_E, *sv_E2;
+  unsigned long long *sv_mask;
 };
+
+// Where the forward keeps those intermediates: after the B*H*NC records.
+struct SavedLayout {
+  size_t e, e2, mask, bytes;  // byte offsets from the workspace base; region size
+};
+inline SavedLayout saved_layout(size_t nct, int Dv) {
+  SavedLayout l;
+  l.e = nct * sizeof(float) * (size_t)kRecFloats;
+  l.e2 = l.e + nct * sizeof(float) * C * Dv;
+  l.mask = l.e2 + nct * sizeof(float) * C * Dv;
+  l.bytes = l.mask + nct * sizeof(unsigned long long) * Dv - l.e;
+  return l;
+}
 
 
 inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
@@ -78,6 +95,8 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.ST = a.ST; p.RT = a.RT; p.S_chunks = a.S_chunks; p.R_chunks = a.R_chunks;
   p.ws = nullptr;
   p.err = nullptr;
+  p.sv_E = p.sv_E2 = nullptr;
+  p.sv_mask = nullptr;
   return p;
 }
 

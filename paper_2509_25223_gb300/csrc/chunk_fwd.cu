@@ -184,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
       uint8_t *img = reinterpret_cast<uint8_t *>(rec);
       img_put(img + IMG_APMQ, 16384, t, i, ap);
       img_put(img + IMG_APMQ, 16384, 64 + t, i, mq);
-      img_put(img + IMG_M2, 8192, t, i, m2);
+      img_put(img + IMG_M2, 8192, t, i, gam[t] * m2);  // the image holds diag(gamma) M2
     } else {
       rec[OFF_AP + e] = ap;
       rec[OFF_MQ + e] = mq;
@@ -501,12 +501,15 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
               : launch_t<64, false, float>(p, s, true, false, img);
 }
 
-FwdPlan plan_fwd(const rdn_fwd_args &a, int /*variant*/) {
+FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   FwdPlan pl;
   pl.NC = (a.T + C - 1) / C;
   pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
-  // per-chunk records, then a 256-byte device status word
-  pl.total_bytes = pl.prep_bytes * (size_t)a.B * a.H * pl.NC + 256;
+  const size_t nct = (size_t)a.B * a.H * pl.NC;
+  // per-chunk records, the saved intermediates if asked for, then a 256-byte
+  // device status word
+  pl.total_bytes = pl.prep_bytes * nct + 256;
+  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) pl.total_bytes += saved_layout(nct, a.Dv).bytes;
   return pl;
 }
 
@@ -524,6 +527,12 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   FwdParams p = make_fwd_params(a);
   p.ws = (float *)a.workspace;
   p.err = (int *)((char *)a.workspace + plan_fwd(a, variant).total_bytes - 256);
+  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) {
+    const SavedLayout l = saved_layout((size_t)a.B * a.H * p.NC, a.Dv);
+    p.sv_E = (float *)((char *)a.workspace + l.e);
+    p.sv_E2 = (float *)((char *)a.workspace + l.e2);
+    p.sv_mask = (unsigned long long *)((char *)a.workspace + l.mask);
+  }
   return launch_fwd_parts(p, a.Dk, variant == 1, a.dtype == RDN_BF16, true, true, s);
 }
 

@@ -16,9 +16,9 @@
 //   MMA5  D3   = R^T  B1^T          -> [Gprev*KR | Gam*QR]
 //         X2   = r - alpha * (Gprev*KR)
 //   MMA6  E2^T = X2^T T_gamma^T
-//   MMA7  D3[:, Q half] += E2^T M2^T -> Oa
+//   MMA7  D1[:, Ob half] += E2^T (diag(gamma) M2)^T
 //   MMA8  U2   = (wR E2)^T K        -> R_C = Gam_C R + U2 (two N=64 halves)
-//         o    = Ob + gamma * Oa
+//         o    = D1[:, Ob half] + gamma * (Gam*QR)   (= Ob + gamma * Oa)
 //
 // RLA skips MMA2 and MMA6 (E = V, E2 = r).  X, E, wS E and their auxiliary
 // counterparts (magnitude ~ |v|) enter the MMAs as bf16 hi + lo pairs, which
@@ -34,7 +34,7 @@
 // (hi*hi + hi*lo + lo*hi).
 //
 // TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) X
-// (X holds E, then U, then D3; D1 holds P|Ob, then E2 | Ob, then U2a | Ob).
+// (X holds E, then U, then D3; D1 holds P|Ob, then E2 | Ob, then U2a | Ob + gamma M2 E2).
 #include "chunk_common.cuh"
 #include "tc_common.cuh"
 
@@ -297,10 +297,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
 
     // ---- (d) E -> EA, wS*E -> WA;  MMA3: D1 += E^T [Ap;Mq]^T,  MMA4: U = (wS E)^T K
+    const size_t ci = (size_t)bh * NC + c;  // chunk index of the saved intermediates
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_X + c0, e);
+        if (p.sv_E) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) p.sv_E[(ci * 64 + c0 + i) * D + j] = e[i];
+        }
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = vval(t0, n, c0 + i);
@@ -323,14 +328,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (tid == 0) load_slot(sm + SM_SLOTB, barB, rec_of(c) + IMG_M2, 16384);
 
     // ---- (e) r = clip(V - P); S = Gam_C S + U (fp32 in TMEM, bf16 copy in SA)
+    unsigned long long msk = 0ull;  // bit t: |x| <= c (the clip passes the gradient)
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float pp[16];
       tmem_ld16(tm + lane + T_D1 + c0, pp);
 #pragma unroll
-      for (int i = 0; i < 16; ++i)
-        rres[c0 + i] = clampf(vval(t0, n, c0 + i) - pp[i], clip);
+      for (int i = 0; i < 16; ++i) {
+        const float x = vval(t0, n, c0 + i) - pp[i];
+        if (fabsf(x) <= clip) msk |= 1ull << (c0 + i);
+        rres[c0 + i] = clampf(x, clip);
+      }
     }
+    if (p.sv_mask) p.sv_mask[ci * D + j] = msk;
     for (int c0 = 0; c0 < D; c0 += 16) {
       float s[16], u[16];
       tmem_ld16(tm + lane + T_S + c0, s);
@@ -369,12 +379,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTA, barA, rec_of(c + 1) + IMG_TB, 16384);
     }
 
-    // ---- (g) E2 -> EA, wR*E2 -> WA;  MMA7: Oa += E2^T M2^T;  MMA8: U2 = (wR E2)^T K
+    // ---- (g) E2 -> EA, wR*E2 -> WA;  MMA7: Ob += E2^T (gamma M2)^T;  MMA8: U2 = (wR E2)^T K
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_D1 + c0, e);
+        if (p.sv_E2) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) p.sv_E2[(ci * 64 + c0 + i) * D + j] = e[i];
+        }
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
@@ -388,7 +402,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       const uint32_t i64 = idesc_bf16(128, 64);
       if (!mbar_wait(barB, phB)) return false;
       phB ^= 1u;
-      mma_split3(tm + T_X + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
+      // the image is diag(gamma) M2: its product lands on Ob directly
+      mma_split3(tm + T_D1 + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 8192, i64, true);
       mma_tile(tm + T_D1, sbase + SM_W, 0, sbase + SM_KT, 0, 4, i64, false);
       mma_tile(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KT, 0, 4, i64, true);
@@ -399,7 +414,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (!alive) break;
     if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTB, barB, rec_of(c + 1) + IMG_APMQ, 32768);
 
-    // ---- (h) o = Ob + gamma * Oa;  R = Gam_C R + U2
+    // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R = Gam_C R + U2
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float ob[16], oa[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);

@@ -64,7 +64,9 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(dtype=7)) == 2
     assert _status(fn, _fwd_args(clip=-1.0)) == 1
     assert _status(fn, _fwd_args(clip=float("nan"))) == 1
-    assert _status(fn, _fwd_args(flags=1)) == 2
+    assert _status(fn, _fwd_args(flags=2)) == 2
+    # RDN_FLAG_SAVE_FOR_BWD: rdn_fwd only, and only with chunk states
+    assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD)) == (2 if fn == "rla_fwd" else 1)
     assert _status(fn, _fwd_args()) == 1  # q is NULL
     assert "q is NULL" in lib.rdn_last_error().decode()
     ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE, o=FAKE)
@@ -72,6 +74,9 @@ def test_fwd_validation(fn):
     mis["v"] = ctypes.c_void_p(0x10004)
     assert _status(fn, _fwd_args(**mis)) == 6
     assert _status(fn, _fwd_args(S_chunks=FAKE, **ok)) == 1  # R_chunks missing
+    if fn == "rdn_fwd":
+        assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, **ok)) == 1
+        assert "S_chunks" in lib.rdn_last_error().decode()
     assert _status(fn, _fwd_args(**ok)) == 5  # no workspace
     assert "workspace" in lib.rdn_last_error().decode()
 
@@ -83,6 +88,12 @@ def test_workspace_size_queries():
     assert n.value > 0
     assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args(Dk=32, Dv=32)), ctypes.byref(n)) == 2
     assert lib.rdn_fwd_workspace_size(ctypes.byref(_fwd_args()), None) == 1
+    m = ctypes.c_size_t(0)
+    a = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD)
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(a), ctypes.byref(m)) == 0
+    # E, E2 (fp32 [64][Dv] each) and the mask (one word per value column) per chunk
+    nct = a.B * a.H * ((a.T + 63) // 64)
+    assert m.value - n.value == nct * (2 * 64 * 128 * 4 + 128 * 8)
 
 
 def test_decode_validation():
@@ -129,6 +140,12 @@ def test_bwd_validation():
     assert "fwd.workspace" in lib.rdn_last_error().decode()
     b.fwd = _fwd_args(workspace=ctypes.c_void_p(0x10008), workspace_bytes=n.value, S_chunks=FAKE,
                       R_chunks=FAKE, **ok)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 5
+    # saved intermediates: need the forward's workspace, sized with the flag
+    b.fwd = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, S_chunks=FAKE, R_chunks=FAKE, **ok)
+    assert lib.rdn_bwd(ctypes.byref(b), None) == 1
+    b.fwd = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, workspace=FAKE, workspace_bytes=n.value,
+                      S_chunks=FAKE, R_chunks=FAKE, **ok)
     assert lib.rdn_bwd(ctypes.byref(b), None) == 5
 
 

@@ -147,19 +147,41 @@ def test_bwd_reuses_forward_records(dtype, D):
         assert_close(d1[name], ref[name], dtype, name)
 
 
+@pytest.mark.parametrize("dtype,D,T", [("bf16", 128, 150), ("bf16", 128, 1), ("bf16", 64, 150),
+                                       ("f32", 128, 150)])
+def test_bwd_uses_forward_saved_intermediates(dtype, D, T):
+    """A forward run with save_for_bwd keeps E, E2 and the clip mask; the
+    backward that reads them matches the one that recomputes them, and the
+    oracle."""
+    x = make_inputs(2, T, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    _condition(x, 1.0, dtype)
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", 2, T, 2, D, tdt, save_for_bwd=True),
+                      dtype=torch.uint8, device="cuda")
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                                    return_chunk_states=True, workspace=wsf, save_for_bwd=True)
+    d1 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True)
+    d2 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc)
+    ref = _ref(x, 1.0)
+    for name in GRADS:
+        torch.testing.assert_close(d1[name].float(), d2[name].float(), atol=1e-5, rtol=8e-3)
+        assert_close(d1[name], ref[name], dtype, name)
+
+
 def test_bwd_full_size_sampled():
     """The bench's fwd+bwd workload (B=8, H=16, T=4096, D=128, bf16) in the
-    bench's launch configuration (chunk states and per-chunk matrices from
-    rdn_fwd); the oracle checks sampled heads."""
+    bench's launch configuration (chunk states, per-chunk matrices and saved
+    intermediates from rdn_fwd); the oracle checks sampled heads."""
     w = WORKLOADS["rdn_fwd_bwd_bf16_B8H16T4096D128"]
     x = make_workload_inputs(w, device="cuda")
     heads = [(0, 0), (5, 9), (7, 15)]
     _condition(x, 1.0, "bf16", heads=heads)
-    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", w.B, w.T, w.H, w.D), dtype=torch.uint8,
-                      device="cuda")
+    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", w.B, w.T, w.H, w.D, save_for_bwd=True),
+                      dtype=torch.uint8, device="cuda")
     o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, return_chunk_states=True,
-                                    workspace=wsf)
-    d = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf)
+                                    workspace=wsf, save_for_bwd=True)
+    d = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True)
     for name in GRADS:
         assert torch.isfinite(d[name].float()).all(), name
     for (b, h), ref in zip(heads, _ref(x, 1.0, heads=heads)):
