@@ -64,7 +64,8 @@ struct TcBwdParams {
   float *acc;            // per-chunk records
   float *Ebuf, *E2buf;   // [B*H*NC][64][128] fp32 (t, j)
   float *dX2buf, *dXbuf; // [B*H*NC][64][128]
-  float *dSc, *dRc;      // [B*H*NC][128][128] (i, j): gradients w.r.t. chunk-end states
+  uint8_t *gimg;         // [B*H*NC][128 KB]: gradients w.r.t. each chunk's end states as
+                         // bf16 images (rows j): dS hi | dR hi | dS lo | dR lo, 32 KB each
   unsigned long long *mask;  // [B*H*NC][128]: bit t = clip inactive (|x| <= c)
   void *dq, *dk;             // outputs of bwd_post
   float *dg, *dbeta, *dgamma;
@@ -192,8 +193,7 @@ __device__ __forceinline__ void cta_row_sum(const float (&v)[64], float *scratch
 namespace rc {
 constexpr uint32_t SA = 0, RA = 32768, B1 = 65536, SLOTA = 98304, SLOTB = 114688;
 constexpr uint32_t XE = 147456, XE_LO = 163840, VEC = 180224;
-constexpr uint32_t RED = VEC + 7 * 64 * 4;       // 4*64 floats
-constexpr uint32_t CTL = RED + 4 * 64 * 4;
+constexpr uint32_t CTL = VEC + 7 * 64 * 4;
 constexpr uint32_t SLOT = CTL + 32;
 constexpr size_t SMEM = SLOT + 16;
 constexpr uint32_t T_D1 = 0, T_D3 = 128, T_X = 256;
@@ -369,13 +369,12 @@ constexpr uint32_t KQ = 0;
 constexpr uint32_t DSH = 32768, DRH = 65536, DSL = 98304, DRL = 131072;
 constexpr uint32_t SLOTA = 163840;   // diag(gamma) M2 -> T_gamma -> T_beta (16 KB)
 constexpr uint32_t SLOTB = 180224;   // Mq -> Ap (hi 8 KB | lo 8 KB)
-constexpr uint32_t DOT = 196608;     // dO^T, exact bf16
+constexpr uint32_t DOT = 196608;     // dO, exact bf16, rows t (two 8 KB column blocks)
 // scratch column tiles (hi, lo) inside the gradient-tile region
 constexpr uint32_t S0H = 32768, S0L = 49152, S1H = 65536, S1L = 81920;
 constexpr uint32_t S2H = 98304, S2L = 114688, S3H = 131072, S3L = 147456;
 constexpr uint32_t VEC = 212992;                 // Gam Gprev wS wR gamma (5 x 64)
-constexpr uint32_t RED = VEC + 5 * 64 * 4;       // 4 x 64 + 64 floats (row sums)
-constexpr uint32_t CTL = RED + 5 * 64 * 4;
+constexpr uint32_t CTL = VEC + 5 * 64 * 4;
 constexpr uint32_t SLOT = CTL + 32;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
@@ -449,6 +448,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       put16(sm + DRH, 16384, j, c0, rh);
       put16(sm + DRL, 16384, j, c0, rl);
     }
+    fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   };
   for (int c0 = 0; c0 < D; c0 += 16) {  // upstream gradients of the final states
     float s[16], r[16];
@@ -468,18 +468,10 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     const int t0 = c * 64, n = min(64, T - t0);
     const float *recf = p.ws + chunk * kRecFloats;
     __syncthreads();
-    {  // gradients w.r.t. this chunk's end states, for bwd_post
-      float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
-      for (int c0 = 0; c0 < D; c0 += 16) {
-        float s[16], r[16];
-        tmem_ld16(tm + lane + T_DS + c0, s);
-        tmem_ld16(tm + lane + T_DR + c0, r);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          gS[(size_t)(c0 + i) * D + j] = s[i];
-          gR[(size_t)(c0 + i) * D + j] = r[i];
-        }
-      }
+    if (tid == 0) {  // gradients w.r.t. this chunk's end states, for bwd_post: the tile images
+      static_assert(DRH == DSH + 32768 && DSL == DRH + 32768 && DRL == DSL + 32768, "contiguous");
+      bulk_s2g(P.gimg + chunk * 131072, sm + DSH, 131072);
+      bulk_commit();
     }
     if (tid < 64) {
       Gam[tid] = recf[OFF_VEC + V_GAM + tid];
@@ -489,31 +481,26 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
     }
     const float GamC = recf[OFF_VEC + V_GAMC];
-    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q (exact bf16) and dO^T
+    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q, dO (exact bf16), rows t
       const int t = e >> 4, chn = e & 15;
-      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv, ov = kv;
       if (t < n) {
         const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
         kv = *reinterpret_cast<const uint4 *>(k + off);
         qv = *reinterpret_cast<const uint4 *>(q + off);
+        ov = *reinterpret_cast<const uint4 *>(dOp + off);
       }
       const int blk = chn >> 3, cc = (chn & 7) * 8;
       *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
       *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+      *reinterpret_cast<uint4 *>(sm + DOT + blk * 8192 + sw128(t, cc)) = ov;
     }
     __syncthreads();
-    float dO[64];
-#pragma unroll
-    for (int t = 0; t < 64; ++t)
-      dO[t] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
     const unsigned long long m = P.mask[chunk * D + j];
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {  // dO^T, exact in bf16
-      float y[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) y[i] = dO[c0 + i];
-      put16(sm + DOT, 0, j, c0, y);
-    }
+    auto dO = [&](int t) {  // dO[t, j] from the tile
+      return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
+          sm + DOT + (j >> 6) * 8192 + sw128(t, j & 63)));
+    };
     // ---- phase A: K dR, K dS (gradients hi + lo), M2^T (gamma dO), Mq^T dO
     ok = phase_run(K, tid, [&] {
       if (!slot_wait(K.barA, K.phA)) return false;
@@ -523,10 +510,12 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       mma_tile(tm + T_R1, sb + DRL, 16384, sb + KQ, 16384, 8, i64, true);
       mma_tile(tm + T_R2, sb + DSH, 16384, sb + KQ, 16384, 8, i64, false);
       mma_tile(tm + T_R2, sb + DSL, 16384, sb + KQ, 16384, 8, i64, true);
-      mma_tile_kmn(tm + T_R3, sb + DOT, 0, sb + SLOTA, 16384, 4, i64, false);
-      mma_tile_kmn(tm + T_R3, sb + DOT, 0, sb + SLOTA + 8192, 16384, 4, i64, true);
-      mma_tile_kmn(tm + T_R4, sb + DOT, 0, sb + SLOTB, 16384, 4, i64, false);
-      mma_tile_kmn(tm + T_R4, sb + DOT, 0, sb + SLOTB + 8192, 16384, 4, i64, true);
+      // dO enters as the MN-major A operand (rows t, value-column atoms 8 KB apart)
+      mma_tile_mnmn(tm + T_R3, sb + DOT, 8192, sb + SLOTA, 16384, 4, i64, false);
+      mma_tile_mnmn(tm + T_R3, sb + DOT, 8192, sb + SLOTA + 8192, 16384, 4, i64, true);
+      mma_tile_mnmn(tm + T_R4, sb + DOT, 8192, sb + SLOTB, 16384, 4, i64, false);
+      mma_tile_mnmn(tm + T_R4, sb + DOT, 8192, sb + SLOTB + 8192, 16384, 4, i64, true);
+      bulk_wait_read();  // the tiles become scratch after this phase
       return true;
     });
     if (!ok) break;
@@ -547,28 +536,11 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
         const int t = c0 + i;
         m2[i] = m2[i] + wR[t] * kdr[i];
         mq[i] = mq[i] + wS[t] * kds[i];
-        dqr[i] = p.scale * Gam[t] * gamv[t] * dO[t];  // Q below is unscaled
+        dqr[i] = p.scale * Gam[t] * gamv[t] * dO(t);  // Q below is unscaled
       }
       tmem_st16(tm + lane + T_R4 + c0, mq);
       put16s(sm + S0H, sm + S0L, j, c0, m2);
       put16s(sm + S1H, sm + S1L, j, c0, dqr);
-    }
-    {  // dwS_t = sum_j (K dS)[t,j] E[t,j], dwR_t = sum_j (K dR)[t,j] E2[t,j]
-      float *red = reinterpret_cast<float *>(sm + RED);
-      float *acc = P.acc + chunk * A8::FLOATS;
-      const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
-      for (int w = 0; w < 2; ++w) {
-        float pr[64];
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) {
-          float kd[16];
-          tmem_ld16(tm + lane + (w == 0 ? T_R2 : T_R1) + c0, kd);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) pr[c0 + i] = kd[i] * (w == 0 ? Eg : E2g)[(c0 + i) * D + j];
-        }
-        cta_row_sum(pr, red, red + 256, tid);
-        if (tid < 64) acc[A8::VEC + (w == 0 ? A8::V_DWS : A8::V_DWR) + tid] = red[256 + tid];
-      }
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
     ok = phase_run(K, tid, [&] {
@@ -630,7 +602,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           a[i] += e[i];
-          dqs[i] = p.scale * Gam[c0 + i] * dO[c0 + i];
+          dqs[i] = p.scale * Gam[c0 + i] * dO(c0 + i);
         }
         put16s(sm + S0H, sm + S0L, j, c0, a);
         put16s(sm + S1H, sm + S1L, j, c0, dqs);
@@ -697,6 +669,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   } else if (tid == 0 && p.err) {
     atomicExch(p.err, RDN_ERR_TIMEOUT);
   }
+  if (tid == 0) bulk_wait_all();
   fence_before_sync();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, 512);
@@ -736,6 +709,7 @@ constexpr int F_DM2 = 0, F_DMQ = TILE, F_DAB = 2 * TILE, F_KK = 3 * TILE, F_DAG 
 static_assert((F_VEC + 9 * 64 + 6 * 4 * 64) * 4 <= (int)XH, "finish scratch");
 // TMEM columns
 constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
+constexpr uint32_t T_KDR = 0, T_KDS = 64;                        // P4, after the read-outs
 constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
 }  // namespace po
 
@@ -781,9 +755,17 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const float *recf = p.ws + chunk * kRecFloats;
   float *acc = P.acc + chunk * A8::FLOATS;
 
+  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
+  const uint8_t *gimg = P.gimg + chunk * 131072;  // dS hi | dR hi | dS lo | dR lo
   Ctl K;
   ctl_init(K, sm + CTL, tid);
   if (warp == 0) tmem_alloc(slot, 512);
+  __syncthreads();  // barriers initialised
+  if (tid == 0) {   // chunk-start states, fp32, staged where their images go
+    mbar_expect_tx(K.barA, 131072);
+    bulk_g2s(sm + SA, S0, 65536, K.barA);
+    bulk_g2s(sm + SB, R0, 65536, K.barA);
+  }
   if (tid < 64) {
     Gam[tid] = recf[OFF_VEC + V_GAM + tid];
     Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
@@ -805,8 +787,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
   const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
-  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
-  const float *gS = P.dSc + chunk * D * D, *gR = P.dRc + chunk * D * D;
   const unsigned long long m = P.mask[chunk * D + j] >> tb;
   // this thread's tokens of dX2, dX, dO
   float x2v[32], xv[32], dov[32];
@@ -817,26 +797,35 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     xv[i] = Xg[t * D + j];
     dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
   }
-  // a [i][j] fp32 state -> rows j of its (hi | lo) image, key rows of half hf
-  auto put_state = [&](const float *src, uint32_t img) {
+  // fp32 [i][j] state staged at `base` -> rows j of its (hi | lo) image at
+  // `base`, key rows of half hf (every thread reads its values before any writes)
+  auto stage_to_image = [&](uint32_t base) {
+    const float *st = reinterpret_cast<const float *>(sm + base);
     float v[64];
 #pragma unroll
-    for (int i = 0; i < 64; ++i) v[i] = src[(size_t)(64 * hf + i) * D + j];
+    for (int i = 0; i < 64; ++i) v[i] = st[(64 * hf + i) * D + j];
+    __syncthreads();
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float w[16];
 #pragma unroll
       for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
-      put16s(sm + img + hf * 16384, sm + img + 32768 + hf * 16384, j, c0, w);
+      put16s(sm + base + hf * 16384, sm + base + 32768 + hf * 16384, j, c0, w);
     }
   };
-  // <src, g> over this thread's 64 entries
-  auto dot_state = [&](const float *src, const float *g) {
+  // sum over this thread's entries of (image at base, hi + lo) * x[i][j]
+  auto dot_image = [&](uint32_t base, const float (&x)[64]) {
     float s = 0.f;
-#pragma unroll 16
-    for (int i = 0; i < 64; ++i) {
-      const size_t o = (size_t)(64 * hf + i) * D + j;
-      s += src[o] * g[o];
+#pragma unroll
+    for (int c8 = 0; c8 < 8; ++c8) {
+      const uint32_t o = base + hf * 16384 + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
+      const uint4 hv = *reinterpret_cast<const uint4 *>(sm + o);
+      const uint4 lv = *reinterpret_cast<const uint4 *>(sm + o + 32768);
+      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
+      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        s += (__bfloat162float(hb[e]) + __bfloat162float(lb[e])) * x[c8 * 8 + e];
     }
     return s;
   };
@@ -854,9 +843,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const uint32_t tm_lane = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
 
-  put_state(S0, SA);
-  put_state(R0, SB);
-  float gdot = dot_state(S0, gS) + dot_state(R0, gR);
+  if (!mbar_wait(K.barA, 0)) *K.flag = 1;  // phase_run below reports it to every thread
+  stage_to_image(SA);
+  stage_to_image(SB);
   // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
   bool ok = phase_run(K, tid, [&] {
     const uint32_t t_ = *slot;
@@ -908,15 +897,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       for (int i = 0; i < 16; ++i) rv[c0 + i] = dp_of(c0 + i) * ks[i];
     }
     cta_row_sum256(rv, red, dGprevS, tid);
-#pragma unroll
-    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
-    if (lane == 0) red[warp] = gdot;
-    __syncthreads();
-    if (tid == 0) {
-      float s = 0.f;
-      for (int w = 0; w < NTP / 32; ++w) s += red[w];
-      *dGamC = s;
-    }
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
     float x[32], y[32];
 #pragma unroll
@@ -933,6 +913,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile_mnmn(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 32768, 8, i128, true);
       return true;
     });
+  }
+  if (ok && tid == 0) {  // R0's image is done with: dR's image into its place
+    mbar_expect_tx(K.barB, 65536);
+    bulk_g2s(sm + SB, gimg + 32768, 32768, K.barB);
+    bulk_g2s(sm + SB + 32768, gimg + 98304, 32768, K.barB);
   }
   if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO
     float x[32], y[32];
@@ -951,15 +936,48 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       return true;
     });
   }
-  if (ok) {  // ---- P4: dK += dR (diag(wR) E2)^T + dS (diag(wS) E)^T
-    put_state(gR, SB);
-    put_state(gS, SA);
+  if (ok && tid == 0) {  // and dS's image into S0's
+    mbar_expect_tx(K.barA, 65536);
+    bulk_g2s(sm + SA, gimg, 32768, K.barA);
+    bulk_g2s(sm + SA + 32768, gimg + 65536, 32768, K.barA);
+  }
+  if (ok) {  // <dR, R0> + <dS, S0> (states re-read from L2), reduced into dGamC
+    float gdot;
+    {
+      float x[64];
+#pragma unroll
+      for (int i = 0; i < 64; ++i) x[i] = R0[(size_t)(64 * hf + i) * D + j];
+      if (!mbar_wait(K.barB, 0)) *K.flag = 1;
+      gdot = dot_image(SB, x);
+#pragma unroll
+      for (int i = 0; i < 64; ++i) x[i] = S0[(size_t)(64 * hf + i) * D + j];
+      if (!mbar_wait(K.barA, 1)) *K.flag = 1;
+      gdot += dot_image(SA, x);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
+    if (lane == 0) red[warp] = gdot;
+    __syncthreads();
+    if (tid == 0) {
+      float s = 0.f;
+      for (int w = 0; w < NTP / 32; ++w) s += red[w];
+      *dGamC = s;
+    }
+    ok = *K.flag == 0;
+  }
+  float e2v[32], ev[32];  // this thread's tokens of E2, E
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    e2v[i] = E2g[(tb + i) * D + j];
+    ev[i] = Eg[(tb + i) * D + j];
+  }
+  if (ok) {  // ---- P4: dK += dR (diag(wR) E2)^T + dS (diag(wS) E)^T ; K dR, K dS read-outs
     float x[32], y[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       const int t = tb + i;
-      x[i] = wR[t] * E2g[t * D + j];
-      y[i] = wS[t] * Eg[t * D + j];
+      x[i] = wR[t] * e2v[i];
+      y[i] = wS[t] * ev[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -970,23 +988,35 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YH, 16384, 8, i64, true);
       mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
       mma_tile_mnmn(tm + T_DKQ, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
+      // (K dR)^T, (K dS)^T (lanes j, columns t; K exact)
+      mma_tile(tm + T_KDR, sb + SB, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile(tm + T_KDR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i64, true);
+      mma_tile(tm + T_KDS, sb + SA, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile(tm + T_KDS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i64, true);
       return true;
     });
+  }
+  if (ok) {  // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
+    for (int w = 0; w < 2; ++w) {
+      float rv[32];
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float kd[16];
+        tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb + c0, kd);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rv[c0 + i] = kd[i] * (w == 0 ? e2v[c0 + i] : ev[c0 + i]);
+      }
+      // parked in the record's slots (shared memory is full); read in the gate pass
+      cta_row_sum256(rv, red, acc + A8::VEC + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
+    }
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
   //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
   //   and the Gram matrices [K ; Q] K^T
   // images: E2 at SA (hi | lo), E at SA + 32 KB, dX at SB; the pair at X / Y
   if (ok) {
-    float x[32], y[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int t = tb + i;
-      x[i] = E2g[t * D + j];
-      y[i] = Eg[t * D + j];
-    }
-    put_tok(x, SA, SA + 16384);
-    put_tok(y, SA + 32768, SA + 49152);
+    put_tok(e2v, SA, SA + 16384);
+    put_tok(ev, SA + 32768, SA + 49152);
     put_tok(xv, SB, SB + 16384);
     put_tok(dov, XH, XL);  // [dO ; dX2]: gamma_t enters in the element-wise pass
     put_tok(x2v, YH, YL);
@@ -1287,9 +1317,8 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.E2buf = x + nct * 64 * D;
   P.dX2buf = x + 2 * nct * 64 * D;
   P.dXbuf = x + 3 * nct * 64 * D;
-  P.dSc = x + 4 * nct * 64 * D;
-  P.dRc = P.dSc + nct * D * D;
-  P.mask = reinterpret_cast<unsigned long long *>(P.dRc + nct * D * D);
+  P.gimg = reinterpret_cast<uint8_t *>(x + 4 * nct * 64 * D);
+  P.mask = reinterpret_cast<unsigned long long *>(P.gimg + nct * 131072);
   const bool saved = f.sv_E && f.sv_E2 && f.sv_mask;  // E, E2, mask kept by the forward
   if (saved) {
     P.Ebuf = f.sv_E;

@@ -50,7 +50,7 @@ constexpr int kTcThreads = 128;
 constexpr uint32_t SM_SA = 0;          // S^T bf16, 128 x 128, two 64-col blocks
 constexpr uint32_t SM_RA = 32768;      // R^T bf16
 constexpr uint32_t SM_B1 = 65536;      // [Gprev K ; Gam Q], 128 x 128
-constexpr uint32_t SM_KT = 98304;      // K^T, 128 (d_k) x 64 (t)
+constexpr uint32_t SM_KT = 98304;      // K, 64 (t) x 128 (d_k), unscaled: MN-major B operand
 constexpr uint32_t SM_SLOTA = 114688;  // T_beta then T_gamma image (hi | lo), 16 KB
 constexpr uint32_t SM_SLOTB = 131072;  // [Ap;Mq] then M2 image (hi | lo), 32 KB
 // value-like operands are split into bf16 hi + lo parts (two MMAs each):
@@ -204,7 +204,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return *flag == 0;
   };
 
-  float rres[64];  // clipped residual r[t] of column j
+  float rres[64];  // v[t] of column j, then (from step e) the clipped residual r[t]
   // v[t, j] of the current chunk (0 beyond the sequence), read from L2/HBM
   auto vval = [&](int t0, int n, int t) -> float {
     return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
@@ -215,6 +215,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     const int n = min(64, T - t0);
     const float *rec = p.ws + ((size_t)bh * NC + c) * kRecFloats;
     __syncthreads();  // every thread is done with the previous chunk's tiles and vectors
+#pragma unroll
+    for (int t = 0; t < 64; ++t) rres[t] = vval(t0, n, t);  // in flight during (a) and MMA1
 
     // ---- (a) chunk inputs -> shared memory
     if (p.S_chunks) {  // chunk-start states for the backward
@@ -262,10 +264,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       const int blk = ch >> 3, cc = (ch & 7) * 8;
       *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(t, cc)) = ks;
       *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc)) = qs;
-      __nv_bfloat16 *kt = reinterpret_cast<__nv_bfloat16 *>(sm + SM_KT);
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        kt[sw128(ch * 8 + i, t) / 2] = kb[i];
+      *reinterpret_cast<uint4 *>(sm + SM_KT + blk * 8192 + sw128(t, cc)) = kv;
     }
 
     // ---- (b) MMA1: D1 = S^T B1^T
@@ -282,7 +281,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         float x[16];
         tmem_ld16(tm + lane + T_D1 + c0, x);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = vval(t0, n, c0 + i) - alpha[c0 + i] * x[i];
+        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - alpha[c0 + i] * x[i];
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
       }
       alive = run_phase([&] {
@@ -308,7 +307,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         }
       } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) e[i] = vval(t0, n, c0 + i);
+        for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
       }
 #pragma unroll
       for (int i = 0; i < 16; ++i) w[i] = wS[c0 + i] * e[i];
@@ -320,8 +319,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       phB ^= 1u;
       mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 16384, idesc_bf16(128, 128), true);
-      mma_tile(tm + T_X, sbase + SM_W, 0, sbase + SM_KT, 0, 4, idesc_bf16(128, 128), false);
-      mma_tile(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT, 0, 4, idesc_bf16(128, 128), true);
+      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KT, 8192, 4, idesc_bf16(128, 128), false);
+      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT, 8192, 4, idesc_bf16(128, 128),
+                   true);
       return true;
     });
     if (!alive) break;
@@ -335,7 +335,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       tmem_ld16(tm + lane + T_D1 + c0, pp);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float x = vval(t0, n, c0 + i) - pp[i];
+        const float x = rres[c0 + i] - pp[i];
         if (fabsf(x) <= clip) msk |= 1ull << (c0 + i);
         rres[c0 + i] = clampf(x, clip);
       }
@@ -405,10 +405,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       // the image is diag(gamma) M2: its product lands on Ob directly
       mma_split3(tm + T_D1 + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 8192, i64, true);
-      mma_tile(tm + T_D1, sbase + SM_W, 0, sbase + SM_KT, 0, 4, i64, false);
-      mma_tile(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KT, 0, 4, i64, true);
-      mma_tile(tm + T_X, sbase + SM_W, 0, sbase + SM_KT + 8192, 0, 4, i64, false);
-      mma_tile(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT + 8192, 0, 4, i64, true);
+      mma_tile_kmn(tm + T_D1, sbase + SM_W, 0, sbase + SM_KT, 8192, 4, i64, false);
+      mma_tile_kmn(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KT, 8192, 4, i64, true);
+      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KT + 8192, 8192, 4, i64, false);
+      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT + 8192, 8192, 4, i64, true);
       return true;
     });
     if (!alive) break;
