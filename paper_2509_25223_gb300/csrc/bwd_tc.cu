@@ -41,18 +41,13 @@ using namespace tc;
 constexpr int D = 128;
 constexpr int NT = 128;  // threads per CTA
 
-template <int DK>
-struct AccL;  // layout of the per-chunk record, identical to chunk_bwd.cu's
-template <>
-struct AccL<128> {
-  static constexpr int DKo = 0, DQo = C * 128;
-  static constexpr int DAP = 2 * C * 128, DMQ = DAP + kCC, DM2 = DMQ + kCC, DAB = DM2 + kCC,
-                       DAG = DAB + kCC, VEC = DAG + kCC;
-  static constexpr int V_DGAM_OUT = 0, V_DGAM = C, V_DGPREV = 2 * C, V_DWS = 3 * C,
-                       V_DWR = 4 * C, V_DGAMC = 5 * C;
-  static constexpr int FLOATS = VEC + 6 * C;
+// Per-chunk row-sum slots in the backward workspace (floats): read-out part of
+// d gamma, dwS, dwR (C each).  Used as scratch by bwd_post, whose shared
+// memory is full.
+struct A8 {
+  static constexpr int V_DGAM_OUT = 0, V_DWS = C, V_DWR = 2 * C;
+  static constexpr int FLOATS = 3 * C;
 };
-using A8 = AccL<128>;
 
 struct TcBwdParams {
   FwdParams f;          // inputs; f.ws = prep records (shared-memory images)
@@ -868,7 +863,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       }
       cta_row_sum256(rv, red, dGamS, tid);
       // parked in the record's slot (shared memory is full); the same thread reads it back
-      if (tid < 64) acc[A8::VEC + A8::V_DGAM_OUT + tid] = dGamS[tid];
+      if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
       __syncthreads();
     }
 #pragma unroll
@@ -1007,7 +1002,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         for (int i = 0; i < 16; ++i) rv[c0 + i] = kd[i] * (w == 0 ? e2v[c0 + i] : ev[c0 + i]);
       }
       // parked in the record's slots (shared memory is full); read in the gate pass
-      cta_row_sum256(rv, red, acc + A8::VEC + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
+      cta_row_sum256(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
     }
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
@@ -1194,9 +1189,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
                 prt[w * 256 + 192 + i];
       const float cC = cum[63];
       const float eC = __expf(cC - cum[i]);
-      const float dwS = acc[A8::VEC + A8::V_DWS + i], dwR = acc[A8::VEC + A8::V_DWR + i];
+      const float dwS = acc[A8::V_DWS + i], dwR = acc[A8::V_DWR + i];
       dbet[i] = s5[3] + dwS * eC;
-      dgam[i] = s5[4] + s5[5] + acc[A8::VEC + A8::V_DGAM_OUT + i] + dwR * eC;
+      dgam[i] = s5[4] + s5[5] + acc[A8::V_DGAM_OUT + i] + dwR * eC;
       dcum[i] = s5[0] - s5[2] - (dwS * bet[i] + dwR * gam[i]) * eC + dGamS[i] * __expf(cum[i]);
       dcprev[i] = s5[1] + dGprevS[i] * __expf(cprev[i]);
     }
@@ -1205,7 +1200,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const float cC = cum[63];
       float s = 0.f;
       for (int t = lane; t < 64; t += 32)
-        s += (acc[A8::VEC + A8::V_DWS + t] * bet[t] + acc[A8::VEC + A8::V_DWR + t] * gam[t]) *
+        s += (acc[A8::V_DWS + t] * bet[t] + acc[A8::V_DWR + t] * gam[t]) *
              __expf(cC - cum[t]);
 #pragma unroll
       for (int off = 16; off; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
@@ -1284,6 +1279,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 }
 
 }  // namespace
+
+size_t bwd_tc_acc_bytes(int B, int H, int NC) {
+  return sizeof(float) * (size_t)B * H * NC * A8::FLOATS;
+}
 
 size_t bwd_tc_extra_bytes(int B, int H, int NC) {
   const size_t nct = (size_t)B * H * NC;

@@ -736,7 +736,8 @@ BwdLayout layout(const rdn_bwd_args &a) {
   BwdLayout l;
   // the forward's records are read from its workspace when it is passed
   l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nct * kRecFloats);
-  l.acc = align256(sizeof(float) * nct * accf);
+  l.acc = use_tc_bwd(f) ? align256(bwd_tc_acc_bytes(f.B, f.H, (f.T + C - 1) / C))
+                        : align256(sizeof(float) * nct * accf);
   const bool need_states = f.S_chunks == nullptr;
   l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;

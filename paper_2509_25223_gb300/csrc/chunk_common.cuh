@@ -110,6 +110,7 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
 
 // Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
 size_t bwd_tc_extra_bytes(int B, int H, int NC);
+size_t bwd_tc_acc_bytes(int B, int H, int NC);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
