@@ -28,6 +28,8 @@
 // sequential pass over chunks carrying S and R slices in shared memory.  Each
 // value column is independent (the clip is elementwise), so slicing d_v is
 // exact; only the prep work is shared between slices.
+#include <type_traits>
+
 #include "chunk_common.cuh"
 
 namespace rdn {
@@ -41,55 +43,6 @@ __device__ __forceinline__ void img_put(uint8_t *tile, uint32_t lo_off, int r, i
   const __nv_bfloat16 hi = __float2bfloat16_rn(x);
   *reinterpret_cast<__nv_bfloat16 *>(tile + o) = hi;
   *reinterpret_cast<__nv_bfloat16 *>(tile + lo_off + o) = __float2bfloat16_rn(x - __bfloat162float(hi));
-}
-
-// (I + A)^-1 for a 64 x 64 strictly lower A (row stride ld), by 16 x 16
-// blocks, with 128 threads (g = thread index within the group):
-//   diagonal blocks  T_ii = (I + A_ii)^-1 by forward substitution (one thread
-//                    per block column, the column kept in registers);
-//   block row i      W_j = sum_{k=j}^{i-1} A_ik T_kj,  T_ij = -T_ii W_j.
-// W is scratch of 3 x 256 floats.  The caller synchronises the block between
-// the calls of the 4 stages (stage 0: diagonal; stage i: block row i).
-__device__ __forceinline__ void inv_diag_blocks(const float *A, float *Tm, int ld, int g) {
-  if (g < 64) {
-    const int blk = g >> 4, col = g & 15, b0 = blk * 16;
-    float x[16];
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      float s = (r == col) ? 1.f : 0.f;
-#pragma unroll
-      for (int m = 0; m < r; ++m) s = fmaf(-A[(b0 + r) * ld + b0 + m], x[m], s);
-      x[r] = (r < col) ? 0.f : s;
-    }
-#pragma unroll
-    for (int r = 0; r < 16; ++r) Tm[(b0 + r) * ld + b0 + col] = x[r];
-  }
-  // zero the strictly upper blocks once
-  for (int e = g; e < 64 * 64; e += 128) {
-    const int r = e >> 6, c = e & 63;
-    if ((c >> 4) > (r >> 4)) Tm[r * ld + c] = 0.f;
-  }
-}
-__device__ __forceinline__ void inv_block_row_w(const float *A, const float *Tm, float *W, int ld,
-                                                int i, int g) {
-  for (int e = g; e < i * 256; e += 128) {
-    const int j = e >> 8, r = (e >> 4) & 15, cc = e & 15;
-    float s = 0.f;
-    for (int k = j; k < i; ++k)
-#pragma unroll
-      for (int m = 0; m < 16; ++m)
-        s = fmaf(A[(16 * i + r) * ld + 16 * k + m], Tm[(16 * k + m) * ld + 16 * j + cc], s);
-    W[e] = s;
-  }
-}
-__device__ __forceinline__ void inv_block_row_t(float *Tm, const float *W, int ld, int i, int g) {
-  for (int e = g; e < i * 256; e += 128) {
-    const int j = e >> 8, r = (e >> 4) & 15, cc = e & 15;
-    float s = 0.f;
-#pragma unroll
-    for (int m = 0; m < 16; ++m) s = fmaf(Tm[(16 * i + r) * ld + 16 * i + m], W[j * 256 + m * 16 + cc], s);
-    Tm[(16 * i + r) * ld + 16 * j + cc] = -s;
-  }
 }
 
 template <int DK, bool RDNV, typename InT, bool IMG>
@@ -454,8 +407,14 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
                                 (int)scan_smem<DK>())) != cudaSuccess)
     return e;
   if (do_prep) {
-    RDN_LAUNCH("chunk_prep", s, prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p));
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    // the images for RDN with bf16 inputs and d = 128 come from the tensor-core prep
+    constexpr bool tc_prep = DK == 128 && RDNV && std::is_same<InT, __nv_bfloat16>::value;
+    if (tc_prep && img) {
+      if ((e = launch_prep_tc(p, s)) != cudaSuccess) return e;
+    } else {
+      RDN_LAUNCH("chunk_prep", s, prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p));
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
   }
   if (do_scan)
     RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.B * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p));

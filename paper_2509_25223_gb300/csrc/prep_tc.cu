@@ -1,0 +1,270 @@
+// prep_tc.cu -- chunk_prep on the tensor cores for RDN with bf16 inputs and
+// d_k = 128: the state-independent matrices of one 64-token chunk (the UT
+// form of the delta rule, Section 3.5's chunkwise algorithm; algebra in
+// chunk_fwd.cu's header), written as the shared-memory images the
+// tensor-core scans copy into their operand slots.
+//
+// One chunk per CTA of 256 threads, two CTAs per SM:
+//   1. the Gram matrices [K ; Q] K^T in one tcgen05 product (bf16 inputs are
+//      exact, fp32 accumulation; the query scale is applied to the result);
+//   2. thread (row, half) turns its TMEM row into the decayed, gated matrices
+//      Ap, Mq, diag(gamma) M2 (written straight to the record as bf16 hi + lo
+//      image rows) and A_beta, A_gamma (fp32, shared memory);
+//   3. T_beta = (I + A_beta)^-1 and T_gamma = (I + A_gamma)^-1 by the blocked
+//      forward substitution of chunk_common.cuh, 128 threads each, in fp32;
+//   4. their image rows and the gate vectors.
+#include "chunk_common.cuh"
+#include "tc_common.cuh"
+
+namespace rdn {
+namespace {
+
+using namespace tc;
+
+constexpr int D = 128;
+constexpr int NTH = 256;
+constexpr int LDC = C + 1;
+
+namespace pp {
+constexpr uint32_t KQ = 0;                   // K rows 0..63, Q rows 64..127, 2 x 16 KB
+constexpr uint32_t AB = 32768;               // fp32 [64][65] each: A_beta, A_gamma, T_beta, T_gamma
+constexpr uint32_t AG = AB + 64 * LDC * 4;
+constexpr uint32_t TB = AG + 64 * LDC * 4;
+constexpr uint32_t TG = TB + 64 * LDC * 4;
+constexpr uint32_t WS = TG + 64 * LDC * 4;   // blocked-inverse scratch, 2 x 768 floats
+constexpr uint32_t VEC = WS + 2 * 768 * 4;   // cum, cprev, beta, gamma, g (5 x 64)
+constexpr uint32_t CTL = VEC + 5 * 64 * 4;   // mbarrier, flag
+constexpr uint32_t SLOT = CTL + 16;          // TMEM base
+constexpr size_t SMEM = SLOT + 16;
+static_assert(2 * (SMEM + 1024) <= 233472, "two CTAs per SM");
+}  // namespace pp
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Row r, columns c0 .. c0+15 (c0 a multiple of 16 below 64) of a 64-column
+// image in global memory: bf16 hi part at `hi`, lo part `lo_off` bytes later.
+__device__ __forceinline__ void img_row16(uint8_t *hi, uint32_t lo_off, int r, int c0,
+                                          const float (&v)[16]) {
+  float a[16], b[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+    b[i] = v[i] - a[i];
+  }
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    const int o = 8 * half;
+    uint4 x, y;
+    x.x = pack2(a[o + 0], a[o + 1]); x.y = pack2(a[o + 2], a[o + 3]);
+    x.z = pack2(a[o + 4], a[o + 5]); x.w = pack2(a[o + 6], a[o + 7]);
+    y.x = pack2(b[o + 0], b[o + 1]); y.y = pack2(b[o + 2], b[o + 3]);
+    y.z = pack2(b[o + 4], b[o + 5]); y.w = pack2(b[o + 6], b[o + 7]);
+    const uint32_t off = sw128(r, c0 + o);
+    *reinterpret_cast<uint4 *>(hi + off) = x;
+    *reinterpret_cast<uint4 *>(hi + lo_off + off) = y;
+  }
+}
+
+__global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
+  using namespace pp;
+  extern __shared__ __align__(1024) uint8_t sm[];
+  const uint32_t sb = smem_u32(sm);
+  if (sb & 1023u) {
+    if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
+    return;
+  }
+  float *cum = reinterpret_cast<float *>(sm + VEC), *cprev = cum + 64, *bet = cum + 128,
+        *gam = cum + 192, *gg = cum + 256;
+  float *Ab = reinterpret_cast<float *>(sm + AB), *Ag = reinterpret_cast<float *>(sm + AG);
+  float *Tb = reinterpret_cast<float *>(sm + TB), *Tg = reinterpret_cast<float *>(sm + TG);
+  float *Wsc = reinterpret_cast<float *>(sm + WS);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(sm + CTL);
+  volatile int *flag = reinterpret_cast<volatile int *>(sm + CTL + 8);
+  uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const size_t chunk = blockIdx.x;
+  const int NC = p.NC, T = p.T, H = p.H;
+  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
+  const int b = bh / H, h = bh % H;
+  const int t0 = c * C, n = min(C, T - t0);
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
+
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    *flag = 0;
+  }
+  if (warp == 0) tmem_alloc(slot, 64);
+  for (int e = tid; e < 64 * 16; e += NTH) {  // K, Q (exact bf16), rows t
+    const int t = e >> 4, chn = e & 15;
+    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
+    if (t < n) {
+      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
+      kv = *reinterpret_cast<const uint4 *>(k + off);
+      qv = *reinterpret_cast<const uint4 *>(q + off);
+    }
+    const int blk = chn >> 3, cc = (chn & 7) * 8;
+    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
+    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+  }
+  if (tid < C) {
+    const int t = tid;
+    float gv = 0.f, bv = 0.f, mv = 0.f;
+    if (t < n) {
+      const size_t off = (size_t)(b * T + t0 + t) * H + h;
+      gv = p.g[off];
+      bv = p.beta[off];
+      mv = p.gamma[off];
+    }
+    gg[t] = gv;
+    bet[t] = bv;
+    gam[t] = mv;
+  }
+  fence_async_smem();
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  if (tid == 0) {  // [K ; Q] K^T: lanes 0..63 K K^T, lanes 64..127 Q K^T (unscaled)
+    mma_tile(tm, sb + KQ, 16384, sb + KQ, 16384, 8, idesc_bf16(128, 64), false);
+    mma_commit(bar);
+  }
+  if (warp == 0) {  // in-chunk cumulative log-decay, while the product runs
+    float a = gg[lane], a2 = gg[32 + lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float ua = __shfl_up_sync(0xffffffffu, a, off);
+      const float ub = __shfl_up_sync(0xffffffffu, a2, off);
+      if (lane >= off) {
+        a += ua;
+        a2 += ub;
+      }
+    }
+    a2 += __shfl_sync(0xffffffffu, a, 31);
+    cum[lane] = a;
+    cum[32 + lane] = a2;
+    cprev[lane] = a - gg[lane];
+    cprev[32 + lane] = a2 - gg[32 + lane];
+  }
+  if (!mbar_wait(bar, 0)) *flag = 1;
+  __syncthreads();
+  fence_after_sync();
+  const bool ok = *flag == 0;
+  uint8_t *img = reinterpret_cast<uint8_t *>(p.ws + chunk * kRecFloats);
+  if (ok) {  // thread (row r, half hf) of the Gram read-out: columns i in [32 hf, 32 hf + 32)
+    const int r = tid & 127, hf = tid >> 7;
+    float gv[32];
+    {
+      const uint32_t ta = tm + ((uint32_t)((warp & 3) * 32) << 16) + 32 * hf;
+      float x[16];
+      tmem_ld16(ta, x);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) gv[i] = x[i];
+      tmem_ld16(ta + 16, x);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) gv[16 + i] = x[i];
+    }
+    if (r < 64) {  // K K^T row t: Ap (previous-token decay), A_beta, A_gamma (strict)
+      const int t = r;
+      const float ct = cum[t], cpt = cprev[t];
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float ap[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int i = 32 * hf + c0 + u;
+          const float kk = gv[c0 + u];
+          float a_p = 0.f, a_b = 0.f, a_g = 0.f;
+          if (i < t) {
+            const float dec = __expf(ct - cum[i]);
+            a_p = __expf(cpt - cum[i]) * bet[i] * kk;
+            a_b = dec * bet[i] * kk;
+            a_g = dec * gam[i] * kk;
+          }
+          ap[u] = a_p;
+          Ab[t * LDC + i] = a_b;
+          Ag[t * LDC + i] = a_g;
+        }
+        img_row16(img + IMG_APMQ, 16384, t, 32 * hf + c0, ap);
+      }
+    } else {  // Q K^T row t: Mq (strict), diag(gamma) M2 (inclusive)
+      const int t = r - 64;
+      const float ct = cum[t], gt = gam[t];
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float mq[16], m2[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int i = 32 * hf + c0 + u;
+          const float qk = p.scale * gv[c0 + u];
+          const float dec = i <= t ? __expf(ct - cum[i]) : 0.f;
+          mq[u] = i < t ? dec * bet[i] * qk : 0.f;
+          m2[u] = gt * dec * gam[i] * qk;
+        }
+        img_row16(img + IMG_APMQ, 16384, 64 + t, 32 * hf + c0, mq);
+        img_row16(img + IMG_M2, 8192, t, 32 * hf + c0, m2);
+      }
+    }
+  }
+  __syncthreads();
+  {  // T_beta (threads 0..127) and T_gamma (128..255)
+    const int g = tid & 127;
+    const float *A = tid < 128 ? Ab : Ag;
+    float *Tm = tid < 128 ? Tb : Tg;
+    float *W = Wsc + (tid < 128 ? 0 : 768);
+    inv_diag_blocks(A, Tm, LDC, g);
+    for (int i = 1; i < 4; ++i) {
+      __syncthreads();
+      inv_block_row_w(A, Tm, W, LDC, i, g);
+      __syncthreads();
+      inv_block_row_t(Tm, W, LDC, i, g);
+    }
+  }
+  __syncthreads();
+  if (ok) {
+    {  // image rows of T: thread (row r, matrix m, half hf)
+      const int r = tid & 63, m = (tid >> 6) & 1, hf = tid >> 7;
+      const float *Tm = m ? Tg : Tb;
+      uint8_t *dst = img + (m ? IMG_TG : IMG_TB);
+#pragma unroll
+      for (int c0 = 0; c0 < 32; c0 += 16) {
+        float v[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = Tm[r * LDC + 32 * hf + c0 + u];
+        img_row16(dst, 8192, r, 32 * hf + c0, v);
+      }
+    }
+    if (tid < C) {
+      float *rec = p.ws + chunk * kRecFloats;
+      const int t = tid;
+      const float cC = cum[C - 1];
+      rec[OFF_VEC + V_GAM + t] = __expf(cum[t]);
+      rec[OFF_VEC + V_GPREV + t] = __expf(cprev[t]);
+      rec[OFF_VEC + V_ALPHA + t] = __expf(gg[t]);
+      rec[OFF_VEC + V_WS + t] = bet[t] * __expf(cC - cum[t]);
+      rec[OFF_VEC + V_WR + t] = gam[t] * __expf(cC - cum[t]);
+      if (t == 0) rec[OFF_VEC + V_GAMC] = __expf(cC);
+    }
+  } else if (tid == 0 && p.err) {
+    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  }
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, 64);
+}
+
+}  // namespace
+
+cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)pp::SMEM);
+  if (e != cudaSuccess) return e;
+  RDN_LAUNCH("chunk_prep", s,
+             prep_tc_kernel<<<(unsigned)(p.B * p.H * p.NC), NTH, pp::SMEM, s>>>(p));
+  return cudaGetLastError();
+}
+
+}  // namespace rdn
