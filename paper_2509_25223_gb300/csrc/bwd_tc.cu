@@ -476,20 +476,16 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
     }
     const float GamC = recf[OFF_VEC + V_GAMC];
-    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q, dO (exact bf16), rows t
+    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q, dO (exact bf16), rows t, asynchronous
       const int t = e >> 4, chn = e & 15;
-      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv, ov = kv;
-      if (t < n) {
-        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
-        kv = *reinterpret_cast<const uint4 *>(k + off);
-        qv = *reinterpret_cast<const uint4 *>(q + off);
-        ov = *reinterpret_cast<const uint4 *>(dOp + off);
-      }
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
       const int blk = chn >> 3, cc = (chn & 7) * 8;
-      *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
-      *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
-      *reinterpret_cast<uint4 *>(sm + DOT + blk * 8192 + sw128(t, cc)) = ov;
+      cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
+      cp_async16(sm + DOT + blk * 8192 + sw128(t, cc), dOp + off, vld);
     }
+    cp_async_wait_all();
     __syncthreads();
     const unsigned long long m = P.mask[chunk * D + j];
     auto dO = [&](int t) {  // dO[t, j] from the tile
@@ -768,17 +764,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     wR[tid] = recf[OFF_VEC + V_WR + tid];
     gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
   }
-  for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16)
+  for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16), asynchronous
     const int t = e >> 4, chn = e & 15;
-    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
-    if (t < n) {
-      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
-      kv = *reinterpret_cast<const uint4 *>(k + off);
-      qv = *reinterpret_cast<const uint4 *>(q + off);
-    }
+    const bool vld = t < n;
+    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
     const int blk = chn >> 3, cc = (chn & 7) * 8;
-    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
-    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+    cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+    cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
   }
   const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
   const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
@@ -838,6 +830,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const uint32_t tm_lane = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
 
+  cp_async_wait_all();  // K, Q tile (published by the barriers below)
   if (!mbar_wait(K.barA, 0)) *K.flag = 1;  // phase_run below reports it to every thread
   stage_to_image(SA);
   stage_to_image(SB);

@@ -217,6 +217,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     __syncthreads();  // every thread is done with the previous chunk's tiles and vectors
 #pragma unroll
     for (int t = 0; t < 64; ++t) rres[t] = vval(t0, n, t);  // in flight during (a) and MMA1
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // K -> KT, Q -> B1's Q rows (raw)
+      const int t = e >> 4, ch = e & 15;
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+      const int blk = ch >> 3, cc = (ch & 7) * 8;
+      cp_async16(sm + SM_KT + blk * 8192 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc), q + off, vld);
+    }
 
     // ---- (a) chunk inputs -> shared memory
     if (p.S_chunks) {  // chunk-start states for the backward
@@ -242,15 +250,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
     }
     const float GamC = rec[OFF_VEC + V_GAMC];
+    cp_async_wait_all();
     __syncthreads();
-    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // K, Q: 64 rows x 16 chunks of 8
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // B1 = [Gprev K ; Gam scale Q]
       const int t = e >> 4, ch = e & 15;
-      uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
-      if (t < n) {
-        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8;
-        kv = *reinterpret_cast<const uint4 *>(k + off);
-        qv = *reinterpret_cast<const uint4 *>(q + off);
-      }
+      const int blk = ch >> 3, cc = (ch & 7) * 8;
+      const uint4 kv = *reinterpret_cast<const uint4 *>(sm + SM_KT + blk * 8192 + sw128(t, cc));
+      uint4 *qp = reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc));
+      const uint4 qv = *qp;
       const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
       const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(&qv);
       const float gk = Gprev[t], gq = Gam[t] * p.scale;
@@ -261,10 +268,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         kw[i] = pack_bf16(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
         qw[i] = pack_bf16(gq * __bfloat162float(qb[2 * i]), gq * __bfloat162float(qb[2 * i + 1]));
       }
-      const int blk = ch >> 3, cc = (ch & 7) * 8;
       *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(t, cc)) = ks;
-      *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc)) = qs;
-      *reinterpret_cast<uint4 *>(sm + SM_KT + blk * 8192 + sw128(t, cc)) = kv;
+      *qp = qs;
     }
 
     // ---- (b) MMA1: D1 = S^T B1^T

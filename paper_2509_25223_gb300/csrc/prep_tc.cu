@@ -98,17 +98,13 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     *flag = 0;
   }
   if (warp == 0) tmem_alloc(slot, 64);
-  for (int e = tid; e < 64 * 16; e += NTH) {  // K, Q (exact bf16), rows t
+  for (int e = tid; e < 64 * 16; e += NTH) {  // K, Q (exact bf16), rows t, asynchronous
     const int t = e >> 4, chn = e & 15;
-    uint4 kv = make_uint4(0, 0, 0, 0), qv = kv;
-    if (t < n) {
-      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8;
-      kv = *reinterpret_cast<const uint4 *>(k + off);
-      qv = *reinterpret_cast<const uint4 *>(q + off);
-    }
+    const bool vld = t < n;
+    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
     const int blk = chn >> 3, cc = (chn & 7) * 8;
-    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(t, cc)) = kv;
-    *reinterpret_cast<uint4 *>(sm + KQ + blk * 16384 + sw128(64 + t, cc)) = qv;
+    cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+    cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
   }
   if (tid < C) {
     const int t = tid;
@@ -123,6 +119,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     bet[t] = bv;
     gam[t] = mv;
   }
+  cp_async_wait_all();
   fence_async_smem();
   fence_before_sync();
   __syncthreads();

@@ -70,6 +70,18 @@ __device__ __forceinline__ void bulk_g2s(void *dst_smem, const void *src_gmem, u
       : "memory");
 }
 
+// 16-byte asynchronous copy global -> shared, zero-filled when !valid (the
+// source is then not read, but must still be a valid address).  Completes at
+// cp_async_wait_all() of the issuing thread; a barrier then publishes it.
+__device__ __forceinline__ void cp_async16(void *dst_smem, const void *src_gmem, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst_smem)),
+               "l"(src_gmem), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
 // Bulk copy shared -> global, tracked by this thread's bulk groups: issue,
 // then bulk_commit(); bulk_wait_read() returns once every committed copy has
 // finished reading shared memory, bulk_wait_all() once they are complete.
