@@ -168,21 +168,6 @@ __device__ __forceinline__ const uint8_t *rec_bytes(const FwdParams &p, size_t c
   return reinterpret_cast<const uint8_t *>(p.ws + chunk * kRecFloats);
 }
 
-// Per-row sums over the CTA's 128 columns of a vector v[64] (one value per
-// token t per thread): out[t] in shared memory.  `scratch` holds 4*64 floats.
-__device__ __forceinline__ void cta_row_sum(const float (&v)[64], float *scratch, float *out,
-                                            int tid) {
-  const int warp = tid >> 5, lane = tid & 31;
-  const int tb = transpose_reduce_tbase(lane);
-  float o2[2];
-  warp_transpose_reduce64(v, o2);
-  scratch[warp * 64 + tb] = o2[0];
-  scratch[warp * 64 + tb + 1] = o2[1];
-  __syncthreads();
-  if (tid < 64) out[tid] = scratch[tid] + scratch[64 + tid] + scratch[128 + tid] + scratch[192 + tid];
-  __syncthreads();
-}
-
 // ======================================================================== 1
 // bwd_recompute: the forward pieces of one chunk from its start states.
 namespace rc {
@@ -204,7 +189,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     return;
   }
   float *vec = reinterpret_cast<float *>(sm + VEC);
-  float *Gam = vec, *Gprev = vec + 64, *alpha = vec + 128, *gamv = vec + 320;
+  float *Gam = vec, *Gprev = vec + 64, *gamv = vec + 320;
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, j = tid;
   const size_t chunk = blockIdx.x;
@@ -226,7 +211,6 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   if (tid < 64) {
     Gam[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GAM + tid];
     Gprev[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GPREV + tid];
-    alpha[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_ALPHA + tid];
     gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
   }
   // chunk-start states -> bf16 A operands (row j = column j of [i][j])
@@ -244,24 +228,16 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     }
   }
   __syncthreads();
-  // B1 = diag(Gprev) K (64 rows)
+  // B1 = K (64 rows, exact bf16); the forward scan's arithmetic: unscaled
+  // read-outs, gates applied in fp32
   for (int e = tid; e < 64 * 16; e += NT) {
     const int t = e >> 4, ch = e & 15;
-    uint4 kv = make_uint4(0, 0, 0, 0);
-    if (t < n) {
-      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8;
-      kv = *reinterpret_cast<const uint4 *>(k + off);
-    }
-    const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
-    const float gk = Gprev[t];
-    uint4 ks;
-    uint32_t *kw = &ks.x;
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      kw[i] = pack2(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
-    const int blk = ch >> 3, cc = (ch & 7) * 8;
-    *reinterpret_cast<uint4 *>(sm + B1 + blk * 16384 + sw128(t, cc)) = ks;
+    const bool vld = t < n;
+    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+    cp_async16(sm + B1 + (ch >> 3) * 16384 + sw128(t, (ch & 7) * 8), k + off, vld);
   }
+  cp_async_wait_all();
+  fence_async_smem();
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
@@ -271,19 +247,23 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
   };
 
-  bool ok = phase_run(K, tid, [&] {  // Gprev KS, Gprev KR
+  bool ok = phase_run(K, tid, [&] {  // KS, KR
     mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
     mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
     return true;
   });
   float r[64];
-  if (ok) {  // X = V - alpha * (Gprev KS) -> E = T_beta X
+  if (ok) {  // X = V - Gam KS -> E = T_beta X; D1 <- Gprev KS (P accumulates onto it)
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
-      float x[16];
-      tmem_ld16(tm + lane + T_D1 + c0, x);
+      float ks[16], x[16];
+      tmem_ld16(tm + lane + T_D1 + c0, ks);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] = vval(c0 + i) - alpha[c0 + i] * x[i];
+      for (int i = 0; i < 16; ++i) {
+        x[i] = vval(c0 + i) - Gam[c0 + i] * ks[i];
+        ks[i] *= Gprev[c0 + i];
+      }
+      tmem_st16(tm + lane + T_D1 + c0, ks);
       put16s(sm + XE, sm + XE_LO, j, c0, x);
     }
     ok = phase_run(K, tid, [&] {
@@ -325,7 +305,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
         const float x = vval(t) - pp[i];
         if (fabsf(x) <= clip) m |= 1ull << t;
         r[t] = clampf(x, clip);
-        x2[i] = r[t] - alpha[t] * kr[i];
+        x2[i] = r[t] - Gam[t] * kr[i];
       }
       put16s(sm + XE, sm + XE_LO, j, c0, x2);
     }

@@ -5,33 +5,35 @@
 // transposed orientation so that every product has the value dimension
 // d_v = 128 as its M dimension: TMEM lane j holds value column j, and thread
 // j of the CTA's 128 threads owns that column end to end.  Per chunk of 64
-// tokens, with B1 = [diag(Gprev) K ; diag(Gam) Q] (128 x d_k, bf16):
+// tokens, with KQ = [K ; Q] (128 x d_k, exact bf16, unscaled):
 //
-//   MMA1  D1   = S^T  B1^T          -> [Gprev*KS | Gam*QS]        (N=128, K=128)
-//         X    = V - alpha * (Gprev*KS)                  (= V - Gam*KS)
+//   MMA1  D1   = S^T  KQ^T          -> [KS | QS], rescaled in TMEM to
+//                                      [Gprev*KS | Gam*scale*QS]  (N=128, K=128)
+//         X    = V - Gam*KS         (= V - alpha * Gprev*KS)
 //   MMA2  E^T  = X^T  T_beta^T                                    (N=64,  K=64)
 //   MMA3  D1  += E^T  [Ap ; Mq]^T   -> [P | Ob]                   (N=128, K=64)
 //   MMA4  U    = (wS E)^T K         -> S_C = Gam_C S + U          (N=128, K=64)
 //         r    = clip(V - P)        (Section 3.3; kept in registers)
-//   MMA5  D3   = R^T  B1^T          -> [Gprev*KR | Gam*QR]
-//         X2   = r - alpha * (Gprev*KR)
+//   MMA5  D3   = R^T  KQ^T          -> [KR | QR]
+//         X2   = r - Gam*KR
 //   MMA6  E2^T = X2^T T_gamma^T
 //   MMA7  D1[:, Ob half] += E2^T (diag(gamma) M2)^T
 //   MMA8  U2   = (wR E2)^T K        -> R_C = Gam_C R + U2 (two N=64 halves)
-//         o    = D1[:, Ob half] + gamma * (Gam*QR)   (= Ob + gamma * Oa)
+//         o    = D1[:, Ob half] + gamma * Gam*scale*QR   (= Ob + gamma * Oa)
 //
 // RLA skips MMA2 and MMA6 (E = V, E2 = r).  X, E, wS E and their auxiliary
 // counterparts (magnitude ~ |v|) enter the MMAs as bf16 hi + lo pairs, which
-// keeps their rounding well below the state's own scale; the other operands
-// (states, scaled K and Q, chunk matrices) are single bf16.  The states S, R live in TMEM in
-// fp32 for the whole sequence; their bf16 copies (the A operands of MMA1 and
-// MMA5) are rewritten in shared memory after each update.  One thread issues
-// the MMAs; every wait is an mbarrier wait with a time limit.  The
-// state-independent chunk matrices (T_beta, T_gamma, Ap, Mq, M2) come from
-// chunk_prep's records as bf16 hi + lo shared-memory images; they are streamed
-// into two slots by bulk copies one phase ahead of their use (slot A: T_beta
-// then T_gamma; slot B: [Ap;Mq] then M2) and enter the MMAs as three products
-// (hi*hi + hi*lo + lo*hi).
+// keeps their rounding well below the state's own scale; the states and the
+// chunk's K, Q are single bf16 (K, Q exactly).  The states S, R live in TMEM
+// in fp32 for the whole sequence; their bf16 copies (the A operands of MMA1
+// and MMA5) are rewritten in shared memory after each update.  The chunk's V
+// and [K ; Q] tiles are fetched by cp.async while the previous chunk
+// finishes.  One thread issues the MMAs; every wait is an mbarrier wait with
+// a time limit.  The state-independent chunk matrices (T_beta, T_gamma, Ap,
+// Mq, diag(gamma) M2) come from chunk_prep's records as bf16 hi + lo
+// shared-memory images; they are streamed into two slots by bulk copies one
+// phase ahead of their use (slot A: T_beta then T_gamma; slot B: [Ap;Mq] then
+// M2) and enter the MMAs as three products (hi*hi + hi*lo + lo*hi).
 //
 // TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) X
 // (X holds E, then U, then D3; D1 holds P|Ob, then E2 | Ob, then U2a | Ob + gamma M2 E2).
@@ -49,8 +51,9 @@ constexpr int kTcThreads = 128;
 // shared-memory carve-up (bytes from the 1024-aligned dynamic base)
 constexpr uint32_t SM_SA = 0;          // S^T bf16, 128 x 128, two 64-col blocks
 constexpr uint32_t SM_RA = 32768;      // R^T bf16
-constexpr uint32_t SM_B1 = 65536;      // [Gprev K ; Gam Q], 128 x 128
-constexpr uint32_t SM_KT = 98304;      // K, 64 (t) x 128 (d_k), unscaled: MN-major B operand
+constexpr uint32_t SM_KQ = 65536;      // [K ; Q] unscaled, 128 rows x 128, two 64-col blocks
+                                       // (K rows also serve as the MN-major B of the updates)
+constexpr uint32_t SM_V = 98304;       // V, 64 rows t x 128 columns j, two 8 KB blocks
 constexpr uint32_t SM_SLOTA = 114688;  // T_beta then T_gamma image (hi | lo), 16 KB
 constexpr uint32_t SM_SLOTB = 131072;  // [Ap;Mq] then M2 image (hi | lo), 32 KB
 // value-like operands are split into bf16 hi + lo parts (two MMAs each):
@@ -58,7 +61,7 @@ constexpr uint32_t SM_XE = 163840;     // X^T then E^T (X2^T then E2^T), hi part
 constexpr uint32_t SM_XE_LO = 180224;  //   lo part
 constexpr uint32_t SM_W = 196608;      // (wS E)^T / (wR E2)^T, hi part
 constexpr uint32_t SM_W_LO = 212992;   //   lo part
-constexpr uint32_t SM_VEC = 229376;    // 7 x 64 fp32: Gam Gprev alpha wS wR gamma, GamC
+constexpr uint32_t SM_VEC = 229376;    // 7 x 64 fp32: Gam Gprev (unused) wS wR gamma, GamC
 constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;  // 3 mbarriers: MMA, slot A, slot B
 constexpr uint32_t SM_SLOT = SM_BAR + 24;
 constexpr uint32_t SM_FLAG = SM_SLOT + 4;
@@ -125,7 +128,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return;
   }
   float *vec = reinterpret_cast<float *>(sm + SM_VEC);
-  float *Gam = vec, *Gprev = vec + 64, *alpha = vec + 128, *wS = vec + 192, *wR = vec + 256,
+  float *Gam = vec, *Gprev = vec + 64, *wS = vec + 192, *wR = vec + 256,
         *gamv = vec + 320;
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + SM_BAR);
   uint64_t *barA = bar + 1, *barB = bar + 2;  // slot A / slot B bulk copies
@@ -170,6 +173,35 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (RDNV) load_slot(sm + SM_SLOTA, barA, rec_of(0) + IMG_TB, 16384);
     load_slot(sm + SM_SLOTB, barB, rec_of(0) + IMG_APMQ, 32768);
   }
+  // chunk tiles (rows t, exact bf16, zero past the sequence end), asynchronous;
+  // the next chunk's are fetched while the current one finishes
+  auto fetch_v = [&](int c) {
+    const int t0 = c * 64, n = min(64, T - t0);
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {
+      const int t = e >> 4, ch = e & 15;
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+      cp_async16(sm + SM_V + (ch >> 3) * 8192 + sw128(t, (ch & 7) * 8), v + off, vld);
+    }
+  };
+  auto fetch_kq = [&](int c) {
+    const int t0 = c * 64, n = min(64, T - t0);
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {
+      const int t = e >> 4, ch = e & 15;
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+      const int blk = ch >> 3, cc = (ch & 7) * 8;
+      cp_async16(sm + SM_KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + SM_KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
+    }
+  };
+  // v[t, j] of the current chunk from its tile
+  auto vs = [&](int t) {
+    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
+        sm + SM_V + (j >> 6) * 8192 + sw128(t, j & 63)));
+  };
+  fetch_v(0);
+  fetch_kq(0);
 
   // initial states -> TMEM (fp32) and bf16 A operands
   for (int c0 = 0; c0 < D; c0 += 16) {
@@ -204,27 +236,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return *flag == 0;
   };
 
-  float rres[64];  // v[t] of column j, then (from step e) the clipped residual r[t]
-  // v[t, j] of the current chunk (0 beyond the sequence), read from L2/HBM
-  auto vval = [&](int t0, int n, int t) -> float {
-    return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
-  };
+  float rres[64];  // clipped residual r[t] of column j
   bool alive = true;
   for (int c = 0; c < NC && alive; ++c) {
     const int t0 = c * 64;
     const int n = min(64, T - t0);
     const float *rec = p.ws + ((size_t)bh * NC + c) * kRecFloats;
-    __syncthreads();  // every thread is done with the previous chunk's tiles and vectors
-#pragma unroll
-    for (int t = 0; t < 64; ++t) rres[t] = vval(t0, n, t);  // in flight during (a) and MMA1
-    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // K -> KT, Q -> B1's Q rows (raw)
-      const int t = e >> 4, ch = e & 15;
-      const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
-      const int blk = ch >> 3, cc = (ch & 7) * 8;
-      cp_async16(sm + SM_KT + blk * 8192 + sw128(t, cc), k + off, vld);
-      cp_async16(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc), q + off, vld);
-    }
+    cp_async_wait_all();  // this chunk's V, K, Q tiles (fetched during the previous chunk)
+    __syncthreads();      // every thread is done with the previous chunk's tiles and vectors
 
     // ---- (a) chunk inputs -> shared memory
     if (p.S_chunks) {  // chunk-start states for the backward
@@ -244,51 +263,42 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (tid < 64) {
       Gam[tid] = rec[OFF_VEC + V_GAM + tid];
       Gprev[tid] = rec[OFF_VEC + V_GPREV + tid];
-      alpha[tid] = rec[OFF_VEC + V_ALPHA + tid];
       wS[tid] = rec[OFF_VEC + V_WS + tid];
       wR[tid] = rec[OFF_VEC + V_WR + tid];
       gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
     }
     const float GamC = rec[OFF_VEC + V_GAMC];
-    cp_async_wait_all();
     __syncthreads();
-    for (int e = tid; e < 64 * 16; e += kTcThreads) {  // B1 = [Gprev K ; Gam scale Q]
-      const int t = e >> 4, ch = e & 15;
-      const int blk = ch >> 3, cc = (ch & 7) * 8;
-      const uint4 kv = *reinterpret_cast<const uint4 *>(sm + SM_KT + blk * 8192 + sw128(t, cc));
-      uint4 *qp = reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(64 + t, cc));
-      const uint4 qv = *qp;
-      const __nv_bfloat16 *kb = reinterpret_cast<const __nv_bfloat16 *>(&kv);
-      const __nv_bfloat16 *qb = reinterpret_cast<const __nv_bfloat16 *>(&qv);
-      const float gk = Gprev[t], gq = Gam[t] * p.scale;
-      uint4 ks, qs;
-      uint32_t *kw = &ks.x, *qw = &qs.x;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        kw[i] = pack_bf16(gk * __bfloat162float(kb[2 * i]), gk * __bfloat162float(kb[2 * i + 1]));
-        qw[i] = pack_bf16(gq * __bfloat162float(qb[2 * i]), gq * __bfloat162float(qb[2 * i + 1]));
-      }
-      *reinterpret_cast<uint4 *>(sm + SM_B1 + blk * 16384 + sw128(t, cc)) = ks;
-      *qp = qs;
-    }
 
-    // ---- (b) MMA1: D1 = S^T B1^T
+    // ---- (b) MMA1: D1 = S^T [K ; Q]^T  (unscaled read-outs K S | Q S)
     alive = run_phase([&] {
-      mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_B1, 16384, 8, idesc_bf16(128, 128),
+      mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
     });
     if (!alive) break;
-
-    // ---- (c) X = V - alpha * (Gprev KS)  ->  MMA2: E^T = X^T T_beta^T
-    if (RDNV) {
-      for (int c0 = 0; c0 < 64; c0 += 16) {
-        float x[16];
-        tmem_ld16(tm + lane + T_D1 + c0, x);
+    // the products below accumulate onto Gprev * KS (-> P) and Gam * scale * QS (-> Ob)
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float x[16];
+      tmem_ld16(tm + lane + T_D1 + 64 + c0, x);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - alpha[c0 + i] * x[i];
-        st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+      for (int i = 0; i < 16; ++i) x[i] *= Gam[c0 + i] * p.scale;
+      tmem_st16(tm + lane + T_D1 + 64 + c0, x);
+    }
+
+    // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T
+    for (int c0 = 0; c0 < 64; c0 += 16) {
+      float ks[16], x[16];
+      tmem_ld16(tm + lane + T_D1 + c0, ks);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        x[i] = vs(c0 + i) - Gam[c0 + i] * ks[i];
+        ks[i] *= Gprev[c0 + i];
       }
+      tmem_st16(tm + lane + T_D1 + c0, ks);
+      if (RDNV) st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+    }
+    if (RDNV) {
       alive = run_phase([&] {
         if (!mbar_wait(barA, phA)) return false;
         phA ^= 1u;
@@ -312,7 +322,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         }
       } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
+        for (int i = 0; i < 16; ++i) e[i] = vs(c0 + i);
       }
 #pragma unroll
       for (int i = 0; i < 16; ++i) w[i] = wS[c0 + i] * e[i];
@@ -324,8 +334,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       phB ^= 1u;
       mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 16384, idesc_bf16(128, 128), true);
-      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KT, 8192, 4, idesc_bf16(128, 128), false);
-      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT, 8192, 4, idesc_bf16(128, 128),
+      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
+                   false);
+      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
                    true);
       return true;
     });
@@ -340,7 +351,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       tmem_ld16(tm + lane + T_D1 + c0, pp);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float x = rres[c0 + i] - pp[i];
+        const float x = vs(c0 + i) - pp[i];
         if (fabsf(x) <= clip) msk |= 1ull << (c0 + i);
         rres[c0 + i] = clampf(x, clip);
       }
@@ -355,22 +366,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       tmem_st16(tm + lane + T_S + c0, s);
       st_row16(sm + SM_SA, 16384, j, c0, s);
     }
-    // MMA5: D3 = R^T B1^T (into X)
+    // MMA5: D3 = R^T [K ; Q]^T (into X; unscaled K R | Q R)
     alive = run_phase([&] {
-      mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_B1, 16384, 8, idesc_bf16(128, 128),
+      mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
     });
     if (!alive) break;
+    if (c + 1 < NC) fetch_v(c + 1);  // every thread is past its last read of V
 
-    // ---- (f) X2 = r - alpha * (Gprev KR);  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
+    // ---- (f) X2 = r - Gam KR;  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
     if (RDNV) {
 #pragma unroll
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float x[16];
         tmem_ld16(tm + lane + T_X + c0, x);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - alpha[c0 + i] * x[i];
+        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - Gam[c0 + i] * x[i];
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
       }
       alive = run_phase([&] {
@@ -410,14 +422,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       // the image is diag(gamma) M2: its product lands on Ob directly
       mma_split3(tm + T_D1 + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 8192, i64, true);
-      mma_tile_kmn(tm + T_D1, sbase + SM_W, 0, sbase + SM_KT, 8192, 4, i64, false);
-      mma_tile_kmn(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KT, 8192, 4, i64, true);
-      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KT + 8192, 8192, 4, i64, false);
-      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KT + 8192, 8192, 4, i64, true);
+      mma_tile_kmn(tm + T_D1, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, i64, false);
+      mma_tile_kmn(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, i64, true);
+      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ + 16384, 16384, 4, i64, false);
+      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KQ + 16384, 16384, 4, i64, true);
       return true;
     });
     if (!alive) break;
     if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTB, barB, rec_of(c + 1) + IMG_APMQ, 32768);
+    if (c + 1 < NC) fetch_kq(c + 1);  // K, Q are done with
 
     // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R = Gam_C R + U2
     for (int c0 = 0; c0 < 64; c0 += 16) {
@@ -429,7 +442,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         const int t = c0 + i;
         if (t < n)
           o[((size_t)(b * T + t0 + t) * H + h) * D + j] =
-              __float2bfloat16_rn(fmaf(gamv[t], oa[i], ob[i]));
+              __float2bfloat16_rn(fmaf(gamv[t] * Gam[t] * p.scale, oa[i], ob[i]));
       }
     }
     for (int c0 = 0; c0 < D; c0 += 16) {
