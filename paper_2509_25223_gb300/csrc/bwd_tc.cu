@@ -437,11 +437,55 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   }
   write_grad_tiles();
 
+  // a chunk's K, Q, dO tiles (rows t, exact bf16, zero past the end), asynchronous
+  auto fetch_kq = [&](int c) {
+    const int t0 = c * 64, n = min(64, T - t0);
+    for (int e = tid; e < 64 * 16; e += NT) {
+      const int t = e >> 4, chn = e & 15;
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
+      const int blk = chn >> 3, cc = (chn & 7) * 8;
+      cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
+    }
+  };
+  auto fetch_do = [&](int c) {
+    const int t0 = c * 64, n = min(64, T - t0);
+    for (int e = tid; e < 64 * 16; e += NT) {
+      const int t = e >> 4, chn = e & 15;
+      const bool vld = t < n;
+      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
+      cp_async16(sm + DOT + (chn >> 3) * 8192 + sw128(t, (chn & 7) * 8), dOp + off, vld);
+    }
+  };
+  // a chunk's gate vectors and clip-mask word, into registers
+  struct Pre {
+    float gam_, gprev, ws_, wr_, g_, gamc;
+    unsigned long long m;
+  };
+  auto fetch_pre = [&](int c) {
+    const size_t ck = (size_t)bh * NC + c;
+    const int t0 = c * 64, n = min(64, T - t0);
+    const float *rf = p.ws + ck * kRecFloats;
+    Pre x;
+    const int t = tid & 63;
+    x.gam_ = rf[OFF_VEC + V_GAM + t];
+    x.gprev = rf[OFF_VEC + V_GPREV + t];
+    x.ws_ = rf[OFF_VEC + V_WS + t];
+    x.wr_ = rf[OFF_VEC + V_WR + t];
+    x.g_ = t < n ? p.gamma[(size_t)(b * T + t0 + t) * H + h] : 0.f;
+    x.gamc = rf[OFF_VEC + V_GAMC];
+    x.m = P.mask[ck * D + j];
+    return x;
+  };
+  fetch_kq(NC - 1);
+  fetch_do(NC - 1);
+  Pre pre = fetch_pre(NC - 1);
+
   bool ok = true;
   for (int c = NC - 1; c >= 0 && ok; --c) {
     const size_t chunk = (size_t)bh * NC + c;
     const int t0 = c * 64, n = min(64, T - t0);
-    const float *recf = p.ws + chunk * kRecFloats;
     __syncthreads();
     if (tid == 0) {  // gradients w.r.t. this chunk's end states, for bwd_post: the tile images
       static_assert(DRH == DSH + 32768 && DSL == DRH + 32768 && DRL == DSL + 32768, "contiguous");
@@ -449,25 +493,16 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       bulk_commit();
     }
     if (tid < 64) {
-      Gam[tid] = recf[OFF_VEC + V_GAM + tid];
-      Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
-      wS[tid] = recf[OFF_VEC + V_WS + tid];
-      wR[tid] = recf[OFF_VEC + V_WR + tid];
-      gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+      Gam[tid] = pre.gam_;
+      Gprev[tid] = pre.gprev;
+      wS[tid] = pre.ws_;
+      wR[tid] = pre.wr_;
+      gamv[tid] = pre.g_;
     }
-    const float GamC = recf[OFF_VEC + V_GAMC];
-    for (int e = tid; e < 64 * 16; e += NT) {  // K, Q, dO (exact bf16), rows t, asynchronous
-      const int t = e >> 4, chn = e & 15;
-      const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
-      const int blk = chn >> 3, cc = (chn & 7) * 8;
-      cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
-      cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
-      cp_async16(sm + DOT + blk * 8192 + sw128(t, cc), dOp + off, vld);
-    }
-    cp_async_wait_all();
+    const float GamC = pre.gamc;
+    const unsigned long long m = pre.m;
+    cp_async_wait_all();  // this chunk's tiles (fetched during the previous one)
     __syncthreads();
-    const unsigned long long m = P.mask[chunk * D + j];
     auto dO = [&](int t) {  // dO[t, j] from the tile
       return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
           sm + DOT + (j >> 6) * 8192 + sw128(t, j & 63)));
@@ -591,6 +626,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     });
     if (!ok) break;
     if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
+    if (c > 0) fetch_do(c - 1);  // every thread is past its last read of this chunk's dO
     {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX
       float *gx = P.dXbuf + chunk * 64 * D;
 #pragma unroll
@@ -616,6 +652,10 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       return true;
     });
     if (!ok) break;
+    if (c > 0) {  // the next chunk's inputs, while this one finishes
+      fetch_kq(c - 1);
+      pre = fetch_pre(c - 1);
+    }
     for (int c0 = 0; c0 < D; c0 += 16) {  // dS update
       float s[16], u[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
