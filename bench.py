@@ -308,8 +308,11 @@ def _traffic(kernel):
         if not ent:
             return None
         import hashlib
-        src = os.path.join(ROOT, ent["source"])
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        srcs = ent["source"] if isinstance(ent["source"], list) else [ent["source"]]
+        hs = hashlib.sha256()
+        for sname in srcs:
+            hs.update(open(os.path.join(ROOT, sname), "rb").read())
+        h = hs.hexdigest()[:16]
         if h != ent["source_sha256_16"]:
             return None
         return float(ent["bytes_per_launch_full_workload"])
