@@ -57,7 +57,7 @@ struct TcBwdParams {
   void *dv;
   float *dS0, *dR0;
   float *acc;            // per-chunk records
-  float *Ebuf, *E2buf;   // [B*H*NC][64][128] fp32 (t, j)
+  uint8_t *Ebuf, *E2buf; // [B*H*NC][32 KB]: images of E^T, E2^T (rows j, columns t; hi | lo)
   float *dX2buf, *dXbuf; // [B*H*NC][64][128]
   uint8_t *gimg;         // [B*H*NC][128 KB]: gradients w.r.t. each chunk's end states as
                          // bf16 images (rows j): dS hi | dR hi | dS lo | dR lo, 32 KB each
@@ -112,7 +112,7 @@ __device__ __forceinline__ void mma_s3_kk(uint32_t d, uint32_t a_hi, uint32_t a_
 
 // Common per-CTA machinery: mbarriers (MMA, slot A, slot B), TMEM, phases.
 struct Ctl {
-  uint64_t *bar, *barA, *barB;
+  uint64_t *bar, *barA, *barB, *barC;
   volatile int *flag;
   uint32_t phase, phA, phB;
 };
@@ -121,12 +121,14 @@ __device__ __forceinline__ void ctl_init(Ctl &k, uint8_t *base, int tid) {
   k.bar = reinterpret_cast<uint64_t *>(base);
   k.barA = k.bar + 1;
   k.barB = k.bar + 2;
-  k.flag = reinterpret_cast<volatile int *>(base + 28);
+  k.barC = k.bar + 3;
+  k.flag = reinterpret_cast<volatile int *>(base + 32);
   k.phase = k.phA = k.phB = 0;
   if (tid == 0) {
     mbar_init(k.bar, 1);
     mbar_init(k.barA, 1);
     mbar_init(k.barB, 1);
+    mbar_init(k.barC, 1);
     fence_mbar_init();
     *k.flag = 0;
   }
@@ -174,7 +176,7 @@ namespace rc {
 constexpr uint32_t SA = 0, RA = 32768, B1 = 65536, SLOTA = 98304, SLOTB = 114688;
 constexpr uint32_t XE = 147456, XE_LO = 163840, VEC = 180224;
 constexpr uint32_t CTL = VEC + 7 * 64 * 4;
-constexpr uint32_t SLOT = CTL + 32;
+constexpr uint32_t SLOT = CTL + 48;
 constexpr size_t SMEM = SLOT + 16;
 constexpr uint32_t T_D1 = 0, T_D3 = 128, T_X = 256;
 }  // namespace rc
@@ -275,19 +277,20 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   }
   if (ok) {
     if (tid == 0) load_slot(sm + SLOTA, K.barA, rec + IMG_TG, 16384);
-    float *Eg = P.Ebuf + chunk * 64 * D;
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float e[16];
       tmem_ld16(tm + lane + T_X + c0, e);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) Eg[(c0 + i) * D + j] = e[i];
       put16s(sm + XE, sm + XE_LO, j, c0, e);
     }
     ok = phase_run(K, tid, [&] {  // D1 += E Ap^T -> P (the Ap rows of the [Ap ; Mq] image)
       if (!slot_wait(K.barB, K.phB)) return false;
       mma_s3_kk(tm + T_D1, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 16384,
                  idesc_bf16(128, 64), true);
+      static_assert(XE_LO == XE + 16384, "contiguous");
+      bulk_s2g(P.Ebuf + chunk * 32768, sm + XE, 32768);  // the E^T image, for bwd_post
+      bulk_commit();
+      bulk_wait_read();
       return true;
     });
   }
@@ -317,18 +320,24 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       return true;
     });
   }
-  if (ok) {
-    float *E2g = P.E2buf + chunk * 64 * D;
+  if (ok) {  // the E2^T image, for bwd_post
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float e[16];
       tmem_ld16(tm + lane + T_X + c0, e);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) E2g[(c0 + i) * D + j] = e[i];
+      put16s(sm + XE, sm + XE_LO, j, c0, e);
+    }
+    fence_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      bulk_s2g(P.E2buf + chunk * 32768, sm + XE, 32768);
+      bulk_commit();
+      bulk_wait_all();
     }
   } else if (tid == 0 && p.err) {
     atomicExch(p.err, RDN_ERR_TIMEOUT);
   }
+  if (tid == 0) bulk_wait_all();
   fence_before_sync();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, 512);
@@ -350,7 +359,7 @@ constexpr uint32_t S0H = 32768, S0L = 49152, S1H = 65536, S1L = 81920;
 constexpr uint32_t S2H = 98304, S2L = 114688, S3H = 131072, S3L = 147456;
 constexpr uint32_t VEC = 212992;                 // Gam Gprev wS wR gamma (5 x 64)
 constexpr uint32_t CTL = VEC + 5 * 64 * 4;
-constexpr uint32_t SLOT = CTL + 32;
+constexpr uint32_t SLOT = CTL + 48;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
 constexpr uint32_t T_DS = 0, T_DR = 128, T_R1 = 256, T_R2 = 320, T_R3 = 384, T_R4 = 448;
@@ -710,7 +719,7 @@ constexpr uint32_t KQ = 196608;         // K rows 0..63, Q rows 64..127, 2 x 16 
 constexpr uint32_t VEC = 229376;        // Gam Gprev wS wR gamma dGam dGprev (7 x 64), dGamC
 constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // 8 warps x 32 floats
 constexpr uint32_t CTL = RED + 8 * 32 * 4;
-constexpr uint32_t SLOT = CTL + 32;
+constexpr uint32_t SLOT = CTL + 48;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
 // element-wise pass: fp32 C x C tiles (row stride 65) over the state images
@@ -720,7 +729,7 @@ constexpr int F_DM2 = 0, F_DMQ = TILE, F_DAB = 2 * TILE, F_KK = 3 * TILE, F_DAG 
 static_assert((F_VEC + 9 * 64 + 6 * 4 * 64) * 4 <= (int)XH, "finish scratch");
 // TMEM columns
 constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
-constexpr uint32_t T_KDR = 0, T_KDS = 64;                        // P4, after the read-outs
+constexpr uint32_t T_KDR = 0, T_KDS = 64, T_U1 = 128, T_U2 = 192;  // P4, after the read-outs
 constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
 }  // namespace po
 
@@ -792,7 +801,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
     cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
   }
-  const float *Eg = P.Ebuf + chunk * 64 * D, *E2g = P.E2buf + chunk * 64 * D;
   const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
   const unsigned long long m = P.mask[chunk * D + j] >> tb;
   // this thread's tokens of dX2, dX, dO
@@ -944,10 +952,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       return true;
     });
   }
-  if (ok && tid == 0) {  // and dS's image into S0's
+  if (ok && tid == 0) {  // and dS's image into S0's; the E2^T, E^T images into the pair's
     mbar_expect_tx(K.barA, 65536);
     bulk_g2s(sm + SA, gimg, 32768, K.barA);
     bulk_g2s(sm + SA + 32768, gimg + 65536, 32768, K.barA);
+    mbar_expect_tx(K.barC, 65536);
+    bulk_g2s(sm + XH, P.E2buf + chunk * 32768, 32768, K.barC);  // hi at XH, lo at XL
+    bulk_g2s(sm + YH, P.Ebuf + chunk * 32768, 32768, K.barC);   // hi at YH, lo at YL
   }
   if (ok) {  // <dR, R0> + <dS, S0> (states re-read from L2), reduced into dGamC
     float gdot;
@@ -973,29 +984,29 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
     ok = *K.flag == 0;
   }
-  float e2v[32], ev[32];  // this thread's tokens of E2, E
+  // this thread's 32 tokens of row j of a (hi | lo) image of a [j][t] matrix
+  auto image_row = [&](uint32_t base, float (&out)[32]) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    e2v[i] = E2g[(tb + i) * D + j];
-    ev[i] = Eg[(tb + i) * D + j];
-  }
-  if (ok) {  // ---- P4: dK += dR (diag(wR) E2)^T + dS (diag(wS) E)^T ; K dR, K dS read-outs
-    float x[32], y[32];
+    for (int k8 = 0; k8 < 4; ++k8) {
+      const int c8 = (tb >> 3) + k8;
+      const uint32_t o = base + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
+      const uint4 hv = *reinterpret_cast<const uint4 *>(sm + o);
+      const uint4 lv = *reinterpret_cast<const uint4 *>(sm + o + 16384);
+      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
+      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int t = tb + i;
-      x[i] = wR[t] * e2v[i];
-      y[i] = wS[t] * ev[i];
+      for (int e = 0; e < 8; ++e) out[k8 * 8 + e] = __bfloat162float(hb[e]) + __bfloat162float(lb[e]);
     }
-    put_tok(x, XH, XL);
-    put_tok(y, YH, YL);
+  };
+  if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs
+    if (!mbar_wait(K.barC, 0)) *K.flag = 1;  // the E images, for every thread
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XH, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YH, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_U1, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_U2, sb + SA, 16384, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_U2, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_U2, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
       // (K dR)^T, (K dS)^T (lanes j, columns t; K exact)
       mma_tile(tm + T_KDR, sb + SB, 16384, sb + KQ, 16384, 8, i64, false);
       mma_tile(tm + T_KDR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i64, true);
@@ -1004,15 +1015,31 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       return true;
     });
   }
-  if (ok) {  // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
+  if (ok) {
+    // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 16) {
+      float a[16], u1[16], u2[16];
+      tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);
+      tmem_ld16(tm + tm_lane + T_U1 + tb + c0, u1);
+      tmem_ld16(tm + tm_lane + T_U2 + tb + c0, u2);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int t = tb + c0 + i;
+        a[i] = fmaf(wR[t], u1[i], fmaf(wS[t], u2[i], a[i]));
+      }
+      tmem_st16(tm + tm_lane + T_DKQ + tb + c0, a);
+    }
+    // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
     for (int w = 0; w < 2; ++w) {
-      float rv[32];
+      float ev[32], rv[32];
+      image_row(w == 0 ? XH : YH, ev);
 #pragma unroll
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float kd[16];
         tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb + c0, kd);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) rv[c0 + i] = kd[i] * (w == 0 ? e2v[c0 + i] : ev[c0 + i]);
+        for (int i = 0; i < 16; ++i) rv[c0 + i] = kd[i] * ev[c0 + i];
       }
       // parked in the record's slots (shared memory is full); read in the gate pass
       cta_row_sum256(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
@@ -1021,21 +1048,20 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
   //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
   //   and the Gram matrices [K ; Q] K^T
-  // images: E2 at SA (hi | lo), E at SA + 32 KB, dX at SB; the pair at X / Y
+  // images: E2 at XH (hi | lo), E at YH (hi | lo); dX at SB; the pairs at SA
+  // (X atom hi SA, lo SA + 16 KB; Y atom hi SA + 32 KB, lo SA + 48 KB)
   if (ok) {
-    put_tok(e2v, SA, SA + 16384);
-    put_tok(ev, SA + 32768, SA + 49152);
     put_tok(xv, SB, SB + 16384);
-    put_tok(dov, XH, XL);  // [dO ; dX2]: gamma_t enters in the element-wise pass
-    put_tok(x2v, YH, YL);
+    put_tok(dov, SA, SA + 16384);  // [dO ; dX2]: gamma_t enters in the element-wise pass
+    put_tok(x2v, SA + 32768, SA + 49152);
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_G1, sb + XH, 32768, sb + SA, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G1, sb + XH, 32768, sb + SA + 16384, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G1, sb + XL, 32768, sb + SA, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G1, sb + SA, 32768, sb + XH, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G1, sb + SA, 32768, sb + XL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G1, sb + SA + 16384, 32768, sb + XH, 16384, 8, i64, true);
       // the second M atom of [dX ; -] is any valid tile: lanes 64..127 are unused
-      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + SA + 32768, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + SA + 49152, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G3, sb + SB + 16384, 32768, sb + SA + 32768, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G3, sb + SB + 16384, 32768, sb + YH, 16384, 8, i64, true);
       mma_tile(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
       return true;
     });
@@ -1044,12 +1070,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     float y[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) y[i] = dp_of(i);
-    put_tok(dov, XH, XL);
-    put_tok(y, YH, YL);
+    put_tok(y, SA + 32768, SA + 49152);  // [dO ; dP]: the dO atom is still in place
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_G2, sb + XH, 32768, sb + SA + 32768, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G2, sb + XH, 32768, sb + SA + 49152, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G2, sb + XL, 32768, sb + SA + 32768, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G2, sb + SA, 32768, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn(tm + T_G2, sb + SA, 32768, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn(tm + T_G2, sb + SA + 16384, 32768, sb + YH, 16384, 8, i64, true);
       return true;
     });
   }
@@ -1325,8 +1350,8 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.acc = acc;
   const size_t nct = (size_t)f.B * f.H * f.NC;
   float *x = reinterpret_cast<float *>(extra);
-  P.Ebuf = x;
-  P.E2buf = x + nct * 64 * D;
+  P.Ebuf = reinterpret_cast<uint8_t *>(x);
+  P.E2buf = reinterpret_cast<uint8_t *>(x + nct * 64 * D);
   P.dX2buf = x + 2 * nct * 64 * D;
   P.dXbuf = x + 3 * nct * 64 * D;
   P.gimg = reinterpret_cast<uint8_t *>(x + 4 * nct * 64 * D);

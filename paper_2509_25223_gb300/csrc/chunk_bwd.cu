@@ -775,8 +775,8 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   p.f.err = (int *)(ws + l.total - 256);
   if (reuse && (f.flags & RDN_FLAG_SAVE_FOR_BWD)) {  // E, E2 and the mask kept by the forward
     const SavedLayout sl = saved_layout((size_t)f.B * f.H * ((f.T + C - 1) / C), f.Dv);
-    p.f.sv_E = (float *)((char *)f.workspace + sl.e);
-    p.f.sv_E2 = (float *)((char *)f.workspace + sl.e2);
+    p.f.sv_E = (uint8_t *)f.workspace + sl.e;
+    p.f.sv_E2 = (uint8_t *)f.workspace + sl.e2;
     p.f.sv_mask = (unsigned long long *)((char *)f.workspace + sl.mask);
   }
   p.f.ST = p.f.RT = nullptr;

@@ -113,8 +113,10 @@ struct FwdParams {
   float *ws;  // NC*B*H records of kRecFloats
   int *err;   // device status word (RDN_ERR_TIMEOUT if a bounded wait gave up) or NULL
   // forward intermediates kept for the backward (RDN_FLAG_SAVE_FOR_BWD) or NULL:
-  // E, E2 as [chunk][t][j] fp32, the clip mask as [chunk][j] (bit t = |x| <= c)
-  float *sv_E, *sv_E2;
+  // E, E2 per chunk as a 32 KB shared-memory image of E^T (rows j, columns t;
+  // bf16 hi 16 KB | lo 16 KB, K-major, 128-byte swizzled), the clip mask as
+  // [chunk][j] (bit t = |x| <= c)
+  uint8_t *sv_E, *sv_E2;
   unsigned long long *sv_mask;
 };
 

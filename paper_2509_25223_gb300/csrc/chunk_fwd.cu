@@ -488,8 +488,8 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   p.err = (int *)((char *)a.workspace + plan_fwd(a, variant).total_bytes - 256);
   if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) {
     const SavedLayout l = saved_layout((size_t)a.B * a.H * p.NC, a.Dv);
-    p.sv_E = (float *)((char *)a.workspace + l.e);
-    p.sv_E2 = (float *)((char *)a.workspace + l.e2);
+    p.sv_E = (uint8_t *)a.workspace + l.e;
+    p.sv_E2 = (uint8_t *)a.workspace + l.e2;
     p.sv_mask = (unsigned long long *)((char *)a.workspace + l.mask);
   }
   return launch_fwd_parts(p, a.Dk, variant == 1, a.dtype == RDN_BF16, true, true, s);

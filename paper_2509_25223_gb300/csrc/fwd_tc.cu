@@ -272,6 +272,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (b) MMA1: D1 = S^T [K ; Q]^T  (unscaled read-outs K S | Q S)
     alive = run_phase([&] {
+      if (p.sv_E2) bulk_wait_read();  // the E2^T tiles of the previous chunk are rewritten next
       mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
@@ -316,10 +317,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_X + c0, e);
-        if (p.sv_E) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) p.sv_E[(ci * 64 + c0 + i) * D + j] = e[i];
-        }
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = vs(c0 + i);
@@ -334,6 +331,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       phB ^= 1u;
       mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 16384, idesc_bf16(128, 128), true);
+      if (p.sv_E) {  // keep the E^T image (hi | lo) for the backward
+        static_assert(SM_XE_LO == SM_XE + 16384, "contiguous");
+        bulk_s2g(p.sv_E + ci * 32768, sm + SM_XE, 32768);
+        bulk_commit();
+      }
       mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
                    false);
       mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
@@ -368,6 +370,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
     // MMA5: D3 = R^T [K ; Q]^T (into X; unscaled K R | Q R)
     alive = run_phase([&] {
+      if (p.sv_E) bulk_wait_read();  // the E^T tiles are rewritten next
       mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
@@ -402,10 +405,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_D1 + c0, e);
-        if (p.sv_E2) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) p.sv_E2[(ci * 64 + c0 + i) * D + j] = e[i];
-        }
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
@@ -422,6 +421,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       // the image is diag(gamma) M2: its product lands on Ob directly
       mma_split3(tm + T_D1 + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 8192, i64, true);
+      if (p.sv_E2) {  // and the E2^T image
+        bulk_s2g(p.sv_E2 + ci * 32768, sm + SM_XE, 32768);
+        bulk_commit();
+      }
       mma_tile_kmn(tm + T_D1, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, i64, false);
       mma_tile_kmn(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, i64, true);
       mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ + 16384, 16384, 4, i64, false);
@@ -456,6 +459,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
   }
 
+  if (tid == 0 && p.sv_E) bulk_wait_all();
   if (alive) {  // final states
     for (int c0 = 0; c0 < D; c0 += 16) {
       float s[16], r[16];
