@@ -781,17 +781,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   ctl_init(K, sm + CTL, tid);
   if (warp == 0) tmem_alloc(slot, 512);
   __syncthreads();  // barriers initialised
-  if (tid == 0) {   // chunk-start states, fp32, staged where their images go
+  if (tid == 0) {  // chunk-start states, fp32, staged where their images go; dX2, dX
+                   // (fp32 [t][j]) staged in the pair's place until P2
     mbar_expect_tx(K.barA, 131072);
     bulk_g2s(sm + SA, S0, 65536, K.barA);
     bulk_g2s(sm + SB, R0, 65536, K.barA);
-  }
-  if (tid < 64) {
-    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
-    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
-    wS[tid] = recf[OFF_VEC + V_WS + tid];
-    wR[tid] = recf[OFF_VEC + V_WR + tid];
-    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    mbar_expect_tx(K.barC, 65536);
+    bulk_g2s(sm + XH, P.dX2buf + chunk * 64 * D, 32768, K.barC);
+    bulk_g2s(sm + YH, P.dXbuf + chunk * 64 * D, 32768, K.barC);
   }
   for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16), asynchronous
     const int t = e >> 4, chn = e & 15;
@@ -801,16 +798,30 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
     cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
   }
-  const float *X2g = P.dX2buf + chunk * 64 * D, *Xg = P.dXbuf + chunk * 64 * D;
   const unsigned long long m = P.mask[chunk * D + j] >> tb;
-  // this thread's tokens of dX2, dX, dO
+  // this thread's tokens of dX2, dX (from the staging, below) and dO
   float x2v[32], xv[32], dov[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
     const int t = tb + i;
-    x2v[i] = X2g[t * D + j];
-    xv[i] = Xg[t * D + j];
     dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  }
+  if (tid < 64) {
+    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
+    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
+    wS[tid] = recf[OFF_VEC + V_WS + tid];
+    wR[tid] = recf[OFF_VEC + V_WR + tid];
+    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+  }
+  if (!mbar_wait(K.barC, 0)) *K.flag = 1;
+  {
+    const float *x2s = reinterpret_cast<const float *>(sm + XH);
+    const float *xs = reinterpret_cast<const float *>(sm + YH);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      x2v[i] = x2s[(tb + i) * D + j];
+      xv[i] = xs[(tb + i) * D + j];
+    }
   }
   // fp32 [i][j] state staged at `base` -> rows j of its (hi | lo) image at
   // `base`, key rows of half hf (every thread reads its values before any writes)
@@ -999,7 +1010,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
   };
   if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs
-    if (!mbar_wait(K.barC, 0)) *K.flag = 1;  // the E images, for every thread
+    if (!mbar_wait(K.barC, 1)) *K.flag = 1;  // the E images, for every thread
     ok = phase_run(K, tid, [&] {
       mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
       mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
