@@ -416,6 +416,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   const uint32_t lane = (uint32_t)(warp * 32) << 16;
   // carried gradients (bf16 hi + lo tiles, rows j) from their fp32 TMEM copy
   auto write_grad_tiles = [&]() {
+#pragma unroll 1
     for (int c0 = 0; c0 < D; c0 += 16) {
       float s[16], r[16], sh[16], sl[16], rh[16], rl[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
@@ -601,6 +602,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     if (!ok) break;
     if (tid == 0 && c > 0) load_mq(chunk - 1);
     {  // dR update (fp32 in TMEM); dE = dE_partial + Ap^T dP; dQS = Gam dO
+#pragma unroll 1
       for (int c0 = 0; c0 < D; c0 += 16) {
         float r[16], u[16];
         tmem_ld16(tm + lane + T_DR + c0, r);
@@ -665,6 +667,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       fetch_kq(c - 1);
       pre = fetch_pre(c - 1);
     }
+#pragma unroll 1
     for (int c0 = 0; c0 < D; c0 += 16) {  // dS update
       float s[16], u[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
@@ -890,10 +893,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
   bool ok = phase_run(K, tid, [&] {
     const uint32_t t_ = *slot;
-    mma_tile(t_ + T_KS, sb + SA, 16384, sb + KQ, 16384, 8, i128, false);
-    mma_tile(t_ + T_KS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i128, true);
-    mma_tile(t_ + T_KR, sb + SB, 16384, sb + KQ, 16384, 8, i128, false);
-    mma_tile(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
+    mma_tile<true>(t_ + T_KS, sb + SA, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile<true>(t_ + T_KS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i128, true);
+    mma_tile<true>(t_ + T_KR, sb + SB, 16384, sb + KQ, 16384, 8, i128, false);
+    mma_tile<true>(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
     return true;
   });
   const uint32_t tm = *slot;
@@ -949,9 +952,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XH, 32768, 8, i128, false);
-      mma_tile_mnmn(tm + T_DKQ, sb + SB, 16384, sb + XL, 32768, 8, i128, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SB, 16384, sb + XH, 32768, 8, i128, false);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SB, 16384, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SB + 32768, 16384, sb + XH, 32768, 8, i128, true);
       return true;
     });
   }
@@ -971,9 +974,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + XH, 32768, 8, i128, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SA, 16384, sb + XL, 32768, 8, i128, true);
-      mma_tile_mnmn(tm + T_DKQ, sb + SA + 32768, 16384, sb + XH, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SA, 16384, sb + XH, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SA, 16384, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_DKQ, sb + SA + 32768, 16384, sb + XH, 32768, 8, i128, true);
       return true;
     });
   }
@@ -1006,23 +1009,23 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs
     if (!mbar_wait(K.barC, 1)) *K.flag = 1;  // the E images, for every thread
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_U1, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_U2, sb + SA, 16384, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_U2, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_U2, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_U1, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_U2, sb + SA, 16384, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_U2, sb + SA, 16384, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_U2, sb + SA + 32768, 16384, sb + YH, 16384, 8, i64, true);
       // (K dR)^T, (K dS)^T (lanes j, columns t; K exact)
-      mma_tile(tm + T_KDR, sb + SB, 16384, sb + KQ, 16384, 8, i64, false);
-      mma_tile(tm + T_KDR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i64, true);
-      mma_tile(tm + T_KDS, sb + SA, 16384, sb + KQ, 16384, 8, i64, false);
-      mma_tile(tm + T_KDS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i64, true);
+      mma_tile<true>(tm + T_KDR, sb + SB, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile<true>(tm + T_KDR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i64, true);
+      mma_tile<true>(tm + T_KDS, sb + SA, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile<true>(tm + T_KDS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i64, true);
       return true;
     });
   }
   if (ok) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
-#pragma unroll
+#pragma unroll 1
     for (int c0 = 0; c0 < 32; c0 += 16) {
       float a[16], u1[16], u2[16];
       tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);
@@ -1060,14 +1063,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     put_tok(dov, SA, SA + 16384);  // [dO ; dX2]: gamma_t enters in the element-wise pass
     put_tok(x2v, SA + 32768, SA + 49152);
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_G1, sb + SA, 32768, sb + XH, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G1, sb + SA, 32768, sb + XL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G1, sb + SA + 16384, 32768, sb + XH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G1, sb + SA + 16384, 32768, sb + XH, 16384, 8, i64, true);
       // the second M atom of [dX ; -] is any valid tile: lanes 64..127 are unused
-      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G3, sb + SB, 32768, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G3, sb + SB + 16384, 32768, sb + YH, 16384, 8, i64, true);
-      mma_tile(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_G3, sb + SB, 32768, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_G3, sb + SB, 32768, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G3, sb + SB + 16384, 32768, sb + YH, 16384, 8, i64, true);
+      mma_tile<true>(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
       return true;
     });
   }
@@ -1077,9 +1080,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     for (int i = 0; i < 32; ++i) y[i] = dp_of(i);
     put_tok(y, SA + 32768, SA + 49152);  // [dO ; dP]: the dO atom is still in place
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn(tm + T_G2, sb + SA, 32768, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn(tm + T_G2, sb + SA, 32768, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn(tm + T_G2, sb + SA + 16384, 32768, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 32768, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 32768, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA + 16384, 32768, sb + YH, 16384, 8, i64, true);
       return true;
     });
   }
@@ -1092,7 +1095,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   if (ok) {
     {
       const int r = j & 63;
-#pragma unroll
+#pragma unroll 1
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float g1[16], g2[16], g3[16], gr[16];
         tmem_ld16(tm + tm_lane + T_G1 + tb + c0, g1);
@@ -1151,7 +1154,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const float ct = cum[t], cpt = cprev[t];
       const float gt = gam[t];
       float rowc = 0.f, rowp = 0.f, dgo = 0.f;
-#pragma unroll 4
+#pragma unroll 1
       for (int ii = 0; ii < 16; ++ii) {
         const int i = 16 * q4 + ii, e = t * LDC + i;
         float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
@@ -1211,7 +1214,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {  // column pass: thread (i, quarter) over t in [16 q, 16 q + 16)
       const int i = tid & 63, q4 = tid >> 6;
       float sg = 0.f, sbv = 0.f, smv = 0.f;
-#pragma unroll 4
+#pragma unroll 1
       for (int tt = 0; tt < 16; ++tt) {
         const int e = (16 * q4 + tt) * LDC + i;
         sg += F[F_DM2 + e];
@@ -1282,10 +1285,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
     // ---- P7: dK, dQ += K^T [dKK + dKK^T ; dQK]^T ; D2 = Q^T dQK
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnk(tm + T_DKQ, sb + KQ, 16384, sb + XH, 4, i128, true);
-      mma_tile_mnk(tm + T_DKQ, sb + KQ, 16384, sb + XL, 4, i128, true);
-      mma_tile_mnmn(tm + T_D2, sb + KQ + 8192, 16384, sb + XH + 8192, 16384, 4, i64, false);
-      mma_tile_mnmn(tm + T_D2, sb + KQ + 8192, 16384, sb + XL + 8192, 16384, 4, i64, true);
+      mma_tile_mnk<true>(tm + T_DKQ, sb + KQ, 16384, sb + XH, 4, i128, true);
+      mma_tile_mnk<true>(tm + T_DKQ, sb + KQ, 16384, sb + XL, 4, i128, true);
+      mma_tile_mnmn<true>(tm + T_D2, sb + KQ + 8192, 16384, sb + XH + 8192, 16384, 4, i64, false);
+      mma_tile_mnmn<true>(tm + T_D2, sb + KQ + 8192, 16384, sb + XL + 8192, 16384, 4, i64, true);
       return true;
     });
   }
@@ -1297,7 +1300,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       P.dgamma[off] = dgam[tid];
     }
     __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
-#pragma unroll
+#pragma unroll 1
     for (int c0 = 0; c0 < 32; c0 += 16) {
       float a[16], d2[16], qv[16];
       tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);

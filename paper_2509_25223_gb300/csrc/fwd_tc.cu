@@ -249,6 +249,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (p.S_chunks) {  // chunk-start states for the backward
       float *sc = p.S_chunks + ((size_t)bh * NC + c) * D * D;
       float *rc = p.R_chunks + ((size_t)bh * NC + c) * D * D;
+#pragma unroll 1
       for (int c0 = 0; c0 < D; c0 += 16) {
         float s[16], r[16];
         tmem_ld16(tm + lane + T_S + c0, s);
@@ -359,6 +360,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       }
     }
     if (p.sv_mask) p.sv_mask[ci * D + j] = msk;
+#pragma unroll 1
     for (int c0 = 0; c0 < D; c0 += 16) {
       float s[16], u[16];
       tmem_ld16(tm + lane + T_S + c0, s);
@@ -448,6 +450,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
               __float2bfloat16_rn(fmaf(gamv[t] * Gam[t] * p.scale, oa[i], ob[i]));
       }
     }
+#pragma unroll 1
     for (int c0 = 0; c0 < D; c0 += 16) {
       float r[16], u[16];
       tmem_ld16(tm + lane + T_R + c0, r);

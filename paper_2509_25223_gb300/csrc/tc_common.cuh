@@ -227,36 +227,62 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
 
 // D (+)= A * B^T over K = 16 * ksteps, A K-major (64-column blocks a_blk
 // apart), B MN-major (K rows, N in 64-wide atoms b_lbo apart).
+template <bool kRolled = false>
 __device__ __forceinline__ void mma_tile_kmn(uint32_t d_tmem, uint32_t a_base, uint32_t a_blk,
                                              uint32_t b_base, uint32_t b_lbo, int ksteps,
                                              uint32_t idesc, bool accumulate_first) {
-  for (int kk = 0; kk < ksteps; ++kk) {
+  auto step = [&](int kk) {
     const uint32_t a = a_base + (uint32_t)(kk >> 2) * a_blk + (uint32_t)(kk & 3) * 32u;
     mma_bf16(d_tmem, sdesc_sw128(a), sdesc_sw128_mn(b_base + (uint32_t)kk * 2048u, b_lbo),
              idesc | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
+  };
+  if constexpr (kRolled) {
+#pragma unroll 1
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  } else {
+#pragma unroll
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
   }
 }
 
 // D (+)= A * B^T over K = 16 * ksteps (<= 4), A MN-major (K rows, M atoms
 // a_lbo apart), B K-major in one 64-column block.
+template <bool kRolled = false>
 __device__ __forceinline__ void mma_tile_mnk(uint32_t d_tmem, uint32_t a_base, uint32_t a_lbo,
                                              uint32_t b_base, int ksteps, uint32_t idesc,
                                              bool accumulate_first) {
-  for (int kk = 0; kk < ksteps; ++kk)
+  auto step = [&](int kk) {
     mma_bf16(d_tmem, sdesc_sw128_mn(a_base + (uint32_t)kk * 2048u, a_lbo),
              sdesc_sw128(b_base + (uint32_t)kk * 32u), idesc | kAMajorMN,
              (kk > 0 || accumulate_first) ? 1u : 0u);
+  };
+  if constexpr (kRolled) {
+#pragma unroll 1
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  } else {
+#pragma unroll
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  }
 }
 
 // D (+)= A * B^T over K = 16 * ksteps with both operands MN-major (K rows;
 // M / N atoms a_lbo / b_lbo apart).
+template <bool kRolled = false>
 __device__ __forceinline__ void mma_tile_mnmn(uint32_t d_tmem, uint32_t a_base, uint32_t a_lbo,
                                               uint32_t b_base, uint32_t b_lbo, int ksteps,
                                               uint32_t idesc, bool accumulate_first) {
-  for (int kk = 0; kk < ksteps; ++kk)
+  auto step = [&](int kk) {
     mma_bf16(d_tmem, sdesc_sw128_mn(a_base + (uint32_t)kk * 2048u, a_lbo),
              sdesc_sw128_mn(b_base + (uint32_t)kk * 2048u, b_lbo),
              idesc | kAMajorMN | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
+  };
+  if constexpr (kRolled) {
+#pragma unroll 1
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  } else {
+#pragma unroll
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  }
 }
 
 // Sum a per-thread vector v[64] over the 32 lanes of a warp by halving
@@ -355,17 +381,27 @@ __device__ __forceinline__ uint32_t sw128(int r, int c) {
   return (uint32_t)(r * 128 + ((((c >> 3) ^ (r & 7)) & 7) << 4) + (c & 7) * 2);
 }
 
+// (kRolled: one issue loop per call site instead of an unrolled sequence --
+// for kernels whose straight-line code would not stay in the instruction cache.)
 // Issue D = A * B^T over K = 16 * ksteps for K-major SW128 tiles A [M][K] and
 // B [N][K] stored as consecutive 64-column blocks (a_blk / b_blk bytes apart).
+template <bool kRolled = false>
 __device__ __forceinline__ void mma_tile(uint32_t d_tmem, uint32_t a_base, uint32_t a_blk,
                                          uint32_t b_base, uint32_t b_blk, int ksteps,
                                          uint32_t idesc, bool accumulate_first) {
-  for (int kk = 0; kk < ksteps; ++kk) {
+  auto step = [&](int kk) {
     const uint32_t off = (uint32_t)(kk & 3) * 32u;
     const uint32_t a = a_base + (uint32_t)(kk >> 2) * a_blk + off;
     const uint32_t b = b_base + (uint32_t)(kk >> 2) * b_blk + off;
     mma_bf16(d_tmem, sdesc_sw128(a), sdesc_sw128(b), idesc,
              (kk > 0 || accumulate_first) ? 1u : 0u);
+  };
+  if constexpr (kRolled) {
+#pragma unroll 1
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  } else {
+#pragma unroll
+    for (int kk = 0; kk < ksteps; ++kk) step(kk);
   }
 }
 
