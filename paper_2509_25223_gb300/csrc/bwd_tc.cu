@@ -863,12 +863,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   };
   // this thread's 32 tokens of a [j][t] atom pair (hi, lo)
   auto put_tok = [&](const float (&x)[32], uint32_t hi, uint32_t lo) {
-#pragma unroll
-    for (int c0 = 0; c0 < 32; c0 += 16) {
+#pragma unroll 1  // one copy of the conversion code per call site
+    for (int h2 = 0; h2 < 2; ++h2) {
       float w[16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) w[i] = x[c0 + i];
-      put16s(sm + hi, sm + lo, j, tb + c0, w);
+      for (int i = 0; i < 16; ++i) w[i] = h2 ? x[16 + i] : x[i];
+      put16s(sm + hi, sm + lo, j, tb + 16 * h2, w);
     }
   };
   auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
@@ -878,8 +878,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   cp_async_wait_all();  // K, Q tile (published by the barriers below)
   if (!mbar_wait(K.barA, 0)) *K.flag = 1;  // phase_run below reports it to every thread
   {  // images of S0, R0; <dS, S0> + <dR, R0> (gradient images: dS hi | dR hi | dS lo | dR lo)
-    float gdot = stage_to_image(SA, gimg, gimg + 65536);
-    gdot += stage_to_image(SB, gimg + 32768, gimg + 98304);
+    float gdot = 0.f;
+#pragma unroll 1
+    for (int s2 = 0; s2 < 2; ++s2)  // S0 with dS, then R0 with dR
+      gdot += stage_to_image(s2 ? SB : SA, gimg + 32768 * s2, gimg + 65536 + 32768 * s2);
 #pragma unroll
     for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
     if (lane == 0) red[warp] = gdot;
@@ -1039,6 +1041,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       tmem_st16(tm + tm_lane + T_DKQ + tb + c0, a);
     }
     // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
+#pragma unroll 1
     for (int w = 0; w < 2; ++w) {
       float ev[32], rv[32];
       image_row(w == 0 ? XH : YH, ev);
