@@ -828,29 +828,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   // fp32 [i][j] state staged at `base` -> rows j of its (hi | lo) image at
   // `base`, key rows of half hf (every thread reads its values before any writes)
-  // Also returns this thread's part of <g, state> for the gradient g w.r.t. the
-  // chunk's end state, read from its image in global memory (hi at gh, lo at gl).
-  auto stage_to_image = [&](uint32_t base, const uint8_t *gh, const uint8_t *gl) {
-    uint4 gv[16];
-#pragma unroll
-    for (int c8 = 0; c8 < 8; ++c8) {
-      const uint32_t o = hf * 16384 + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
-      gv[c8] = __ldg(reinterpret_cast<const uint4 *>(gh + o));
-      gv[8 + c8] = __ldg(reinterpret_cast<const uint4 *>(gl + o));
-    }
+  auto stage_to_image = [&](uint32_t base) {
     const float *st = reinterpret_cast<const float *>(sm + base);
     float v[64];
 #pragma unroll
     for (int i = 0; i < 64; ++i) v[i] = st[(64 * hf + i) * D + j];
-    float dot = 0.f;
-#pragma unroll
-    for (int c8 = 0; c8 < 8; ++c8) {
-      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&gv[c8]);
-      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&gv[8 + c8]);
-#pragma unroll
-      for (int e = 0; e < 8; ++e)
-        dot += (__bfloat162float(hb[e]) + __bfloat162float(lb[e])) * v[c8 * 8 + e];
-    }
     __syncthreads();
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
@@ -859,7 +841,22 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
       put16s(sm + base + hf * 16384, sm + base + 32768 + hf * 16384, j, c0, w);
     }
-    return dot;
+  };
+  // sum over this thread's entries of (image at base, hi + lo) * x[i][j]
+  auto dot_image = [&](uint32_t base, const float (&x)[64]) {
+    float s = 0.f;
+#pragma unroll
+    for (int c8 = 0; c8 < 8; ++c8) {
+      const uint32_t o = base + hf * 16384 + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
+      const uint4 hv = *reinterpret_cast<const uint4 *>(sm + o);
+      const uint4 lv = *reinterpret_cast<const uint4 *>(sm + o + 32768);
+      const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
+      const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        s += (__bfloat162float(hb[e]) + __bfloat162float(lb[e])) * x[c8 * 8 + e];
+    }
+    return s;
   };
   // this thread's 32 tokens of a [j][t] atom pair (hi, lo)
   auto put_tok = [&](const float (&x)[32], uint32_t hi, uint32_t lo) {
@@ -877,21 +874,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 
   cp_async_wait_all();  // K, Q tile (published by the barriers below)
   if (!mbar_wait(K.barA, 0)) *K.flag = 1;  // phase_run below reports it to every thread
-  {  // images of S0, R0; <dS, S0> + <dR, R0> (gradient images: dS hi | dR hi | dS lo | dR lo)
-    float gdot = 0.f;
 #pragma unroll 1
-    for (int s2 = 0; s2 < 2; ++s2)  // S0 with dS, then R0 with dR
-      gdot += stage_to_image(s2 ? SB : SA, gimg + 32768 * s2, gimg + 65536 + 32768 * s2);
-#pragma unroll
-    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
-    if (lane == 0) red[warp] = gdot;
-    __syncthreads();
-    if (tid == 0) {
-      float s = 0.f;
-      for (int w = 0; w < NTP / 32; ++w) s += red[w];
-      *dGamC = s;
-    }
-  }
+  for (int s2 = 0; s2 < 2; ++s2) stage_to_image(s2 ? SB : SA);  // images of S0, R0
   // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
   bool ok = phase_run(K, tid, [&] {
     const uint32_t t_ = *slot;
@@ -990,9 +974,26 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     bulk_g2s(sm + XH, P.E2buf + chunk * 32768, 32768, K.barC);  // hi at XH, lo at XL
     bulk_g2s(sm + YH, P.Ebuf + chunk * 32768, 32768, K.barC);   // hi at YH, lo at YL
   }
-  if (ok) {  // the dR, dS images (issued after P2, P3), for every thread
-    if (!mbar_wait(K.barB, 0)) *K.flag = 1;
-    if (!mbar_wait(K.barA, 1)) *K.flag = 1;
+  if (ok) {  // <dR, R0> + <dS, S0> (states re-read from L2, images in place), into dGamC
+    float gdot = 0.f;
+#pragma unroll 1
+    for (int s2 = 0; s2 < 2; ++s2) {
+      const float *st = s2 ? S0 : R0;
+      float x[64];
+#pragma unroll
+      for (int i = 0; i < 64; ++i) x[i] = st[(size_t)(64 * hf + i) * D + j];
+      if (!mbar_wait(s2 ? K.barA : K.barB, s2 ? 1 : 0)) *K.flag = 1;
+      gdot += dot_image(s2 ? SA : SB, x);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
+    if (lane == 0) red[warp] = gdot;
+    __syncthreads();
+    if (tid == 0) {
+      float s = 0.f;
+      for (int w = 0; w < NTP / 32; ++w) s += red[w];
+      *dGamC = s;
+    }
   }
   // this thread's 32 tokens of row j of a (hi | lo) image of a [j][t] matrix
   auto image_row = [&](uint32_t base, float (&out)[32]) {
