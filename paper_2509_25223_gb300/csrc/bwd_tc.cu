@@ -159,6 +159,29 @@ __device__ __forceinline__ bool phase_run(Ctl &k, int tid, F issue) {
   return *k.flag == 0;
 }
 
+// The same phase in two halves, for work that overlaps the MMAs: publish and
+// issue ...
+template <typename F>
+__device__ __forceinline__ void phase_issue(Ctl &k, int tid, F issue) {
+  fence_async_smem();
+  fence_before_sync();
+  __syncthreads();
+  if (tid == 0) {
+    fence_after_sync();
+    if (!issue()) *k.flag = 1;
+    mma_commit(k.bar);
+  }
+}
+// ... then wait for them (every thread).
+__device__ __forceinline__ bool phase_wait(Ctl &k) {
+  const bool ok = mbar_wait(k.bar, k.phase);
+  k.phase ^= 1u;
+  if (!ok) *k.flag = 1;
+  __syncthreads();
+  fence_after_sync();
+  return *k.flag == 0;
+}
+
 // thread 0: wait for a slot's bulk copy
 __device__ __forceinline__ bool slot_wait(uint64_t *bar, uint32_t &ph) {
   const bool ok = mbar_wait(bar, ph);
@@ -801,31 +824,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
     cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
   }
-  const unsigned long long m = P.mask[chunk * D + j] >> tb;
-  // this thread's tokens of dX2, dX (from the staging, below) and dO
+  // this thread's tokens of dX2, dX (from the staging) and dO: read after P1 is
+  // issued, so that the MMA issue does not wait behind them
   float x2v[32], xv[32], dov[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    const int t = tb + i;
-    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
-  }
-  if (tid < 64) {
-    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
-    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
-    wS[tid] = recf[OFF_VEC + V_WS + tid];
-    wR[tid] = recf[OFF_VEC + V_WR + tid];
-    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
-  }
-  if (!mbar_wait(K.barC, 0)) *K.flag = 1;
-  {
-    const float *x2s = reinterpret_cast<const float *>(sm + XH);
-    const float *xs = reinterpret_cast<const float *>(sm + YH);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      x2v[i] = x2s[(tb + i) * D + j];
-      xv[i] = xs[(tb + i) * D + j];
-    }
-  }
   // fp32 [i][j] state staged at `base` -> rows j of its (hi | lo) image at
   // `base`, key rows of half hf (every thread reads its values before any writes)
   auto stage_to_image = [&](uint32_t base) {
@@ -868,7 +869,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       put16s(sm + hi, sm + lo, j, tb + 16 * h2, w);
     }
   };
-  auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
   const uint32_t tm_lane = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
 
@@ -877,7 +877,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll 1
   for (int s2 = 0; s2 < 2; ++s2) stage_to_image(s2 ? SB : SA);  // images of S0, R0
   // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
-  bool ok = phase_run(K, tid, [&] {
+  phase_issue(K, tid, [&] {
     const uint32_t t_ = *slot;
     mma_tile<true>(t_ + T_KS, sb + SA, 16384, sb + KQ, 16384, 8, i128, false);
     mma_tile<true>(t_ + T_KS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i128, true);
@@ -885,7 +885,33 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     mma_tile<true>(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
     return true;
   });
+  // while P1 runs: this thread's dO, the gate vectors, dX2 and dX from their staging
+  const unsigned long long m = P.mask[chunk * D + j] >> tb;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int t = tb + i;
+    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+  }
+  if (tid < 64) {
+    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
+    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
+    wS[tid] = recf[OFF_VEC + V_WS + tid];
+    wR[tid] = recf[OFF_VEC + V_WR + tid];
+    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+  }
+  if (!mbar_wait(K.barC, 0)) *K.flag = 1;
+  {
+    const float *x2s = reinterpret_cast<const float *>(sm + XH);
+    const float *xs = reinterpret_cast<const float *>(sm + YH);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      x2v[i] = x2s[(tb + i) * D + j];
+      xv[i] = xs[(tb + i) * D + j];
+    }
+  }
+  bool ok = phase_wait(K);  // (its barrier also publishes the gate vectors)
   const uint32_t tm = *slot;
+  auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
     float rv[32];
     {  // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
