@@ -215,6 +215,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     tmem_st16(tm + lane + T_R + c0, r);
     st_row16(sm + SM_SA, 16384, j, c0, s);
     st_row16(sm + SM_RA, 16384, j, c0, r);
+    if (p.S_chunks) {  // the first chunk's start states, for the backward
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        p.S_chunks[(size_t)bh * NC * D * D + (size_t)(c0 + i) * D + j] = s[i];
+        p.R_chunks[(size_t)bh * NC * D * D + (size_t)(c0 + i) * D + j] = r[i];
+      }
+    }
   }
 
   // one MMA phase: make smem writes visible, issue, wait.  Returns false on
@@ -245,22 +252,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     cp_async_wait_all();  // this chunk's V, K, Q tiles (fetched during the previous chunk)
     __syncthreads();      // every thread is done with the previous chunk's tiles and vectors
 
-    // ---- (a) chunk inputs -> shared memory
-    if (p.S_chunks) {  // chunk-start states for the backward
-      float *sc = p.S_chunks + ((size_t)bh * NC + c) * D * D;
-      float *rc = p.R_chunks + ((size_t)bh * NC + c) * D * D;
-#pragma unroll 1
-      for (int c0 = 0; c0 < D; c0 += 16) {
-        float s[16], r[16];
-        tmem_ld16(tm + lane + T_S + c0, s);
-        tmem_ld16(tm + lane + T_R + c0, r);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          sc[(size_t)(c0 + i) * D + j] = s[i];
-          rc[(size_t)(c0 + i) * D + j] = r[i];
-        }
-      }
-    }
+    // ---- (a) chunk inputs -> shared memory (the chunk-start states for the
+    // backward were stored by the previous chunk's updates)
+    float *sc_next = (p.S_chunks && c + 1 < NC) ? p.S_chunks + ((size_t)bh * NC + c + 1) * D * D
+                                                : nullptr;
+    float *rc_next = sc_next ? p.R_chunks + ((size_t)bh * NC + c + 1) * D * D : nullptr;
     if (tid < 64) {
       Gam[tid] = rec[OFF_VEC + V_GAM + tid];
       Gprev[tid] = rec[OFF_VEC + V_GPREV + tid];
@@ -369,6 +365,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
       tmem_st16(tm + lane + T_S + c0, s);
       st_row16(sm + SM_SA, 16384, j, c0, s);
+      if (sc_next) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sc_next[(size_t)(c0 + i) * D + j] = s[i];
+      }
     }
     // MMA5: D3 = R^T [K ; Q]^T (into X; unscaled K R | Q R)
     alive = run_phase([&] {
@@ -459,6 +459,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
       tmem_st16(tm + lane + T_R + c0, r);
       st_row16(sm + SM_RA, 16384, j, c0, r);
+      if (rc_next) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rc_next[(size_t)(c0 + i) * D + j] = r[i];
+      }
     }
   }
 
