@@ -437,24 +437,26 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   fence_after_sync();
   const uint32_t tm = *slot;
   const uint32_t lane = (uint32_t)(warp * 32) << 16;
-  // carried gradients (bf16 hi + lo tiles, rows j) from their fp32 TMEM copy
+  // a carried gradient's bf16 hi + lo tiles (rows j), 16 of its key rows
+  auto put_grad16 = [&](uint32_t hi, uint32_t lo, int c0, const float (&g)[16]) {
+    float gh[16], gl[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      gh[i] = __bfloat162float(__float2bfloat16_rn(g[i]));
+      gl[i] = g[i] - gh[i];
+    }
+    put16(sm + hi, 16384, j, c0, gh);
+    put16(sm + lo, 16384, j, c0, gl);
+  };
+  // both carried gradients' tiles from their fp32 TMEM copies
   auto write_grad_tiles = [&]() {
 #pragma unroll 1
     for (int c0 = 0; c0 < D; c0 += 16) {
-      float s[16], r[16], sh[16], sl[16], rh[16], rl[16];
+      float s[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
       tmem_ld16(tm + lane + T_DR + c0, r);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        sh[i] = __bfloat162float(__float2bfloat16_rn(s[i]));
-        sl[i] = s[i] - sh[i];
-        rh[i] = __bfloat162float(__float2bfloat16_rn(r[i]));
-        rl[i] = r[i] - rh[i];
-      }
-      put16(sm + DSH, 16384, j, c0, sh);
-      put16(sm + DSL, 16384, j, c0, sl);
-      put16(sm + DRH, 16384, j, c0, rh);
-      put16(sm + DRL, 16384, j, c0, rl);
+      put_grad16(DSH, DSL, c0, s);
+      put_grad16(DRH, DRL, c0, r);
     }
     fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   };
@@ -690,16 +692,21 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       fetch_kq(c - 1);
       pre = fetch_pre(c - 1);
     }
+    // dS update, and the carried gradients' tiles: the A operands of the next
+    // chunk's phase A (the scratch tiles in their place are done with)
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {  // dS update
-      float s[16], u[16];
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float s[16], u[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
       tmem_ld16(tm + lane + T_R1 + c0, u);
+      tmem_ld16(tm + lane + T_DR + c0, r);
 #pragma unroll
       for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
       tmem_st16(tm + lane + T_DS + c0, s);
+      put_grad16(DSH, DSL, c0, s);
+      put_grad16(DRH, DRL, c0, r);
     }
-    write_grad_tiles();  // A operands of the next chunk's phase A
+    fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   }
   if (ok) {
     for (int c0 = 0; c0 < D; c0 += 16) {
