@@ -797,40 +797,61 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int j = tid & 127, hf = tid >> 7, tb = 32 * hf;
-  const size_t chunk = blockIdx.x;
   const int NC = p.NC, T = p.T, H = p.H;
-  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
-  const int b = bh / H, h = bh % H;
-  const int t0 = c * 64, n = min(64, T - t0);
+  const size_t nct = (size_t)p.B * H * NC;
   const float scale = p.scale;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
-  const float *recf = p.ws + chunk * kRecFloats;
-  float *acc = P.acc + chunk * A8::FLOATS;
-
-  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
-  const uint8_t *gimg = P.gimg + chunk * 131072;  // dS hi | dR hi | dS lo | dR lo
   Ctl K;
   ctl_init(K, sm + CTL, tid);
   if (warp == 0) tmem_alloc(slot, 512);
-  __syncthreads();  // barriers initialised
-  if (tid == 0) {  // chunk-start states, fp32, staged where their images go; dX2, dX
-                   // (fp32 [t][j]) staged in the pair's place until P2
-    mbar_expect_tx(K.barA, 131072);
-    bulk_g2s(sm + SA, S0, 65536, K.barA);
-    bulk_g2s(sm + SB, R0, 65536, K.barA);
-    mbar_expect_tx(K.barC, 65536);
-    bulk_g2s(sm + XH, P.dX2buf + chunk * 64 * D, 32768, K.barC);
-    bulk_g2s(sm + YH, P.dXbuf + chunk * 64 * D, 32768, K.barC);
+  fence_before_sync();
+  __syncthreads();  // barriers initialised, TMEM allocated
+  fence_after_sync();
+  const uint32_t tm = *slot;
+  // A chunk's inputs are fetched in two parts, each during the previous chunk
+  // (this CTA loops over chunks): the chunk-start states, fp32, staged where
+  // their images go; then dX2, dX (fp32 [t][j], staged in the pair's place
+  // until P2) and the K, Q tile.
+  auto fetch_states = [&](size_t ck) {
+    if (tid == 0) {
+      mbar_expect_tx(K.barA, 131072);
+      bulk_g2s(sm + SA, P.Sc + ck * D * D, 65536, K.barA);
+      bulk_g2s(sm + SB, P.Rc + ck * D * D, 65536, K.barA);
+    }
+  };
+  auto fetch_rest = [&](size_t ck) {
+    if (tid == 0) {
+      mbar_expect_tx(K.barC, 65536);
+      bulk_g2s(sm + XH, P.dX2buf + ck * 64 * D, 32768, K.barC);
+      bulk_g2s(sm + YH, P.dXbuf + ck * 64 * D, 32768, K.barC);
+    }
+    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
+    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * 64, n_ = min(64, T - t0_);
+    for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16), asynchronous
+      const int t = e >> 4, chn = e & 15;
+      const bool vld = t < n_;
+      const size_t off = ((size_t)(b_ * T + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
+      const int blk = chn >> 3, cc = (chn & 7) * 8;
+      cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
+    }
+  };
+  if (blockIdx.x < nct) {
+    fetch_states(blockIdx.x);
+    fetch_rest(blockIdx.x);
   }
-  for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16), asynchronous
-    const int t = e >> 4, chn = e & 15;
-    const bool vld = t < n;
-    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
-    const int blk = chn >> 3, cc = (chn & 7) * 8;
-    cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
-    cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
-  }
+  bool ok = true;
+  uint32_t it = 0;  // chunks done by this CTA: the parity of barrier B
+  for (size_t chunk = blockIdx.x; chunk < nct && ok; chunk += gridDim.x, ++it) {
+  const size_t next = chunk + gridDim.x;
+  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
+  const int b = bh / H, h = bh % H;
+  const int t0 = c * 64, n = min(64, T - t0);
+  const float *recf = p.ws + chunk * kRecFloats;
+  float *acc = P.acc + chunk * A8::FLOATS;
+  const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
+  const uint8_t *gimg = P.gimg + chunk * 131072;  // dS hi | dR hi | dS lo | dR lo
   // this thread's tokens of dX2, dX (from the staging) and dO: read after P1 is
   // issued, so that the MMA issue does not wait behind them
   float x2v[32], xv[32], dov[32];
@@ -916,8 +937,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       xv[i] = xs[(tb + i) * D + j];
     }
   }
-  bool ok = phase_wait(K);  // (its barrier also publishes the gate vectors)
-  const uint32_t tm = *slot;
+  ok = phase_wait(K);  // (its barrier also publishes the gate vectors)
   auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
     float rv[32];
@@ -1015,7 +1035,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       float x[64];
 #pragma unroll
       for (int i = 0; i < 64; ++i) x[i] = st[(size_t)(64 * hf + i) * D + j];
-      if (!mbar_wait(s2 ? K.barA : K.barB, s2 ? 1 : 0)) *K.flag = 1;
+      if (!mbar_wait(s2 ? K.barA : K.barB, s2 ? 1u : (it & 1u))) *K.flag = 1;
       gdot += dot_image(s2 ? SA : SB, x);
     }
 #pragma unroll
@@ -1129,6 +1149,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   float *cum = F + F_VEC, *cprev = cum + 64, *bet = cum + 128, *gam = cum + 192, *gg = cum + 256,
         *dcum = cum + 320, *dcprev = cum + 384, *dbet = cum + 448, *dgam = cum + 512;
   float *prt = cum + 576;  // [6][4][64] partial sums
+  float o_dg = 0.f, o_dbeta = 0.f, o_dgamma = 0.f;  // this thread's token's gate gradients
   if (ok) {
     {
       const int r = j & 63;
@@ -1321,20 +1342,29 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       put16s(sm + XH, sm + XL, 64 + t, 16 * q4, w);
     }
     // ---- P7: dK, dQ += K^T [dKK + dKK^T ; dQK]^T ; D2 = Q^T dQK
-    ok = phase_run(K, tid, [&] {
+    phase_issue(K, tid, [&] {
       mma_tile_mnk<true>(tm + T_DKQ, sb + KQ, 16384, sb + XH, 4, i128, true);
       mma_tile_mnk<true>(tm + T_DKQ, sb + KQ, 16384, sb + XL, 4, i128, true);
       mma_tile_mnmn<true>(tm + T_D2, sb + KQ + 8192, 16384, sb + XH + 8192, 16384, 4, i64, false);
       mma_tile_mnmn<true>(tm + T_D2, sb + KQ + 8192, 16384, sb + XL + 8192, 16384, 4, i64, true);
       return true;
     });
+    if (tid < n) {  // the vectors live where the next chunk's states are staged
+      o_dg = gg[tid];
+      o_dbeta = dbet[tid];
+      o_dgamma = dgam[tid];
+    }
+    __syncthreads();
+    if (next < nct) fetch_states(next);  // the state images and the fp32 tiles are done with
+    ok = phase_wait(K);
+    if (ok && next < nct) fetch_rest(next);  // K, Q and the pair region are done with
   }
   if (ok) {
     if (tid < n) {
       const size_t off = (size_t)(b * T + t0 + tid) * H + h;
-      P.dg[off] = gg[tid];
-      P.dbeta[off] = dbet[tid];
-      P.dgamma[off] = dgam[tid];
+      P.dg[off] = o_dg;
+      P.dbeta[off] = o_dbeta;
+      P.dgamma[off] = o_dgamma;
     }
     __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
 #pragma unroll 1
@@ -1353,9 +1383,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         }
       }
     }
-  } else if (tid == 0 && p.err) {
-    atomicExch(p.err, RDN_ERR_TIMEOUT);
   }
+  }  // chunks
+  if (!ok && tid == 0 && p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+  cp_async_wait_all();  // no copy of this CTA outlives it (a fetch for a chunk not reached)
   fence_before_sync();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, 512);
@@ -1423,7 +1454,12 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   }
   RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NT, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<(unsigned)nct, po::NTP, po::SMEM, s>>>(P));
+  int dev = 0, nsm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return e;
+  const unsigned post_grid = (unsigned)(nct < (size_t)nsm ? nct : (size_t)nsm);  // one CTA per SM
+  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<post_grid, po::NTP, po::SMEM, s>>>(P));
   return cudaGetLastError();
 }
 
