@@ -596,8 +596,9 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     if (!ok) break;
     if (tid == 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TB, 16384);
     float dP[64];
-    {  // dX2 -> dP = -mask dX2, dKR = -Gam dX2
-      float *gx = P.dX2buf + chunk * 64 * D;
+    {  // dX2 -> dP = -mask dX2, dKR = -Gam dX2; dX2 itself (fp32 [t][j]) for bwd_post,
+       // staged in the free scratch tiles and bulk-copied
+      float *stg = reinterpret_cast<float *>(sm + S0H);
 #pragma unroll
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float x[16], dkr[16], dp[16];
@@ -605,7 +606,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
-          gx[t * D + j] = x[i];
+          stg[t * D + j] = x[i];
           dp[i] = ((m >> t) & 1ull) ? -x[i] : 0.f;
           dP[t] = dp[i];
           dkr[i] = -Gam[t] * x[i];
@@ -616,12 +617,16 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     }
     // ---- phase C: U_R += K^T dKR ; Ap^T dP
     ok = phase_run(K, tid, [&] {
+      static_assert(S0L == S0H + 16384, "contiguous");
+      bulk_s2g(P.dX2buf + chunk * 64 * D, sm + S0H, 32768);  // (published by this barrier)
+      bulk_commit();
       if (!slot_wait(K.barB, K.phB)) return false;
       const uint32_t i128 = idesc_bf16(128, 128);
       mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
       mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
       mma_s3_kmn(tm + T_R3, sb + S3H, sb + S3L, sb + SLOTB, sb + SLOTB + 8192, 16384,
                  idesc_bf16(128, 64), false);
+      bulk_wait_read();  // the staging is rewritten next
       return true;
     });
     if (!ok) break;
@@ -663,8 +668,10 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     if (!ok) break;
     if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
     if (c > 0) fetch_do(c - 1);  // every thread is past its last read of this chunk's dO
-    {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX
-      float *gx = P.dXbuf + chunk * 64 * D;
+    {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX; dX (fp32 [t][j]) and dv
+       // (bf16 [t][j]) staged in the free scratch tiles
+      float *stg = reinterpret_cast<float *>(sm + S0H);
+      __nv_bfloat16 *dvs = reinterpret_cast<__nv_bfloat16 *>(sm + S1H);
 #pragma unroll
       for (int c0 = 0; c0 < 64; c0 += 16) {
         float x[16], dks[16];
@@ -672,12 +679,23 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
-          gx[t * D + j] = x[i];
-          if (t < n)
-            dv[((size_t)(b * T + t0 + t) * H + h) * D + j] = __float2bfloat16_rn(x[i] - dP[t]);
+          stg[t * D + j] = x[i];
+          dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[t]);
           dks[i] = Gprev[t] * dP[t] - Gam[t] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
+      }
+      fence_async_smem();
+      __syncthreads();
+      if (tid == 0) {
+        bulk_s2g(P.dXbuf + chunk * 64 * D, sm + S0H, 32768);
+        bulk_commit();
+      }
+      for (int e = tid; e < 64 * 16; e += NT) {  // dv rows, 16 bytes at a time
+        const int t = e >> 4, chn = e & 15;
+        if (t < n)
+          *reinterpret_cast<uint4 *>(dv + ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8) =
+              *reinterpret_cast<const uint4 *>(sm + S1H + t * 256 + chn * 16);
       }
     }
     // ---- phase E: U_S += K^T dKS
@@ -685,6 +703,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       const uint32_t i128 = idesc_bf16(128, 128);
       mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
       mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
+      bulk_wait_read();  // the staging is rewritten next (the gradient tiles)
       return true;
     });
     if (!ok) break;
