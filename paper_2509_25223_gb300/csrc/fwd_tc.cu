@@ -438,6 +438,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (c + 1 < NC) fetch_kq(c + 1);  // K, Q are done with
 
     // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R = Gam_C R + U2
+    // o is staged as a [t][j] bf16 tile in W's place (free after MMA8) and stored
+    // 16 bytes at a time
+    __nv_bfloat16 *ostg = reinterpret_cast<__nv_bfloat16 *>(sm + SM_W);
+#pragma unroll 1
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float ob[16], oa[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);
@@ -445,9 +449,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
-        if (t < n)
-          o[((size_t)(b * T + t0 + t) * H + h) * D + j] =
-              __float2bfloat16_rn(fmaf(gamv[t] * Gam[t] * p.scale, oa[i], ob[i]));
+        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gamv[t] * Gam[t] * p.scale, oa[i], ob[i]));
       }
     }
 #pragma unroll 1
@@ -463,6 +465,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) rc_next[(size_t)(c0 + i) * D + j] = r[i];
       }
+    }
+    __syncthreads();  // the o tile
+    for (int e = tid; e < 64 * 16; e += kTcThreads) {
+      const int t = e >> 4, ch = e & 15;
+      if (t < n)
+        *reinterpret_cast<uint4 *>(o + ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8) =
+            *reinterpret_cast<const uint4 *>(sm + SM_W + t * 256 + ch * 16);
     }
   }
 
