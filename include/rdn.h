@@ -184,6 +184,8 @@ rdn_status_t rdn_fwd(const rdn_fwd_args *args, rdn_stream_t stream);
  * library (RDN_NOALLOC_SCRATCH_BYTES, held on every GPU that loads the
  * library until the process exits) instead of args->workspace, which is
  * ignored.  It allocates nothing.
+ *   - RDN_FLAG_SAVE_FOR_BWD is rejected (RDN_ERR_UNSUPPORTED): what it saves
+ *     would stay in the built-in scratch, out of rdn_bwd's reach.
  *   - Size limit: the scratch holds one 83,456-byte record per 64-token
  *     chunk, so B * H * ceil(T/64) must be at most 804; larger problems
  *     return RDN_ERR_WORKSPACE (with a message giving both sizes) and

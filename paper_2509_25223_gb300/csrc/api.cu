@@ -227,6 +227,9 @@ rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a, rdn_stream_t stream) {
   const char *fn = "rdn_fwd_noalloc";
   rdn_status_t st = check_fwd_shapes(fn, a);
   if (st != RDN_OK) return st;
+  if (a->flags & RDN_FLAG_SAVE_FOR_BWD)  // what it saves would stay in the built-in scratch
+    return fail(RDN_ERR_UNSUPPORTED,
+                "%s: RDN_FLAG_SAVE_FOR_BWD needs a caller workspace (use rdn_fwd)", fn);
   if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
   const size_t need = rdn::plan_fwd(*a, 1).total_bytes;
   if (need > (size_t)RDN_NOALLOC_SCRATCH_BYTES) {

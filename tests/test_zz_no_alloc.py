@@ -70,3 +70,18 @@ def test_noalloc_rejects_problems_beyond_its_scratch():
     assert lib.rdn_fwd_noalloc(ctypes.byref(a), None) == 5
     msg = lib.rdn_last_error().decode()
     assert "built-in scratch" in msg and "804" in msg
+
+
+def test_noalloc_rejects_the_save_for_backward_flag():
+    """Its scratch is internal, so intermediates saved there would be out of
+    rdn_bwd's reach: the flag is refused before anything is launched."""
+    lib = _abi.load()
+    a = _abi.FwdArgs()
+    a.B, a.T, a.H, a.Dk, a.Dv = 1, 64, 1, 128, 128
+    a.dtype, a.clip, a.scale = _abi.RDN_BF16, 1.0, 1.0
+    a.flags = _abi.RDN_FLAG_SAVE_FOR_BWD
+    fake = ctypes.c_void_p(0x10000)
+    a.q = a.k = a.v = a.g = a.beta = a.gamma = a.o = fake
+    a.S_chunks = a.R_chunks = fake
+    assert lib.rdn_fwd_noalloc(ctypes.byref(a), None) == 2
+    assert "caller workspace" in lib.rdn_last_error().decode()
