@@ -24,7 +24,9 @@
 //     matrices' entries turned into dq, dk, dg, dbeta, dgamma (the work that
 //     bwd_finish of chunk_bwd.cu does on the SIMT path).
 //
-// Orientation: thread j of 128 owns value column j = TMEM lane j for every
+// Orientation: value column j = TMEM lane j, owned by thread j of a group of
+// 128 threads (bwd_chain: 4 groups, group g taking the token and key columns
+// [16g, 16g + 16) and [64 + 16g, 80 + 16g); bwd_post: 2 groups), for every
 // column quantity (X, E, dO, dX2, ...), which is kept as a bf16 hi + lo tile
 // [j][t] (K-major for products over t).  Products over j use the same tiles
 // as MN-major operands.  The chunk matrices come from chunk_prep's images
@@ -39,7 +41,8 @@ namespace {
 using namespace tc;
 
 constexpr int D = 128;
-constexpr int NT = 128;  // threads per CTA
+constexpr int NT = 128;   // threads per CTA of bwd_recompute
+constexpr int NTC = 512;  // threads per CTA of bwd_chain (4 warps per TMEM lane quadrant)
 
 // Per-chunk row-sum slots in the backward workspace (floats): read-out part of
 // d gamma, dwS, dwR (C each).  Used as scratch by bwd_post, whose shared
@@ -388,7 +391,7 @@ static_assert(SMEM <= 232448, "shared memory");
 constexpr uint32_t T_DS = 0, T_DR = 128, T_R1 = 256, T_R2 = 320, T_R3 = 384, T_R4 = 448;
 }  // namespace ch
 
-__global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
+__global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
   using namespace ch;
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sb = smem_u32(sm);
@@ -400,7 +403,8 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   float *vec = reinterpret_cast<float *>(sm + VEC);
   float *Gam = vec, *Gprev = vec + 64, *wS = vec + 128, *wR = vec + 192, *gamv = vec + 256;
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
-  const int tid = threadIdx.x, warp = tid >> 5, j = tid;
+  const int tid = threadIdx.x, warp = tid >> 5, j = tid & 127;
+  const int g16 = (warp >> 2) * 16;  // this thread's token (and key) columns start
   const int bh = blockIdx.x;
   const int NC = p.NC, T = p.T, H = p.H;
   const int b = bh / H, h = bh % H;
@@ -436,7 +440,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   __syncthreads();
   fence_after_sync();
   const uint32_t tm = *slot;
-  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   // a carried gradient's bf16 hi + lo tiles (rows j), 16 of its key rows
   auto put_grad16 = [&](uint32_t hi, uint32_t lo, int c0, const float (&g)[16]) {
     float gh[16], gl[16];
@@ -451,7 +455,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   // both carried gradients' tiles from their fp32 TMEM copies
   auto write_grad_tiles = [&]() {
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
       tmem_ld16(tm + lane + T_DR + c0, r);
@@ -460,7 +464,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     }
     fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   };
-  for (int c0 = 0; c0 < D; c0 += 16) {  // upstream gradients of the final states
+  for (int c0 = g16; c0 < D; c0 += 64) {  // upstream gradients of the final states
     float s[16], r[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -475,7 +479,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   // a chunk's K, Q, dO tiles (rows t, exact bf16, zero past the end), asynchronous
   auto fetch_kq = [&](int c) {
     const int t0 = c * 64, n = min(64, T - t0);
-    for (int e = tid; e < 64 * 16; e += NT) {
+    for (int e = tid; e < 64 * 16; e += NTC) {
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n;
       const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
@@ -486,31 +490,36 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
   };
   auto fetch_do = [&](int c) {
     const int t0 = c * 64, n = min(64, T - t0);
-    for (int e = tid; e < 64 * 16; e += NT) {
+    for (int e = tid; e < 64 * 16; e += NTC) {
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n;
       const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
       cp_async16(sm + DOT + (chn >> 3) * 8192 + sw128(t, (chn & 7) * 8), dOp + off, vld);
     }
   };
-  // a chunk's gate vectors and clip-mask word, into registers
+  // a chunk's gate vectors (threads 0..63, one token each) and this thread's
+  // 16 bits of the clip-mask word, into registers
   struct Pre {
     float gam_, gprev, ws_, wr_, g_, gamc;
-    unsigned long long m;
+    unsigned m;
   };
   auto fetch_pre = [&](int c) {
     const size_t ck = (size_t)bh * NC + c;
     const int t0 = c * 64, n = min(64, T - t0);
     const float *rf = p.ws + ck * kRecFloats;
     Pre x;
-    const int t = tid & 63;
-    x.gam_ = rf[OFF_VEC + V_GAM + t];
-    x.gprev = rf[OFF_VEC + V_GPREV + t];
-    x.ws_ = rf[OFF_VEC + V_WS + t];
-    x.wr_ = rf[OFF_VEC + V_WR + t];
-    x.g_ = t < n ? p.gamma[(size_t)(b * T + t0 + t) * H + h] : 0.f;
+    x.gam_ = x.gprev = x.ws_ = x.wr_ = x.g_ = 0.f;
+    if (tid < 64) {
+      const int t = tid;
+      x.gam_ = rf[OFF_VEC + V_GAM + t];
+      x.gprev = rf[OFF_VEC + V_GPREV + t];
+      x.ws_ = rf[OFF_VEC + V_WS + t];
+      x.wr_ = rf[OFF_VEC + V_WR + t];
+      x.g_ = t < n ? p.gamma[(size_t)(b * T + t0 + t) * H + h] : 0.f;
+    }
     x.gamc = rf[OFF_VEC + V_GAMC];
-    x.m = P.mask[ck * D + j];
+    // bits [g16, g16 + 16) of the column's 64-bit word (little-endian)
+    x.m = reinterpret_cast<const uint16_t *>(P.mask + ck * D + j)[g16 >> 4];
     return x;
   };
   fetch_kq(NC - 1);
@@ -535,7 +544,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       gamv[tid] = pre.g_;
     }
     const float GamC = pre.gamc;
-    const unsigned long long m = pre.m;
+    const unsigned m = pre.m;  // bit i: clip inactive at t = g16 + i
     cp_async_wait_all();  // this chunk's tiles (fetched during the previous one)
     __syncthreads();
     auto dO = [&](int t) {  // dO[t, j] from the tile
@@ -565,23 +574,25 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
       load_ap(chunk);
     }
     // dE2 = M2^T dOa + wR K dR ; dE (partial) = Mq^T dO + wS K dS ; dQR = Gam gamma dO
+    {
+      const int c0 = g16;
+      float x[16], y[16];
+      tmem_ld16(tm + lane + T_R1 + c0, x);
+      tmem_ld16(tm + lane + T_R3 + c0, y);
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
-      float kdr[16], kds[16], m2[16], mq[16], dqr[16];
-      tmem_ld16(tm + lane + T_R1 + c0, kdr);
-      tmem_ld16(tm + lane + T_R2 + c0, kds);
-      tmem_ld16(tm + lane + T_R3 + c0, m2);
-      tmem_ld16(tm + lane + T_R4 + c0, mq);
+      for (int i = 0; i < 16; ++i) y[i] += wR[c0 + i] * x[i];
+      put16s(sm + S0H, sm + S0L, j, c0, y);
+      tmem_ld16(tm + lane + T_R2 + c0, x);
+      tmem_ld16(tm + lane + T_R4 + c0, y);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) y[i] += wS[c0 + i] * x[i];
+      tmem_st16(tm + lane + T_R4 + c0, y);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
-        m2[i] = m2[i] + wR[t] * kdr[i];
-        mq[i] = mq[i] + wS[t] * kds[i];
-        dqr[i] = p.scale * Gam[t] * gamv[t] * dO(t);  // Q below is unscaled
+        x[i] = p.scale * Gam[t] * gamv[t] * dO(t);  // dQR (Q below is unscaled)
       }
-      tmem_st16(tm + lane + T_R4 + c0, mq);
-      put16s(sm + S0H, sm + S0L, j, c0, m2);
-      put16s(sm + S1H, sm + S1L, j, c0, dqr);
+      put16s(sm + S1H, sm + S1L, j, c0, x);
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
     ok = phase_run(K, tid, [&] {
@@ -595,20 +606,20 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     });
     if (!ok) break;
     if (tid == 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TB, 16384);
-    float dP[64];
+    float dP[16];  // t in [g16, g16 + 16)
     {  // dX2 -> dP = -mask dX2, dKR = -Gam dX2; dX2 itself (fp32 [t][j]) for bwd_post,
        // staged in the free scratch tiles and bulk-copied
       float *stg = reinterpret_cast<float *>(sm + S0H);
-#pragma unroll
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      {
+        const int c0 = g16;
         float x[16], dkr[16], dp[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
-          dp[i] = ((m >> t) & 1ull) ? -x[i] : 0.f;
-          dP[t] = dp[i];
+          dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
+          dP[i] = dp[i];
           dkr[i] = -Gam[t] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dkr);
@@ -633,7 +644,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     if (tid == 0 && c > 0) load_mq(chunk - 1);
     {  // dR update (fp32 in TMEM); dE = dE_partial + Ap^T dP; dQS = Gam dO
 #pragma unroll 1
-      for (int c0 = 0; c0 < D; c0 += 16) {
+      for (int c0 = g16; c0 < D; c0 += 64) {
         float r[16], u[16];
         tmem_ld16(tm + lane + T_DR + c0, r);
         tmem_ld16(tm + lane + T_R1 + c0, u);
@@ -641,8 +652,8 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
         for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
         tmem_st16(tm + lane + T_DR + c0, r);
       }
-#pragma unroll
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      {
+        const int c0 = g16;
         float a[16], e[16], dqs[16];
         tmem_ld16(tm + lane + T_R4 + c0, a);
         tmem_ld16(tm + lane + T_R3 + c0, e);
@@ -672,16 +683,16 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
        // (bf16 [t][j]) staged in the free scratch tiles
       float *stg = reinterpret_cast<float *>(sm + S0H);
       __nv_bfloat16 *dvs = reinterpret_cast<__nv_bfloat16 *>(sm + S1H);
-#pragma unroll
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      {
+        const int c0 = g16;
         float x[16], dks[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
-          dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[t]);
-          dks[i] = Gprev[t] * dP[t] - Gam[t] * x[i];
+          dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
+          dks[i] = Gprev[t] * dP[i] - Gam[t] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
       }
@@ -691,7 +702,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
         bulk_s2g(P.dXbuf + chunk * 64 * D, sm + S0H, 32768);
         bulk_commit();
       }
-      for (int e = tid; e < 64 * 16; e += NT) {  // dv rows, 16 bytes at a time
+      for (int e = tid; e < 64 * 16; e += NTC) {  // dv rows, 16 bytes at a time
         const int t = e >> 4, chn = e & 15;
         if (t < n)
           *reinterpret_cast<uint4 *>(dv + ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8) =
@@ -714,7 +725,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     // dS update, and the carried gradients' tiles: the A operands of the next
     // chunk's phase A (the scratch tiles in their place are done with)
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], u[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
       tmem_ld16(tm + lane + T_R1 + c0, u);
@@ -728,7 +739,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_chain_kernel(TcBwdParams P) {
     fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   }
   if (ok) {
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
       tmem_ld16(tm + lane + T_DR + c0, r);
@@ -1471,7 +1482,7 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
     RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NT, ch::SMEM, s>>>(P));
+  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NTC, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   int dev = 0, nsm = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;

@@ -3,8 +3,11 @@
 //
 // Same chunk algebra as chunk_fwd.cu (see its header), computed in the
 // transposed orientation so that every product has the value dimension
-// d_v = 128 as its M dimension: TMEM lane j holds value column j, and thread
-// j of the CTA's 128 threads owns that column end to end.  Per chunk of 64
+// d_v = 128 as its M dimension: TMEM lane j holds value column j.  The CTA's
+// 16 warps form 4 groups of 128 threads; thread j of group g owns value
+// column j for the token columns t in [16g, 16g + 16) of the chunk (and the
+// state columns [16g, 16g + 16) and [64 + 16g, 80 + 16g)), so that the four
+// warps sharing a TMEM lane quadrant hide one another's latencies.  Per chunk of 64
 // tokens, with KQ = [K ; Q] (128 x d_k, exact bf16, unscaled):
 //
 //   MMA1  D1   = S^T  KQ^T          -> [KS | QS], rescaled in TMEM to
@@ -46,7 +49,9 @@ namespace {
 using namespace tc;
 
 constexpr int D = 128;
-constexpr int kTcThreads = 128;
+constexpr int kTcThreads = 512;
+constexpr int kGroups = kTcThreads / 128;  // threads sharing a value column
+static_assert(kGroups == 4, "each group owns 16 of a chunk's 64 token columns");
 
 // shared-memory carve-up (bytes from the 1024-aligned dynamic base)
 constexpr uint32_t SM_SA = 0;          // S^T bf16, 128 x 128, two 64-col blocks
@@ -136,7 +141,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   volatile int *flag = reinterpret_cast<volatile int *>(sm + SM_FLAG);
 
   const int tid = threadIdx.x, warp = tid >> 5;
-  const int j = tid;  // value column == TMEM lane
+  const int j = tid & 127;       // value column == TMEM lane
+  const int g16 = (warp >> 2) * 16;  // this thread's token (and state) columns start
   const int bh = blockIdx.x;
   const int b = bh / p.H, h = bh % p.H;
   const int T = p.T, H = p.H, NC = p.NC;
@@ -159,7 +165,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   __syncthreads();
   fence_after_sync();
   const uint32_t tm = *slot;
-  const uint32_t lane = (uint32_t)(warp * 32) << 16;
+  const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   uint32_t phase = 0, phA = 0, phB = 0;  // phA/phB: tracked by thread 0 only
   auto rec_of = [&](int c) {
     return reinterpret_cast<const uint8_t *>(p.ws + ((size_t)bh * NC + c) * kRecFloats);
@@ -204,7 +210,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   fetch_kq(0);
 
   // initial states -> TMEM (fp32) and bf16 A operands
-  for (int c0 = 0; c0 < D; c0 += 16) {
+  for (int c0 = g16; c0 < D; c0 += 64) {
     float s[16], r[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -243,7 +249,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return *flag == 0;
   };
 
-  float rres[64];  // clipped residual r[t] of column j
+  float rres[16];  // clipped residual r[t] of column j, t in [g16, g16 + 16)
   bool alive = true;
   for (int c = 0; c < NC && alive; ++c) {
     const int t0 = c * 64;
@@ -276,7 +282,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     });
     if (!alive) break;
     // the products below accumulate onto Gprev * KS (-> P) and Gam * scale * QS (-> Ob)
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
       float x[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, x);
 #pragma unroll
@@ -285,7 +292,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
 
     // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
       float ks[16], x[16];
       tmem_ld16(tm + lane + T_D1 + c0, ks);
 #pragma unroll
@@ -310,7 +318,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (d) E -> EA, wS*E -> WA;  MMA3: D1 += E^T [Ap;Mq]^T,  MMA4: U = (wS E)^T K
     const size_t ci = (size_t)bh * NC + c;  // chunk index of the saved intermediates
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_X + c0, e);
@@ -343,21 +352,22 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (tid == 0) load_slot(sm + SM_SLOTB, barB, rec_of(c) + IMG_M2, 16384);
 
     // ---- (e) r = clip(V - P); S = Gam_C S + U (fp32 in TMEM, bf16 copy in SA)
-    unsigned long long msk = 0ull;  // bit t: |x| <= c (the clip passes the gradient)
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
+      unsigned msk = 0u;  // bit i: |x| <= c at t = c0 + i (the clip passes the gradient)
       float pp[16];
       tmem_ld16(tm + lane + T_D1 + c0, pp);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const float x = vs(c0 + i) - pp[i];
-        if (fabsf(x) <= clip) msk |= 1ull << (c0 + i);
-        rres[c0 + i] = clampf(x, clip);
+        if (fabsf(x) <= clip) msk |= 1u << i;
+        rres[i] = clampf(x, clip);
       }
+      // bits [c0, c0 + 16) of the column's 64-bit mask word (little-endian)
+      if (p.sv_mask) reinterpret_cast<uint16_t *>(p.sv_mask + ci * D + j)[c0 >> 4] = (uint16_t)msk;
     }
-    if (p.sv_mask) p.sv_mask[ci * D + j] = msk;
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], u[16];
       tmem_ld16(tm + lane + T_S + c0, s);
       tmem_ld16(tm + lane + T_X + c0, u);
@@ -382,12 +392,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (f) X2 = r - Gam KR;  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
     if (RDNV) {
-#pragma unroll
-      for (int c0 = 0; c0 < 64; c0 += 16) {
+      {
+        const int c0 = g16;
         float x[16];
         tmem_ld16(tm + lane + T_X + c0, x);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = rres[c0 + i] - Gam[c0 + i] * x[i];
+        for (int i = 0; i < 16; ++i) x[i] = rres[i] - Gam[c0 + i] * x[i];
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
       }
       alive = run_phase([&] {
@@ -402,14 +412,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
 
     // ---- (g) E2 -> EA, wR*E2 -> WA;  MMA7: Ob += E2^T (gamma M2)^T;  MMA8: U2 = (wR E2)^T K
-#pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
       float e[16], w[16];
       if (RDNV) {
         tmem_ld16(tm + lane + T_D1 + c0, e);
       } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) e[i] = rres[c0 + i];
+        for (int i = 0; i < 16; ++i) e[i] = rres[i];
       }
 #pragma unroll
       for (int i = 0; i < 16; ++i) w[i] = wR[c0 + i] * e[i];
@@ -441,8 +451,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     // o is staged as a [t][j] bf16 tile in W's place (free after MMA8) and stored
     // 16 bytes at a time
     __nv_bfloat16 *ostg = reinterpret_cast<__nv_bfloat16 *>(sm + SM_W);
-#pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    {
+      const int c0 = g16;
       float ob[16], oa[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);
       tmem_ld16(tm + lane + T_X + 64 + c0, oa);
@@ -453,7 +463,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       }
     }
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float r[16], u[16];
       tmem_ld16(tm + lane + T_R + c0, r);
       tmem_ld16(tm + lane + (c0 < 64 ? T_D1 + c0 : T_X + c0 - 64), u);
@@ -477,7 +487,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
   if (tid == 0 && p.sv_E) bulk_wait_all();
   if (alive) {  // final states
-    for (int c0 = 0; c0 < D; c0 += 16) {
+    for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], r[16];
       tmem_ld16(tm + lane + T_S + c0, s);
       tmem_ld16(tm + lane + T_R + c0, r);
