@@ -97,6 +97,21 @@ __device__ __forceinline__ void put16s(uint8_t *hi, uint8_t *lo, int r, int c0,
   put16(hi, 0, r, c0, a);
   put16(lo, 0, r, c0, b);
 }
+// the same for 8 values (one 16-byte chunk of each tile)
+__device__ __forceinline__ void put8s(uint8_t *hi, uint8_t *lo, int r, int c0,
+                                      const float (&v)[8]) {
+  float a[8], b[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
+    b[i] = v[i] - a[i];
+  }
+  uint4 x, y;
+  x.x = pack2(a[0], a[1]); x.y = pack2(a[2], a[3]); x.z = pack2(a[4], a[5]); x.w = pack2(a[6], a[7]);
+  y.x = pack2(b[0], b[1]); y.y = pack2(b[2], b[3]); y.z = pack2(b[4], b[5]); y.w = pack2(b[6], b[7]);
+  *reinterpret_cast<uint4 *>(hi + sw128(r, c0)) = x;
+  *reinterpret_cast<uint4 *>(lo + sw128(r, c0)) = y;
+}
 // K-major A (single block, K = 64) times MN-major B, split both: 3 products
 __device__ __forceinline__ void mma_s3_kmn(uint32_t d, uint32_t a_hi, uint32_t a_lo,
                                            uint32_t b_hi, uint32_t b_lo, uint32_t b_lbo,
@@ -761,9 +776,9 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
 // ======================================================================== 3
 // bwd_post: everything that reduces over the value dimension, followed by the
 // chunk-matrix part of the gradients (the work bwd_finish of chunk_bwd.cu does
-// for the SIMT path), one chunk per CTA of 256 threads.  Thread (j, hf) owns
-// value column j = TMEM lane j and half hf of the chunk's tokens (or of the
-// key rows of a state).
+// for the SIMT path), one persistent CTA of 512 threads per SM walking the
+// chunks.  Thread (j, qd) owns value column j = TMEM lane j and quarter qd of
+// the chunk's tokens (or of the key rows of a state).
 //
 // dK and dQ are accumulated transposed in TMEM (lane = key dimension d,
 // column t for dK_t, 64 + t for dQ_t):
@@ -775,13 +790,13 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
 // Q enters the tensor-core products unscaled; the scale is applied to the
 // fp32 results.
 namespace po {
-constexpr int NTP = 256;
+constexpr int NTP = 512;
 constexpr uint32_t SA = 0, SB = 65536;  // state images: hi 2 x 16 KB | lo 2 x 16 KB, rows j
 constexpr uint32_t XH = 131072, XL = 147456, YH = 163840, YL = 180224;  // [j][t] atoms
 constexpr uint32_t KQ = 196608;         // K rows 0..63, Q rows 64..127, 2 x 16 KB
 constexpr uint32_t VEC = 229376;        // Gam Gprev wS wR gamma dGam dGprev (7 x 64), dGamC
-constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // 8 warps x 32 floats
-constexpr uint32_t CTL = RED + 8 * 32 * 4;
+constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // 16 warps x 16 floats
+constexpr uint32_t CTL = RED + 16 * 16 * 4;
 constexpr uint32_t SLOT = CTL + 48;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
@@ -789,24 +804,27 @@ static_assert(SMEM <= 232448, "shared memory");
 constexpr int LDC = 65, TILE = 64 * LDC;
 constexpr int F_DM2 = 0, F_DMQ = TILE, F_DAB = 2 * TILE, F_KK = 3 * TILE, F_DAG = 4 * TILE,
               F_DAP = 5 * TILE, F_QK = 6 * TILE, F_VEC = 7 * TILE;
-static_assert((F_VEC + 9 * 64 + 6 * 4 * 64) * 4 <= (int)XH, "finish scratch");
+static_assert((F_VEC + 9 * 64 + 6 * 8 * 64) * 4 <= (int)XH, "finish scratch");
 // TMEM columns
 constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
 constexpr uint32_t T_KDR = 0, T_KDS = 64, T_U1 = 128, T_U2 = 192;  // P4, after the read-outs
 constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
 }  // namespace po
 
-// Sums over the 128 value columns: thread (j, hf) holds v[t - 32 hf] for the
-// tokens t of its half; out[t] for t in [0, 64).
-__device__ __forceinline__ void cta_row_sum256(const float (&v)[32], float *red, float *out,
+// Sums over the 128 value columns: thread (j, qd) holds v[t - 16 qd] for the
+// tokens t of its quarter; out[t] for t in [0, 64).  Warp 4 qd + w covers
+// columns [32 w, 32 w + 32); after the warp's transposed reduction lane 2 i
+// holds its sum for token 16 qd + i.
+__device__ __forceinline__ void cta_row_sum512(const float (&v)[16], float *red, float *out,
                                                int tid) {
-  const float o = warp_transpose_reduce32(v);
-  red[tid] = o;  // red[warp * 32 + lane]
+  const float o = warp_transpose_reduce16(v);
+  const int warp = tid >> 5, lane = tid & 31;
+  if (!(lane & 1)) red[warp * 16 + (lane >> 1)] = o;
   __syncthreads();
   if (tid < 64) {
-    const int hh = tid >> 5, l = tid & 31;
-    out[tid] = red[(4 * hh) * 32 + l] + red[(4 * hh + 1) * 32 + l] + red[(4 * hh + 2) * 32 + l] +
-               red[(4 * hh + 3) * 32 + l];
+    const int g = tid >> 4, i = tid & 15;
+    out[tid] = red[(4 * g) * 16 + i] + red[(4 * g + 1) * 16 + i] + red[(4 * g + 2) * 16 + i] +
+               red[(4 * g + 3) * 16 + i];
   }
   __syncthreads();
 }
@@ -826,7 +844,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   float *red = reinterpret_cast<float *>(sm + RED);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int j = tid & 127, hf = tid >> 7, tb = 32 * hf;
+  const int j = tid & 127, qd = tid >> 7, tb = 16 * qd;
   const int NC = p.NC, T = p.T, H = p.H;
   const size_t nct = (size_t)p.B * H * NC;
   const float scale = p.scale;
@@ -884,48 +902,47 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const uint8_t *gimg = P.gimg + chunk * 131072;  // dS hi | dR hi | dS lo | dR lo
   // this thread's tokens of dX2, dX (from the staging) and dO: read after P1 is
   // issued, so that the MMA issue does not wait behind them
-  float x2v[32], xv[32], dov[32];
+  float x2v[16], xv[16], dov[16];
+  // this thread's key rows of a state: [32 qd, 32 qd + 32), the columns
+  // [32 (qd & 1), +32) of 64-row block qd >> 1 of the image
+  const uint32_t kblk = (uint32_t)(qd >> 1) * 16384u;
+  const int kc0 = 32 * (qd & 1);
   // fp32 [i][j] state staged at `base` -> rows j of its (hi | lo) image at
-  // `base`, key rows of half hf (every thread reads its values before any writes)
+  // `base` (every thread reads its values before any writes)
   auto stage_to_image = [&](uint32_t base) {
     const float *st = reinterpret_cast<const float *>(sm + base);
-    float v[64];
+    float v[32];
 #pragma unroll
-    for (int i = 0; i < 64; ++i) v[i] = st[(64 * hf + i) * D + j];
+    for (int i = 0; i < 32; ++i) v[i] = st[(32 * qd + i) * D + j];
     __syncthreads();
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 16) {
+    for (int c0 = 0; c0 < 32; c0 += 16) {
       float w[16];
 #pragma unroll
       for (int i = 0; i < 16; ++i) w[i] = v[c0 + i];
-      put16s(sm + base + hf * 16384, sm + base + 32768 + hf * 16384, j, c0, w);
+      put16s(sm + base + kblk, sm + base + 32768 + kblk, j, kc0 + c0, w);
     }
   };
   // sum over this thread's entries of (image at base, hi + lo) * x[i][j]
-  auto dot_image = [&](uint32_t base, const float (&x)[64]) {
+  auto dot_image = [&](uint32_t base, const float (&x)[32]) {
     float s = 0.f;
 #pragma unroll
-    for (int c8 = 0; c8 < 8; ++c8) {
-      const uint32_t o = base + hf * 16384 + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
+    for (int k8 = 0; k8 < 4; ++k8) {
+      const int c8 = (kc0 >> 3) + k8;
+      const uint32_t o = base + kblk + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
       const uint4 hv = *reinterpret_cast<const uint4 *>(sm + o);
       const uint4 lv = *reinterpret_cast<const uint4 *>(sm + o + 32768);
       const __nv_bfloat16 *hb = reinterpret_cast<const __nv_bfloat16 *>(&hv);
       const __nv_bfloat16 *lb = reinterpret_cast<const __nv_bfloat16 *>(&lv);
 #pragma unroll
       for (int e = 0; e < 8; ++e)
-        s += (__bfloat162float(hb[e]) + __bfloat162float(lb[e])) * x[c8 * 8 + e];
+        s += (__bfloat162float(hb[e]) + __bfloat162float(lb[e])) * x[k8 * 8 + e];
     }
     return s;
   };
-  // this thread's 32 tokens of a [j][t] atom pair (hi, lo)
-  auto put_tok = [&](const float (&x)[32], uint32_t hi, uint32_t lo) {
-#pragma unroll 1  // one copy of the conversion code per call site
-    for (int h2 = 0; h2 < 2; ++h2) {
-      float w[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) w[i] = h2 ? x[16 + i] : x[i];
-      put16s(sm + hi, sm + lo, j, tb + 16 * h2, w);
-    }
+  // this thread's 16 tokens of a [j][t] atom pair (hi, lo)
+  auto put_tok = [&](const float (&x)[16], uint32_t hi, uint32_t lo) {
+    put16s(sm + hi, sm + lo, j, tb, x);
   };
   const uint32_t tm_lane = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
@@ -946,7 +963,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // while P1 runs: this thread's dO, the gate vectors, dX2 and dX from their staging
   const unsigned long long m = P.mask[chunk * D + j] >> tb;
 #pragma unroll
-  for (int i = 0; i < 32; ++i) {
+  for (int i = 0; i < 16; ++i) {
     const int t = tb + i;
     dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
   }
@@ -962,7 +979,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     const float *x2s = reinterpret_cast<const float *>(sm + XH);
     const float *xs = reinterpret_cast<const float *>(sm + YH);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       x2v[i] = x2s[(tb + i) * D + j];
       xv[i] = xs[(tb + i) * D + j];
     }
@@ -970,50 +987,39 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   ok = phase_wait(K);  // (its barrier also publishes the gate vectors)
   auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
-    float rv[32];
+    float rv[16];
     {  // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
+      float qr[16];
+      tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
 #pragma unroll
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float qr[16];
-        tmem_ld16(tm + tm_lane + T_KR + 64 + tb + c0, qr);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) rv[c0 + i] = scale * Gam[tb + c0 + i] * dov[c0 + i] * qr[i];
-      }
-      cta_row_sum256(rv, red, dGamS, tid);
+      for (int i = 0; i < 16; ++i) rv[i] = scale * Gam[tb + i] * dov[i] * qr[i];
+      cta_row_sum512(rv, red, dGamS, tid);
       // parked in the record's slot (shared memory is full); the same thread reads it back
       if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
       __syncthreads();
     }
-#pragma unroll
-    for (int c0 = 0; c0 < 32; c0 += 16) {
+    {
       float qs[16], qr[16];
-      tmem_ld16(tm + tm_lane + T_KS + 64 + tb + c0, qs);
-      tmem_ld16(tm + tm_lane + T_KR + 64 + tb + c0, qr);
+      tmem_ld16(tm + tm_lane + T_KS + 64 + tb, qs);
+      tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
 #pragma unroll
-      for (int i = 0; i < 16; ++i)
-        rv[c0 + i] = scale * dov[c0 + i] * (qs[i] + gamv[tb + c0 + i] * qr[i]);
+      for (int i = 0; i < 16; ++i) rv[i] = scale * dov[i] * (qs[i] + gamv[tb + i] * qr[i]);
     }
-#pragma unroll
-    for (int c0 = 0; c0 < 32; c0 += 16) {
+    {
       float ks[16], kr[16];
-      tmem_ld16(tm + tm_lane + T_KS + tb + c0, ks);
-      tmem_ld16(tm + tm_lane + T_KR + tb + c0, kr);
+      tmem_ld16(tm + tm_lane + T_KS + tb, ks);
+      tmem_ld16(tm + tm_lane + T_KR + tb, kr);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[c0 + i] -= x2v[c0 + i] * kr[i] + xv[c0 + i] * ks[i];
+      for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
+      cta_row_sum512(rv, red, dGamS, tid);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) rv[i] = dp_of(i) * ks[i];
     }
-    cta_row_sum256(rv, red, dGamS, tid);
-#pragma unroll
-    for (int c0 = 0; c0 < 32; c0 += 16) {
-      float ks[16];
-      tmem_ld16(tm + tm_lane + T_KS + tb + c0, ks);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) rv[c0 + i] = dp_of(c0 + i) * ks[i];
-    }
-    cta_row_sum256(rv, red, dGprevS, tid);
+    cta_row_sum512(rv, red, dGprevS, tid);
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
-    float x[32], y[32];
+    float x[16], y[16];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       const int t = tb + i;
       x[i] = -Gam[t] * x2v[i];
       y[i] = Gam[t] * gamv[t] * dov[i];
@@ -1033,9 +1039,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     bulk_g2s(sm + SB + 32768, gimg + 98304, 32768, K.barB);
   }
   if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO
-    float x[32], y[32];
+    float x[16], y[16];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       const int t = tb + i;
       x[i] = Gprev[t] * dp_of(i) - Gam[t] * xv[i];
       y[i] = Gam[t] * dov[i];
@@ -1062,9 +1068,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll 1
     for (int s2 = 0; s2 < 2; ++s2) {
       const float *st = s2 ? S0 : R0;
-      float x[64];
+      float x[32];
 #pragma unroll
-      for (int i = 0; i < 64; ++i) x[i] = st[(size_t)(64 * hf + i) * D + j];
+      for (int i = 0; i < 32; ++i) x[i] = st[(size_t)(32 * qd + i) * D + j];
       if (!mbar_wait(s2 ? K.barA : K.barB, s2 ? 1u : (it & 1u))) *K.flag = 1;
       gdot += dot_image(s2 ? SA : SB, x);
     }
@@ -1078,10 +1084,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       *dGamC = s;
     }
   }
-  // this thread's 32 tokens of row j of a (hi | lo) image of a [j][t] matrix
-  auto image_row = [&](uint32_t base, float (&out)[32]) {
+  // this thread's 16 tokens of row j of a (hi | lo) image of a [j][t] matrix
+  auto image_row = [&](uint32_t base, float (&out)[16]) {
 #pragma unroll
-    for (int k8 = 0; k8 < 4; ++k8) {
+    for (int k8 = 0; k8 < 2; ++k8) {
       const int c8 = (tb >> 3) + k8;
       const uint32_t o = base + j * 128 + (((c8 ^ (j & 7)) & 7) << 4);
       const uint4 hv = *reinterpret_cast<const uint4 *>(sm + o);
@@ -1111,33 +1117,28 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   if (ok) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
-#pragma unroll 1
-    for (int c0 = 0; c0 < 32; c0 += 16) {
+    {
       float a[16], u1[16], u2[16];
-      tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);
-      tmem_ld16(tm + tm_lane + T_U1 + tb + c0, u1);
-      tmem_ld16(tm + tm_lane + T_U2 + tb + c0, u2);
+      tmem_ld16(tm + tm_lane + T_DKQ + tb, a);
+      tmem_ld16(tm + tm_lane + T_U1 + tb, u1);
+      tmem_ld16(tm + tm_lane + T_U2 + tb, u2);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const int t = tb + c0 + i;
+        const int t = tb + i;
         a[i] = fmaf(wR[t], u1[i], fmaf(wS[t], u2[i], a[i]));
       }
-      tmem_st16(tm + tm_lane + T_DKQ + tb + c0, a);
+      tmem_st16(tm + tm_lane + T_DKQ + tb, a);
     }
     // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
 #pragma unroll 1
     for (int w = 0; w < 2; ++w) {
-      float ev[32], rv[32];
+      float ev[16], rv[16];
       image_row(w == 0 ? XH : YH, ev);
+      tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb, rv);
 #pragma unroll
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float kd[16];
-        tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb + c0, kd);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) rv[c0 + i] = kd[i] * ev[c0 + i];
-      }
+      for (int i = 0; i < 16; ++i) rv[i] *= ev[i];
       // parked in the record's slots (shared memory is full); read in the gate pass
-      cta_row_sum256(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
+      cta_row_sum512(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
     }
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
@@ -1162,9 +1163,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     });
   }
   if (ok) {
-    float y[32];
+    float y[16];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) y[i] = dp_of(i);
+    for (int i = 0; i < 16; ++i) y[i] = dp_of(i);
     put_tok(y, SA + 32768, SA + 49152);  // [dO ; dP]: the dO atom is still in place
     ok = phase_run(K, tid, [&] {
       mma_tile_mnmn<true>(tm + T_G2, sb + SA, 32768, sb + YH, 16384, 8, i64, false);
@@ -1178,21 +1179,20 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   float *F = reinterpret_cast<float *>(sm);
   float *cum = F + F_VEC, *cprev = cum + 64, *bet = cum + 128, *gam = cum + 192, *gg = cum + 256,
         *dcum = cum + 320, *dcprev = cum + 384, *dbet = cum + 448, *dgam = cum + 512;
-  float *prt = cum + 576;  // [6][4][64] partial sums
+  float *prt = cum + 576;  // [6][8][64] partial sums
   float o_dg = 0.f, o_dbeta = 0.f, o_dgamma = 0.f;  // this thread's token's gate gradients
   if (ok) {
     {
       const int r = j & 63;
-#pragma unroll 1
-      for (int c0 = 0; c0 < 32; c0 += 16) {
+      {
         float g1[16], g2[16], g3[16], gr[16];
-        tmem_ld16(tm + tm_lane + T_G1 + tb + c0, g1);
-        tmem_ld16(tm + tm_lane + T_G2 + tb + c0, g2);
-        tmem_ld16(tm + tm_lane + T_G3 + tb + c0, g3);
-        tmem_ld16(tm + tm_lane + T_GR + tb + c0, gr);
+        tmem_ld16(tm + tm_lane + T_G1 + tb, g1);
+        tmem_ld16(tm + tm_lane + T_G2 + tb, g2);
+        tmem_ld16(tm + tm_lane + T_G3 + tb, g3);
+        tmem_ld16(tm + tm_lane + T_GR + tb, gr);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int e = r * LDC + tb + c0 + i;
+          const int e = r * LDC + tb + i;
           if (j < 64) {
             F[F_DM2 + e] = g1[i];
             F[F_DMQ + e] = g2[i];
@@ -1237,14 +1237,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       cprev[32 + lane] = a2 - gg[32 + lane];
     }
     __syncthreads();
-    {  // row pass: thread (t, quarter) over i in [16 q, 16 q + 16)
-      const int t = tid & 63, q4 = tid >> 6;
+    {  // row pass: thread (t, eighth) over i in [8 q8, 8 q8 + 8)
+      const int t = tid & 63, q8 = tid >> 6;
       const float ct = cum[t], cpt = cprev[t];
       const float gt = gam[t];
       float rowc = 0.f, rowp = 0.f, dgo = 0.f;
 #pragma unroll 1
-      for (int ii = 0; ii < 16; ++ii) {
-        const int i = 16 * q4 + ii, e = t * LDC + i;
+      for (int ii = 0; ii < 8; ++ii) {
+        const int i = 8 * q8 + ii, e = t * LDC + i;
         float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
         if (i <= t) {
           const float dec = __expf(ct - cum[i]);
@@ -1294,33 +1294,36 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         F[F_DMQ + e] = cb;
         F[F_DAB + e] = cm;
       }
-      prt[0 * 256 + q4 * 64 + t] = rowc;
-      prt[1 * 256 + q4 * 64 + t] = rowp;
-      prt[5 * 256 + q4 * 64 + t] = dgo;
+      prt[0 * 512 + q8 * 64 + t] = rowc;
+      prt[1 * 512 + q8 * 64 + t] = rowp;
+      prt[5 * 512 + q8 * 64 + t] = dgo;
     }
     __syncthreads();
-    {  // column pass: thread (i, quarter) over t in [16 q, 16 q + 16)
-      const int i = tid & 63, q4 = tid >> 6;
+    {  // column pass: thread (i, eighth) over t in [8 q8, 8 q8 + 8)
+      const int i = tid & 63, q8 = tid >> 6;
       float sg = 0.f, sbv = 0.f, smv = 0.f;
-#pragma unroll 1
-      for (int tt = 0; tt < 16; ++tt) {
-        const int e = (16 * q4 + tt) * LDC + i;
+#pragma unroll
+      for (int tt = 0; tt < 8; ++tt) {
+        const int e = (8 * q8 + tt) * LDC + i;
         sg += F[F_DM2 + e];
         sbv += F[F_DMQ + e];
         smv += F[F_DAB + e];
       }
-      prt[2 * 256 + q4 * 64 + i] = sg;
-      prt[3 * 256 + q4 * 64 + i] = sbv;
-      prt[4 * 256 + q4 * 64 + i] = smv;
+      prt[2 * 512 + q8 * 64 + i] = sg;
+      prt[3 * 512 + q8 * 64 + i] = sbv;
+      prt[4 * 512 + q8 * 64 + i] = smv;
     }
     __syncthreads();
     if (tid < 64) {
       const int i = tid;
       float s5[6];
 #pragma unroll
-      for (int w = 0; w < 6; ++w)
-        s5[w] = prt[w * 256 + i] + prt[w * 256 + 64 + i] + prt[w * 256 + 128 + i] +
-                prt[w * 256 + 192 + i];
+      for (int w = 0; w < 6; ++w) {
+        float a = 0.f;
+#pragma unroll
+        for (int q8 = 0; q8 < 8; ++q8) a += prt[w * 512 + q8 * 64 + i];
+        s5[w] = a;
+      }
       const float cC = cum[63];
       const float eC = __expf(cC - cum[i]);
       const float dwS = acc[A8::V_DWS + i], dwR = acc[A8::V_DWR + i];
@@ -1360,16 +1363,16 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       gg[31 - lane] = a2 + (pb - dcprev[31 - lane]);
     }
     {  // B operand [dKK + dKK^T ; dQK] (rows t, columns i), hi | lo
-      const int t = tid & 63, q4 = tid >> 6;
-      float v[16], w[16];
+      const int t = tid & 63, q8 = tid >> 6;
+      float v[8], w[8];
 #pragma unroll
-      for (int ii = 0; ii < 16; ++ii) {
-        const int i = 16 * q4 + ii;
+      for (int ii = 0; ii < 8; ++ii) {
+        const int i = 8 * q8 + ii;
         v[ii] = i == t ? 2.f * F[F_KK + t * LDC + t] : F[F_KK + t * LDC + i] + F[F_KK + i * LDC + t];
         w[ii] = F[F_QK + t * LDC + i];
       }
-      put16s(sm + XH, sm + XL, t, 16 * q4, v);
-      put16s(sm + XH, sm + XL, 64 + t, 16 * q4, w);
+      put8s(sm + XH, sm + XL, t, 8 * q8, v);
+      put8s(sm + XH, sm + XL, 64 + t, 8 * q8, w);
     }
     // ---- P7: dK, dQ += K^T [dKK + dKK^T ; dQK]^T ; D2 = Q^T dQK
     phase_issue(K, tid, [&] {
@@ -1397,15 +1400,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       P.dgamma[off] = o_dgamma;
     }
     __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
-#pragma unroll 1
-    for (int c0 = 0; c0 < 32; c0 += 16) {
+    {
       float a[16], d2[16], qv[16];
-      tmem_ld16(tm + tm_lane + T_DKQ + tb + c0, a);
-      tmem_ld16(tm + tm_lane + T_D2 + tb + c0, d2);
-      tmem_ld16(tm + tm_lane + T_DKQ + 64 + tb + c0, qv);
+      tmem_ld16(tm + tm_lane + T_DKQ + tb, a);
+      tmem_ld16(tm + tm_lane + T_D2 + tb, d2);
+      tmem_ld16(tm + tm_lane + T_DKQ + 64 + tb, qv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const int t = tb + c0 + i;
+        const int t = tb + i;
         if (t < n) {
           const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + j;
           dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);

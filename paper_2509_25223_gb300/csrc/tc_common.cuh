@@ -370,6 +370,30 @@ __device__ __forceinline__ float warp_transpose_reduce32(const float (&v)[32]) {
   return (hi ? d[1] : d[0]) + __shfl_xor_sync(0xffffffffu, hi ? d[0] : d[1], 1);
 }
 
+// The same for v[16]: afterwards lanes 2 i and 2 i + 1 hold the warp sum of v[i].
+__device__ __forceinline__ float warp_transpose_reduce16(const float (&v)[16]) {
+  const int lane = threadIdx.x & 31;
+  float a[8], b[4], c[2];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const bool hi = lane & 16;
+    a[k] = (hi ? v[8 + k] : v[k]) + __shfl_xor_sync(0xffffffffu, hi ? v[k] : v[8 + k], 16);
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const bool hi = lane & 8;
+    b[k] = (hi ? a[4 + k] : a[k]) + __shfl_xor_sync(0xffffffffu, hi ? a[k] : a[4 + k], 8);
+  }
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const bool hi = lane & 4;
+    c[k] = (hi ? b[2 + k] : b[k]) + __shfl_xor_sync(0xffffffffu, hi ? b[k] : b[2 + k], 4);
+  }
+  const bool hi = lane & 2;
+  const float d = (hi ? c[1] : c[0]) + __shfl_xor_sync(0xffffffffu, hi ? c[0] : c[1], 2);
+  return d + __shfl_xor_sync(0xffffffffu, d, 1);
+}
+
 __device__ __forceinline__ int transpose_reduce_tbase(int lane) {
   return ((lane >> 4) & 1) * 32 + ((lane >> 3) & 1) * 16 + ((lane >> 2) & 1) * 8 +
          ((lane >> 1) & 1) * 4 + (lane & 1) * 2;
