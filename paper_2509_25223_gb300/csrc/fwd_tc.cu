@@ -249,11 +249,32 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return *flag == 0;
   };
 
+  // L2 prefetch of a chunk's record and V, K, Q rows and gammas, one chunk
+  // ahead of the cp.async and bulk copies that read them
+  auto prefetch_chunk = [&](int c) {
+    const int t0_ = c * 64, n_ = min(64, T - t0_);
+    if (tid == 0) {
+      const uint8_t *r = rec_of(c);
+      static_assert((kRecFloats * 4) % 16 == 0 && kRecFloats * 4 > 65536, "record");
+      prefetch_l2_bulk(r, 65536);
+      prefetch_l2_bulk(r + 65536, kRecFloats * 4 - 65536);
+    }
+    if (tid < 384) {
+      const int rr = tid >> 1, t = rr & 63, w = rr >> 6;
+      const __nv_bfloat16 *src = w == 0 ? v : (w == 1 ? k : q);
+      if (t < n_) prefetch_l2_line(src + ((size_t)(b * T + t0_ + t) * H + h) * D + (tid & 1) * 64);
+    } else if (tid < 416) {
+      const int t = 2 * (tid - 384);
+      if (t < n_) prefetch_l2_line(p.gamma + (size_t)(b * T + t0_ + t) * H + h);
+    }
+  };
+
   float rres[16];  // clipped residual r[t] of column j, t in [g16, g16 + 16)
   bool alive = true;
   for (int c = 0; c < NC && alive; ++c) {
     const int t0 = c * 64;
     const int n = min(64, T - t0);
+    if (c + 1 < NC) prefetch_chunk(c + 1);
     const float *rec = p.ws + ((size_t)bh * NC + c) * kRecFloats;
     cp_async_wait_all();  // this chunk's V, K, Q tiles (fetched during the previous chunk)
     __syncthreads();      // every thread is done with the previous chunk's tiles and vectors
