@@ -213,6 +213,11 @@ __device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t saddr, uint32_t lbo)
   return d;
 }
 
+// A byte offset as an increment of a descriptor's start-address field (the
+// field holds address / 16 in 14 bits; shared-memory addresses stay below
+// 256 KB, so an in-range offset never carries out of it).
+__device__ __forceinline__ uint64_t desc_off(uint32_t bytes) { return (uint64_t)(bytes >> 4); }
+
 constexpr uint32_t kAMajorMN = 1u << 15, kBMajorMN = 1u << 16;
 
 // D[tmem] (+)= A * B^T for one K = 16 slice, issued by one thread.
@@ -248,8 +253,17 @@ __device__ __forceinline__ void mma_tile_kmn(uint32_t d_tmem, uint32_t a_base, u
              idesc | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
   };
   if constexpr (kRolled) {
+    const uint64_t a0 = sdesc_sw128(a_base), b0 = sdesc_sw128_mn(b_base, b_lbo);
 #pragma unroll 1
-    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+    for (int kb = 0; kb < ksteps; kb += 4) {
+      const uint64_t a = a0 + desc_off((uint32_t)(kb >> 2) * a_blk);
+      const uint64_t b = b0 + desc_off((uint32_t)kb * 2048u);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (kb + j < ksteps)
+          mma_bf16(d_tmem, a + desc_off(32u * j), b + desc_off(2048u * j), idesc | kBMajorMN,
+                   (kb + j > 0 || accumulate_first) ? 1u : 0u);
+    }
   } else {
 #pragma unroll
     for (int kk = 0; kk < ksteps; ++kk) step(kk);
@@ -267,9 +281,13 @@ __device__ __forceinline__ void mma_tile_mnk(uint32_t d_tmem, uint32_t a_base, u
              sdesc_sw128(b_base + (uint32_t)kk * 32u), idesc | kAMajorMN,
              (kk > 0 || accumulate_first) ? 1u : 0u);
   };
-  if constexpr (kRolled) {
-#pragma unroll 1
-    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+  if constexpr (kRolled) {  // ksteps <= 4: one group
+    const uint64_t a0 = sdesc_sw128_mn(a_base, a_lbo), b0 = sdesc_sw128(b_base);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (j < ksteps)
+        mma_bf16(d_tmem, a0 + desc_off(2048u * j), b0 + desc_off(32u * j), idesc | kAMajorMN,
+                 (j > 0 || accumulate_first) ? 1u : 0u);
   } else {
 #pragma unroll
     for (int kk = 0; kk < ksteps; ++kk) step(kk);
@@ -288,8 +306,16 @@ __device__ __forceinline__ void mma_tile_mnmn(uint32_t d_tmem, uint32_t a_base, 
              idesc | kAMajorMN | kBMajorMN, (kk > 0 || accumulate_first) ? 1u : 0u);
   };
   if constexpr (kRolled) {
+    const uint64_t a0 = sdesc_sw128_mn(a_base, a_lbo), b0 = sdesc_sw128_mn(b_base, b_lbo);
 #pragma unroll 1
-    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+    for (int kb = 0; kb < ksteps; kb += 4) {
+      const uint64_t a = a0 + desc_off((uint32_t)kb * 2048u), b = b0 + desc_off((uint32_t)kb * 2048u);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (kb + j < ksteps)
+          mma_bf16(d_tmem, a + desc_off(2048u * j), b + desc_off(2048u * j),
+                   idesc | kAMajorMN | kBMajorMN, (kb + j > 0 || accumulate_first) ? 1u : 0u);
+    }
   } else {
 #pragma unroll
     for (int kk = 0; kk < ksteps; ++kk) step(kk);
@@ -416,8 +442,11 @@ __device__ __forceinline__ uint32_t sw128(int r, int c) {
   return (uint32_t)(r * 128 + ((((c >> 3) ^ (r & 7)) & 7) << 4) + (c & 7) * 2);
 }
 
-// (kRolled: one issue loop per call site instead of an unrolled sequence --
-// for kernels whose straight-line code would not stay in the instruction cache.)
+// (kRolled: a loop over groups of 4 K-steps per call site instead of an
+// unrolled sequence -- for kernels whose straight-line code would not stay in
+// the instruction cache.  The descriptors are built once and advanced by
+// adding to their address field, so that the issuing thread keeps up with the
+// tensor pipe: rebuilding both per step costs about 90 cycles an MMA.)
 // Issue D = A * B^T over K = 16 * ksteps for K-major SW128 tiles A [M][K] and
 // B [N][K] stored as consecutive 64-column blocks (a_blk / b_blk bytes apart).
 template <bool kRolled = false>
@@ -432,8 +461,17 @@ __device__ __forceinline__ void mma_tile(uint32_t d_tmem, uint32_t a_base, uint3
              (kk > 0 || accumulate_first) ? 1u : 0u);
   };
   if constexpr (kRolled) {
+    const uint64_t a0 = sdesc_sw128(a_base), b0 = sdesc_sw128(b_base);
 #pragma unroll 1
-    for (int kk = 0; kk < ksteps; ++kk) step(kk);
+    for (int kb = 0; kb < ksteps; kb += 4) {
+      const uint64_t a = a0 + desc_off((uint32_t)(kb >> 2) * a_blk);
+      const uint64_t b = b0 + desc_off((uint32_t)(kb >> 2) * b_blk);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (kb + j < ksteps)
+          mma_bf16(d_tmem, a + desc_off(32u * j), b + desc_off(32u * j), idesc,
+                   (kb + j > 0 || accumulate_first) ? 1u : 0u);
+    }
   } else {
 #pragma unroll
     for (int kk = 0; kk < ksteps; ++kk) step(kk);
