@@ -389,29 +389,59 @@ def run_ours(args):
             "algorithmic_flop_per_launch": dom_flop, "mean_launch_ms": dom_mean}
     step_tflops = fl["step"] * token_heads / (ms_per_step * 1e-3) / 1e12
 
-    # ---- end to end through the public API: pinned host in, host out
+    # ---- end to end through the public API: pinned host in, host out.  Each
+    # step copies its inputs in from pinned host memory and all its results
+    # out; the copies run on their own streams, so that step i + 1's inputs
+    # arrive and step i's results leave while a step computes (two device
+    # buffer sets, ordered by events).
     host = {n: x[n].cpu().pin_memory() for n in names + ("dO",)}
-    dev_in = {n: torch.empty_like(x[n]) for n in host}
+    dev_in = [{n: torch.empty_like(x[n]) for n in host} for _ in range(2)]
+    outs = [(torch.empty_like(o), {n: torch.empty_like(t) for n, t in grads.items()})
+            for _ in range(2)]
     host_out = {n: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
                 for n, t in list(grads.items()) + [("o", o)]}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev = lambda: torch.cuda.Event()
+    in_ready, in_free = [ev(), ev()], [ev(), ev()]
+    out_ready, out_free = [ev(), ev()], [ev(), ev()]
 
-    def e2e_step():
-        for n, t in host.items():
-            dev_in[n].copy_(t, non_blocking=True)
-        step(dev_in)
-        for n, t in host_out.items():
-            t.copy_(o if n == "o" else grads[n], non_blocking=True)
+    def e2e_step(i):
+        bsel = i % 2
+        with torch.cuda.stream(s_in):
+            if i >= 2:
+                s_in.wait_event(in_free[bsel])
+            for n, t in host.items():
+                dev_in[bsel][n].copy_(t, non_blocking=True)
+            in_ready[bsel].record(s_in)
+        oo, gg = outs[bsel]
+        stream.wait_event(in_ready[bsel])
+        if i >= 2:
+            stream.wait_event(out_free[bsel])
+        _, _, _, Sc, Rc = rdn.rdn_fwd(*(dev_in[bsel][n] for n in names), clip=w.clip,
+                                      return_chunk_states=True, out=oo, workspace=wsf,
+                                      save_for_bwd=True)
+        rdn.rdn_bwd(*(dev_in[bsel][n] for n in names), dev_in[bsel]["dO"], clip=w.clip,
+                    S_chunks=Sc, R_chunks=Rc, workspace=wsb, out=gg, fwd_workspace=wsf,
+                    fwd_saved=True)
+        in_free[bsel].record(stream)
+        out_ready[bsel].record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(out_ready[bsel])
+            for n, t in host_out.items():
+                t.copy_(oo if n == "o" else gg[n], non_blocking=True)
+            out_free[bsel].record(s_out)
 
-    e2e_steps = max(1, min(args.steps, 5))
-    e2e_step()
+    e2e_steps = max(2, min(args.steps, 10))
+    for i in range(2):
+        e2e_step(i)
     torch.cuda.synchronize()
     barrier(dist)
-    e0.record(stream)
-    for _ in range(e2e_steps):
-        e2e_step()
-    e1.record(stream)
+    e0.record(s_in)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    e1.record(s_out)
     torch.cuda.synchronize()
     barrier(dist)
     _, e2e_val = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * e2e_steps)
@@ -468,7 +498,9 @@ def run_ours(args):
                 "step_frac_of_bf16_peak": step_tflops / peak,
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                        "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                        "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                        "copies": "pinned host, own streams, overlapped with the compute "
+                                  "of the neighbouring steps (two device buffer sets)"},
                 "gpu_launches": lt.launches,
                 "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
                                 "share": t / sum(v[1] for v in kern.values())}
