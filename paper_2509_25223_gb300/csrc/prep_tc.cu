@@ -10,8 +10,11 @@
 //   2. thread (row, half) turns its TMEM row into the decayed, gated matrices
 //      Ap, Mq, diag(gamma) M2 (written straight to the record as bf16 hi + lo
 //      image rows) and A_beta, A_gamma (fp32, shared memory);
-//   3. T_beta = (I + A_beta)^-1 and T_gamma = (I + A_gamma)^-1 by the blocked
-//      forward substitution of chunk_common.cuh, 128 threads each, in fp32;
+//   3. T_beta = (I + A_beta)^-1 and T_gamma = (I + A_gamma)^-1, 128 threads
+//      each, in fp32, as a recursive 2 x 2 block inverse of the unit-lower
+//      matrix: diagonal 16 x 16 blocks by forward substitution, then
+//      T_ij = -T_ii A_ij T_jj for the 16-row blocks (1,0), (3,2) and the
+//      32-row block (1,0), the products register-tiled;
 //   4. their image rows and the gate vectors.
 #include "chunk_common.cuh"
 #include "tc_common.cuh"
@@ -23,16 +26,19 @@ using namespace tc;
 
 constexpr int D = 128;
 constexpr int NTH = 256;
-constexpr int LDC = C + 1;
+constexpr int LDA = C + 1;  // A_beta, A_gamma: rows written by the row pass, read as scalars
+constexpr int LDT = C + 4;  // T_beta, T_gamma: rows read as 16-byte vectors
+constexpr int LDW = 36;     // product scratch W, 32 x 32
 
 namespace pp {
 constexpr uint32_t KQ = 0;                   // K rows 0..63, Q rows 64..127, 2 x 16 KB
-constexpr uint32_t AB = 32768;               // fp32 [64][65] each: A_beta, A_gamma, T_beta, T_gamma
-constexpr uint32_t AG = AB + 64 * LDC * 4;
-constexpr uint32_t TB = AG + 64 * LDC * 4;
-constexpr uint32_t TG = TB + 64 * LDC * 4;
-constexpr uint32_t WS = TG + 64 * LDC * 4;   // blocked-inverse scratch, 2 x 768 floats
-constexpr uint32_t VEC = WS + 2 * 768 * 4;   // cum, cprev, beta, gamma, g (5 x 64)
+constexpr uint32_t AB = 32768;               // fp32 A_beta, A_gamma [64][LDA]
+constexpr uint32_t AG = AB + 64 * LDA * 4;
+constexpr uint32_t TB = AG + 64 * LDA * 4;   // fp32 T_beta, T_gamma [64][LDT]
+constexpr uint32_t TG = TB + 64 * LDT * 4;
+constexpr uint32_t WS = TG + 64 * LDT * 4;   // product scratch, 2 x [32][LDW]
+constexpr uint32_t VEC = WS + 2 * 32 * LDW * 4;  // cum, cprev, beta, gamma, g (5 x 64)
+static_assert(TB % 16 == 0 && TG % 16 == 0 && WS % 16 == 0, "16-byte rows");
 constexpr uint32_t CTL = VEC + 5 * 64 * 4;   // mbarrier, flag
 constexpr uint32_t SLOT = CTL + 16;          // TMEM base
 constexpr size_t SMEM = SLOT + 16;
@@ -65,6 +71,92 @@ __device__ __forceinline__ void img_row16(uint8_t *hi, uint32_t lo_off, int r, i
     const uint32_t off = sw128(r, c0 + o);
     *reinterpret_cast<uint4 *>(hi + off) = x;
     *reinterpret_cast<uint4 *>(hi + lo_off + off) = y;
+  }
+}
+
+// T = (I + A)^-1 for a strictly lower 64 x 64 A, by 128 threads (g = thread
+// index in the group); W is 32 x LDW scratch.  The caller synchronises the
+// block between the stages (0: diagonal blocks; 1, 2: the 16-row blocks; 3, 4:
+// the 32-row block), all groups of the block running the same stage.
+__device__ __forceinline__ void inv64_stage(int stage, const float *A, float *Tm, float *W, int g) {
+  if (stage == 0) {
+    // diagonal 16 x 16 blocks: thread (block, column) forward-substitutes its
+    // column; the blocks above the diagonal are zero
+    if (g < 64) {
+      const int b0 = (g >> 4) * 16, col = g & 15;
+      float x[16];
+#pragma unroll
+      for (int r = 0; r < 16; ++r) {
+        float s = (r == col) ? 1.f : 0.f;
+#pragma unroll
+        for (int m = 0; m < r; ++m) s = fmaf(-A[(b0 + r) * LDA + b0 + m], x[m], s);
+        x[r] = (r < col) ? 0.f : s;
+      }
+#pragma unroll
+      for (int r = 0; r < 16; ++r) Tm[(b0 + r) * LDT + b0 + col] = x[r];
+    }
+    for (int e = g; e < 64 * 64; e += 128) {
+      const int r = e >> 6, c = e & 63;
+      if ((c >> 4) > (r >> 4)) Tm[r * LDT + c] = 0.f;
+    }
+  } else if (stage <= 2) {
+    // 16-row blocks (i, j) = (1, 0) and (3, 2): W = A_ij T_jj, then
+    // T_ij = -T_ii W; thread (block, row r, columns 4q .. 4q + 3)
+    const int bi = 2 * (g >> 6) + 1, bj = bi - 1, r = (g >> 2) & 15, q = g & 3;
+    float *w = W + (g >> 6) * 16 * LDW;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (stage == 1) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const float a = A[(16 * bi + r) * LDA + 16 * bj + k];
+        const float4 t = *reinterpret_cast<const float4 *>(Tm + (16 * bj + k) * LDT + 16 * bj + 4 * q);
+        acc[0] = fmaf(a, t.x, acc[0]); acc[1] = fmaf(a, t.y, acc[1]);
+        acc[2] = fmaf(a, t.z, acc[2]); acc[3] = fmaf(a, t.w, acc[3]);
+      }
+      *reinterpret_cast<float4 *>(w + r * LDW + 4 * q) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const float a = Tm[(16 * bi + r) * LDT + 16 * bi + k];
+        const float4 t = *reinterpret_cast<const float4 *>(w + k * LDW + 4 * q);
+        acc[0] = fmaf(a, t.x, acc[0]); acc[1] = fmaf(a, t.y, acc[1]);
+        acc[2] = fmaf(a, t.z, acc[2]); acc[3] = fmaf(a, t.w, acc[3]);
+      }
+      *reinterpret_cast<float4 *>(Tm + (16 * bi + r) * LDT + 16 * bj + 4 * q) =
+          make_float4(-acc[0], -acc[1], -acc[2], -acc[3]);
+    }
+  } else {
+    // the 32-row block: W = A[32:64, 0:32] T[0:32, 0:32], then
+    // T[32:64, 0:32] = -T[32:64, 32:64] W; thread (rows rp, rp + 16, columns 4q .. 4q + 3)
+    const int q = g & 7, rp = g >> 3;
+    float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+    if (stage == 3) {
+#pragma unroll 8
+      for (int k = 0; k < 32; ++k) {
+        const float x0 = A[(32 + rp) * LDA + k], x1 = A[(48 + rp) * LDA + k];
+        const float4 t = *reinterpret_cast<const float4 *>(Tm + k * LDT + 4 * q);
+        a0[0] = fmaf(x0, t.x, a0[0]); a0[1] = fmaf(x0, t.y, a0[1]);
+        a0[2] = fmaf(x0, t.z, a0[2]); a0[3] = fmaf(x0, t.w, a0[3]);
+        a1[0] = fmaf(x1, t.x, a1[0]); a1[1] = fmaf(x1, t.y, a1[1]);
+        a1[2] = fmaf(x1, t.z, a1[2]); a1[3] = fmaf(x1, t.w, a1[3]);
+      }
+      *reinterpret_cast<float4 *>(W + rp * LDW + 4 * q) = make_float4(a0[0], a0[1], a0[2], a0[3]);
+      *reinterpret_cast<float4 *>(W + (rp + 16) * LDW + 4 * q) = make_float4(a1[0], a1[1], a1[2], a1[3]);
+    } else {
+#pragma unroll 8
+      for (int k = 0; k < 32; ++k) {
+        const float x0 = Tm[(32 + rp) * LDT + 32 + k], x1 = Tm[(48 + rp) * LDT + 32 + k];
+        const float4 t = *reinterpret_cast<const float4 *>(W + k * LDW + 4 * q);
+        a0[0] = fmaf(x0, t.x, a0[0]); a0[1] = fmaf(x0, t.y, a0[1]);
+        a0[2] = fmaf(x0, t.z, a0[2]); a0[3] = fmaf(x0, t.w, a0[3]);
+        a1[0] = fmaf(x1, t.x, a1[0]); a1[1] = fmaf(x1, t.y, a1[1]);
+        a1[2] = fmaf(x1, t.z, a1[2]); a1[3] = fmaf(x1, t.w, a1[3]);
+      }
+      *reinterpret_cast<float4 *>(Tm + (32 + rp) * LDT + 4 * q) =
+          make_float4(-a0[0], -a0[1], -a0[2], -a0[3]);
+      *reinterpret_cast<float4 *>(Tm + (48 + rp) * LDT + 4 * q) =
+          make_float4(-a1[0], -a1[1], -a1[2], -a1[3]);
+    }
   }
 }
 
@@ -182,8 +274,8 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
             a_g = dec * gam[i] * kk;
           }
           ap[u] = a_p;
-          Ab[t * LDC + i] = a_b;
-          Ag[t * LDC + i] = a_g;
+          Ab[t * LDA + i] = a_b;
+          Ag[t * LDA + i] = a_g;
         }
         img_row16(img + IMG_APMQ, 16384, t, 32 * hf + c0, ap);
       }
@@ -211,13 +303,11 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     const int g = tid & 127;
     const float *A = tid < 128 ? Ab : Ag;
     float *Tm = tid < 128 ? Tb : Tg;
-    float *W = Wsc + (tid < 128 ? 0 : 768);
-    inv_diag_blocks(A, Tm, LDC, g);
-    for (int i = 1; i < 4; ++i) {
-      __syncthreads();
-      inv_block_row_w(A, Tm, W, LDC, i, g);
-      __syncthreads();
-      inv_block_row_t(Tm, W, LDC, i, g);
+    float *W = Wsc + (tid < 128 ? 0 : 32 * LDW);
+#pragma unroll 1
+    for (int stage = 0; stage < 5; ++stage) {
+      if (stage) __syncthreads();
+      inv64_stage(stage, A, Tm, W, g);
     }
   }
   __syncthreads();
@@ -230,7 +320,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
 #pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = Tm[r * LDC + 32 * hf + c0 + u];
+        for (int u = 0; u < 16; ++u) v[u] = Tm[r * LDT + 32 * hf + c0 + u];
         img_row16(dst, 8192, r, 32 * hf + c0, v);
       }
     }
