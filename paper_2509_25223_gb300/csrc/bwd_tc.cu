@@ -177,6 +177,27 @@ __device__ __forceinline__ bool phase_run(Ctl &k, int tid, F issue) {
   return *k.flag == 0;
 }
 
+// The same, running `during` (work the MMAs do not touch) between the issue
+// and the wait.
+template <typename F, typename G>
+__device__ __forceinline__ bool phase_run_with(Ctl &k, int tid, F issue, G during) {
+  fence_async_smem();
+  fence_before_sync();
+  __syncthreads();
+  if (tid == 0) {
+    fence_after_sync();
+    if (!issue()) *k.flag = 1;
+    mma_commit(k.bar);
+  }
+  during();
+  const bool ok = mbar_wait(k.bar, k.phase);
+  k.phase ^= 1u;
+  if (!ok) *k.flag = 1;
+  __syncthreads();
+  fence_after_sync();
+  return *k.flag == 0;
+}
+
 // The same phase in two halves, for work that overlaps the MMAs: publish and
 // issue ...
 template <typename F>
@@ -479,6 +500,18 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     }
     fence_async_smem();  // the tiles are read by the MMAs and by a bulk copy
   };
+  // a carried gradient's TMEM copy times the chunk's total decay, in place
+  // (this chunk's products accumulate onto it); this thread's columns
+  auto scale_grad = [&](uint32_t col, float f) {
+#pragma unroll 1
+    for (int c0 = g16; c0 < D; c0 += 64) {
+      float x[16];
+      tmem_ld16(tm + lane + col + c0, x);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] *= f;
+      tmem_st16(tm + lane + col + c0, x);
+    }
+  };
   for (int c0 = g16; c0 < D; c0 += 64) {  // upstream gradients of the final states
     float s[16], r[16];
 #pragma unroll
@@ -566,8 +599,10 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
           sm + DOT + (j >> 6) * 8192 + sw128(t, j & 63)));
     };
-    // ---- phase A: K dR, K dS (gradients hi + lo), M2^T (gamma dO), Mq^T dO
-    ok = phase_run(K, tid, [&] {
+    // ---- phase A: K dR, K dS (gradients hi + lo), M2^T (gamma dO), Mq^T dO; meanwhile
+    // dR, dS (TMEM) times Gam_C, onto which the products of phases B .. E accumulate
+    // (the MMAs read their shared-memory tiles)
+    ok = phase_run_with(K, tid, [&] {
       if (!slot_wait(K.barA, K.phA)) return false;
       if (!slot_wait(K.barB, K.phB)) return false;
       const uint32_t i64 = idesc_bf16(128, 64);
@@ -582,6 +617,9 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       mma_tile_mnmn(tm + T_R4, sb + DOT, 8192, sb + SLOTB + 8192, 16384, 4, i64, true);
       bulk_wait_read();  // the tiles become scratch after this phase
       return true;
+    }, [&] {
+      scale_grad(T_DR, GamC);
+      scale_grad(T_DS, GamC);
     });
     if (!ok) break;
     if (tid == 0) {
@@ -615,8 +653,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
                  idesc_bf16(128, 64), false);
       const uint32_t i128 = idesc_bf16(128, 128);
-      mma_tile_kmn(tm + T_R1, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, false);
-      mma_tile_kmn(tm + T_R1, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DR, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DR, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
       return true;
     });
     if (!ok) break;
@@ -648,8 +686,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       bulk_commit();
       if (!slot_wait(K.barB, K.phB)) return false;
       const uint32_t i128 = idesc_bf16(128, 128);
-      mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
-      mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DR, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DR, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
       mma_s3_kmn(tm + T_R3, sb + S3H, sb + S3L, sb + SLOTB, sb + SLOTB + 8192, 16384,
                  idesc_bf16(128, 64), false);
       bulk_wait_read();  // the staging is rewritten next
@@ -657,16 +695,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     });
     if (!ok) break;
     if (tid == 0 && c > 0) load_mq(chunk - 1);
-    {  // dR update (fp32 in TMEM); dE = dE_partial + Ap^T dP; dQS = Gam dO
-#pragma unroll 1
-      for (int c0 = g16; c0 < D; c0 += 64) {
-        float r[16], u[16];
-        tmem_ld16(tm + lane + T_DR + c0, r);
-        tmem_ld16(tm + lane + T_R1 + c0, u);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
-        tmem_st16(tm + lane + T_DR + c0, r);
-      }
+    {  // dE = dE_partial + Ap^T dP; dQS = Gam dO (dR is complete in TMEM)
       {
         const int c0 = g16;
         float a[16], e[16], dqs[16];
@@ -687,8 +716,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
                  idesc_bf16(128, 64), false);
       const uint32_t i128 = idesc_bf16(128, 128);
-      mma_tile_kmn(tm + T_R1, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, false);
-      mma_tile_kmn(tm + T_R1, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DS, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DS, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
       return true;
     });
     if (!ok) break;
@@ -727,8 +756,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     // ---- phase E: U_S += K^T dKS
     ok = phase_run(K, tid, [&] {
       const uint32_t i128 = idesc_bf16(128, 128);
-      mma_tile_kmn(tm + T_R1, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
-      mma_tile_kmn(tm + T_R1, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DS, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
+      mma_tile_kmn(tm + T_DS, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
       bulk_wait_read();  // the staging is rewritten next (the gradient tiles)
       return true;
     });
@@ -737,17 +766,13 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       fetch_kq(c - 1);
       pre = fetch_pre(c - 1);
     }
-    // dS update, and the carried gradients' tiles: the A operands of the next
-    // chunk's phase A (the scratch tiles in their place are done with)
+    // the carried gradients' tiles (dS, dR complete in TMEM): the A operands of
+    // the next chunk's phase A (the scratch tiles in their place are done with)
 #pragma unroll 1
     for (int c0 = g16; c0 < D; c0 += 64) {
-      float s[16], u[16], r[16];
+      float s[16], r[16];
       tmem_ld16(tm + lane + T_DS + c0, s);
-      tmem_ld16(tm + lane + T_R1 + c0, u);
       tmem_ld16(tm + lane + T_DR + c0, r);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
-      tmem_st16(tm + lane + T_DS + c0, s);
       put_grad16(DSH, DSL, c0, s);
       put_grad16(DRH, DRL, c0, r);
     }
@@ -1389,6 +1414,21 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
     __syncthreads();
     if (next < nct) fetch_states(next);  // the state images and the fp32 tiles are done with
+    if (next < nct) {  // the next chunk's dO rows, mask words and gate vectors into L1
+      const int cb = (int)(next / NC), cc_ = (int)(next % NC);
+      const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * 64, n_ = min(64, T - t0_);
+      if (tid < 128) {  // 64 rows of 256 bytes
+        const int t = tid >> 1;
+        if (t < n_) prefetch_l1_line(dOp + ((size_t)(b_ * T + t0_ + t) * H + h_) * D + (tid & 1) * 64);
+      } else if (tid < 136) {  // 128 mask words
+        prefetch_l1_line(P.mask + next * D + (tid - 128) * 16);
+      } else if (tid < 148) {  // the record's 6 x 64 gate floats
+        prefetch_l1_line(p.ws + next * kRecFloats + OFF_VEC + (tid - 136) * 32);
+      } else if (tid < 180) {  // gamma, one line per two tokens
+        const int t = 2 * (tid - 148);
+        if (t < n_) prefetch_l1_line(p.gamma + (size_t)(b_ * T + t0_ + t) * H + h_);
+      }
+    }
     ok = phase_wait(K);
     if (ok && next < nct) fetch_rest(next);  // K, Q and the pair region are done with
   }

@@ -10,18 +10,19 @@
 // warps sharing a TMEM lane quadrant hide one another's latencies.  Per chunk of 64
 // tokens, with KQ = [K ; Q] (128 x d_k, exact bf16, unscaled):
 //
-//   MMA1  D1   = S^T  KQ^T          -> [KS | QS], rescaled in TMEM to
-//                                      [Gprev*KS | Gam*scale*QS]  (N=128, K=128)
-//         X    = V - Gam*KS         (= V - alpha * Gprev*KS)
-//   MMA2  E^T  = X^T  T_beta^T                                    (N=64,  K=64)
+//   MMA1  D1   = S^T  KQ^T          -> [KS | QS]                  (N=128, K=128)
+//   MMA5  D3   = R^T  KQ^T          -> [KR | QR] (chunk-start R, issued with MMA1)
+//         X    = V - Gam*KS         (= V - alpha * Gprev*KS); QS rescaled in TMEM
+//                                      to Gam*scale*QS
+//   MMA2  E^T  = X^T  T_beta^T      (over KS; Gprev*KS back in its place after)
 //   MMA3  D1  += E^T  [Ap ; Mq]^T   -> [P | Ob]                   (N=128, K=64)
-//   MMA4  U    = (wS E)^T K         -> S_C = Gam_C S + U          (N=128, K=64)
+//   MMA4  S   += (wS E)^T K         onto S scaled by Gam_C in TMEM while MMA1
+//                                      ran: S_C = Gam_C S + U       (N=128, K=64)
 //         r    = clip(V - P)        (Section 3.3; kept in registers)
-//   MMA5  D3   = R^T  KQ^T          -> [KR | QR]
 //         X2   = r - Gam*KR
 //   MMA6  E2^T = X2^T T_gamma^T
 //   MMA7  D1[:, Ob half] += E2^T (diag(gamma) M2)^T
-//   MMA8  U2   = (wR E2)^T K        -> R_C = Gam_C R + U2 (two N=64 halves)
+//   MMA8  R   += (wR E2)^T K        onto R scaled by Gam_C during MMA1: R_C
 //         o    = D1[:, Ob half] + gamma * Gam*scale*QR   (= Ob + gamma * Oa)
 //
 // RLA skips MMA2 and MMA6 (E = V, E2 = r).  X, E, wS E and their auxiliary
@@ -38,8 +39,8 @@
 // phase ahead of their use (slot A: T_beta then T_gamma; slot B: [Ap;Mq] then
 // M2) and enter the MMAs as three products (hi*hi + hi*lo + lo*hi).
 //
-// TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) X
-// (X holds E, then U, then D3; D1 holds P|Ob, then E2 | Ob, then U2a | Ob + gamma M2 E2).
+// TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) D3
+// (D1 holds KS|QS, then E | Ob, Gprev KS + Ap E = P | Ob, then E2 | Ob + gamma M2 E2).
 #include "chunk_common.cuh"
 #include "tc_common.cuh"
 
@@ -74,7 +75,7 @@ constexpr uint32_t SM_BYTES = SM_FLAG + 4;
 constexpr size_t kTcSmem = SM_BYTES;
 static_assert(kTcSmem <= 232448, "shared memory");
 
-constexpr uint32_t T_S = 0, T_R = 128, T_D1 = 256, T_X = 384;
+constexpr uint32_t T_S = 0, T_R = 128, T_D1 = 256, T_X = 384;  // T_X: D3
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
@@ -230,9 +231,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
   }
 
-  // one MMA phase: make smem writes visible, issue, wait.  Returns false on
-  // timeout (the caller aborts).
-  auto run_phase = [&](auto issue) -> bool {
+  // one MMA phase: make smem writes visible, issue, run `during` (work that
+  // the MMAs do not touch), wait.  Returns false on timeout (the caller aborts).
+  auto run_phase = [&](auto issue, auto during) -> bool {
     fence_async_smem();
     fence_before_sync();
     __syncthreads();
@@ -241,6 +242,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       if (!issue()) *flag = 1;  // a slot's bulk copy did not arrive in time
       mma_commit(bar);
     }
+    during();
     const bool ok = mbar_wait(bar, phase);
     phase ^= 1u;
     if (!ok) *flag = 1;
@@ -269,6 +271,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
   };
 
+  auto nothing = [] {};
+  // a state's TMEM copy times the chunk's total decay, in place (its updates
+  // accumulate onto it); this thread's columns
+  auto scale_state = [&](uint32_t col, float f) {
+#pragma unroll 1
+    for (int c0 = g16; c0 < D; c0 += 64) {
+      float x[16];
+      tmem_ld16(tm + lane + col + c0, x);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] *= f;
+      tmem_st16(tm + lane + col + c0, x);
+    }
+  };
+
   float rres[16];  // clipped residual r[t] of column j, t in [g16, g16 + 16)
   bool alive = true;
   for (int c = 0; c < NC && alive; ++c) {
@@ -294,15 +310,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     const float GamC = rec[OFF_VEC + V_GAMC];
     __syncthreads();
 
-    // ---- (b) MMA1: D1 = S^T [K ; Q]^T  (unscaled read-outs K S | Q S)
+    // ---- (b) MMA1: D1 = S^T [K ; Q]^T and MMA5: X = R^T [K ; Q]^T (unscaled
+    // read-outs K S | Q S and K R | Q R; both from the chunk-start states);
+    // meanwhile the TMEM states are scaled by Gam_C, for MMA4 and MMA8 to
+    // accumulate onto (the MMAs read the states' bf16 copies)
     alive = run_phase([&] {
       if (p.sv_E2) bulk_wait_read();  // the E2^T tiles of the previous chunk are rewritten next
       mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
+      mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
+               false);
       return true;
+    }, [&] {
+      scale_state(T_S, GamC);
+      scale_state(T_R, GamC);
     });
     if (!alive) break;
-    // the products below accumulate onto Gprev * KS (-> P) and Gam * scale * QS (-> Ob)
+    // Ob accumulates onto Gam * scale * QS
     {
       const int c0 = g16;
       float x[16];
@@ -312,38 +336,44 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       tmem_st16(tm + lane + T_D1 + 64 + c0, x);
     }
 
-    // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T
+    // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T into
+    // D1[0,64) (over KS); P accumulates onto Gprev KS, kept in registers until then
+    float gks[16];
     {
       const int c0 = g16;
-      float ks[16], x[16];
-      tmem_ld16(tm + lane + T_D1 + c0, ks);
+      float x[16];
+      tmem_ld16(tm + lane + T_D1 + c0, gks);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        x[i] = vs(c0 + i) - Gam[c0 + i] * ks[i];
-        ks[i] *= Gprev[c0 + i];
+        x[i] = vs(c0 + i) - Gam[c0 + i] * gks[i];
+        gks[i] *= Gprev[c0 + i];
       }
-      tmem_st16(tm + lane + T_D1 + c0, ks);
-      if (RDNV) st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+      if (RDNV)
+        st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
+      else
+        tmem_st16(tm + lane + T_D1 + c0, gks);
     }
     if (RDNV) {
       alive = run_phase([&] {
         if (!mbar_wait(barA, phA)) return false;
         phA ^= 1u;
-        mma_split3(tm + T_X, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
+        mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
                    sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
         return true;
-      });
+      }, nothing);
       if (!alive) break;
       if (tid == 0) load_slot(sm + SM_SLOTA, barA, rec_of(c) + IMG_TG, 16384);
     }
 
-    // ---- (d) E -> EA, wS*E -> WA;  MMA3: D1 += E^T [Ap;Mq]^T,  MMA4: U = (wS E)^T K
+    // ---- (d) E -> EA, wS*E -> WA, Gprev KS -> D1[0,64);  MMA3: D1 += E^T [Ap;Mq]^T,
+    // MMA4: S += (wS E)^T K
     const size_t ci = (size_t)bh * NC + c;  // chunk index of the saved intermediates
     {
       const int c0 = g16;
       float e[16], w[16];
       if (RDNV) {
-        tmem_ld16(tm + lane + T_X + c0, e);
+        tmem_ld16(tm + lane + T_D1 + c0, e);
+        tmem_st16(tm + lane + T_D1 + c0, gks);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = vs(c0 + i);
@@ -363,16 +393,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         bulk_s2g(p.sv_E + ci * 32768, sm + SM_XE, 32768);
         bulk_commit();
       }
-      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
-                   false);
-      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
+      mma_tile_kmn(tm + T_S, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
+                   true);
+      mma_tile_kmn(tm + T_S, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
                    true);
       return true;
-    });
+    }, nothing);
     if (!alive) break;
     if (tid == 0) load_slot(sm + SM_SLOTB, barB, rec_of(c) + IMG_M2, 16384);
 
-    // ---- (e) r = clip(V - P); S = Gam_C S + U (fp32 in TMEM, bf16 copy in SA)
+    // ---- (e) r = clip(V - P); S (= Gam_C S + U, fp32 in TMEM) -> bf16 copy in SA
     {
       const int c0 = g16;
       unsigned msk = 0u;  // bit i: |x| <= c at t = c0 + i (the clip passes the gradient)
@@ -389,26 +419,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
 #pragma unroll 1
     for (int c0 = g16; c0 < D; c0 += 64) {
-      float s[16], u[16];
+      float s[16];
       tmem_ld16(tm + lane + T_S + c0, s);
-      tmem_ld16(tm + lane + T_X + c0, u);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) s[i] = fmaf(GamC, s[i], u[i]);
-      tmem_st16(tm + lane + T_S + c0, s);
       st_row16(sm + SM_SA, 16384, j, c0, s);
       if (sc_next) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) sc_next[(size_t)(c0 + i) * D + j] = s[i];
       }
     }
-    // MMA5: D3 = R^T [K ; Q]^T (into X; unscaled K R | Q R)
-    alive = run_phase([&] {
-      if (p.sv_E) bulk_wait_read();  // the E^T tiles are rewritten next
-      mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
-               false);
-      return true;
-    });
-    if (!alive) break;
+    if (tid == 0 && p.sv_E) bulk_wait_read();  // the E^T tiles are rewritten next
+    __syncthreads();
     if (c + 1 < NC) fetch_v(c + 1);  // every thread is past its last read of V
 
     // ---- (f) X2 = r - Gam KR;  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
@@ -427,7 +447,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
                    sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
         return true;
-      });
+      }, nothing);
       if (!alive) break;
       if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTA, barA, rec_of(c + 1) + IMG_TB, 16384);
     }
@@ -458,17 +478,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         bulk_s2g(p.sv_E2 + ci * 32768, sm + SM_XE, 32768);
         bulk_commit();
       }
-      mma_tile_kmn(tm + T_D1, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, i64, false);
-      mma_tile_kmn(tm + T_D1, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, i64, true);
-      mma_tile_kmn(tm + T_X, sbase + SM_W, 0, sbase + SM_KQ + 16384, 16384, 4, i64, false);
-      mma_tile_kmn(tm + T_X, sbase + SM_W_LO, 0, sbase + SM_KQ + 16384, 16384, 4, i64, true);
+      mma_tile_kmn(tm + T_R, sbase + SM_W, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128), true);
+      mma_tile_kmn(tm + T_R, sbase + SM_W_LO, 0, sbase + SM_KQ, 16384, 4, idesc_bf16(128, 128),
+                   true);
       return true;
-    });
+    }, nothing);
     if (!alive) break;
     if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTB, barB, rec_of(c + 1) + IMG_APMQ, 32768);
     if (c + 1 < NC) fetch_kq(c + 1);  // K, Q are done with
 
-    // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R = Gam_C R + U2
+    // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R (= Gam_C R + U2) -> RA
     // o is staged as a [t][j] bf16 tile in W's place (free after MMA8) and stored
     // 16 bytes at a time
     __nv_bfloat16 *ostg = reinterpret_cast<__nv_bfloat16 *>(sm + SM_W);
@@ -485,12 +504,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
 #pragma unroll 1
     for (int c0 = g16; c0 < D; c0 += 64) {
-      float r[16], u[16];
+      float r[16];
       tmem_ld16(tm + lane + T_R + c0, r);
-      tmem_ld16(tm + lane + (c0 < 64 ? T_D1 + c0 : T_X + c0 - 64), u);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) r[i] = fmaf(GamC, r[i], u[i]);
-      tmem_st16(tm + lane + T_R + c0, r);
       st_row16(sm + SM_RA, 16384, j, c0, r);
       if (rc_next) {
 #pragma unroll

@@ -70,15 +70,20 @@ __device__ __forceinline__ void bulk_g2s(void *dst_smem, const void *src_gmem, u
       : "memory");
 }
 
-// Hints that bring global memory into L2 ahead of its use (no completion to
-// wait for; the later loads find the lines in L2): a contiguous range
-// (16-byte aligned address and size) and the 128-byte line of one address.
+// Hints that bring global memory closer ahead of its use (no completion to
+// wait for; the later loads find the lines cached): into L2, a contiguous
+// range (16-byte aligned address and size) or the 128-byte line of one address.
 __device__ __forceinline__ void prefetch_l2_bulk(const void *src_gmem, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src_gmem), "r"(bytes)
                : "memory");
 }
 __device__ __forceinline__ void prefetch_l2_line(const void *src_gmem) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(src_gmem));
+}
+// ... and the line of one address into this SM's L1, for loads a few
+// thousand cycles later
+__device__ __forceinline__ void prefetch_l1_line(const void *src_gmem) {
+  asm volatile("prefetch.global.L1 [%0];" ::"l"(src_gmem));
 }
 
 // 16-byte asynchronous copy global -> shared, zero-filled when !valid (the
