@@ -85,32 +85,26 @@ __device__ __forceinline__ void put16(uint8_t *tile, uint32_t blk, int r, int c0
   *reinterpret_cast<uint4 *>(b + sw128(r, cc)) = x;
   *reinterpret_cast<uint4 *>(b + sw128(r, cc + 8)) = y;
 }
-// hi / lo split of 16 values into two single-block tiles
+// hi / lo split (split_pack_bf16) of 16 values into two single-block tiles
 __device__ __forceinline__ void put16s(uint8_t *hi, uint8_t *lo, int r, int c0,
                                        const float (&v)[16]) {
-  float a[16], b[16];
+  uint32_t h[8], l[8];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
-    b[i] = v[i] - a[i];
-  }
-  put16(hi, 0, r, c0, a);
-  put16(lo, 0, r, c0, b);
+  for (int i = 0; i < 8; ++i) split_pack_bf16(v[2 * i], v[2 * i + 1], h[i], l[i]);
+  const int cc = c0 & 63;
+  *reinterpret_cast<uint4 *>(hi + sw128(r, cc)) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4 *>(hi + sw128(r, cc + 8)) = make_uint4(h[4], h[5], h[6], h[7]);
+  *reinterpret_cast<uint4 *>(lo + sw128(r, cc)) = make_uint4(l[0], l[1], l[2], l[3]);
+  *reinterpret_cast<uint4 *>(lo + sw128(r, cc + 8)) = make_uint4(l[4], l[5], l[6], l[7]);
 }
 // the same for 8 values (one 16-byte chunk of each tile)
 __device__ __forceinline__ void put8s(uint8_t *hi, uint8_t *lo, int r, int c0,
                                       const float (&v)[8]) {
-  float a[8], b[8];
+  uint32_t h[4], l[4];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
-    b[i] = v[i] - a[i];
-  }
-  uint4 x, y;
-  x.x = pack2(a[0], a[1]); x.y = pack2(a[2], a[3]); x.z = pack2(a[4], a[5]); x.w = pack2(a[6], a[7]);
-  y.x = pack2(b[0], b[1]); y.y = pack2(b[2], b[3]); y.z = pack2(b[4], b[5]); y.w = pack2(b[6], b[7]);
-  *reinterpret_cast<uint4 *>(hi + sw128(r, c0)) = x;
-  *reinterpret_cast<uint4 *>(lo + sw128(r, c0)) = y;
+  for (int i = 0; i < 4; ++i) split_pack_bf16(v[2 * i], v[2 * i + 1], h[i], l[i]);
+  *reinterpret_cast<uint4 *>(hi + sw128(r, c0)) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4 *>(lo + sw128(r, c0)) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 // K-major A (single block, K = 64) times MN-major B, split both: 3 products
 __device__ __forceinline__ void mma_s3_kmn(uint32_t d, uint32_t a_hi, uint32_t a_lo,
@@ -479,14 +473,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
   const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   // a carried gradient's bf16 hi + lo tiles (rows j), 16 of its key rows
   auto put_grad16 = [&](uint32_t hi, uint32_t lo, int c0, const float (&g)[16]) {
-    float gh[16], gl[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      gh[i] = __bfloat162float(__float2bfloat16_rn(g[i]));
-      gl[i] = g[i] - gh[i];
-    }
-    put16(sm + hi, 16384, j, c0, gh);
-    put16(sm + lo, 16384, j, c0, gl);
+    put16s(sm + hi + (c0 >> 6) * 16384, sm + lo + (c0 >> 6) * 16384, j, c0, g);
   };
   // both carried gradients' tiles from their fp32 TMEM copies
   auto write_grad_tiles = [&]() {

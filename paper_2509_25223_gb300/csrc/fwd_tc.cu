@@ -101,18 +101,17 @@ __device__ __forceinline__ void st_row16(uint8_t *tile, uint32_t blk_bytes, int 
   *reinterpret_cast<uint4 *>(blk + sw128(r, cc + 8)) = b;
 }
 
-// Same, split: hi = bf16(v), lo = bf16(v - hi) into two tiles, so that
-// hi + lo carries about 16 significant bits.
+// Same, split into bf16 hi + lo parts (split_pack_bf16) in two tiles.
 __device__ __forceinline__ void st_row16_split(uint8_t *hi, uint8_t *lo, int r, int c0,
                                                const float (&v)[16]) {
-  float a[16], b[16];
+  uint32_t h[8], l[8];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
-    b[i] = v[i] - a[i];
-  }
-  st_row16(hi, 0, r, c0, a);
-  st_row16(lo, 0, r, c0, b);
+  for (int i = 0; i < 8; ++i) split_pack_bf16(v[2 * i], v[2 * i + 1], h[i], l[i]);
+  const int cc = c0 & 63;
+  *reinterpret_cast<uint4 *>(hi + sw128(r, cc)) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4 *>(hi + sw128(r, cc + 8)) = make_uint4(h[4], h[5], h[6], h[7]);
+  *reinterpret_cast<uint4 *>(lo + sw128(r, cc)) = make_uint4(l[0], l[1], l[2], l[3]);
+  *reinterpret_cast<uint4 *>(lo + sw128(r, cc + 8)) = make_uint4(l[4], l[5], l[6], l[7]);
 }
 
 // D (+)= (A_hi + A_lo)(B_hi + B_lo)^T without the lo*lo term: three MMAs

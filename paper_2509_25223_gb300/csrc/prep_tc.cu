@@ -45,32 +45,20 @@ constexpr size_t SMEM = SLOT + 16;
 static_assert(2 * (SMEM + 1024) <= 233472, "two CTAs per SM");
 }  // namespace pp
 
-__device__ __forceinline__ uint32_t pack2(float a, float b) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t *>(&v);
-}
-
 // Row r, columns c0 .. c0+15 (c0 a multiple of 16 below 64) of a 64-column
 // image in global memory: bf16 hi part at `hi`, lo part `lo_off` bytes later.
 __device__ __forceinline__ void img_row16(uint8_t *hi, uint32_t lo_off, int r, int c0,
                                           const float (&v)[16]) {
-  float a[16], b[16];
+  uint32_t h[8], l[8];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    a[i] = __bfloat162float(__float2bfloat16_rn(v[i]));
-    b[i] = v[i] - a[i];
-  }
+  for (int i = 0; i < 8; ++i) split_pack_bf16(v[2 * i], v[2 * i + 1], h[i], l[i]);
 #pragma unroll
   for (int half = 0; half < 2; ++half) {
-    const int o = 8 * half;
-    uint4 x, y;
-    x.x = pack2(a[o + 0], a[o + 1]); x.y = pack2(a[o + 2], a[o + 3]);
-    x.z = pack2(a[o + 4], a[o + 5]); x.w = pack2(a[o + 6], a[o + 7]);
-    y.x = pack2(b[o + 0], b[o + 1]); y.y = pack2(b[o + 2], b[o + 3]);
-    y.z = pack2(b[o + 4], b[o + 5]); y.w = pack2(b[o + 6], b[o + 7]);
-    const uint32_t off = sw128(r, c0 + o);
-    *reinterpret_cast<uint4 *>(hi + off) = x;
-    *reinterpret_cast<uint4 *>(hi + lo_off + off) = y;
+    const uint32_t off = sw128(r, c0 + 8 * half);
+    *reinterpret_cast<uint4 *>(hi + off) =
+        make_uint4(h[4 * half], h[4 * half + 1], h[4 * half + 2], h[4 * half + 3]);
+    *reinterpret_cast<uint4 *>(hi + lo_off + off) =
+        make_uint4(l[4 * half], l[4 * half + 1], l[4 * half + 2], l[4 * half + 3]);
   }
 }
 

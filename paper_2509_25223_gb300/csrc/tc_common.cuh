@@ -86,6 +86,18 @@ __device__ __forceinline__ void prefetch_l1_line(const void *src_gmem) {
   asm volatile("prefetch.global.L1 [%0];" ::"l"(src_gmem));
 }
 
+// Two floats as bf16 hi + lo parts, each pair packed in 32 bits (a in the low
+// half): hi is a's upper 16 bits (bf16 truncation, exact, no conversion), lo
+// the remainder a - hi (exact in fp32) rounded to bf16; hi + lo carries about
+// 16 significant bits (relative error below 2^-17).
+__device__ __forceinline__ void split_pack_bf16(float a, float b, uint32_t &hi, uint32_t &lo) {
+  const uint32_t ua = __float_as_uint(a), ub = __float_as_uint(b);
+  hi = __byte_perm(ua, ub, 0x7632);
+  const __nv_bfloat162 r = __floats2bfloat162_rn(a - __uint_as_float(ua & 0xFFFF0000u),
+                                                 b - __uint_as_float(ub & 0xFFFF0000u));
+  lo = *reinterpret_cast<const uint32_t *>(&r);
+}
+
 // 16-byte asynchronous copy global -> shared, zero-filled when !valid (the
 // source is then not read, but must still be a valid address).  Completes at
 // cp_async_wait_all() of the issuing thread; a barrier then publishes it.
