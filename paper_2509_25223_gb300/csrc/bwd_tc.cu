@@ -616,22 +616,23 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     // dE2 = M2^T dOa + wR K dR ; dE (partial) = Mq^T dO + wS K dS ; dQR = Gam gamma dO
     {
       const int c0 = g16;
-      float x[16], y[16];
+      float x[16], y[16], w[16];
       tmem_ld16(tm + lane + T_R1 + c0, x);
       tmem_ld16(tm + lane + T_R3 + c0, y);
+      lds16(wR + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) y[i] += wR[c0 + i] * x[i];
+      for (int i = 0; i < 16; ++i) y[i] += w[i] * x[i];
       put16s(sm + S0H, sm + S0L, j, c0, y);
       tmem_ld16(tm + lane + T_R2 + c0, x);
       tmem_ld16(tm + lane + T_R4 + c0, y);
+      lds16(wS + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) y[i] += wS[c0 + i] * x[i];
+      for (int i = 0; i < 16; ++i) y[i] += w[i] * x[i];
       tmem_st16(tm + lane + T_R4 + c0, y);
+      lds16(Gam + c0, x);
+      lds16(gamv + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = c0 + i;
-        x[i] = p.scale * Gam[t] * gamv[t] * dO(t);  // dQR (Q below is unscaled)
-      }
+      for (int i = 0; i < 16; ++i) x[i] = p.scale * x[i] * w[i] * dO(c0 + i);  // dQR (Q unscaled)
       put16s(sm + S1H, sm + S1L, j, c0, x);
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
@@ -654,13 +655,14 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         const int c0 = g16;
         float x[16], dkr[16], dp[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
+        lds16(Gam + c0, dkr);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
           dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
           dP[i] = dp[i];
-          dkr[i] = -Gam[t] * x[i];
+          dkr[i] = -dkr[i] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dkr);
         put16s(sm + S3H, sm + S3L, j, c0, dp);
@@ -688,10 +690,11 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         float a[16], e[16], dqs[16];
         tmem_ld16(tm + lane + T_R4 + c0, a);
         tmem_ld16(tm + lane + T_R3 + c0, e);
+        lds16(Gam + c0, dqs);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           a[i] += e[i];
-          dqs[i] = p.scale * Gam[c0 + i] * dO(c0 + i);
+          dqs[i] = p.scale * dqs[i] * dO(c0 + i);
         }
         put16s(sm + S0H, sm + S0L, j, c0, a);
         put16s(sm + S1H, sm + S1L, j, c0, dqs);
@@ -716,14 +719,16 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       __nv_bfloat16 *dvs = reinterpret_cast<__nv_bfloat16 *>(sm + S1H);
       {
         const int c0 = g16;
-        float x[16], dks[16];
+        float x[16], dks[16], gm[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
+        lds16(Gprev + c0, dks);
+        lds16(Gam + c0, gm);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
           dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
-          dks[i] = Gprev[t] * dP[i] - Gam[t] * x[i];
+          dks[i] = dks[i] * dP[i] - gm[i] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
       }
@@ -1003,8 +1008,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {  // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
       float qr[16];
       tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
+      lds16(Gam + tb, rv);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] = scale * Gam[tb + i] * dov[i] * qr[i];
+      for (int i = 0; i < 16; ++i) rv[i] = scale * rv[i] * dov[i] * qr[i];
       cta_row_sum512(rv, red, dGamS, tid);
       // parked in the record's slot (shared memory is full); the same thread reads it back
       if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
@@ -1014,8 +1020,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       float qs[16], qr[16];
       tmem_ld16(tm + tm_lane + T_KS + 64 + tb, qs);
       tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
+      lds16(gamv + tb, rv);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] = scale * dov[i] * (qs[i] + gamv[tb + i] * qr[i]);
+      for (int i = 0; i < 16; ++i) rv[i] = scale * dov[i] * (qs[i] + rv[i] * qr[i]);
     }
     {
       float ks[16], kr[16];
@@ -1030,11 +1037,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     cta_row_sum512(rv, red, dGprevS, tid);
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
     float x[16], y[16];
+    lds16(Gam + tb, x);
+    lds16(gamv + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      const int t = tb + i;
-      x[i] = -Gam[t] * x2v[i];
-      y[i] = Gam[t] * gamv[t] * dov[i];
+      y[i] *= x[i] * dov[i];
+      x[i] = -x[i] * x2v[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1052,11 +1060,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO
     float x[16], y[16];
+    lds16(Gprev + tb, x);
+    lds16(Gam + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      const int t = tb + i;
-      x[i] = Gprev[t] * dp_of(i) - Gam[t] * xv[i];
-      y[i] = Gam[t] * dov[i];
+      x[i] = x[i] * dp_of(i) - y[i] * xv[i];
+      y[i] *= dov[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1130,15 +1139,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   if (ok) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
     {
-      float a[16], u1[16], u2[16];
+      float a[16], u1[16], u2[16], wr[16], ws[16];
       tmem_ld16(tm + tm_lane + T_DKQ + tb, a);
       tmem_ld16(tm + tm_lane + T_U1 + tb, u1);
       tmem_ld16(tm + tm_lane + T_U2 + tb, u2);
+      lds16(wR + tb, wr);
+      lds16(wS + tb, ws);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = tb + i;
-        a[i] = fmaf(wR[t], u1[i], fmaf(wS[t], u2[i], a[i]));
-      }
+      for (int i = 0; i < 16; ++i) a[i] = fmaf(wr[i], u1[i], fmaf(ws[i], u2[i], a[i]));
       tmem_st16(tm + tm_lane + T_DKQ + tb, a);
     }
     // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]

@@ -328,24 +328,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     // Ob accumulates onto Gam * scale * QS
     {
       const int c0 = g16;
-      float x[16];
+      float x[16], gm[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, x);
+      lds16(Gam + c0, gm);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] *= Gam[c0 + i] * p.scale;
+      for (int i = 0; i < 16; ++i) x[i] *= gm[i] * p.scale;
       tmem_st16(tm + lane + T_D1 + 64 + c0, x);
     }
 
     // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T into
     // D1[0,64) (over KS); P accumulates onto Gprev KS, kept in registers until then
-    float gks[16];
+    float gks[16], vv[16];  // vv: this thread's V entries, until (e)
     {
       const int c0 = g16;
-      float x[16];
+      float x[16], gm[16], gp[16];
       tmem_ld16(tm + lane + T_D1 + c0, gks);
+      lds16(Gam + c0, gm);
+      lds16(Gprev + c0, gp);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        x[i] = vs(c0 + i) - Gam[c0 + i] * gks[i];
-        gks[i] *= Gprev[c0 + i];
+        vv[i] = vs(c0 + i);
+        x[i] = vv[i] - gm[i] * gks[i];
+        gks[i] *= gp[i];
       }
       if (RDNV)
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
@@ -375,10 +379,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         tmem_st16(tm + lane + T_D1 + c0, gks);
       } else {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) e[i] = vs(c0 + i);
+        for (int i = 0; i < 16; ++i) e[i] = vv[i];
       }
+      lds16(wS + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) w[i] = wS[c0 + i] * e[i];
+      for (int i = 0; i < 16; ++i) w[i] *= e[i];
       st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, e);
       st_row16_split(sm + SM_W, sm + SM_W_LO, j, c0, w);
     }
@@ -409,7 +414,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       tmem_ld16(tm + lane + T_D1 + c0, pp);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float x = vs(c0 + i) - pp[i];
+        const float x = vv[i] - pp[i];
         if (fabsf(x) <= clip) msk |= 1u << i;
         rres[i] = clampf(x, clip);
       }
@@ -434,10 +439,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (RDNV) {
       {
         const int c0 = g16;
-        float x[16];
+        float x[16], gm[16];
         tmem_ld16(tm + lane + T_X + c0, x);
+        lds16(Gam + c0, gm);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = rres[i] - Gam[c0 + i] * x[i];
+        for (int i = 0; i < 16; ++i) x[i] = rres[i] - gm[i] * x[i];
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
       }
       alive = run_phase([&] {
@@ -461,8 +467,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) e[i] = rres[i];
       }
+      lds16(wR + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) w[i] = wR[c0 + i] * e[i];
+      for (int i = 0; i < 16; ++i) w[i] *= e[i];
       st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, e);
       st_row16_split(sm + SM_W, sm + SM_W_LO, j, c0, w);
     }
@@ -492,13 +499,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     __nv_bfloat16 *ostg = reinterpret_cast<__nv_bfloat16 *>(sm + SM_W);
     {
       const int c0 = g16;
-      float ob[16], oa[16];
+      float ob[16], oa[16], gm[16], gv[16];
       tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);
       tmem_ld16(tm + lane + T_X + 64 + c0, oa);
+      lds16(Gam + c0, gm);
+      lds16(gamv + c0, gv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
-        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gamv[t] * Gam[t] * p.scale, oa[i], ob[i]));
+        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gv[i] * gm[i] * p.scale, oa[i], ob[i]));
       }
     }
 #pragma unroll 1

@@ -86,6 +86,20 @@ __device__ __forceinline__ void prefetch_l1_line(const void *src_gmem) {
   asm volatile("prefetch.global.L1 [%0];" ::"l"(src_gmem));
 }
 
+// 16 consecutive floats of shared memory at a 16-byte aligned address, by
+// four 16-byte loads
+__device__ __forceinline__ void lds16(const float *p, float (&v)[16]) {
+  const float4 *q = reinterpret_cast<const float4 *>(p);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float4 a = q[k];
+    v[4 * k] = a.x;
+    v[4 * k + 1] = a.y;
+    v[4 * k + 2] = a.z;
+    v[4 * k + 3] = a.w;
+  }
+}
+
 // Two floats as bf16 hi + lo parts, each pair packed in 32 bits (a in the low
 // half): hi is a's upper 16 bits (bf16 truncation, exact, no conversion), lo
 // the remainder a - hi (exact in fp32) rounded to bf16; hi + lo carries about
