@@ -480,8 +480,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll 1
     for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], r[16];
-      tmem_ld16(tm + lane + T_DS + c0, s);
-      tmem_ld16(tm + lane + T_DR + c0, r);
+      tmem_ld16x2(tm + lane + T_DS + c0, s, tm + lane + T_DR + c0, r);
       put_grad16(DSH, DSL, c0, s);
       put_grad16(DRH, DRL, c0, r);
     }
@@ -490,14 +489,15 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
   // a carried gradient's TMEM copy times the chunk's total decay, in place
   // (this chunk's products accumulate onto it); this thread's columns
   auto scale_grad = [&](uint32_t col, float f) {
-#pragma unroll 1
-    for (int c0 = g16; c0 < D; c0 += 64) {
-      float x[16];
-      tmem_ld16(tm + lane + col + c0, x);
+    float x[16], y[16];
+    tmem_ld16x2(tm + lane + col + g16, x, tm + lane + col + g16 + 64, y);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] *= f;
-      tmem_st16(tm + lane + col + c0, x);
+    for (int i = 0; i < 16; ++i) {
+      x[i] *= f;
+      y[i] *= f;
     }
+    tmem_st16(tm + lane + col + g16, x);
+    tmem_st16(tm + lane + col + g16 + 64, y);
   };
   for (int c0 = g16; c0 < D; c0 += 64) {  // upstream gradients of the final states
     float s[16], r[16];
@@ -617,14 +617,12 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     {
       const int c0 = g16;
       float x[16], y[16], w[16];
-      tmem_ld16(tm + lane + T_R1 + c0, x);
-      tmem_ld16(tm + lane + T_R3 + c0, y);
+      tmem_ld16x2(tm + lane + T_R1 + c0, x, tm + lane + T_R3 + c0, y);
       lds16(wR + c0, w);
 #pragma unroll
       for (int i = 0; i < 16; ++i) y[i] += w[i] * x[i];
       put16s(sm + S0H, sm + S0L, j, c0, y);
-      tmem_ld16(tm + lane + T_R2 + c0, x);
-      tmem_ld16(tm + lane + T_R4 + c0, y);
+      tmem_ld16x2(tm + lane + T_R2 + c0, x, tm + lane + T_R4 + c0, y);
       lds16(wS + c0, w);
 #pragma unroll
       for (int i = 0; i < 16; ++i) y[i] += w[i] * x[i];
@@ -688,8 +686,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       {
         const int c0 = g16;
         float a[16], e[16], dqs[16];
-        tmem_ld16(tm + lane + T_R4 + c0, a);
-        tmem_ld16(tm + lane + T_R3 + c0, e);
+        tmem_ld16x2(tm + lane + T_R4 + c0, a, tm + lane + T_R3 + c0, e);
         lds16(Gam + c0, dqs);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -763,8 +760,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
 #pragma unroll 1
     for (int c0 = g16; c0 < D; c0 += 64) {
       float s[16], r[16];
-      tmem_ld16(tm + lane + T_DS + c0, s);
-      tmem_ld16(tm + lane + T_DR + c0, r);
+      tmem_ld16x2(tm + lane + T_DS + c0, s, tm + lane + T_DR + c0, r);
       put_grad16(DSH, DSL, c0, s);
       put_grad16(DRH, DRL, c0, r);
     }
@@ -1005,9 +1001,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
     float rv[16];
-    {  // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
-      float qr[16];
-      tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
+    {
+      float qs[16], qr[16];
+      tmem_ld16x2(tm + tm_lane + T_KS + 64 + tb, qs, tm + tm_lane + T_KR + 64 + tb, qr);
+      // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
       lds16(Gam + tb, rv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = scale * rv[i] * dov[i] * qr[i];
@@ -1015,19 +1012,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       // parked in the record's slot (shared memory is full); the same thread reads it back
       if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
       __syncthreads();
-    }
-    {
-      float qs[16], qr[16];
-      tmem_ld16(tm + tm_lane + T_KS + 64 + tb, qs);
-      tmem_ld16(tm + tm_lane + T_KR + 64 + tb, qr);
       lds16(gamv + tb, rv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = scale * dov[i] * (qs[i] + rv[i] * qr[i]);
     }
     {
       float ks[16], kr[16];
-      tmem_ld16(tm + tm_lane + T_KS + tb, ks);
-      tmem_ld16(tm + tm_lane + T_KR + tb, kr);
+      tmem_ld16x2(tm + tm_lane + T_KS + tb, ks, tm + tm_lane + T_KR + tb, kr);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
       cta_row_sum512(rv, red, dGamS, tid);
@@ -1140,8 +1131,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
     {
       float a[16], u1[16], u2[16], wr[16], ws[16];
-      tmem_ld16(tm + tm_lane + T_DKQ + tb, a);
-      tmem_ld16(tm + tm_lane + T_U1 + tb, u1);
+      tmem_ld16x2(tm + tm_lane + T_DKQ + tb, a, tm + tm_lane + T_U1 + tb, u1);
       tmem_ld16(tm + tm_lane + T_U2 + tb, u2);
       lds16(wR + tb, wr);
       lds16(wS + tb, ws);
@@ -1206,10 +1196,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const int r = j & 63;
       {
         float g1[16], g2[16], g3[16], gr[16];
-        tmem_ld16(tm + tm_lane + T_G1 + tb, g1);
-        tmem_ld16(tm + tm_lane + T_G2 + tb, g2);
-        tmem_ld16(tm + tm_lane + T_G3 + tb, g3);
-        tmem_ld16(tm + tm_lane + T_GR + tb, gr);
+        tmem_ld16x2(tm + tm_lane + T_G1 + tb, g1, tm + tm_lane + T_G2 + tb, g2);
+        tmem_ld16x2(tm + tm_lane + T_G3 + tb, g3, tm + tm_lane + T_GR + tb, gr);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int e = r * LDC + tb + i;
@@ -1437,8 +1425,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
     {
       float a[16], d2[16], qv[16];
-      tmem_ld16(tm + tm_lane + T_DKQ + tb, a);
-      tmem_ld16(tm + tm_lane + T_D2 + tb, d2);
+      tmem_ld16x2(tm + tm_lane + T_DKQ + tb, a, tm + tm_lane + T_D2 + tb, d2);
       tmem_ld16(tm + tm_lane + T_DKQ + 64 + tb, qv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {

@@ -274,15 +274,38 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   // a state's TMEM copy times the chunk's total decay, in place (its updates
   // accumulate onto it); this thread's columns
   auto scale_state = [&](uint32_t col, float f) {
-#pragma unroll 1
-    for (int c0 = g16; c0 < D; c0 += 64) {
-      float x[16];
-      tmem_ld16(tm + lane + col + c0, x);
+    float x[16], y[16];
+    tmem_ld16x2(tm + lane + col + g16, x, tm + lane + col + g16 + 64, y);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] *= f;
-      tmem_st16(tm + lane + col + c0, x);
+    for (int i = 0; i < 16; ++i) {
+      x[i] *= f;
+      y[i] *= f;
     }
+    tmem_st16(tm + lane + col + g16, x);
+    tmem_st16(tm + lane + col + g16 + 64, y);
   };
+
+  // a chunk's gate values (threads 0..63, one token each) and its total decay,
+  // loaded into registers one chunk ahead of their use
+  struct Pre {
+    float gm, gp, ws, wr, g, gc;
+  };
+  auto fetch_pre = [&](int c) {
+    const float *rc = p.ws + ((size_t)bh * NC + c) * kRecFloats;
+    const int t0_ = c * 64, n_ = min(64, T - t0_);
+    Pre x;
+    x.gm = x.gp = x.ws = x.wr = x.g = 0.f;
+    if (tid < 64) {
+      x.gm = rc[OFF_VEC + V_GAM + tid];
+      x.gp = rc[OFF_VEC + V_GPREV + tid];
+      x.ws = rc[OFF_VEC + V_WS + tid];
+      x.wr = rc[OFF_VEC + V_WR + tid];
+      x.g = tid < n_ ? p.gamma[(size_t)(b * T + t0_ + tid) * H + h] : 0.f;
+    }
+    x.gc = rc[OFF_VEC + V_GAMC];
+    return x;
+  };
+  Pre pre = fetch_pre(0);
 
   float rres[16];  // clipped residual r[t] of column j, t in [g16, g16 + 16)
   bool alive = true;
@@ -290,7 +313,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     const int t0 = c * 64;
     const int n = min(64, T - t0);
     if (c + 1 < NC) prefetch_chunk(c + 1);
-    const float *rec = p.ws + ((size_t)bh * NC + c) * kRecFloats;
     cp_async_wait_all();  // this chunk's V, K, Q tiles (fetched during the previous chunk)
     __syncthreads();      // every thread is done with the previous chunk's tiles and vectors
 
@@ -300,13 +322,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
                                                 : nullptr;
     float *rc_next = sc_next ? p.R_chunks + ((size_t)bh * NC + c + 1) * D * D : nullptr;
     if (tid < 64) {
-      Gam[tid] = rec[OFF_VEC + V_GAM + tid];
-      Gprev[tid] = rec[OFF_VEC + V_GPREV + tid];
-      wS[tid] = rec[OFF_VEC + V_WS + tid];
-      wR[tid] = rec[OFF_VEC + V_WR + tid];
-      gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+      Gam[tid] = pre.gm;
+      Gprev[tid] = pre.gp;
+      wS[tid] = pre.ws;
+      wR[tid] = pre.wr;
+      gamv[tid] = pre.g;
     }
-    const float GamC = rec[OFF_VEC + V_GAMC];
+    const float GamC = pre.gc;
+    if (c + 1 < NC) pre = fetch_pre(c + 1);  // in flight during this chunk
     __syncthreads();
 
     // ---- (b) MMA1: D1 = S^T [K ; Q]^T and MMA5: X = R^T [K ; Q]^T (unscaled
@@ -326,10 +349,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     });
     if (!alive) break;
     // Ob accumulates onto Gam * scale * QS
+    float gks[16], vv[16];  // gks: K S, then Gprev K S; vv: this thread's V entries, until (e)
     {
       const int c0 = g16;
       float x[16], gm[16];
-      tmem_ld16(tm + lane + T_D1 + 64 + c0, x);
+      tmem_ld16x2(tm + lane + T_D1 + 64 + c0, x, tm + lane + T_D1 + c0, gks);
       lds16(Gam + c0, gm);
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] *= gm[i] * p.scale;
@@ -338,11 +362,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (c) X = V - Gam KS (= V - alpha Gprev KS)  ->  MMA2: E^T = X^T T_beta^T into
     // D1[0,64) (over KS); P accumulates onto Gprev KS, kept in registers until then
-    float gks[16], vv[16];  // vv: this thread's V entries, until (e)
     {
       const int c0 = g16;
       float x[16], gm[16], gp[16];
-      tmem_ld16(tm + lane + T_D1 + c0, gks);
       lds16(Gam + c0, gm);
       lds16(Gprev + c0, gp);
 #pragma unroll
@@ -421,14 +443,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       // bits [c0, c0 + 16) of the column's 64-bit mask word (little-endian)
       if (p.sv_mask) reinterpret_cast<uint16_t *>(p.sv_mask + ci * D + j)[c0 >> 4] = (uint16_t)msk;
     }
-#pragma unroll 1
-    for (int c0 = g16; c0 < D; c0 += 64) {
-      float s[16];
-      tmem_ld16(tm + lane + T_S + c0, s);
-      st_row16(sm + SM_SA, 16384, j, c0, s);
+    {
+      float s0[16], s1[16];
+      tmem_ld16x2(tm + lane + T_S + g16, s0, tm + lane + T_S + g16 + 64, s1);
+      st_row16(sm + SM_SA, 16384, j, g16, s0);
+      st_row16(sm + SM_SA, 16384, j, g16 + 64, s1);
       if (sc_next) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) sc_next[(size_t)(c0 + i) * D + j] = s[i];
+        for (int i = 0; i < 16; ++i) {
+          sc_next[(size_t)(g16 + i) * D + j] = s0[i];
+          sc_next[(size_t)(g16 + 64 + i) * D + j] = s1[i];
+        }
       }
     }
     if (tid == 0 && p.sv_E) bulk_wait_read();  // the E^T tiles are rewritten next
@@ -500,8 +525,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     {
       const int c0 = g16;
       float ob[16], oa[16], gm[16], gv[16];
-      tmem_ld16(tm + lane + T_D1 + 64 + c0, ob);
-      tmem_ld16(tm + lane + T_X + 64 + c0, oa);
+      tmem_ld16x2(tm + lane + T_D1 + 64 + c0, ob, tm + lane + T_X + 64 + c0, oa);
       lds16(Gam + c0, gm);
       lds16(gamv + c0, gv);
 #pragma unroll
@@ -510,14 +534,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         ostg[t * D + j] = __float2bfloat16_rn(fmaf(gv[i] * gm[i] * p.scale, oa[i], ob[i]));
       }
     }
-#pragma unroll 1
-    for (int c0 = g16; c0 < D; c0 += 64) {
-      float r[16];
-      tmem_ld16(tm + lane + T_R + c0, r);
-      st_row16(sm + SM_RA, 16384, j, c0, r);
+    {
+      float r0[16], r1[16];
+      tmem_ld16x2(tm + lane + T_R + g16, r0, tm + lane + T_R + g16 + 64, r1);
+      st_row16(sm + SM_RA, 16384, j, g16, r0);
+      st_row16(sm + SM_RA, 16384, j, g16 + 64, r1);
       if (rc_next) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) rc_next[(size_t)(c0 + i) * D + j] = r[i];
+        for (int i = 0; i < 16; ++i) {
+          rc_next[(size_t)(g16 + i) * D + j] = r0[i];
+          rc_next[(size_t)(g16 + 64 + i) * D + j] = r1[i];
+        }
       }
     }
     __syncthreads();  // the o tile
