@@ -1049,7 +1049,18 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     bulk_g2s(sm + SB, gimg + 32768, 32768, K.barB);
     bulk_g2s(sm + SB + 32768, gimg + 98304, 32768, K.barB);
   }
-  if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO
+  // <dR, R0> + <dS, S0> into dGamC, each computed while MMAs run: the states
+  // are re-read from L2 (not through L1, which holds the prefetched dO rows),
+  // the gradients' images are in the states' places
+  float gdot = 0.f;
+  auto dot_state = [&](const float *st, uint32_t img) {
+    float x[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] = __ldcg(st + (size_t)(32 * qd + i) * D + j);
+    return dot_image(img, x);
+  };
+  if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO;
+             // meanwhile <dR, R0>
     float x[16], y[16];
     lds16(Gprev + tb, x);
     lds16(Gam + tb, y);
@@ -1060,11 +1071,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
-    ok = phase_run(K, tid, [&] {
+    ok = phase_run_with(K, tid, [&] {
       mma_tile_mnmn<true>(tm + T_DKQ, sb + SA, 16384, sb + XH, 32768, 8, i128, true);
       mma_tile_mnmn<true>(tm + T_DKQ, sb + SA, 16384, sb + XL, 32768, 8, i128, true);
       mma_tile_mnmn<true>(tm + T_DKQ, sb + SA + 32768, 16384, sb + XH, 32768, 8, i128, true);
       return true;
+    }, [&] {
+      if (!mbar_wait(K.barB, it & 1u)) *K.flag = 1;  // dR's image
+      gdot = dot_state(R0, SB);
     });
   }
   if (ok && tid == 0) {  // and dS's image into S0's; the E2^T, E^T images into the pair's
@@ -1074,27 +1088,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     mbar_expect_tx(K.barC, 65536);
     bulk_g2s(sm + XH, P.E2buf + chunk * 32768, 32768, K.barC);  // hi at XH, lo at XL
     bulk_g2s(sm + YH, P.Ebuf + chunk * 32768, 32768, K.barC);   // hi at YH, lo at YL
-  }
-  if (ok) {  // <dR, R0> + <dS, S0> (states re-read from L2, images in place), into dGamC
-    float gdot = 0.f;
-#pragma unroll 1
-    for (int s2 = 0; s2 < 2; ++s2) {
-      const float *st = s2 ? S0 : R0;
-      float x[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) x[i] = st[(size_t)(32 * qd + i) * D + j];
-      if (!mbar_wait(s2 ? K.barA : K.barB, s2 ? 1u : (it & 1u))) *K.flag = 1;
-      gdot += dot_image(s2 ? SA : SB, x);
-    }
-#pragma unroll
-    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
-    if (lane == 0) red[warp] = gdot;
-    __syncthreads();
-    if (tid == 0) {
-      float s = 0.f;
-      for (int w = 0; w < NTP / 32; ++w) s += red[w];
-      *dGamC = s;
-    }
   }
   // this thread's 16 tokens of row j of a (hi | lo) image of a [j][t] matrix
   auto image_row = [&](uint32_t base, float (&out)[16]) {
@@ -1110,9 +1103,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       for (int e = 0; e < 8; ++e) out[k8 * 8 + e] = __bfloat162float(hb[e]) + __bfloat162float(lb[e]);
     }
   };
-  if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs
+  if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs;
+             // meanwhile <dS, S0> and the dGamC reduction
     if (!mbar_wait(K.barC, 1)) *K.flag = 1;  // the E images, for every thread
-    ok = phase_run(K, tid, [&] {
+    if (!mbar_wait(K.barA, 1)) *K.flag = 1;  // dS's image
+    phase_issue(K, tid, [&] {
       mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
       mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
       mma_tile_mnmn<true>(tm + T_U1, sb + SB + 32768, 16384, sb + XH, 16384, 8, i64, true);
@@ -1126,6 +1121,17 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile<true>(tm + T_KDS, sb + SA + 32768, 16384, sb + KQ, 16384, 8, i64, true);
       return true;
     });
+    gdot += dot_state(S0, SA);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
+    if (lane == 0) red[warp] = gdot;
+    __syncthreads();
+    if (tid == 0) {
+      float s = 0.f;
+      for (int w = 0; w < NTP / 32; ++w) s += red[w];
+      *dGamC = s;
+    }
+    ok = phase_wait(K);
   }
   if (ok) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
