@@ -4,7 +4,8 @@
 // chunk_fwd.cu's header), written as the shared-memory images the
 // tensor-core scans copy into their operand slots.
 //
-// One chunk per CTA of 256 threads, two CTAs per SM:
+// Two persistent CTAs of 256 threads per SM, each walking chunks (the next
+// chunk's K, Q and gates are fetched while the current one finishes):
 //   1. the Gram matrices [K ; Q] K^T in one tcgen05 product (bf16 inputs are
 //      exact, fp32 accumulation; the query scale is applied to the result);
 //   2. thread (row, half) turns its TMEM row into the decayed, gated matrices
@@ -37,9 +38,10 @@ constexpr uint32_t AG = AB + 64 * LDA * 4;
 constexpr uint32_t TB = AG + 64 * LDA * 4;   // fp32 T_beta, T_gamma [64][LDT]
 constexpr uint32_t TG = TB + 64 * LDT * 4;
 constexpr uint32_t WS = TG + 64 * LDT * 4;   // product scratch, 2 x [32][LDW]
-constexpr uint32_t VEC = WS + 2 * 32 * LDW * 4;  // cum, cprev, beta, gamma, g (5 x 64)
-static_assert(TB % 16 == 0 && TG % 16 == 0 && WS % 16 == 0, "16-byte rows");
-constexpr uint32_t CTL = VEC + 5 * 64 * 4;   // mbarrier, flag
+// cum, cprev, beta, gamma, g, and cum, cprev times log2(e) (7 x 64)
+constexpr uint32_t VEC = WS + 2 * 32 * LDW * 4;
+static_assert(TB % 16 == 0 && TG % 16 == 0 && WS % 16 == 0 && VEC % 16 == 0, "16-byte rows");
+constexpr uint32_t CTL = VEC + 7 * 64 * 4;   // mbarrier, flag
 constexpr uint32_t SLOT = CTL + 16;          // TMEM base
 constexpr size_t SMEM = SLOT + 16;
 static_assert(2 * (SMEM + 1024) <= 233472, "two CTAs per SM");
@@ -157,7 +159,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     return;
   }
   float *cum = reinterpret_cast<float *>(sm + VEC), *cprev = cum + 64, *bet = cum + 128,
-        *gam = cum + 192, *gg = cum + 256;
+        *gam = cum + 192, *gg = cum + 256, *cum2 = cum + 320, *cprev2 = cum + 384;
   float *Ab = reinterpret_cast<float *>(sm + AB), *Ag = reinterpret_cast<float *>(sm + AG);
   float *Tb = reinterpret_cast<float *>(sm + TB), *Tg = reinterpret_cast<float *>(sm + TG);
   float *Wsc = reinterpret_cast<float *>(sm + WS);
@@ -165,12 +167,10 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
   volatile int *flag = reinterpret_cast<volatile int *>(sm + CTL + 8);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const size_t chunk = blockIdx.x;
   const int NC = p.NC, T = p.T, H = p.H;
-  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
-  const int b = bh / H, h = bh % H;
-  const int t0 = c * C, n = min(C, T - t0);
+  const size_t nct = (size_t)p.B * H * NC;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
+  constexpr float kLog2e = 1.4426950408889634f;
 
   if (tid == 0) {
     mbar_init(bar, 1);
@@ -178,128 +178,172 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     *flag = 0;
   }
   if (warp == 0) tmem_alloc(slot, 64);
-  for (int e = tid; e < 64 * 16; e += NTH) {  // K, Q (exact bf16), rows t, asynchronous
-    const int t = e >> 4, chn = e & 15;
-    const bool vld = t < n;
-    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
-    const int blk = chn >> 3, cc = (chn & 7) * 8;
-    cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
-    cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
-  }
-  if (tid < C) {
-    const int t = tid;
-    float gv = 0.f, bv = 0.f, mv = 0.f;
-    if (t < n) {
-      const size_t off = (size_t)(b * T + t0 + t) * H + h;
-      gv = p.g[off];
-      bv = p.beta[off];
-      mv = p.gamma[off];
+  // a chunk's K, Q (exact bf16, rows t, zero past the end), asynchronous, and
+  // its gates into registers (threads 0..63); fetched while the previous chunk
+  // of this CTA finishes
+  auto fetch_kq = [&](size_t ck) {
+    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
+    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * C, n_ = min(C, T - t0_);
+    for (int e = tid; e < 64 * 16; e += NTH) {
+      const int t = e >> 4, chn = e & 15;
+      const bool vld = t < n_;
+      const size_t off = ((size_t)(b_ * T + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
+      const int blk = chn >> 3, cc = (chn & 7) * 8;
+      cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
+      cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
     }
-    gg[t] = gv;
-    bet[t] = bv;
-    gam[t] = mv;
+  };
+  struct Gates {
+    float g, b, m;
+  };
+  auto fetch_gates = [&](size_t ck) {
+    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
+    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * C, n_ = min(C, T - t0_);
+    Gates x{0.f, 0.f, 0.f};
+    if (tid < C && tid < n_) {
+      const size_t off = (size_t)(b_ * T + t0_ + tid) * H + h_;
+      x.g = p.g[off];
+      x.b = p.beta[off];
+      x.m = p.gamma[off];
+    }
+    return x;
+  };
+  Gates gt{0.f, 0.f, 0.f};
+  if (blockIdx.x < nct) {
+    fetch_kq(blockIdx.x);
+    gt = fetch_gates(blockIdx.x);
   }
-  cp_async_wait_all();
-  fence_async_smem();
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   const uint32_t tm = *slot;
-  if (tid == 0) {  // [K ; Q] K^T: lanes 0..63 K K^T, lanes 64..127 Q K^T (unscaled)
-    mma_tile(tm, sb + KQ, 16384, sb + KQ, 16384, 8, idesc_bf16(128, 64), false);
-    mma_commit(bar);
-  }
-  if (warp == 0) {  // in-chunk cumulative log-decay, while the product runs
-    float a = gg[lane], a2 = gg[32 + lane];
+
+  bool ok = true;
+  uint32_t it = 0;  // chunks done by this CTA: the MMA barrier's parity
+  for (size_t chunk = blockIdx.x; chunk < nct && ok; chunk += gridDim.x, ++it) {
+    const size_t next = chunk + gridDim.x;
+    if (tid < C) {
+      gg[tid] = gt.g;
+      bet[tid] = gt.b;
+      gam[tid] = gt.m;
+    }
+    cp_async_wait_all();  // this chunk's K, Q
+    fence_async_smem();
+    fence_before_sync();
+    __syncthreads();  // (also: every thread is done with the previous chunk)
+    fence_after_sync();
+    if (tid == 0) {  // [K ; Q] K^T: lanes 0..63 K K^T, lanes 64..127 Q K^T (unscaled)
+      mma_tile(tm, sb + KQ, 16384, sb + KQ, 16384, 8, idesc_bf16(128, 64), false);
+      mma_commit(bar);
+    }
+    if (warp == 0) {  // in-chunk cumulative log-decay, while the product runs
+      float a = gg[lane], a2 = gg[32 + lane];
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const float ua = __shfl_up_sync(0xffffffffu, a, off);
-      const float ub = __shfl_up_sync(0xffffffffu, a2, off);
-      if (lane >= off) {
-        a += ua;
-        a2 += ub;
+      for (int off = 1; off < 32; off <<= 1) {
+        const float ua = __shfl_up_sync(0xffffffffu, a, off);
+        const float ub = __shfl_up_sync(0xffffffffu, a2, off);
+        if (lane >= off) {
+          a += ua;
+          a2 += ub;
+        }
       }
+      a2 += __shfl_sync(0xffffffffu, a, 31);
+      const float p1 = a - gg[lane], p2 = a2 - gg[32 + lane];
+      cum[lane] = a;
+      cum[32 + lane] = a2;
+      cprev[lane] = p1;
+      cprev[32 + lane] = p2;
+      cum2[lane] = a * kLog2e;
+      cum2[32 + lane] = a2 * kLog2e;
+      cprev2[lane] = p1 * kLog2e;
+      cprev2[32 + lane] = p2 * kLog2e;
     }
-    a2 += __shfl_sync(0xffffffffu, a, 31);
-    cum[lane] = a;
-    cum[32 + lane] = a2;
-    cprev[lane] = a - gg[lane];
-    cprev[32 + lane] = a2 - gg[32 + lane];
-  }
-  if (!mbar_wait(bar, 0)) *flag = 1;
-  __syncthreads();
-  fence_after_sync();
-  const bool ok = *flag == 0;
-  uint8_t *img = reinterpret_cast<uint8_t *>(p.ws + chunk * kRecFloats);
-  if (ok) {  // thread (row r, half hf) of the Gram read-out: columns i in [32 hf, 32 hf + 32)
-    const int r = tid & 127, hf = tid >> 7;
-    float gv[32];
-    {
-      const uint32_t ta = tm + ((uint32_t)((warp & 3) * 32) << 16) + 32 * hf;
-      float x[16];
-      tmem_ld16(ta, x);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) gv[i] = x[i];
-      tmem_ld16(ta + 16, x);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) gv[16 + i] = x[i];
+    if (!mbar_wait(bar, it & 1u)) *flag = 1;
+    __syncthreads();
+    fence_after_sync();
+    ok = *flag == 0;
+    if (!ok) break;
+    if (next < nct) {  // K, Q are done with: the next chunk's, during this one
+      fetch_kq(next);
+      gt = fetch_gates(next);
     }
-    if (r < 64) {  // K K^T row t: Ap (previous-token decay), A_beta, A_gamma (strict)
-      const int t = r;
-      const float ct = cum[t], cpt = cprev[t];
+    uint8_t *img = reinterpret_cast<uint8_t *>(p.ws + chunk * kRecFloats);
+    {  // thread (row r, half hf) of the Gram read-out: columns i in [32 hf, 32 hf + 32)
+      const int r = tid & 127, hf = tid >> 7;
+      float gv[32];
+      {
+        const uint32_t ta = tm + ((uint32_t)((warp & 3) * 32) << 16) + 32 * hf;
+        float x0[16], x1[16];
+        tmem_ld16x2(ta, x0, ta + 16, x1);
 #pragma unroll
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float ap[16];
+        for (int i = 0; i < 16; ++i) {
+          gv[i] = x0[i];
+          gv[16 + i] = x1[i];
+        }
+      }
+      if (r < 64) {  // K K^T row t: Ap (previous-token decay), A_beta, A_gamma (strict);
+                     // e^{b_t - b_i} = e^{b_{t-1} - b_i} e^{g_t}, both factors <= 1
+        const int t = r;
+        const float cp2 = cprev2[t], al = exp2f(cum2[t] - cp2);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int i = 32 * hf + c0 + u;
-          const float kk = gv[c0 + u];
-          float a_p = 0.f, a_b = 0.f, a_g = 0.f;
-          if (i < t) {
-            const float dec = __expf(ct - cum[i]);
-            a_p = __expf(cpt - cum[i]) * bet[i] * kk;
-            a_b = dec * bet[i] * kk;
-            a_g = dec * gam[i] * kk;
+        for (int c0 = 0; c0 < 32; c0 += 16) {
+          const int i0 = 32 * hf + c0;
+          float c2[16], bt[16], gm[16], ap[16];
+          lds16(cum2 + i0, c2);
+          lds16(bet + i0, bt);
+          lds16(gam + i0, gm);
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int i = i0 + u;
+            float a_p = 0.f, a_b = 0.f, a_g = 0.f;
+            if (i < t) {
+              const float dk = exp2f(cp2 - c2[u]) * gv[c0 + u];
+              a_p = dk * bt[u];
+              a_b = a_p * al;
+              a_g = dk * al * gm[u];
+            }
+            ap[u] = a_p;
+            Ab[t * LDA + i] = a_b;
+            Ag[t * LDA + i] = a_g;
           }
-          ap[u] = a_p;
-          Ab[t * LDA + i] = a_b;
-          Ag[t * LDA + i] = a_g;
+          img_row16(img + IMG_APMQ, 16384, t, i0, ap);
         }
-        img_row16(img + IMG_APMQ, 16384, t, 32 * hf + c0, ap);
-      }
-    } else {  // Q K^T row t: Mq (strict), diag(gamma) M2 (inclusive)
-      const int t = r - 64;
-      const float ct = cum[t], gt = gam[t];
+      } else {  // Q K^T row t: Mq (strict), diag(gamma) M2 (inclusive)
+        const int t = r - 64;
+        const float ct2 = cum2[t], gtt = gam[t];
 #pragma unroll
-      for (int c0 = 0; c0 < 32; c0 += 16) {
-        float mq[16], m2[16];
+        for (int c0 = 0; c0 < 32; c0 += 16) {
+          const int i0 = 32 * hf + c0;
+          float c2[16], bt[16], gm[16], mq[16], m2[16];
+          lds16(cum2 + i0, c2);
+          lds16(bet + i0, bt);
+          lds16(gam + i0, gm);
 #pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int i = 32 * hf + c0 + u;
-          const float qk = p.scale * gv[c0 + u];
-          const float dec = i <= t ? __expf(ct - cum[i]) : 0.f;
-          mq[u] = i < t ? dec * bet[i] * qk : 0.f;
-          m2[u] = gt * dec * gam[i] * qk;
+          for (int u = 0; u < 16; ++u) {
+            const int i = i0 + u;
+            const float qk = p.scale * gv[c0 + u];
+            const float dec = i <= t ? exp2f(ct2 - c2[u]) * qk : 0.f;
+            mq[u] = i < t ? dec * bt[u] : 0.f;
+            m2[u] = gtt * dec * gm[u];
+          }
+          img_row16(img + IMG_APMQ, 16384, 64 + t, i0, mq);
+          img_row16(img + IMG_M2, 8192, t, i0, m2);
         }
-        img_row16(img + IMG_APMQ, 16384, 64 + t, 32 * hf + c0, mq);
-        img_row16(img + IMG_M2, 8192, t, 32 * hf + c0, m2);
       }
     }
-  }
-  __syncthreads();
-  {  // T_beta (threads 0..127) and T_gamma (128..255)
-    const int g = tid & 127;
-    const float *A = tid < 128 ? Ab : Ag;
-    float *Tm = tid < 128 ? Tb : Tg;
-    float *W = Wsc + (tid < 128 ? 0 : 32 * LDW);
+    __syncthreads();
+    {  // T_beta (threads 0..127) and T_gamma (128..255)
+      const int g = tid & 127;
+      const float *A = tid < 128 ? Ab : Ag;
+      float *Tm = tid < 128 ? Tb : Tg;
+      float *W = Wsc + (tid < 128 ? 0 : 32 * LDW);
 #pragma unroll 1
-    for (int stage = 0; stage < 5; ++stage) {
-      if (stage) __syncthreads();
-      inv64_stage(stage, A, Tm, W, g);
+      for (int stage = 0; stage < 5; ++stage) {
+        if (stage) __syncthreads();
+        inv64_stage(stage, A, Tm, W, g);
+      }
     }
-  }
-  __syncthreads();
-  if (ok) {
+    __syncthreads();
     {  // image rows of T: thread (row r, matrix m, half hf)
       const int r = tid & 63, m = (tid >> 6) & 1, hf = tid >> 7;
       const float *Tm = m ? Tg : Tb;
@@ -307,8 +351,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
 #pragma unroll
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) v[u] = Tm[r * LDT + 32 * hf + c0 + u];
+        lds16(Tm + r * LDT + 32 * hf + c0, v);
         img_row16(dst, 8192, r, 32 * hf + c0, v);
       }
     }
@@ -323,9 +366,9 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
       rec[OFF_VEC + V_WR + t] = gam[t] * __expf(cC - cum[t]);
       if (t == 0) rec[OFF_VEC + V_GAMC] = __expf(cC);
     }
-  } else if (tid == 0 && p.err) {
-    atomicExch(p.err, RDN_ERR_TIMEOUT);
   }
+  if (!ok && tid == 0 && p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+  cp_async_wait_all();  // no copy of this CTA outlives it (a fetch for a chunk not reached)
   fence_before_sync();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, 64);
@@ -337,8 +380,13 @@ cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)pp::SMEM);
   if (e != cudaSuccess) return e;
-  RDN_LAUNCH("chunk_prep", s,
-             prep_tc_kernel<<<(unsigned)(p.B * p.H * p.NC), NTH, pp::SMEM, s>>>(p));
+  int dev = 0, nsm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return e;
+  const size_t nct = (size_t)p.B * p.H * p.NC;
+  const unsigned grid = (unsigned)(nct < 2 * (size_t)nsm ? nct : 2 * (size_t)nsm);  // two per SM
+  RDN_LAUNCH("chunk_prep", s, prep_tc_kernel<<<grid, NTH, pp::SMEM, s>>>(p));
   return cudaGetLastError();
 }
 
