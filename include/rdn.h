@@ -205,6 +205,12 @@ rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *args, rdn_stream_t stream);
  * Supports RDN_BF16 with Dk = Dv in {64, 128} and RDN_F32 likewise. */
 rdn_status_t rdn_bwd(const rdn_bwd_args *args, rdn_stream_t stream);
 
+/* Backward of rla_fwd, Section 3.4 (left formulation): the same arguments,
+ * layouts, ownership and errors as rdn_bwd, for the RLA recurrence.
+ * fwd.workspace / fwd.S_chunks refer to an rla_fwd call; fwd.flags must be 0
+ * (RDN_FLAG_SAVE_FOR_BWD is rdn_fwd's; RDN_ERR_UNSUPPORTED otherwise). */
+rdn_status_t rla_bwd(const rdn_bwd_args *args, rdn_stream_t stream);
+
 /* One recurrent step (Section 3.4 recurrence at a single t), states in
  * place; memory-bound: reads and writes S and R once. */
 rdn_status_t rdn_decode_step(const rdn_decode_args *args, rdn_stream_t stream);
@@ -213,6 +219,7 @@ rdn_status_t rdn_decode_step(const rdn_decode_args *args, rdn_stream_t stream);
  * Return RDN_OK and set *bytes, or an error for invalid shapes. */
 rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
 rdn_status_t rdn_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
+rdn_status_t rla_bwd_workspace_size(const rdn_bwd_args *args, size_t *bytes);
 rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *args, size_t *bytes);
 
 /* Message describing the last non-OK status returned on this thread

@@ -23,7 +23,7 @@ import torch
 from . import _abi
 from ._abi import BwdArgs, DecodeArgs, FwdArgs
 
-__all__ = ["rla_fwd", "rdn_fwd", "rdn_bwd", "rdn_decode_step", "RdnError", "library",
+__all__ = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "RdnError", "library",
            "CHUNK"]
 
 CHUNK = 64
@@ -148,6 +148,21 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     fwd_workspace: with them, the workspace that forward call used, whose
     per-chunk matrices are then reused instead of recomputed.
     fwd_saved: that forward ran with save_for_bwd=True."""
+    return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
+                R_chunks, workspace, out, fwd_workspace, fwd_saved)
+
+
+def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
+            scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
+            fwd_workspace=None):
+    """Backward of rla_fwd; the same arguments and results as rdn_bwd (no
+    saved intermediates: rla_fwd has no save_for_bwd)."""
+    return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
+                R_chunks, workspace, out, fwd_workspace, False)
+
+
+def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
+         workspace, out, fwd_workspace, fwd_saved):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -172,13 +187,14 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"])
     a.dS0, a.dR0 = _ptr(out.get("dS0")), _ptr(out.get("dR0"))
     nbytes = ctypes.c_size_t(0)
-    _check("rdn_bwd_workspace_size", lib.rdn_bwd_workspace_size(ctypes.byref(a), ctypes.byref(nbytes)))
+    _check(name + "_workspace_size",
+           getattr(lib, name + "_workspace_size")(ctypes.byref(a), ctypes.byref(nbytes)))
     ws = workspace
     if ws is None or ws.numel() < nbytes.value:
         ws = _alloc_ws(nbytes.value, dev)
     a.workspace = _ptr(ws)
     a.workspace_bytes = nbytes.value if ws is not None else 0
-    _check("rdn_bwd", lib.rdn_bwd(ctypes.byref(a), _stream(q)))
+    _check(name, getattr(lib, name)(ctypes.byref(a), _stream(q)))
     return out
 
 
@@ -237,7 +253,7 @@ class LaunchTimer:
 
 
 def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False):
-    """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rdn_bwd)."""
+    """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rla_bwd | rdn_bwd)."""
     lib = _abi.load()
     a = FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
@@ -245,10 +261,10 @@ def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False):
     a.clip, a.scale = 1.0, 1.0
     a.flags = _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0
     n = ctypes.c_size_t(0)
-    if op == "rdn_bwd":
+    if op in ("rla_bwd", "rdn_bwd"):
         b = BwdArgs()
         b.fwd = a
-        _check(op, lib.rdn_bwd_workspace_size(ctypes.byref(b), ctypes.byref(n)))
+        _check(op, getattr(lib, op + "_workspace_size")(ctypes.byref(b), ctypes.byref(n)))
     else:
         _check(op, getattr(lib, op + "_workspace_size")(ctypes.byref(a), ctypes.byref(n)))
     return n.value

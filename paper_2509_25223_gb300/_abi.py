@@ -16,9 +16,9 @@ STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "R
           4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}
 
 # every function the header declares (checked by the CPU tests)
-EXPORTS = ["rla_fwd", "rdn_fwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
-           "rdn_fwd_workspace_size", "rdn_bwd_workspace_size", "rdn_last_error", "rdn_version",
-           "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc"]
+EXPORTS = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
+           "rdn_fwd_workspace_size", "rla_bwd_workspace_size", "rdn_bwd_workspace_size",
+           "rdn_last_error", "rdn_version", "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc"]
 
 
 class ProfRecord(ctypes.Structure):
@@ -71,10 +71,12 @@ def load(build_if_missing: bool = True):
     for name, argt in [("rla_fwd", [ctypes.POINTER(FwdArgs), P]),
                        ("rdn_fwd", [ctypes.POINTER(FwdArgs), P]),
                        ("rdn_fwd_noalloc", [ctypes.POINTER(FwdArgs), P]),
+                       ("rla_bwd", [ctypes.POINTER(BwdArgs), P]),
                        ("rdn_bwd", [ctypes.POINTER(BwdArgs), P]),
                        ("rdn_decode_step", [ctypes.POINTER(DecodeArgs), P]),
                        ("rla_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rdn_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
+                       ("rla_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rdn_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)])]:
         fn = getattr(lib, name)
         fn.argtypes = argt

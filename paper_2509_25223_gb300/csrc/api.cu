@@ -294,18 +294,18 @@ rdn_status_t rdn_fwd(const rdn_fwd_args *a, rdn_stream_t stream) {
   return fwd_common("rdn_fwd", a, 1, (cudaStream_t)stream);
 }
 
-rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *a, size_t *bytes) {
-  const char *fn = "rdn_bwd_workspace_size";
+namespace {
+rdn_status_t bwd_workspace_common(const char *fn, const rdn_bwd_args *a, int variant,
+                                  size_t *bytes) {
   if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
   rdn_status_t st = check_fwd_shapes(fn, &a->fwd);
   if (st != RDN_OK) return st;
   if (!bytes) return fail(RDN_ERR_INVALID_ARG, "%s: bytes is NULL", fn);
-  *bytes = rdn::plan_bwd(*a).total_bytes;
+  *bytes = rdn::plan_bwd(*a, variant).total_bytes;
   return ok();
 }
 
-rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
-  const char *fn = "rdn_bwd";
+rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a, int variant, cudaStream_t stream) {
   if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
   rdn_status_t st = check_fwd_shapes(fn, &a->fwd);
   if (st != RDN_OK) return st;
@@ -331,6 +331,8 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
   OPTIONAL_PTR(f->R_chunks);
   if ((f->S_chunks == nullptr) != (f->R_chunks == nullptr))
     return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
+  if ((f->flags & RDN_FLAG_SAVE_FOR_BWD) && variant != 1)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: RDN_FLAG_SAVE_FOR_BWD is for rdn_fwd / rdn_bwd", fn);
   if ((f->flags & RDN_FLAG_SAVE_FOR_BWD) && !f->workspace && f->T > 0)
     return fail(RDN_ERR_INVALID_ARG,
                 "%s: RDN_FLAG_SAVE_FOR_BWD in fwd.flags needs the forward's fwd.workspace", fn);
@@ -340,7 +342,7 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
                   "%s: fwd.workspace is reused only together with fwd.S_chunks/R_chunks", fn);
     if (!aligned16(f->workspace))
       return fail(RDN_ERR_WORKSPACE, "%s: fwd.workspace is not 16-byte aligned", fn);
-    const size_t fneed = rdn::plan_fwd(*f, 1).total_bytes;
+    const size_t fneed = rdn::plan_fwd(*f, variant).total_bytes;
     if (f->workspace_bytes < fneed)
       return fail(RDN_ERR_WORKSPACE, "%s: fwd.workspace of %zu bytes required (got %zu)", fn, fneed,
                   f->workspace_bytes);
@@ -349,7 +351,7 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
   OPTIONAL_PTR(a->dRT);
   OPTIONAL_PTR(a->dS0);
   OPTIONAL_PTR(a->dR0);
-  const rdn::BwdPlan plan = rdn::plan_bwd(*a);
+  const rdn::BwdPlan plan = rdn::plan_bwd(*a, variant);
   if (plan.total_bytes > 0) {
     if (!a->workspace || a->workspace_bytes < plan.total_bytes)
       return fail(RDN_ERR_WORKSPACE, "%s: workspace of %zu bytes required (got %zu)", fn,
@@ -357,7 +359,24 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
     if (!aligned16(a->workspace))
       return fail(RDN_ERR_WORKSPACE, "%s: workspace is not 16-byte aligned", fn);
   }
-  return cuda_status(fn, rdn::launch_bwd(*a, (cudaStream_t)stream));
+  return cuda_status(fn, rdn::launch_bwd(*a, variant, stream));
+}
+}  // namespace
+
+rdn_status_t rla_bwd_workspace_size(const rdn_bwd_args *a, size_t *bytes) {
+  return bwd_workspace_common("rla_bwd_workspace_size", a, 0, bytes);
+}
+
+rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *a, size_t *bytes) {
+  return bwd_workspace_common("rdn_bwd_workspace_size", a, 1, bytes);
+}
+
+rdn_status_t rla_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
+  return bwd_common("rla_bwd", a, 0, (cudaStream_t)stream);
+}
+
+rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
+  return bwd_common("rdn_bwd", a, 1, (cudaStream_t)stream);
 }
 
 rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {

@@ -720,8 +720,11 @@ struct BwdLayout {
   size_t prep, acc, states, o, tc, total;
 };
 
-// bf16 inputs with d = 128 take the tensor-core backward
-bool use_tc_bwd(const rdn_fwd_args &f) { return f.dtype == RDN_BF16 && f.Dk == 128; }
+// RDN with bf16 inputs and d = 128 takes the tensor-core backward (RLA, whose
+// forward stays on the fp32 SIMT scan, the SIMT backward)
+bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
+  return variant == 1 && f.dtype == RDN_BF16 && f.Dk == 128;
+}
 
 // The forward's per-chunk records are valid input when the caller passes the
 // forward's workspace with its chunk-start states.  Both passes pick the same
@@ -729,32 +732,33 @@ bool use_tc_bwd(const rdn_fwd_args &f) { return f.dtype == RDN_BF16 && f.Dk == 1
 // and backward), fp32 otherwise.
 bool reuse_fwd_records(const rdn_fwd_args &f) { return f.workspace && f.S_chunks; }
 
-BwdLayout layout(const rdn_bwd_args &a) {
+BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const rdn_fwd_args &f = a.fwd;
+  const bool tc = use_tc_bwd(f, variant);
   const size_t nct = (size_t)f.B * f.H * ((f.T + C - 1) / C);
   const size_t accf = f.Dk == 128 ? Acc<128>::FLOATS : Acc<64>::FLOATS;
   BwdLayout l;
   // the forward's records are read from its workspace when it is passed
   l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nct * kRecFloats);
-  l.acc = use_tc_bwd(f) ? align256(bwd_tc_acc_bytes(f.B, f.H, (f.T + C - 1) / C))
-                        : align256(sizeof(float) * nct * accf);
+  l.acc = tc ? align256(bwd_tc_acc_bytes(f.B, f.H, (f.T + C - 1) / C))
+            : align256(sizeof(float) * nct * accf);
   const bool need_states = f.S_chunks == nullptr;
   l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
-  l.tc = use_tc_bwd(f) ? align256(bwd_tc_extra_bytes(f.B, f.H, (f.T + C - 1) / C)) : 0;
+  l.tc = tc ? align256(bwd_tc_extra_bytes(f.B, f.H, (f.T + C - 1) / C)) : 0;
   l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + 256;  // + device status word
   return l;
 }
 
 }  // namespace
 
-BwdPlan plan_bwd(const rdn_bwd_args &a) {
+BwdPlan plan_bwd(const rdn_bwd_args &a, int variant) {
   if (a.fwd.T == 0) return BwdPlan{0};
-  return BwdPlan{layout(a).total};
+  return BwdPlan{layout(a, variant).total};
 }
 
-cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
+cudaError_t launch_bwd(const rdn_bwd_args &a, int variant, cudaStream_t s) {
   const rdn_fwd_args &f = a.fwd;
   const size_t sbytes = sizeof(float) * (size_t)f.B * f.H * f.Dk * f.Dv;
   if (f.T == 0) {  // no tokens: the initial-state gradients are the upstream ones
@@ -766,7 +770,7 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
                 : cudaMemsetAsync(a.dR0, 0, sbytes, s);
     return e;
   }
-  const BwdLayout l = layout(a);
+  const BwdLayout l = layout(a, variant);
   char *ws = (char *)a.workspace;
   BwdParams p;
   p.f = make_fwd_params(f);
@@ -781,9 +785,9 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
   }
   p.f.ST = p.f.RT = nullptr;
   const bool bf = f.dtype == RDN_BF16;
-  const bool rdnv = true;
-  const bool tc = use_tc_bwd(f);
-  cudaError_t e;
+  const bool rdnv = variant == 1;
+  const bool tc = use_tc_bwd(f, variant);
+  cudaError_t e = cudaSuccess;  // (nothing to launch first when both the states and records are reused)
   if (f.S_chunks == nullptr) {  // recompute the chunk-start states
     p.f.S_chunks = (float *)(ws + l.prep + l.acc);
     p.f.R_chunks = (float *)(ws + l.prep + l.acc + l.states);
@@ -791,7 +795,7 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
     // the tensor-core forward leaves its records as shared-memory images,
     // which the tensor-core backward reads too; the SIMT backward needs fp32
-    if (e == cudaSuccess && bf && f.Dk == 128 && !tc)
+    if (e == cudaSuccess && rdnv && bf && f.Dk == 128 && !tc)
       e = launch_prep(p.f, f.Dk, rdnv, bf, false, s);
   } else if (!reuse) {
     e = launch_prep(p.f, f.Dk, rdnv, bf, tc, s);
@@ -816,8 +820,12 @@ cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s) {
                          a.dgamma, a.dS0, a.dR0, p.acc, ws + l.prep + l.acc + 2 * l.states + l.o,
                          s);
   if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
-  if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
-  return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
+  if (rdnv) {
+    if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
+    return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
+  }
+  if (f.Dk == 128) return bf ? launch_t<128, false, __nv_bfloat16>(p, s) : launch_t<128, false, float>(p, s);
+  return bf ? launch_t<64, false, __nv_bfloat16>(p, s) : launch_t<64, false, float>(p, s);
 }
 
 }  // namespace rdn

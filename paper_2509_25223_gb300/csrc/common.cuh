@@ -62,6 +62,6 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s);
 struct BwdPlan {
   size_t total_bytes;
 };
-BwdPlan plan_bwd(const rdn_bwd_args &a);
-cudaError_t launch_bwd(const rdn_bwd_args &a, cudaStream_t s);
+BwdPlan plan_bwd(const rdn_bwd_args &a, int variant);
+cudaError_t launch_bwd(const rdn_bwd_args &a, int variant, cudaStream_t s);
 }  // namespace rdn

@@ -149,6 +149,33 @@ def test_bwd_validation():
     assert lib.rdn_bwd(ctypes.byref(b), None) == 5
 
 
+def test_rla_bwd_validation():
+    """rla_bwd shares rdn_bwd's checks; the saved-intermediates flag is rdn_fwd's
+    and is refused; its workspace query answers for the RLA forward's layout."""
+    lib = _abi.load()
+    b = _abi.BwdArgs()
+    b.fwd = _fwd_args()
+    assert lib.rla_bwd(ctypes.byref(b), None) == 1
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE)
+    for f in ("dO", "dq", "dk", "dv", "dg", "dbeta", "dgamma"):
+        setattr(b, f, FAKE)
+    b.fwd = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, workspace=FAKE, workspace_bytes=1 << 40,
+                      S_chunks=FAKE, R_chunks=FAKE, **ok)
+    assert lib.rla_bwd(ctypes.byref(b), None) == 2
+    assert "RDN_FLAG_SAVE_FOR_BWD" in lib.rdn_last_error().decode()
+    n_rla, n_rdn = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    b.fwd = _fwd_args()
+    assert lib.rla_bwd_workspace_size(ctypes.byref(b), ctypes.byref(n_rla)) == 0
+    assert lib.rdn_bwd_workspace_size(ctypes.byref(b), ctypes.byref(n_rdn)) == 0
+    assert n_rla.value > 0 and n_rdn.value > 0
+    # the forward's workspace must be at least what rla_fwd asks for
+    nf = ctypes.c_size_t(0)
+    assert lib.rla_fwd_workspace_size(ctypes.byref(_fwd_args()), ctypes.byref(nf)) == 0
+    b.fwd = _fwd_args(workspace=FAKE, workspace_bytes=nf.value - 16, S_chunks=FAKE, R_chunks=FAKE,
+                      **ok)
+    assert lib.rla_bwd(ctypes.byref(b), None) == 5
+
+
 def test_binding_rejects_cpu_tensors():
     import torch
     x = torch.zeros(1, 64, 1, 64)

@@ -21,7 +21,7 @@ GRADS = ("dq", "dk", "dv", "dg", "dbeta", "dgamma", "dS0", "dR0")
 MARGIN = 1e-2
 
 
-def _condition(x, clip, dtype, heads=None):
+def _condition(x, clip, dtype, heads=None, variant=oracle.RDN):
     """Move v (in place on the device tensor) so the fp64 clip decisions have
     a margin; only the listed (b, h) heads when given."""
     sel = heads if heads is not None else [(b, h) for b in range(x["q"].shape[0])
@@ -30,16 +30,16 @@ def _condition(x, clip, dtype, heads=None):
         sl = {n: as64(x[n][b:b + 1, :, h:h + 1]) for n in NAMES}
         S0 = None if x["S0"] is None else as64(x["S0"][b:b + 1, h:h + 1])
         R0 = None if x["R0"] is None else as64(x["R0"][b:b + 1, h:h + 1])
-        v2, _ = oracle.clip_margin_condition(oracle.RDN, sl["q"], sl["k"], sl["v"], sl["g"],
+        v2, _ = oracle.clip_margin_condition(variant, sl["q"], sl["k"], sl["v"], sl["g"],
                                              sl["beta"], sl["gamma"], clip, S0, R0,
                                              margin=MARGIN, quant=dtype)
         x["v"][b, :, h] = torch.from_numpy(v2[0, :, 0]).to(x["v"].dtype).to(x["v"].device)
 
 
-def _ref(x, clip, dST=None, dRT=None, heads=None, scale=1.0):
+def _ref(x, clip, dST=None, dRT=None, heads=None, scale=1.0, variant=oracle.RDN):
     if heads is None:
-        return oracle.rdn_bwd(*(as64(x[n]) for n in NAMES), clip, as64(x["S0"]), as64(x["R0"]),
-                              as64(x["dO"]), as64(dST), as64(dRT), scale=scale)
+        return oracle.bwd(variant, *(as64(x[n]) for n in NAMES), clip, as64(x["S0"]),
+                          as64(x["R0"]), as64(x["dO"]), as64(dST), as64(dRT), scale=scale)
     outs = []
     for b, h in heads:
         sl = lambda t: None if t is None else as64(t[b:b + 1, :, h:h + 1])
@@ -49,9 +49,10 @@ def _ref(x, clip, dST=None, dRT=None, heads=None, scale=1.0):
     return outs
 
 
-def _gpu(x, clip, dST=None, dRT=None, **kw):
-    d = rdn.rdn_bwd(*(x[n] for n in NAMES), x["dO"], clip=clip, S0=x["S0"], R0=x["R0"],
-                    dST=dST, dRT=dRT, **kw)
+def _gpu(x, clip, dST=None, dRT=None, variant="rdn", **kw):
+    fn = rdn.rdn_bwd if variant == "rdn" else rdn.rla_bwd
+    d = fn(*(x[n] for n in NAMES), x["dO"], clip=clip, S0=x["S0"], R0=x["R0"], dST=dST, dRT=dRT,
+           **kw)
     torch.cuda.synchronize()
     return d
 
@@ -199,3 +200,55 @@ def test_dalpha_from_dg():
     ref = _ref(x, 1.0)
     alpha = np.exp(as64(x["g"]))
     np.testing.assert_allclose(as64(d["dg"]) / alpha, ref["dg"] / alpha, atol=2e-4, rtol=1e-4)
+
+
+# ------------------------------------------------------------------ rla_bwd
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("T", [1, 64, 65, 200])
+def test_rla_bwd_small(dtype, D, T):
+    """rla_bwd against the oracle's RLA back-propagation through time (nonzero
+    states, upstream state gradients, several chunks and a ragged tail)."""
+    clip = 1.0
+    x = make_inputs(2, T, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    gen = torch.Generator(device="cpu").manual_seed(17)
+    dST = torch.randn(x["S0"].shape, generator=gen).cuda()
+    dRT = torch.randn(x["R0"].shape, generator=gen).cuda()
+    _condition(x, clip, dtype, variant=oracle.RLA)
+    d = _gpu(x, clip, dST, dRT, variant="rla")
+    ref = _ref(x, clip, dST, dRT, variant=oracle.RLA)
+    for name in GRADS:
+        assert_close(d[name], ref[name], dtype, name)
+
+
+@pytest.mark.parametrize("clip", [0.3, float("inf")])
+def test_rla_bwd_clip_and_scale(clip):
+    scale = 128 ** -0.5
+    x = make_inputs(1, 130, 2, 128, dtype="bf16", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    _condition(x, clip, "bf16", variant=oracle.RLA)
+    d = _gpu(x, clip, variant="rla", scale=scale)
+    ref = _ref(x, clip, variant=oracle.RLA, scale=scale)
+    for name in GRADS:
+        assert_close(d[name], ref[name], "bf16", name)
+
+
+@pytest.mark.parametrize("dtype,D", [("bf16", 128), ("f32", 64)])
+def test_rla_bwd_reuses_forward(dtype, D):
+    """rla_bwd reading rla_fwd's chunk-start states and records gives the
+    recomputing backward's gradients, and the oracle's."""
+    x = make_inputs(2, 150, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    _condition(x, 1.0, dtype, variant=oracle.RLA)
+    nb = rdn.workspace_bytes("rla_fwd", 2, 150, 2, D,
+                             dtype=torch.bfloat16 if dtype == "bf16" else torch.float32)
+    ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    _, _, _, Sc, Rc = rdn.rla_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                                  return_chunk_states=True, workspace=ws)
+    d1 = _gpu(x, 1.0, variant="rla", S_chunks=Sc, R_chunks=Rc, fwd_workspace=ws)
+    d2 = _gpu(x, 1.0, variant="rla")
+    ref = _ref(x, 1.0, variant=oracle.RLA)
+    for name in GRADS:
+        torch.testing.assert_close(d1[name].float(), d2[name].float(), atol=1e-5, rtol=8e-3)
+        assert_close(d1[name], ref[name], dtype, name)
