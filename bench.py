@@ -485,6 +485,38 @@ def run_ours(args):
                "l2": "no flush: 1.07 GB of state per step, larger than L2"}
         del y, S, R
 
+    # ---- RLA fwd+bwd on the same workload (rla_fwd -> rla_bwd, chunk states
+    # and records reused as in the RDN step)
+    rla = None
+    if not args.no_rla:
+        wsr = torch.empty(rdn.workspace_bytes("rla_fwd", B, T, H, D), dtype=torch.uint8,
+                          device=dev)
+
+        def rstep(inp):
+            _, _, _, Sc_, Rc_ = rdn.rla_fwd(*(inp[n] for n in names), clip=w.clip,
+                                            return_chunk_states=True, out=o, workspace=wsr)
+            rdn.rla_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
+                        R_chunks=Rc_, out=grads, fwd_workspace=wsr)
+
+        rsteps = max(1, args.rla_steps)
+        rstep(x)
+        torch.cuda.synchronize()
+        barrier(dist)
+        with rdn.LaunchTimer() as ltr:
+            e0.record(stream)
+            for _ in range(rsteps):
+                rstep(x)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        barrier(dist)
+        tr, rval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * rsteps)
+        rla = {"workload": w.name.replace("rdn_", "rla_"), "value": rval, "unit": "tokens/s",
+               "steps": rsteps, "ms_per_step": tr / rsteps,
+               "path": "fp32 SIMT chunk kernels (RLA keeps fp32 state operands)",
+               "kernels": {k: {"launches": n, "mean_ms": m}
+                           for k, (n, t, m) in ltr.summary().items()}}
+        del wsr
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = time_oracle_sample(target_s=args.cpu_seconds)
@@ -505,7 +537,7 @@ def run_ours(args):
                 "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
                                 "share": t / sum(v[1] for v in kern.values())}
                             for k, (n, t, m) in kern.items()},
-                "clocks": clk.summary(), "decode": dec}
+                "clocks": clk.summary(), "decode": dec, "rla": rla}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -520,6 +552,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--decode-steps", type=int, default=1000)
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--rla-steps", type=int, default=3)
+    ap.add_argument("--no-rla", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")
