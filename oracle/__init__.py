@@ -190,6 +190,36 @@ def decode_step(variant, q, k, v, g, beta, gamma, c, S, R, scale=1.0):
     return o, S, R
 
 
+# ----------------------------------------------------------- q, k prologue
+# Section 3.4 leaves out of its equations the SiLU activation and the L2
+# normalisation that the model applies to queries and keys before the
+# recurrence; the reading here: SiLU first, then normalisation over the head
+# dimension, with the norm floored at eps like the listing's normalisation.
+
+def qk_prologue(x, eps=1e-12):
+    """y = u / max(||u||_2, eps), u = SiLU(x) = x * sigmoid(x), over the last
+    axis of x (rows of q or k, [..., D])."""
+    x = _f64(x)
+    u = x / (1.0 + np.exp(-x))
+    n = np.sqrt((u * u).sum(-1, keepdims=True))
+    return u / np.maximum(n, eps)
+
+
+def qk_prologue_bwd(x, dy, eps=1e-12):
+    """Gradient of <dy, qk_prologue(x)> w.r.t. x, by the chain rule through the
+    two steps: with y = u / n (n = ||u|| > eps) du = (dy - y <y, dy>) / n, with
+    n <= eps du = dy / eps; then dx = du * SiLU'(x), SiLU'(x) = s (1 + x (1 - s)),
+    s = sigmoid(x)."""
+    x, dy = _f64(x), _f64(dy)
+    s = 1.0 / (1.0 + np.exp(-x))
+    u = x * s
+    n = np.sqrt((u * u).sum(-1, keepdims=True))
+    big = n > eps
+    y = u / np.maximum(n, eps)
+    du = np.where(big, (dy - y * (y * dy).sum(-1, keepdims=True)) / np.maximum(n, eps), dy / eps)
+    return du * s * (1.0 + x * (1.0 - s))
+
+
 QUANT = {"f64": 0, "f32": 1, "bf16": 2}
 
 

@@ -513,3 +513,55 @@ def test_chunkwise_backward_equals_bptt(variant, name, C):
                     x["R0"], x["dO"], dST, dRT, C=C, scale=0.7)
     for key in ref:
         np.testing.assert_allclose(got[key], ref[key], atol=1e-10, err_msg=key)
+
+
+# ------------------------------------------------ q, k prologue (SiLU, L2 norm)
+def test_qk_prologue_rows_have_unit_norm_and_silu_direction():
+    """Each row of the output is the unit vector along SiLU(x): norm 1, and
+    parallel to x * sigmoid(x) computed with scipy's logistic function."""
+    from scipy.special import expit
+    x = np.random.default_rng(3).standard_normal((5, 7, 128)) * 2.0
+    y = oracle.qk_prologue(x)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=-1), 1.0, atol=1e-14)
+    u = x * expit(x)
+    np.testing.assert_allclose(y * np.linalg.norm(u, axis=-1, keepdims=True), u, atol=1e-12)
+
+
+def test_qk_prologue_closed_forms():
+    """One-element rows: y = sign(SiLU(x)) (SiLU(x) > 0 iff x > 0); an all-zero
+    row falls under the floor and stays zero; x = ln 3 has sigmoid 3/4."""
+    x = np.array([[2.0], [-0.5], [0.0]])
+    y = oracle.qk_prologue(x)
+    np.testing.assert_array_equal(y[:, 0], [1.0, -1.0, 0.0])
+    x2 = np.array([[np.log(3.0), 0.0]])  # SiLU = (ln 3) 3/4 and 0: the unit row (1, 0)
+    np.testing.assert_allclose(oracle.qk_prologue(x2), [[1.0, 0.0]], atol=1e-15)
+    # the norm floor: y = u / eps for rows whose SiLU is tiny
+    tiny = np.array([[1e-14, -2e-14]])
+    u = tiny / (1.0 + np.exp(-tiny))
+    np.testing.assert_allclose(oracle.qk_prologue(tiny, eps=1e-12), u / 1e-12, rtol=1e-12)
+
+
+def test_qk_prologue_backward_matches_autograd():
+    """Against fp64 autograd of torch's silu and normalize (library routines)."""
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal((3, 4, 64)) * 1.5
+    dy = rng.standard_normal(x.shape)
+    t = torch.tensor(x, requires_grad=True)
+    y = torch.nn.functional.normalize(torch.nn.functional.silu(t), dim=-1, eps=1e-12)
+    (y * torch.from_numpy(dy)).sum().backward()
+    np.testing.assert_allclose(oracle.qk_prologue(x), y.detach().numpy(), atol=1e-14)
+    np.testing.assert_allclose(oracle.qk_prologue_bwd(x, dy), t.grad.numpy(), atol=1e-12)
+
+
+def test_qk_prologue_backward_finite_differences():
+    rng = np.random.default_rng(6)
+    x = rng.standard_normal((2, 16))
+    dy = rng.standard_normal(x.shape)
+    g = oracle.qk_prologue_bwd(x, dy)
+    eps = 1e-6
+    for idx in [(0, 0), (0, 7), (1, 3), (1, 15)]:
+        xp, xm = x.copy(), x.copy()
+        xp[idx] += eps
+        xm[idx] -= eps
+        fd = ((oracle.qk_prologue(xp) - oracle.qk_prologue(xm)) * dy).sum() / (2 * eps)
+        assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
