@@ -517,6 +517,39 @@ def run_ours(args):
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr
 
+    # ---- q, k prologue (SiLU + L2 norm) and its backward on the bench
+    # workload's q, k: algorithmic bytes = each element read and written once
+    # (the backward also reads dy), against the measured HBM peak
+    pro = None
+    if not args.no_prologue:
+        dq_, dk_ = torch.empty_like(x["q"]), torch.empty_like(x["k"])
+        yq_, yk_ = torch.empty_like(x["q"]), torch.empty_like(x["k"])
+
+        def pstep():
+            rdn.qk_prologue(x["q"], x["k"], out=(yq_, yk_))
+            rdn.qk_prologue_bwd(x["q"], x["k"], x["dO"], x["dO"])
+
+        psteps = 20
+        for _ in range(3):
+            pstep()
+        torch.cuda.synchronize()
+        with rdn.LaunchTimer(capacity=2 * psteps + 8) as ltp:
+            for _ in range(psteps):
+                pstep()
+            torch.cuda.synchronize()
+        kp = ltp.summary()
+        elem = x["q"].numel() * x["q"].element_size()  # bytes of one tensor
+        fwd_bytes, bwd_bytes = 4 * elem, 6 * elem
+        mf, mb = kp["qk_prologue"][2], kp["qk_prologue_bwd"][2]
+        pro = {"workload": "qk_prologue_bf16_B8T4096H16D128 (q and k)",
+               "fwd_ms": mf, "fwd_gbs": fwd_bytes / (mf * 1e-3) / 1e9,
+               "bwd_ms": mb, "bwd_gbs": bwd_bytes / (mb * 1e-3) / 1e9,
+               "fwd_frac_of_hbm_peak": fwd_bytes / (mf * 1e-3) / 1e9 / peaks["hbm"],
+               "bwd_frac_of_hbm_peak": bwd_bytes / (mb * 1e-3) / 1e9 / peaks["hbm"],
+               "bytes": {"fwd": fwd_bytes, "bwd": bwd_bytes}, "launches": psteps,
+               "l2": "no flush: 268 MB of q, k per pass, larger than L2"}
+        del dq_, dk_, yq_, yk_
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = time_oracle_sample(target_s=args.cpu_seconds)
@@ -537,7 +570,7 @@ def run_ours(args):
                 "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
                                 "share": t / sum(v[1] for v in kern.values())}
                             for k, (n, t, m) in kern.items()},
-                "clocks": clk.summary(), "decode": dec, "rla": rla}
+                "clocks": clk.summary(), "decode": dec, "rla": rla, "prologue": pro}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -554,6 +587,7 @@ def main(argv=None):
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--rla-steps", type=int, default=3)
     ap.add_argument("--no-rla", action="store_true")
+    ap.add_argument("--no-prologue", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")

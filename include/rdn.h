@@ -165,6 +165,39 @@ typedef struct {
   void *o;
 } rdn_decode_args;
 
+/* Arguments of rdn_qk_prologue / rdn_qk_prologue_bwd: the activation and
+ * normalisation the model applies to queries and keys before the recurrence
+ * (Section 3.4 leaves them out of its equations): per row of D elements
+ *     u = SiLU(x) = x * sigmoid(x),   y = u / max(||u||_2, eps).
+ *   rows              number of rows of each tensor (B*T*H for q or k), >= 1.
+ *   D                 row length, 64 or 128.
+ *   dtype             RDN_BF16 or RDN_F32 for every tensor below.
+ *   eps               norm floor, > 0 and finite (1e-12 matches common
+ *                     normalisation defaults).
+ *   x[i]              pre-activation rows [rows][D] (q in x[0], k in x[1];
+ *                     x[1] may be NULL for one tensor).  Read only.
+ *   y[i]              (prologue) outputs [rows][D], may not alias x.
+ *   dy[i], dx[i]      (backward) upstream gradients of y and the gradients
+ *                     w.r.t. x [rows][D]; the backward recomputes y from x.
+ * Every pointer is a caller-owned 16-byte aligned device pointer; unused
+ * fields are ignored.  Errors: RDN_ERR_INVALID_ARG (rows < 1, eps, NULL
+ * pointers), RDN_ERR_UNSUPPORTED (D, dtype), RDN_ERR_MISALIGNED. */
+typedef struct {
+  long long rows;
+  int D;
+  int dtype; /* rdn_dtype_t */
+  float eps;
+  const void *x[2];
+  void *y[2];
+  const void *dy[2];
+  void *dx[2];
+} rdn_prologue_args;
+
+/* y = SiLU(x) / max(||SiLU(x)||, eps) row-wise for one or two tensors. */
+rdn_status_t rdn_qk_prologue(const rdn_prologue_args *args, rdn_stream_t stream);
+/* dx = d<dy, y>/dx of the same map. */
+rdn_status_t rdn_qk_prologue_bwd(const rdn_prologue_args *args, rdn_stream_t stream);
+
 /* RLA forward, Section 3.4 (left formulation).  Chunkwise-parallel form:
  * additive base state, no triangular solves. */
 rdn_status_t rla_fwd(const rdn_fwd_args *args, rdn_stream_t stream);

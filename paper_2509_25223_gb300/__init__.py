@@ -23,7 +23,7 @@ import torch
 from . import _abi
 from ._abi import BwdArgs, DecodeArgs, FwdArgs
 
-__all__ = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "RdnError", "library",
+__all__ = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "qk_prologue", "qk_prologue_bwd", "rdn_decode_step", "RdnError", "library",
            "CHUNK"]
 
 CHUNK = 64
@@ -196,6 +196,45 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
     a.workspace_bytes = nbytes.value if ws is not None else 0
     _check(name, getattr(lib, name)(ctypes.byref(a), _stream(q)))
     return out
+
+
+def _prologue_args(x0, x1, eps):
+    a = _abi.PrologueArgs()
+    D = x0.shape[-1]
+    a.rows = x0.numel() // D
+    a.D = D
+    a.dtype = _dtype_code(x0)
+    a.eps = float(eps)
+    a.x[0], a.x[1] = _ptr(x0), _ptr(x1)
+    if x1 is not None and x1.shape != x0.shape:
+        raise ValueError("q and k must have the same shape")
+    return a
+
+
+def qk_prologue(q, k=None, eps=1e-12, out=None):
+    """SiLU then L2 normalisation over the last axis, of q and (optionally) k
+    in one launch: y = SiLU(x) / max(||SiLU(x)||, eps).  Returns (q', k') (k'
+    None when k is None)."""
+    lib = _abi.load()
+    yq = out[0] if out is not None else torch.empty_like(q)
+    yk = (out[1] if out is not None else torch.empty_like(k)) if k is not None else None
+    a = _prologue_args(q, k, eps)
+    a.y[0], a.y[1] = _ptr(yq), _ptr(yk)
+    _check("rdn_qk_prologue", lib.rdn_qk_prologue(ctypes.byref(a), _stream(q)))
+    return yq, yk
+
+
+def qk_prologue_bwd(q, k, dyq, dyk=None, eps=1e-12):
+    """Gradients w.r.t. the pre-activation q, k of <dyq, q'> + <dyk, k'>
+    (q', k' from qk_prologue; recomputed from q, k).  k / dyk may be None."""
+    lib = _abi.load()
+    dq = torch.empty_like(q)
+    dk = torch.empty_like(k) if k is not None else None
+    a = _prologue_args(q, k, eps)
+    a.dy[0], a.dy[1] = _ptr(dyq), _ptr(dyk)
+    a.dx[0], a.dx[1] = _ptr(dq), _ptr(dk)
+    _check("rdn_qk_prologue_bwd", lib.rdn_qk_prologue_bwd(ctypes.byref(a), _stream(q)))
+    return dq, dk
 
 
 def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant="rdn", out=None):

@@ -18,7 +18,8 @@ STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "R
 # every function the header declares (checked by the CPU tests)
 EXPORTS = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
            "rdn_fwd_workspace_size", "rla_bwd_workspace_size", "rdn_bwd_workspace_size",
-           "rdn_last_error", "rdn_version", "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc"]
+           "rdn_last_error", "rdn_version", "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc",
+           "rdn_qk_prologue", "rdn_qk_prologue_bwd"]
 
 
 class ProfRecord(ctypes.Structure):
@@ -49,6 +50,12 @@ class DecodeArgs(ctypes.Structure):
                 ("S", P), ("R", P), ("o", P)]
 
 
+class PrologueArgs(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_longlong), ("D", ctypes.c_int), ("dtype", ctypes.c_int),
+                ("eps", ctypes.c_float), ("x", P * 2), ("y", P * 2), ("dy", P * 2),
+                ("dx", P * 2)]
+
+
 _lib = None
 
 
@@ -74,6 +81,8 @@ def load(build_if_missing: bool = True):
                        ("rla_bwd", [ctypes.POINTER(BwdArgs), P]),
                        ("rdn_bwd", [ctypes.POINTER(BwdArgs), P]),
                        ("rdn_decode_step", [ctypes.POINTER(DecodeArgs), P]),
+                       ("rdn_qk_prologue", [ctypes.POINTER(PrologueArgs), P]),
+                       ("rdn_qk_prologue_bwd", [ctypes.POINTER(PrologueArgs), P]),
                        ("rla_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rdn_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rla_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)]),

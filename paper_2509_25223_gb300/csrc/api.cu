@@ -379,6 +379,41 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
   return bwd_common("rdn_bwd", a, 1, (cudaStream_t)stream);
 }
 
+namespace {
+rdn_status_t prologue_common(const char *fn, const rdn_prologue_args *a, bool bwd,
+                             cudaStream_t stream) {
+  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  if (a->rows < 1 || a->rows > (1ll << 40))
+    return fail(RDN_ERR_INVALID_ARG, "%s: rows must be in [1, 2^40] (got %lld)", fn, a->rows);
+  if (a->D != 64 && a->D != 128)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: supported row lengths are D in {64, 128}", fn);
+  if (a->dtype != RDN_F32 && a->dtype != RDN_BF16)
+    return fail(RDN_ERR_UNSUPPORTED, "%s: dtype %d unsupported", fn, a->dtype);
+  if (!(a->eps > 0.f) || isinf(a->eps))
+    return fail(RDN_ERR_INVALID_ARG, "%s: eps must be positive and finite", fn);
+  for (int i = 0; i < 2; ++i) {
+    if (i == 1 && !a->x[1]) break;
+    REQUIRE_PTR(a->x[i]);
+    if (!bwd) {
+      REQUIRE_PTR(a->y[i]);
+      if (a->y[i] == a->x[i]) return fail(RDN_ERR_INVALID_ARG, "%s: y aliases x", fn);
+    } else {
+      REQUIRE_PTR(a->dy[i]);
+      REQUIRE_PTR(a->dx[i]);
+    }
+  }
+  return cuda_status(fn, rdn::launch_prologue(*a, bwd, stream));
+}
+}  // namespace
+
+rdn_status_t rdn_qk_prologue(const rdn_prologue_args *a, rdn_stream_t stream) {
+  return prologue_common("rdn_qk_prologue", a, false, (cudaStream_t)stream);
+}
+
+rdn_status_t rdn_qk_prologue_bwd(const rdn_prologue_args *a, rdn_stream_t stream) {
+  return prologue_common("rdn_qk_prologue_bwd", a, true, (cudaStream_t)stream);
+}
+
 rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {
   const char *fn = "rdn_decode_step";
   if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);

@@ -50,6 +50,7 @@ void end(cudaStream_t s);
 // launches.
 namespace rdn {
 cudaError_t launch_decode(const rdn_decode_args &a, cudaStream_t s);
+cudaError_t launch_prologue(const rdn_prologue_args &a, bool bwd, cudaStream_t s);
 
 struct FwdPlan {
   int NC;                // chunks per sequence

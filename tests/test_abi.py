@@ -182,3 +182,57 @@ def test_binding_rejects_cpu_tensors():
     g = torch.zeros(1, 64, 1)
     with pytest.raises(ValueError):
         rdn.rla_fwd(x, x, x, g, g, g)
+
+
+_STRUCTS = {
+    "rdn_fwd_args": ("FwdArgs", ["B", "q", "clip", "S0", "scale", "flags", "workspace",
+                                 "workspace_bytes"]),
+    "rdn_bwd_args": ("BwdArgs", ["fwd", "dO", "dq", "dS0", "dR0", "workspace",
+                                 "workspace_bytes"]),
+    "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o"]),
+    "rdn_prologue_args": ("PrologueArgs", ["rows", "D", "dtype", "eps", "x", "y", "dy", "dx"]),
+}
+
+
+def test_binding_struct_layouts_match_the_header(tmp_path):
+    """sizeof and field offsets of every argument struct, as the C compiler lays
+    them out from include/rdn.h, equal those of the ctypes binding."""
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "rdn.h"', "int main(void) {"]
+    for cname, (_, fields) in _STRUCTS.items():
+        src.append(f'  printf("{cname} size %zu\\n", sizeof({cname}));')
+        for f in fields:
+            src.append(f'  printf("{cname} {f} %zu\\n", offsetof({cname}, {f}));')
+    src += ["  return 0;", "}"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    got = {tuple(ln.split()[:2]): int(ln.split()[2]) for ln in out if ln.strip()}
+    for cname, (pyname, fields) in _STRUCTS.items():
+        st = getattr(_abi, pyname)
+        assert got[(cname, "size")] == ctypes.sizeof(st), cname
+        for f in fields:
+            assert got[(cname, f)] == getattr(st, f).offset, (cname, f)
+
+
+def test_prologue_validation():
+    lib = _abi.load()
+    a = _abi.PrologueArgs()
+    a.rows, a.D, a.dtype, a.eps = 16, 128, _abi.RDN_BF16, 1e-12
+    assert lib.rdn_qk_prologue(ctypes.byref(a), None) == 1  # x[0] NULL
+    a.x[0], a.y[0] = FAKE, ctypes.c_void_p(0x20000)
+    a.D = 96
+    assert lib.rdn_qk_prologue(ctypes.byref(a), None) == 2
+    a.D = 128
+    a.eps = 0.0
+    assert lib.rdn_qk_prologue(ctypes.byref(a), None) == 1
+    a.eps = 1e-12
+    a.y[0] = FAKE  # aliases x
+    assert lib.rdn_qk_prologue(ctypes.byref(a), None) == 1
+    a.y[0] = ctypes.c_void_p(0x20004)  # misaligned
+    assert lib.rdn_qk_prologue(ctypes.byref(a), None) == 6
+    a.rows = 0
+    assert lib.rdn_qk_prologue_bwd(ctypes.byref(a), None) == 1
+    a.rows = 16
+    assert lib.rdn_qk_prologue_bwd(ctypes.byref(a), None) == 1  # dy[0] NULL
