@@ -76,6 +76,14 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  * backward; on the others the flag only reserves the space. */
 #define RDN_FLAG_SAVE_FOR_BWD 0x1u
 
+/* RDN_FLAG_TIED_GAMMA (all four entry points): the residual rate is tied to
+ * the base rate, gamma_t = beta_t (the paper's tied-gate ablation): `gamma`
+ * is ignored (may be NULL) and `beta` serves as both.  rla_bwd / rdn_bwd then
+ * return in dbeta the gradient w.r.t. the shared gate (the sum of the two
+ * gates' gradients of the untied computation); dgamma may be NULL, and if
+ * given receives the gamma part alone.  The backward's fwd.flags carries it. */
+#define RDN_FLAG_TIED_GAMMA 0x2u
+
 /* Arguments of rla_fwd / rdn_fwd.
  *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
  *                     S0/R0 to ST/RT).
@@ -94,7 +102,8 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *                     stored).  rdn_bwd can consume them instead of
  *                     recomputing.
  *   scale             multiplies q (the paper uses 1).
- *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd (above).
+ *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd and / or
+ *                     RDN_FLAG_TIED_GAMMA (above).
  *   workspace         device scratch of *_fwd_workspace_size() bytes.     */
 typedef struct {
   int B, T, H, Dk, Dv;
@@ -127,7 +136,8 @@ typedef struct {
  *                     gamma, scale and clip as in that call are the caller's
  *                     responsibility (not checked).  It is only read.
  *   fwd.flags         RDN_FLAG_SAVE_FOR_BWD if that forward ran with it
- *                     (then fwd.workspace is required), else 0.
+ *                     (then fwd.workspace is required), and
+ *                     RDN_FLAG_TIED_GAMMA for tied gates; else 0.
  *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
  *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
  *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype.

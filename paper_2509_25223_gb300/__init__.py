@@ -90,7 +90,7 @@ def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
          return_final_state=True, return_chunk_states=False, out=None, workspace=None,
-         save_for_bwd=False):
+         save_for_bwd=False, tied_gamma=False):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -106,7 +106,8 @@ def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
         Rc = torch.empty_like(Sc)
     a = FwdArgs()
     _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale,
-              _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0)
+              (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0)
+              | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0))
     nbytes = ctypes.c_size_t(0)
     _check(name + "_workspace_size",
            getattr(lib, name + "_workspace_size")(ctypes.byref(a), ctypes.byref(nbytes)))
@@ -140,7 +141,7 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, fwd_saved=False):
+            fwd_workspace=None, fwd_saved=False, tied_gamma=False):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
@@ -149,20 +150,20 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     per-chunk matrices are then reused instead of recomputed.
     fwd_saved: that forward ran with save_for_bwd=True."""
     return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, fwd_saved)
+                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma)
 
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None):
+            fwd_workspace=None, tied_gamma=False):
     """Backward of rla_fwd; the same arguments and results as rdn_bwd (no
     saved intermediates: rla_fwd has no save_for_bwd)."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, False)
+                R_chunks, workspace, out, fwd_workspace, False, tied_gamma)
 
 
 def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
-         workspace, out, fwd_workspace, fwd_saved):
+         workspace, out, fwd_workspace, fwd_saved, tied_gamma=False):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -180,11 +181,11 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
     if fwd_workspace is not None:
         a.fwd.workspace = _ptr(fwd_workspace)
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
-    if fwd_saved:
-        a.fwd.flags = _abi.RDN_FLAG_SAVE_FOR_BWD
+    a.fwd.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if fwd_saved else 0) \
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0)
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
-    a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out["dgamma"])
+    a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out.get("dgamma"))
     a.dS0, a.dR0 = _ptr(out.get("dS0")), _ptr(out.get("dR0"))
     nbytes = ctypes.c_size_t(0)
     _check(name + "_workspace_size",

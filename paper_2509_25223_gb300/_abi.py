@@ -11,6 +11,7 @@ F = ctypes.POINTER(ctypes.c_float)
 
 RDN_F32, RDN_BF16 = 0, 1
 RDN_FLAG_SAVE_FOR_BWD = 0x1  # rdn_fwd_args.flags (include/rdn.h)
+RDN_FLAG_TIED_GAMMA = 0x2
 
 STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "RDN_ERR_CUDA",
           4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}

@@ -98,7 +98,7 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
   if ((long long)a->B * a->T * a->H > (1ll << 31) / 128)
     return fail(RDN_ERR_UNSUPPORTED, "%s: B*T*H = %lld too large", fn,
                 (long long)a->B * a->T * a->H);
-  if (a->flags & ~RDN_FLAG_SAVE_FOR_BWD)
+  if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
   if (isnan(a->scale) || isinf(a->scale))
     return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
@@ -128,14 +128,23 @@ rdn_status_t check_fwd_ptrs(const char *fn, const rdn_fwd_args *a) {
   return RDN_OK;
 }
 
+// The arguments with the tied-gate flag resolved: gamma is beta.
+rdn_fwd_args untied(const rdn_fwd_args &a) {
+  rdn_fwd_args u = a;
+  if (a.flags & RDN_FLAG_TIED_GAMMA) u.gamma = a.beta;
+  return u;
+}
+
 rdn_status_t cuda_status(const char *fn, cudaError_t e) {
   if (e == cudaSuccess) return ok();
   return fail(RDN_ERR_CUDA, "%s: CUDA error %d (%s)", fn, (int)e, cudaGetErrorString(e));
 }
 
-rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a, int variant, cudaStream_t s) {
-  rdn_status_t st = check_fwd_shapes(fn, a);
+rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a0, int variant, cudaStream_t s) {
+  rdn_status_t st = check_fwd_shapes(fn, a0);
   if (st != RDN_OK) return st;
+  const rdn_fwd_args ua = untied(*a0);
+  const rdn_fwd_args *a = &ua;
   if (variant == 0 && (a->flags & RDN_FLAG_SAVE_FOR_BWD))
     return fail(RDN_ERR_UNSUPPORTED, "%s: RDN_FLAG_SAVE_FOR_BWD is for rdn_fwd", fn);
   if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
@@ -223,10 +232,12 @@ std::mutex g_noalloc_mu;
 void *g_noalloc_ptr[kMaxDevices] = {};
 }  // namespace
 
-rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a, rdn_stream_t stream) {
+rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a0, rdn_stream_t stream) {
   const char *fn = "rdn_fwd_noalloc";
-  rdn_status_t st = check_fwd_shapes(fn, a);
+  rdn_status_t st = check_fwd_shapes(fn, a0);
   if (st != RDN_OK) return st;
+  const rdn_fwd_args ua = untied(*a0);
+  const rdn_fwd_args *a = &ua;
   if (a->flags & RDN_FLAG_SAVE_FOR_BWD)  // what it saves would stay in the built-in scratch
     return fail(RDN_ERR_UNSUPPORTED,
                 "%s: RDN_FLAG_SAVE_FOR_BWD needs a caller workspace (use rdn_fwd)", fn);
@@ -305,10 +316,13 @@ rdn_status_t bwd_workspace_common(const char *fn, const rdn_bwd_args *a, int var
   return ok();
 }
 
-rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a, int variant, cudaStream_t stream) {
-  if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
-  rdn_status_t st = check_fwd_shapes(fn, &a->fwd);
+rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a0, int variant, cudaStream_t stream) {
+  if (!a0) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
+  rdn_status_t st = check_fwd_shapes(fn, &a0->fwd);
   if (st != RDN_OK) return st;
+  rdn_bwd_args ua = *a0;
+  ua.fwd = untied(a0->fwd);
+  const rdn_bwd_args *a = &ua;
   const rdn_fwd_args *f = &a->fwd;
   if (f->T > 0) {
     REQUIRE_PTR(f->q);
@@ -323,8 +337,9 @@ rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a, int variant, cuda
     REQUIRE_PTR(a->dv);
     REQUIRE_PTR(a->dg);
     REQUIRE_PTR(a->dbeta);
-    REQUIRE_PTR(a->dgamma);
+    if (!(f->flags & RDN_FLAG_TIED_GAMMA)) REQUIRE_PTR(a->dgamma);
   }
+  OPTIONAL_PTR(a->dgamma);
   OPTIONAL_PTR(f->S0);
   OPTIONAL_PTR(f->R0);
   OPTIONAL_PTR(f->S_chunks);

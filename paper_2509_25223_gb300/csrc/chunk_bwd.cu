@@ -717,7 +717,7 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct BwdLayout {
-  size_t prep, acc, states, o, tc, total;
+  size_t prep, acc, states, o, tc, tied, total;
 };
 
 // RDN with bf16 inputs and d = 128 takes the tensor-core backward (RLA, whose
@@ -747,7 +747,11 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
   l.tc = tc ? align256(bwd_tc_extra_bytes(f.B, f.H, (f.T + C - 1) / C)) : 0;
-  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + 256;  // + device status word
+  // tied gates without a dgamma buffer: the gamma part is made here, then added
+  l.tied = (f.flags & RDN_FLAG_TIED_GAMMA) && !a.dgamma
+               ? align256(sizeof(float) * (size_t)f.B * f.T * f.H)
+               : 0;
+  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.tied + 256;  // + device status word
   return l;
 }
 
@@ -758,7 +762,32 @@ BwdPlan plan_bwd(const rdn_bwd_args &a, int variant) {
   return BwdPlan{layout(a, variant).total};
 }
 
-cudaError_t launch_bwd(const rdn_bwd_args &a, int variant, cudaStream_t s) {
+static __global__ void add_inplace_kernel(float *__restrict__ a, const float *__restrict__ b,
+                                          size_t n) {
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x)
+    a[i] += b[i];
+}
+
+static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStream_t s);
+
+cudaError_t launch_bwd(const rdn_bwd_args &a0, int variant, cudaStream_t s) {
+  const rdn_fwd_args &f = a0.fwd;
+  if (!(f.flags & RDN_FLAG_TIED_GAMMA) || f.T == 0) return launch_bwd_impl(a0, variant, s);
+  // tied gates (gamma is beta): the untied gradients, then dbeta += dgamma
+  rdn_bwd_args a = a0;
+  const BwdLayout l = layout(a0, variant);
+  // (after what the untied backward uses: its own plan is l.total - l.tied bytes)
+  if (!a.dgamma) a.dgamma = (float *)((char *)a.workspace + l.total - l.tied);
+  cudaError_t e = launch_bwd_impl(a, variant, s);
+  if (e != cudaSuccess) return e;
+  const size_t n = (size_t)f.B * f.T * f.H;
+  const unsigned grid = (unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
+  RDN_LAUNCH("tied_gate_grad", s, add_inplace_kernel<<<grid, 256, 0, s>>>(a.dbeta, a.dgamma, n));
+  return cudaGetLastError();
+}
+
+static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStream_t s) {
   const rdn_fwd_args &f = a.fwd;
   const size_t sbytes = sizeof(float) * (size_t)f.B * f.H * f.Dk * f.Dv;
   if (f.T == 0) {  // no tokens: the initial-state gradients are the upstream ones

@@ -64,7 +64,12 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(dtype=7)) == 2
     assert _status(fn, _fwd_args(clip=-1.0)) == 1
     assert _status(fn, _fwd_args(clip=float("nan"))) == 1
-    assert _status(fn, _fwd_args(flags=2)) == 2
+    assert _status(fn, _fwd_args(flags=4)) == 2
+    # tied gates: gamma may be NULL (beta serves as both); the call then gets
+    # as far as the workspace check
+    tied = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, o=FAKE)
+    assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_TIED_GAMMA, **tied)) == 5
+    assert _status(fn, _fwd_args(flags=0, **tied)) == 1  # untied: gamma is required
     # RDN_FLAG_SAVE_FOR_BWD: rdn_fwd only, and only with chunk states
     assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD)) == (2 if fn == "rla_fwd" else 1)
     assert _status(fn, _fwd_args()) == 1  # q is NULL

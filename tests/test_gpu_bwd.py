@@ -252,3 +252,36 @@ def test_rla_bwd_reuses_forward(dtype, D):
     for name in GRADS:
         torch.testing.assert_close(d1[name].float(), d2[name].float(), atol=1e-5, rtol=8e-3)
         assert_close(d1[name], ref[name], dtype, name)
+
+
+# ------------------------------------------------------------- tied gates
+@pytest.mark.parametrize("variant,dtype,D", [("rdn", "bf16", 128), ("rdn", "f32", 64),
+                                             ("rla", "bf16", 128)])
+def test_tied_gates(variant, dtype, D):
+    """RDN_FLAG_TIED_GAMMA: the forward with gamma omitted equals the oracle at
+    gamma = beta, and the backward returns the shared gate's gradient in dbeta
+    (dgamma not requested: the library keeps the gamma part in its workspace)."""
+    ov = oracle.RDN if variant == "rdn" else oracle.RLA
+    x = make_inputs(2, 130, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    x["gamma"] = x["beta"]
+    _condition(x, 1.0, dtype, variant=ov)
+    fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
+    o, ST, RT = fwd(*(x[n] for n in NAMES[:5]), None, clip=1.0, S0=x["S0"], R0=x["R0"],
+                    tied_gamma=True)
+    ref_o, ref_ST, _ = oracle.fwd(ov, *(as64(x[n]) for n in NAMES), 1.0, as64(x["S0"]),
+                                  as64(x["R0"]))
+    assert_close(o, ref_o, dtype, "o")
+    assert_close(ST, ref_ST, dtype, "ST")
+    B, T, H = x["g"].shape
+    out = dict(dq=torch.empty_like(x["q"]), dk=torch.empty_like(x["k"]), dv=torch.empty_like(x["v"]),
+               dg=torch.empty(B, T, H, device="cuda"), dbeta=torch.empty(B, T, H, device="cuda"),
+               dS0=torch.empty_like(x["S0"]), dR0=torch.empty_like(x["R0"]))
+    bwd = rdn.rdn_bwd if variant == "rdn" else rdn.rla_bwd
+    d = bwd(*(x[n] for n in NAMES[:5]), None, x["dO"], clip=1.0, S0=x["S0"], R0=x["R0"],
+            out=out, tied_gamma=True)
+    torch.cuda.synchronize()
+    ref = _ref(x, 1.0, variant=ov)
+    assert_close(d["dbeta"], ref["dbeta"] + ref["dgamma"], dtype, "dbeta (tied)")
+    for name in ("dq", "dk", "dv", "dg", "dS0", "dR0"):
+        assert_close(d[name], ref[name], dtype, name)

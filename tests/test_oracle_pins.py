@@ -565,3 +565,20 @@ def test_qk_prologue_backward_finite_differences():
         xm[idx] -= eps
         fd = ((oracle.qk_prologue(xp) - oracle.qk_prologue(xm)) * dy).sum() / (2 * eps)
         assert abs(fd - g[idx]) < 1e-7, (idx, fd, g[idx])
+
+
+@pytest.mark.parametrize("variant", [RLA, RDN])
+def test_tied_gate_gradient_matches_autograd(variant):
+    """Tied gates (gamma = beta, the paper's tied-gate ablation): the gradient
+    w.r.t. the shared gate, formed from the oracle as dbeta + dgamma of the
+    untied computation at gamma = beta, equals fp64 autograd of the recurrence
+    driven by one gate tensor."""
+    x = _inputs(B=1, T=40, H=2, D=5, Dv=4, seed=8)
+    c = 0.7
+    T_ = {n: torch.tensor(a, requires_grad=True) for n, a in x.items() if a is not None and n != "dO"}
+    o, ST, RT = _torch_recurrence(variant, T_["q"], T_["k"], T_["v"], torch.exp(T_["g"]),
+                                  T_["beta"], T_["beta"], c, T_["S0"], T_["R0"])
+    (o * torch.from_numpy(x["dO"])).sum().backward()
+    d = oracle.bwd(variant, x["q"], x["k"], x["v"], x["g"], x["beta"], x["beta"], c, x["S0"],
+                   x["R0"], x["dO"])
+    np.testing.assert_allclose(d["dbeta"] + d["dgamma"], T_["beta"].grad.numpy(), atol=1e-11)
