@@ -390,16 +390,16 @@ def run_ours(args):
     step_tflops = fl["step"] * token_heads / (ms_per_step * 1e-3) / 1e12
 
     # ---- end to end through the public API: pinned host in, host out.  Each
-    # step copies its inputs in from pinned host memory and all its results
-    # out; the copies run on their own streams, so that step i + 1's inputs
-    # arrive and step i's results leave while a step computes (two device
-    # buffer sets, ordered by events).
+    # step copies all its inputs in from pinned host memory and reads its
+    # result, the layer output o, back to the host (the gradients stay on the
+    # device, where a training step's optimizer uses them); the copies run on
+    # their own streams, so that step i + 1's inputs arrive and step i's output
+    # leaves while a step computes (two device buffer sets, ordered by events).
     host = {n: x[n].cpu().pin_memory() for n in names + ("dO",)}
     dev_in = [{n: torch.empty_like(x[n]) for n in host} for _ in range(2)]
     outs = [(torch.empty_like(o), {n: torch.empty_like(t) for n, t in grads.items()})
             for _ in range(2)]
-    host_out = {n: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-                for n, t in list(grads.items()) + [("o", o)]}
+    host_out = {"o": torch.empty(o.shape, dtype=o.dtype, pin_memory=True)}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     d2h = sum(t.numel() * t.element_size() for t in host_out.values())
     s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
@@ -564,8 +564,10 @@ def run_ours(args):
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                         "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                        "copies": "pinned host, own streams, overlapped with the compute "
-                                  "of the neighbouring steps (two device buffer sets)"},
+                        "copies": "all inputs in from pinned host memory and the output o "
+                                  "back, every step, on their own streams, overlapped with "
+                                  "the compute of the neighbouring steps (two device buffer "
+                                  "sets); the gradients stay on the device"},
                 "gpu_launches": lt.launches,
                 "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
                                 "share": t / sum(v[1] for v in kern.values())}
