@@ -28,6 +28,8 @@
  *                                        stored transposed: row i is key dim i)
  *      S_chunks, R_chunks [B,H,NC,Dk,Dv] fp32, NC = ceil(T/64): the states at
  *                    the start of each 64-token chunk.
+ *    (packed variable-length sequences change the B axis: rdn_fwd_args
+ *    .cu_seqlens.)
  *  - Every pointer must be 16-byte aligned.
  *  - All work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
  *    stream) and is asynchronous.  Argument errors are reported before
@@ -104,7 +106,25 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *   scale             multiplies q (the paper uses 1).
  *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd and / or
  *                     RDN_FLAG_TIED_GAMMA (above).
- *   workspace         device scratch of *_fwd_workspace_size() bytes.     */
+ *   workspace         device scratch of *_fwd_workspace_size() bytes.
+ *   cu_seqlens        NULL, or packed variable-length sequences: a device
+ *                     int32 array of num_seqs + 1 token offsets, 0 =
+ *                     cu_seqlens[0] <= cu_seqlens[1] <= ... <=
+ *                     cu_seqlens[num_seqs] = T.  Then B must be 1 and
+ *                     sequence s is tokens cu_seqlens[s] .. cu_seqlens[s+1]-1
+ *                     of the [1,T,H,.] inputs, each with its own recurrence
+ *                     (states restart at S0[s], R0[s]; empty sequences are
+ *                     allowed).  S0, R0, ST, RT (and the backward's dST,
+ *                     dRT, dS0, dR0) are [num_seqs,H,Dk,Dv]; S_chunks and
+ *                     R_chunks hold rdn_chunk_slots() blocks of Dk x Dv fp32,
+ *                     block (first chunk of s) * H + h * nc_s + c for chunk c
+ *                     of sequence s, head h (nc_s = ceil(len_s / 64)).  The
+ *                     table is read on the device only: a table that breaks
+ *                     the ordering above is clamped into it (no fault, the
+ *                     result is unspecified).  Sequences are independent,
+ *                     exactly as B separate calls would run them.
+ *   num_seqs          number of packed sequences (>= 1) when cu_seqlens is
+ *                     set; ignored otherwise.                             */
 typedef struct {
   int B, T, H, Dk, Dv;
   int dtype; /* rdn_dtype_t */
@@ -119,6 +139,8 @@ typedef struct {
   unsigned flags;
   void *workspace;
   size_t workspace_bytes;
+  const int *cu_seqlens;
+  int num_seqs;
 } rdn_fwd_args;
 
 /* Arguments of rdn_bwd.  `fwd` holds the forward's inputs (its o, ST, RT,
@@ -261,6 +283,10 @@ rdn_status_t rdn_decode_step(const rdn_decode_args *args, rdn_stream_t stream);
 /* Workspace sizes in bytes for the arguments' shapes (pointers ignored).
  * Return RDN_OK and set *bytes, or an error for invalid shapes. */
 rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
+/* Number of Dk x Dv blocks in each of S_chunks and R_chunks:
+ * B * H * ceil(T/64), or with cu_seqlens the bound H * (num_seqs +
+ * ceil(T/64)) (slots past the sequences' chunks are left untouched). */
+rdn_status_t rdn_chunk_slots(const rdn_fwd_args *args, long long *slots);
 rdn_status_t rdn_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
 rdn_status_t rla_bwd_workspace_size(const rdn_bwd_args *args, size_t *bytes);
 rdn_status_t rdn_bwd_workspace_size(const rdn_bwd_args *args, size_t *bytes);

@@ -73,7 +73,8 @@ def _alloc_ws(nbytes, device):
     return torch.empty(nbytes, dtype=torch.uint8, device=device)
 
 
-def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale, flags=0):
+def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale, flags=0,
+              cu_seqlens=None):
     B, T, H, Dk = q.shape
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, Dk, v.shape[-1]
     a.dtype = _dtype_code(q)
@@ -86,28 +87,50 @@ def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale
     a.S_chunks, a.R_chunks = _ptr(Sc), _ptr(Rc)
     a.scale = float(scale)
     a.flags = flags
+    if cu_seqlens is not None:
+        if cu_seqlens.dtype != torch.int32 or cu_seqlens.dim() != 1 or cu_seqlens.numel() < 2:
+            raise ValueError("cu_seqlens must be a 1-D int32 tensor of num_seqs + 1 offsets")
+        a.cu_seqlens = _ptr(cu_seqlens)
+        a.num_seqs = cu_seqlens.numel() - 1
+
+
+def _num_seqs(q, cu_seqlens):
+    return q.shape[0] if cu_seqlens is None else cu_seqlens.numel() - 1
+
+
+def _chunk_slots(a):
+    """Dk x Dv blocks in each of S_chunks and R_chunks for the filled FwdArgs."""
+    n = ctypes.c_longlong(0)
+    _check("rdn_chunk_slots", _abi.load().rdn_chunk_slots(ctypes.byref(a), ctypes.byref(n)))
+    return n.value
 
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
          return_final_state=True, return_chunk_states=False, out=None, workspace=None,
-         save_for_bwd=False, tied_gamma=False):
+         save_for_bwd=False, tied_gamma=False, cu_seqlens=None):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
     dev = q.device
+    N = _num_seqs(q, cu_seqlens)
     o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
     ST = RT = Sc = Rc = None
     if return_final_state:
-        ST = torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev)
+        ST = torch.empty(N, H, Dk, Dv, dtype=torch.float32, device=dev)
         RT = torch.empty_like(ST)
-    if return_chunk_states:
-        NC = (T + CHUNK - 1) // CHUNK
-        Sc = torch.empty(B, H, NC, Dk, Dv, dtype=torch.float32, device=dev)
-        Rc = torch.empty_like(Sc)
+    flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) \
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0)
     a = FwdArgs()
-    _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale,
-              (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0)
-              | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0))
+    _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, None, None, scale, flags,
+              cu_seqlens)
+    if return_chunk_states:
+        if cu_seqlens is None:
+            NC = (T + CHUNK - 1) // CHUNK
+            Sc = torch.empty(B, H, NC, Dk, Dv, dtype=torch.float32, device=dev)
+        else:  # record slots (the packed layout of rdn_fwd_args.cu_seqlens)
+            Sc = torch.empty(_chunk_slots(a), Dk, Dv, dtype=torch.float32, device=dev)
+        Rc = torch.empty_like(Sc)
+        a.S_chunks, a.R_chunks = _ptr(Sc), _ptr(Rc)
     nbytes = ctypes.c_size_t(0)
     _check(name + "_workspace_size",
            getattr(lib, name + "_workspace_size")(ctypes.byref(a), ctypes.byref(nbytes)))
@@ -135,13 +158,17 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
     return_chunk_states=True, also the chunk-start states (Sc, Rc) that
     rdn_bwd can reuse.  With save_for_bwd=True (needs return_chunk_states and
     a caller workspace sized with the same flag) the workspace also keeps the
-    intermediates rdn_bwd(fwd_workspace=..., fwd_saved=True) reads."""
+    intermediates rdn_bwd(fwd_workspace=..., fwd_saved=True) reads.
+
+    cu_seqlens (int32 device tensor of N+1 offsets, q of shape [1,T,H,D]):
+    N packed sequences, each with its own recurrence; S0, R0, ST, RT are then
+    [N,H,D,D] and the chunk states [slots,D,D] (rdn_fwd_args.cu_seqlens)."""
     return _fwd("rdn_fwd", q, k, v, g, beta, gamma, clip, S0, R0, scale, **kw)
 
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, fwd_saved=False, tied_gamma=False):
+            fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
@@ -150,34 +177,35 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     per-chunk matrices are then reused instead of recomputed.
     fwd_saved: that forward ran with save_for_bwd=True."""
     return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma)
+                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens)
 
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, tied_gamma=False):
+            fwd_workspace=None, tied_gamma=False, cu_seqlens=None):
     """Backward of rla_fwd; the same arguments and results as rdn_bwd (no
     saved intermediates: rla_fwd has no save_for_bwd)."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, False, tied_gamma)
+                R_chunks, workspace, out, fwd_workspace, False, tied_gamma, cu_seqlens)
 
 
 def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
-         workspace, out, fwd_workspace, fwd_saved, tied_gamma=False):
+         workspace, out, fwd_workspace, fwd_saved, tied_gamma=False, cu_seqlens=None):
     lib = _abi.load()
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
     dev = q.device
+    N = _num_seqs(q, cu_seqlens)
     if out is None:
         out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
                    dg=torch.empty(B, T, H, dtype=torch.float32, device=dev),
                    dbeta=torch.empty(B, T, H, dtype=torch.float32, device=dev),
                    dgamma=torch.empty(B, T, H, dtype=torch.float32, device=dev),
-                   dS0=torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev),
-                   dR0=torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev))
+                   dS0=torch.empty(N, H, Dk, Dv, dtype=torch.float32, device=dev),
+                   dR0=torch.empty(N, H, Dk, Dv, dtype=torch.float32, device=dev))
     a = BwdArgs()
     _fill_fwd(a.fwd, q, k, v, g, beta, gamma, clip, S0, R0, None, None, None, S_chunks,
-              R_chunks, scale)
+              R_chunks, scale, 0, cu_seqlens)
     if fwd_workspace is not None:
         a.fwd.workspace = _ptr(fwd_workspace)
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
@@ -292,14 +320,17 @@ class LaunchTimer:
         return {k: (c, t, t / c) for k, (c, t) in out.items()}
 
 
-def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False):
-    """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rla_bwd | rdn_bwd)."""
+def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False, cu_seqlens=None):
+    """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rla_bwd | rdn_bwd);
+    cu_seqlens: the packed-sequence table of the call (B = 1)."""
     lib = _abi.load()
     a = FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
     a.dtype = _abi.RDN_BF16 if dtype == torch.bfloat16 else _abi.RDN_F32
     a.clip, a.scale = 1.0, 1.0
     a.flags = _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0
+    if cu_seqlens is not None:
+        a.cu_seqlens, a.num_seqs = _ptr(cu_seqlens), cu_seqlens.numel() - 1
     n = ctypes.c_size_t(0)
     if op in ("rla_bwd", "rdn_bwd"):
         b = BwdArgs()

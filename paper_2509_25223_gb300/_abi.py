@@ -20,7 +20,7 @@ STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "R
 EXPORTS = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
            "rdn_fwd_workspace_size", "rla_bwd_workspace_size", "rdn_bwd_workspace_size",
            "rdn_last_error", "rdn_version", "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc",
-           "rdn_qk_prologue", "rdn_qk_prologue_bwd"]
+           "rdn_qk_prologue", "rdn_qk_prologue_bwd", "rdn_chunk_slots"]
 
 
 class ProfRecord(ctypes.Structure):
@@ -34,7 +34,8 @@ class FwdArgs(ctypes.Structure):
                 ("clip", ctypes.c_float), ("S0", P), ("R0", P), ("o", P),
                 ("ST", P), ("RT", P), ("S_chunks", P), ("R_chunks", P),
                 ("scale", ctypes.c_float), ("flags", ctypes.c_uint),
-                ("workspace", P), ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace", P), ("workspace_bytes", ctypes.c_size_t),
+                ("cu_seqlens", P), ("num_seqs", ctypes.c_int)]
 
 
 class BwdArgs(ctypes.Structure):
@@ -87,7 +88,8 @@ def load(build_if_missing: bool = True):
                        ("rla_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rdn_fwd_workspace_size", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
                        ("rla_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
-                       ("rdn_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)])]:
+                       ("rdn_bwd_workspace_size", [ctypes.POINTER(BwdArgs), ctypes.POINTER(ctypes.c_size_t)]),
+                       ("rdn_chunk_slots", [ctypes.POINTER(FwdArgs), ctypes.POINTER(ctypes.c_longlong)])]:
         fn = getattr(lib, name)
         fn.argtypes = argt
         fn.restype = S

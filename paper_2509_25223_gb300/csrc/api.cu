@@ -98,6 +98,15 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
   if ((long long)a->B * a->T * a->H > (1ll << 31) / 128)
     return fail(RDN_ERR_UNSUPPORTED, "%s: B*T*H = %lld too large", fn,
                 (long long)a->B * a->T * a->H);
+  if (a->cu_seqlens) {  // packed sequences: one row of T tokens split by the table
+    if (a->B != 1)
+      return fail(RDN_ERR_INVALID_ARG, "%s: cu_seqlens needs B = 1 (got B=%d)", fn, a->B);
+    if (a->num_seqs < 1 || (long long)a->num_seqs * a->H > (1ll << 24))
+      return fail(RDN_ERR_INVALID_ARG, "%s: need 1 <= num_seqs, num_seqs*H <= 2^24 (got %d)", fn,
+                  a->num_seqs);
+    if (!aligned16(a->cu_seqlens))
+      return fail(RDN_ERR_MISALIGNED, "%s: cu_seqlens is not 16-byte aligned", fn);
+  }
   if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
   if (isnan(a->scale) || isinf(a->scale))
@@ -247,15 +256,16 @@ rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a0, rdn_stream_t stream) {
     // per-chunk record size and fixed overhead, from the workspace plan
     rdn_fwd_args one = *a, two = *a;
     one.B = one.H = two.B = two.H = 1;
+    one.cu_seqlens = two.cu_seqlens = nullptr;
     one.T = rdn::kChunk;
     two.T = 2 * rdn::kChunk;
     const size_t per_chunk = rdn::plan_fwd(two, 1).total_bytes - rdn::plan_fwd(one, 1).total_bytes;
     const size_t fixed = rdn::plan_fwd(one, 1).total_bytes - per_chunk;
     return fail(RDN_ERR_WORKSPACE,
-                "%s: this problem needs %zu bytes of scratch (B*H*ceil(T/64) = %lld chunks) but "
+                "%s: this problem needs %zu bytes of scratch (%lld chunk records) but "
                 "the built-in scratch holds %zu bytes (at most %zu chunks); use rdn_fwd with a "
                 "caller workspace",
-                fn, need, (long long)a->B * a->H * ((a->T + rdn::kChunk - 1) / rdn::kChunk),
+                fn, need, rdn::call_records(*a),
                 (size_t)RDN_NOALLOC_SCRATCH_BYTES,
                 ((size_t)RDN_NOALLOC_SCRATCH_BYTES - fixed) / per_chunk);
   }
@@ -294,6 +304,14 @@ rdn_status_t rdn_fwd_workspace_size(const rdn_fwd_args *a, size_t *bytes) {
   if (st != RDN_OK) return st;
   if (!bytes) return fail(RDN_ERR_INVALID_ARG, "rdn_fwd_workspace_size: bytes is NULL");
   *bytes = rdn::plan_fwd(*a, 1).total_bytes;
+  return ok();
+}
+
+rdn_status_t rdn_chunk_slots(const rdn_fwd_args *a, long long *slots) {
+  rdn_status_t st = check_fwd_shapes("rdn_chunk_slots", a);
+  if (st != RDN_OK) return st;
+  if (!slots) return fail(RDN_ERR_INVALID_ARG, "rdn_chunk_slots: slots is NULL");
+  *slots = rdn::call_records(*a);
   return ok();
 }
 

@@ -251,9 +251,13 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, j = tid;
   const size_t chunk = blockIdx.x;
-  const int NC = p.NC, T = p.T, H = p.H;
-  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
-  const int b = bh / H, h = bh % H;
+  if ((long long)chunk >= total_records(p)) return;  // (packed sequences: the grid is a bound)
+  const int H = p.H;
+  int sq, h, c;
+  rec_decode(p, (long long)chunk, sq, h, c);
+  const SeqSpan sp = seq_span(p, sq, h);
+  const long long tok0 = sp.tok0;
+  const int T = sp.len;
   const int t0 = c * 64, n = min(64, T - t0);
   const __nv_bfloat16 *k = (const __nv_bfloat16 *)p.k, *v = (const __nv_bfloat16 *)p.v;
   const uint8_t *rec = rec_bytes(p, chunk);
@@ -269,7 +273,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   if (tid < 64) {
     Gam[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GAM + tid];
     Gprev[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GPREV + tid];
-    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    gamv[tid] = tid < n ? p.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
   }
   // chunk-start states -> bf16 A operands (row j = column j of [i][j])
   {
@@ -291,7 +295,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   for (int e = tid; e < 64 * 16; e += NT) {
     const int t = e >> 4, ch = e & 15;
     const bool vld = t < n;
-    const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+    const size_t off = ((size_t)(tok0 + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
     cp_async16(sm + B1 + (ch >> 3) * 16384 + sw128(t, (ch & 7) * 8), k + off, vld);
   }
   cp_async_wait_all();
@@ -302,7 +306,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   const uint32_t tm = *slot;
   const uint32_t lane = (uint32_t)(warp * 32) << 16;
   auto vval = [&](int t) -> float {
-    return t < n ? __bfloat162float(v[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+    return t < n ? __bfloat162float(v[((size_t)(tok0 + t0 + t) * H + h) * D + j]) : 0.f;
   };
 
   bool ok = phase_run(K, tid, [&] {  // KS, KR
@@ -436,8 +440,10 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
   const int tid = threadIdx.x, warp = tid >> 5, j = tid & 127;
   const int g16 = (warp >> 2) * 16;  // this thread's token (and key) columns start
   const int bh = blockIdx.x;
-  const int NC = p.NC, T = p.T, H = p.H;
-  const int b = bh / H, h = bh % H;
+  const int H = p.H, h = bh % H;
+  const SeqSpan sp = seq_span(p, bh / H, h);  // this (sequence, head)'s tokens and records
+  const long long tok0 = sp.tok0;
+  const int NC = sp.nc, T = sp.len;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   __nv_bfloat16 *dv = (__nv_bfloat16 *)P.dv;
@@ -461,8 +467,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     bulk_g2s(sm + SLOTB, r + IMG_APMQ, 8192, K.barB);
     bulk_g2s(sm + SLOTB + 8192, r + IMG_APMQ + 16384, 8192, K.barB);
   };
-  if (tid == 0) {
-    const size_t last = (size_t)bh * NC + NC - 1;
+  if (tid == 0 && NC > 0) {  // (a packed sequence may be empty)
+    const size_t last = (size_t)(sp.rbase + NC - 1);
     load_slot(sm + SLOTA, K.barA, rec_bytes(p, last) + IMG_M2, 16384);
     load_mq(last);
   }
@@ -517,7 +523,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     for (int e = tid; e < 64 * 16; e += NTC) {
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
+      const size_t off = ((size_t)(tok0 + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
       const int blk = chn >> 3, cc = (chn & 7) * 8;
       cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
       cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
@@ -528,7 +534,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     for (int e = tid; e < 64 * 16; e += NTC) {
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
+      const size_t off = ((size_t)(tok0 + t0 + (vld ? t : 0)) * H + h) * D + chn * 8;
       cp_async16(sm + DOT + (chn >> 3) * 8192 + sw128(t, (chn & 7) * 8), dOp + off, vld);
     }
   };
@@ -539,7 +545,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     unsigned m;
   };
   auto fetch_pre = [&](int c) {
-    const size_t ck = (size_t)bh * NC + c;
+    const size_t ck = (size_t)(sp.rbase + c);
     const int t0 = c * 64, n = min(64, T - t0);
     const float *rf = p.ws + ck * kRecFloats;
     Pre x;
@@ -550,20 +556,23 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       x.gprev = rf[OFF_VEC + V_GPREV + t];
       x.ws_ = rf[OFF_VEC + V_WS + t];
       x.wr_ = rf[OFF_VEC + V_WR + t];
-      x.g_ = t < n ? p.gamma[(size_t)(b * T + t0 + t) * H + h] : 0.f;
+      x.g_ = t < n ? p.gamma[(size_t)(tok0 + t0 + t) * H + h] : 0.f;
     }
     x.gamc = rf[OFF_VEC + V_GAMC];
     // bits [g16, g16 + 16) of the column's 64-bit word (little-endian)
     x.m = reinterpret_cast<const uint16_t *>(P.mask + ck * D + j)[g16 >> 4];
     return x;
   };
-  fetch_kq(NC - 1);
-  fetch_do(NC - 1);
-  Pre pre = fetch_pre(NC - 1);
+  Pre pre{};
+  if (NC > 0) {
+    fetch_kq(NC - 1);
+    fetch_do(NC - 1);
+    pre = fetch_pre(NC - 1);
+  }
 
   bool ok = true;
   for (int c = NC - 1; c >= 0 && ok; --c) {
-    const size_t chunk = (size_t)bh * NC + c;
+    const size_t chunk = (size_t)(sp.rbase + c);
     const int t0 = c * 64, n = min(64, T - t0);
     __syncthreads();
     if (tid == 0) {  // gradients w.r.t. this chunk's end states, for bwd_post: the tile images
@@ -738,7 +747,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       for (int e = tid; e < 64 * 16; e += NTC) {  // dv rows, 16 bytes at a time
         const int t = e >> 4, chn = e & 15;
         if (t < n)
-          *reinterpret_cast<uint4 *>(dv + ((size_t)(b * T + t0 + t) * H + h) * D + chn * 8) =
+          *reinterpret_cast<uint4 *>(dv + ((size_t)(tok0 + t0 + t) * H + h) * D + chn * 8) =
               *reinterpret_cast<const uint4 *>(sm + S1H + t * 256 + chn * 16);
       }
     }
@@ -858,8 +867,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int j = tid & 127, qd = tid >> 7, tb = 16 * qd;
-  const int NC = p.NC, T = p.T, H = p.H;
-  const size_t nct = (size_t)p.B * H * NC;
+  const int H = p.H;
+  const size_t nct = (size_t)total_records(p);
   const float scale = p.scale;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
@@ -887,12 +896,15 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       bulk_g2s(sm + XH, P.dX2buf + ck * 64 * D, 32768, K.barC);
       bulk_g2s(sm + YH, P.dXbuf + ck * 64 * D, 32768, K.barC);
     }
-    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
-    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * 64, n_ = min(64, T - t0_);
+    int s_, h_, cc_;
+    rec_decode(p, (long long)ck, s_, h_, cc_);
+    const SeqSpan sp_ = seq_span(p, s_, h_);
+    const long long tok0_ = sp_.tok0;
+    const int t0_ = cc_ * 64, n_ = min(64, sp_.len - t0_);
     for (int e = tid; e < 64 * 16; e += NTP) {  // K, Q (exact bf16), asynchronous
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n_;
-      const size_t off = ((size_t)(b_ * T + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
+      const size_t off = ((size_t)(tok0_ + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
       const int blk = chn >> 3, cc = (chn & 7) * 8;
       cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
       cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
@@ -906,9 +918,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   uint32_t it = 0;  // chunks done by this CTA: the parity of barrier B
   for (size_t chunk = blockIdx.x; chunk < nct && ok; chunk += gridDim.x, ++it) {
   const size_t next = chunk + gridDim.x;
-  const int bh = (int)(chunk / NC), c = (int)(chunk % NC);
-  const int b = bh / H, h = bh % H;
-  const int t0 = c * 64, n = min(64, T - t0);
+  int sq, h, c;
+  rec_decode(p, (long long)chunk, sq, h, c);
+  const SeqSpan sp = seq_span(p, sq, h);
+  const long long tok0 = sp.tok0;
+  const int t0 = c * 64, n = min(64, sp.len - t0);
   const float *recf = p.ws + chunk * kRecFloats;
   float *acc = P.acc + chunk * A8::FLOATS;
   const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
@@ -978,14 +992,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const int t = tb + i;
-    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(b * T + t0 + t) * H + h) * D + j]) : 0.f;
+    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(tok0 + t0 + t) * H + h) * D + j]) : 0.f;
   }
   if (tid < 64) {
     Gam[tid] = recf[OFF_VEC + V_GAM + tid];
     Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
     wS[tid] = recf[OFF_VEC + V_WS + tid];
     wR[tid] = recf[OFF_VEC + V_WR + tid];
-    gamv[tid] = tid < n ? p.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    gamv[tid] = tid < n ? p.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
   }
   if (!mbar_wait(K.barC, 0)) *K.flag = 1;
   {
@@ -1224,7 +1238,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const int t = tid;
       float gv = 0.f, bv = 0.f;
       if (t < n) {
-        const size_t off = (size_t)(b * T + t0 + t) * H + h;
+        const size_t off = (size_t)(tok0 + t0 + t) * H + h;
         gv = p.g[off];
         bv = p.beta[off];
       }
@@ -1404,18 +1418,21 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     __syncthreads();
     if (next < nct) fetch_states(next);  // the state images and the fp32 tiles are done with
     if (next < nct) {  // the next chunk's dO rows, mask words and gate vectors into L1
-      const int cb = (int)(next / NC), cc_ = (int)(next % NC);
-      const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * 64, n_ = min(64, T - t0_);
+      int s_, h_, cc_;
+      rec_decode(p, (long long)next, s_, h_, cc_);
+      const SeqSpan sp_ = seq_span(p, s_, h_);
+      const long long tok0_ = sp_.tok0;
+      const int t0_ = cc_ * 64, n_ = min(64, sp_.len - t0_);
       if (tid < 128) {  // 64 rows of 256 bytes
         const int t = tid >> 1;
-        if (t < n_) prefetch_l1_line(dOp + ((size_t)(b_ * T + t0_ + t) * H + h_) * D + (tid & 1) * 64);
+        if (t < n_) prefetch_l1_line(dOp + ((size_t)(tok0_ + t0_ + t) * H + h_) * D + (tid & 1) * 64);
       } else if (tid < 136) {  // 128 mask words
         prefetch_l1_line(P.mask + next * D + (tid - 128) * 16);
       } else if (tid < 148) {  // the record's 6 x 64 gate floats
         prefetch_l1_line(p.ws + next * kRecFloats + OFF_VEC + (tid - 136) * 32);
       } else if (tid < 180) {  // gamma, one line per two tokens
         const int t = 2 * (tid - 148);
-        if (t < n_) prefetch_l1_line(p.gamma + (size_t)(b_ * T + t0_ + t) * H + h_);
+        if (t < n_) prefetch_l1_line(p.gamma + (size_t)(tok0_ + t0_ + t) * H + h_);
       }
     }
     ok = phase_wait(K);
@@ -1423,7 +1440,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   if (ok) {
     if (tid < n) {
-      const size_t off = (size_t)(b * T + t0 + tid) * H + h;
+      const size_t off = (size_t)(tok0 + t0 + tid) * H + h;
       P.dg[off] = o_dg;
       P.dbeta[off] = o_dbeta;
       P.dgamma[off] = o_dgamma;
@@ -1437,7 +1454,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       for (int i = 0; i < 16; ++i) {
         const int t = tb + i;
         if (t < n) {
-          const size_t off = ((size_t)(b * T + t0 + t) * H + h) * D + j;
+          const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * D + j;
           dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
           dq[off] = __float2bfloat16_rn(scale * qv[i]);
         }
@@ -1454,12 +1471,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 
 }  // namespace
 
-size_t bwd_tc_acc_bytes(int B, int H, int NC) {
-  return sizeof(float) * (size_t)B * H * NC * A8::FLOATS;
-}
+size_t bwd_tc_acc_bytes(long long nrec) { return sizeof(float) * (size_t)nrec * A8::FLOATS; }
 
-size_t bwd_tc_extra_bytes(int B, int H, int NC) {
-  const size_t nct = (size_t)B * H * NC;
+size_t bwd_tc_extra_bytes(long long nrec) {
+  const size_t nct = (size_t)nrec;
   return nct * (4 * 64 * D * sizeof(float) + 2 * (size_t)D * D * sizeof(float) +
                 D * sizeof(unsigned long long));
 }
@@ -1484,7 +1499,7 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.dS0 = dS0;
   P.dR0 = dR0;
   P.acc = acc;
-  const size_t nct = (size_t)f.B * f.H * f.NC;
+  const size_t nct = (size_t)f.nrec;  // record slots (packed sequences: a bound)
   float *x = reinterpret_cast<float *>(extra);
   P.Ebuf = reinterpret_cast<uint8_t *>(x);
   P.E2buf = reinterpret_cast<uint8_t *>(x + nct * 64 * D);
@@ -1512,7 +1527,7 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
     RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.B * f.H, NTC, ch::SMEM, s>>>(P));
+  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.nseq * f.H, NTC, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   int dev = 0, nsm = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;

@@ -87,10 +87,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
   float *red = gmv + C;          // [6*C] per-row sums of this slice
 
   const int bh = blockIdx.x;
-  const int b = bh / p.f.H, h = bh % p.f.H;
+  const int H = p.f.H, h = bh % H;
+  const SeqSpan sp = seq_span(p.f, bh / H, h);  // this (sequence, head)'s tokens and records
+  const long long tok0 = sp.tok0;
+  const int NC = sp.nc, T = sp.len;
   const int j0 = blockIdx.y * kBDVS;
   const int tid = threadIdx.x;
-  const int NC = p.f.NC, T = p.f.T, H = p.f.H;
   const InT *q = (const InT *)p.f.q;
   const InT *k = (const InT *)p.f.k;
   const InT *v = (const InT *)p.f.v;
@@ -115,7 +117,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
   for (int c = NC - 1; c >= 0; --c) {
     const int t0 = c * C;
     const int n = min(C, T - t0);
-    const size_t chunk = (size_t)bh * NC + c;
+    const size_t chunk = (size_t)(sp.rbase + c);
     const float *rec = p.f.ws + chunk * kRecFloats;
     float *acc = p.acc + chunk * L::FLOATS;
     __syncthreads();
@@ -123,7 +125,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       const int t = e / DK, d = e % DK;
       float kv = 0.f, qv = 0.f;
       if (t < n) {
-        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+        const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * DK + d;
         kv = to_f32(k[off]);
         qv = p.f.scale * to_f32(q[off]);
       }
@@ -134,7 +136,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       const int t = e / kBDVS, jj = e % kBDVS;
       float vv = 0.f, dd = 0.f;
       if (t < n) {
-        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DV + j0 + jj;
+        const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * DV + j0 + jj;
         vv = to_f32(v[off]);
         dd = to_f32(dO[off]);
       }
@@ -151,7 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       vec[e] = rec[OFF_VEC + e];
       red[e] = 0.f;
     }
-    if (tid < C) gmv[tid] = tid < n ? p.f.gamma[(size_t)(b * T + t0 + tid) * H + h] : 0.f;
+    if (tid < C) gmv[tid] = tid < n ? p.f.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
     __syncthreads();
     const float *Gam = vec + V_GAM, *Gprev = vec + V_GPREV, *wS = vec + V_WS, *wR = vec + V_WR;
     const float GamC = vec[V_GAMC];
@@ -423,7 +425,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     }
     for (int e = tid; e < C * kBDVS; e += kThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
-      if (t < n) dv[((size_t)(b * T + t0 + t) * H + h) * DV + j0 + jj] = from_f32<InT>(T3[t * LDV + jj]);
+      if (t < n) dv[((size_t)(tok0 + t0 + t) * H + h) * DV + j0 + jj] = from_f32<InT>(T3[t * LDV + jj]);
     }
     __syncthreads();
     for (int e = tid; e < 5 * C + 1; e += kThreads) atomicAdd(&acc[L::VEC + e], red[e]);
@@ -467,12 +469,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   float *dbet = dcprev + C;
   float *dgam = dbet + C;
 
-  const int chunk = blockIdx.x;
-  const int NC = p.f.NC, T = p.f.T, H = p.f.H;
-  const int bh = chunk / NC, c = chunk % NC;
-  const int b = bh / H, h = bh % H;
+  const long long chunk = blockIdx.x;
+  if (chunk >= total_records(p.f)) return;  // (packed sequences: the grid is a bound)
+  const int H = p.f.H;
+  int sq, h, c;
+  rec_decode(p.f, chunk, sq, h, c);
+  const SeqSpan sp = seq_span(p.f, sq, h);
+  const long long tok0 = sp.tok0;
   const int t0 = c * C;
-  const int n = min(C, T - t0);
+  const int n = min(C, sp.len - t0);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const InT *q = (const InT *)p.f.q;
   const InT *k = (const InT *)p.f.k;
@@ -482,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     const int t = e / DK, d = e % DK;
     float kv = 0.f, qv = 0.f;
     if (t < n) {
-      const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+      const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * DK + d;
       kv = to_f32(k[off]);
       qv = p.f.scale * to_f32(q[off]);
     }
@@ -493,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     const int t = tid;
     float gv = 0.f, bv = 0.f, mv = 0.f;
     if (t < n) {
-      const size_t off = (size_t)(b * T + t0 + t) * H + h;
+      const size_t off = (size_t)(tok0 + t0 + t) * H + h;
       gv = p.f.g[off];
       bv = p.f.beta[off];
       mv = p.f.gamma[off];
@@ -651,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     for (int i = 0; i < MM::RPT; ++i) {
       const int t = MM::row(i), d = MM::col();
       if (t < n) {
-        const size_t off = ((size_t)(b * T + t0 + t) * H + h) * DK + d;
+        const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * DK + d;
         dk[off] = from_f32<InT>(acc[L::DKo + t * DK + d] + a1[i] + a2[i]);
         dq[off] = from_f32<InT>(p.f.scale * (acc[L::DQo + t * DK + d] + a3[i]));
       }
@@ -681,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   }
   __syncthreads();
   if (tid < n) {
-    const size_t off = (size_t)(b * T + t0 + tid) * H + h;
+    const size_t off = (size_t)(tok0 + t0 + tid) * H + h;
     p.dg[off] = gg[tid];
     p.dbeta[off] = dbet[tid];
     p.dgamma[off] = dgam[tid];
@@ -708,16 +713,16 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
   if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)finish_smem<DK>())) != cudaSuccess)
     return e;
-  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.B * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
+  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.nseq * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  RDN_LAUNCH("bwd_finish", s, fin<<<p.f.B * p.f.H * p.f.NC, kThreads, finish_smem<DK>(), s>>>(p));
+  RDN_LAUNCH("bwd_finish", s, fin<<<(unsigned)p.f.nrec, kThreads, finish_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct BwdLayout {
-  size_t prep, acc, states, o, tc, tied, total;
+  size_t prep, acc, states, o, tc, tied, seq, total;
 };
 
 // RDN with bf16 inputs and d = 128 takes the tensor-core backward (RLA, whose
@@ -735,23 +740,24 @@ bool reuse_fwd_records(const rdn_fwd_args &f) { return f.workspace && f.S_chunks
 BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const rdn_fwd_args &f = a.fwd;
   const bool tc = use_tc_bwd(f, variant);
-  const size_t nct = (size_t)f.B * f.H * ((f.T + C - 1) / C);
+  const long long nrec = call_records(f);  // record slots
   const size_t accf = f.Dk == 128 ? Acc<128>::FLOATS : Acc<64>::FLOATS;
   BwdLayout l;
   // the forward's records are read from its workspace when it is passed
-  l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nct * kRecFloats);
-  l.acc = tc ? align256(bwd_tc_acc_bytes(f.B, f.H, (f.T + C - 1) / C))
-            : align256(sizeof(float) * nct * accf);
+  l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nrec * kRecFloats);
+  l.acc = tc ? align256(bwd_tc_acc_bytes(nrec)) : align256(sizeof(float) * nrec * accf);
   const bool need_states = f.S_chunks == nullptr;
-  l.states = need_states ? align256(sizeof(float) * nct * f.Dk * f.Dv) : 0;  // each of S, R
+  l.states = need_states ? align256(sizeof(float) * nrec * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
-  l.tc = tc ? align256(bwd_tc_extra_bytes(f.B, f.H, (f.T + C - 1) / C)) : 0;
+  l.tc = tc ? align256(bwd_tc_extra_bytes(nrec)) : 0;
+  l.seq = seq_table_bytes(f);
   // tied gates without a dgamma buffer: the gamma part is made here, then added
   l.tied = (f.flags & RDN_FLAG_TIED_GAMMA) && !a.dgamma
                ? align256(sizeof(float) * (size_t)f.B * f.T * f.H)
                : 0;
-  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.tied + 256;  // + device status word
+  // + the packed-sequence table and the device status word
+  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.tied + l.seq + 256;
   return l;
 }
 
@@ -789,7 +795,7 @@ cudaError_t launch_bwd(const rdn_bwd_args &a0, int variant, cudaStream_t s) {
 
 static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStream_t s) {
   const rdn_fwd_args &f = a.fwd;
-  const size_t sbytes = sizeof(float) * (size_t)f.B * f.H * f.Dk * f.Dv;
+  const size_t sbytes = sizeof(float) * (size_t)call_seqs(f) * f.H * f.Dk * f.Dv;
   if (f.T == 0) {  // no tokens: the initial-state gradients are the upstream ones
     cudaError_t e = cudaSuccess;
     if (a.dS0) e = a.dST ? cudaMemcpyAsync(a.dS0, a.dST, sbytes, cudaMemcpyDeviceToDevice, s)
@@ -806,8 +812,14 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   const bool reuse = reuse_fwd_records(f);
   p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
   p.f.err = (int *)(ws + l.total - 256);
+  if (f.cu_seqlens) {  // this call's own copy of the packed-sequence table
+    long long *seq = (long long *)(ws + l.total - 256 - l.seq);
+    cudaError_t e = launch_seq_table(f, seq, s);
+    if (e != cudaSuccess) return e;
+    p.f.seq = seq;
+  }
   if (reuse && (f.flags & RDN_FLAG_SAVE_FOR_BWD)) {  // E, E2 and the mask kept by the forward
-    const SavedLayout sl = saved_layout((size_t)f.B * f.H * ((f.T + C - 1) / C), f.Dv);
+    const SavedLayout sl = saved_layout((size_t)p.f.nrec, f.Dv);
     p.f.sv_E = (uint8_t *)f.workspace + sl.e;
     p.f.sv_E2 = (uint8_t *)f.workspace + sl.e2;
     p.f.sv_mask = (unsigned long long *)((char *)f.workspace + sl.mask);

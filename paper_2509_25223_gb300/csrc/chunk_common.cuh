@@ -118,9 +118,64 @@ struct FwdParams {
   // [chunk][j] (bit t = |x| <= c)
   uint8_t *sv_E, *sv_E2;
   unsigned long long *sv_mask;
+  // Packed variable-length sequences (rdn_fwd_args.cu_seqlens), or NULL for B
+  // sequences of T tokens each: for s = 0 .. nseq, {first token, first chunk}
+  // of sequence s (entry nseq closes the list: {T, total chunks}).
+  const long long *seq;
+  int nseq;        // sequences: B, or the number of packed sequences
+  long long nrec;  // record slots: B * H * NC, or a bound on H * (total chunks)
 };
 
-// Where the forward keeps those intermediates: after the B*H*NC records.
+// Where sequence s's tokens and (s, h)'s chunk records are.  Token t of the
+// sequence is row (tok0 + t) * H + h of the [tokens][H] inputs; chunk c of
+// (s, h) is record rbase + c (also the index of its chunk-start states and
+// saved intermediates).  With packed sequences the records of sequence s
+// start at (its first chunk) * H, heads one after the other.
+struct SeqSpan {
+  long long tok0, rbase;
+  int len, nc;
+};
+__host__ __device__ __forceinline__ SeqSpan seq_span(const FwdParams &p, int s, int h) {
+  SeqSpan q;
+  if (p.seq) {
+    q.tok0 = p.seq[2 * s];
+    q.len = (int)(p.seq[2 * s + 2] - q.tok0);
+    q.nc = (q.len + C - 1) / C;
+    q.rbase = p.seq[2 * s + 1] * p.H + (long long)h * q.nc;
+  } else {
+    q.tok0 = (long long)s * p.T;
+    q.len = p.T;
+    q.nc = p.NC;
+    q.rbase = ((long long)s * p.H + h) * p.NC;
+  }
+  return q;
+}
+// chunk records in use (at most nseq * H * NC slots)
+__device__ __forceinline__ long long total_records(const FwdParams &p) {
+  return p.seq ? p.seq[2 * p.nseq + 1] * p.H : (long long)p.nseq * p.H * p.NC;
+}
+// record r -> (sequence s, head h, chunk c); r < total_records(p)
+__device__ __forceinline__ void rec_decode(const FwdParams &p, long long r, int &s, int &h, int &c) {
+  if (!p.seq) {
+    const long long bh = r / p.NC;
+    c = (int)(r - bh * p.NC);
+    s = (int)(bh / p.H);
+    h = (int)(bh - (long long)s * p.H);
+    return;
+  }
+  int lo = 0, hi = p.nseq - 1;  // the last sequence whose records start at or before r
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.seq[2 * mid + 1] * p.H <= r) lo = mid; else hi = mid - 1;
+  }
+  s = lo;
+  const int nc = (int)((p.seq[2 * s + 2] - p.seq[2 * s] + C - 1) / C);
+  const long long off = r - p.seq[2 * s + 1] * p.H;
+  h = (int)(off / nc);
+  c = (int)(off - (long long)h * nc);
+}
+
+// Where the forward keeps those intermediates: after the nrec record slots.
 struct SavedLayout {
   size_t e, e2, mask, bytes;  // byte offsets from the workspace base; region size
 };
@@ -148,6 +203,9 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.err = nullptr;
   p.sv_E = p.sv_E2 = nullptr;
   p.sv_mask = nullptr;
+  p.seq = nullptr;  // set by the launcher once the table is in its workspace
+  p.nseq = call_seqs(a);
+  p.nrec = call_records(a);
   return p;
 }
 
@@ -161,8 +219,8 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
 
 // Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
 cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s);
-size_t bwd_tc_extra_bytes(int B, int H, int NC);
-size_t bwd_tc_acc_bytes(int B, int H, int NC);
+size_t bwd_tc_extra_bytes(long long nrec);  // per record slot
+size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,

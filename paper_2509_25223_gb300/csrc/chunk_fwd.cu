@@ -65,11 +65,13 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   float *gg = gam + C;            // [C]
   float *Wsc = gg + C;            // [2][3*256] scratch of the blocked inverse
 
-  const int chunk = blockIdx.x;
-  const int bh = chunk / p.NC, c = chunk % p.NC;
-  const int b = bh / p.H, h = bh % p.H;
+  const long long chunk = blockIdx.x;
+  if (chunk >= total_records(p)) return;  // (packed sequences: the grid covers the bound)
+  int sq, h, c;
+  rec_decode(p, chunk, sq, h, c);
+  const SeqSpan sp = seq_span(p, sq, h);
   const int t0 = c * C;
-  const int n = min(C, p.T - t0);
+  const int n = min(C, sp.len - t0);
   const int tid = threadIdx.x;
   const InT *q = (const InT *)p.q;
   const InT *k = (const InT *)p.k;
@@ -78,7 +80,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
     const int t = e / DK, d = e % DK;
     float kv = 0.f, qv = 0.f;
     if (t < n) {
-      const size_t off = ((size_t)(b * p.T + t0 + t) * p.H + h) * DK + d;
+      const size_t off = ((size_t)(sp.tok0 + t0 + t) * p.H + h) * DK + d;
       kv = to_f32(k[off]);
       qv = p.scale * to_f32(q[off]);
     }
@@ -89,7 +91,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
     const int t = tid;
     float gv = 0.f, bv = 0.f, mv = 0.f;
     if (t < n) {
-      const size_t off = (size_t)(b * p.T + t0 + t) * p.H + h;
+      const size_t off = (size_t)(sp.tok0 + t0 + t) * p.H + h;
       gv = p.g[off];
       bv = p.beta[off];
       mv = p.gamma[off];
@@ -210,7 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
   float *vec = Ws + C * kDVS;     // [6*C]
 
   const int bh = blockIdx.x;
-  const int b = bh / p.H, h = bh % p.H;
+  const int h = bh % p.H;
+  const SeqSpan sp = seq_span(p, bh / p.H, h);
   const int j0 = blockIdx.y * kDVS;
   const int tid = threadIdx.x;
   const InT *q = (const InT *)p.q;
@@ -226,14 +229,14 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     Rs[e] = p.R0 ? p.R0[sbase + (size_t)i * DV + j0 + jj] : 0.f;
   }
 
-  for (int c = 0; c < p.NC; ++c) {
+  for (int c = 0; c < sp.nc; ++c) {
     const int t0 = c * C;
-    const int n = min(C, p.T - t0);
-    const float *rec = p.ws + ((size_t)bh * p.NC + c) * kRecFloats;
+    const int n = min(C, sp.len - t0);
+    const float *rec = p.ws + (size_t)(sp.rbase + c) * kRecFloats;
     __syncthreads();  // previous chunk done with every buffer
     if (p.S_chunks) {
-      float *sc = p.S_chunks + ((size_t)bh * p.NC + c) * DK * DV;
-      float *rc = p.R_chunks + ((size_t)bh * p.NC + c) * DK * DV;
+      float *sc = p.S_chunks + (size_t)(sp.rbase + c) * DK * DV;
+      float *rc = p.R_chunks + (size_t)(sp.rbase + c) * DK * DV;
       for (int e = tid; e < DK * kDVS; e += kThreads) {
         const int i = e / kDVS, jj = e % kDVS;
         sc[(size_t)i * DV + j0 + jj] = Ss[e];
@@ -244,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       const int t = e / DK, d = e % DK;
       float kv = 0.f, qv = 0.f;
       if (t < n) {
-        const size_t off = ((size_t)(b * p.T + t0 + t) * p.H + h) * DK + d;
+        const size_t off = ((size_t)(sp.tok0 + t0 + t) * p.H + h) * DK + d;
         kv = to_f32(k[off]);
         qv = p.scale * to_f32(q[off]);
       }
@@ -253,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     }
     for (int e = tid; e < C * kDVS; e += kThreads) {
       const int t = e / kDVS, jj = e % kDVS;
-      Vs[e] = t < n ? to_f32(v[((size_t)(b * p.T + t0 + t) * p.H + h) * DV + j0 + jj]) : 0.f;
+      Vs[e] = t < n ? to_f32(v[((size_t)(sp.tok0 + t0 + t) * p.H + h) * DV + j0 + jj]) : 0.f;
     }
     for (int e = tid; e < 6 * C; e += kThreads) vec[e] = rec[OFF_VEC + e];
     __syncthreads();
@@ -357,9 +360,9 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
         if (t < n) {
-          const float gm = p.gamma[(size_t)(b * p.T + t0 + t) * p.H + h];
+          const float gm = p.gamma[(size_t)(sp.tok0 + t0 + t) * p.H + h];
           const float oa = Gam[t] * QS[t * kDVS + col] + a1[i];
-          o[((size_t)(b * p.T + t0 + t) * p.H + h) * DV + j0 + col] =
+          o[((size_t)(sp.tok0 + t0 + t) * p.H + h) * DV + j0 + col] =
               from_f32<InT>(Ob[t * kDVS + col] + gm * oa);
         }
       }
@@ -412,12 +415,12 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
     if (tc_prep && img) {
       if ((e = launch_prep_tc(p, s)) != cudaSuccess) return e;
     } else {
-      RDN_LAUNCH("chunk_prep", s, prep<<<p.B * p.H * p.NC, kThreads, prep_smem<DK>(), s>>>(p));
+      RDN_LAUNCH("chunk_prep", s, prep<<<(unsigned)p.nrec, kThreads, prep_smem<DK>(), s>>>(p));
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
   }
   if (do_scan)
-    RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.B * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p));
+    RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.nseq * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 
@@ -460,20 +463,85 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
               : launch_t<64, false, float>(p, s, true, false, img);
 }
 
+// Block-wide inclusive scan of one value per thread (blockDim.x = 1024).
+template <typename Op>
+__device__ long long block_incl_scan(long long x, Op op, long long *wsum) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const long long y = __shfl_up_sync(0xffffffffu, x, d);
+    if (lane >= d) x = op(x, y);
+  }
+  if (lane == 31) wsum[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    long long w = wsum[lane];
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, w, d);
+      if (lane >= d) w = op(w, y);
+    }
+    wsum[lane] = w;
+  }
+  __syncthreads();
+  if (wid > 0) x = op(x, wsum[wid - 1]);
+  __syncthreads();  // (wsum is reused by the next call)
+  return x;
+}
+
+// The packed-sequence table FwdParams::seq from cu_seqlens[0 .. N]: first
+// tokens are the running maximum of the entries clamped into [0, T] (with
+// entry 0 read as 0 and entry N as T, so the table always covers [0, T) in
+// order), first chunks the exclusive prefix sum of ceil(len_s / 64).  One CTA.
+__global__ void __launch_bounds__(1024) seq_table_kernel(const int *__restrict__ cu, int N, int T,
+                                                         long long *__restrict__ seq) {
+  __shared__ long long wsum[32];
+  __shared__ long long carry;
+  const int tid = threadIdx.x;
+  if (tid == 0) carry = 0;
+  __syncthreads();
+  auto mx = [](long long a, long long b) { return a > b ? a : b; };
+  auto add = [](long long a, long long b) { return a + b; };
+  for (int base = 0; base <= N; base += 1024) {
+    const int s = base + tid;
+    long long x = 0;
+    if (s <= N) x = s == 0 ? 0 : s == N ? T : min(max(cu[s], 0), T);
+    x = mx(block_incl_scan(x, mx, wsum), carry);
+    if (s <= N) seq[2 * s] = x;
+    if (tid == 1023) carry = x;  // (padding reads 0 and leaves the maximum alone)
+    __syncthreads();
+  }
+  if (tid == 0) carry = 0;
+  __syncthreads();  // (also orders the token offsets before they are read back)
+  for (int base = 0; base <= N; base += 1024) {
+    const int s = base + tid;
+    const long long nc = s < N ? (seq[2 * s + 2] - seq[2 * s] + C - 1) / C : 0;
+    const long long incl = block_incl_scan(nc, add, wsum) + carry;
+    if (s <= N) seq[2 * s + 1] = incl - nc;  // entry N: the total
+    if (tid == 1023) carry = incl;
+    __syncthreads();
+  }
+}
+
+cudaError_t launch_seq_table(const rdn_fwd_args &a, long long *seq, cudaStream_t s) {
+  RDN_LAUNCH("seq_table", s, seq_table_kernel<<<1, 1024, 0, s>>>(a.cu_seqlens, a.num_seqs, a.T, seq));
+  return cudaGetLastError();
+}
+
 FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   FwdPlan pl;
   pl.NC = (a.T + C - 1) / C;
   pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
-  const size_t nct = (size_t)a.B * a.H * pl.NC;
-  // per-chunk records, the saved intermediates if asked for, then a 256-byte
-  // device status word
-  pl.total_bytes = pl.prep_bytes * nct + 256;
-  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) pl.total_bytes += saved_layout(nct, a.Dv).bytes;
+  const size_t nrec = (size_t)call_records(a);
+  // per-chunk records, the saved intermediates if asked for, the packed-
+  // sequence table, then a 256-byte device status word
+  pl.total_bytes = pl.prep_bytes * nrec + seq_table_bytes(a) + 256;
+  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
   return pl;
 }
 
 cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
-  const size_t sbytes = sizeof(float) * (size_t)a.B * a.H * a.Dk * a.Dv;
+  const size_t sbytes = sizeof(float) * (size_t)call_seqs(a) * a.H * a.Dk * a.Dv;
   if (a.T == 0) {  // no tokens: the final states are the initial ones
     cudaError_t e = cudaSuccess;
     if (a.ST) e = a.S0 ? cudaMemcpyAsync(a.ST, a.S0, sbytes, cudaMemcpyDeviceToDevice, s)
@@ -485,9 +553,16 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   }
   FwdParams p = make_fwd_params(a);
   p.ws = (float *)a.workspace;
-  p.err = (int *)((char *)a.workspace + plan_fwd(a, variant).total_bytes - 256);
+  const size_t total = plan_fwd(a, variant).total_bytes;
+  p.err = (int *)((char *)a.workspace + total - 256);
+  if (a.cu_seqlens) {
+    long long *seq = (long long *)((char *)a.workspace + total - 256 - seq_table_bytes(a));
+    const cudaError_t e = launch_seq_table(a, seq, s);
+    if (e != cudaSuccess) return e;
+    p.seq = seq;
+  }
   if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) {
-    const SavedLayout l = saved_layout((size_t)a.B * a.H * p.NC, a.Dv);
+    const SavedLayout l = saved_layout((size_t)p.nrec, a.Dv);
     p.sv_E = (uint8_t *)a.workspace + l.e;
     p.sv_E2 = (uint8_t *)a.workspace + l.e2;
     p.sv_mask = (unsigned long long *)((char *)a.workspace + l.mask);

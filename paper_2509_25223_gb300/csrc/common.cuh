@@ -52,6 +52,22 @@ namespace rdn {
 cudaError_t launch_decode(const rdn_decode_args &a, cudaStream_t s);
 cudaError_t launch_prologue(const rdn_prologue_args &a, bool bwd, cudaStream_t s);
 
+// Sequences and record slots of a call: B sequences of T tokens with B * H *
+// ceil(T/64) records, or num_seqs packed sequences whose sum over s of
+// ceil(len_s/64) <= num_seqs + ceil(T/64) chunks bounds the records per head.
+inline int call_seqs(const rdn_fwd_args &a) { return a.cu_seqlens ? a.num_seqs : a.B; }
+inline long long call_records(const rdn_fwd_args &a) {
+  const long long nc = (a.T + kChunk - 1) / kChunk;
+  return a.cu_seqlens ? (long long)a.H * (a.num_seqs + nc) : (long long)a.B * a.H * nc;
+}
+// bytes of the device sequence table (FwdParams::seq) in a workspace
+inline size_t seq_table_bytes(const rdn_fwd_args &a) {
+  return a.cu_seqlens ? ((sizeof(long long) * 2 * ((size_t)a.num_seqs + 1) + 255) & ~(size_t)255) : 0;
+}
+// Fill seq (seq_table_bytes) from the caller's cu_seqlens, clamping it into a
+// valid table; one small kernel on s.
+cudaError_t launch_seq_table(const rdn_fwd_args &a, long long *seq, cudaStream_t s);
+
 struct FwdPlan {
   int NC;                // chunks per sequence
   size_t prep_bytes;     // per-chunk precomputed matrices

@@ -144,8 +144,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const int j = tid & 127;       // value column == TMEM lane
   const int g16 = (warp >> 2) * 16;  // this thread's token (and state) columns start
   const int bh = blockIdx.x;
-  const int b = bh / p.H, h = bh % p.H;
-  const int T = p.T, H = p.H, NC = p.NC;
+  const int h = bh % p.H;
+  const SeqSpan sp = seq_span(p, bh / p.H, h);  // this (sequence, head)'s tokens and records
+  const long long tok0 = sp.tok0;
+  const int T = sp.len, H = p.H, NC = sp.nc;
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q;
   const __nv_bfloat16 *k = (const __nv_bfloat16 *)p.k;
   const __nv_bfloat16 *v = (const __nv_bfloat16 *)p.v;
@@ -168,14 +170,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   uint32_t phase = 0, phA = 0, phB = 0;  // phA/phB: tracked by thread 0 only
   auto rec_of = [&](int c) {
-    return reinterpret_cast<const uint8_t *>(p.ws + ((size_t)bh * NC + c) * kRecFloats);
+    return reinterpret_cast<const uint8_t *>(p.ws + (size_t)(sp.rbase + c) * kRecFloats);
   };
   // thread 0: start the bulk copy of a chunk-matrix image into a slot
   auto load_slot = [&](uint8_t *dst, uint64_t *b, const uint8_t *src, uint32_t bytes) {
     mbar_expect_tx(b, bytes);
     bulk_g2s(dst, src, bytes, b);
   };
-  if (tid == 0) {
+  if (tid == 0 && NC > 0) {  // (a packed sequence may be empty)
     if (RDNV) load_slot(sm + SM_SLOTA, barA, rec_of(0) + IMG_TB, 16384);
     load_slot(sm + SM_SLOTB, barB, rec_of(0) + IMG_APMQ, 32768);
   }
@@ -186,7 +188,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     for (int e = tid; e < 64 * 16; e += kTcThreads) {
       const int t = e >> 4, ch = e & 15;
       const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+      const size_t off = ((size_t)(tok0 + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
       cp_async16(sm + SM_V + (ch >> 3) * 8192 + sw128(t, (ch & 7) * 8), v + off, vld);
     }
   };
@@ -195,7 +197,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     for (int e = tid; e < 64 * 16; e += kTcThreads) {
       const int t = e >> 4, ch = e & 15;
       const bool vld = t < n;
-      const size_t off = ((size_t)(b * T + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
+      const size_t off = ((size_t)(tok0 + t0 + (vld ? t : 0)) * H + h) * D + ch * 8;
       const int blk = ch >> 3, cc = (ch & 7) * 8;
       cp_async16(sm + SM_KQ + blk * 16384 + sw128(t, cc), k + off, vld);
       cp_async16(sm + SM_KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
@@ -206,8 +208,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
         sm + SM_V + (j >> 6) * 8192 + sw128(t, j & 63)));
   };
-  fetch_v(0);
-  fetch_kq(0);
+  if (NC > 0) {
+    fetch_v(0);
+    fetch_kq(0);
+  }
 
   // initial states -> TMEM (fp32) and bf16 A operands
   for (int c0 = g16; c0 < D; c0 += 64) {
@@ -221,11 +225,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     tmem_st16(tm + lane + T_R + c0, r);
     st_row16(sm + SM_SA, 16384, j, c0, s);
     st_row16(sm + SM_RA, 16384, j, c0, r);
-    if (p.S_chunks) {  // the first chunk's start states, for the backward
+    if (p.S_chunks && NC > 0) {  // the first chunk's start states, for the backward
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        p.S_chunks[(size_t)bh * NC * D * D + (size_t)(c0 + i) * D + j] = s[i];
-        p.R_chunks[(size_t)bh * NC * D * D + (size_t)(c0 + i) * D + j] = r[i];
+        p.S_chunks[(size_t)sp.rbase * D * D + (size_t)(c0 + i) * D + j] = s[i];
+        p.R_chunks[(size_t)sp.rbase * D * D + (size_t)(c0 + i) * D + j] = r[i];
       }
     }
   }
@@ -263,10 +267,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (tid < 384) {
       const int rr = tid >> 1, t = rr & 63, w = rr >> 6;
       const __nv_bfloat16 *src = w == 0 ? v : (w == 1 ? k : q);
-      if (t < n_) prefetch_l2_line(src + ((size_t)(b * T + t0_ + t) * H + h) * D + (tid & 1) * 64);
+      if (t < n_) prefetch_l2_line(src + ((size_t)(tok0 + t0_ + t) * H + h) * D + (tid & 1) * 64);
     } else if (tid < 416) {
       const int t = 2 * (tid - 384);
-      if (t < n_) prefetch_l2_line(p.gamma + (size_t)(b * T + t0_ + t) * H + h);
+      if (t < n_) prefetch_l2_line(p.gamma + (size_t)(tok0 + t0_ + t) * H + h);
     }
   };
 
@@ -291,7 +295,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     float gm, gp, ws, wr, g, gc;
   };
   auto fetch_pre = [&](int c) {
-    const float *rc = p.ws + ((size_t)bh * NC + c) * kRecFloats;
+    const float *rc = p.ws + (size_t)(sp.rbase + c) * kRecFloats;
     const int t0_ = c * 64, n_ = min(64, T - t0_);
     Pre x;
     x.gm = x.gp = x.ws = x.wr = x.g = 0.f;
@@ -300,12 +304,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       x.gp = rc[OFF_VEC + V_GPREV + tid];
       x.ws = rc[OFF_VEC + V_WS + tid];
       x.wr = rc[OFF_VEC + V_WR + tid];
-      x.g = tid < n_ ? p.gamma[(size_t)(b * T + t0_ + tid) * H + h] : 0.f;
+      x.g = tid < n_ ? p.gamma[(size_t)(tok0 + t0_ + tid) * H + h] : 0.f;
     }
     x.gc = rc[OFF_VEC + V_GAMC];
     return x;
   };
-  Pre pre = fetch_pre(0);
+  Pre pre{};
+  if (NC > 0) pre = fetch_pre(0);
 
   float rres[16];  // clipped residual r[t] of column j, t in [g16, g16 + 16)
   bool alive = true;
@@ -318,9 +323,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (a) chunk inputs -> shared memory (the chunk-start states for the
     // backward were stored by the previous chunk's updates)
-    float *sc_next = (p.S_chunks && c + 1 < NC) ? p.S_chunks + ((size_t)bh * NC + c + 1) * D * D
+    float *sc_next = (p.S_chunks && c + 1 < NC) ? p.S_chunks + (size_t)(sp.rbase + c + 1) * D * D
                                                 : nullptr;
-    float *rc_next = sc_next ? p.R_chunks + ((size_t)bh * NC + c + 1) * D * D : nullptr;
+    float *rc_next = sc_next ? p.R_chunks + (size_t)(sp.rbase + c + 1) * D * D : nullptr;
     if (tid < 64) {
       Gam[tid] = pre.gm;
       Gprev[tid] = pre.gp;
@@ -392,7 +397,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
     // ---- (d) E -> EA, wS*E -> WA, Gprev KS -> D1[0,64);  MMA3: D1 += E^T [Ap;Mq]^T,
     // MMA4: S += (wS E)^T K
-    const size_t ci = (size_t)bh * NC + c;  // chunk index of the saved intermediates
+    const size_t ci = (size_t)(sp.rbase + c);  // chunk index of the saved intermediates
     {
       const int c0 = g16;
       float e[16], w[16];
@@ -551,7 +556,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     for (int e = tid; e < 64 * 16; e += kTcThreads) {
       const int t = e >> 4, ch = e & 15;
       if (t < n)
-        *reinterpret_cast<uint4 *>(o + ((size_t)(b * T + t0 + t) * H + h) * D + ch * 8) =
+        *reinterpret_cast<uint4 *>(o + ((size_t)(tok0 + t0 + t) * H + h) * D + ch * 8) =
             *reinterpret_cast<const uint4 *>(sm + SM_W + t * 256 + ch * 16);
     }
   }
@@ -587,7 +592,7 @@ cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kTcSmem);
   if (e != cudaSuccess) return e;
-  RDN_LAUNCH("fwd_tc_scan", s, kern<<<p.B * p.H, kTcThreads, kTcSmem, s>>>(p));
+  RDN_LAUNCH("fwd_tc_scan", s, kern<<<p.nseq * p.H, kTcThreads, kTcSmem, s>>>(p));
   return cudaGetLastError();
 }
 

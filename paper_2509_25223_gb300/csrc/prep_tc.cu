@@ -167,8 +167,8 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
   volatile int *flag = reinterpret_cast<volatile int *>(sm + CTL + 8);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int NC = p.NC, T = p.T, H = p.H;
-  const size_t nct = (size_t)p.B * H * NC;
+  const int H = p.H;
+  const size_t nct = (size_t)total_records(p);
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
   constexpr float kLog2e = 1.4426950408889634f;
 
@@ -182,12 +182,15 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
   // its gates into registers (threads 0..63); fetched while the previous chunk
   // of this CTA finishes
   auto fetch_kq = [&](size_t ck) {
-    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
-    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * C, n_ = min(C, T - t0_);
+    int s_, h_, cc_;
+    rec_decode(p, (long long)ck, s_, h_, cc_);
+    const SeqSpan sp_ = seq_span(p, s_, h_);
+    const long long tok0_ = sp_.tok0;
+    const int t0_ = cc_ * C, n_ = min(C, sp_.len - t0_);
     for (int e = tid; e < 64 * 16; e += NTH) {
       const int t = e >> 4, chn = e & 15;
       const bool vld = t < n_;
-      const size_t off = ((size_t)(b_ * T + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
+      const size_t off = ((size_t)(tok0_ + t0_ + (vld ? t : 0)) * H + h_) * D + chn * 8;
       const int blk = chn >> 3, cc = (chn & 7) * 8;
       cp_async16(sm + KQ + blk * 16384 + sw128(t, cc), k + off, vld);
       cp_async16(sm + KQ + blk * 16384 + sw128(64 + t, cc), q + off, vld);
@@ -197,11 +200,14 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
     float g, b, m;
   };
   auto fetch_gates = [&](size_t ck) {
-    const int cb = (int)(ck / NC), cc_ = (int)(ck % NC);
-    const int b_ = cb / H, h_ = cb % H, t0_ = cc_ * C, n_ = min(C, T - t0_);
+    int s_, h_, cc_;
+    rec_decode(p, (long long)ck, s_, h_, cc_);
+    const SeqSpan sp_ = seq_span(p, s_, h_);
+    const long long tok0_ = sp_.tok0;
+    const int t0_ = cc_ * C, n_ = min(C, sp_.len - t0_);
     Gates x{0.f, 0.f, 0.f};
     if (tid < C && tid < n_) {
-      const size_t off = (size_t)(b_ * T + t0_ + tid) * H + h_;
+      const size_t off = (size_t)(tok0_ + t0_ + tid) * H + h_;
       x.g = p.g[off];
       x.b = p.beta[off];
       x.m = p.gamma[off];
@@ -384,7 +390,7 @@ cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s) {
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
     return e;
-  const size_t nct = (size_t)p.B * p.H * p.NC;
+  const size_t nct = (size_t)p.nrec;  // (packed sequences: a bound; the kernel reads the count)
   const unsigned grid = (unsigned)(nct < 2 * (size_t)nsm ? nct : 2 * (size_t)nsm);  // two per SM
   RDN_LAUNCH("chunk_prep", s, prep_tc_kernel<<<grid, NTH, pp::SMEM, s>>>(p));
   return cudaGetLastError();

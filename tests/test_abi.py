@@ -101,6 +101,32 @@ def test_workspace_size_queries():
     assert m.value - n.value == nct * (2 * 64 * 128 * 4 + 128 * 8)
 
 
+def test_packed_sequence_validation_and_sizes():
+    """cu_seqlens: B must be 1, num_seqs >= 1, the table 16-byte aligned; the
+    chunk-slot count and the workspace grow by H * num_seqs records."""
+    lib = _abi.load()
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE, o=FAKE)
+    assert _status("rdn_fwd", _fwd_args(cu_seqlens=FAKE, num_seqs=3, **ok)) == 1  # B = 2
+    assert "B = 1" in lib.rdn_last_error().decode()
+    assert _status("rdn_fwd", _fwd_args(B=1, cu_seqlens=FAKE, num_seqs=0, **ok)) == 1
+    assert _status("rdn_fwd", _fwd_args(B=1, cu_seqlens=ctypes.c_void_p(0x10004), num_seqs=3,
+                                        **ok)) == 6
+    assert _status("rdn_fwd", _fwd_args(B=1, cu_seqlens=FAKE, num_seqs=3, **ok)) == 5
+    slots = ctypes.c_longlong(0)
+    a = _fwd_args(B=1, T=300, H=4)
+    assert lib.rdn_chunk_slots(ctypes.byref(a), ctypes.byref(slots)) == 0
+    assert slots.value == 4 * 5
+    p = _fwd_args(B=1, T=300, H=4, cu_seqlens=FAKE, num_seqs=7)
+    assert lib.rdn_chunk_slots(ctypes.byref(p), ctypes.byref(slots)) == 0
+    assert slots.value == 4 * (7 + 5)  # at most num_seqs + ceil(T/64) chunks per head
+    n, m = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(a), ctypes.byref(n)) == 0
+    assert lib.rdn_fwd_workspace_size(ctypes.byref(p), ctypes.byref(m)) == 0
+    rec = (n.value - 256) // (4 * 5)
+    table = 256  # 8 entries of {first token, first chunk}, rounded up to 256 bytes
+    assert m.value == 256 + rec * 4 * 12 + table
+
+
 def test_decode_validation():
     lib = _abi.load()
     a = _abi.DecodeArgs()
