@@ -26,6 +26,8 @@ import sys
 import tempfile
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
@@ -517,6 +519,60 @@ def run_ours(args):
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr
 
+    # ---- packed variable-length sequences: the same B*T tokens per head as
+    # one packed row of seeded log-uniform lengths in [64, 8192] (the last one
+    # cut to fill the row), RDN fwd+bwd exactly as the step above
+    vl = None
+    if not args.no_varlen:
+        rng = np.random.default_rng(1234)
+        lens, tot = [], 0
+        while tot < B * T:
+            L = int(np.exp(rng.uniform(np.log(64), np.log(8192))))
+            L = min(L, B * T - tot)
+            lens.append(L)
+            tot += L
+        cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
+        N = len(lens)
+        xv = {n: x[n].view(1, B * T, *x[n].shape[2:]) for n in names + ("dO",)}
+        ov = o.view(1, B * T, H, D)
+        wsfv = torch.empty(rdn.workspace_bytes("rdn_fwd", 1, B * T, H, D, save_for_bwd=True,
+                                               cu_seqlens=cu), dtype=torch.uint8, device=dev)
+        wsbv = torch.empty(rdn.workspace_bytes("rdn_bwd", 1, B * T, H, D, cu_seqlens=cu),
+                           dtype=torch.uint8, device=dev)
+        gv = {n: (t.view(1, B * T, *t.shape[2:]) if n not in ("dS0", "dR0") else
+                  torch.empty(N, H, D, D, device=dev)) for n, t in grads.items()}
+
+        def vstep(inp):
+            _, _, _, Sc_, Rc_ = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
+                                            return_chunk_states=True, out=ov, workspace=wsfv,
+                                            save_for_bwd=True, cu_seqlens=cu)
+            rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
+                        R_chunks=Rc_, workspace=wsbv, out=gv, fwd_workspace=wsfv,
+                        fwd_saved=True, cu_seqlens=cu)
+
+        vsteps = max(1, args.steps)
+        for _ in range(3):
+            vstep(xv)
+        torch.cuda.synchronize()
+        barrier(dist)
+        with rdn.LaunchTimer() as ltv:
+            e0.record(stream)
+            for _ in range(vsteps):
+                vstep(xv)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        barrier(dist)
+        tv, vval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * vsteps)
+        vl = {"workload": f"rdn_fwd_bwd_packed_bf16_N{N}_T{B * T}H{H}D{D}", "value": vval,
+              "unit": "tokens/s", "steps": vsteps, "ms_per_step": tv / vsteps,
+              "num_seqs": N, "lengths": {"min": int(min(lens)), "max": int(max(lens)),
+                                         "mean": float(np.mean(lens))},
+              "chunks_per_head": int(sum((L + C - 1) // C for L in lens)),
+              "vs_fixed_length": vval / value,
+              "kernels": {k: {"launches": n, "mean_ms": m}
+                          for k, (n, t, m) in ltv.summary().items()}}
+        del wsfv, wsbv, gv
+
     # ---- q, k prologue (SiLU + L2 norm) and its backward on the bench
     # workload's q, k: algorithmic bytes = each element read and written once
     # (the backward also reads dy), against the measured HBM peak
@@ -572,7 +628,8 @@ def run_ours(args):
                 "kernels": {k: {"launches": n, "total_ms": t, "mean_ms": m,
                                 "share": t / sum(v[1] for v in kern.values())}
                             for k, (n, t, m) in kern.items()},
-                "clocks": clk.summary(), "decode": dec, "rla": rla, "prologue": pro}
+                "clocks": clk.summary(), "decode": dec, "rla": rla, "prologue": pro,
+                "varlen": vl}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -590,6 +647,7 @@ def main(argv=None):
     ap.add_argument("--rla-steps", type=int, default=3)
     ap.add_argument("--no-rla", action="store_true")
     ap.add_argument("--no-prologue", action="store_true")
+    ap.add_argument("--no-varlen", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")

@@ -35,6 +35,10 @@ _lock = threading.Lock()
 _lib = None
 
 RLA, RDN = 0, 1
+# variant bits (rdn_oracle.c, orc_fwd_mod): residual against a_t S_{t-1} k_t;
+# ungated combine o = S_{t-1} q + R_t q; c tanh(x / c) residual; stateless
+# correction R_t = r_t k_t^T
+DECAYED, PLAIN, TANH, STATELESS = 1, 2, 4, 8
 
 
 def build(force: bool = False) -> str:
@@ -63,17 +67,19 @@ def _load():
             for name in ("orc_rla_fwd", "orc_rdn_fwd"):
                 getattr(lib, name).argtypes = fwd_sig
                 getattr(lib, name).restype = None
-            lib.orc_fwd_with_residual.argtypes = [I] + fwd_sig + [P]
-            lib.orc_fwd_with_residual.restype = None
+            lib.orc_fwd_mod.argtypes = [I, I] + fwd_sig + [P]
+            lib.orc_fwd_mod.restype = None
             bwd_sig = [I, I, I, I, I, P, P, P, P, P, P, D, D, P, P, P, P, P,
                        P, P, P, P, P, P, P, P]
             for name in ("orc_rla_bwd", "orc_rdn_bwd"):
                 getattr(lib, name).argtypes = bwd_sig
                 getattr(lib, name).restype = None
+            lib.orc_bwd_mod.argtypes = [I, I] + bwd_sig
+            lib.orc_bwd_mod.restype = None
             lib.orc_decode_step.argtypes = [I, I, I, I, I, P, P, P, P, P, P, D, D, P, P, P]
             lib.orc_decode_step.restype = None
             lib.orc_clip_margin_condition.argtypes = [I, I, I, I, I, I, P, P, P, P, P, P,
-                                                      D, D, P, P, D, I]
+                                                      D, D, P, P, D, I, I]
             lib.orc_clip_margin_condition.restype = ctypes.c_long
             lib.orc_max_threads.restype = I
             lib.orc_set_threads.argtypes = [I]
@@ -108,8 +114,9 @@ def _dims(q, v):
 
 
 def fwd(variant, q, k, v, g, beta, gamma, c=1.0, S0=None, R0=None, scale=1.0,
-        return_residual=False):
-    """Forward of RLA (variant=RLA) or RDN (variant=RDN).
+        return_residual=False, mods=0):
+    """Forward of RLA (variant=RLA) or RDN (variant=RDN), with the variant
+    bits `mods` (DECAYED | PLAIN | TANH | STATELESS, 0 = the method).
 
     Returns (o, ST, RT) as float64 arrays, plus r (the clipped residuals,
     [B,T,H,Dv]) when return_residual is set."""
@@ -123,10 +130,10 @@ def fwd(variant, q, k, v, g, beta, gamma, c=1.0, S0=None, R0=None, scale=1.0,
     args = (B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta),
             _ptr(gamma), float(c), float(scale), _ptr(S0), _ptr(R0), _ptr(o),
             _ptr(ST), _ptr(RT))
-    if return_residual:
-        r = np.zeros((B, T, H, Dv))
-        lib.orc_fwd_with_residual(int(variant), *args, _ptr(r))
-        return o, ST, RT, r
+    if return_residual or mods:
+        r = np.zeros((B, T, H, Dv)) if return_residual else None
+        lib.orc_fwd_mod(int(variant), int(mods), *args, _ptr(r))
+        return (o, ST, RT, r) if return_residual else (o, ST, RT)
     (lib.orc_rdn_fwd if variant == RDN else lib.orc_rla_fwd)(*args)
     return o, ST, RT
 
@@ -142,7 +149,7 @@ def rla_fwd(*a, **kw):
 
 
 def bwd(variant, q, k, v, g, beta, gamma, c, S0, R0, dO, dST=None, dRT=None,
-        scale=1.0):
+        scale=1.0, mods=0):
     """Back-propagation through time of the forward above.
 
     Returns a dict with dq, dk, dv, dg (w.r.t. the log-decay g), dbeta,
@@ -156,6 +163,8 @@ def bwd(variant, q, k, v, g, beta, gamma, c, S0, R0, dO, dST=None, dRT=None,
                dbeta=np.zeros((B, T, H)), dgamma=np.zeros((B, T, H)),
                dS0=np.zeros((B, H, Dk, Dv)), dR0=np.zeros((B, H, Dk, Dv)))
     fn = lib.orc_rdn_bwd if variant == RDN else lib.orc_rla_bwd
+    if mods:
+        fn = lambda *a: lib.orc_bwd_mod(int(variant), int(mods), *a)  # noqa: E731
     fn(B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta),
        _ptr(gamma), float(c), float(scale), _ptr(S0), _ptr(R0), _ptr(dO),
        _ptr(dST), _ptr(dRT), _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]),
@@ -224,7 +233,7 @@ QUANT = {"f64": 0, "f32": 1, "bf16": 2}
 
 
 def clip_margin_condition(variant, q, k, v, g, beta, gamma, c, S0=None, R0=None,
-                          scale=1.0, margin=4e-3, quant="bf16"):
+                          scale=1.0, margin=4e-3, quant="bf16", mods=0):
     """Return (v_conditioned, n_moved): v moved, in token order and in steps
     representable in `quant`, so that every |v - S_{t-1}k| of the fp64
     forward is at least `margin` away from the clip threshold c.  Makes the
@@ -237,5 +246,5 @@ def clip_margin_condition(variant, q, k, v, g, beta, gamma, c, S0=None, R0=None,
     n = lib.orc_clip_margin_condition(int(variant), B, T, H, Dk, Dv, _ptr(q), _ptr(k),
                                       _ptr(v), _ptr(g), _ptr(beta), _ptr(gamma),
                                       float(c), float(scale), _ptr(S0), _ptr(R0),
-                                      float(margin), QUANT[quant])
+                                      float(margin), QUANT[quant], int(mods))
     return v, int(n)

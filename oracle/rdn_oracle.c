@@ -33,6 +33,20 @@
  *    (the tie |x| == c passes the gradient through);
  *  - q is multiplied by `scale` (the paper uses 1, i.e. no 1/sqrt(d)).
  *
+ * The paper's variants, selected by the `mods` bits of the *_mod entry
+ * points (any combination; 0 is the method above):
+ *  - ORC_DECAYED: the residual against the decayed prediction,
+ *    r_t = Clip(v_t - a_t S_{t-1} k_t) (the gated-delta error; Section 3.2's
+ *    table and Section 3.4's discussion of which prediction to fit);
+ *  - ORC_PLAIN: the ungated combine o_t = S_{t-1} q_t + R_t q_t (the output
+ *    combination ablation, Section 4.4);
+ *  - ORC_TANH: the log-cosh residual of Appendix B, read with the threshold
+ *    as a scale, r_t = c tanh((v_t - S_{t-1} k_t) / c) (c = 1 is the
+ *    paper's tanh; c = inf is no limit, c = 0 is r = 0);
+ *  - ORC_STATELESS: the stateless correction of the residual-fitting
+ *    ablation (Section 4.4), R_t = r_t k_t^T in place of the recurrence for
+ *    R (R0 unused; RT = r_T k_T^T, or R0 when T = 0).
+ *
  * The backward is hand-written reverse-mode through the same token loop
  * (back-propagation through time), with the states re-computed from
  * checkpoints taken every ORC_CKPT tokens.  The paper has no backward; it is
@@ -54,11 +68,27 @@
 #define ORC_CKPT 64
 
 enum { ORC_RLA = 0, ORC_RDN = 1 };
+enum { ORC_DECAYED = 1, ORC_PLAIN = 2, ORC_TANH = 4, ORC_STATELESS = 8 };
 
 static double clampd(double x, double c) {
   if (x < -c) return -c;
   if (x > c) return c;
   return x;
+}
+
+/* the residual nonlinearity and its derivative */
+static double resid(double x, double c, int mods) {
+  if (!(mods & ORC_TANH)) return clampd(x, c);
+  if (isinf(c)) return x;
+  if (c == 0.0) return 0.0;
+  return c * tanh(x / c);
+}
+static double resid_grad(double x, double c, int mods) {
+  if (!(mods & ORC_TANH)) return fabs(x) <= c ? 1.0 : 0.0;
+  if (isinf(c)) return 1.0;
+  if (c == 0.0) return 0.0;
+  const double t = tanh(x / c);
+  return 1.0 - t * t;
 }
 
 int orc_max_threads(void) {
@@ -80,7 +110,7 @@ void orc_set_threads(int n) {
 /* One token of the recurrence for one (b,h).  S,R [Dk][Dv] are updated in
  * place; o[Dv] receives the output.  p, rk are scratch of length Dv.
  * Returns nothing; r (length Dv, may be NULL) receives the clipped residual. */
-static void token_step(int variant, int Dk, int Dv, const double *q,
+static void token_step(int variant, int mods, int Dk, int Dv, const double *q,
                        const double *k, const double *v, double alpha,
                        double beta, double gamma, double c, double scale,
                        double *S, double *R, double *o, double *p, double *rk,
@@ -95,16 +125,20 @@ static void token_step(int variant, int Dk, int Dv, const double *q,
       rkj += k[i] * R[i * Dv + j];
     }
     p[j] = pj;
-    o[j] = alpha * sqj; /* base prediction a_t S_{t-1} q_t */
+    /* base prediction a_t S_{t-1} q_t (ORC_PLAIN: S_{t-1} q_t) */
+    o[j] = (mods & ORC_PLAIN ? 1.0 : alpha) * sqj;
     rk[j] = rkj;
   }
   for (int j = 0; j < Dv; ++j) {
-    double rj = clampd(v[j] - p[j], c); /* Section 3.3 */
+    const double x = v[j] - (mods & ORC_DECAYED ? alpha * p[j] : p[j]);
+    double rj = resid(x, c, mods); /* Section 3.3 */
     if (r_out) r_out[j] = rj;
     /* auxiliary state update */
     for (int i = 0; i < Dk; ++i) {
       double Rij = R[i * Dv + j];
-      if (variant == ORC_RDN)
+      if (mods & ORC_STATELESS)
+        R[i * Dv + j] = k[i] * rj;
+      else if (variant == ORC_RDN)
         R[i * Dv + j] = alpha * Rij - alpha * gamma * k[i] * rk[j] + gamma * k[i] * rj;
       else
         R[i * Dv + j] = alpha * Rij + gamma * k[i] * rj;
@@ -122,11 +156,11 @@ static void token_step(int variant, int Dk, int Dv, const double *q,
   for (int j = 0; j < Dv; ++j) {
     double aq = 0.0;
     for (int i = 0; i < Dk; ++i) aq += scale * q[i] * R[i * Dv + j];
-    o[j] += gamma * aq;
+    o[j] += (mods & ORC_PLAIN ? 1.0 : gamma) * aq;
   }
 }
 
-static void fwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
+static void fwd_impl(int variant, int mods, int B, int T, int H, int Dk, int Dv,
                      const double *q, const double *k, const double *v,
                      const double *g, const double *beta, const double *gamma,
                      double c, double scale, const double *S0, const double *R0,
@@ -143,7 +177,7 @@ static void fwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
     if (R0) memcpy(R, R0 + bh * SD, sizeof(double) * SD); else memset(R, 0, sizeof(double) * SD);
     for (long t = 0; t < T; ++t) {
       const long tok = (b * T + t) * H + h; /* index into [B,T,H] */
-      token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+      token_step(variant, mods, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
                  exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R,
                  o + tok * Dv, p, rk, r_all ? r_all + tok * Dv : NULL);
     }
@@ -159,7 +193,7 @@ void orc_rla_fwd(int B, int T, int H, int Dk, int Dv, const double *q,
                  const double *beta, const double *gamma, double c,
                  double scale, const double *S0, const double *R0, double *o,
                  double *ST, double *RT) {
-  fwd_impl(ORC_RLA, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+  fwd_impl(ORC_RLA, 0, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
            o, ST, RT, NULL);
 }
 
@@ -169,19 +203,19 @@ void orc_rdn_fwd(int B, int T, int H, int Dk, int Dv, const double *q,
                  const double *beta, const double *gamma, double c,
                  double scale, const double *S0, const double *R0, double *o,
                  double *ST, double *RT) {
-  fwd_impl(ORC_RDN, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+  fwd_impl(ORC_RDN, 0, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
            o, ST, RT, NULL);
 }
 
-/* Forward that also returns the clipped residuals r [B,T,H,Dv]
- * (variant 0 = RLA, 1 = RDN).  Used by tests of the residual itself. */
-void orc_fwd_with_residual(int variant, int B, int T, int H, int Dk, int Dv,
+/* Forward with the variant bits `mods` that also returns the residuals r
+ * [B,T,H,Dv] when r is not NULL (variant 0 = RLA, 1 = RDN). */
+void orc_fwd_mod(int variant, int mods, int B, int T, int H, int Dk, int Dv,
                            const double *q, const double *k, const double *v,
                            const double *g, const double *beta,
                            const double *gamma, double c, double scale,
                            const double *S0, const double *R0, double *o,
                            double *ST, double *RT, double *r) {
-  fwd_impl(variant, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+  fwd_impl(variant, mods, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
            o, ST, RT, r);
 }
 
@@ -197,7 +231,7 @@ void orc_decode_step(int variant, int N, int H, int Dk, int Dv, const double *q,
   for (long nh = 0; nh < (long)N * H; ++nh) {
     double *p = (double *)malloc(sizeof(double) * Dv);
     double *rk = (double *)malloc(sizeof(double) * Dv);
-    token_step(variant, Dk, Dv, q + nh * Dk, k + nh * Dk, v + nh * Dv,
+    token_step(variant, 0, Dk, Dv, q + nh * Dk, k + nh * Dk, v + nh * Dv,
                exp(g[nh]), beta[nh], gamma[nh], c, scale, S + nh * SD,
                R + nh * SD, o + nh * Dv, p, rk, NULL);
     free(p); free(rk);
@@ -231,8 +265,15 @@ void orc_decode_step(int variant, int N, int H, int Dk, int Dv, const double *q,
  *            dv += b w; dk += b dS' v; dS += a dS'
  *   p = S^T k: dk += S dp;  dS += k dp^T
  *   dg = a * da.
+ * The variant bits change these steps as follows:
+ *   ORC_DECAYED    x = v - a p:  dp = -a dx (not -dx), da -= dx.p
+ *   ORC_PLAIN      output weights 1 for a and gam: no da, dgam from the
+ *                  output; dq = S_{t-1}^T dO + R_t^T dO; dS, dR' get q dO^T
+ *   ORC_TANH       dx = dr * (1 - (r/c)^2) (the derivative of c tanh(x/c))
+ *   ORC_STATELESS  R_t = k r^T:  u = dR'^T k,  dr = u,  dk += dR' r,
+ *                  dR_{t-1} = 0 (R0 does not enter)
  * ------------------------------------------------------------------------ */
-static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
+static void bwd_impl(int variant, int mods, int B, int T, int H, int Dk, int Dv,
                      const double *q, const double *k, const double *v,
                      const double *g, const double *beta, const double *gamma,
                      double c, double scale, const double *S0,
@@ -275,7 +316,7 @@ static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
       const int t0 = sgi * ORC_CKPT, t1 = t0 + ORC_CKPT < T ? t0 + ORC_CKPT : T;
       for (int t = t0; t < t1; ++t) {
         const long tok = (b * T + t) * H + h;
-        token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+        token_step(variant, mods, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
                    exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R, ob, p,
                    rk, NULL);
       }
@@ -292,7 +333,7 @@ static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
         const long tok = (b * T + t) * H + h;
         memcpy(segS + (t - t0) * SD, S, sizeof(double) * SD);
         memcpy(segR + (t - t0) * SD, R, sizeof(double) * SD);
-        token_step(variant, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
+        token_step(variant, mods, Dk, Dv, q + tok * Dk, k + tok * Dk, v + tok * Dv,
                    exp(g[tok]), beta[tok], gamma[tok], c, scale, S, R, ob, p,
                    rk, NULL);
       }
@@ -316,35 +357,41 @@ static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
             rkj += kt[i] * Rp[i * Dv + j];
           }
           p[j] = pj; rk[j] = rkj;
-          r[j] = clampd(vt[j] - pj, c);
+          r[j] = resid(vt[j] - (mods & ORC_DECAYED ? a * pj : pj), c, mods);
         }
         for (int i = 0; i < Dk; ++i)
           for (int j = 0; j < Dv; ++j) {
             const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
-            Rt[i * Dv + j] = a * Rp[i * Dv + j] + gm * kt[i] * e2;
+            Rt[i * Dv + j] = mods & ORC_STATELESS ? kt[i] * r[j]
+                                                  : a * Rp[i * Dv + j] + gm * kt[i] * e2;
           }
 
-        /* output o = a S_{t-1} q + gam R_t q (q scaled) */
+        /* output o = ws S_{t-1} q + wr R_t q (q scaled): ws = a, wr = gam,
+           or 1 and 1 for the plain combine */
+        const int plain = (mods & ORC_PLAIN) != 0;
+        const double ws = plain ? 1.0 : a, wr = plain ? 1.0 : gm;
         for (int j = 0; j < Dv; ++j) {
           double sq = 0.0, rq = 0.0;
           for (int i = 0; i < Dk; ++i) {
             sq += scale * qt[i] * Sp[i * Dv + j];
             rq += scale * qt[i] * Rt[i * Dv + j];
           }
-          da += dOt[j] * sq;
-          dgm += dOt[j] * rq;
+          if (!plain) {
+            da += dOt[j] * sq;
+            dgm += dOt[j] * rq;
+          }
         }
         for (int i = 0; i < Dk; ++i) {
           double acc = 0.0;
           for (int j = 0; j < Dv; ++j)
-            acc += (a * Sp[i * Dv + j] + gm * Rt[i * Dv + j]) * dOt[j];
+            acc += (ws * Sp[i * Dv + j] + wr * Rt[i * Dv + j]) * dOt[j];
           dqt[i] = scale * acc;
         }
-        /* dR' += gam (scale q) dO^T ; dS_{t-1} starts at a (scale q) dO^T */
+        /* dR' += wr (scale q) dO^T ; dS_{t-1} starts at ws (scale q) dO^T */
         for (int i = 0; i < Dk; ++i)
           for (int j = 0; j < Dv; ++j) {
-            dR[i * Dv + j] += gm * scale * qt[i] * dOt[j];
-            dSp[i * Dv + j] = a * scale * qt[i] * dOt[j];
+            dR[i * Dv + j] += wr * scale * qt[i] * dOt[j];
+            dSp[i * Dv + j] = ws * scale * qt[i] * dOt[j];
           }
 
         /* R step */
@@ -353,40 +400,49 @@ static void bwd_impl(int variant, int B, int T, int H, int Dk, int Dv,
           for (int i = 0; i < Dk; ++i) uj += kt[i] * dR[i * Dv + j];
           u[j] = uj;
         }
-        {
+        if (mods & ORC_STATELESS) { /* R_t = k r^T: no decay, rate or R_{t-1} */
+          for (int i = 0; i < Dk; ++i) {
+            double acc = 0.0;
+            for (int j = 0; j < Dv; ++j) acc += dR[i * Dv + j] * r[j];
+            dkt[i] += acc;
+          }
+          memset(dRp, 0, sizeof(double) * SD);
+        } else {
           double dRR = 0.0;
           for (long e = 0; e < SD; ++e) dRR += dR[e] * Rp[e];
           da += dRR;
-        }
-        for (int j = 0; j < Dv; ++j) {
-          const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
-          if (variant == ORC_RDN) da -= gm * u[j] * rk[j];
-          dgm += u[j] * e2;
-        }
-        for (int i = 0; i < Dk; ++i) {
-          double acc = 0.0, acc2 = 0.0;
           for (int j = 0; j < Dv; ++j) {
             const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
-            acc += dR[i * Dv + j] * e2;
-            acc2 += Rp[i * Dv + j] * u[j];
+            if (variant == ORC_RDN) da -= gm * u[j] * rk[j];
+            dgm += u[j] * e2;
           }
-          dkt[i] += gm * acc;
-          if (variant == ORC_RDN) dkt[i] -= a * gm * acc2;
+          for (int i = 0; i < Dk; ++i) {
+            double acc = 0.0, acc2 = 0.0;
+            for (int j = 0; j < Dv; ++j) {
+              const double e2 = variant == ORC_RDN ? r[j] - a * rk[j] : r[j];
+              acc += dR[i * Dv + j] * e2;
+              acc2 += Rp[i * Dv + j] * u[j];
+            }
+            dkt[i] += gm * acc;
+            if (variant == ORC_RDN) dkt[i] -= a * gm * acc2;
+          }
+          for (int i = 0; i < Dk; ++i)
+            for (int j = 0; j < Dv; ++j) {
+              double nv = a * dR[i * Dv + j];
+              if (variant == ORC_RDN) nv -= a * gm * kt[i] * u[j];
+              dRp[i * Dv + j] = nv;
+            }
         }
-        for (int i = 0; i < Dk; ++i)
-          for (int j = 0; j < Dv; ++j) {
-            double nv = a * dR[i * Dv + j];
-            if (variant == ORC_RDN) nv -= a * gm * kt[i] * u[j];
-            dRp[i * Dv + j] = nv;
-          }
 
-        /* clip */
+        /* clip (or tanh) of x = v - p (ORC_DECAYED: v - a p) */
         for (int j = 0; j < Dv; ++j) {
-          const double x = vt[j] - p[j];
-          const double dr = gm * u[j];
-          const double dx = fabs(x) <= c ? dr : 0.0;
+          const int dec = (mods & ORC_DECAYED) != 0;
+          const double x = vt[j] - (dec ? a * p[j] : p[j]);
+          const double dr = mods & ORC_STATELESS ? u[j] : gm * u[j];
+          const double dx = dr * resid_grad(x, c, mods);
           dvt[j] += dx;
-          dp[j] = -dx;
+          dp[j] = dec ? -a * dx : -dx;
+          if (dec) da -= dx * p[j];
         }
 
         /* S step */
@@ -446,7 +502,7 @@ void orc_rdn_bwd(int B, int T, int H, int Dk, int Dv, const double *q,
                  const double *dO, const double *dST, const double *dRT,
                  double *dq, double *dk, double *dv, double *dg, double *dbeta,
                  double *dgamma, double *dS0, double *dR0) {
-  bwd_impl(ORC_RDN, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+  bwd_impl(ORC_RDN, 0, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
            dO, dST, dRT, dq, dk, dv, dg, dbeta, dgamma, dS0, dR0);
 }
 
@@ -457,7 +513,18 @@ void orc_rla_bwd(int B, int T, int H, int Dk, int Dv, const double *q,
                  const double *dO, const double *dST, const double *dRT,
                  double *dq, double *dk, double *dv, double *dg, double *dbeta,
                  double *dgamma, double *dS0, double *dR0) {
-  bwd_impl(ORC_RLA, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+  bwd_impl(ORC_RLA, 0, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
+           dO, dST, dRT, dq, dk, dv, dg, dbeta, dgamma, dS0, dR0);
+}
+
+/* Backward with the variant bits `mods` (orc_fwd_mod). */
+void orc_bwd_mod(int variant, int mods, int B, int T, int H, int Dk, int Dv,
+                 const double *q, const double *k, const double *v, const double *g,
+                 const double *beta, const double *gamma, double c, double scale,
+                 const double *S0, const double *R0, const double *dO, const double *dST,
+                 const double *dRT, double *dq, double *dk, double *dv, double *dg,
+                 double *dbeta, double *dgamma, double *dS0, double *dR0) {
+  bwd_impl(variant, mods, B, T, H, Dk, Dv, q, k, v, g, beta, gamma, c, scale, S0, R0,
            dO, dST, dRT, dq, dk, dv, dg, dbeta, dgamma, dS0, dR0);
 }
 
@@ -475,7 +542,8 @@ void orc_rla_bwd(int B, int T, int H, int Dk, int Dv, const double *q,
  * representable in the input dtype (quant: 0 = double, 1 = fp32, 2 = bf16).
  * Because p_t depends only on tokens before t, fixing v in token order leaves
  * every later decision well defined.  v [B,T,H,Dv] is modified in place;
- * returns the number of moved elements.  variant 0 = RLA, 1 = RDN.
+ * returns the number of moved elements.  variant 0 = RLA, 1 = RDN; mods as
+ * in orc_fwd_mod (ORC_TANH has a smooth derivative: nothing is moved).
  * ------------------------------------------------------------------------ */
 static double quantize(double x, int quant) {
   if (quant == 1) return (double)(float)x;
@@ -506,7 +574,7 @@ long orc_clip_margin_condition(int variant, int B, int T, int H, int Dk,
                                double *v, const double *g, const double *beta,
                                const double *gamma, double c, double scale,
                                const double *S0, const double *R0,
-                               double margin, int quant) {
+                               double margin, int quant, int mods) {
   const long SD = (long)Dk * Dv;
   long moved = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(+ : moved)
@@ -526,20 +594,22 @@ long orc_clip_margin_condition(int variant, int B, int T, int H, int Dk,
       for (int j = 0; j < Dv; ++j) {
         double pj = 0.0;
         for (int i = 0; i < Dk; ++i) pj += kt[i] * S[i * Dv + j];
-        double x = vt[j] - pj;
-        if (fabs(fabs(x) - c) < margin) {
+        const double a = exp(g[tok]);
+        double x = vt[j] - (mods & ORC_DECAYED ? a * pj : pj);
+        if (!(mods & ORC_TANH) && fabs(fabs(x) - c) < margin) {
           const double sgn_x = x >= 0.0 ? 1.0 : -1.0;
           /* outside (|x| >= c): grow |x|; inside: shrink |x| unless that
              would cross zero before leaving the band */
           double dir = fabs(x) >= c ? sgn_x : -sgn_x;
           if (fabs(x) < c && fabs(x) < 2.0 * margin) dir = sgn_x;
           int guard = 0;
-          while (fabs(fabs(vt[j] - pj) - c) < margin && guard++ < 100000)
+          const double pe = mods & ORC_DECAYED ? a * pj : pj;
+          while (fabs(fabs(vt[j] - pe) - c) < margin && guard++ < 100000)
             vt[j] = step_away(vt[j], dir, quant);
           ++moved;
         }
       }
-      token_step(variant, Dk, Dv, q + tok * Dk, kt, vt, exp(g[tok]), beta[tok],
+      token_step(variant, mods, Dk, Dv, q + tok * Dk, kt, vt, exp(g[tok]), beta[tok],
                  gamma[tok], c, scale, S, R, o, p, rk, NULL);
     }
     free(S); free(R); free(p); free(rk); free(o);
