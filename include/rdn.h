@@ -86,6 +86,26 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  * given receives the gamma part alone.  The backward's fwd.flags carries it. */
 #define RDN_FLAG_TIED_GAMMA 0x2u
 
+/* The paper's variants of the method (all four entry points; any
+ * combination; the backward's fwd.flags carries them):
+ *   RDN_FLAG_DECAYED_RESIDUAL  the residual against the decayed prediction,
+ *       r_t = Clip(v_t - a_t S_{t-1} k_t) (the gated-delta error);
+ *   RDN_FLAG_PLAIN_COMBINE     the ungated output o_t = S_{t-1} q_t + R_t q_t
+ *       (output-combination ablation, Section 4.4);
+ *   RDN_FLAG_TANH_RESIDUAL     the log-cosh residual of Appendix B with the
+ *       threshold as its scale, r_t = c tanh((v_t - S_{t-1} k_t) / c)
+ *       (c = 1 is the paper's tanh; c = INFINITY no limit; c = 0 gives 0);
+ *   RDN_FLAG_STATELESS_AUX     the stateless correction of the residual-
+ *       fitting ablation (Section 4.4): R_t = r_t k_t^T replaces the
+ *       recurrence for R, so R0 is ignored (dR0 = 0 unless T = 0) and RT =
+ *       r_T k_T^T.
+ * These run on the fp32 chunk kernels for every dtype and head dimension
+ * (the tensor-core kernels implement the method itself). */
+#define RDN_FLAG_DECAYED_RESIDUAL 0x4u
+#define RDN_FLAG_PLAIN_COMBINE 0x8u
+#define RDN_FLAG_TANH_RESIDUAL 0x10u
+#define RDN_FLAG_STATELESS_AUX 0x20u
+
 /* Arguments of rla_fwd / rdn_fwd.
  *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
  *                     S0/R0 to ST/RT).
@@ -105,7 +125,7 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *                     recomputing.
  *   scale             multiplies q (the paper uses 1).
  *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd and / or
- *                     RDN_FLAG_TIED_GAMMA (above).
+ *                     RDN_FLAG_TIED_GAMMA and the variant flags (above).
  *   workspace         device scratch of *_fwd_workspace_size() bytes.
  *   cu_seqlens        NULL, or packed variable-length sequences: a device
  *                     int32 array of num_seqs + 1 token offsets, 0 =

@@ -22,6 +22,13 @@ import torch
 
 from . import _abi
 from ._abi import BwdArgs, DecodeArgs, FwdArgs
+# variant flags (variant_flags= of the forward and backward calls): residual
+# against a_t S_{t-1} k_t; ungated combine S_{t-1} q + R_t q; c tanh(x / c)
+# residual; stateless correction R_t = r_t k_t^T
+from ._abi import (RDN_FLAG_DECAYED_RESIDUAL as DECAYED_RESIDUAL,  # noqa: F401
+                   RDN_FLAG_PLAIN_COMBINE as PLAIN_COMBINE,
+                   RDN_FLAG_STATELESS_AUX as STATELESS_AUX,
+                   RDN_FLAG_TANH_RESIDUAL as TANH_RESIDUAL)
 
 __all__ = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "qk_prologue", "qk_prologue_bwd", "rdn_decode_step", "RdnError", "library",
            "CHUNK"]
@@ -73,6 +80,11 @@ def _alloc_ws(nbytes, device):
     return torch.empty(nbytes, dtype=torch.uint8, device=device)
 
 
+def _check_variant_flags(f):
+    if f & ~_abi.RDN_FLAG_VARIANTS:
+        raise ValueError(f"variant_flags 0x{f:x}: only the variant bits are accepted")
+
+
 def _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, Sc, Rc, scale, flags=0,
               cu_seqlens=None):
     B, T, H, Dk = q.shape
@@ -107,8 +119,9 @@ def _chunk_slots(a):
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
          return_final_state=True, return_chunk_states=False, out=None, workspace=None,
-         save_for_bwd=False, tied_gamma=False, cu_seqlens=None):
+         save_for_bwd=False, tied_gamma=False, cu_seqlens=None, variant_flags=0):
     lib = _abi.load()
+    _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
     dev = q.device
@@ -119,7 +132,7 @@ def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
         ST = torch.empty(N, H, Dk, Dv, dtype=torch.float32, device=dev)
         RT = torch.empty_like(ST)
     flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) \
-        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0)
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
     a = FwdArgs()
     _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, None, None, scale, flags,
               cu_seqlens)
@@ -168,7 +181,8 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None):
+            fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
+            variant_flags=0):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
@@ -177,21 +191,25 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     per-chunk matrices are then reused instead of recomputed.
     fwd_saved: that forward ran with save_for_bwd=True."""
     return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens)
+                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
+                variant_flags)
 
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, tied_gamma=False, cu_seqlens=None):
+            fwd_workspace=None, tied_gamma=False, cu_seqlens=None, variant_flags=0):
     """Backward of rla_fwd; the same arguments and results as rdn_bwd (no
     saved intermediates: rla_fwd has no save_for_bwd)."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, False, tied_gamma, cu_seqlens)
+                R_chunks, workspace, out, fwd_workspace, False, tied_gamma, cu_seqlens,
+                variant_flags)
 
 
 def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
-         workspace, out, fwd_workspace, fwd_saved, tied_gamma=False, cu_seqlens=None):
+         workspace, out, fwd_workspace, fwd_saved, tied_gamma=False, cu_seqlens=None,
+         variant_flags=0):
     lib = _abi.load()
+    _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
     dev = q.device
@@ -210,7 +228,7 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
         a.fwd.workspace = _ptr(fwd_workspace)
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
     a.fwd.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if fwd_saved else 0) \
-        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0)
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out.get("dgamma"))

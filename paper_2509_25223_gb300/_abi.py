@@ -12,6 +12,12 @@ F = ctypes.POINTER(ctypes.c_float)
 RDN_F32, RDN_BF16 = 0, 1
 RDN_FLAG_SAVE_FOR_BWD = 0x1  # rdn_fwd_args.flags (include/rdn.h)
 RDN_FLAG_TIED_GAMMA = 0x2
+# the paper's variants of the method
+RDN_FLAG_DECAYED_RESIDUAL = 0x4
+RDN_FLAG_PLAIN_COMBINE = 0x8
+RDN_FLAG_TANH_RESIDUAL = 0x10
+RDN_FLAG_STATELESS_AUX = 0x20
+RDN_FLAG_VARIANTS = 0x3C
 
 STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "RDN_ERR_CUDA",
           4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}

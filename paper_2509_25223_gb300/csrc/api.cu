@@ -107,7 +107,7 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
     if (!aligned16(a->cu_seqlens))
       return fail(RDN_ERR_MISALIGNED, "%s: cu_seqlens is not 16-byte aligned", fn);
   }
-  if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA))
+  if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
   if (isnan(a->scale) || isinf(a->scale))
     return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);

@@ -100,6 +100,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
   InT *dv = (InT *)p.dv;
   const float clip = p.f.clip;
   const size_t sbase = (size_t)bh * DK * DV;
+  const bool dec_res = p.f.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = p.f.mods & RDN_FLAG_PLAIN_COMBINE;
+  const bool tnh = p.f.mods & RDN_FLAG_TANH_RESIDUAL;
+  const bool stl = p.f.mods & RDN_FLAG_STATELESS_AUX;
+  const bool rdn_aux = RDNV && !stl;  // the auxiliary pass runs the delta rule
 
   using MMk = BlockMM<C, kBDVS, DK>;   // [C x DK] @ [DK x DVS]
   using MMc = BlockMM<C, kBDVS, C>;    // [C x C] @ [C x DVS]
@@ -170,8 +175,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
         const int t = MMk::row(i);
         KS[t * LDV + col] = a1[i];
         QS[t * LDV + col] = a2[i];
-        KR[t * LDV + col] = a3[i];
-        QR[t * LDV + col] = a4[i];
+        KR[t * LDV + col] = stl ? 0.f : a3[i];  // (the stateless R carries nothing)
+        QR[t * LDV + col] = stl ? 0.f : a4[i];
         if (RDNV) T1[t * LDV + col] = Vs[t * LDV + col] - Gam[t] * a1[i];
       }
     }
@@ -194,14 +199,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
-        const float x = Vs[t * LDV + col] - (Gprev[t] * KS[t * LDV + col] + a1[i]);
+        const float x =
+            Vs[t * LDV + col] - ((dec_res ? Gam[t] : Gprev[t]) * KS[t * LDV + col] + a1[i]);
         XR[t * LDV + col] = x;
-        if (RDNV) T1[t * LDV + col] = clampf(x, clip) - Gam[t] * KR[t * LDV + col];
-        else E2[t * LDV + col] = clampf(x, clip);
+        if (rdn_aux) T1[t * LDV + col] = resid_map(x, clip, tnh) - Gam[t] * KR[t * LDV + col];
+        else E2[t * LDV + col] = resid_map(x, clip, tnh);
       }
     }
     __syncthreads();
-    if (RDNV) {
+    if (rdn_aux) {
       for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
@@ -220,9 +226,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
         const int t = MMc::row(i);
         const float oa = Gam[t] * QR[t * LDV + col] + a1[i];
         const float dOv = dOs[t * LDV + col];
-        const float doa = gmv[t] * dOv;
+        const float doa = plain ? dOv : gmv[t] * dOv;
         T3[t * LDV + col] = doa;
-        atomicAdd(&red[L::V_DGAM_OUT + t], dOv * oa);
+        if (!plain) atomicAdd(&red[L::V_DGAM_OUT + t], dOv * oa);
         atomicAdd(&red[L::V_DGAM + t], doa * QR[t * LDV + col]);
       }
     }
@@ -237,8 +243,10 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
         T1[t * LDV + col] = a1[i] + wR[t] * kd[i];  // dE2
-        atomicAdd(&red[L::V_DWR + t], kd[i] * E2[t * LDV + col]);
-        QR[t * LDV + col] = Gam[t] * T3[t * LDV + col];  // dQR
+        if (!stl) {  // (stateless: wR is a constant and R0 does not enter)
+          atomicAdd(&red[L::V_DWR + t], kd[i] * E2[t * LDV + col]);
+          QR[t * LDV + col] = Gam[t] * T3[t * LDV + col];  // dQR
+        }
       }
       float g1[MMg::RPT];
       MMg::run(T3, LDV, 1, E2, 1, LDV, g1);  // dM2 = dOa E2^T (inclusive)
@@ -250,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     }
     __syncthreads();
     const float *dRv = T1;
-    if (RDNV) {
+    if (rdn_aux) {
       for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
@@ -283,34 +291,36 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     {
       float g1[MMd::RPT];
       MMd::run(T3, LDV, 1, dR, 1, LDV, dKacc);
-      if (RDNV) {
+      if (rdn_aux) {
         MMd::run(T1, LDV, 1, R0, 1, LDV, g1);
 #pragma unroll
         for (int i = 0; i < MMd::RPT; ++i) dKacc[i] += g1[i];
       }
       MMd::run(QR, LDV, 1, R0, 1, LDV, dQacc);
       float s = 0.f;
-      for (int e = tid; e < DK * kBDVS; e += kThreads) {
-        const int i = e / kBDVS, jj = e % kBDVS;
-        s += dR[i * LDV + jj] * R0[i * LDV + jj];
-      }
+      if (!stl)
+        for (int e = tid; e < DK * kBDVS; e += kThreads) {
+          const int i = e / kBDVS, jj = e % kBDVS;
+          s += dR[i * LDV + jj] * R0[i * LDV + jj];
+        }
       atomicAdd(&red[L::V_DGAMC], s);
     }
     __syncthreads();
-    {  // dR0 = Gam_C dR + K^T dKR + Q^T dQR
+    {  // dR0 = Gam_C dR + K^T dKR + Q^T dQR (stateless: 0)
       float u1[MMu::RPT], u2[MMu::RPT];
       MMu::run(Qs, 1, LDK, QR, LDV, 1, u2);
-      if (RDNV) MMu::run(Ks, 1, LDK, T1, LDV, 1, u1);
+      if (rdn_aux) MMu::run(Ks, 1, LDK, T1, LDV, 1, u1);
 #pragma unroll
       for (int i = 0; i < MMu::RPT; ++i) {
         const int r = MMu::row(i);
-        dR[r * LDV + col] = GamC * dR[r * LDV + col] + u2[i] + (RDNV ? u1[i] : 0.f);
+        dR[r * LDV + col] =
+            stl ? 0.f : GamC * dR[r * LDV + col] + u2[i] + (rdn_aux ? u1[i] : 0.f);
       }
     }
-    // clip: dV = dRv * [|x| <= c] into T3 (dP = -dV)
+    // clip: dV = dRv * [|x| <= c] into T3 (dP = -dV; tanh: times 1 - (r/c)^2)
     for (int e = tid; e < C * kBDVS; e += kThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
-      T3[t * LDV + jj] = fabsf(XR[t * LDV + jj]) <= clip ? dRv[t * LDV + jj] : 0.f;
+      T3[t * LDV + jj] = dRv[t * LDV + jj] * resid_grad(XR[t * LDV + jj], clip, tnh);
     }
     __syncthreads();
 
@@ -345,11 +355,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
         const float dv_ = T3[t * LDV + col];
         T1[t * LDV + col] = de[i] - a1[i] + wS[t] * kd[i];  // dE
         atomicAdd(&red[L::V_DWS + t], kd[i] * E[t * LDV + col]);
-        atomicAdd(&red[L::V_DGPREV + t], -dv_ * KS[t * LDV + col]);
-        T2[t * LDV + col] = -Gprev[t] * dv_;  // dKS (base part)
+        // the prediction's state term: Gprev KS (decayed residual: Gam KS)
+        atomicAdd(&red[(dec_res ? L::V_DGAM : L::V_DGPREV) + t], -dv_ * KS[t * LDV + col]);
+        T2[t * LDV + col] = -(dec_res ? Gam[t] : Gprev[t]) * dv_;  // dKS (base part)
         const float dOv = dOs[t * LDV + col];
-        atomicAdd(&red[L::V_DGAM + t], dOv * QS[t * LDV + col]);
-        QS[t * LDV + col] = Gam[t] * dOv;  // dQS
+        // the base read-out Gam QS (plain combine: Gprev QS)
+        atomicAdd(&red[(plain ? L::V_DGPREV : L::V_DGAM) + t], dOv * QS[t * LDV + col]);
+        QS[t * LDV + col] = (plain ? Gprev[t] : Gam[t]) * dOv;  // dQS
       }
     }
     __syncthreads();
@@ -482,6 +494,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   const InT *q = (const InT *)p.f.q;
   const InT *k = (const InT *)p.f.k;
   const float *acc = p.acc + (size_t)chunk * L::FLOATS;
+  const bool dec_res = p.f.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = p.f.mods & RDN_FLAG_PLAIN_COMBINE;
+  const bool stl = p.f.mods & RDN_FLAG_STATELESS_AUX;
 
   for (int e = tid; e < C * DK; e += kThreads) {
     const int t = e / DK, d = e % DK;
@@ -549,7 +564,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
         const float dec = expf(cum[t] - cum[i]);
         const float kk = KK[t * LDC + i], qk = QK[t * LDC + i];
         const float bi = bet[i], gi = gam[i];
-        {  // M2: inclusive, gamma, QK
+        if (stl) {  // M2 = diag(QK): no decay, no rate
+          if (i == t) dqk += acc[L::DM2 + e];
+        } else {  // M2: inclusive, gamma, QK
           const float dm = acc[L::DM2 + e];
           const float G = dm * dec * gi * qk;
           rowc += G;
@@ -559,21 +576,23 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
         }
         if (i < t) {
           const float decp = expf(cprev[t] - cum[i]);
-          {  // Ap: strict, beta, KK, previous-token decay
+          {  // Ap: strict, beta, KK, previous-token decay (decayed residual: to t)
+            const float dA = dec_res ? dec : decp;
             const float dm = acc[L::DAP + e];
-            const float G = dm * decp * bi * kk;
-            rowp += G;
+            const float G = dm * dA * bi * kk;
+            if (dec_res) rowc += G; else rowp += G;
             cg += G;
-            cb += dm * decp * kk;
-            dkk += dm * decp * bi;
+            cb += dm * dA * kk;
+            dkk += dm * dA * bi;
           }
-          {  // Mq: strict, beta, QK
+          {  // Mq: strict, beta, QK (plain combine: decay to t-1)
+            const float dA = plain ? decp : dec;
             const float dm = acc[L::DMQ + e];
-            const float G = dm * dec * bi * qk;
-            rowc += G;
+            const float G = dm * dA * bi * qk;
+            if (plain) rowp += G; else rowc += G;
             cg += G;
-            cb += dm * dec * qk;
-            dqk += dm * dec * bi;
+            cb += dm * dA * qk;
+            dqk += dm * dA * bi;
           }
           if (RDNV) {
             const float da = acc[L::DAB + e], dg2 = acc[L::DAG + e];
@@ -728,7 +747,7 @@ struct BwdLayout {
 // RDN with bf16 inputs and d = 128 takes the tensor-core backward (RLA, whose
 // forward stays on the fp32 SIMT scan, the SIMT backward)
 bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
-  return variant == 1 && f.dtype == RDN_BF16 && f.Dk == 128;
+  return variant == 1 && f.dtype == RDN_BF16 && f.Dk == 128 && !(f.flags & RDN_FLAG_VARIANTS);
 }
 
 // The forward's per-chunk records are valid input when the caller passes the
@@ -836,7 +855,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
     // the tensor-core forward leaves its records as shared-memory images,
     // which the tensor-core backward reads too; the SIMT backward needs fp32
-    if (e == cudaSuccess && rdnv && bf && f.Dk == 128 && !tc)
+    if (e == cudaSuccess && rdnv && bf && f.Dk == 128 && !tc && p.f.mods == 0)
       e = launch_prep(p.f, f.Dk, rdnv, bf, false, s);
   } else if (!reuse) {
     e = launch_prep(p.f, f.Dk, rdnv, bf, tc, s);

@@ -124,6 +124,7 @@ struct FwdParams {
   const long long *seq;
   int nseq;        // sequences: B, or the number of packed sequences
   long long nrec;  // record slots: B * H * NC, or a bound on H * (total chunks)
+  unsigned mods;   // the variant flags (RDN_FLAG_VARIANTS bits of rdn_fwd_args.flags)
 };
 
 // Where sequence s's tokens and (s, h)'s chunk records are.  Token t of the
@@ -206,6 +207,7 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.seq = nullptr;  // set by the launcher once the table is in its workspace
   p.nseq = call_seqs(a);
   p.nrec = call_records(a);
+  p.mods = a.flags & RDN_FLAG_VARIANTS;
   return p;
 }
 

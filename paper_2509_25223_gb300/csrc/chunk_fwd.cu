@@ -122,15 +122,22 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
   }
   __syncthreads();
   float *rec = p.ws + (size_t)chunk * kRecFloats;
+  // variants: the decayed residual predicts with a_t S_{t-1} k_t, so Ap takes
+  // the decay to t (not t-1); the plain combine reads S_{t-1} q_t, so Mq takes
+  // the decay to t-1; the stateless correction reads r_t (q_t.k_t) alone
+  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = p.mods & RDN_FLAG_PLAIN_COMBINE;
+  const bool stl = p.mods & RDN_FLAG_STATELESS_AUX;
   for (int e = tid; e < C * C; e += kThreads) {
     const int t = e / C, i = e % C;
     float ap = 0.f, mq = 0.f, m2 = 0.f, ab = 0.f, ag = 0.f;
     if (i <= t) {
       const float dec = expf(cum[t] - cum[i]);
-      m2 = dec * gam[i] * QK[t * LDC + i];
+      m2 = stl ? (i == t ? QK[t * LDC + i] : 0.f) : dec * gam[i] * QK[t * LDC + i];
       if (i < t) {
-        ap = expf(cprev[t] - cum[i]) * bet[i] * KK[t * LDC + i];
-        mq = dec * bet[i] * QK[t * LDC + i];
+        const float decp = expf(cprev[t] - cum[i]);
+        ap = (dec_res ? dec : decp) * bet[i] * KK[t * LDC + i];
+        mq = (plain ? decp : dec) * bet[i] * QK[t * LDC + i];
         ab = dec * bet[i] * KK[t * LDC + i];
         ag = dec * gam[i] * KK[t * LDC + i];
       }
@@ -157,7 +164,8 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
     rec[OFF_VEC + V_GPREV + t] = expf(cprev[t]);
     rec[OFF_VEC + V_ALPHA + t] = expf(gg[t]);
     rec[OFF_VEC + V_WS + t] = bet[t] * expf(cC - cum[t]);
-    rec[OFF_VEC + V_WR + t] = gam[t] * expf(cC - cum[t]);
+    // (stateless correction: R at the chunk end is k r^T of its last token)
+    rec[OFF_VEC + V_WR + t] = stl ? (t == n - 1 ? 1.f : 0.f) : gam[t] * expf(cC - cum[t]);
     if (t == 0) rec[OFF_VEC + V_GAMC] = expf(cC);
   }
   if (RDNV) {
@@ -221,6 +229,11 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
   const InT *v = (const InT *)p.v;
   InT *o = (InT *)p.o;
   const float clip = p.clip;
+  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = p.mods & RDN_FLAG_PLAIN_COMBINE;
+  const bool tnh = p.mods & RDN_FLAG_TANH_RESIDUAL;
+  const bool stl = p.mods & RDN_FLAG_STATELESS_AUX;
+  const bool rdn_aux = RDNV && !stl;  // the auxiliary pass runs the delta rule
 
   const size_t sbase = (size_t)bh * DK * DV;
   for (int e = tid; e < DK * kDVS; e += kThreads) {
@@ -299,8 +312,9 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
-        const float pt = Gprev[t] * KS[t * kDVS + col] + a1[i];
-        Ps[t * kDVS + col] = clampf(Vs[t * kDVS + col] - pt, clip);  // r, Section 3.3
+        // P_t = S_{t-1}^T k_t (decayed residual: a_t S_{t-1}^T k_t)
+        const float pt = (dec_res ? Gam[t] : Gprev[t]) * KS[t * kDVS + col] + a1[i];
+        Ps[t * kDVS + col] = resid_map(Vs[t * kDVS + col] - pt, clip, tnh);  // r, Section 3.3
       }
     }
     __syncthreads();
@@ -312,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
-        Ob[t * kDVS + col] = Gam[t] * QS[t * kDVS + col] + a1[i];
+        Ob[t * kDVS + col] = (plain ? Gprev[t] : Gam[t]) * QS[t * kDVS + col] + a1[i];
       }
     }
     // S_C = Gam_C S0 + K^T diag(wS) E   (W = wS * E)
@@ -336,12 +350,12 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMk::RPT; ++i) {
         const int t = MMk::row(i);
-        QS[t * kDVS + col] = a2[i];  // Q R0
-        if (RDNV) Ws[t * kDVS + col] = Ps[t * kDVS + col] - Gam[t] * a1[i];
+        QS[t * kDVS + col] = stl ? 0.f : a2[i];  // Q R0 (the stateless R carries nothing)
+        if (rdn_aux) Ws[t * kDVS + col] = Ps[t * kDVS + col] - Gam[t] * a1[i];
       }
     }
     const float *E2 = Ps;
-    if (RDNV) {
+    if (rdn_aux) {
       for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
@@ -360,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       for (int i = 0; i < MMc::RPT; ++i) {
         const int t = MMc::row(i);
         if (t < n) {
-          const float gm = p.gamma[(size_t)(sp.tok0 + t0 + t) * p.H + h];
+          const float gm = plain ? 1.f : p.gamma[(size_t)(sp.tok0 + t0 + t) * p.H + h];
           const float oa = Gam[t] * QS[t * kDVS + col] + a1[i];
           o[((size_t)(sp.tok0 + t0 + t) * p.H + h) * DV + j0 + col] =
               from_f32<InT>(Ob[t * kDVS + col] + gm * oa);
@@ -376,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMu::RPT; ++i) {
         const int r = MMu::row(i);
-        Rs[r * kDVS + col] = GamC * Rs[r * kDVS + col] + a1[i];
+        Rs[r * kDVS + col] = (stl ? 0.f : GamC) * Rs[r * kDVS + col] + a1[i];
       }
     }
   }
@@ -412,7 +426,7 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
   if (do_prep) {
     // the images for RDN with bf16 inputs and d = 128 come from the tensor-core prep
     constexpr bool tc_prep = DK == 128 && RDNV && std::is_same<InT, __nv_bfloat16>::value;
-    if (tc_prep && img) {
+    if (tc_prep && img && p.mods == 0) {
       if ((e = launch_prep_tc(p, s)) != cudaSuccess) return e;
     } else {
       RDN_LAUNCH("chunk_prep", s, prep<<<(unsigned)p.nrec, kThreads, prep_smem<DK>(), s>>>(p));
@@ -432,7 +446,7 @@ cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, b
   // else the fp32 SIMT one.  (RLA's state is not contracted by the delta
   // term, and its output error with single-bf16 state operands reaches the
   // 2e-2 RMS bound, so RLA stays on the fp32 path.)
-  const bool tc_scan = do_scan && bf16 && DK == 128 && rdnv;
+  const bool tc_scan = do_scan && bf16 && DK == 128 && rdnv && p.mods == 0;
   cudaError_t e = cudaSuccess;
   // (the tensor-core scan reads the records as shared-memory images)
   if (DK == 128) {

@@ -10,6 +10,10 @@ namespace rdn {
 
 // Chunk length of the chunkwise-parallel forms (tokens per chunk).
 constexpr int kChunk = 64;
+// the variant flags of rdn.h, which the fp32 chunk kernels implement
+#define RDN_FLAG_VARIANTS                                                             \
+  (RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE | RDN_FLAG_TANH_RESIDUAL | \
+   RDN_FLAG_STATELESS_AUX)
 
 template <typename T> __device__ __forceinline__ float to_f32(T x);
 template <> __device__ __forceinline__ float to_f32<float>(float x) { return x; }
@@ -24,6 +28,23 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 }
 
 __device__ __forceinline__ float clampf(float x, float c) { return fminf(fmaxf(x, -c), c); }
+
+// The residual map of Section 3.3 (clip to [-c, c]) or, with tnh, the
+// log-cosh residual c tanh(x / c) of Appendix B; and their derivatives (the
+// clip's taken as 1 on |x| <= c).
+__device__ __forceinline__ float resid_map(float x, float c, bool tnh) {
+  if (!tnh) return clampf(x, c);
+  if (isinf(c)) return x;
+  if (c == 0.f) return 0.f;
+  return c * tanhf(x / c);
+}
+__device__ __forceinline__ float resid_grad(float x, float c, bool tnh) {
+  if (!tnh) return fabsf(x) <= c ? 1.f : 0.f;
+  if (isinf(c)) return 1.f;
+  if (c == 0.f) return 0.f;
+  const float t = tanhf(x / c);
+  return 1.f - t * t;
+}
 
 }  // namespace rdn
 

@@ -64,7 +64,7 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(dtype=7)) == 2
     assert _status(fn, _fwd_args(clip=-1.0)) == 1
     assert _status(fn, _fwd_args(clip=float("nan"))) == 1
-    assert _status(fn, _fwd_args(flags=4)) == 2
+    assert _status(fn, _fwd_args(flags=0x40)) == 2
     # tied gates: gamma may be NULL (beta serves as both); the call then gets
     # as far as the workspace check
     tied = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, o=FAKE)
