@@ -519,6 +519,37 @@ def run_ours(args):
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr
 
+    # ---- the paper's variants (variant_flags, fp32 chunk kernels) on the
+    # bench workload: RDN fwd+bwd with each flag, as the RDN step above
+    var = None
+    if not args.no_variants:
+        var = {"workload": w.name, "path": "fp32 SIMT chunk kernels", "steps": 1, "flags": {}}
+        wsbv_ = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D,
+                                                variant_flags=rdn.DECAYED_RESIDUAL),
+                            dtype=torch.uint8, device=dev)
+        for fname, fl in (("decayed_residual", rdn.DECAYED_RESIDUAL),
+                          ("plain_combine", rdn.PLAIN_COMBINE),
+                          ("tanh_residual", rdn.TANH_RESIDUAL),
+                          ("stateless_aux", rdn.STATELESS_AUX)):
+            def fstep(inp):
+                _, _, _, Sc_, Rc_ = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
+                                                return_chunk_states=True, out=o, workspace=wsf,
+                                                variant_flags=fl)
+                rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
+                            R_chunks=Rc_, workspace=wsbv_, out=grads, fwd_workspace=wsf,
+                            variant_flags=fl)
+            fstep(x)
+            torch.cuda.synchronize()
+            barrier(dist)
+            e0.record(stream)
+            fstep(x)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            barrier(dist)
+            tf, fval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step)
+            var["flags"][fname] = {"value": fval, "unit": "tokens/s", "ms_per_step": tf}
+        del wsbv_
+
     # ---- packed variable-length sequences: the same B*T tokens per head as
     # one packed row of seeded log-uniform lengths in [64, 8192] (the last one
     # cut to fill the row), RDN fwd+bwd exactly as the step above
@@ -629,7 +660,7 @@ def run_ours(args):
                                 "share": t / sum(v[1] for v in kern.values())}
                             for k, (n, t, m) in kern.items()},
                 "clocks": clk.summary(), "decode": dec, "rla": rla, "prologue": pro,
-                "varlen": vl}
+                "varlen": vl, "variants": var}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -648,6 +679,7 @@ def main(argv=None):
     ap.add_argument("--no-rla", action="store_true")
     ap.add_argument("--no-prologue", action="store_true")
     ap.add_argument("--no-varlen", action="store_true")
+    ap.add_argument("--no-variants", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")

@@ -204,7 +204,10 @@ typedef struct {
  *   q, k [N,H,Dk]; v, o [N,H,Dv]; g, beta, gamma [N,H] fp32.
  *   S, R [N,H,Dk,Dv] fp32, read and updated IN PLACE (must not alias any
  *   other argument).
- *   variant           0 = RLA, 1 = RDN.                                   */
+ *   variant           0 = RLA, 1 = RDN.
+ *   flags             0, or RDN_FLAG_TIED_GAMMA (gamma ignored, beta serves
+ *                     as both rates) and / or the variant flags: the same
+ *                     token step as the forward with those flags.        */
 typedef struct {
   int N, H, Dk, Dv;
   int dtype;
@@ -215,6 +218,7 @@ typedef struct {
   float scale;
   float *S, *R;
   void *o;
+  unsigned flags;
 } rdn_decode_args;
 
 /* Arguments of rdn_qk_prologue / rdn_qk_prologue_bwd: the activation and

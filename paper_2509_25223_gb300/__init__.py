@@ -284,10 +284,13 @@ def qk_prologue_bwd(q, k, dyq, dyk=None, eps=1e-12):
     return dq, dk
 
 
-def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant="rdn", out=None):
+def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant="rdn", out=None,
+                    tied_gamma=False, variant_flags=0):
     """One recurrent step for N sequences; S, R [N,H,Dk,Dv] fp32 are updated
-    in place.  q, k [N,H,Dk]; v [N,H,Dv]; gates [N,H].  Returns o [N,H,Dv]."""
+    in place.  q, k [N,H,Dk]; v [N,H,Dv]; gates [N,H].  Returns o [N,H,Dv].
+    tied_gamma / variant_flags: as for the forward."""
     lib = _abi.load()
+    _check_variant_flags(variant_flags)
     N, H, Dk = q.shape
     Dv = v.shape[-1]
     o = out if out is not None else torch.empty(N, H, Dv, dtype=q.dtype, device=q.device)
@@ -299,6 +302,7 @@ def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant=
     a.g, a.beta, a.gamma = _ptr(g), _ptr(beta), _ptr(gamma)
     a.clip, a.scale = float(clip), float(scale)
     a.S, a.R, a.o = _ptr(S), _ptr(R), _ptr(o)
+    a.flags = (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
     _check("rdn_decode_step", lib.rdn_decode_step(ctypes.byref(a), _stream(q)))
     return o
 
@@ -338,15 +342,18 @@ class LaunchTimer:
         return {k: (c, t, t / c) for k, (c, t) in out.items()}
 
 
-def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False, cu_seqlens=None):
+def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False, cu_seqlens=None,
+                    variant_flags=0):
     """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rla_bwd | rdn_bwd);
-    cu_seqlens: the packed-sequence table of the call (B = 1)."""
+    cu_seqlens: the packed-sequence table of the call (B = 1); variant_flags:
+    the variant bits of the call."""
     lib = _abi.load()
     a = FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
     a.dtype = _abi.RDN_BF16 if dtype == torch.bfloat16 else _abi.RDN_F32
     a.clip, a.scale = 1.0, 1.0
-    a.flags = _abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0
+    _check_variant_flags(variant_flags)
+    a.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) | variant_flags
     if cu_seqlens is not None:
         a.cu_seqlens, a.num_seqs = _ptr(cu_seqlens), cu_seqlens.numel() - 1
     n = ctypes.c_size_t(0)

@@ -463,17 +463,21 @@ rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {
   rdn_status_t st = check_clip(fn, a->clip);
   if (st != RDN_OK) return st;
   if (isnan(a->scale) || isinf(a->scale)) return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
+  if (a->flags & ~(RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS))
+    return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
   REQUIRE_PTR(a->q);
   REQUIRE_PTR(a->k);
   REQUIRE_PTR(a->v);
   REQUIRE_PTR(a->g);
   REQUIRE_PTR(a->beta);
-  REQUIRE_PTR(a->gamma);
+  if (!(a->flags & RDN_FLAG_TIED_GAMMA)) REQUIRE_PTR(a->gamma);
   REQUIRE_PTR(a->S);
   REQUIRE_PTR(a->R);
   REQUIRE_PTR(a->o);
   if (a->S == a->R) return fail(RDN_ERR_INVALID_ARG, "%s: S and R alias", fn);
-  return cuda_status(fn, rdn::launch_decode(*a, (cudaStream_t)stream));
+  rdn_decode_args b = *a;
+  if (a->flags & RDN_FLAG_TIED_GAMMA) b.gamma = a->beta;
+  return cuda_status(fn, rdn::launch_decode(b, (cudaStream_t)stream));
 }
 
 }  // extern "C"

@@ -16,6 +16,10 @@
 //     o  = a sq + gam (q^T R') = a sq + gam (a rq + gam (k.q) e2)
 // which is the right (RDN) / left (RLA) formulation of Section 3.4 with the
 // delta-rule product expanded: a S (I - b k k^T) + b k v^T = a S + b k (v - a S^T k)^T.
+// The variant flags change the step as in the chunk kernels: r = resid(v - a p)
+// (decayed residual), c tanh(x / c) (tanh residual), R' = k r^T without
+// reading R (stateless correction, o's correction term gam (k.q) r), and
+// o = sq + q^T R' (plain combine).
 #include "common.cuh"
 
 namespace rdn {
@@ -30,7 +34,7 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
               const InT *__restrict__ v, const float *__restrict__ g,
               const float *__restrict__ beta, const float *__restrict__ gam,
               float clip, float scale, float *__restrict__ S, float *__restrict__ R,
-              InT *__restrict__ o) {
+              InT *__restrict__ o, unsigned mods) {
   constexpr int RPT = D / 16;             // rows per thread (16 row groups)
   constexpr int NSLICE = D / kSliceCols;  // column slices per (n,h)
   __shared__ float q_s[D], k_s[D];
@@ -44,6 +48,10 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
   const int cg = tid & 15, rg = tid >> 4;
   const int warp = tid >> 5;
   const size_t sbase = (size_t)nh * D * D + (size_t)slice * kSliceCols + 4 * cg;
+  const bool dec_res = mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = mods & RDN_FLAG_PLAIN_COMBINE;
+  const bool tnh = mods & RDN_FLAG_TANH_RESIDUAL;
+  const bool stl = mods & RDN_FLAG_STATELESS_AUX;
 
   // issue the state loads first: they are the whole cost of the step
   float4 s_reg[RPT], r_reg[RPT];
@@ -51,7 +59,8 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
   for (int i = 0; i < RPT; ++i) {
     const size_t off = sbase + (size_t)(rg * RPT + i) * D;
     s_reg[i] = __ldcs(reinterpret_cast<const float4 *>(S + off));
-    r_reg[i] = __ldcs(reinterpret_cast<const float4 *>(R + off));
+    r_reg[i] = stl ? make_float4(0.f, 0.f, 0.f, 0.f)  // (the stateless R is not read)
+                   : __ldcs(reinterpret_cast<const float4 *>(R + off));
   }
   for (int i = tid; i < D; i += kDecThreads) {
     q_s[i] = scale * to_f32(q[(size_t)nh * D + i]);
@@ -114,27 +123,31 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
     const int col = 4 * cg + c;
     const float vj = to_f32(v[(size_t)nh * D + slice * kSliceCols + col]);
     const float p = tot[0][col], rk = tot[2][col];
-    const float r = clampf(vj - p, clip);
+    const float r = resid_map(vj - (dec_res ? alpha * p : p), clip, tnh);
     e[c] = RDN_VARIANT ? vj - alpha * p : vj;
-    e2[c] = RDN_VARIANT ? r - alpha * rk : r;
+    e2[c] = stl ? r : RDN_VARIANT ? r - alpha * rk : r;
     if (rg == 0) {
-      const float oj = alpha * tot[1][col] + gm * (alpha * tot[3][col] + gm * kq * e2[c]);
+      // q^T R' = a rq + gam (k.q) e2, or (k.q) r for the stateless R' = k r^T
+      const float qr = stl ? kq * r : alpha * tot[3][col] + gm * kq * e2[c];
+      const float oj = plain ? tot[1][col] + qr : alpha * tot[1][col] + gm * qr;
       o[(size_t)nh * D + slice * kSliceCols + col] = from_f32<InT>(oj);
     }
   }
+  // R' = a R + gam k e2^T, or k r^T for the stateless correction
+  const float ra = stl ? 0.f : alpha, rgm = stl ? 1.f : gm;
 #pragma unroll
   for (int i = 0; i < RPT; ++i) {
     const float ki = k_s[rg * RPT + i];
-    const float bk = b * ki, gk = gm * ki;
+    const float bk = b * ki, gk = rgm * ki;
     float4 sn, rn;
     sn.x = fmaf(alpha, s_reg[i].x, bk * e[0]);
     sn.y = fmaf(alpha, s_reg[i].y, bk * e[1]);
     sn.z = fmaf(alpha, s_reg[i].z, bk * e[2]);
     sn.w = fmaf(alpha, s_reg[i].w, bk * e[3]);
-    rn.x = fmaf(alpha, r_reg[i].x, gk * e2[0]);
-    rn.y = fmaf(alpha, r_reg[i].y, gk * e2[1]);
-    rn.z = fmaf(alpha, r_reg[i].z, gk * e2[2]);
-    rn.w = fmaf(alpha, r_reg[i].w, gk * e2[3]);
+    rn.x = fmaf(ra, r_reg[i].x, gk * e2[0]);
+    rn.y = fmaf(ra, r_reg[i].y, gk * e2[1]);
+    rn.z = fmaf(ra, r_reg[i].z, gk * e2[2]);
+    rn.w = fmaf(ra, r_reg[i].w, gk * e2[3]);
     const size_t off = sbase + (size_t)(rg * RPT + i) * D;
     __stcs(reinterpret_cast<float4 *>(S + off), sn);
     __stcs(reinterpret_cast<float4 *>(R + off), rn);
@@ -148,12 +161,12 @@ cudaError_t launch_decode_t(const rdn_decode_args &a, cudaStream_t s) {
     RDN_LAUNCH("decode", s,
                decode_kernel<D, true, InT><<<grid, kDecThreads, 0, s>>>(
                    a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
-                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o));
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS));
   else
     RDN_LAUNCH("decode", s,
                decode_kernel<D, false, InT><<<grid, kDecThreads, 0, s>>>(
                    a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
-                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o));
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS));
   return cudaGetLastError();
 }
 

@@ -145,6 +145,9 @@ def test_decode_validation():
     a.clip = -2.0
     assert lib.rdn_decode_step(ctypes.byref(a), None) == 1
     a.clip = math.inf
+    a.flags = 0x40
+    assert lib.rdn_decode_step(ctypes.byref(a), None) == 2  # not a variant flag
+    a.flags = 0
     a.Dk = a.Dv = 256
     assert lib.rdn_decode_step(ctypes.byref(a), None) == 2
 

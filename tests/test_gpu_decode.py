@@ -72,3 +72,32 @@ def test_decode_no_clip_and_zero_clip():
         (o, S, R), (oref, Sref, Rref) = _step(x, 0, "rdn", clip=clip)
         assert_close(o, oref, "bf16", f"o clip={clip}")
         assert_close(R, Rref, "f32", f"R clip={clip}")
+
+
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
+@pytest.mark.parametrize("flags", [rdn.DECAYED_RESIDUAL, rdn.PLAIN_COMBINE, rdn.TANH_RESIDUAL,
+                                   rdn.STATELESS_AUX,
+                                   rdn.DECAYED_RESIDUAL | rdn.TANH_RESIDUAL | rdn.PLAIN_COMBINE])
+@pytest.mark.parametrize("tied", [False, True])
+def test_decode_variants(variant, flags, tied):
+    """The variant flags and tied gates in the decode step equal one token of
+    the oracle's forward with the same variant bits (S0, R0 = the states)."""
+    x = make_decode_inputs(5, 3, 128, steps=1, device="cuda", state_std=0.3)
+    mods = {rdn.DECAYED_RESIDUAL: oracle.DECAYED, rdn.PLAIN_COMBINE: oracle.PLAIN,
+            rdn.TANH_RESIDUAL: oracle.TANH, rdn.STATELESS_AUX: oracle.STATELESS}
+    m = sum(o for f, o in mods.items() if flags & f)
+    gam = x["beta"][0] if tied else x["gamma"][0]
+    S, R = x["S"].clone(), x["R"].clone()
+    o = rdn.rdn_decode_step(x["q"][0], x["k"][0], x["v"][0], x["g"][0], x["beta"][0],
+                            None if tied else gam, S, R, clip=0.7, variant=variant,
+                            tied_gamma=tied, variant_flags=flags)
+    torch.cuda.synchronize()
+    tok = lambda t: as64(t)[:, None]  # [N,H,...] -> [N,1,H,...]: one token of the forward
+    oref, Sref, Rref = oracle.fwd(oracle.RDN if variant == "rdn" else oracle.RLA,
+                                  tok(x["q"][0]), tok(x["k"][0]), tok(x["v"][0]), tok(x["g"][0]),
+                                  tok(x["beta"][0]), tok(gam), 0.7, as64(x["S"]), as64(x["R"]),
+                                  mods=m)
+    assert_close(o, oref[:, 0], "bf16", "o")
+    assert_close(S, Sref, "f32", "S")
+    assert_close(R, Rref, "f32", "R")
+
