@@ -33,6 +33,7 @@ namespace rdn {
 namespace {
 
 constexpr int kBDVS = 16;       // value columns per backward scan CTA
+constexpr int kScanThreads = 512;  // threads of a backward scan CTA (latency bound: 16 warps)
 constexpr int LDV = kBDVS + 1;  // padded row stride of the [C][kBDVS] tiles
 
 template <int DK>
@@ -58,7 +59,7 @@ struct BwdParams {
 
 // ---------------------------------------------------------------- kernel 1
 template <int DK, bool RDNV, typename InT>
-__global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
+__global__ void __launch_bounds__(kScanThreads, 1) bwd_scan_kernel(BwdParams p) {
   constexpr int DV = DK;
   constexpr int LDK = DK + 1;
   using L = Acc<DK>;
@@ -106,14 +107,14 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
   const bool stl = p.f.mods & RDN_FLAG_STATELESS_AUX;
   const bool rdn_aux = RDNV && !stl;  // the auxiliary pass runs the delta rule
 
-  using MMk = BlockMM<C, kBDVS, DK>;   // [C x DK] @ [DK x DVS]
-  using MMc = BlockMM<C, kBDVS, C>;    // [C x C] @ [C x DVS]
-  using MMg = BlockMM<C, C, kBDVS>;    // [C x DVS] @ [DVS x C]
-  using MMd = BlockMM<C, DK, kBDVS>;   // [C x DVS] @ [DVS x DK]
-  using MMu = BlockMM<DK, kBDVS, C>;   // [DK x C] @ [C x DVS]
+  using MMk = BlockMM<C, kBDVS, DK, kScanThreads>;   // [C x DK] @ [DK x DVS]
+  using MMc = BlockMM<C, kBDVS, C, kScanThreads>;    // [C x C] @ [C x DVS]
+  using MMg = BlockMM<C, C, kBDVS, kScanThreads>;    // [C x DVS] @ [DVS x C]
+  using MMd = BlockMM<C, DK, kBDVS, kScanThreads>;   // [C x DVS] @ [DVS x DK]
+  using MMu = BlockMM<DK, kBDVS, C, kScanThreads>;   // [DK x C] @ [C x DVS]
   const int col = MMk::col();
 
-  for (int e = tid; e < DK * kBDVS; e += kThreads) {
+  for (int e = tid; e < DK * kBDVS; e += kScanThreads) {
     const int i = e / kBDVS, jj = e % kBDVS;
     dS[i * LDV + jj] = p.dST ? p.dST[sbase + (size_t)i * DV + j0 + jj] : 0.f;
     dR[i * LDV + jj] = p.dRT ? p.dRT[sbase + (size_t)i * DV + j0 + jj] : 0.f;
@@ -126,7 +127,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     const float *rec = p.f.ws + chunk * kRecFloats;
     float *acc = p.acc + chunk * L::FLOATS;
     __syncthreads();
-    for (int e = tid; e < C * DK; e += kThreads) {
+    for (int e = tid; e < C * DK; e += kScanThreads) {
       const int t = e / DK, d = e % DK;
       float kv = 0.f, qv = 0.f;
       if (t < n) {
@@ -137,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       Ks[t * LDK + d] = kv;
       Qs[t * LDK + d] = qv;
     }
-    for (int e = tid; e < C * kBDVS; e += kThreads) {
+    for (int e = tid; e < C * kBDVS; e += kScanThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
       float vv = 0.f, dd = 0.f;
       if (t < n) {
@@ -148,13 +149,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       Vs[t * LDV + jj] = vv;
       dOs[t * LDV + jj] = dd;
     }
-    for (int e = tid; e < DK * kBDVS; e += kThreads) {
+    for (int e = tid; e < DK * kBDVS; e += kScanThreads) {
       const int i = e / kBDVS, jj = e % kBDVS;
       const size_t off = chunk * DK * DV + (size_t)i * DV + j0 + jj;
       S0[i * LDV + jj] = p.Sc[off];
       R0[i * LDV + jj] = p.Rc[off];
     }
-    for (int e = tid; e < 6 * C; e += kThreads) {
+    for (int e = tid; e < 6 * C; e += kScanThreads) {
       vec[e] = rec[OFF_VEC + e];
       red[e] = 0.f;
     }
@@ -182,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     }
     const float *E = Vs;
     if (RDNV) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TB + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, C, 1, T1, LDV, 1, a1);
@@ -191,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       E = Es;
     }
     __syncthreads();
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_AP + e];
     __syncthreads();
     {
       float a1[MMc::RPT];
@@ -208,7 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     }
     __syncthreads();
     if (rdn_aux) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, C, 1, T1, LDV, 1, a1);
@@ -216,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       for (int i = 0; i < MMc::RPT; ++i) E2[MMc::row(i) * LDV + col] = a1[i];
       __syncthreads();
     }
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_M2 + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_M2 + e];
     __syncthreads();
     {  // Oa -> T2, dOa -> T3, row sums d(gamma)_out and dGam
       float a1[MMc::RPT];
@@ -259,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     __syncthreads();
     const float *dRv = T1;
     if (rdn_aux) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, 1, C, T1, LDV, 1, a1);  // dX2 = Tg^T dE2
@@ -282,7 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       dRv = T2;
     }
     // T3 <- diag(wR) E2 for dK += diag(wR) E2 dR^T
-    for (int e = tid; e < C * kBDVS; e += kThreads) {
+    for (int e = tid; e < C * kBDVS; e += kScanThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
       T3[t * LDV + jj] = wR[t] * E2[t * LDV + jj];
     }
@@ -299,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       MMd::run(QR, LDV, 1, R0, 1, LDV, dQacc);
       float s = 0.f;
       if (!stl)
-        for (int e = tid; e < DK * kBDVS; e += kThreads) {
+        for (int e = tid; e < DK * kBDVS; e += kScanThreads) {
           const int i = e / kBDVS, jj = e % kBDVS;
           s += dR[i * LDV + jj] * R0[i * LDV + jj];
         }
@@ -318,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       }
     }
     // clip: dV = dRv * [|x| <= c] into T3 (dP = -dV; tanh: times 1 - (r/c)^2)
-    for (int e = tid; e < C * kBDVS; e += kThreads) {
+    for (int e = tid; e < C * kBDVS; e += kScanThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
       T3[t * LDV + jj] = dRv[t * LDV + jj] * resid_grad(XR[t * LDV + jj], clip, tnh);
     }
@@ -338,12 +339,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
         }
       }
     }
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_MQ + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_MQ + e];
     __syncthreads();
     float de[MMc::RPT];
     MMc::run(CC, 1, C, dOs, LDV, 1, de);  // Mq^T dO
     __syncthreads();
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_AP + e];
     __syncthreads();
     {
       float a1[MMc::RPT], kd[MMk::RPT];
@@ -366,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
     }
     __syncthreads();
     if (RDNV) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TB + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, 1, C, T1, LDV, 1, a1);  // dX = Tb^T dE
@@ -388,13 +389,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
         if (ii < t) atomicAdd(&acc[L::DAB + t * C + ii], -g1[i]);
       }
     } else {
-      for (int e = tid; e < C * kBDVS; e += kThreads) {
+      for (int e = tid; e < C * kBDVS; e += kScanThreads) {
         const int t = e / kBDVS, jj = e % kBDVS;
         T3[t * LDV + jj] += T1[t * LDV + jj];  // dV += dE
       }
     }
     // XR <- diag(wS) E for dK += diag(wS) E dS^T
-    for (int e = tid; e < C * kBDVS; e += kThreads) {
+    for (int e = tid; e < C * kBDVS; e += kScanThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
       XR[t * LDV + jj] = wS[t] * E[t * LDV + jj];
     }
@@ -411,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
 #pragma unroll
       for (int i = 0; i < MMd::RPT; ++i) dQacc[i] += g1[i];
       float s = 0.f;
-      for (int e = tid; e < DK * kBDVS; e += kThreads) {
+      for (int e = tid; e < DK * kBDVS; e += kScanThreads) {
         const int i = e / kBDVS, jj = e % kBDVS;
         s += dS[i * LDV + jj] * S0[i * LDV + jj];
       }
@@ -435,15 +436,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
       atomicAdd(&acc[L::DKo + t * DK + d], dKacc[i]);
       atomicAdd(&acc[L::DQo + t * DK + d], dQacc[i]);
     }
-    for (int e = tid; e < C * kBDVS; e += kThreads) {
+    for (int e = tid; e < C * kBDVS; e += kScanThreads) {
       const int t = e / kBDVS, jj = e % kBDVS;
       if (t < n) dv[((size_t)(tok0 + t0 + t) * H + h) * DV + j0 + jj] = from_f32<InT>(T3[t * LDV + jj]);
     }
     __syncthreads();
-    for (int e = tid; e < 5 * C + 1; e += kThreads) atomicAdd(&acc[L::VEC + e], red[e]);
+    for (int e = tid; e < 5 * C + 1; e += kScanThreads) atomicAdd(&acc[L::VEC + e], red[e]);
   }
   __syncthreads();
-  for (int e = tid; e < DK * kBDVS; e += kThreads) {
+  for (int e = tid; e < DK * kBDVS; e += kScanThreads) {
     const int i = e / kBDVS, jj = e % kBDVS;
     if (p.dS0) p.dS0[sbase + (size_t)i * DV + j0 + jj] = dS[i * LDV + jj];
     if (p.dR0) p.dR0[sbase + (size_t)i * DV + j0 + jj] = dR[i * LDV + jj];
@@ -451,13 +452,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_scan_kernel(BwdParams p) {
 }
 
 // ---------------------------------------------------------------- kernel 2
-// One CTA per chunk.  Each warp owns 8 rows t of the C x C gradients; lane l
+// One CTA per chunk.  Each warp owns 4 rows t of the C x C gradients; lane l
 // handles columns l and l + 32.  Row sums (d cum_t, d cprev_t) are reduced
 // with shuffles; column sums (d cum_i, dbeta_i, dgamma_i) go through
 // shared-memory tiles and a column pass, so no shared-memory atomics are
 // contended.
 template <int DK, bool RDNV, typename InT>
-__global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
+__global__ void __launch_bounds__(kScanThreads, 1) bwd_finish_kernel(BwdParams p) {
   constexpr int LDK = DK + 1;
   constexpr int LDC = C + 1;
   using L = Acc<DK>;
@@ -498,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   const bool plain = p.f.mods & RDN_FLAG_PLAIN_COMBINE;
   const bool stl = p.f.mods & RDN_FLAG_STATELESS_AUX;
 
-  for (int e = tid; e < C * DK; e += kThreads) {
+  for (int e = tid; e < C * DK; e += kScanThreads) {
     const int t = e / DK, d = e % DK;
     float kv = 0.f, qv = 0.f;
     if (t < n) {
@@ -541,7 +542,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     cprev[32 + lane] = b2 - gg[32 + lane];
   }
   {
-    using MM = BlockMM<C, C, DK>;
+    using MM = BlockMM<C, C, DK, kScanThreads>;
     float a[MM::RPT];
     MM::run(Ks, LDK, 1, Ks, 1, LDK, a);
 #pragma unroll
@@ -552,8 +553,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   }
   __syncthreads();
   // ---- row pass over the C x C gradients
-  for (int rr = 0; rr < C / 8; ++rr) {
-    const int t = warp * (C / 8) + rr;
+  constexpr int kRowsPerWarp = C / (kScanThreads / 32);
+  for (int rr = 0; rr < kRowsPerWarp; ++rr) {
+    const int t = warp * kRowsPerWarp + rr;
     float rowc = 0.f, rowp = 0.f;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -652,7 +654,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
     if (lane == 0) dcum[C - 1] += s + acc[L::VEC + L::V_DGAMC] * expf(cC);
   }
   // symmetrise: dK gets (dKK + dKK^T) K
-  for (int e = tid; e < C * C; e += kThreads) {
+  for (int e = tid; e < C * C; e += kScanThreads) {
     const int t = e / C, i = e % C;
     if (i < t) {
       const float s2 = dKK[t * LDC + i] + dKK[i * LDC + t];
@@ -664,7 +666,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_finish_kernel(BwdParams p) {
   }
   __syncthreads();
   {
-    using MM = BlockMM<C, DK, C>;
+    using MM = BlockMM<C, DK, C, kScanThreads>;
     float a1[MM::RPT], a2[MM::RPT], a3[MM::RPT];
     MM::run(dKK, LDC, 1, Ks, LDK, 1, a1);   // (dKK + dKK^T) K
     MM::run(dQK, 1, LDC, Qs, LDK, 1, a2);   // dQK^T Q
@@ -732,9 +734,9 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
   if ((e = cudaFuncSetAttribute(fin, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)finish_smem<DK>())) != cudaSuccess)
     return e;
-  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.nseq * p.f.H, DK / kBDVS), kThreads, scan_smem<DK>(), s>>>(p));
+  RDN_LAUNCH("bwd_scan", s, scan<<<dim3(p.f.nseq * p.f.H, DK / kBDVS), kScanThreads, scan_smem<DK>(), s>>>(p));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  RDN_LAUNCH("bwd_finish", s, fin<<<(unsigned)p.f.nrec, kThreads, finish_smem<DK>(), s>>>(p));
+  RDN_LAUNCH("bwd_finish", s, fin<<<(unsigned)p.f.nrec, kScanThreads, finish_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 

@@ -28,15 +28,15 @@ constexpr int kRecFloats = OFF_VEC + 6 * C;
 constexpr int IMG_TB = 0, IMG_APMQ = 16384, IMG_TG = 49152, IMG_M2 = 65536;
 static_assert(IMG_M2 + 16384 == OFF_VEC * 4, "image fills the matrix part of the record");
 
-// Block-level fp32 product over shared memory: the calling thread gets
-// acc[i] = sum_k A(m_i, k) B(k, n) for n = tid % N and m_i = tid / N + i * (256 / N).
+// Block-level fp32 product over shared memory (NT threads): the calling thread
+// gets acc[i] = sum_k A(m_i, k) B(k, n) for n = tid % N and m_i = tid / N + i * (NT / N).
 // A(m,k) = A[m*a_m + k*a_k], B(k,n) = B[k*b_k + n*b_n].  With N >= 32 the lanes
 // of a warp share m, so A reads are broadcasts.
-template <int M, int N, int K>
+template <int M, int N, int K, int NT = kThreads>
 struct BlockMM {
-  static constexpr int RG = kThreads / N;
+  static constexpr int RG = NT / N;
   static constexpr int RPT = M / RG;
-  static_assert(kThreads % N == 0 && M % RG == 0, "tile");
+  static_assert(NT % N == 0 && M % RG == 0, "tile");
   __device__ static __forceinline__ void run(const float *A, int a_m, int a_k, const float *B,
                                              int b_k, int b_n, float (&acc)[RPT]) {
     const int n = threadIdx.x % N, rg = threadIdx.x / N;

@@ -201,8 +201,10 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
 }
 
 // ---------------------------------------------------------------- kernel 2
+constexpr int kScanThreads = 512;  // threads of a scan CTA (latency bound: 16 warps)
+
 template <int DK, bool RDNV, typename InT>
-__global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
+__global__ void __launch_bounds__(kScanThreads, 1) chunk_scan_kernel(FwdParams p) {
   constexpr int DV = DK;
   extern __shared__ float sm[];
   float *Ks = sm;                 // [C][DK]
@@ -236,7 +238,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
   const bool rdn_aux = RDNV && !stl;  // the auxiliary pass runs the delta rule
 
   const size_t sbase = (size_t)bh * DK * DV;
-  for (int e = tid; e < DK * kDVS; e += kThreads) {
+  for (int e = tid; e < DK * kDVS; e += kScanThreads) {
     const int i = e / kDVS, jj = e % kDVS;
     Ss[e] = p.S0 ? p.S0[sbase + (size_t)i * DV + j0 + jj] : 0.f;
     Rs[e] = p.R0 ? p.R0[sbase + (size_t)i * DV + j0 + jj] : 0.f;
@@ -250,13 +252,13 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     if (p.S_chunks) {
       float *sc = p.S_chunks + (size_t)(sp.rbase + c) * DK * DV;
       float *rc = p.R_chunks + (size_t)(sp.rbase + c) * DK * DV;
-      for (int e = tid; e < DK * kDVS; e += kThreads) {
+      for (int e = tid; e < DK * kDVS; e += kScanThreads) {
         const int i = e / kDVS, jj = e % kDVS;
         sc[(size_t)i * DV + j0 + jj] = Ss[e];
         rc[(size_t)i * DV + j0 + jj] = Rs[e];
       }
     }
-    for (int e = tid; e < C * DK; e += kThreads) {
+    for (int e = tid; e < C * DK; e += kScanThreads) {
       const int t = e / DK, d = e % DK;
       float kv = 0.f, qv = 0.f;
       if (t < n) {
@@ -267,19 +269,19 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       Ks[e] = kv;
       Qs[e] = qv;
     }
-    for (int e = tid; e < C * kDVS; e += kThreads) {
+    for (int e = tid; e < C * kDVS; e += kScanThreads) {
       const int t = e / kDVS, jj = e % kDVS;
       Vs[e] = t < n ? to_f32(v[((size_t)(sp.tok0 + t0 + t) * p.H + h) * DV + j0 + jj]) : 0.f;
     }
-    for (int e = tid; e < 6 * C; e += kThreads) vec[e] = rec[OFF_VEC + e];
+    for (int e = tid; e < 6 * C; e += kScanThreads) vec[e] = rec[OFF_VEC + e];
     __syncthreads();
     const float *Gam = vec + V_GAM, *Gprev = vec + V_GPREV;
     const float *wS = vec + V_WS, *wR = vec + V_WR;
     const float GamC = vec[V_GAMC];
 
-    using MMk = BlockMM<C, kDVS, DK>;  // [C x DK] @ [DK x DVS]
-    using MMc = BlockMM<C, kDVS, C>;   // [C x C] @ [C x DVS]
-    using MMu = BlockMM<DK, kDVS, C>;  // [DK x C] @ [C x DVS]
+    using MMk = BlockMM<C, kDVS, DK, kScanThreads>;  // [C x DK] @ [DK x DVS]
+    using MMc = BlockMM<C, kDVS, C, kScanThreads>;   // [C x C] @ [C x DVS]
+    using MMu = BlockMM<DK, kDVS, C, kScanThreads>;  // [DK x C] @ [C x DVS]
     const int col = MMk::col();
     {
       float a1[MMk::RPT], a2[MMk::RPT];
@@ -295,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     }
     const float *E = Vs;
     if (RDNV) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TB + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TB + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, C, 1, Ws, kDVS, 1, a1);
@@ -304,7 +306,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       E = Es;
     }
     __syncthreads();
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_AP + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_AP + e];
     __syncthreads();
     {
       float a1[MMc::RPT];
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       }
     }
     __syncthreads();
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_MQ + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_MQ + e];
     __syncthreads();
     {
       float a1[MMc::RPT];
@@ -330,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       }
     }
     // S_C = Gam_C S0 + K^T diag(wS) E   (W = wS * E)
-    for (int e = tid; e < C * kDVS; e += kThreads) Ws[e] = wS[e / kDVS] * E[e];
+    for (int e = tid; e < C * kDVS; e += kScanThreads) Ws[e] = wS[e / kDVS] * E[e];
     __syncthreads();
     {
       float a1[MMu::RPT];
@@ -356,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     }
     const float *E2 = Ps;
     if (rdn_aux) {
-      for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_TG + e];
+      for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_TG + e];
       __syncthreads();
       float a1[MMc::RPT];
       MMc::run(CC, C, 1, Ws, kDVS, 1, a1);
@@ -365,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       E2 = Es;
     }
     __syncthreads();
-    for (int e = tid; e < C * C; e += kThreads) CC[e] = rec[OFF_M2 + e];
+    for (int e = tid; e < C * C; e += kScanThreads) CC[e] = rec[OFF_M2 + e];
     __syncthreads();
     {
       float a1[MMc::RPT];
@@ -382,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
       }
     }
     // R_C = Gam_C R0 + K^T diag(wR) E2
-    for (int e = tid; e < C * kDVS; e += kThreads) Ws[e] = wR[e / kDVS] * E2[e];
+    for (int e = tid; e < C * kDVS; e += kScanThreads) Ws[e] = wR[e / kDVS] * E2[e];
     __syncthreads();
     {
       float a1[MMu::RPT];
@@ -395,7 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_scan_kernel(FwdParams p) {
     }
   }
   __syncthreads();
-  for (int e = tid; e < DK * kDVS; e += kThreads) {
+  for (int e = tid; e < DK * kDVS; e += kScanThreads) {
     const int i = e / kDVS, jj = e % kDVS;
     if (p.ST) p.ST[sbase + (size_t)i * DV + j0 + jj] = Ss[e];
     if (p.RT) p.RT[sbase + (size_t)i * DV + j0 + jj] = Rs[e];
@@ -434,7 +436,7 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
     }
   }
   if (do_scan)
-    RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.nseq * p.H, DK / kDVS), kThreads, scan_smem<DK>(), s>>>(p));
+    RDN_LAUNCH("chunk_scan", s, scan<<<dim3(p.nseq * p.H, DK / kDVS), kScanThreads, scan_smem<DK>(), s>>>(p));
   return cudaGetLastError();
 }
 
