@@ -519,6 +519,43 @@ def run_ours(args):
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr
 
+    # ---- forward-only workloads (RDN forward, B=8 T=2048, and the long
+    # context B=2 T=16384 with initial states and final states returned):
+    # tokens/s and the forward's algorithmic flop rate against the tensor peak
+    fwd = None
+    if not args.no_forward:
+        fwd = {}
+        for wname in ("rdn_fwd_bf16_B8H16T2048D128", "rdn_fwd_bf16_B2H16T16384D128_state"):
+            wf = WORKLOADS[wname]
+            xf = make_workload_inputs(wf, device=dev, device_rng=True, seed=rank)
+            of = torch.empty(wf.B, wf.T, wf.H, wf.D, dtype=torch.bfloat16, device=dev)
+            wsff = torch.empty(rdn.workspace_bytes("rdn_fwd", wf.B, wf.T, wf.H, wf.D),
+                               dtype=torch.uint8, device=dev)
+            ret = wf.nonzero_state
+
+            def fwd_step():
+                rdn.rdn_fwd(*(xf[n] for n in names), clip=wf.clip, S0=xf["S0"], R0=xf["R0"],
+                            return_final_state=ret, out=of, workspace=wsff)
+
+            for _ in range(3):
+                fwd_step()
+            torch.cuda.synchronize()
+            barrier(dist)
+            fsteps = max(3, args.steps)
+            e0.record(stream)
+            for _ in range(fsteps):
+                fwd_step()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            barrier(dist)
+            tfw, fvals = aggregate(dist, e0.elapsed_time(e1), wf.B * wf.T * fsteps)
+            ms_f = tfw / fsteps
+            tfl = fl["fwd"] * wf.B * wf.T * wf.H / (ms_f * 1e-3) / 1e12
+            fwd[wname] = {"value": fvals, "unit": "tokens/s", "ms_per_step": ms_f,
+                          "steps": fsteps, "tflops": tfl, "frac_of_bf16_peak": tfl / peak,
+                          "states": "S0, R0 in, S_T, R_T out" if ret else "zero, not returned"}
+            del xf, of, wsff
+
     # ---- the paper's variants (variant_flags, fp32 chunk kernels) on the
     # bench workload: RDN fwd+bwd with each flag, as the RDN step above
     var = None
@@ -660,7 +697,7 @@ def run_ours(args):
                                 "share": t / sum(v[1] for v in kern.values())}
                             for k, (n, t, m) in kern.items()},
                 "clocks": clk.summary(), "decode": dec, "rla": rla, "prologue": pro,
-                "varlen": vl, "variants": var}
+                "varlen": vl, "variants": var, "forward": fwd}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
@@ -680,6 +717,7 @@ def main(argv=None):
     ap.add_argument("--no-prologue", action="store_true")
     ap.add_argument("--no-varlen", action="store_true")
     ap.add_argument("--no-variants", action="store_true")
+    ap.add_argument("--no-forward", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")
