@@ -50,12 +50,14 @@ C = 64
 #   (the tensor-core bwd_post does the last two; the SIMT path splits them
 #   into bwd_scan and bwd_finish).  Recomputation of forward pieces is not
 #   algorithmic work (counted 0).
+#   The same work with every C x C x d product counted as a dense tile (the
+#   triangular ones at full size): forward + 7 C d per token-head.
 def flops_per_token_head(d=128, c=C):
     scan = 12 * d * d + 5 * c * d
     prep = 2 * c * d + (4.0 / 3.0) * c * c
     return dict(fwd=scan + prep, fwd_scan=scan, fwd_prep=prep, bwd_scan=2 * scan,
                 bwd_chain=scan, bwd_post=scan + 2 * prep, bwd_finish=2 * prep, recompute=0.0,
-                step=3 * (scan + prep))
+                step=3 * (scan + prep), step_dense_tiles=3 * (scan + prep + 7 * c * d))
 
 
 # kernel name (as recorded by the library) -> algorithmic flop per token-head
@@ -330,7 +332,7 @@ def run_ours(args):
     dist = init_dist(ws)
     torch.cuda.set_device(local)
     import paper_2509_25223_gb300 as rdn
-    from rdn_synthetic import WORKLOADS, make_decode_inputs, make_workload_inputs
+    from rdn_synthetic import WORKLOADS, make_decode_inputs, make_workload_inputs, packed_lengths
 
     rdn.library()  # fails loudly when the CUDA library is missing
     w = _workload(args)
@@ -390,6 +392,7 @@ def run_ours(args):
             "peak_kind": f"bf16 dense, {peaks['source']} sustained (kernel timed inside a long step)",
             "algorithmic_flop_per_launch": dom_flop, "mean_launch_ms": dom_mean}
     step_tflops = fl["step"] * token_heads / (ms_per_step * 1e-3) / 1e12
+    step_tflops_dense = fl["step_dense_tiles"] * token_heads / (ms_per_step * 1e-3) / 1e12
 
     # ---- end to end through the public API: pinned host in, host out.  Each
     # step copies all its inputs in from pinned host memory and reads its
@@ -592,13 +595,7 @@ def run_ours(args):
     # cut to fill the row), RDN fwd+bwd exactly as the step above
     vl = None
     if not args.no_varlen:
-        rng = np.random.default_rng(1234)
-        lens, tot = [], 0
-        while tot < B * T:
-            L = int(np.exp(rng.uniform(np.log(64), np.log(8192))))
-            L = min(L, B * T - tot)
-            lens.append(L)
-            tot += L
+        lens = packed_lengths(B * T)
         cu = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device=dev)
         N = len(lens)
         xv = {n: x[n].view(1, B * T, *x[n].shape[2:]) for n in names + ("dO",)}
@@ -685,6 +682,8 @@ def run_ours(args):
                 "dtype": "bf16", "data": "synthetic", "config": _config(w),
                 "roofline": roof, "step_tflops": step_tflops,
                 "step_frac_of_bf16_peak": step_tflops / peak,
+                "step_tflops_dense_tiles": step_tflops_dense,
+                "step_frac_of_bf16_peak_dense_tiles": step_tflops_dense / peak,
                 "cpu_baseline": cpu,
                 "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                         "d2h_bytes_per_step": d2h, "steps": e2e_steps,

@@ -128,3 +128,17 @@ def make_decode_inputs(N, H, D, steps=1, seed=0, device="cpu", device_rng=False,
     td = TORCH_DTYPE[dtype]
     out = dict(S=S, R=R, q=q.to(td), k=k.to(td), v=v.to(td), g=g, beta=beta, gamma=gamma)
     return {n: t.to(device).contiguous() for n, t in out.items()}
+
+
+def packed_lengths(total, lo=64, hi=8192, seed=1234):
+    """Sequence lengths for a packed batch of `total` tokens: log-uniform in
+    [lo, hi] from a seeded numpy generator, the last one cut to fill the row
+    (a pretraining-style mix of short and long documents)."""
+    import numpy as np
+    rng = np.random.default_rng(seed)
+    lens, tot = [], 0
+    while tot < total:
+        L = min(int(np.exp(rng.uniform(np.log(lo), np.log(hi)))), total - tot)
+        lens.append(L)
+        tot += L
+    return lens

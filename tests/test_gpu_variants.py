@@ -136,3 +136,34 @@ def test_variant_packed_sequences_and_tied_gates():
         assert_close(d["dbeta"][:, t0:t1], ref["dbeta"] + ref["dgamma"], "bf16", f"dbeta[{s}]")
         assert_close(d["dS0"][s:s + 1], ref["dS0"], "bf16", f"dS0[{s}]")
         assert_close(d["dR0"][s:s + 1], ref["dR0"], "bf16", f"dR0[{s}]")
+
+
+@pytest.mark.parametrize("flags", [rdn.DECAYED_RESIDUAL | rdn.PLAIN_COMBINE | rdn.STATELESS_AUX,
+                                   rdn.TANH_RESIDUAL])
+def test_variant_bench_shape_sampled(flags):
+    """RDN fwd + bwd with variant flags at the bench's sequence length and
+    head count (B = 2, T = 4096, H = 16, d = 128, bf16), two sampled heads
+    against the oracle."""
+    m = _mods(flags)
+    x = make_inputs(2, 4096, 16, 128, dtype="bf16", with_grad_out=True, device="cuda", seed=8)
+    picks = [(0, 2), (1, 13)]
+    for b, h in picks:
+        sl = {n: as64(x[n][b:b + 1, :, h:h + 1]) for n in NAMES}
+        v2, _ = oracle.clip_margin_condition(oracle.RDN, *(sl[n] for n in NAMES), 1.0,
+                                             margin=1e-2, quant="bf16", mods=m)
+        x["v"][b, :, h] = torch.from_numpy(v2[0, :, 0]).to(x["v"].dtype).cuda()
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, return_chunk_states=True,
+                                    variant_flags=flags)
+    d = rdn.rdn_bwd(*(x[n] for n in NAMES), x["dO"], clip=1.0, S_chunks=Sc, R_chunks=Rc,
+                    variant_flags=flags)
+    torch.cuda.synchronize()
+    for b, h in picks:
+        sl = {n: as64(x[n][b:b + 1, :, h:h + 1]) for n in NAMES + ("dO",)}
+        oref, Sref, Rref = oracle.fwd(oracle.RDN, *(sl[n] for n in NAMES), 1.0, mods=m)
+        assert_close(o[b:b + 1, :, h:h + 1], oref, "bf16", f"o[{b},{h}]")
+        assert_close(ST[b:b + 1, h:h + 1], Sref, "bf16", f"ST[{b},{h}]")
+        assert_close(RT[b:b + 1, h:h + 1], Rref, "bf16", f"RT[{b},{h}]")
+        ref = oracle.bwd(oracle.RDN, *(sl[n] for n in NAMES), 1.0, None, None, sl["dO"], mods=m)
+        for name in ("dq", "dk", "dv", "dg", "dbeta", "dgamma"):
+            assert_close(d[name][b:b + 1, :, h:h + 1], ref[name], "bf16", f"{name}[{b},{h}]")
+        assert_close(d["dS0"][b:b + 1, h:h + 1], ref["dS0"], "bf16", f"dS0[{b},{h}]")

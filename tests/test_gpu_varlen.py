@@ -199,3 +199,43 @@ def test_packed_table_clamped():
     o2, ST2, RT2 = _fwd("rdn", x, 1.0)
     assert torch.equal(o, o2) and torch.equal(ST, ST2) and torch.equal(RT, RT2)
     x["cu"] = good
+
+
+def test_packed_bench_shape_sampled():
+    """The bench's packed workload (32,768 tokens x 16 heads, d = 128, 15
+    log-uniform lengths), fwd + bwd as the bench runs it (chunk states and
+    saved intermediates reused); the shortest, a middle and the longest
+    sequence checked against the oracle on one head each."""
+    from rdn_synthetic import packed_lengths
+    lens = packed_lengths(32768)
+    T, H, D = sum(lens), 16, 128
+    x = make_inputs(1, T, H, D, dtype="bf16", with_grad_out=True, device="cuda", seed=2)
+    cu_h = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    x["cu"], x["cu_host"] = torch.from_numpy(cu_h).cuda(), cu_h
+    order = np.argsort(lens)
+    picks = [(int(order[0]), 3), (int(order[len(lens) // 2]), 9), (int(order[-1]), 14)]
+    for s, h in picks:  # margin on the sampled heads' clip decisions
+        t0, t1 = int(cu_h[s]), int(cu_h[s + 1])
+        sl = {n: as64(x[n][:, t0:t1, h:h + 1]) for n in NAMES}
+        v2, _ = oracle.clip_margin_condition(oracle.RDN, *(sl[n] for n in NAMES), 1.0,
+                                             margin=MARGIN, quant="bf16")
+        x["v"][0, t0:t1, h] = torch.from_numpy(v2[0, :, 0]).to(x["v"].dtype).cuda()
+    ws = torch.empty(rdn.workspace_bytes("rdn_fwd", 1, T, H, D, save_for_bwd=True,
+                                         cu_seqlens=x["cu"]), dtype=torch.uint8, device="cuda")
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, cu_seqlens=x["cu"],
+                                    return_chunk_states=True, workspace=ws, save_for_bwd=True)
+    d = rdn.rdn_bwd(*(x[n] for n in NAMES), x["dO"], clip=1.0, cu_seqlens=x["cu"], S_chunks=Sc,
+                    R_chunks=Rc, fwd_workspace=ws, fwd_saved=True)
+    torch.cuda.synchronize()
+    for s, h in picks:
+        t0, t1 = int(cu_h[s]), int(cu_h[s + 1])
+        sl = {n: as64(x[n][:, t0:t1, h:h + 1]) for n in NAMES + ("dO",)}
+        oref, Sref, Rref = oracle.fwd(oracle.RDN, *(sl[n] for n in NAMES), 1.0)
+        assert_close(o[:, t0:t1, h:h + 1], oref, "bf16", f"o[{s},{h}]")
+        assert_close(ST[s:s + 1, h:h + 1], Sref, "bf16", f"ST[{s},{h}]")
+        assert_close(RT[s:s + 1, h:h + 1], Rref, "bf16", f"RT[{s},{h}]")
+        ref = oracle.bwd(oracle.RDN, *(sl[n] for n in NAMES), 1.0, None, None, sl["dO"])
+        for name in GRADS:
+            assert_close(d[name][:, t0:t1, h:h + 1], ref[name], "bf16", f"{name}[{s},{h}]")
+        assert_close(d["dS0"][s:s + 1, h:h + 1], ref["dS0"], "bf16", f"dS0[{s},{h}]")
+        assert_close(d["dR0"][s:s + 1, h:h + 1], ref["dR0"], "bf16", f"dR0[{s},{h}]")
