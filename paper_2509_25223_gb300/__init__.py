@@ -271,12 +271,16 @@ def qk_prologue(q, k=None, eps=1e-12, out=None):
     return yq, yk
 
 
-def qk_prologue_bwd(q, k, dyq, dyk=None, eps=1e-12):
+def qk_prologue_bwd(q, k, dyq, dyk=None, eps=1e-12, out=None):
     """Gradients w.r.t. the pre-activation q, k of <dyq, q'> + <dyk, k'>
-    (q', k' from qk_prologue; recomputed from q, k).  k / dyk may be None."""
+    (q', k' from qk_prologue; recomputed from q, k).  k / dyk may be None;
+    out: (dq, dk) buffers to write into."""
     lib = _abi.load()
-    dq = torch.empty_like(q)
-    dk = torch.empty_like(k) if k is not None else None
+    if out is not None:
+        dq, dk = out
+    else:
+        dq = torch.empty_like(q)
+        dk = torch.empty_like(k) if k is not None else None
     a = _prologue_args(q, k, eps)
     a.dy[0], a.dy[1] = _ptr(dyq), _ptr(dyk)
     a.dx[0], a.dx[1] = _ptr(dq), _ptr(dk)

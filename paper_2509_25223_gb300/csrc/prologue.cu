@@ -6,13 +6,15 @@
 //     dx = du * sigmoid(x) (1 + x (1 - sigmoid(x))).
 //
 // Memory-bound (read x, write y; the backward reads x and dy and writes dx,
-// recomputing u and the norm instead of saving them).  One warp per row, each
-// lane holding D/32 consecutive elements (one 4- to 16-byte access, kept
-// packed in registers until used, which keeps four rows in flight per warp
-// at full occupancy: 70-77 % of the measured HBM bandwidth), the
-// row's norm and <y, dy> reduced with shuffles; the q and k rows form one
-// grid-stride range.  Loads and stores are streaming (every element is
-// touched once).
+// recomputing u and the norm instead of saving them).  In the forward each
+// lane holds 16 consecutive bytes of a row (one 16-byte access, kept packed
+// in registers until used), so a row takes D * size / 16 lanes and a warp has
+// 2 to 8 rows per access; the backward, which holds x and dy, gives a row a
+// whole warp (D / 32 elements per lane, fewer registers, more warps).  Four
+// accesses are in flight per warp; the row's norm and <y, dy> are reduced
+// with shuffles within its lanes; q and k are the two rows of the grid
+// (blockIdx.y), each a grid-stride range.  Loads and stores are streaming
+// (every element is touched once).
 #include "common.cuh"
 
 namespace rdn {
@@ -64,6 +66,29 @@ struct Vec<__nv_bfloat16, 4> {
   }
 };
 template <>
+struct Vec<__nv_bfloat16, 8> {
+  using Raw = uint4;
+  __device__ static Raw ldr(const __nv_bfloat16 *p) { return __ldcs(reinterpret_cast<const uint4 *>(p)); }
+  __device__ static void unpack(const Raw &a, float (&v)[8]) {
+    const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&w[i]);
+      v[2 * i] = __low2float(b);
+      v[2 * i + 1] = __high2float(b);
+    }
+  }
+  __device__ static void st(__nv_bfloat16 *p, const float (&v)[8]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 b = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+      w[i] = *reinterpret_cast<const uint32_t *>(&b);
+    }
+    __stcs(reinterpret_cast<uint4 *>(p), make_uint4(w[0], w[1], w[2], w[3]));
+  }
+};
+template <>
 struct Vec<__nv_bfloat16, 2> {
   using Raw = unsigned;
   __device__ static Raw ldr(const __nv_bfloat16 *p) { return __ldcs(reinterpret_cast<const unsigned *>(p)); }
@@ -77,43 +102,53 @@ struct Vec<__nv_bfloat16, 2> {
   }
 };
 
-__device__ __forceinline__ float warp_sum(float v) {
+// sum over the LPR lanes of a row (aligned groups of LPR lanes)
+template <int LPR>
+__device__ __forceinline__ float row_sum(float v) {
 #pragma unroll
-  for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  for (int off = LPR / 2; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
   return v;
 }
 
 struct ProP {
-  long long rows, total;  // rows per tensor; rows of all tensors
+  long long rows;  // rows per tensor (blockIdx.y picks the tensor: q, then k)
   float eps;
-  const void *x0, *x1, *dy0, *dy1;
-  void *o0, *o1;  // y (forward) or dx (backward)
+  const void *x[2], *dy[2];
+  void *o[2];  // y (forward) or dx (backward)
 };
 
 template <typename InT, int D, bool BWD>
 __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
-  constexpr int E = D / 32;
+  // elements per lane: one 16-byte access (the backward, which holds x and
+  // dy, one warp per row: D / 32 elements per lane, fewer registers)
+  constexpr int E = BWD ? D / 32 : 16 / (int)sizeof(InT);
+  constexpr int LPR = D / E;                 // lanes per row
+  constexpr int RPW = 32 / LPR;              // rows per warp access
+  constexpr int ROWS = kRowsInFlight * RPW;  // rows a warp has in flight
   using V = Vec<InT, E>;
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, sub = lane / LPR, li = lane % LPR;
   const long long warp = ((long long)blockIdx.x * kProThreads + threadIdx.x) >> 5;
   const long long nwarps = ((long long)gridDim.x * kProThreads) >> 5;
-  for (long long base = warp * kRowsInFlight; base < p.total; base += nwarps * kRowsInFlight) {
+  const InT *X = reinterpret_cast<const InT *>(p.x[blockIdx.y]);
+  const InT *DY = reinterpret_cast<const InT *>(p.dy[blockIdx.y]);
+  InT *O = reinterpret_cast<InT *>(p.o[blockIdx.y]);
+  for (long long base = warp * ROWS; base < p.rows; base += nwarps * ROWS) {
     typename V::Raw xr[kRowsInFlight], gr[kRowsInFlight];  // packed until used
     // the loads of all rows first
 #pragma unroll
     for (int u = 0; u < kRowsInFlight; ++u) {
-      const long long r = base + u;
-      if (r < p.total) {
-        const bool second = r >= p.rows;
-        const size_t off = (size_t)(second ? r - p.rows : r) * D + lane * E;
-        xr[u] = V::ldr(reinterpret_cast<const InT *>(second ? p.x1 : p.x0) + off);
-        if (BWD) gr[u] = V::ldr(reinterpret_cast<const InT *>(second ? p.dy1 : p.dy0) + off);
+      const long long r = base + u * RPW + sub;
+      xr[u] = typename V::Raw{};
+      gr[u] = typename V::Raw{};
+      if (r < p.rows) {
+        const size_t off = (size_t)r * D + li * E;
+        xr[u] = V::ldr(X + off);
+        if (BWD) gr[u] = V::ldr(DY + off);
       }
     }
 #pragma unroll
     for (int u = 0; u < kRowsInFlight; ++u) {
-      const long long r = base + u;
-      if (r >= p.total) break;  // (uniform across the warp)
+      const long long r = base + u * RPW + sub;  // (rows past the end: computed, not stored)
       float x[E], g[E], s[E], uu[E], ss = 0.f;
       V::unpack(xr[u], x);
       if (BWD) V::unpack(gr[u], g);
@@ -123,7 +158,7 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
         uu[e] = x[e] * s[e];
         ss = fmaf(uu[e], uu[e], ss);
       }
-      const float n = sqrtf(warp_sum(ss));
+      const float n = sqrtf(row_sum<LPR>(ss));
       const float m = fmaxf(n, p.eps), inv = 1.f / m;
       float out[E];
       if (!BWD) {
@@ -133,7 +168,7 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
         float dot = 0.f;
 #pragma unroll
         for (int e = 0; e < E; ++e) dot = fmaf(uu[e] * inv, g[e], dot);
-        dot = warp_sum(dot);
+        dot = row_sum<LPR>(dot);
         const bool big = n > p.eps;
 #pragma unroll
         for (int e = 0; e < E; ++e) {
@@ -141,9 +176,7 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
           out[e] = du * s[e] * (1.f + x[e] * (1.f - s[e]));
         }
       }
-      const bool second = r >= p.rows;
-      const size_t off = (size_t)(second ? r - p.rows : r) * D + lane * E;
-      V::st(reinterpret_cast<InT *>(second ? p.o1 : p.o0) + off, out);
+      if (r < p.rows) V::st(O + (size_t)r * D + li * E, out);
     }
   }
 }
@@ -155,14 +188,16 @@ cudaError_t launch_t(const ProP &p, bool bwd, cudaStream_t s) {
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
     return e;
-  const long long warps = (p.total + kRowsInFlight - 1) / kRowsInFlight;
+  const int rows_per_warp = bwd ? kRowsInFlight : kRowsInFlight * 32 / (D * (int)sizeof(InT) / 16);
+  const int nt = p.x[1] ? 2 : 1;  // tensors: grid.y
+  const long long warps = (p.rows + rows_per_warp - 1) / rows_per_warp;
   const long long want = (warps + kProThreads / 32 - 1) / (kProThreads / 32);
   int occ = 0;  // a few waves of resident CTAs, grid-stride beyond
   e = bwd ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, prologue_kernel<InT, D, true>, kProThreads, 0)
           : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, prologue_kernel<InT, D, false>, kProThreads, 0);
   if (e != cudaSuccess) return e;
-  const long long cap = (long long)nsm * (occ > 0 ? occ : 1) * kWaves;
-  const unsigned grid = (unsigned)(want < cap ? want : cap);
+  const long long cap = ((long long)nsm * (occ > 0 ? occ : 1) * kWaves + nt - 1) / nt;
+  const dim3 grid((unsigned)(want < cap ? want : cap), nt);
   if (bwd)
     RDN_LAUNCH("qk_prologue_bwd", s, prologue_kernel<InT, D, true><<<grid, kProThreads, 0, s>>>(p));
   else
@@ -175,14 +210,12 @@ cudaError_t launch_t(const ProP &p, bool bwd, cudaStream_t s) {
 cudaError_t launch_prologue(const rdn_prologue_args &a, bool bwd, cudaStream_t s) {
   ProP p;
   p.rows = a.rows;
-  p.total = a.x[1] ? 2 * a.rows : a.rows;
   p.eps = a.eps;
-  p.x0 = a.x[0];
-  p.x1 = a.x[1];
-  p.dy0 = bwd ? a.dy[0] : nullptr;
-  p.dy1 = bwd ? a.dy[1] : nullptr;
-  p.o0 = bwd ? a.dx[0] : a.y[0];
-  p.o1 = bwd ? a.dx[1] : a.y[1];
+  for (int i = 0; i < 2; ++i) {
+    p.x[i] = a.x[i];
+    p.dy[i] = bwd ? a.dy[i] : nullptr;
+    p.o[i] = bwd ? a.dx[i] : a.y[i];
+  }
   if (a.dtype == RDN_BF16)
     return a.D == 128 ? launch_t<__nv_bfloat16, 128>(p, bwd, s) : launch_t<__nv_bfloat16, 64>(p, bwd, s);
   return a.D == 128 ? launch_t<float, 128>(p, bwd, s) : launch_t<float, 64>(p, bwd, s);
