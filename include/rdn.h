@@ -307,6 +307,16 @@ rdn_status_t rdn_decode_step(const rdn_decode_args *args, rdn_stream_t stream);
 /* Workspace sizes in bytes for the arguments' shapes (pointers ignored).
  * Return RDN_OK and set *bytes, or an error for invalid shapes. */
 rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
+/* Device-side failures.  A kernel whose bounded wait for its own copies or
+ * tensor-core work gives up (RDN_ERR_TIMEOUT), or that finds its shared
+ * memory misaligned (RDN_ERR_CUDA), records the code in a per-device status
+ * word, skips the rest of its work and exits, leaving the context usable;
+ * the outputs of that call are then invalid.  rdn_device_status waits for
+ * `stream`, returns in *status the code recorded since the previous query
+ * (RDN_OK if none) and clears it.  The word is shared by all streams of the
+ * device. */
+rdn_status_t rdn_device_status(rdn_stream_t stream, int *status);
+
 /* Number of Dk x Dv blocks in each of S_chunks and R_chunks:
  * B * H * ceil(T/64), or with cu_seqlens the bound H * (num_seqs +
  * ceil(T/64)) (slots past the sequences' chunks are left untouched). */

@@ -311,6 +311,16 @@ def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant=
     return o
 
 
+def device_status(stream=None):
+    """Wait for the stream (default: torch's current stream) and return the
+    device-side failure code recorded since the last call (0 = none; 4 = a
+    bounded wait gave up, the outputs of that call are invalid), clearing it."""
+    st = ctypes.c_int(0)
+    s = torch.cuda.current_stream().cuda_stream if stream is None else stream.cuda_stream
+    _check("rdn_device_status", _abi.load().rdn_device_status(s, ctypes.byref(st)))
+    return st.value
+
+
 class LaunchTimer:
     """Context manager recording the device time of every launch of the
     library's kernels (CUDA events on each kernel's own stream).

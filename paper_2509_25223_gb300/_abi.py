@@ -26,7 +26,7 @@ STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "R
 EXPORTS = ["rla_fwd", "rdn_fwd", "rla_bwd", "rdn_bwd", "rdn_decode_step", "rla_fwd_workspace_size",
            "rdn_fwd_workspace_size", "rla_bwd_workspace_size", "rdn_bwd_workspace_size",
            "rdn_last_error", "rdn_version", "rdn_prof_start", "rdn_prof_stop", "rdn_fwd_noalloc",
-           "rdn_qk_prologue", "rdn_qk_prologue_bwd", "rdn_chunk_slots"]
+           "rdn_qk_prologue", "rdn_qk_prologue_bwd", "rdn_chunk_slots", "rdn_device_status"]
 
 
 class ProfRecord(ctypes.Structure):
@@ -104,6 +104,8 @@ def load(build_if_missing: bool = True):
     lib.rdn_prof_stop.argtypes = [ctypes.POINTER(ProfRecord), ctypes.c_int,
                                   ctypes.POINTER(ctypes.c_int)]
     lib.rdn_prof_stop.restype = S
+    lib.rdn_device_status.argtypes = [P, ctypes.POINTER(ctypes.c_int)]
+    lib.rdn_device_status.restype = S
     lib.rdn_last_error.restype = ctypes.c_char_p
     lib.rdn_last_error.argtypes = []
     lib.rdn_version.restype = ctypes.c_char_p

@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "status.cuh"
 
 namespace rdn {
 namespace prof {
@@ -240,6 +241,48 @@ constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
 void *g_noalloc_ptr[kMaxDevices] = {};
 }  // namespace
+
+// The status word (status.cuh): one per device, looked up like the scratch.
+static __device__ int g_status;
+namespace {
+std::mutex g_status_mu;
+void *g_status_ptr[kMaxDevices] = {};
+}  // namespace
+
+}  // extern "C"
+
+namespace rdn {
+int *status_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(g_status_mu);
+  if (!g_status_ptr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = p;
+  }
+  return static_cast<int *>(g_status_ptr[dev]);
+}
+}  // namespace rdn
+
+extern "C" {
+
+rdn_status_t rdn_device_status(rdn_stream_t stream, int *status) {
+  const char *fn = "rdn_device_status";
+  if (!status) return fail(RDN_ERR_INVALID_ARG, "%s: status is NULL", fn);
+  int *w = rdn::status_word();
+  if (!w) return fail(RDN_ERR_CUDA, "%s: the status word of this device is not available", fn);
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  int v = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&v, w, sizeof v, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && v != 0) {
+    const int zero = 0;
+    e = cudaMemcpy(w, &zero, sizeof zero, cudaMemcpyHostToDevice);
+  }
+  if (e != cudaSuccess) return cuda_status(fn, e);
+  *status = v;
+  return ok();
+}
 
 rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a0, rdn_stream_t stream) {
   const char *fn = "rdn_fwd_noalloc";

@@ -28,6 +28,7 @@
 // Kernel bwd_finish: one CTA per chunk, folds the accumulator into dq, dk,
 // dg, dbeta, dgamma.
 #include "chunk_common.cuh"
+#include "status.cuh"
 
 namespace rdn {
 namespace {
@@ -777,7 +778,7 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   l.tied = (f.flags & RDN_FLAG_TIED_GAMMA) && !a.dgamma
                ? align256(sizeof(float) * (size_t)f.B * f.T * f.H)
                : 0;
-  // + the packed-sequence table and the device status word
+  // + the packed-sequence table and a 256-byte tail
   l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.tied + l.seq + 256;
   return l;
 }
@@ -832,7 +833,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   p.f = make_fwd_params(f);
   const bool reuse = reuse_fwd_records(f);
   p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
-  p.f.err = (int *)(ws + l.total - 256);
+  p.f.err = status_word();
   if (f.cu_seqlens) {  // this call's own copy of the packed-sequence table
     long long *seq = (long long *)(ws + l.total - 256 - l.seq);
     cudaError_t e = launch_seq_table(f, seq, s);

@@ -31,6 +31,7 @@
 #include <type_traits>
 
 #include "chunk_common.cuh"
+#include "status.cuh"
 
 namespace rdn {
 namespace {
@@ -550,7 +551,7 @@ FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
   const size_t nrec = (size_t)call_records(a);
   // per-chunk records, the saved intermediates if asked for, the packed-
-  // sequence table, then a 256-byte device status word
+  // sequence table, then a 256-byte tail
   pl.total_bytes = pl.prep_bytes * nrec + seq_table_bytes(a) + 256;
   if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
   return pl;
@@ -570,7 +571,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   FwdParams p = make_fwd_params(a);
   p.ws = (float *)a.workspace;
   const size_t total = plan_fwd(a, variant).total_bytes;
-  p.err = (int *)((char *)a.workspace + total - 256);
+  p.err = status_word();
   if (a.cu_seqlens) {
     long long *seq = (long long *)((char *)a.workspace + total - 256 - seq_table_bytes(a));
     const cudaError_t e = launch_seq_table(a, seq, s);

@@ -127,6 +127,12 @@ def test_packed_sequence_validation_and_sizes():
     assert m.value == 256 + rec * 4 * 12 + table
 
 
+def test_device_status_validation():
+    lib = _abi.load()
+    assert lib.rdn_device_status(None, None) == 1  # status pointer NULL, before any CUDA call
+    assert "status is NULL" in lib.rdn_last_error().decode()
+
+
 def test_decode_validation():
     lib = _abi.load()
     a = _abi.DecodeArgs()

@@ -128,3 +128,17 @@ def test_rdn_fwd_full_size_sampled(wname, heads):
         assert_close(o[b:b + 1, :, h:h + 1], oref, "bf16", f"o{b},{h}")
         assert_close(ST[b:b + 1, h:h + 1], Sref, "bf16", f"ST{b},{h}")
         assert_close(RT[b:b + 1, h:h + 1], Rref, "bf16", f"RT{b},{h}")
+
+
+def test_device_status_clear_after_normal_calls():
+    """No bounded wait gives up on a normal forward and backward: the device
+    status word reads 0 (and reading clears it)."""
+    x = make_inputs(2, 200, 2, 128, dtype="bf16", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    rdn.device_status()  # whatever an earlier test left
+    for variant in ("rdn", "rla"):
+        fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
+        bwd = rdn.rdn_bwd if variant == "rdn" else rdn.rla_bwd
+        fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"])
+        bwd(*(x[n] for n in NAMES), x["dO"], clip=1.0, S0=x["S0"], R0=x["R0"])
+        assert rdn.device_status() == 0, variant
