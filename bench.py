@@ -232,7 +232,16 @@ def time_oracle_sample(target_s=15.0, max_heads=None):
             nh = min(nh, max_heads)
         dt = run(nh)
     tokens = nh * w.T / w.H
+    # one head on one thread: the oracle's single-core rate
+    oracle.set_threads(1)
+    try:
+        dt1 = run(1)
+    finally:
+        oracle.set_threads(threads)
+    single = (w.T / w.H) / dt1
     return dict(value=tokens / dt, unit="tokens/s", cores=min(threads, nh), kind="oracle",
+                single_thread_value=single, single_thread_sample=f"1 (b,h) head, T={w.T}, "
+                f"{dt1:.1f} s on 1 thread",
                 sample=f"fp64 oracle fwd+bwd on {nh} of the workload's (b,h) heads, "
                        f"full T={w.T} each ({nh * w.T} token-heads = {tokens:.0f} tokens), "
                        f"{dt:.1f} s on {min(threads, nh)} OpenMP threads")

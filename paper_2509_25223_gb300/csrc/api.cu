@@ -10,6 +10,8 @@
 #include <mutex>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 #include "status.cuh"
 
@@ -150,7 +152,15 @@ rdn_status_t cuda_status(const char *fn, cudaError_t e) {
   return fail(RDN_ERR_CUDA, "%s: CUDA error %d (%s)", fn, (int)e, cudaGetErrorString(e));
 }
 
+// An NVTX range named after the entry point for the duration of the call
+// (host side: validation and enqueueing), seen by profilers and free without one.
+struct CallRange {
+  explicit CallRange(const char *fn) { nvtxRangePushA(fn); }
+  ~CallRange() { nvtxRangePop(); }
+};
+
 rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a0, int variant, cudaStream_t s) {
+  CallRange range(fn);
   rdn_status_t st = check_fwd_shapes(fn, a0);
   if (st != RDN_OK) return st;
   const rdn_fwd_args ua = untied(*a0);
@@ -286,6 +296,7 @@ rdn_status_t rdn_device_status(rdn_stream_t stream, int *status) {
 
 rdn_status_t rdn_fwd_noalloc(const rdn_fwd_args *a0, rdn_stream_t stream) {
   const char *fn = "rdn_fwd_noalloc";
+  CallRange range(fn);
   rdn_status_t st = check_fwd_shapes(fn, a0);
   if (st != RDN_OK) return st;
   const rdn_fwd_args ua = untied(*a0);
@@ -378,6 +389,7 @@ rdn_status_t bwd_workspace_common(const char *fn, const rdn_bwd_args *a, int var
 }
 
 rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a0, int variant, cudaStream_t stream) {
+  CallRange range(fn);
   if (!a0) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
   rdn_status_t st = check_fwd_shapes(fn, &a0->fwd);
   if (st != RDN_OK) return st;
@@ -458,6 +470,7 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *a, rdn_stream_t stream) {
 namespace {
 rdn_status_t prologue_common(const char *fn, const rdn_prologue_args *a, bool bwd,
                              cudaStream_t stream) {
+  CallRange range(fn);
   if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
   if (a->rows < 1 || a->rows > (1ll << 40))
     return fail(RDN_ERR_INVALID_ARG, "%s: rows must be in [1, 2^40] (got %lld)", fn, a->rows);
@@ -492,6 +505,7 @@ rdn_status_t rdn_qk_prologue_bwd(const rdn_prologue_args *a, rdn_stream_t stream
 
 rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {
   const char *fn = "rdn_decode_step";
+  CallRange range(fn);
   if (!a) return fail(RDN_ERR_INVALID_ARG, "%s: args is NULL", fn);
   if (a->N < 1 || a->H < 1)
     return fail(RDN_ERR_INVALID_ARG, "%s: need N >= 1, H >= 1 (got N=%d H=%d)", fn, a->N, a->H);
