@@ -529,7 +529,8 @@ def run_ours(args):
         tr, rval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * rsteps)
         rla = {"workload": w.name.replace("rdn_", "rla_"), "value": rval, "unit": "tokens/s",
                "steps": rsteps, "ms_per_step": tr / rsteps,
-               "path": "fp32 SIMT chunk kernels (RLA keeps fp32 state operands)",
+               "path": "tensor-core forward (hi + lo copy of S for the read-outs), "
+                       "fp32 chunk-kernel backward",
                "kernels": {k: {"launches": n, "mean_ms": m}
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr

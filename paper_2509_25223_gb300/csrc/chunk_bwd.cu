@@ -754,10 +754,16 @@ bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
 }
 
 // The forward's per-chunk records are valid input when the caller passes the
-// forward's workspace with its chunk-start states.  Both passes pick the same
-// record format: shared-memory images for bf16, d = 128 (tensor-core forward
-// and backward), fp32 otherwise.
-bool reuse_fwd_records(const rdn_fwd_args &f) { return f.workspace && f.S_chunks; }
+// forward's workspace with its chunk-start states and they are in the format
+// this backward reads: shared-memory images where the forward ran the
+// tensor-core scan, read by the tensor-core backward (RDN); fp32 otherwise.
+// (RLA at bf16, d = 128 runs the tensor-core forward and the fp32 backward,
+// which then recomputes its records.)
+bool reuse_fwd_records(const rdn_fwd_args &f, int variant) {
+  const FwdParams fp = make_fwd_params(f);
+  return f.workspace && f.S_chunks &&
+         fwd_uses_tc(fp, f.Dk, f.dtype == RDN_BF16) == use_tc_bwd(f, variant);
+}
 
 BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const rdn_fwd_args &f = a.fwd;
@@ -766,7 +772,7 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const size_t accf = f.Dk == 128 ? Acc<128>::FLOATS : Acc<64>::FLOATS;
   BwdLayout l;
   // the forward's records are read from its workspace when it is passed
-  l.prep = reuse_fwd_records(f) ? 0 : align256(sizeof(float) * nrec * kRecFloats);
+  l.prep = reuse_fwd_records(f, variant) ? 0 : align256(sizeof(float) * nrec * kRecFloats);
   l.acc = tc ? align256(bwd_tc_acc_bytes(nrec)) : align256(sizeof(float) * nrec * accf);
   const bool need_states = f.S_chunks == nullptr;
   l.states = need_states ? align256(sizeof(float) * nrec * f.Dk * f.Dv) : 0;  // each of S, R
@@ -831,7 +837,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   char *ws = (char *)a.workspace;
   BwdParams p;
   p.f = make_fwd_params(f);
-  const bool reuse = reuse_fwd_records(f);
+  const bool reuse = reuse_fwd_records(f, variant);
   p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
   p.f.err = status_word();
   if (f.cu_seqlens) {  // this call's own copy of the packed-sequence table
@@ -858,7 +864,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
     e = launch_fwd_parts(p.f, f.Dk, rdnv, bf, true, true, s);
     // the tensor-core forward leaves its records as shared-memory images,
     // which the tensor-core backward reads too; the SIMT backward needs fp32
-    if (e == cudaSuccess && rdnv && bf && f.Dk == 128 && !tc && p.f.mods == 0)
+    if (e == cudaSuccess && fwd_uses_tc(p.f, f.Dk, bf) && !tc)
       e = launch_prep(p.f, f.Dk, rdnv, bf, false, s);
   } else if (!reuse) {
     e = launch_prep(p.f, f.Dk, rdnv, bf, tc, s);

@@ -211,6 +211,13 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   return p;
 }
 
+// Whether the forward runs the tensor-core scan (and its records are
+// shared-memory images): bf16 inputs, d = 128, the method itself (no variant
+// flags), for RDN and RLA alike.
+inline bool fwd_uses_tc(const FwdParams &p, int DK, bool bf16) {
+  return bf16 && DK == 128 && p.mods == 0;
+}
+
 // Tensor-core scan (fwd_tc.cu): bf16 inputs with d_k = d_v = 128.
 bool fwd_tc_supported(const rdn_fwd_args &a);
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s);

@@ -445,11 +445,10 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
 
 cudaError_t launch_fwd_parts(const FwdParams &p, int DK, bool rdnv, bool bf16, bool do_prep,
                              bool do_scan, cudaStream_t s) {
-  // RDN with bf16 inputs and d = 128 runs the tensor-core scan; everything
-  // else the fp32 SIMT one.  (RLA's state is not contracted by the delta
-  // term, and its output error with single-bf16 state operands reaches the
-  // 2e-2 RMS bound, so RLA stays on the fp32 path.)
-  const bool tc_scan = do_scan && bf16 && DK == 128 && rdnv && p.mods == 0;
+  // bf16 inputs with d = 128 (RDN, and RLA with a hi + lo copy of S for its
+  // read-outs) run the tensor-core scan; everything else, and the variants,
+  // the fp32 SIMT one
+  const bool tc_scan = do_scan && fwd_uses_tc(p, DK, bf16);
   cudaError_t e = cudaSuccess;
   // (the tensor-core scan reads the records as shared-memory images)
   if (DK == 128) {

@@ -169,6 +169,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const uint32_t tm = *slot;
   const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   uint32_t phase = 0, phA = 0, phB = 0;  // phA/phB: tracked by thread 0 only
+  // RLA: S - bf16(S) as a bf16 image (rows j; key block 0 in slot A, block 1
+  // in the E^T lo tile: RLA has no T matrices, and the E lo tile is free from
+  // the end of a chunk to the next one's MMA3), so that the read-outs K S,
+  // Q S use S to ~16 bits: RLA's state is not contracted by a delta term and
+  // its prediction S k is a large sum the residual v - S k cancels against
+  auto store_state_lo = [&](int c0, const float (&s)[16]) {
+    float lo[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) lo[i] = s[i] - __bfloat162float(__float2bfloat16_rn(s[i]));
+    st_row16(sm + SM_SLOTA, SM_XE_LO - SM_SLOTA, j, c0, lo);
+  };
   auto rec_of = [&](int c) {
     return reinterpret_cast<const uint8_t *>(p.ws + (size_t)(sp.rbase + c) * kRecFloats);
   };
@@ -225,6 +236,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     tmem_st16(tm + lane + T_R + c0, r);
     st_row16(sm + SM_SA, 16384, j, c0, s);
     st_row16(sm + SM_RA, 16384, j, c0, r);
+    if (!RDNV) store_state_lo(c0, s);
     if (p.S_chunks && NC > 0) {  // the first chunk's start states, for the backward
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
@@ -345,6 +357,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       if (p.sv_E2) bulk_wait_read();  // the E2^T tiles of the previous chunk are rewritten next
       mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
+      if (!RDNV)  // (RLA) + the state's lo part: its prediction carries no delta contraction
+        mma_tile(tm + T_D1, sbase + SM_SLOTA, SM_XE_LO - SM_SLOTA, sbase + SM_KQ, 16384, 8,
+                 idesc_bf16(128, 128), true);
       mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
@@ -551,6 +566,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
           rc_next[(size_t)(g16 + 64 + i) * D + j] = r1[i];
         }
       }
+    }
+    if (!RDNV) {  // (RLA) the updated state's lo part, for the next chunk's read-outs
+      float s0[16], s1[16];
+      tmem_ld16x2(tm + lane + T_S + g16, s0, tm + lane + T_S + g16 + 64, s1);
+      store_state_lo(g16, s0);
+      store_state_lo(g16 + 64, s1);
     }
     __syncthreads();  // the o tile
     for (int e = tid; e < 64 * 16; e += kTcThreads) {

@@ -130,6 +130,24 @@ def test_rdn_fwd_full_size_sampled(wname, heads):
         assert_close(RT[b:b + 1, h:h + 1], Rref, "bf16", f"RT{b},{h}")
 
 
+@pytest.mark.parametrize("wname,heads", [
+    ("rdn_fwd_bf16_B8H16T2048D128", [(0, 1), (7, 14)]),
+    ("rdn_fwd_bf16_B2H16T16384D128_state", [(0, 3), (1, 10)]),
+])
+def test_rla_fwd_full_size_sampled(wname, heads):
+    """RLA on the same full-size inputs (tensor-core forward, hi + lo state
+    for the read-outs): the state is not contracted by a delta term and grows
+    over the 16,384 tokens, the case its precision is made for."""
+    w = WORKLOADS[wname]
+    x = make_workload_inputs(w, device="cuda")
+    o, ST, RT = _gpu("rla", x)
+    assert torch.isfinite(o.float()).all()
+    for (b, h), (oref, Sref, Rref) in zip(heads, _ref("rla", x, heads=heads)):
+        assert_close(o[b:b + 1, :, h:h + 1], oref, "bf16", f"o{b},{h}")
+        assert_close(ST[b:b + 1, h:h + 1], Sref, "bf16", f"ST{b},{h}")
+        assert_close(RT[b:b + 1, h:h + 1], Rref, "bf16", f"RT{b},{h}")
+
+
 def test_device_status_clear_after_normal_calls():
     """No bounded wait gives up on a normal forward and backward: the device
     status word reads 0 (and reading clears it)."""
