@@ -67,6 +67,11 @@ struct TcBwdParams {
   unsigned long long *mask;  // [B*H*NC][128]: bit t = clip inactive (|x| <= c)
   void *dq, *dk;             // outputs of bwd_post
   float *dg, *dbeta, *dgamma;
+  // RLA: the records carry T_beta = T_gamma = I and the deltas are absent
+  // (E = V, E2 = r), so the terms through -Gam K S0, -Gam K R0 and the
+  // gradients of A_beta, A_gamma drop out; the chunk-start state enters the
+  // recomputed prediction with a lo part (RLA's S is not contracted)
+  bool rla;
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
@@ -233,7 +238,9 @@ constexpr uint32_t SA = 0, RA = 32768, B1 = 65536, SLOTA = 98304, SLOTB = 114688
 constexpr uint32_t XE = 147456, XE_LO = 163840, VEC = 180224;
 constexpr uint32_t CTL = VEC + 7 * 64 * 4;
 constexpr uint32_t SLOT = CTL + 48;
-constexpr size_t SMEM = SLOT + 16;
+constexpr uint32_t SA_LO = 183296;  // (RLA) S0 - bf16(S0), two 16 KB blocks
+static_assert(SA_LO >= SLOT + 16 && SA_LO % 1024 == 0, "layout");
+constexpr size_t SMEM = SA_LO + 32768;
 constexpr uint32_t T_D1 = 0, T_D3 = 128, T_X = 256;
 }  // namespace rc
 
@@ -287,6 +294,11 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       }
       put16(sm + SA, 16384, j, c0, s);
       put16(sm + RA, 16384, j, c0, r);
+      if (P.rla) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) s[i] -= __bfloat162float(__float2bfloat16_rn(s[i]));
+        put16(sm + SA_LO, 16384, j, c0, s);
+      }
     }
   }
   __syncthreads();
@@ -311,6 +323,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
 
   bool ok = phase_run(K, tid, [&] {  // KS, KR
     mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
+    if (P.rla) mma_tile(tm + T_D1, sb + SA_LO, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), true);
     mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
     return true;
   });
@@ -322,7 +335,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       tmem_ld16(tm + lane + T_D1 + c0, ks);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        x[i] = vval(c0 + i) - Gam[c0 + i] * ks[i];
+        x[i] = vval(c0 + i) - (P.rla ? 0.f : Gam[c0 + i] * ks[i]);
         ks[i] *= Gprev[c0 + i];
       }
       tmem_st16(tm + lane + T_D1 + c0, ks);
@@ -368,7 +381,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
         const float x = vval(t) - pp[i];
         if (fabsf(x) <= clip) m |= 1ull << t;
         r[t] = clampf(x, clip);
-        x2[i] = r[t] - Gam[t] * kr[i];
+        x2[i] = r[t] - (P.rla ? 0.f : Gam[t] * kr[i]);
       }
       put16s(sm + XE, sm + XE_LO, j, c0, x2);
     }
@@ -669,7 +682,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
           stg[t * D + j] = x[i];
           dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
           dP[i] = dp[i];
-          dkr[i] = -dkr[i] * x[i];
+          dkr[i] = P.rla ? 0.f : -dkr[i] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dkr);
         put16s(sm + S3H, sm + S3L, j, c0, dp);
@@ -734,7 +747,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
           dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
-          dks[i] = dks[i] * dP[i] - gm[i] * x[i];
+          dks[i] = dks[i] * dP[i] - (P.rla ? 0.f : gm[i] * x[i]);
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
       }
@@ -1034,7 +1047,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       float ks[16], kr[16];
       tmem_ld16x2(tm + tm_lane + T_KS + tb, ks, tm + tm_lane + T_KR + tb, kr);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
+      if (!P.rla) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
+      }
       cta_row_sum512(rv, red, dGamS, tid);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = dp_of(i) * ks[i];
@@ -1047,7 +1063,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       y[i] *= x[i] * dov[i];
-      x[i] = -x[i] * x2v[i];
+      x[i] = P.rla ? 0.f : -x[i] * x2v[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1080,7 +1096,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     lds16(Gam + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      x[i] = x[i] * dp_of(i) - y[i] * xv[i];
+      x[i] = x[i] * dp_of(i) - (P.rla ? 0.f : y[i] * xv[i]);
       y[i] *= dov[i];
     }
     put_tok(x, XH, XL);
@@ -1224,10 +1240,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
           if (j < 64) {
             F[F_DM2 + e] = g1[i];
             F[F_DMQ + e] = g2[i];
-            F[F_DAB + e] = -g3[i];
+            F[F_DAB + e] = P.rla ? 0.f : -g3[i];
             F[F_KK + e] = gr[i];
           } else {
-            F[F_DAG + e] = -g1[i];
+            F[F_DAG + e] = P.rla ? 0.f : -g1[i];
             F[F_DAP + e] = g2[i];
             F[F_QK + e] = scale * gr[i];
           }
@@ -1482,8 +1498,9 @@ size_t bwd_tc_extra_bytes(long long nrec) {
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, cudaStream_t s) {
+                          char *extra, bool rla, cudaStream_t s) {
   TcBwdParams P;
+  P.rla = rla;
   P.dq = dq;
   P.dk = dk;
   P.dg = dg;

@@ -747,10 +747,11 @@ struct BwdLayout {
   size_t prep, acc, states, o, tc, tied, seq, total;
 };
 
-// RDN with bf16 inputs and d = 128 takes the tensor-core backward (RLA, whose
-// forward stays on the fp32 SIMT scan, the SIMT backward)
+// bf16 inputs with d = 128 take the tensor-core backward (RDN, and RLA with
+// identity T matrices in its records), the variants the fp32 one
 bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
-  return variant == 1 && f.dtype == RDN_BF16 && f.Dk == 128 && !(f.flags & RDN_FLAG_VARIANTS);
+  (void)variant;
+  return f.dtype == RDN_BF16 && f.Dk == 128 && !(f.flags & RDN_FLAG_VARIANTS);
 }
 
 // The forward's per-chunk records are valid input when the caller passes the
@@ -887,7 +888,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   if (tc)  // the accumulator words it reads are written by its own kernels
     return launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dq, a.dk, a.dv, a.dg, a.dbeta,
                          a.dgamma, a.dS0, a.dR0, p.acc, ws + l.prep + l.acc + 2 * l.states + l.o,
-                         s);
+                         !rdnv, s);
   if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
   if (rdnv) {
     if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);

@@ -233,7 +233,7 @@ size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, cudaStream_t s);
+                          char *extra, bool rla, cudaStream_t s);
 
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).

@@ -198,6 +198,15 @@ __global__ void __launch_bounds__(kThreads, 1) chunk_prep_kernel(FwdParams p) {
         rec[OFF_TG + e] = Tg[t * LDC + i];
       }
     }
+  } else if (IMG) {
+    // RLA has no delta rule: T_beta = T_gamma = I, which the tensor-core
+    // backward reads in their place
+    for (int e = tid; e < C * C; e += kThreads) {
+      const int t = e / C, i = e % C;
+      uint8_t *img = reinterpret_cast<uint8_t *>(rec);
+      img_put(img + IMG_TB, 8192, t, i, t == i ? 1.f : 0.f);
+      img_put(img + IMG_TG, 8192, t, i, t == i ? 1.f : 0.f);
+    }
   }
 }
 
