@@ -506,14 +506,16 @@ def run_ours(args):
     # and records reused as in the RDN step)
     rla = None
     if not args.no_rla:
-        wsr = torch.empty(rdn.workspace_bytes("rla_fwd", B, T, H, D), dtype=torch.uint8,
-                          device=dev)
+        wsr = torch.empty(rdn.workspace_bytes("rla_fwd", B, T, H, D, save_for_bwd=True),
+                          dtype=torch.uint8, device=dev)
 
         def rstep(inp):
             _, _, _, Sc_, Rc_ = rdn.rla_fwd(*(inp[n] for n in names), clip=w.clip,
-                                            return_chunk_states=True, out=o, workspace=wsr)
+                                            return_chunk_states=True, out=o, workspace=wsr,
+                                            save_for_bwd=True)
             rdn.rla_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
-                        R_chunks=Rc_, out=grads, fwd_workspace=wsr)
+                        R_chunks=Rc_, workspace=wsb, out=grads, fwd_workspace=wsr,
+                        fwd_saved=True)
 
         rsteps = max(1, args.rla_steps)
         rstep(x)
@@ -529,8 +531,8 @@ def run_ours(args):
         tr, rval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * rsteps)
         rla = {"workload": w.name.replace("rdn_", "rla_"), "value": rval, "unit": "tokens/s",
                "steps": rsteps, "ms_per_step": tr / rsteps,
-               "path": "tensor-core forward (hi + lo copy of S for the read-outs), "
-                       "fp32 chunk-kernel backward",
+               "path": "tensor-core kernels as the RDN step (hi + lo copies of S where "
+                       "RLA's uncontracted state needs them; identity T matrices)",
                "kernels": {k: {"launches": n, "mean_ms": m}
                            for k, (n, t, m) in ltr.summary().items()}}
         del wsr

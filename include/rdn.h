@@ -68,13 +68,13 @@ typedef enum {
 
 typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
 
-/* rdn_fwd_args.flags.  RDN_FLAG_SAVE_FOR_BWD (rdn_fwd only; needs S_chunks
- * and R_chunks): the forward also keeps, in its workspace after the per-chunk
- * matrices, the delta errors E and E2 of both passes and the clip mask of
- * every chunk (Section 3.5's intermediates of the residual pass); ask
- * rdn_fwd_workspace_size with the flag set.  rdn_bwd given that workspace
- * (fwd.workspace) and the same flag in fwd.flags reads them instead of
- * recomputing them.  On the bf16, Dk = 128 path this removes a pass of the
+/* rdn_fwd_args.flags.  RDN_FLAG_SAVE_FOR_BWD (rla_fwd / rdn_fwd; needs
+ * S_chunks and R_chunks): the forward also keeps, in its workspace after the
+ * per-chunk matrices, the delta errors E and E2 of both passes (RLA: V and r)
+ * and the clip mask of every chunk (the intermediates of the residual pass);
+ * ask *_fwd_workspace_size with the flag set.  rla_bwd / rdn_bwd given that
+ * workspace (fwd.workspace) and the same flag in fwd.flags reads them instead
+ * of recomputing them.  On the bf16, Dk = 128 path this removes a pass of the
  * backward; on the others the flag only reserves the space. */
 #define RDN_FLAG_SAVE_FOR_BWD 0x1u
 
@@ -124,7 +124,7 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *                     stored).  rdn_bwd can consume them instead of
  *                     recomputing.
  *   scale             multiplies q (the paper uses 1).
- *   flags             0, or RDN_FLAG_SAVE_FOR_BWD for rdn_fwd and / or
+ *   flags             0, or RDN_FLAG_SAVE_FOR_BWD and / or
  *                     RDN_FLAG_TIED_GAMMA and the variant flags (above).
  *   workspace         device scratch of *_fwd_workspace_size() bytes.
  *   cu_seqlens        NULL, or packed variable-length sequences: a device
@@ -296,8 +296,7 @@ rdn_status_t rdn_bwd(const rdn_bwd_args *args, rdn_stream_t stream);
 
 /* Backward of rla_fwd, Section 3.4 (left formulation): the same arguments,
  * layouts, ownership and errors as rdn_bwd, for the RLA recurrence.
- * fwd.workspace / fwd.S_chunks refer to an rla_fwd call; fwd.flags must be 0
- * (RDN_FLAG_SAVE_FOR_BWD is rdn_fwd's; RDN_ERR_UNSUPPORTED otherwise). */
+ * fwd.workspace / fwd.S_chunks / fwd.flags refer to an rla_fwd call. */
 rdn_status_t rla_bwd(const rdn_bwd_args *args, rdn_stream_t stream);
 
 /* One recurrent step (Section 3.4 recurrence at a single t), states in

@@ -197,11 +197,11 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
-            fwd_workspace=None, tied_gamma=False, cu_seqlens=None, variant_flags=0):
-    """Backward of rla_fwd; the same arguments and results as rdn_bwd (no
-    saved intermediates: rla_fwd has no save_for_bwd)."""
+            fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
+            variant_flags=0):
+    """Backward of rla_fwd; the same arguments and results as rdn_bwd."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
-                R_chunks, workspace, out, fwd_workspace, False, tied_gamma, cu_seqlens,
+                R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
                 variant_flags)
 
 

@@ -165,8 +165,6 @@ rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a0, int variant, cud
   if (st != RDN_OK) return st;
   const rdn_fwd_args ua = untied(*a0);
   const rdn_fwd_args *a = &ua;
-  if (variant == 0 && (a->flags & RDN_FLAG_SAVE_FOR_BWD))
-    return fail(RDN_ERR_UNSUPPORTED, "%s: RDN_FLAG_SAVE_FOR_BWD is for rdn_fwd", fn);
   if ((st = check_fwd_ptrs(fn, a)) != RDN_OK) return st;
   const rdn::FwdPlan plan = rdn::plan_fwd(*a, variant);
   if (plan.total_bytes > 0) {
@@ -419,8 +417,6 @@ rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a0, int variant, cud
   OPTIONAL_PTR(f->R_chunks);
   if ((f->S_chunks == nullptr) != (f->R_chunks == nullptr))
     return fail(RDN_ERR_INVALID_ARG, "%s: S_chunks and R_chunks must be both set or both NULL", fn);
-  if ((f->flags & RDN_FLAG_SAVE_FOR_BWD) && variant != 1)
-    return fail(RDN_ERR_UNSUPPORTED, "%s: RDN_FLAG_SAVE_FOR_BWD is for rdn_fwd / rdn_bwd", fn);
   if ((f->flags & RDN_FLAG_SAVE_FOR_BWD) && !f->workspace && f->T > 0)
     return fail(RDN_ERR_INVALID_ARG,
                 "%s: RDN_FLAG_SAVE_FOR_BWD in fwd.flags needs the forward's fwd.workspace", fn);

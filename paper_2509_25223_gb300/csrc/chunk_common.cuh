@@ -227,7 +227,7 @@ cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s);
 cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool img, cudaStream_t s);
 
 // Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
-cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s);
+cudaError_t launch_prep_tc(const FwdParams &p, bool rla, cudaStream_t s);
 size_t bwd_tc_extra_bytes(long long nrec);  // per record slot
 size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,

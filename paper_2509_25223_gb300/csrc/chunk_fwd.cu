@@ -436,10 +436,10 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
                                 (int)scan_smem<DK>())) != cudaSuccess)
     return e;
   if (do_prep) {
-    // the images for RDN with bf16 inputs and d = 128 come from the tensor-core prep
-    constexpr bool tc_prep = DK == 128 && RDNV && std::is_same<InT, __nv_bfloat16>::value;
+    // the images for bf16 inputs and d = 128 come from the tensor-core prep
+    constexpr bool tc_prep = DK == 128 && std::is_same<InT, __nv_bfloat16>::value;
     if (tc_prep && img && p.mods == 0) {
-      if ((e = launch_prep_tc(p, s)) != cudaSuccess) return e;
+      if ((e = launch_prep_tc(p, !RDNV, s)) != cudaSuccess) return e;
     } else {
       RDN_LAUNCH("chunk_prep", s, prep<<<(unsigned)p.nrec, kThreads, prep_smem<DK>(), s>>>(p));
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -561,7 +561,7 @@ FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   // per-chunk records, the saved intermediates if asked for, the packed-
   // sequence table, then a 256-byte tail
   pl.total_bytes = pl.prep_bytes * nrec + seq_table_bytes(a) + 256;
-  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
+  if (a.flags & RDN_FLAG_SAVE_FOR_BWD) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
   return pl;
 }
 
@@ -586,7 +586,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     p.seq = seq;
   }
-  if (variant == 1 && (a.flags & RDN_FLAG_SAVE_FOR_BWD)) {
+  if (a.flags & RDN_FLAG_SAVE_FOR_BWD) {
     const SavedLayout l = saved_layout((size_t)p.nrec, a.Dv);
     p.sv_E = (uint8_t *)a.workspace + l.e;
     p.sv_E2 = (uint8_t *)a.workspace + l.e2;

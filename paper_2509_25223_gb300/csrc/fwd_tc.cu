@@ -568,6 +568,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       }
     }
     if (!RDNV) {  // (RLA) the updated state's lo part, for the next chunk's read-outs
+      if (p.sv_E2) {  // (into the E^T lo tile: its bulk store to the saved E2 must be done)
+        if (tid == 0) bulk_wait_read();
+        __syncthreads();
+      }
       float s0[16], s1[16];
       tmem_ld16x2(tm + lane + T_S + g16, s0, tm + lane + T_S + g16 + 64, s1);
       store_state_lo(g16, s0);

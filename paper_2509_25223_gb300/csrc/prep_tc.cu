@@ -150,7 +150,9 @@ __device__ __forceinline__ void inv64_stage(int stage, const float *A, float *Tm
   }
 }
 
-__global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
+// rla: RLA's records (no delta rule: T_beta = T_gamma = I, written as such
+// for the tensor-core backward; Ap, Mq, M2 and the vectors are RDN's)
+__global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) {
   using namespace pp;
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sb = smem_u32(sm);
@@ -338,7 +340,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
       }
     }
     __syncthreads();
-    {  // T_beta (threads 0..127) and T_gamma (128..255)
+    if (!rla) {  // T_beta (threads 0..127) and T_gamma (128..255)
       const int g = tid & 127;
       const float *A = tid < 128 ? Ab : Ag;
       float *Tm = tid < 128 ? Tb : Tg;
@@ -357,7 +359,12 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
 #pragma unroll
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        lds16(Tm + r * LDT + 32 * hf + c0, v);
+        if (rla) {
+#pragma unroll
+          for (int u = 0; u < 16; ++u) v[u] = r == 32 * hf + c0 + u ? 1.f : 0.f;
+        } else {
+          lds16(Tm + r * LDT + 32 * hf + c0, v);
+        }
         img_row16(dst, 8192, r, 32 * hf + c0, v);
       }
     }
@@ -382,7 +389,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p) {
 
 }  // namespace
 
-cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s) {
+cudaError_t launch_prep_tc(const FwdParams &p, bool rla, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)pp::SMEM);
   if (e != cudaSuccess) return e;
@@ -392,7 +399,7 @@ cudaError_t launch_prep_tc(const FwdParams &p, cudaStream_t s) {
     return e;
   const size_t nct = (size_t)p.nrec;  // (packed sequences: a bound; the kernel reads the count)
   const unsigned grid = (unsigned)(nct < 2 * (size_t)nsm ? nct : 2 * (size_t)nsm);  // two per SM
-  RDN_LAUNCH("chunk_prep", s, prep_tc_kernel<<<grid, NTH, pp::SMEM, s>>>(p));
+  RDN_LAUNCH("chunk_prep", s, prep_tc_kernel<<<grid, NTH, pp::SMEM, s>>>(p, rla));
   return cudaGetLastError();
 }
 

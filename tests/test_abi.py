@@ -70,8 +70,8 @@ def test_fwd_validation(fn):
     tied = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, o=FAKE)
     assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_TIED_GAMMA, **tied)) == 5
     assert _status(fn, _fwd_args(flags=0, **tied)) == 1  # untied: gamma is required
-    # RDN_FLAG_SAVE_FOR_BWD: rdn_fwd only, and only with chunk states
-    assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD)) == (2 if fn == "rla_fwd" else 1)
+    # RDN_FLAG_SAVE_FOR_BWD: only with chunk states
+    assert _status(fn, _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD)) == 1  # needs S_chunks
     assert _status(fn, _fwd_args()) == 1  # q is NULL
     assert "q is NULL" in lib.rdn_last_error().decode()
     ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE, o=FAKE)
@@ -190,8 +190,9 @@ def test_bwd_validation():
 
 
 def test_rla_bwd_validation():
-    """rla_bwd shares rdn_bwd's checks; the saved-intermediates flag is rdn_fwd's
-    and is refused; its workspace query answers for the RLA forward's layout."""
+    """rla_bwd shares rdn_bwd's checks, the saved-intermediates flag included
+    (it needs the forward's workspace); its workspace query answers for the
+    RLA forward's layout."""
     lib = _abi.load()
     b = _abi.BwdArgs()
     b.fwd = _fwd_args()
@@ -199,9 +200,8 @@ def test_rla_bwd_validation():
     ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE)
     for f in ("dO", "dq", "dk", "dv", "dg", "dbeta", "dgamma"):
         setattr(b, f, FAKE)
-    b.fwd = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, workspace=FAKE, workspace_bytes=1 << 40,
-                      S_chunks=FAKE, R_chunks=FAKE, **ok)
-    assert lib.rla_bwd(ctypes.byref(b), None) == 2
+    b.fwd = _fwd_args(flags=_abi.RDN_FLAG_SAVE_FOR_BWD, S_chunks=FAKE, R_chunks=FAKE, **ok)
+    assert lib.rla_bwd(ctypes.byref(b), None) == 1  # the flag without the forward's workspace
     assert "RDN_FLAG_SAVE_FOR_BWD" in lib.rdn_last_error().decode()
     n_rla, n_rdn = ctypes.c_size_t(0), ctypes.c_size_t(0)
     b.fwd = _fwd_args()

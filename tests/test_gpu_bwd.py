@@ -44,8 +44,8 @@ def _ref(x, clip, dST=None, dRT=None, heads=None, scale=1.0, variant=oracle.RDN)
     for b, h in heads:
         sl = lambda t: None if t is None else as64(t[b:b + 1, :, h:h + 1])
         st = lambda t: None if t is None else as64(t[b:b + 1, h:h + 1])
-        outs.append(oracle.rdn_bwd(*(sl(x[n]) for n in NAMES), clip, st(x["S0"]), st(x["R0"]),
-                                   sl(x["dO"]), st(dST), st(dRT)))
+        outs.append(oracle.bwd(variant, *(sl(x[n]) for n in NAMES), clip, st(x["S0"]),
+                               st(x["R0"]), sl(x["dO"]), st(dST), st(dRT)))
     return outs
 
 
@@ -148,44 +148,52 @@ def test_bwd_reuses_forward_records(dtype, D):
         assert_close(d1[name], ref[name], dtype, name)
 
 
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
 @pytest.mark.parametrize("dtype,D,T", [("bf16", 128, 150), ("bf16", 128, 1), ("bf16", 64, 150),
                                        ("f32", 128, 150)])
-def test_bwd_uses_forward_saved_intermediates(dtype, D, T):
+def test_bwd_uses_forward_saved_intermediates(variant, dtype, D, T):
     """A forward run with save_for_bwd keeps E, E2 and the clip mask; the
     backward that reads them matches the one that recomputes them, and the
     oracle."""
+    ov = oracle.RDN if variant == "rdn" else oracle.RLA
     x = make_inputs(2, T, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,
                     device="cuda", state_std=0.1)
-    _condition(x, 1.0, dtype)
+    _condition(x, 1.0, dtype, variant=ov)
     tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
-    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", 2, T, 2, D, tdt, save_for_bwd=True),
+    wsf = torch.empty(rdn.workspace_bytes(f"{variant}_fwd", 2, T, 2, D, tdt, save_for_bwd=True),
                       dtype=torch.uint8, device="cuda")
-    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
-                                    return_chunk_states=True, workspace=wsf, save_for_bwd=True)
-    d1 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True)
-    d2 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc)
-    ref = _ref(x, 1.0)
+    fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
+    o, ST, RT, Sc, Rc = fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                            return_chunk_states=True, workspace=wsf, save_for_bwd=True)
+    d1 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True,
+              variant=variant)
+    d2 = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, variant=variant)
+    ref = _ref(x, 1.0, variant=ov)
     for name in GRADS:
         torch.testing.assert_close(d1[name].float(), d2[name].float(), atol=1e-5, rtol=8e-3)
         assert_close(d1[name], ref[name], dtype, name)
 
 
-def test_bwd_full_size_sampled():
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
+def test_bwd_full_size_sampled(variant):
     """The bench's fwd+bwd workload (B=8, H=16, T=4096, D=128, bf16) in the
     bench's launch configuration (chunk states, per-chunk matrices and saved
-    intermediates from rdn_fwd); the oracle checks sampled heads."""
+    intermediates from the forward); the oracle checks sampled heads."""
+    ov = oracle.RDN if variant == "rdn" else oracle.RLA
     w = WORKLOADS["rdn_fwd_bwd_bf16_B8H16T4096D128"]
     x = make_workload_inputs(w, device="cuda")
     heads = [(0, 0), (5, 9), (7, 15)]
-    _condition(x, 1.0, "bf16", heads=heads)
-    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", w.B, w.T, w.H, w.D, save_for_bwd=True),
-                      dtype=torch.uint8, device="cuda")
-    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, return_chunk_states=True,
-                                    workspace=wsf, save_for_bwd=True)
-    d = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True)
+    _condition(x, 1.0, "bf16", heads=heads, variant=ov)
+    wsf = torch.empty(rdn.workspace_bytes(f"{variant}_fwd", w.B, w.T, w.H, w.D,
+                                          save_for_bwd=True), dtype=torch.uint8, device="cuda")
+    fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
+    o, ST, RT, Sc, Rc = fwd(*(x[n] for n in NAMES), clip=1.0, return_chunk_states=True,
+                            workspace=wsf, save_for_bwd=True)
+    d = _gpu(x, 1.0, S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True,
+             variant=variant)
     for name in GRADS:
         assert torch.isfinite(d[name].float()).all(), name
-    for (b, h), ref in zip(heads, _ref(x, 1.0, heads=heads)):
+    for (b, h), ref in zip(heads, _ref(x, 1.0, heads=heads, variant=ov)):
         for name in GRADS:
             g = d[name][b:b + 1, h:h + 1] if name in ("dS0", "dR0") else d[name][b:b + 1, :, h:h + 1]
             assert_close(g, ref[name], "bf16", f"{name} ({b},{h})")
