@@ -336,7 +336,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         x[i] = vval(c0 + i) - (P.rla ? 0.f : Gam[c0 + i] * ks[i]);
-        ks[i] *= Gprev[c0 + i];
+        ks[i] *= (p.mods & RDN_FLAG_DECAYED_RESIDUAL) ? Gam[c0 + i] : Gprev[c0 + i];
       }
       tmem_st16(tm + lane + T_D1 + c0, ks);
       put16s(sm + XE, sm + XE_LO, j, c0, x);
@@ -740,7 +740,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         const int c0 = g16;
         float x[16], dks[16], gm[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
-        lds16(Gprev + c0, dks);
+        // the prediction's state term: Gprev K S0 (decayed residual: Gam K S0)
+        lds16((p.mods & RDN_FLAG_DECAYED_RESIDUAL) ? Gam + c0 : Gprev + c0, dks);
         lds16(Gam + c0, gm);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -883,6 +884,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const int H = p.H;
   const size_t nct = (size_t)total_records(p);
   const float scale = p.scale;
+  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;  // residual against a_t S_{t-1} k_t
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   Ctl K;
@@ -1046,14 +1048,18 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {
       float ks[16], kr[16];
       tmem_ld16x2(tm + tm_lane + T_KS + tb, ks, tm + tm_lane + T_KR + tb, kr);
-#pragma unroll
       if (!P.rla) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
       }
+      // the prediction's state term: Gprev K S0 (decayed residual: Gam K S0)
+      if (dec_res) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rv[i] += dp_of(i) * ks[i];
+      }
       cta_row_sum512(rv, red, dGamS, tid);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] = dp_of(i) * ks[i];
+      for (int i = 0; i < 16; ++i) rv[i] = dec_res ? 0.f : dp_of(i) * ks[i];
     }
     cta_row_sum512(rv, red, dGprevS, tid);
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
@@ -1092,7 +1098,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   if (ok) {  // ---- P3: dK, dQ += S0 [dKS ; dQS]^T, dKS = Gprev dP - Gam dX, dQS = Gam dO;
              // meanwhile <dR, R0>
     float x[16], y[16];
-    lds16(Gprev + tb, x);
+    lds16(dec_res ? Gam + tb : Gprev + tb, x);
     lds16(Gam + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -1305,13 +1311,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
           }
           if (i < t) {
             const float decp = __expf(cpt - cum[i]);
-            {  // Ap: strict, beta, K K^T, previous-token decay
+            {  // Ap: strict, beta, K K^T, previous-token decay (decayed residual: to t)
+              const float dA = dec_res ? dec : decp;
               const float dm = F[F_DAP + e];
-              const float G = dm * decp * bi * kk;
-              rowp += G;
+              const float G = dm * dA * bi * kk;
+              if (dec_res) rowc += G; else rowp += G;
               cg += G;
-              cb += dm * decp * kk;
-              dkk += dm * decp * bi;
+              cb += dm * dA * kk;
+              dkk += dm * dA * bi;
             }
             {  // Mq: strict, beta, Q K^T
               const float dm = F[F_DMQ + e];

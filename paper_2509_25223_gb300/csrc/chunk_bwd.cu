@@ -751,7 +751,7 @@ struct BwdLayout {
 // identity T matrices in its records), the variants the fp32 one
 bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
   (void)variant;
-  return f.dtype == RDN_BF16 && f.Dk == 128 && !(f.flags & RDN_FLAG_VARIANTS);
+  return f.dtype == RDN_BF16 && f.Dk == 128 && !(f.flags & RDN_FLAG_VARIANTS & ~kTcVariants);
 }
 
 // The forward's per-chunk records are valid input when the caller passes the

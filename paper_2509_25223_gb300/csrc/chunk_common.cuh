@@ -211,11 +211,14 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   return p;
 }
 
+// The variant flags the tensor-core kernels implement (the others run on the
+// fp32 chunk kernels): the decayed residual.
+constexpr unsigned kTcVariants = RDN_FLAG_DECAYED_RESIDUAL;
 // Whether the forward runs the tensor-core scan (and its records are
-// shared-memory images): bf16 inputs, d = 128, the method itself (no variant
-// flags), for RDN and RLA alike.
+// shared-memory images): bf16 inputs, d = 128, no variant flag outside
+// kTcVariants, for RDN and RLA alike.
 inline bool fwd_uses_tc(const FwdParams &p, int DK, bool bf16) {
-  return bf16 && DK == 128 && p.mods == 0;
+  return bf16 && DK == 128 && (p.mods & ~kTcVariants) == 0;
 }
 
 // Tensor-core scan (fwd_tc.cu): bf16 inputs with d_k = d_v = 128.

@@ -438,7 +438,7 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
   if (do_prep) {
     // the images for bf16 inputs and d = 128 come from the tensor-core prep
     constexpr bool tc_prep = DK == 128 && std::is_same<InT, __nv_bfloat16>::value;
-    if (tc_prep && img && p.mods == 0) {
+    if (tc_prep && img && (p.mods & ~kTcVariants) == 0) {
       if ((e = launch_prep_tc(p, !RDNV, s)) != cudaSuccess) return e;
     } else {
       RDN_LAUNCH("chunk_prep", s, prep<<<(unsigned)p.nrec, kThreads, prep_smem<DK>(), s>>>(p));

@@ -153,6 +153,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const __nv_bfloat16 *v = (const __nv_bfloat16 *)p.v;
   __nv_bfloat16 *o = (__nv_bfloat16 *)p.o;
   const float clip = p.clip;
+  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
   const size_t st_base = (size_t)bh * D * D;
 
   if (tid == 0) {
@@ -391,7 +392,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       for (int i = 0; i < 16; ++i) {
         vv[i] = vs(c0 + i);
         x[i] = vv[i] - gm[i] * gks[i];
-        gks[i] *= gp[i];
+        gks[i] *= dec_res ? gm[i] : gp[i];  // (decayed residual: P = a S_{t-1} k)
       }
       if (RDNV)
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);

@@ -173,6 +173,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
   const size_t nct = (size_t)total_records(p);
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
   constexpr float kLog2e = 1.4426950408889634f;
+  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
 
   if (tid == 0) {
     mbar_init(bar, 1);
@@ -310,7 +311,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
               a_b = a_p * al;
               a_g = dk * al * gm[u];
             }
-            ap[u] = a_p;
+            ap[u] = dec_res ? a_b : a_p;  // (decayed residual: Ap decays to t)
             Ab[t * LDA + i] = a_b;
             Ag[t * LDA + i] = a_g;
           }
