@@ -438,11 +438,16 @@ static_assert(SMEM <= 232448, "shared memory");
 constexpr uint32_t T_DS = 0, T_DR = 128, T_R1 = 256, T_R2 = 320, T_R3 = 384, T_R4 = 448;
 }  // namespace ch
 
+// kGeneric: the RLA mode and the variant flags (TcBwdParams::rla, FwdParams::mods)
+// are read; the RDN method's instance has them folded away
+template <bool kGeneric>
 __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
   using namespace ch;
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sb = smem_u32(sm);
   const FwdParams &p = P.f;
+  const bool rla = kGeneric && P.rla;
+  const unsigned mods = kGeneric ? p.mods : 0u;
   if (sb & 1023u) {
     if (threadIdx.x == 0 && p.err) atomicExch(p.err, RDN_ERR_CUDA);
     return;
@@ -652,7 +657,9 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       lds16(Gam + c0, x);
       lds16(gamv + c0, w);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] = p.scale * x[i] * w[i] * dO(c0 + i);  // dQR (Q unscaled)
+      const bool plain = mods & RDN_FLAG_PLAIN_COMBINE;  // (no gamma_t in the output)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = p.scale * x[i] * (plain ? 1.f : w[i]) * dO(c0 + i);  // dQR (Q unscaled)
       put16s(sm + S1H, sm + S1L, j, c0, x);
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
@@ -682,7 +689,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
           stg[t * D + j] = x[i];
           dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
           dP[i] = dp[i];
-          dkr[i] = P.rla ? 0.f : -dkr[i] * x[i];
+          dkr[i] = rla ? 0.f : -dkr[i] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dkr);
         put16s(sm + S3H, sm + S3L, j, c0, dp);
@@ -709,7 +716,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         const int c0 = g16;
         float a[16], e[16], dqs[16];
         tmem_ld16x2(tm + lane + T_R4 + c0, a, tm + lane + T_R3 + c0, e);
-        lds16(Gam + c0, dqs);
+        // the base read-out Gam Q S0 (plain combine: Gprev Q S0)
+        lds16((mods & RDN_FLAG_PLAIN_COMBINE) ? Gprev + c0 : Gam + c0, dqs);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           a[i] += e[i];
@@ -741,14 +749,14 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         float x[16], dks[16], gm[16];
         tmem_ld16(tm + lane + T_R3 + c0, x);
         // the prediction's state term: Gprev K S0 (decayed residual: Gam K S0)
-        lds16((p.mods & RDN_FLAG_DECAYED_RESIDUAL) ? Gam + c0 : Gprev + c0, dks);
+        lds16((mods & RDN_FLAG_DECAYED_RESIDUAL) ? Gam + c0 : Gprev + c0, dks);
         lds16(Gam + c0, gm);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
           dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
-          dks[i] = dks[i] * dP[i] - (P.rla ? 0.f : gm[i] * x[i]);
+          dks[i] = dks[i] * dP[i] - (rla ? 0.f : gm[i] * x[i]);
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
       }
@@ -865,6 +873,7 @@ __device__ __forceinline__ void cta_row_sum512(const float (&v)[16], float *red,
   __syncthreads();
 }
 
+template <bool kGeneric>  // (as bwd_chain_kernel's)
 __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   using namespace po;
   extern __shared__ __align__(1024) uint8_t sm[];
@@ -884,7 +893,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const int H = p.H;
   const size_t nct = (size_t)total_records(p);
   const float scale = p.scale;
-  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;  // residual against a_t S_{t-1} k_t
+  const bool rla = kGeneric && P.rla;
+  // residual against a_t S_{t-1} k_t; o = S_{t-1} q_t + R_t q_t
+  const bool dec_res = kGeneric && (p.mods & RDN_FLAG_DECAYED_RESIDUAL);
+  const bool plain = kGeneric && (p.mods & RDN_FLAG_PLAIN_COMBINE);
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   Ctl K;
@@ -1036,19 +1048,20 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
       lds16(Gam + tb, rv);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] = scale * rv[i] * dov[i] * qr[i];
+      for (int i = 0; i < 16; ++i) rv[i] = plain ? 0.f : scale * rv[i] * dov[i] * qr[i];
       cta_row_sum512(rv, red, dGamS, tid);
       // parked in the record's slot (shared memory is full); the same thread reads it back
       if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
       __syncthreads();
       lds16(gamv + tb, rv);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] = scale * dov[i] * (qs[i] + rv[i] * qr[i]);
+      for (int i = 0; i < 16; ++i)  // (plain combine: Gprev Q S0 and no gamma_t)
+        rv[i] = plain ? scale * dov[i] * qr[i] : scale * dov[i] * (qs[i] + rv[i] * qr[i]);
     }
     {
       float ks[16], kr[16];
       tmem_ld16x2(tm + tm_lane + T_KS + tb, ks, tm + tm_lane + T_KR + tb, kr);
-      if (!P.rla) {
+      if (!rla) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
       }
@@ -1060,6 +1073,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       cta_row_sum512(rv, red, dGamS, tid);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = dec_res ? 0.f : dp_of(i) * ks[i];
+      if (plain) {  // the base read-out's gate is Gprev
+        float qs[16];
+        tmem_ld16(tm + tm_lane + T_KS + 64 + tb, qs);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rv[i] += scale * dov[i] * qs[i];
+      }
     }
     cta_row_sum512(rv, red, dGprevS, tid);
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
@@ -1068,8 +1087,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     lds16(gamv + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      y[i] *= x[i] * dov[i];
-      x[i] = P.rla ? 0.f : -x[i] * x2v[i];
+      y[i] = (plain ? 1.f : y[i]) * x[i] * dov[i];
+      x[i] = rla ? 0.f : -x[i] * x2v[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1101,9 +1120,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     lds16(dec_res ? Gam + tb : Gprev + tb, x);
     lds16(Gam + tb, y);
 #pragma unroll
+    float gq[16];  // the base read-out's gate: Gam (plain combine: Gprev)
+    lds16(plain ? Gprev + tb : Gam + tb, gq);
+#pragma unroll
     for (int i = 0; i < 16; ++i) {
-      x[i] = x[i] * dp_of(i) - (P.rla ? 0.f : y[i] * xv[i]);
-      y[i] *= dov[i];
+      x[i] = x[i] * dp_of(i) - (rla ? 0.f : y[i] * xv[i]);
+      y[i] = gq[i] * dov[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1246,10 +1268,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
           if (j < 64) {
             F[F_DM2 + e] = g1[i];
             F[F_DMQ + e] = g2[i];
-            F[F_DAB + e] = P.rla ? 0.f : -g3[i];
+            F[F_DAB + e] = rla ? 0.f : -g3[i];
             F[F_KK + e] = gr[i];
           } else {
-            F[F_DAG + e] = P.rla ? 0.f : -g1[i];
+            F[F_DAG + e] = rla ? 0.f : -g1[i];
             F[F_DAP + e] = g2[i];
             F[F_QK + e] = scale * gr[i];
           }
@@ -1301,8 +1323,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
           const float kk = F[F_KK + e], qk = F[F_QK + e], bi = bet[i], gi = gam[i];
           {  // M2: inclusive, gamma, Q K^T; G1 holds dO E2^T, dM2 = gamma_t dO E2^T
             const float g1 = F[F_DM2 + e];
-            dgo += dec * gi * qk * g1;  // d gamma_t += (M2 E2)_t . dO_t
-            const float dm = gt * g1;
+            if (!plain) dgo += dec * gi * qk * g1;  // d gamma_t += (M2 E2)_t . dO_t
+            const float dm = plain ? g1 : gt * g1;
             const float G = dm * dec * gi * qk;
             rowc += G;
             cg += G;
@@ -1320,13 +1342,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
               cb += dm * dA * kk;
               dkk += dm * dA * bi;
             }
-            {  // Mq: strict, beta, Q K^T
+            {  // Mq: strict, beta, Q K^T (plain combine: decay to t-1)
+              const float dA = plain ? decp : dec;
               const float dm = F[F_DMQ + e];
-              const float G = dm * dec * bi * qk;
-              rowc += G;
+              const float G = dm * dA * bi * qk;
+              if (plain) rowp += G; else rowc += G;
               cg += G;
-              cb += dm * dec * qk;
-              dqk += dm * dec * bi;
+              cb += dm * dA * qk;
+              dqk += dm * dA * bi;
             }
             {  // A_beta, A_gamma: strict, K K^T
               const float da = F[F_DAB + e], dg2 = F[F_DAG + e];
@@ -1541,24 +1564,27 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   if ((e = cudaFuncSetAttribute(bwd_recompute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)rc::SMEM)) != cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(bwd_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const bool generic = rla || f.mods != 0;
+  auto chain = generic ? bwd_chain_kernel<true> : bwd_chain_kernel<false>;
+  auto post = generic ? bwd_post_kernel<true> : bwd_post_kernel<false>;
+  if ((e = cudaFuncSetAttribute(chain, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)ch::SMEM)) != cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(bwd_post_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(post, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)po::SMEM)) != cudaSuccess)
     return e;
   if (!saved) {
     RDN_LAUNCH("bwd_recompute", s, bwd_recompute_kernel<<<(unsigned)nct, NT, rc::SMEM, s>>>(P));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  RDN_LAUNCH("bwd_chain", s, bwd_chain_kernel<<<f.nseq * f.H, NTC, ch::SMEM, s>>>(P));
+  RDN_LAUNCH("bwd_chain", s, chain<<<f.nseq * f.H, NTC, ch::SMEM, s>>>(P));
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   int dev = 0, nsm = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
     return e;
   const unsigned post_grid = (unsigned)(nct < (size_t)nsm ? nct : (size_t)nsm);  // one CTA per SM
-  RDN_LAUNCH("bwd_post", s, bwd_post_kernel<<<post_grid, po::NTP, po::SMEM, s>>>(P));
+  RDN_LAUNCH("bwd_post", s, post<<<post_grid, po::NTP, po::SMEM, s>>>(P));
   return cudaGetLastError();
 }
 

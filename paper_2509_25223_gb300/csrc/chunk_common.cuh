@@ -212,8 +212,8 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
 }
 
 // The variant flags the tensor-core kernels implement (the others run on the
-// fp32 chunk kernels): the decayed residual.
-constexpr unsigned kTcVariants = RDN_FLAG_DECAYED_RESIDUAL;
+// fp32 chunk kernels): the decayed residual and the plain combine.
+constexpr unsigned kTcVariants = RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE;
 // Whether the forward runs the tensor-core scan (and its records are
 // shared-memory images): bf16 inputs, d = 128, no variant flag outside
 // kTcVariants, for RDN and RLA alike.

@@ -124,7 +124,9 @@ __device__ __forceinline__ void mma_split3(uint32_t d, uint32_t a_hi, uint32_t a
   mma_tile(d, a_lo, 0, b_hi, 0, 4, idesc, true);
 }
 
-template <bool RDNV>
+// kGeneric: the variant flags (FwdParams::mods) are read; the method's
+// instances have them folded away
+template <bool RDNV, bool kGeneric>
 __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sbase = smem_u32(sm);
@@ -153,7 +155,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const __nv_bfloat16 *v = (const __nv_bfloat16 *)p.v;
   __nv_bfloat16 *o = (__nv_bfloat16 *)p.o;
   const float clip = p.clip;
-  const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool dec_res = kGeneric && (p.mods & RDN_FLAG_DECAYED_RESIDUAL);
+  const bool plain = kGeneric && (p.mods & RDN_FLAG_PLAIN_COMBINE);  // o = S_{t-1} q + R_t q
   const size_t st_base = (size_t)bh * D * D;
 
   if (tid == 0) {
@@ -375,7 +378,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       const int c0 = g16;
       float x[16], gm[16];
       tmem_ld16x2(tm + lane + T_D1 + 64 + c0, x, tm + lane + T_D1 + c0, gks);
-      lds16(Gam + c0, gm);
+      lds16(plain ? Gprev + c0 : Gam + c0, gm);
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] *= gm[i] * p.scale;
       tmem_st16(tm + lane + T_D1 + 64 + c0, x);
@@ -552,7 +555,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
-        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gv[i] * gm[i] * p.scale, oa[i], ob[i]));
+        const float gg = plain ? 1.f : gv[i];
+        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gg * gm[i] * p.scale, oa[i], ob[i]));
       }
     }
     {
@@ -614,7 +618,9 @@ bool fwd_tc_supported(const rdn_fwd_args &a) {
 }  // (the dispatcher uses it for RDN only)
 
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
-  auto kern = rdnv ? fwd_tc_kernel<true> : fwd_tc_kernel<false>;
+  const bool generic = p.mods != 0;
+  auto kern = rdnv ? (generic ? fwd_tc_kernel<true, true> : fwd_tc_kernel<true, false>)
+                   : (generic ? fwd_tc_kernel<false, true> : fwd_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kTcSmem);
   if (e != cudaSuccess) return e;

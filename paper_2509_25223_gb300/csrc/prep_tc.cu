@@ -174,6 +174,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
   constexpr float kLog2e = 1.4426950408889634f;
   const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
+  const bool plain = p.mods & RDN_FLAG_PLAIN_COMBINE;
 
   if (tid == 0) {
     mbar_init(bar, 1);
@@ -319,7 +320,9 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
         }
       } else {  // Q K^T row t: Mq (strict), diag(gamma) M2 (inclusive)
         const int t = r - 64;
-        const float ct2 = cum2[t], gtt = gam[t];
+        // (plain combine: S_{t-1} q_t reads Mq decayed to t-1, and the output
+        // has no gamma_t, so the image is M2 itself)
+        const float ct2 = cum2[t], gtt = plain ? 1.f : gam[t], cq2 = plain ? cprev2[t] : ct2;
 #pragma unroll
         for (int c0 = 0; c0 < 32; c0 += 16) {
           const int i0 = 32 * hf + c0;
@@ -332,7 +335,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
             const int i = i0 + u;
             const float qk = p.scale * gv[c0 + u];
             const float dec = i <= t ? exp2f(ct2 - c2[u]) * qk : 0.f;
-            mq[u] = i < t ? dec * bt[u] : 0.f;
+            mq[u] = i < t ? (plain ? exp2f(cq2 - c2[u]) * qk : dec) * bt[u] : 0.f;
             m2[u] = gtt * dec * gm[u];
           }
           img_row16(img + IMG_APMQ, 16384, 64 + t, i0, mq);
