@@ -99,8 +99,9 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *       fitting ablation (Section 4.4): R_t = r_t k_t^T replaces the
  *       recurrence for R, so R0 is ignored (dR0 = 0 unless T = 0) and RT =
  *       r_T k_T^T.
- * These run on the fp32 chunk kernels for every dtype and head dimension
- * (the tensor-core kernels implement the method itself). */
+ * The decayed residual and the plain combine also run on the tensor-core
+ * kernels (bf16, Dk = 128); the tanh residual and the stateless correction
+ * run on the fp32 chunk kernels, for every dtype and head dimension. */
 #define RDN_FLAG_DECAYED_RESIDUAL 0x4u
 #define RDN_FLAG_PLAIN_COMBINE 0x8u
 #define RDN_FLAG_TANH_RESIDUAL 0x10u
