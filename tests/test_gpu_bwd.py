@@ -59,7 +59,7 @@ def _gpu(x, clip, dST=None, dRT=None, variant="rdn", **kw):
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("D", [64, 128])
-@pytest.mark.parametrize("T", [1, 64, 65, 200])
+@pytest.mark.parametrize("T", [1, 2, 7, 8, 63, 64, 65, 200])
 def test_bwd_small(dtype, D, T):
     clip = 1.0
     x = make_inputs(2, T, 2, D, dtype=dtype, nonzero_state=True, with_grad_out=True,

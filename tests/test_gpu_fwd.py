@@ -53,7 +53,7 @@ def test_rla_fwd_f32_workload():
 @pytest.mark.parametrize("variant", ["rdn", "rla"])
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("D", [64, 128])
-@pytest.mark.parametrize("T", [1, 63, 64, 65, 200])
+@pytest.mark.parametrize("T", [1, 2, 3, 7, 8, 63, 64, 65, 200])
 def test_fwd_small(variant, dtype, D, T):
     """Several chunks plus a ragged tail, nonzero initial states."""
     x = make_inputs(2, T, 3, D, dtype=dtype, nonzero_state=True, device="cuda", state_std=0.1)
