@@ -578,7 +578,9 @@ def run_ours(args):
     # bench workload: RDN fwd+bwd with each flag, as the RDN step above
     var = None
     if not args.no_variants:
-        var = {"workload": w.name, "path": "fp32 SIMT chunk kernels", "steps": 1, "flags": {}}
+        var = {"workload": w.name, "steps": 1, "flags": {},
+               "path": "tensor-core kernels for the decayed residual and the plain combine, "
+                       "fp32 chunk kernels for the tanh residual and the stateless correction"}
         wsbv_ = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D,
                                                 variant_flags=rdn.DECAYED_RESIDUAL),
                             dtype=torch.uint8, device=dev)
@@ -586,13 +588,13 @@ def run_ours(args):
                           ("plain_combine", rdn.PLAIN_COMBINE),
                           ("tanh_residual", rdn.TANH_RESIDUAL),
                           ("stateless_aux", rdn.STATELESS_AUX)):
-            def fstep(inp):
+            def fstep(inp):  # (the RDN step's options: chunk states, saved intermediates)
                 _, _, _, Sc_, Rc_ = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
                                                 return_chunk_states=True, out=o, workspace=wsf,
-                                                variant_flags=fl)
+                                                save_for_bwd=True, variant_flags=fl)
                 rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
                             R_chunks=Rc_, workspace=wsbv_, out=grads, fwd_workspace=wsf,
-                            variant_flags=fl)
+                            fwd_saved=True, variant_flags=fl)
             fstep(x)
             torch.cuda.synchronize()
             barrier(dist)
