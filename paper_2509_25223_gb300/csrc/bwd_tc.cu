@@ -1,5 +1,6 @@
 // bwd_tc.cu -- tensor-core (tcgen05 / TMEM) backward of the chunkwise RDN
-// forward, bf16 inputs, d_k = d_v = 128.
+// forward, bf16 inputs, d_k = d_v = 128; RLA (TcBwdParams::rla) and two of
+// the variant flags are runtime modes of separate kernel instances.
 //
 // Reverse mode of the chunk algebra of chunk_fwd.cu (the same steps as
 // chunk_bwd.cu, whose header lists them), split by what depends on the

@@ -1,4 +1,6 @@
-// chunk_bwd.cu -- backward of the chunkwise RLA / RDN forward (fp32 SIMT).
+// chunk_bwd.cu -- backward of the chunkwise RLA / RDN forward (fp32 SIMT:
+// fp32 inputs, d = 64, the tanh residual and the stateless correction), and
+// the dispatcher of both backward paths.
 //
 // Reverse mode of the chunk algebra in chunk_fwd.cu (the paper gives no
 // backward; this is the adjoint of the forward as computed).  Per chunk,
@@ -757,9 +759,8 @@ bool use_tc_bwd(const rdn_fwd_args &f, int variant) {
 // The forward's per-chunk records are valid input when the caller passes the
 // forward's workspace with its chunk-start states and they are in the format
 // this backward reads: shared-memory images where the forward ran the
-// tensor-core scan, read by the tensor-core backward (RDN); fp32 otherwise.
-// (RLA at bf16, d = 128 runs the tensor-core forward and the fp32 backward,
-// which then recomputes its records.)
+// tensor-core scan, read by the tensor-core backward; fp32 otherwise (the
+// two choices agree for every argument set, so the check only guards them).
 bool reuse_fwd_records(const rdn_fwd_args &f, int variant) {
   const FwdParams fp = make_fwd_params(f);
   return f.workspace && f.S_chunks &&

@@ -222,7 +222,6 @@ inline bool fwd_uses_tc(const FwdParams &p, int DK, bool bf16) {
 }
 
 // Tensor-core scan (fwd_tc.cu): bf16 inputs with d_k = d_v = 128.
-bool fwd_tc_supported(const rdn_fwd_args &a);
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s);
 
 // Prep kernel alone; img selects the shared-memory-image record format read

@@ -613,10 +613,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 
 }  // namespace
 
-bool fwd_tc_supported(const rdn_fwd_args &a) {
-  return a.dtype == RDN_BF16 && a.Dk == 128 && a.Dv == 128;
-}  // (the dispatcher uses it for RDN only)
-
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
   const bool generic = p.mods != 0;
   auto kern = rdnv ? (generic ? fwd_tc_kernel<true, true> : fwd_tc_kernel<true, false>)

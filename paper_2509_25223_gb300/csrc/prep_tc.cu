@@ -1,5 +1,5 @@
-// prep_tc.cu -- chunk_prep on the tensor cores for RDN with bf16 inputs and
-// d_k = 128: the state-independent matrices of one 64-token chunk (the UT
+// prep_tc.cu -- chunk_prep on the tensor cores for RDN and RLA with bf16
+// inputs and d_k = 128: the state-independent matrices of one 64-token chunk (the UT
 // form of the delta rule, Section 3.5's chunkwise algorithm; algebra in
 // chunk_fwd.cu's header), written as the shared-memory images the
 // tensor-core scans copy into their operand slots.
