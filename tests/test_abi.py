@@ -226,10 +226,10 @@ def test_binding_rejects_cpu_tensors():
 
 _STRUCTS = {
     "rdn_fwd_args": ("FwdArgs", ["B", "q", "clip", "S0", "scale", "flags", "workspace",
-                                 "workspace_bytes"]),
+                                 "workspace_bytes", "cu_seqlens", "num_seqs"]),
     "rdn_bwd_args": ("BwdArgs", ["fwd", "dO", "dq", "dS0", "dR0", "workspace",
                                  "workspace_bytes"]),
-    "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o"]),
+    "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o", "flags"]),
     "rdn_prologue_args": ("PrologueArgs", ["rows", "D", "dtype", "eps", "x", "y", "dy", "dx"]),
 }
 
@@ -254,6 +254,18 @@ def test_binding_struct_layouts_match_the_header(tmp_path):
         assert got[(cname, "size")] == ctypes.sizeof(st), cname
         for f in fields:
             assert got[(cname, f)] == getattr(st, f).offset, (cname, f)
+
+
+def test_binding_flag_values_match_the_header():
+    """Every RDN_FLAG_* of include/rdn.h has the same value in the binding."""
+    src = open(os.path.join(ROOT, "include", "rdn.h")).read()
+    flags = dict(re.findall(r"#define\s+(RDN_FLAG_\w+)\s+(0x[0-9a-fA-F]+)u", src))
+    assert len(flags) == 6, flags
+    for name, val in flags.items():
+        assert getattr(_abi, name) == int(val, 16), name
+    variants = ("RDN_FLAG_DECAYED_RESIDUAL", "RDN_FLAG_PLAIN_COMBINE", "RDN_FLAG_TANH_RESIDUAL",
+                "RDN_FLAG_STATELESS_AUX")
+    assert _abi.RDN_FLAG_VARIANTS == sum(int(flags[n], 16) for n in variants)
 
 
 def test_prologue_validation():
