@@ -288,3 +288,43 @@ def test_prologue_validation():
     assert lib.rdn_qk_prologue_bwd(ctypes.byref(a), None) == 1
     a.rows = 16
     assert lib.rdn_qk_prologue_bwd(ctypes.byref(a), None) == 1  # dy[0] NULL
+
+
+def test_plain_c_consumer(tmp_path):
+    """A C program that includes only include/rdn.h and links librdn.so uses
+    the boundary without Python: version, sizes and argument validation (no
+    device work, so it runs without a GPU)."""
+    _abi.load()
+    src = r"""
+#include <stdio.h>
+#include <string.h>
+#include "rdn.h"
+int main(void) {
+  rdn_fwd_args a;
+  memset(&a, 0, sizeof a);
+  a.B = 2; a.T = 300; a.H = 4; a.Dk = 128; a.Dv = 128; a.dtype = RDN_BF16;
+  a.clip = 1.0f; a.scale = 1.0f;
+  size_t ws = 0;
+  long long slots = 0;
+  if (rdn_fwd_workspace_size(&a, &ws) != RDN_OK || ws == 0) return 1;
+  if (rdn_chunk_slots(&a, &slots) != RDN_OK || slots != 2 * 4 * 5) return 2;
+  if (rdn_fwd(&a, NULL) != RDN_ERR_INVALID_ARG) return 3;      /* q is NULL */
+  if (strstr(rdn_last_error(), "q is NULL") == NULL) return 4;
+  a.flags = RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_TIED_GAMMA;
+  if (rdn_fwd_workspace_size(&a, &ws) != RDN_OK) return 5;
+  a.flags = 0x40u;
+  if (rdn_fwd_workspace_size(&a, &ws) != RDN_ERR_UNSUPPORTED) return 6;
+  printf("%s\n", rdn_version());
+  return 0;
+}
+"""
+    c = tmp_path / "consumer.c"
+    c.write_text(src)
+    exe = tmp_path / "consumer"
+    libdir = os.path.dirname(_abi.lib_path())
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe),
+                    "-L", libdir, "-l:" + os.path.basename(_abi.lib_path()),
+                    "-Wl,-rpath," + libdir], check=True)
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, (r.returncode, r.stdout, r.stderr)
+    assert r.stdout.startswith("rdn-gb300")
