@@ -91,12 +91,12 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *   RDN_FLAG_DECAYED_RESIDUAL  the residual against the decayed prediction,
  *       r_t = Clip(v_t - a_t S_{t-1} k_t) (the gated-delta error);
  *   RDN_FLAG_PLAIN_COMBINE     the ungated output o_t = S_{t-1} q_t + R_t q_t
- *       (output-combination ablation, Section 4.4);
+ *       (output-combination ablation, Section 4.3);
  *   RDN_FLAG_TANH_RESIDUAL     the log-cosh residual of Appendix B with the
  *       threshold as its scale, r_t = c tanh((v_t - S_{t-1} k_t) / c)
  *       (c = 1 is the paper's tanh; c = INFINITY no limit; c = 0 gives 0);
  *   RDN_FLAG_STATELESS_AUX     the stateless correction of the residual-
- *       fitting ablation (Section 4.4): R_t = r_t k_t^T replaces the
+ *       fitting ablation (Section 4.3): R_t = r_t k_t^T replaces the
  *       recurrence for R, so R0 is ignored (dR0 = 0 unless T = 0) and RT =
  *       r_T k_T^T.
  * The decayed residual and the plain combine also run on the tensor-core
@@ -173,7 +173,7 @@ typedef struct {
  *   fwd.workspace     NULL, or (only together with S_chunks/R_chunks) the
  *                     workspace of the rdn_fwd call that wrote them, READ
  *                     as that forward left it: its per-chunk matrices
- *                     (Section 3.5's T, A and M blocks) are reused instead of
+ *                     (the chunk form's T, A and M blocks) are reused instead of
  *                     recomputed.  fwd.workspace_bytes must be at least
  *                     rdn_fwd_workspace_size(&fwd); the same q, k, g, beta,
  *                     gamma, scale and clip as in that call are the caller's

@@ -23,7 +23,7 @@
  * [d_k][d_v] row-major, so "S k" is sum_i k_i S[i][j].  That is a transpose
  * of storage only.
  *
- * Readings taken where the paper leaves room (each listed in the design doc):
+ * Readings taken where the paper leaves room:
  *  - the residual uses the undecayed S_{t-1} k_t (Section 3.3 and 3.4),
  *    not a_t S_{t-1} k_t;
  *  - the output uses S_{t-1} (before the update) and R_t (after it);
@@ -36,15 +36,15 @@
  * The paper's variants, selected by the `mods` bits of the *_mod entry
  * points (any combination; 0 is the method above):
  *  - ORC_DECAYED: the residual against the decayed prediction,
- *    r_t = Clip(v_t - a_t S_{t-1} k_t) (the gated-delta error; Section 3.2's
- *    table and Section 3.4's discussion of which prediction to fit);
+ *    r_t = Clip(v_t - a_t S_{t-1} k_t) (the gated-delta error; Table 1 of
+ *    Section 2.3 and Section 3.4's discussion of which prediction to fit);
  *  - ORC_PLAIN: the ungated combine o_t = S_{t-1} q_t + R_t q_t (the output
- *    combination ablation, Section 4.4);
+ *    combination ablation, Section 4.3);
  *  - ORC_TANH: the log-cosh residual of Appendix B, read with the threshold
  *    as a scale, r_t = c tanh((v_t - S_{t-1} k_t) / c) (c = 1 is the
  *    paper's tanh; c = inf is no limit, c = 0 is r = 0);
  *  - ORC_STATELESS: the stateless correction of the residual-fitting
- *    ablation (Section 4.4), R_t = r_t k_t^T in place of the recurrence for
+ *    ablation (Section 4.3), R_t = r_t k_t^T in place of the recurrence for
  *    R (R0 unused; RT = r_T k_T^T, or R0 when T = 0).
  *
  * The backward is hand-written reverse-mode through the same token loop

@@ -657,7 +657,6 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
       tmem_st16(tm + lane + T_R4 + c0, y);
       lds16(Gam + c0, x);
       lds16(gamv + c0, w);
-#pragma unroll
       const bool plain = mods & RDN_FLAG_PLAIN_COMBINE;  // (no gamma_t in the output)
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] = p.scale * x[i] * (plain ? 1.f : w[i]) * dO(c0 + i);  // dQR (Q unscaled)

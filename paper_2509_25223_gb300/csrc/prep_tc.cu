@@ -1,7 +1,7 @@
 // prep_tc.cu -- chunk_prep on the tensor cores for RDN and RLA with bf16
 // inputs and d_k = 128: the state-independent matrices of one 64-token chunk (the UT
-// form of the delta rule, Section 3.5's chunkwise algorithm; algebra in
-// chunk_fwd.cu's header), written as the shared-memory images the
+// form of the delta rule over a chunk of Section 3.4's recurrence; algebra
+// in chunk_fwd.cu's header), written as the shared-memory images the
 // tensor-core scans copy into their operand slots.
 //
 // Two persistent CTAs of 256 threads per SM, each walking chunks (the next

@@ -56,7 +56,7 @@ def test_reference_arm_nonzero_rank_does_no_work(monkeypatch):
     assert bench.run_reference(A()) == 0
 
 
-def test_flop_model_matches_survey_figures():
+def test_flop_model_matches_hand_counts():
     import bench
     f = bench.flops_per_token_head(128, 64)
     assert round(f["fwd"]) == 259413

@@ -2,11 +2,11 @@
 checked against what the paper and mathematics fix (CPU only).
 
   DECAYED    residual against the decayed prediction a_t S_{t-1} k_t, the
-             gated-delta error (Section 3.2's table, Section 3.4)
-  PLAIN      ungated combine o_t = S_{t-1} q_t + R_t q_t (Section 4.4, output
+             gated-delta error (Table 1 of Section 2.3, Section 3.4)
+  PLAIN      ungated combine o_t = S_{t-1} q_t + R_t q_t (Section 4.3, output
              combination ablation)
   TANH       log-cosh residual c tanh(x / c) (Appendix B)
-  STATELESS  R_t = r_t k_t^T, no accumulated auxiliary state (Section 4.4,
+  STATELESS  R_t = r_t k_t^T, no accumulated auxiliary state (Section 4.3,
              residual-fitting ablation)
 
 The pins use special cases where a variant must coincide with something
@@ -70,7 +70,7 @@ def test_residual_variants_from_the_base_path(variant, mods):
 
 
 def test_gated_delta_net_identity():
-    """Section 3.2's table: Gated DeltaNet is the stateless correction of the
+    """Table 1 (Section 2.3): Gated DeltaNet is the stateless correction of the
     decayed residual with gamma = beta, so RDN with STATELESS | DECAYED,
     gamma = beta and no clip reads o_t = S_t q_t, the updated base state
     (from the base path on the first t tokens) against q_t."""
