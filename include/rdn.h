@@ -107,6 +107,17 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
 #define RDN_FLAG_TANH_RESIDUAL 0x10u
 #define RDN_FLAG_STATELESS_AUX 0x20u
 
+/* RDN_FLAG_F32_OUT: results in fp32 for bf16 inputs -- the forward's o
+ * (rla_fwd / rdn_fwd) and, given in the backward's fwd.flags, dq, dk, dv
+ * (rla_bwd / rdn_bwd; dO stays in fwd.dtype).  Every accumulation is fp32 in
+ * either case; the flag only skips the final rounding to bf16, so a caller
+ * can compare the computation itself against a reference without the bf16
+ * storage rounding of the results (half a bf16 ulp, 2^-9 relative).
+ * Supported where the tensor-core kernels run (RDN_BF16, Dk = Dv = 128, no
+ * variant flag outside RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE)
+ * and, as a no-op, for RDN_F32; otherwise RDN_ERR_UNSUPPORTED. */
+#define RDN_FLAG_F32_OUT 0x40u
+
 /* Arguments of rla_fwd / rdn_fwd.
  *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
  *                     S0/R0 to ST/RT).
@@ -119,7 +130,7 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *   clip              the threshold c of Section 3.3; INFINITY = no clip;
  *                     c < 0 or NaN -> RDN_ERR_INVALID_ARG.
  *   S0, R0            initial states or NULL (= zero).
- *   o                 output [B,T,H,Dv] in `dtype`.
+ *   o                 output [B,T,H,Dv] in `dtype` (fp32 with RDN_FLAG_F32_OUT).
  *   ST, RT            final states or NULL (= not returned).
  *   S_chunks,R_chunks optional chunk-start states (outputs; NULL = not
  *                     stored).  rdn_bwd can consume them instead of
@@ -183,7 +194,8 @@ typedef struct {
  *                     RDN_FLAG_TIED_GAMMA for tied gates; else 0.
  *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
  *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
- *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype.
+ *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype
+ *                     (all three fp32 with RDN_FLAG_F32_OUT in fwd.flags).
  *   dg, dbeta, dgamma [B,T,H] fp32.  dg is the gradient w.r.t. the
  *                     log-decay g; the gradient w.r.t. alpha is dg / alpha.
  *   dS0, dR0          [B,H,Dk,Dv] fp32, or NULL (= not returned).

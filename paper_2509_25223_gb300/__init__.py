@@ -119,20 +119,22 @@ def _chunk_slots(a):
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
          return_final_state=True, return_chunk_states=False, out=None, workspace=None,
-         save_for_bwd=False, tied_gamma=False, cu_seqlens=None, variant_flags=0):
+         save_for_bwd=False, tied_gamma=False, cu_seqlens=None, variant_flags=0, f32_out=False):
     lib = _abi.load()
     _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
     dev = q.device
     N = _num_seqs(q, cu_seqlens)
-    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    odt = torch.float32 if f32_out else q.dtype
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=odt, device=dev)
     ST = RT = Sc = Rc = None
     if return_final_state:
         ST = torch.empty(N, H, Dk, Dv, dtype=torch.float32, device=dev)
         RT = torch.empty_like(ST)
     flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) \
-        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags \
+        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0)
     a = FwdArgs()
     _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, None, None, scale, flags,
               cu_seqlens)
@@ -182,32 +184,34 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
             fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
-            variant_flags=0):
+            variant_flags=0, f32_out=False):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
     S_chunks/R_chunks: the forward's chunk-start states (return_chunk_states).
     fwd_workspace: with them, the workspace that forward call used, whose
     per-chunk matrices are then reused instead of recomputed.
-    fwd_saved: that forward ran with save_for_bwd=True."""
+    fwd_saved: that forward ran with save_for_bwd=True.
+    f32_out: dq, dk, dv in fp32 for bf16 inputs (RDN_FLAG_F32_OUT); the
+    forward takes the same keyword for o."""
     return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
                 R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
-                variant_flags)
+                variant_flags, f32_out)
 
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
             fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
-            variant_flags=0):
+            variant_flags=0, f32_out=False):
     """Backward of rla_fwd; the same arguments and results as rdn_bwd."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
                 R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
-                variant_flags)
+                variant_flags, f32_out)
 
 
 def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
          workspace, out, fwd_workspace, fwd_saved, tied_gamma=False, cu_seqlens=None,
-         variant_flags=0):
+         variant_flags=0, f32_out=False):
     lib = _abi.load()
     _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
@@ -215,7 +219,9 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
     dev = q.device
     N = _num_seqs(q, cu_seqlens)
     if out is None:
-        out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
+        gdt = torch.float32 if f32_out else q.dtype
+        out = dict(dq=torch.empty_like(q, dtype=gdt), dk=torch.empty_like(k, dtype=gdt),
+                   dv=torch.empty_like(v, dtype=gdt),
                    dg=torch.empty(B, T, H, dtype=torch.float32, device=dev),
                    dbeta=torch.empty(B, T, H, dtype=torch.float32, device=dev),
                    dgamma=torch.empty(B, T, H, dtype=torch.float32, device=dev),
@@ -228,7 +234,8 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
         a.fwd.workspace = _ptr(fwd_workspace)
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
     a.fwd.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if fwd_saved else 0) \
-        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
+        | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags \
+        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0)
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out.get("dgamma"))

@@ -18,6 +18,7 @@ RDN_FLAG_PLAIN_COMBINE = 0x8
 RDN_FLAG_TANH_RESIDUAL = 0x10
 RDN_FLAG_STATELESS_AUX = 0x20
 RDN_FLAG_VARIANTS = 0x3C
+RDN_FLAG_F32_OUT = 0x40  # fp32 results for bf16 inputs
 
 STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "RDN_ERR_CUDA",
           4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}

@@ -110,8 +110,14 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
     if (!aligned16(a->cu_seqlens))
       return fail(RDN_ERR_MISALIGNED, "%s: cu_seqlens is not 16-byte aligned", fn);
   }
-  if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS))
+  if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS |
+                   RDN_FLAG_F32_OUT))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
+  if ((a->flags & RDN_FLAG_F32_OUT) && a->dtype == RDN_BF16 &&
+      !(a->Dk == 128 && !(a->flags & (RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_STATELESS_AUX))))
+    return fail(RDN_ERR_UNSUPPORTED,
+                "%s: RDN_FLAG_F32_OUT with bf16 inputs needs Dk = 128 and the tensor-core "
+                "variants only", fn);
   if (isnan(a->scale) || isinf(a->scale))
     return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
   return check_clip(fn, a->clip);
@@ -147,6 +153,15 @@ rdn_fwd_args untied(const rdn_fwd_args &a) {
   return u;
 }
 
+// The failures RDN_FAULT_INJECT asks for (rdn::fault_injection), after validation.
+rdn_status_t injected(const char *fn) {
+  switch (rdn::fault_injection()) {
+    case 1: return fail(RDN_ERR_WORKSPACE, "%s: workspace check failed (injected)", fn);
+    case 2: return fail(RDN_ERR_CUDA, "%s: launch failed (injected)", fn);
+    default: return RDN_OK;
+  }
+}
+
 rdn_status_t cuda_status(const char *fn, cudaError_t e) {
   if (e == cudaSuccess) return ok();
   return fail(RDN_ERR_CUDA, "%s: CUDA error %d (%s)", fn, (int)e, cudaGetErrorString(e));
@@ -174,6 +189,7 @@ rdn_status_t fwd_common(const char *fn, const rdn_fwd_args *a0, int variant, cud
     if (!aligned16(a->workspace))
       return fail(RDN_ERR_WORKSPACE, "%s: workspace is not 16-byte aligned", fn);
   }
+  if ((st = injected(fn)) != RDN_OK) return st;
   return cuda_status(fn, rdn::launch_fwd(*a, variant, s));
 }
 
@@ -260,6 +276,15 @@ void *g_status_ptr[kMaxDevices] = {};
 }  // extern "C"
 
 namespace rdn {
+int fault_injection() {
+  const char *e = getenv("RDN_FAULT_INJECT");
+  if (!e) return 0;
+  if (!strcmp(e, "workspace")) return 1;
+  if (!strcmp(e, "launch")) return 2;
+  if (!strcmp(e, "device_wait")) return 3;
+  return 0;
+}
+
 int *status_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
@@ -443,6 +468,7 @@ rdn_status_t bwd_common(const char *fn, const rdn_bwd_args *a0, int variant, cud
     if (!aligned16(a->workspace))
       return fail(RDN_ERR_WORKSPACE, "%s: workspace is not 16-byte aligned", fn);
   }
+  if ((st = injected(fn)) != RDN_OK) return st;
   return cuda_status(fn, rdn::launch_bwd(*a, variant, stream));
 }
 }  // namespace

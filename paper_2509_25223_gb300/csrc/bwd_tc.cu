@@ -73,6 +73,7 @@ struct TcBwdParams {
   // gradients of A_beta, A_gamma drop out; the chunk-start state enters the
   // recomputed prediction with a lo part (RLA's S is not contracted)
   bool rla;
+  bool f32g;  // dq, dk, dv stored in fp32 (RDN_FLAG_F32_OUT), else bf16
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
@@ -239,7 +240,7 @@ constexpr uint32_t SA = 0, RA = 32768, B1 = 65536, SLOTA = 98304, SLOTB = 114688
 constexpr uint32_t XE = 147456, XE_LO = 163840, VEC = 180224;
 constexpr uint32_t CTL = VEC + 7 * 64 * 4;
 constexpr uint32_t SLOT = CTL + 48;
-constexpr uint32_t SA_LO = 183296;  // (RLA) S0 - bf16(S0), two 16 KB blocks
+constexpr uint32_t SA_LO = 183296;  // S0 - bf16(S0), two 16 KB blocks
 static_assert(SA_LO >= SLOT + 16 && SA_LO % 1024 == 0, "layout");
 constexpr size_t SMEM = SA_LO + 32768;
 constexpr uint32_t T_D1 = 0, T_D3 = 128, T_X = 256;
@@ -295,7 +296,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       }
       put16(sm + SA, 16384, j, c0, s);
       put16(sm + RA, 16384, j, c0, r);
-      if (P.rla) {
+      {  // S0 - bf16(S0), as the forward scan's read-outs use it
 #pragma unroll
         for (int i = 0; i < 16; ++i) s[i] -= __bfloat162float(__float2bfloat16_rn(s[i]));
         put16(sm + SA_LO, 16384, j, c0, s);
@@ -324,7 +325,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
 
   bool ok = phase_run(K, tid, [&] {  // KS, KR
     mma_tile(tm + T_D1, sb + SA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
-    if (P.rla) mma_tile(tm + T_D1, sb + SA_LO, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), true);
+    mma_tile(tm + T_D1, sb + SA_LO, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), true);
     mma_tile(tm + T_D3, sb + RA, 16384, sb + B1, 16384, 8, idesc_bf16(128, 64), false);
     return true;
   });
@@ -744,6 +745,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
        // (bf16 [t][j]) staged in the free scratch tiles
       float *stg = reinterpret_cast<float *>(sm + S0H);
       __nv_bfloat16 *dvs = reinterpret_cast<__nv_bfloat16 *>(sm + S1H);
+      float *dvs32 = reinterpret_cast<float *>(sm + S1H);  // (fp32 dv: over S1H and S1L)
+      static_assert(S1L == S1H + 16384, "fp32 dv staging spans the pair");
       {
         const int c0 = g16;
         float x[16], dks[16], gm[16];
@@ -755,7 +758,10 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
-          dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
+          if (P.f32g)
+            dvs32[t * D + j] = x[i] - dP[i];
+          else
+            dvs[t * D + j] = __float2bfloat16_rn(x[i] - dP[i]);
           dks[i] = dks[i] * dP[i] - (rla ? 0.f : gm[i] * x[i]);
         }
         put16s(sm + S2H, sm + S2L, j, c0, dks);
@@ -766,11 +772,21 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         bulk_s2g(P.dXbuf + chunk * 64 * D, sm + S0H, 32768);
         bulk_commit();
       }
-      for (int e = tid; e < 64 * 16; e += NTC) {  // dv rows, 16 bytes at a time
-        const int t = e >> 4, chn = e & 15;
-        if (t < n)
-          *reinterpret_cast<uint4 *>(dv + ((size_t)(tok0 + t0 + t) * H + h) * D + chn * 8) =
-              *reinterpret_cast<const uint4 *>(sm + S1H + t * 256 + chn * 16);
+      if (P.f32g) {  // dv rows, 16 bytes at a time
+        float *dvf = (float *)P.dv;
+        for (int e = tid; e < 64 * 32; e += NTC) {
+          const int t = e >> 5, chn = e & 31;
+          if (t < n)
+            *reinterpret_cast<uint4 *>(dvf + ((size_t)(tok0 + t0 + t) * H + h) * D + chn * 4) =
+                *reinterpret_cast<const uint4 *>(sm + S1H + t * 512 + chn * 16);
+        }
+      } else {
+        for (int e = tid; e < 64 * 16; e += NTC) {
+          const int t = e >> 4, chn = e & 15;
+          if (t < n)
+            *reinterpret_cast<uint4 *>(dv + ((size_t)(tok0 + t0 + t) * H + h) * D + chn * 8) =
+                *reinterpret_cast<const uint4 *>(sm + S1H + t * 256 + chn * 16);
+        }
       }
     }
     // ---- phase E: U_S += K^T dKS
@@ -1119,7 +1135,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     float x[16], y[16];
     lds16(dec_res ? Gam + tb : Gprev + tb, x);
     lds16(Gam + tb, y);
-#pragma unroll
     float gq[16];  // the base read-out's gate: Gam (plain combine: Gprev)
     lds16(plain ? Gprev + tb : Gam + tb, gq);
 #pragma unroll
@@ -1501,8 +1516,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         const int t = tb + i;
         if (t < n) {
           const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * D + j;
-          dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
-          dq[off] = __float2bfloat16_rn(scale * qv[i]);
+          if (P.f32g) {
+            ((float *)P.dk)[off] = a[i] + scale * d2[i];
+            ((float *)P.dq)[off] = scale * qv[i];
+          } else {
+            dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
+            dq[off] = __float2bfloat16_rn(scale * qv[i]);
+          }
         }
       }
     }
@@ -1528,9 +1548,10 @@ size_t bwd_tc_extra_bytes(long long nrec) {
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, cudaStream_t s) {
+                          char *extra, bool rla, bool grad_f32, cudaStream_t s) {
   TcBwdParams P;
   P.rla = rla;
+  P.f32g = grad_f32;
   P.dq = dq;
   P.dk = dk;
   P.dg = dg;

@@ -839,6 +839,10 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   char *ws = (char *)a.workspace;
   BwdParams p;
   p.f = make_fwd_params(f);
+  // fp32 results (RDN_FLAG_F32_OUT in fwd.flags) are the backward's dq, dk, dv;
+  // a forward recomputed here keeps its o in fwd.dtype
+  const bool grad_f32 = p.f.f32out != 0;
+  p.f.f32out = 0;
   const bool reuse = reuse_fwd_records(f, variant);
   p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
   p.f.err = status_word();
@@ -889,7 +893,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   if (tc)  // the accumulator words it reads are written by its own kernels
     return launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dq, a.dk, a.dv, a.dg, a.dbeta,
                          a.dgamma, a.dS0, a.dR0, p.acc, ws + l.prep + l.acc + 2 * l.states + l.o,
-                         !rdnv, s);
+                         !rdnv, grad_f32, s);
   if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
   if (rdnv) {
     if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);

@@ -125,6 +125,8 @@ struct FwdParams {
   int nseq;        // sequences: B, or the number of packed sequences
   long long nrec;  // record slots: B * H * NC, or a bound on H * (total chunks)
   unsigned mods;   // the variant flags (RDN_FLAG_VARIANTS bits of rdn_fwd_args.flags)
+  int f32out;      // o stored in fp32 (RDN_FLAG_F32_OUT on the tensor-core forward)
+  int inject;      // 1: the tensor-core scan skips its first MMA completion signal (tests)
 };
 
 // Where sequence s's tokens and (s, h)'s chunk records are.  Token t of the
@@ -208,6 +210,8 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.nseq = call_seqs(a);
   p.nrec = call_records(a);
   p.mods = a.flags & RDN_FLAG_VARIANTS;
+  p.f32out = (a.flags & RDN_FLAG_F32_OUT) && a.dtype == RDN_BF16;
+  p.inject = 0;
   return p;
 }
 
@@ -235,7 +239,7 @@ size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, cudaStream_t s);
+                          char *extra, bool rla, bool grad_f32, cudaStream_t s);
 
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).

@@ -580,6 +580,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
   p.ws = (float *)a.workspace;
   const size_t total = plan_fwd(a, variant).total_bytes;
   p.err = status_word();
+  p.inject = fault_injection() == 3 ? 1 : 0;
   if (a.cu_seqlens) {
     long long *seq = (long long *)((char *)a.workspace + total - 256 - seq_table_bytes(a));
     const cudaError_t e = launch_seq_table(a, seq, s);

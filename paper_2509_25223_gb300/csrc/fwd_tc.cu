@@ -27,10 +27,11 @@
 //
 // RLA skips MMA2 and MMA6 (E = V, E2 = r).  X, E, wS E and their auxiliary
 // counterparts (magnitude ~ |v|) enter the MMAs as bf16 hi + lo pairs, which
-// keeps their rounding well below the state's own scale; the states and the
-// chunk's K, Q are single bf16 (K, Q exactly).  The states S, R live in TMEM
-// in fp32 for the whole sequence; their bf16 copies (the A operands of MMA1
-// and MMA5) are rewritten in shared memory after each update.  The chunk's V
+// keeps their rounding well below the state's own scale; so does S in MMA1
+// (hi + lo copies); R and the chunk's K, Q are single bf16 (K, Q exactly).
+// The states S, R live in TMEM in fp32 for the whole sequence; their bf16
+// copies (the A operands of MMA1 and MMA5) are rewritten in shared memory
+// after each update.  The chunk's V
 // and [K ; Q] tiles are fetched by cp.async while the previous chunk
 // finishes.  One thread issues the MMAs; every wait is an mbarrier wait with
 // a time limit.  The state-independent chunk matrices (T_beta, T_gamma, Ap,
@@ -68,8 +69,8 @@ constexpr uint32_t SM_XE_LO = 180224;  //   lo part
 constexpr uint32_t SM_W = 196608;      // (wS E)^T / (wR E2)^T, hi part
 constexpr uint32_t SM_W_LO = 212992;   //   lo part
 constexpr uint32_t SM_VEC = 229376;    // 7 x 64 fp32: Gam Gprev (unused) wS wR gamma, GamC
-constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;  // 3 mbarriers: MMA, slot A, slot B
-constexpr uint32_t SM_SLOT = SM_BAR + 24;
+constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;  // 4 mbarriers: MMA, slot A, slot B, drain
+constexpr uint32_t SM_SLOT = SM_BAR + 32;
 constexpr uint32_t SM_FLAG = SM_SLOT + 4;
 constexpr uint32_t SM_BYTES = SM_FLAG + 4;
 constexpr size_t kTcSmem = SM_BYTES;
@@ -139,6 +140,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         *gamv = vec + 320;
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + SM_BAR);
   uint64_t *barA = bar + 1, *barB = bar + 2;  // slot A / slot B bulk copies
+  uint64_t *barD = bar + 3;  // the drain after a wait that gave up
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SM_SLOT);
   volatile int *flag = reinterpret_cast<volatile int *>(sm + SM_FLAG);
 
@@ -163,6 +165,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     mbar_init(bar, 1);
     mbar_init(barA, 1);
     mbar_init(barB, 1);
+    mbar_init(barD, 1);
     fence_mbar_init();
     *flag = 0;
   }
@@ -173,16 +176,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const uint32_t tm = *slot;
   const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
   uint32_t phase = 0, phA = 0, phB = 0;  // phA/phB: tracked by thread 0 only
-  // RLA: S - bf16(S) as a bf16 image (rows j; key block 0 in slot A, block 1
-  // in the E^T lo tile: RLA has no T matrices, and the E lo tile is free from
-  // the end of a chunk to the next one's MMA3), so that the read-outs K S,
-  // Q S use S to ~16 bits: RLA's state is not contracted by a delta term and
-  // its prediction S k is a large sum the residual v - S k cancels against
+  bool pendA = false, pendB = false;      // (thread 0) a slot copy armed and not yet waited for
+  // the waits on the MMAs: normally about a second; a test (p.inject) skips the
+  // first phase's completion signal and waits about 5 ms for it instead
+  const long long mma_limit = p.inject ? 10000000ll : 2000000000ll;
+  bool skip_commit = p.inject != 0;
+  // S - bf16(S) as a second bf16 image (rows j), so that the read-outs K S,
+  // Q S use S to ~16 bits.  RLA's state is not contracted by a delta term and
+  // its prediction S k is a large sum the residual v - S k cancels against;
+  // RDN's single-bf16 read-outs put the output error of the long-context
+  // workload (T = 16384) at the 2e-2 RMS bound.  The image lives in tiles that
+  // are free from the end of a chunk to the next one's MMA1 / MMA3: RDN the
+  // X/E^T pair (key blocks 0 | 1), RLA (no T matrices) slot A and the E^T lo tile.
+  constexpr uint32_t kSloBase = RDNV ? SM_XE : SM_SLOTA;
+  constexpr uint32_t kSloBlk = RDNV ? SM_XE_LO - SM_XE : SM_XE_LO - SM_SLOTA;
   auto store_state_lo = [&](int c0, const float (&s)[16]) {
     float lo[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) lo[i] = s[i] - __bfloat162float(__float2bfloat16_rn(s[i]));
-    st_row16(sm + SM_SLOTA, SM_XE_LO - SM_SLOTA, j, c0, lo);
+    st_row16(sm + kSloBase, kSloBlk, j, c0, lo);
   };
   auto rec_of = [&](int c) {
     return reinterpret_cast<const uint8_t *>(p.ws + (size_t)(sp.rbase + c) * kRecFloats);
@@ -191,6 +203,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   auto load_slot = [&](uint8_t *dst, uint64_t *b, const uint8_t *src, uint32_t bytes) {
     mbar_expect_tx(b, bytes);
     bulk_g2s(dst, src, bytes, b);
+    (b == barA ? pendA : pendB) = true;
   };
   if (tid == 0 && NC > 0) {  // (a packed sequence may be empty)
     if (RDNV) load_slot(sm + SM_SLOTA, barA, rec_of(0) + IMG_TB, 16384);
@@ -240,7 +253,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     tmem_st16(tm + lane + T_R + c0, r);
     st_row16(sm + SM_SA, 16384, j, c0, s);
     st_row16(sm + SM_RA, 16384, j, c0, r);
-    if (!RDNV) store_state_lo(c0, s);
+    store_state_lo(c0, s);
     if (p.S_chunks && NC > 0) {  // the first chunk's start states, for the backward
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
@@ -259,10 +272,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (tid == 0) {
       fence_after_sync();
       if (!issue()) *flag = 1;  // a slot's bulk copy did not arrive in time
-      mma_commit(bar);
+      if (!skip_commit) mma_commit(bar);
+      skip_commit = false;
     }
     during();
-    const bool ok = mbar_wait(bar, phase);
+    const bool ok = mbar_wait(bar, phase, mma_limit);
     phase ^= 1u;
     if (!ok) *flag = 1;
     __syncthreads();
@@ -361,9 +375,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       if (p.sv_E2) bulk_wait_read();  // the E2^T tiles of the previous chunk are rewritten next
       mma_tile(tm + T_D1, sbase + SM_SA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
-      if (!RDNV)  // (RLA) + the state's lo part: its prediction carries no delta contraction
-        mma_tile(tm + T_D1, sbase + SM_SLOTA, SM_XE_LO - SM_SLOTA, sbase + SM_KQ, 16384, 8,
-                 idesc_bf16(128, 128), true);
+      // + the state's lo part
+      mma_tile(tm + T_D1, sbase + kSloBase, kSloBlk, sbase + SM_KQ, 16384, 8,
+               idesc_bf16(128, 128), true);
       mma_tile(tm + T_X, sbase + SM_RA, 16384, sbase + SM_KQ, 16384, 8, idesc_bf16(128, 128),
                false);
       return true;
@@ -406,6 +420,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       alive = run_phase([&] {
         if (!mbar_wait(barA, phA)) return false;
         phA ^= 1u;
+        pendA = false;
         mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
                    sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
         return true;
@@ -436,6 +451,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     alive = run_phase([&] {
       if (!mbar_wait(barB, phB)) return false;
       phB ^= 1u;
+      pendB = false;
       mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 16384, idesc_bf16(128, 128), true);
       if (p.sv_E) {  // keep the E^T image (hi | lo) for the backward
@@ -498,6 +514,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       alive = run_phase([&] {
         if (!mbar_wait(barA, phA)) return false;
         phA ^= 1u;
+        pendA = false;
         mma_split3(tm + T_D1, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTA,
                    sbase + SM_SLOTA + 8192, idesc_bf16(128, 64), false);
         return true;
@@ -526,6 +543,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       const uint32_t i64 = idesc_bf16(128, 64);
       if (!mbar_wait(barB, phB)) return false;
       phB ^= 1u;
+      pendB = false;
       // the image is diag(gamma) M2: its product lands on Ob directly
       mma_split3(tm + T_D1 + 64, sbase + SM_XE, sbase + SM_XE_LO, sbase + SM_SLOTB,
                  sbase + SM_SLOTB + 8192, i64, true);
@@ -543,9 +561,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     if (c + 1 < NC) fetch_kq(c + 1);  // K, Q are done with
 
     // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R (= Gam_C R + U2) -> RA
-    // o is staged as a [t][j] bf16 tile in W's place (free after MMA8) and stored
-    // 16 bytes at a time
+    // o is staged as a [t][j] tile in W's place (free after MMA8; bf16, or fp32
+    // over W and its lo part) and stored 16 bytes at a time
     __nv_bfloat16 *ostg = reinterpret_cast<__nv_bfloat16 *>(sm + SM_W);
+    float *ostg32 = reinterpret_cast<float *>(sm + SM_W);
+    static_assert(SM_W_LO == SM_W + 16384, "fp32 o staging spans W and its lo part");
     {
       const int c0 = g16;
       float ob[16], oa[16], gm[16], gv[16];
@@ -556,7 +576,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
         const float gg = plain ? 1.f : gv[i];
-        ostg[t * D + j] = __float2bfloat16_rn(fmaf(gg * gm[i] * p.scale, oa[i], ob[i]));
+        const float ov = fmaf(gg * gm[i] * p.scale, oa[i], ob[i]);
+        if (p.f32out)
+          ostg32[t * D + j] = ov;
+        else
+          ostg[t * D + j] = __float2bfloat16_rn(ov);
       }
     }
     {
@@ -572,8 +596,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         }
       }
     }
-    if (!RDNV) {  // (RLA) the updated state's lo part, for the next chunk's read-outs
-      if (p.sv_E2) {  // (into the E^T lo tile: its bulk store to the saved E2 must be done)
+    {  // the updated state's lo part, for the next chunk's read-outs
+      if (p.sv_E2) {  // (over the E2^T tiles: their bulk store to the saved E2 must be done)
         if (tid == 0) bulk_wait_read();
         __syncthreads();
       }
@@ -583,11 +607,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       store_state_lo(g16 + 64, s1);
     }
     __syncthreads();  // the o tile
-    for (int e = tid; e < 64 * 16; e += kTcThreads) {
-      const int t = e >> 4, ch = e & 15;
-      if (t < n)
-        *reinterpret_cast<uint4 *>(o + ((size_t)(tok0 + t0 + t) * H + h) * D + ch * 8) =
-            *reinterpret_cast<const uint4 *>(sm + SM_W + t * 256 + ch * 16);
+    if (p.f32out) {
+      float *of = (float *)p.o;
+      for (int e = tid; e < 64 * 32; e += kTcThreads) {
+        const int t = e >> 5, ch = e & 31;
+        if (t < n)
+          *reinterpret_cast<uint4 *>(of + ((size_t)(tok0 + t0 + t) * H + h) * D + ch * 4) =
+              *reinterpret_cast<const uint4 *>(sm + SM_W + t * 512 + ch * 16);
+      }
+    } else {
+      for (int e = tid; e < 64 * 16; e += kTcThreads) {
+        const int t = e >> 4, ch = e & 15;
+        if (t < n)
+          *reinterpret_cast<uint4 *>(o + ((size_t)(tok0 + t0 + t) * H + h) * D + ch * 8) =
+              *reinterpret_cast<const uint4 *>(sm + SM_W + t * 256 + ch * 16);
+      }
     }
   }
 
@@ -603,8 +637,21 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         if (p.RT) p.RT[st_base + (size_t)(c0 + i) * D + j] = r[i];
       }
     }
-  } else if (tid == 0 && p.err) {
-    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  } else {
+    // a bounded wait gave up: record it, then let every operation of this CTA
+    // still in flight finish (again with bounded waits) before its shared
+    // memory and TMEM are released -- the MMAs this thread issued (one commit
+    // covers them all), the slot copies armed and not waited for, the
+    // cp.async tile copies and the bulk stores
+    if (tid == 0) {
+      if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+      mma_commit(barD);
+      mbar_wait(barD, 0);
+      if (pendA) mbar_wait(barA, phA);
+      if (pendB) mbar_wait(barB, phB);
+      bulk_wait_all();
+    }
+    cp_async_wait_all();
   }
   fence_before_sync();
   __syncthreads();

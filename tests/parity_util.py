@@ -58,3 +58,28 @@ def assert_close(gpu, ref, dtype, name=""):
     excess = np.abs(g - r) - bound
     assert excess.size == 0 or float(excess.max()) <= 0.0, (name, s)
     return s
+
+
+def excess_count(gpu, ref):
+    """Elements whose error exceeds the plain bound 2e-2 * RMS(ref) (for a
+    bf16-typed result these pass only by its half-ulp store rounding)."""
+    g, r = as64(gpu), as64(ref)
+    rms = float(np.sqrt(np.mean(r * r))) if r.size else 0.0
+    return int((np.abs(g - r) > TOL_BF16_REL * rms + ABS_FLOOR).sum())
+
+
+def record(test, tensor, gpu, ref, **extra):
+    """Append one line of error statistics to the file named by the
+    RDN_PARITY_REPORT environment variable (nothing when it is unset)."""
+    import json
+    import os
+    path = os.environ.get("RDN_PARITY_REPORT")
+    s = err_stats(gpu, ref)
+    s.update(test=test, tensor=tensor, elements=int(np.asarray(as64(ref)).size),
+             beyond_plain_bound=excess_count(gpu, ref),
+             stored_bf16=bool(isinstance(gpu, torch.Tensor) and gpu.dtype == torch.bfloat16),
+             **extra)
+    if path:
+        with open(path, "a") as f:
+            f.write(json.dumps(s) + "\n")
+    return s

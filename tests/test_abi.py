@@ -64,7 +64,17 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(dtype=7)) == 2
     assert _status(fn, _fwd_args(clip=-1.0)) == 1
     assert _status(fn, _fwd_args(clip=float("nan"))) == 1
-    assert _status(fn, _fwd_args(flags=0x40)) == 2
+    assert _status(fn, _fwd_args(flags=0x80)) == 2
+    # fp32 results: bf16 inputs need the tensor-core path (Dk = 128, no tanh /
+    # stateless variant); fp32 inputs take the flag as a no-op (then the call
+    # gets as far as the NULL pointer check)
+    F32 = _abi.RDN_FLAG_F32_OUT
+    assert _status(fn, _fwd_args(flags=F32, Dk=64, Dv=64)) == 2
+    assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_TANH_RESIDUAL)) == 2
+    assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_STATELESS_AUX)) == 2
+    assert _status(fn, _fwd_args(flags=F32)) == 1
+    assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_DECAYED_RESIDUAL)) == 1
+    assert _status(fn, _fwd_args(flags=F32, dtype=_abi.RDN_F32, Dk=64, Dv=64)) == 1
     # tied gates: gamma may be NULL (beta serves as both); the call then gets
     # as far as the workspace check
     tied = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, o=FAKE)
@@ -260,7 +270,7 @@ def test_binding_flag_values_match_the_header():
     """Every RDN_FLAG_* of include/rdn.h has the same value in the binding."""
     src = open(os.path.join(ROOT, "include", "rdn.h")).read()
     flags = dict(re.findall(r"#define\s+(RDN_FLAG_\w+)\s+(0x[0-9a-fA-F]+)u", src))
-    assert len(flags) == 6, flags
+    assert len(flags) == 7, flags
     for name, val in flags.items():
         assert getattr(_abi, name) == int(val, 16), name
     variants = ("RDN_FLAG_DECAYED_RESIDUAL", "RDN_FLAG_PLAIN_COMBINE", "RDN_FLAG_TANH_RESIDUAL",
@@ -312,7 +322,7 @@ int main(void) {
   if (strstr(rdn_last_error(), "q is NULL") == NULL) return 4;
   a.flags = RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_TIED_GAMMA;
   if (rdn_fwd_workspace_size(&a, &ws) != RDN_OK) return 5;
-  a.flags = 0x40u;
+  a.flags = 0x80u;
   if (rdn_fwd_workspace_size(&a, &ws) != RDN_ERR_UNSUPPORTED) return 6;
   printf("%s\n", rdn_version());
   return 0;
@@ -328,3 +338,32 @@ int main(void) {
     r = subprocess.run([str(exe)], capture_output=True, text=True)
     assert r.returncode == 0, (r.returncode, r.stdout, r.stderr)
     assert r.stdout.startswith("rdn-gb300")
+
+
+@pytest.mark.parametrize("fn", ["rdn_fwd", "rla_fwd", "rdn_bwd", "rla_bwd"])
+def test_fault_injection(fn, monkeypatch):
+    """RDN_FAULT_INJECT (host side, no GPU needed): a call that passes argument
+    validation and the workspace check fails as asked -- "workspace" with
+    RDN_ERR_WORKSPACE, "launch" with RDN_ERR_CUDA -- before anything is
+    enqueued, and says that the failure was injected."""
+    lib = _abi.load()
+    ok = dict(q=FAKE, k=FAKE, v=FAKE, g=FAKE, beta=FAKE, gamma=FAKE, o=FAKE)
+    n = ctypes.c_size_t(0)
+    if fn.endswith("_fwd"):
+        a = _fwd_args(**ok)
+        assert lib[fn + "_workspace_size"](ctypes.byref(a), ctypes.byref(n)) == 0
+    else:
+        a = _abi.BwdArgs()
+        a.fwd = _fwd_args(**ok)
+        for f in ("dO", "dq", "dk", "dv", "dg", "dbeta", "dgamma"):
+            setattr(a, f, FAKE)
+        assert lib[fn + "_workspace_size"](ctypes.byref(a), ctypes.byref(n)) == 0
+    a.workspace, a.workspace_bytes = FAKE, n.value
+    for what, status in (("workspace", 5), ("launch", 3)):
+        monkeypatch.setenv("RDN_FAULT_INJECT", what)
+        assert lib[fn](ctypes.byref(a), None) == status, what
+        assert "injected" in lib.rdn_last_error().decode(), what
+    # a too-small workspace is still reported as such (validation comes first)
+    a.workspace_bytes = n.value - 16
+    assert lib[fn](ctypes.byref(a), None) == 5
+    assert "injected" not in lib.rdn_last_error().decode()

@@ -117,8 +117,6 @@ def test_packed_fwd_bitwise_equals_separate_calls(variant, dtype, D):
 @pytest.mark.parametrize("dtype,D", [("bf16", 128), ("f32", 64)])
 @pytest.mark.parametrize("reuse", ["recompute", "chunk_states", "saved"])
 def test_packed_bwd_matches_oracle_per_sequence(variant, dtype, D, reuse):
-    if reuse == "saved" and variant == "rla":
-        pytest.skip("rla_fwd keeps no intermediates")
     clip = 1.0
     v = oracle.RDN if variant == "rdn" else oracle.RLA
     x = _packed(LENS, 2, D, dtype, seed=5)
@@ -127,7 +125,7 @@ def test_packed_bwd_matches_oracle_per_sequence(variant, dtype, D, reuse):
     if reuse != "recompute":
         ws = None
         if reuse == "saved":
-            nbytes = rdn.workspace_bytes("rdn_fwd", 1, x["q"].shape[1], 2, D,
+            nbytes = rdn.workspace_bytes(f"{variant}_fwd", 1, x["q"].shape[1], 2, D,
                                          torch.bfloat16 if dtype == "bf16" else torch.float32,
                                          save_for_bwd=True, cu_seqlens=x["cu"])
             ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
