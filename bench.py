@@ -90,12 +90,15 @@ class ClockSampler:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index):
+    def __init__(self, gpu_index, enabled=True):
         self.gpu = gpu_index
+        self.enabled = enabled
         self.proc = None
         self.path = None
 
     def __enter__(self):
+        if not self.enabled:
+            return self
         fd, self.path = tempfile.mkstemp(prefix="rdn_clocks_", suffix=".csv")
         os.close(fd)
         try:
@@ -118,6 +121,8 @@ class ClockSampler:
         return False
 
     def summary(self):
+        if not self.enabled:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["not sampled (--profile)"]}
         if self.proc is None or not self.path:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         rows = []
@@ -247,6 +252,101 @@ def time_oracle_sample(target_s=15.0, max_heads=None):
                        f"{dt:.1f} s on {min(threads, nh)} OpenMP threads")
 
 
+def cpu_model():
+    """The host CPU's model name, as the OS reports it."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.startswith("Model name:"):
+                return ln.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith("model name"):
+                    return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def time_oracle_configs(target_s=2.0):
+    """The oracle on the other workloads, on the host's cores and on one
+    thread: the forward workloads (one whole-T head per thread, and one head
+    on one thread; rate = heads x T / H / time) and the decode step (a sample
+    of the N sequences, all H heads, for one step, scaled to all of them)."""
+    import oracle
+    from rdn_synthetic import WORKLOADS, make_decode_inputs, make_workload_inputs
+
+    oracle.build()
+    threads = oracle.max_threads()
+    out = {}
+
+    def heads_as_batch(t, nh):
+        t = np.moveaxis(t, 2, 1)
+        t = t.reshape(-1, *t.shape[2:])[:nh]
+        return np.ascontiguousarray(np.expand_dims(t, 2))
+
+    def fwd_rate(w, nh):
+        x = make_workload_inputs(w, seed=3)
+        a = {n: (None if t is None else t.double().numpy()) for n, t in x.items()}
+        nh = min(nh, w.B * w.H)
+        q, k, v, g, be, gm = (heads_as_batch(a[n], nh) for n in ("q", "k", "v", "g", "beta",
+                                                                 "gamma"))
+        st = lambda t: None if t is None else np.ascontiguousarray(
+            t.reshape(-1, 1, *t.shape[2:])[:nh])
+        variant = oracle.RLA if w.op == "rla_fwd" else oracle.RDN
+        t0 = time.perf_counter()
+        oracle.fwd(variant, q, k, v, g, be, gm, w.clip, st(a["S0"]), st(a["R0"]))
+        dt = time.perf_counter() - t0
+        return nh, dt, nh * w.T / w.H / dt  # tokens/s (a token = all H heads)
+
+    for name in ("rla_fwd_f32_B1H2T256D64", "rdn_fwd_bf16_B8H16T2048D128",
+                 "rdn_fwd_bf16_B2H16T16384D128_state"):
+        w = WORKLOADS[name]
+        nh, dt, val = fwd_rate(w, threads)  # one whole-T head per thread
+        oracle.set_threads(1)
+        try:
+            nh1, dt1, val1 = fwd_rate(w, 1)
+        finally:
+            oracle.set_threads(threads)
+        out[name] = {"value": val, "unit": "tokens/s", "cores": min(threads, nh),
+                     "single_thread_value": val1,
+                     "sample": f"fp64 oracle forward of {nh} of the {w.B * w.H} (b,h) heads, "
+                               f"T={w.T} each, {dt:.2f} s; one head on one thread "
+                               f"{dt1:.2f} s (rate = heads x T / H / time)"}
+    wd = WORKLOADS["rdn_decode_N256H16D128"]
+
+    def dec_rate(n_seq):
+        y = make_decode_inputs(n_seq, wd.H, wd.D, steps=1, seed=4)
+        a = {k_: t.double().numpy() for k_, t in y.items()}
+        t0 = time.perf_counter()
+        oracle.decode_step(oracle.RDN, a["q"][0], a["k"][0], a["v"][0], a["g"][0],
+                           a["beta"][0], a["gamma"][0], wd.clip, a["S"], a["R"])
+        return time.perf_counter() - t0
+
+    nseq = 8
+    dt = dec_rate(nseq)
+    nseq = max(1, min(wd.B, int(nseq * target_s / max(dt, 1e-4))))
+    dt = dec_rate(nseq)
+    oracle.set_threads(1)
+    try:
+        dt1 = dec_rate(1)
+    finally:
+        oracle.set_threads(threads)
+    scale = wd.B / nseq
+    out[wd.name] = {"value": 1.0 / (dt * scale), "unit": "steps/s (all 256 x 16 heads)",
+                    "cores": min(threads, nseq * wd.H),
+                    "single_thread_value": 1.0 / (dt1 * wd.B),
+                    "sample": f"one fp64 oracle decode step of {nseq} of the {wd.B} sequences "
+                              f"(x {wd.H} heads), {dt:.3f} s, scaled by {scale:.0f} to all "
+                              f"{wd.B}; one sequence on one thread {dt1:.3f} s, scaled by "
+                              f"{wd.B}"}
+    return out
+
+
 # ------------------------------------------------------------ reference arm
 def run_reference(args):
     ws, rank, _ = dist_env()
@@ -374,7 +474,7 @@ def run_ours(args):
     barrier(dist)
     stream = torch.cuda.current_stream()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
+    with ClockSampler(local, enabled=not args.profile) as clk:
         with rdn.LaunchTimer() as lt:
             torch.cuda.synchronize()
             e0.record(stream)
@@ -409,59 +509,61 @@ def run_ours(args):
     # device, where a training step's optimizer uses them); the copies run on
     # their own streams, so that step i + 1's inputs arrive and step i's output
     # leaves while a step computes (two device buffer sets, ordered by events).
-    host = {n: x[n].cpu().pin_memory() for n in names + ("dO",)}
-    dev_in = [{n: torch.empty_like(x[n]) for n in host} for _ in range(2)]
-    outs = [(torch.empty_like(o), {n: torch.empty_like(t) for n, t in grads.items()})
-            for _ in range(2)]
-    host_out = {"o": torch.empty(o.shape, dtype=o.dtype, pin_memory=True)}
-    h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
-    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-    ev = lambda: torch.cuda.Event()
-    in_ready, in_free = [ev(), ev()], [ev(), ev()]
-    out_ready, out_free = [ev(), ev()], [ev(), ev()]
+    e2e_val = h2d = d2h = e2e_steps = None
+    if not args.profile:  # (profiler captures time the step alone)
+        host = {n: x[n].cpu().pin_memory() for n in names + ("dO",)}
+        dev_in = [{n: torch.empty_like(x[n]) for n in host} for _ in range(2)]
+        outs = [(torch.empty_like(o), {n: torch.empty_like(t) for n, t in grads.items()})
+                for _ in range(2)]
+        host_out = {"o": torch.empty(o.shape, dtype=o.dtype, pin_memory=True)}
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        ev = lambda: torch.cuda.Event()
+        in_ready, in_free = [ev(), ev()], [ev(), ev()]
+        out_ready, out_free = [ev(), ev()], [ev(), ev()]
 
-    def e2e_step(i):
-        bsel = i % 2
-        with torch.cuda.stream(s_in):
+        def e2e_step(i):
+            bsel = i % 2
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(in_free[bsel])
+                for n, t in host.items():
+                    dev_in[bsel][n].copy_(t, non_blocking=True)
+                in_ready[bsel].record(s_in)
+            oo, gg = outs[bsel]
+            stream.wait_event(in_ready[bsel])
             if i >= 2:
-                s_in.wait_event(in_free[bsel])
-            for n, t in host.items():
-                dev_in[bsel][n].copy_(t, non_blocking=True)
-            in_ready[bsel].record(s_in)
-        oo, gg = outs[bsel]
-        stream.wait_event(in_ready[bsel])
-        if i >= 2:
-            stream.wait_event(out_free[bsel])
-        _, _, _, Sc, Rc = rdn.rdn_fwd(*(dev_in[bsel][n] for n in names), clip=w.clip,
-                                      return_chunk_states=True, out=oo, workspace=wsf,
-                                      save_for_bwd=True)
-        rdn.rdn_bwd(*(dev_in[bsel][n] for n in names), dev_in[bsel]["dO"], clip=w.clip,
-                    S_chunks=Sc, R_chunks=Rc, workspace=wsb, out=gg, fwd_workspace=wsf,
-                    fwd_saved=True)
-        in_free[bsel].record(stream)
-        out_ready[bsel].record(stream)
-        with torch.cuda.stream(s_out):
-            s_out.wait_event(out_ready[bsel])
-            for n, t in host_out.items():
-                t.copy_(oo if n == "o" else gg[n], non_blocking=True)
-            out_free[bsel].record(s_out)
+                stream.wait_event(out_free[bsel])
+            _, _, _, Sc, Rc = rdn.rdn_fwd(*(dev_in[bsel][n] for n in names), clip=w.clip,
+                                          return_chunk_states=True, out=oo, workspace=wsf,
+                                          save_for_bwd=True)
+            rdn.rdn_bwd(*(dev_in[bsel][n] for n in names), dev_in[bsel]["dO"], clip=w.clip,
+                        S_chunks=Sc, R_chunks=Rc, workspace=wsb, out=gg, fwd_workspace=wsf,
+                        fwd_saved=True)
+            in_free[bsel].record(stream)
+            out_ready[bsel].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(out_ready[bsel])
+                for n, t in host_out.items():
+                    t.copy_(oo if n == "o" else gg[n], non_blocking=True)
+                out_free[bsel].record(s_out)
 
-    # (steady state of the two-deep pipeline: the first input copy and the last
-    # output read are not overlapped with compute, so they are spread over
-    # at least 30 steps, as over the many steps of a training run)
-    e2e_steps = max(30, min(args.steps, 60))
-    for i in range(2):
-        e2e_step(i)
-    torch.cuda.synchronize()
-    barrier(dist)
-    e0.record(s_in)
-    for i in range(e2e_steps):
-        e2e_step(i)
-    e1.record(s_out)
-    torch.cuda.synchronize()
-    barrier(dist)
-    _, e2e_val = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * e2e_steps)
+        # (steady state of the two-deep pipeline: the first input copy and the last
+        # output read are not overlapped with compute, so they are spread over
+        # at least 30 steps, as over the many steps of a training run)
+        e2e_steps = max(30, min(args.steps, 60))
+        for i in range(2):
+            e2e_step(i)
+        torch.cuda.synchronize()
+        barrier(dist)
+        e0.record(s_in)
+        for i in range(e2e_steps):
+            e2e_step(i)
+        e1.record(s_out)
+        torch.cuda.synchronize()
+        barrier(dist)
+        _, e2e_val = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * e2e_steps)
 
     # ---- decode: N=256, H=16, D=128, 1000 steps in place
     dec = None
@@ -693,6 +795,8 @@ def run_ours(args):
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = time_oracle_sample(target_s=args.cpu_seconds)
+        cpu["cpu_model"] = cpu_model()
+        cpu["configs"] = time_oracle_configs()
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws,
@@ -739,10 +843,16 @@ def main(argv=None):
     ap.add_argument("--no-variants", action="store_true")
     ap.add_argument("--no-forward", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="for profiler captures: the timed step only -- no clock sampler, "
+                         "end-to-end leg, CPU baseline or other workloads")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")
     ap.add_argument("--T", type=int, default=0, help="override T (profiling captures only)")
     args = ap.parse_args(argv)
+    if args.profile:
+        args.no_decode = args.no_rla = args.no_prologue = args.no_varlen = True
+        args.no_variants = args.no_forward = args.no_cpu_baseline = True
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":

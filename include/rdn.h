@@ -326,7 +326,18 @@ rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
  * the outputs of that call are then invalid.  rdn_device_status waits for
  * `stream`, returns in *status the code recorded since the previous query
  * (RDN_OK if none) and clears it.  The word is shared by all streams of the
- * device. */
+ * device.
+ * Device state held by the library: the status word and the built-in
+ * scratch of rdn_fwd_noalloc are device variables whose addresses the
+ * library looks up once per device and keeps for the life of the process.
+ * cudaDeviceReset on a device invalidates them: after a reset, do not call
+ * the library on that device again in the same process.
+ * Test instrumentation: with the environment variable RDN_FAULT_INJECT set
+ * to "workspace" or "launch", the forward and backward entry points fail
+ * with RDN_ERR_WORKSPACE or RDN_ERR_CUDA after validating their arguments,
+ * before enqueueing anything; with "device_wait" the tensor-core forward
+ * scan (bf16, Dk = 128) makes its first bounded wait give up, records
+ * RDN_ERR_TIMEOUT here and drains its work in flight. */
 rdn_status_t rdn_device_status(rdn_stream_t stream, int *status);
 
 /* Number of Dk x Dv blocks in each of S_chunks and R_chunks:

@@ -22,12 +22,13 @@ pytestmark = pytest.mark.gpu
 NAMES = ("q", "k", "v", "g", "beta", "gamma")
 
 
-def _noalloc(x, clip=1.0):
+def _noalloc(x, clip=1.0, cu=None):
     """Call rdn_fwd_noalloc through the C ABI; no workspace is passed."""
     lib = _abi.load()
     B, T, H, D = x["q"].shape
+    N = B if cu is None else cu.numel() - 1
     o = torch.empty(B, T, H, D, dtype=x["q"].dtype, device=x["q"].device)
-    ST = torch.empty(B, H, D, D, device=x["q"].device)
+    ST = torch.empty(N, H, D, D, device=x["q"].device)
     RT = torch.empty_like(ST)
     a = _abi.FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
@@ -39,6 +40,8 @@ def _noalloc(x, clip=1.0):
     a.S0, a.R0 = p(x["S0"]), p(x["R0"])
     a.o, a.ST, a.RT = p(o), p(ST), p(RT)
     a.workspace, a.workspace_bytes = None, 0
+    if cu is not None:
+        a.cu_seqlens, a.num_seqs = p(cu), N
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     st = lib.rdn_fwd_noalloc(ctypes.byref(a), stream)
     assert st == 0, lib.rdn_last_error().decode()
@@ -46,18 +49,40 @@ def _noalloc(x, clip=1.0):
     return o, ST, RT
 
 
-def test_noalloc_matches_rdn_fwd_two_calls_in_a_row():
-    # two different problems back to back: the second call must not see the
-    # first one's leftovers in the shared scratch
-    for seed, (B, T, H, D) in ((0, (2, 300, 4, 128)), (1, (1, 130, 3, 64))):
+def _compare(x, dtype, cu=None, what=""):
+    o, ST, RT = _noalloc(x, cu=cu)
+    kw = {} if cu is None else dict(cu_seqlens=cu)
+    o2, ST2, RT2 = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"], **kw)
+    torch.cuda.synchronize()
+    assert_close(o, o2.float().cpu().double().numpy(), dtype, f"{what} o")
+    assert_close(ST, ST2.cpu().double().numpy(), "f32", f"{what} ST")
+    assert_close(RT, RT2.cpu().double().numpy(), "f32", f"{what} RT")
+
+
+def test_noalloc_matches_rdn_fwd_call_after_call():
+    """Problems of growing size back to back -- a small one, a larger one,
+    another of that size on new inputs (every scratch word it reads was left
+    by the previous call), then exactly the largest the scratch holds
+    (1 x 12 heads x 67 chunks = 804 chunk records) -- then packed sequences
+    (whose table sits after the records) and fp32 inputs: each must equal
+    rdn_fwd on the same inputs."""
+    cases = [((1, 130, 3, 64), 0), ((2, 300, 4, 128), 1), ((2, 300, 4, 128), 2),
+             ((1, 67 * 64, 12, 128), 3)]
+    for (B, T, H, D), seed in cases:
         x = make_inputs(B, T, H, D, dtype="bf16", nonzero_state=True, device="cuda",
                         seed=seed, state_std=0.1)
-        o, ST, RT = _noalloc(x)
-        o2, ST2, RT2 = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"])
-        torch.cuda.synchronize()
-        assert_close(o, o2.float().cpu().double().numpy(), "bf16", "o")
-        assert_close(ST, ST2.cpu().double().numpy(), "f32", "ST")
-        assert_close(RT, RT2.cpu().double().numpy(), "f32", "RT")
+        _compare(x, "bf16", what=f"B{B} T{T} H{H} D{D}")
+    # packed sequences: lengths 70, 0, 130, 64 (an empty one and a ragged tail)
+    lens = [70, 0, 130, 64]
+    x = make_inputs(1, sum(lens), 2, 128, dtype="bf16", device="cuda", seed=4)
+    gen = torch.Generator(device="cpu").manual_seed(15)
+    for n in ("S0", "R0"):
+        x[n] = (0.1 * torch.randn(len(lens), 2, 128, 128, generator=gen)).cuda()
+    cu = torch.tensor([0, 70, 70, 200, 264], dtype=torch.int32, device="cuda")
+    _compare(x, "bf16", cu=cu, what="packed")
+    x = make_inputs(2, 150, 2, 64, dtype="f32", nonzero_state=True, device="cuda", seed=5,
+                    state_std=0.1)
+    _compare(x, "f32", what="fp32")
 
 
 def test_noalloc_rejects_problems_beyond_its_scratch():
@@ -70,6 +95,10 @@ def test_noalloc_rejects_problems_beyond_its_scratch():
     assert lib.rdn_fwd_noalloc(ctypes.byref(a), None) == 5
     msg = lib.rdn_last_error().decode()
     assert "built-in scratch" in msg and "804" in msg
+    # one chunk record beyond it: 1 x 5 heads x 161 chunks = 805
+    a.B, a.T, a.H = 1, 161 * 64, 5
+    assert lib.rdn_fwd_noalloc(ctypes.byref(a), None) == 5
+    assert "805 chunk records" in lib.rdn_last_error().decode()
 
 
 def test_noalloc_rejects_the_save_for_backward_flag():
