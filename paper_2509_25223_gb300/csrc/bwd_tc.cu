@@ -74,6 +74,12 @@ struct TcBwdParams {
   // recomputed prediction with a lo part (RLA's S is not contracted)
   bool rla;
   bool f32g;  // dq, dk, dv stored in fp32 (RDN_FLAG_F32_OUT), else bf16
+  // tensor maps (CUtensorMap, 64-byte aligned) over k, q, dO as [tokens][H][D]
+  // with a 64-token x 64-column box (make_tile_map); tma: they are valid
+  alignas(64) unsigned char map_k[128];
+  alignas(64) unsigned char map_q[128];
+  alignas(64) unsigned char map_do[128];
+  bool tma;
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
@@ -443,7 +449,7 @@ constexpr uint32_t T_DS = 0, T_DR = 128, T_R1 = 256, T_R2 = 320, T_R3 = 384, T_R
 // kGeneric: the RLA mode and the variant flags (TcBwdParams::rla, FwdParams::mods)
 // are read; the RDN method's instance has them folded away
 template <bool kGeneric>
-__global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
+__global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant__ TcBwdParams P) {
   using namespace ch;
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sb = smem_u32(sm);
@@ -589,6 +595,27 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     fetch_do(NC - 1);
     pre = fetch_pre(NC - 1);
   }
+  // Chunks before the last are whole 64-token chunks: with tensor maps, thread 0
+  // brings their dO (after phase D) and K, Q (after phase E) tiles by tiled bulk
+  // copies, all on one phase of barrier C; the last chunk, which may be ragged,
+  // is fetched above by cp.async with zero fill.
+  const bool tma = P.tma;
+  uint32_t tma_ph = 0;    // phases of barrier C waited for
+  uint32_t tma_arms = 0;  // (thread 0) phases armed, and of those seen complete
+  uint32_t tma_seen = 0;
+  auto tma_do = [&](int cc) {  // (thread 0) arms barrier C for the whole chunk
+    const int row = (int)(tok0 + (long long)cc * 64);
+    ++tma_arms;
+    mbar_expect_tx(K.barC, 49152);
+    for (int kb = 0; kb < 2; ++kb) tma_load_3d(sm + DOT + kb * 8192, P.map_do, 64 * kb, h, row, K.barC);
+  };
+  auto tma_kq = [&](int cc) {
+    const int row = (int)(tok0 + (long long)cc * 64);
+    for (int kb = 0; kb < 2; ++kb) {
+      tma_load_3d(sm + KQ + kb * 16384, P.map_k, 64 * kb, h, row, K.barC);
+      tma_load_3d(sm + KQ + kb * 16384 + 8192, P.map_q, 64 * kb, h, row, K.barC);
+    }
+  };
 
   bool ok = true;
   for (int c = NC - 1; c >= 0 && ok; --c) {
@@ -610,7 +637,18 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     const float GamC = pre.gamc;
     const unsigned m = pre.m;  // bit i: clip inactive at t = g16 + i
     cp_async_wait_all();  // this chunk's tiles (fetched during the previous one)
+    if (tma && c < NC - 1) {  // (by tiled bulk copies)
+      if (mbar_wait(K.barC, tma_ph & 1u))
+        tma_seen = tma_ph + 1;
+      else
+        *K.flag = 1;
+      ++tma_ph;
+    }
     __syncthreads();
+    if (*K.flag) {
+      ok = false;
+      break;
+    }
     auto dO = [&](int t) {  // dO[t, j] from the tile
       return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
           sm + DOT + (j >> 6) * 8192 + sw128(t, j & 63)));
@@ -740,7 +778,12 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     });
     if (!ok) break;
     if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
-    if (c > 0) fetch_do(c - 1);  // every thread is past its last read of this chunk's dO
+    if (c > 0) {  // every thread is past its last read of this chunk's dO
+      if (!tma)
+        fetch_do(c - 1);
+      else if (tid == 0)
+        tma_do(c - 1);
+    }
     {  // dX -> dv = -dP + dX ; dKS = Gprev dP - Gam dX; dX (fp32 [t][j]) and dv
        // (bf16 [t][j]) staged in the free scratch tiles
       float *stg = reinterpret_cast<float *>(sm + S0H);
@@ -799,7 +842,10 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
     });
     if (!ok) break;
     if (c > 0) {  // the next chunk's inputs, while this one finishes
-      fetch_kq(c - 1);
+      if (!tma)
+        fetch_kq(c - 1);
+      else if (tid == 0)
+        tma_kq(c - 1);
       pre = fetch_pre(c - 1);
     }
     // the carried gradients' tiles (dS, dR complete in TMEM): the A operands of
@@ -824,9 +870,12 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(TcBwdParams P) {
         if (P.dR0) P.dR0[st_base + (size_t)(c0 + i) * D + j] = r[i];
       }
     }
-  } else if (tid == 0 && p.err) {
-    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  } else if (tid == 0) {
+    if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+    // no copy into this CTA's shared memory outlives it (bounded waits)
+    for (; tma_seen < tma_arms; ++tma_seen) mbar_wait(K.barC, tma_seen & 1u);
   }
+  cp_async_wait_all();
   if (tid == 0) bulk_wait_all();
   fence_before_sync();
   __syncthreads();
@@ -1575,6 +1624,10 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.dXbuf = x + 3 * nct * 64 * D;
   P.gimg = reinterpret_cast<uint8_t *>(x + 4 * nct * 64 * D);
   P.mask = reinterpret_cast<unsigned long long *>(P.gimg + nct * 131072);
+  // the chain's tiles of whole chunks by tensor-map copies (else cp.async)
+  const long long rows = (long long)f.B * f.T;
+  P.tma = make_tile_map(P.map_k, f.k, D, f.H, rows) && make_tile_map(P.map_q, f.q, D, f.H, rows) &&
+          make_tile_map(P.map_do, dO, D, f.H, rows);
   const bool saved = f.sv_E && f.sv_E2 && f.sv_mask;  // E, E2, mask kept by the forward
   if (saved) {
     P.Ebuf = f.sv_E;

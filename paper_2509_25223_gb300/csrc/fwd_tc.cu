@@ -42,6 +42,9 @@
 //
 // TMEM (512 columns): [0,128) S   [128,256) R   [256,384) D1   [384,512) D3
 // (D1 holds KS|QS, then E | Ob, Gprev KS + Ap E = P | Ob, then E2 | Ob + gamma M2 E2).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "chunk_common.cuh"
 #include "tc_common.cuh"
 
@@ -659,6 +662,37 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
 }
 
 }  // namespace
+
+namespace {
+// the driver's tensor-map encoder, looked up once through the runtime (no
+// link against the driver library)
+PFN_cuTensorMapEncodeTiled_v12000 tile_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      f = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }();
+  return fn;
+}
+}  // namespace
+
+bool make_tile_map(void *map128, const void *base, int D, int H, long long rows) {
+  static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
+  const auto enc = tile_map_encoder();
+  if (!enc || !base || rows < 1) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)rows};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};  // bytes, dims 1, 2
+  const cuuint32_t box[3] = {64, 1, 64};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(reinterpret_cast<CUtensorMap *>(map128), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+             const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
   const bool generic = p.mods != 0;

@@ -70,6 +70,21 @@ __device__ __forceinline__ void bulk_g2s(void *dst_smem, const void *src_gmem, u
       : "memory");
 }
 
+// Tiled (tensor-map) bulk copy global -> shared of a 3-D box at coordinates
+// (c0, c1, c2), innermost first; completion is signalled on `bar` as
+// transaction bytes.  `map` is the address of a CUtensorMap in kernel
+// parameter space (a __grid_constant__ parameter).  The destination is
+// 1024-byte aligned for the 128-byte swizzled layout; c0 times the element
+// size is a multiple of 16 bytes.
+__device__ __forceinline__ void tma_load_3d(void *dst_smem, const void *map, int c0, int c1,
+                                            int c2, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst_smem)),
+      "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // Hints that bring global memory closer ahead of its use (no completion to
 // wait for; the later loads find the lines cached): into L2, a contiguous
 // range (16-byte aligned address and size) or the 128-byte line of one address.
@@ -535,4 +550,11 @@ __device__ __forceinline__ void mma_tile(uint32_t d_tmem, uint32_t a_base, uint3
 }
 
 }  // namespace tc
+
+// Host: a tensor map over a token-major bf16 tensor [rows][H][D] (q, k, v, dO:
+// rows = B*T tokens) whose box is 64 tokens x 1 head x 64 columns, landing in
+// shared memory as a K-major 128-byte swizzled tile of 64 rows (8 KB): the
+// layout the tensor-core kernels' operand tiles use.  Out-of-range rows read
+// as zero.  Returns false if the driver's encoder is unavailable or refuses.
+bool make_tile_map(void *map128, const void *base, int D, int H, long long rows);
 }  // namespace rdn
