@@ -792,6 +792,42 @@ def run_ours(args):
                "l2": "no flush: 268 MB of q, k per pass, larger than L2"}
         del dq_, dk_, yq_, yk_
 
+        # the same map inside the library (RDN_FLAG_QK_NORM): the RDN step
+        # above with q, k taken as raw projections -- the forward's per-chunk
+        # pass normalises the rows it loads; the backward leaves dq, dk in
+        # fp32 and one streaming pass applies the map's Jacobian
+        wsfq = torch.empty(rdn.workspace_bytes("rdn_fwd", B, T, H, D, save_for_bwd=True,
+                                               qk_norm=True), dtype=torch.uint8, device=dev)
+
+        def qstep(inp):
+            _, _, _, Sc_, Rc_ = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
+                                            return_chunk_states=True, out=o, workspace=wsfq,
+                                            save_for_bwd=True, qk_norm=True)
+            rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
+                        R_chunks=Rc_, workspace=wsb, out=grads, fwd_workspace=wsfq,
+                        fwd_saved=True, qk_norm=True)
+
+        qsteps = max(3, args.steps)
+        for _ in range(3):
+            qstep(x)
+        torch.cuda.synchronize()
+        barrier(dist)
+        with rdn.LaunchTimer() as ltq:
+            e0.record(stream)
+            for _ in range(qsteps):
+                qstep(x)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        barrier(dist)
+        tq, qval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step * qsteps)
+        pro["fused_step"] = {
+            "workload": w.name + " with RDN_FLAG_QK_NORM", "value": qval, "unit": "tokens/s",
+            "steps": qsteps, "ms_per_step": tq / qsteps,
+            "overhead_ms_vs_step": tq / qsteps - ms_per_step,
+            "separate_passes_ms": mf + mb,
+            "kernels": {k: {"launches": n, "mean_ms": m} for k, (n, t, m) in ltq.summary().items()}}
+        del wsfq
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = time_oracle_sample(target_s=args.cpu_seconds)

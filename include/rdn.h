@@ -118,6 +118,21 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  * and, as a no-op, for RDN_F32; otherwise RDN_ERR_UNSUPPORTED. */
 #define RDN_FLAG_F32_OUT 0x40u
 
+/* RDN_FLAG_QK_NORM (rla_fwd / rdn_fwd, and in the backward's fwd.flags): q
+ * and k are the raw projections x, and the library applies the activation and
+ * normalisation of rdn_qk_prologue to them itself, per row of Dk elements
+ *     y = SiLU(x) / max(||SiLU(x)||_2, qk_eps),
+ * before the recurrence; the backward returns dq and dk with respect to x
+ * (the map's transposed Jacobian applied to the gradients w.r.t. y).  On the
+ * tensor-core path (RDN_BF16, Dk = Dv = 128) the forward's per-chunk pass
+ * normalises the rows it loads and keeps y (bf16) in the workspace for the
+ * scan and the backward, and the backward's final kernel applies the
+ * Jacobian as it writes dq and dk; elsewhere the rdn_qk_prologue kernels run
+ * as passes of their own.  Needs qk_eps > 0 and finite (else
+ * RDN_ERR_INVALID_ARG); *_fwd_workspace_size and *_bwd_workspace_size grow
+ * by the normalised copies (2 B T H Dk elements of dtype). */
+#define RDN_FLAG_QK_NORM 0x80u
+
 /* Arguments of rla_fwd / rdn_fwd.
  *   B, T, H           batch, tokens, heads; B, H >= 1, T >= 0 (T = 0 copies
  *                     S0/R0 to ST/RT).
@@ -137,7 +152,9 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *                     recomputing.
  *   scale             multiplies q (the paper uses 1).
  *   flags             0, or RDN_FLAG_SAVE_FOR_BWD and / or
- *                     RDN_FLAG_TIED_GAMMA and the variant flags (above).
+ *                     RDN_FLAG_TIED_GAMMA, the variant flags,
+ *                     RDN_FLAG_F32_OUT, RDN_FLAG_QK_NORM (above).
+ *   qk_eps            (last field) norm floor for RDN_FLAG_QK_NORM.
  *   workspace         device scratch of *_fwd_workspace_size() bytes.
  *   cu_seqlens        NULL, or packed variable-length sequences: a device
  *                     int32 array of num_seqs + 1 token offsets, 0 =
@@ -173,6 +190,7 @@ typedef struct {
   size_t workspace_bytes;
   const int *cu_seqlens;
   int num_seqs;
+  float qk_eps; /* the norm floor of RDN_FLAG_QK_NORM; ignored without it */
 } rdn_fwd_args;
 
 /* Arguments of rdn_bwd.  `fwd` holds the forward's inputs (its o, ST, RT,
@@ -191,7 +209,9 @@ typedef struct {
  *                     responsibility (not checked).  It is only read.
  *   fwd.flags         RDN_FLAG_SAVE_FOR_BWD if that forward ran with it
  *                     (then fwd.workspace is required), and
- *                     RDN_FLAG_TIED_GAMMA for tied gates; else 0.
+ *                     RDN_FLAG_TIED_GAMMA for tied gates, the variant
+ *                     flags, RDN_FLAG_F32_OUT and RDN_FLAG_QK_NORM (with
+ *                     fwd.qk_eps) as the forward had them; else 0.
  *   dO                upstream gradient of o, [B,T,H,Dv] in fwd.dtype.
  *   dST, dRT          upstream gradients of ST, RT, or NULL (= 0).
  *   dq, dk            [B,T,H,Dk] in fwd.dtype;  dv [B,T,H,Dv] in fwd.dtype

@@ -119,7 +119,8 @@ def _chunk_slots(a):
 
 def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
          return_final_state=True, return_chunk_states=False, out=None, workspace=None,
-         save_for_bwd=False, tied_gamma=False, cu_seqlens=None, variant_flags=0, f32_out=False):
+         save_for_bwd=False, tied_gamma=False, cu_seqlens=None, variant_flags=0, f32_out=False,
+         qk_norm=False, qk_eps=1e-12):
     lib = _abi.load()
     _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
@@ -134,10 +135,11 @@ def _fwd(name, q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0,
         RT = torch.empty_like(ST)
     flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) \
         | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags \
-        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0)
+        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0) | (_abi.RDN_FLAG_QK_NORM if qk_norm else 0)
     a = FwdArgs()
     _fill_fwd(a, q, k, v, g, beta, gamma, clip, S0, R0, o, ST, RT, None, None, scale, flags,
               cu_seqlens)
+    a.qk_eps = float(qk_eps)
     if return_chunk_states:
         if cu_seqlens is None:
             NC = (T + CHUNK - 1) // CHUNK
@@ -177,14 +179,18 @@ def rdn_fwd(q, k, v, g, beta, gamma, clip=1.0, S0=None, R0=None, scale=1.0, **kw
 
     cu_seqlens (int32 device tensor of N+1 offsets, q of shape [1,T,H,D]):
     N packed sequences, each with its own recurrence; S0, R0, ST, RT are then
-    [N,H,D,D] and the chunk states [slots,D,D] (rdn_fwd_args.cu_seqlens)."""
+    [N,H,D,D] and the chunk states [slots,D,D] (rdn_fwd_args.cu_seqlens).
+
+    qk_norm: q and k are the raw projections x; the library applies
+    y = SiLU(x) / max(||SiLU(x)||, qk_eps) per row first (RDN_FLAG_QK_NORM;
+    the backward takes the same keywords and returns dq, dk w.r.t. x)."""
     return _fwd("rdn_fwd", q, k, v, g, beta, gamma, clip, S0, R0, scale, **kw)
 
 
 def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
             fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
-            variant_flags=0, f32_out=False):
+            variant_flags=0, f32_out=False, qk_norm=False, qk_eps=1e-12):
     """Backward of rdn_fwd.  Returns a dict with dq, dk, dv (input dtype),
     dg (w.r.t. the log-decay), dbeta, dgamma (fp32), dS0, dR0 (fp32).
 
@@ -193,25 +199,27 @@ def rdn_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, d
     per-chunk matrices are then reused instead of recomputed.
     fwd_saved: that forward ran with save_for_bwd=True.
     f32_out: dq, dk, dv in fp32 for bf16 inputs (RDN_FLAG_F32_OUT); the
-    forward takes the same keyword for o."""
+    forward takes the same keyword for o.
+    qk_norm, qk_eps: as given to the forward (RDN_FLAG_QK_NORM): q, k are the
+    raw x and dq, dk are returned w.r.t. x."""
     return _bwd("rdn_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
                 R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
-                variant_flags, f32_out)
+                variant_flags, f32_out, qk_norm, qk_eps)
 
 
 def rla_bwd(q, k, v, g, beta, gamma, dO, clip=1.0, S0=None, R0=None, dST=None, dRT=None,
             scale=1.0, S_chunks=None, R_chunks=None, workspace=None, out=None,
             fwd_workspace=None, fwd_saved=False, tied_gamma=False, cu_seqlens=None,
-            variant_flags=0, f32_out=False):
+            variant_flags=0, f32_out=False, qk_norm=False, qk_eps=1e-12):
     """Backward of rla_fwd; the same arguments and results as rdn_bwd."""
     return _bwd("rla_bwd", q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks,
                 R_chunks, workspace, out, fwd_workspace, fwd_saved, tied_gamma, cu_seqlens,
-                variant_flags, f32_out)
+                variant_flags, f32_out, qk_norm, qk_eps)
 
 
 def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chunks, R_chunks,
          workspace, out, fwd_workspace, fwd_saved, tied_gamma=False, cu_seqlens=None,
-         variant_flags=0, f32_out=False):
+         variant_flags=0, f32_out=False, qk_norm=False, qk_eps=1e-12):
     lib = _abi.load()
     _check_variant_flags(variant_flags)
     B, T, H, Dk = q.shape
@@ -235,7 +243,8 @@ def _bwd(name, q, k, v, g, beta, gamma, dO, clip, S0, R0, dST, dRT, scale, S_chu
         a.fwd.workspace_bytes = fwd_workspace.numel() * fwd_workspace.element_size()
     a.fwd.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if fwd_saved else 0) \
         | (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags \
-        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0)
+        | (_abi.RDN_FLAG_F32_OUT if f32_out else 0) | (_abi.RDN_FLAG_QK_NORM if qk_norm else 0)
+    a.fwd.qk_eps = float(qk_eps)
     a.dO, a.dST, a.dRT = _ptr(dO), _ptr(dST), _ptr(dRT)
     a.dq, a.dk, a.dv = _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"])
     a.dg, a.dbeta, a.dgamma = _ptr(out["dg"]), _ptr(out["dbeta"]), _ptr(out.get("dgamma"))
@@ -364,17 +373,19 @@ class LaunchTimer:
 
 
 def workspace_bytes(op, B, T, H, D, dtype=torch.bfloat16, save_for_bwd=False, cu_seqlens=None,
-                    variant_flags=0):
+                    variant_flags=0, qk_norm=False):
     """Workspace size the library asks for (op: rla_fwd | rdn_fwd | rla_bwd | rdn_bwd);
     cu_seqlens: the packed-sequence table of the call (B = 1); variant_flags:
-    the variant bits of the call."""
+    the variant bits of the call; qk_norm: the call normalises q, k."""
     lib = _abi.load()
     a = FwdArgs()
     a.B, a.T, a.H, a.Dk, a.Dv = B, T, H, D, D
     a.dtype = _abi.RDN_BF16 if dtype == torch.bfloat16 else _abi.RDN_F32
     a.clip, a.scale = 1.0, 1.0
     _check_variant_flags(variant_flags)
-    a.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) | variant_flags
+    a.flags = (_abi.RDN_FLAG_SAVE_FOR_BWD if save_for_bwd else 0) | variant_flags \
+        | (_abi.RDN_FLAG_QK_NORM if qk_norm else 0)
+    a.qk_eps = 1e-12
     if cu_seqlens is not None:
         a.cu_seqlens, a.num_seqs = _ptr(cu_seqlens), cu_seqlens.numel() - 1
     n = ctypes.c_size_t(0)

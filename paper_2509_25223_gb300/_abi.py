@@ -19,6 +19,7 @@ RDN_FLAG_TANH_RESIDUAL = 0x10
 RDN_FLAG_STATELESS_AUX = 0x20
 RDN_FLAG_VARIANTS = 0x3C
 RDN_FLAG_F32_OUT = 0x40  # fp32 results for bf16 inputs
+RDN_FLAG_QK_NORM = 0x80  # q, k are raw x: SiLU + L2 normalisation applied in the library
 
 STATUS = {0: "RDN_OK", 1: "RDN_ERR_INVALID_ARG", 2: "RDN_ERR_UNSUPPORTED", 3: "RDN_ERR_CUDA",
           4: "RDN_ERR_TIMEOUT", 5: "RDN_ERR_WORKSPACE", 6: "RDN_ERR_MISALIGNED"}
@@ -42,7 +43,7 @@ class FwdArgs(ctypes.Structure):
                 ("ST", P), ("RT", P), ("S_chunks", P), ("R_chunks", P),
                 ("scale", ctypes.c_float), ("flags", ctypes.c_uint),
                 ("workspace", P), ("workspace_bytes", ctypes.c_size_t),
-                ("cu_seqlens", P), ("num_seqs", ctypes.c_int)]
+                ("cu_seqlens", P), ("num_seqs", ctypes.c_int), ("qk_eps", ctypes.c_float)]
 
 
 class BwdArgs(ctypes.Structure):

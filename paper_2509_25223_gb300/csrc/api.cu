@@ -111,8 +111,11 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
       return fail(RDN_ERR_MISALIGNED, "%s: cu_seqlens is not 16-byte aligned", fn);
   }
   if (a->flags & ~(RDN_FLAG_SAVE_FOR_BWD | RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS |
-                   RDN_FLAG_F32_OUT))
+                   RDN_FLAG_F32_OUT | RDN_FLAG_QK_NORM))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
+  if ((a->flags & RDN_FLAG_QK_NORM) && !(a->qk_eps > 0.f && !isinf(a->qk_eps)))
+    return fail(RDN_ERR_INVALID_ARG, "%s: RDN_FLAG_QK_NORM needs qk_eps > 0 and finite (got %g)",
+                fn, a->qk_eps);
   if ((a->flags & RDN_FLAG_F32_OUT) && a->dtype == RDN_BF16 &&
       !(a->Dk == 128 && !(a->flags & (RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_STATELESS_AUX))))
     return fail(RDN_ERR_UNSUPPORTED,

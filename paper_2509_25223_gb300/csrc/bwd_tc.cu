@@ -73,7 +73,8 @@ struct TcBwdParams {
   // gradients of A_beta, A_gamma drop out; the chunk-start state enters the
   // recomputed prediction with a lo part (RLA's S is not contracted)
   bool rla;
-  bool f32g;  // dq, dk, dv stored in fp32 (RDN_FLAG_F32_OUT), else bf16
+  bool f32g;    // dq, dk, dv stored in fp32 (RDN_FLAG_F32_OUT), else bf16
+  bool f32qk;   // dq, dk stored in fp32 whatever f32g (for a step that follows)
   // tensor maps (CUtensorMap, 64-byte aligned) over k, q, dO as [tokens][H][D]
   // with a 64-token x 64-column box (make_tile_map); tma: they are valid
   alignas(64) unsigned char map_k[128];
@@ -1565,7 +1566,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         const int t = tb + i;
         if (t < n) {
           const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * D + j;
-          if (P.f32g) {
+          if (P.f32qk) {
             ((float *)P.dk)[off] = a[i] + scale * d2[i];
             ((float *)P.dq)[off] = scale * qv[i];
           } else {
@@ -1597,10 +1598,11 @@ size_t bwd_tc_extra_bytes(long long nrec) {
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, bool grad_f32, cudaStream_t s) {
+                          char *extra, bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s) {
   TcBwdParams P;
   P.rla = rla;
   P.f32g = grad_f32;
+  P.f32qk = grad_f32 || dqk_f32;
   P.dq = dq;
   P.dk = dk;
   P.dg = dg;

@@ -58,6 +58,9 @@ struct BwdParams {
   void *dq, *dk, *dv;
   float *dg, *dbeta, *dgamma, *dS0, *dR0;
   float *acc;  // [B*H*NC] accumulator records
+  // RDN_FLAG_QK_NORM with bf16 inputs: dq, dk (w.r.t. the normalised q, k)
+  // stored here in fp32 for the normalisation's backward; else NULL
+  float *gq32, *gk32;
 };
 
 // ---------------------------------------------------------------- kernel 1
@@ -681,8 +684,15 @@ __global__ void __launch_bounds__(kScanThreads, 1) bwd_finish_kernel(BwdParams p
       const int t = MM::row(i), d = MM::col();
       if (t < n) {
         const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * DK + d;
-        dk[off] = from_f32<InT>(acc[L::DKo + t * DK + d] + a1[i] + a2[i]);
-        dq[off] = from_f32<InT>(p.f.scale * (acc[L::DQo + t * DK + d] + a3[i]));
+        const float gk = acc[L::DKo + t * DK + d] + a1[i] + a2[i];
+        const float gq = p.f.scale * (acc[L::DQo + t * DK + d] + a3[i]);
+        if (p.gq32) {
+          p.gk32[off] = gk;
+          p.gq32[off] = gq;
+        } else {
+          dk[off] = from_f32<InT>(gk);
+          dq[off] = from_f32<InT>(gq);
+        }
       }
     }
   }
@@ -746,7 +756,7 @@ cudaError_t launch_t(const BwdParams &p, cudaStream_t s) {
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct BwdLayout {
-  size_t prep, acc, states, o, tc, tied, seq, total;
+  size_t prep, acc, states, o, tc, qk, g32, tied, seq, total;
 };
 
 // bf16 inputs with d = 128 take the tensor-core backward (RDN, and RLA with
@@ -781,13 +791,21 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
   l.tc = tc ? align256(bwd_tc_extra_bytes(nrec)) : 0;
+  // normalised q, k (RDN_FLAG_QK_NORM), unless the forward's workspace has them
+  l.qk = reuse_fwd_records(f, variant) ? 0 : align256(qk_norm_bytes(f));
+  // and, with bf16 inputs, dq, dk (w.r.t. the normalised q, k) in fp32 for
+  // the normalisation's backward: its projection (dy - y <y, dy>) would
+  // otherwise start from bf16-rounded dy
+  l.g32 = (f.flags & RDN_FLAG_QK_NORM) && f.dtype == RDN_BF16
+              ? align256(2 * sizeof(float) * (size_t)f.B * f.T * f.H * f.Dk)
+              : 0;
   l.seq = seq_table_bytes(f);
   // tied gates without a dgamma buffer: the gamma part is made here, then added
   l.tied = (f.flags & RDN_FLAG_TIED_GAMMA) && !a.dgamma
                ? align256(sizeof(float) * (size_t)f.B * f.T * f.H)
                : 0;
   // + the packed-sequence table and a 256-byte tail
-  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.tied + l.seq + 256;
+  l.total = l.prep + l.acc + 2 * l.states + l.o + l.tc + l.qk + l.g32 + l.tied + l.seq + 256;
   return l;
 }
 
@@ -852,6 +870,9 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
     if (e != cudaSuccess) return e;
     p.f.seq = seq;
   }
+  if (p.f.qk_norm)  // the normalised q, k: the forward's, or made with this call's records
+    set_qk_norm_copies(p.f, f, reuse ? (char *)f.workspace + qk_norm_offset(f)
+                                     : ws + l.prep + l.acc + 2 * l.states + l.o + l.tc);
   if (reuse && (f.flags & RDN_FLAG_SAVE_FOR_BWD)) {  // E, E2 and the mask kept by the forward
     const SavedLayout sl = saved_layout((size_t)p.f.nrec, f.Dv);
     p.f.sv_E = (uint8_t *)f.workspace + sl.e;
@@ -890,17 +911,46 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   p.dgamma = a.dgamma;
   p.dS0 = a.dS0;
   p.dR0 = a.dR0;
-  if (tc)  // the accumulator words it reads are written by its own kernels
-    return launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, a.dq, a.dk, a.dv, a.dg, a.dbeta,
-                         a.dgamma, a.dS0, a.dR0, p.acc, ws + l.prep + l.acc + 2 * l.states + l.o,
-                         !rdnv, grad_f32, s);
-  if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
-  if (rdnv) {
-    if (f.Dk == 128) return bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
-    return bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
+  p.gq32 = p.gk32 = nullptr;
+  if (l.g32) {
+    p.gq32 = (float *)(ws + l.prep + l.acc + 2 * l.states + l.o + l.tc + l.qk);
+    p.gk32 = p.gq32 + (size_t)f.B * f.T * f.H * f.Dk;
   }
-  if (f.Dk == 128) return bf ? launch_t<128, false, __nv_bfloat16>(p, s) : launch_t<128, false, float>(p, s);
-  return bf ? launch_t<64, false, __nv_bfloat16>(p, s) : launch_t<64, false, float>(p, s);
+  if (tc) {  // the accumulator words it reads are written by its own kernels
+    // (with the normalisation: dq, dk into the fp32 copies, as fp32 results)
+    e = launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, p.gq32 ? p.gq32 : a.dq,
+                      p.gk32 ? p.gk32 : a.dk, a.dv, a.dg, a.dbeta, a.dgamma, a.dS0, a.dR0, p.acc,
+                      ws + l.prep + l.acc + 2 * l.states + l.o, !rdnv, grad_f32,
+                      p.gq32 != nullptr, s);
+  } else {
+    if ((e = cudaMemsetAsync(p.acc, 0, l.acc, s)) != cudaSuccess) return e;
+    if (rdnv) {
+      if (f.Dk == 128) e = bf ? launch_t<128, true, __nv_bfloat16>(p, s) : launch_t<128, true, float>(p, s);
+      else e = bf ? launch_t<64, true, __nv_bfloat16>(p, s) : launch_t<64, true, float>(p, s);
+    } else {
+      if (f.Dk == 128) e = bf ? launch_t<128, false, __nv_bfloat16>(p, s) : launch_t<128, false, float>(p, s);
+      else e = bf ? launch_t<64, false, __nv_bfloat16>(p, s) : launch_t<64, false, float>(p, s);
+    }
+  }
+  if (e != cudaSuccess || !p.f.qk_norm) return e;
+  // dq, dk w.r.t. the caller's x: the normalisation's transposed Jacobian, in place
+  rdn_prologue_args pa{};
+  pa.rows = (long long)f.B * f.T * f.H;
+  pa.D = f.Dk;
+  pa.dtype = f.dtype;
+  pa.eps = f.qk_eps;
+  pa.x[0] = f.q;
+  pa.x[1] = f.k;
+  pa.dx[0] = a.dq;
+  pa.dx[1] = a.dk;
+  if (p.gq32) {  // from the fp32 copies
+    pa.dy[0] = p.gq32;
+    pa.dy[1] = p.gk32;
+    return launch_prologue_bwd_f32dy(pa, grad_f32, s);
+  }
+  pa.dy[0] = a.dq;
+  pa.dy[1] = a.dk;
+  return launch_prologue(pa, true, s);
 }
 
 }  // namespace rdn

@@ -127,6 +127,12 @@ struct FwdParams {
   unsigned mods;   // the variant flags (RDN_FLAG_VARIANTS bits of rdn_fwd_args.flags)
   int f32out;      // o stored in fp32 (RDN_FLAG_F32_OUT on the tensor-core forward)
   int inject;      // 1: the tensor-core scan skips its first MMA completion signal (tests)
+  // RDN_FLAG_QK_NORM: q and k above are then the normalised copies
+  // SiLU(x) / max(||SiLU(x)||, qk_eps), written by the pass that makes the
+  // chunk records (launch_t in chunk_fwd.cu), and qraw, kraw the caller's x
+  const void *qraw, *kraw;
+  float qk_eps;
+  int qk_norm;
 };
 
 // Where sequence s's tokens and (s, h)'s chunk records are.  Token t of the
@@ -212,7 +218,32 @@ inline FwdParams make_fwd_params(const rdn_fwd_args &a) {
   p.mods = a.flags & RDN_FLAG_VARIANTS;
   p.f32out = (a.flags & RDN_FLAG_F32_OUT) && a.dtype == RDN_BF16;
   p.inject = 0;
+  p.qraw = a.q;
+  p.kraw = a.k;
+  p.qk_eps = a.qk_eps;
+  p.qk_norm = (a.flags & RDN_FLAG_QK_NORM) ? 1 : 0;
   return p;
+}
+
+// RDN_FLAG_QK_NORM: the normalised q, then k, [tokens][H][Dk] in dtype, at
+// qk_norm_offset bytes into the forward's workspace (after the records and
+// the saved intermediates) and in the backward's when it makes its own records.
+inline size_t qk_norm_bytes(const rdn_fwd_args &a) {
+  if (!(a.flags & RDN_FLAG_QK_NORM)) return 0;
+  const size_t esz = a.dtype == RDN_BF16 ? 2 : 4;
+  return 2 * esz * (size_t)a.B * a.T * a.H * a.Dk;  // (a multiple of 256)
+}
+inline size_t qk_norm_offset(const rdn_fwd_args &a) {
+  const size_t nrec = (size_t)call_records(a);
+  size_t off = sizeof(float) * (size_t)kRecFloats * nrec;
+  if (a.flags & RDN_FLAG_SAVE_FOR_BWD) off += saved_layout(nrec, a.Dv).bytes;
+  return off;
+}
+// Points p.q, p.k at the normalised copies starting at `base`.
+inline void set_qk_norm_copies(FwdParams &p, const rdn_fwd_args &a, char *base) {
+  const size_t half = qk_norm_bytes(a) / 2;
+  p.q = base;
+  p.k = base + half;
 }
 
 // The variant flags the tensor-core kernels implement (the others run on the
@@ -239,7 +270,7 @@ size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
                           float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, bool grad_f32, cudaStream_t s);
+                          char *extra, bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s);
 
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).

@@ -436,9 +436,24 @@ cudaError_t launch_t(const FwdParams &p, cudaStream_t s, bool do_prep, bool do_s
                                 (int)scan_smem<DK>())) != cudaSuccess)
     return e;
   if (do_prep) {
-    // the images for bf16 inputs and d = 128 come from the tensor-core prep
+    // the images for bf16 inputs and d = 128 come from the tensor-core prep,
+    // which also normalises q and k (RDN_FLAG_QK_NORM) as it loads them; for
+    // the other preps the prologue kernel writes the normalised copies first
     constexpr bool tc_prep = DK == 128 && std::is_same<InT, __nv_bfloat16>::value;
-    if (tc_prep && img && (p.mods & ~kTcVariants) == 0) {
+    const bool use_tc_prep = tc_prep && img && (p.mods & ~kTcVariants) == 0;
+    if (p.qk_norm && !use_tc_prep) {
+      rdn_prologue_args pa{};
+      pa.rows = (long long)p.B * p.T * p.H;
+      pa.D = DK;
+      pa.dtype = std::is_same<InT, __nv_bfloat16>::value ? RDN_BF16 : RDN_F32;
+      pa.eps = p.qk_eps;
+      pa.x[0] = p.qraw;
+      pa.x[1] = p.kraw;
+      pa.y[0] = const_cast<void *>(p.q);
+      pa.y[1] = const_cast<void *>(p.k);
+      if ((e = launch_prologue(pa, false, s)) != cudaSuccess) return e;
+    }
+    if (use_tc_prep) {
       if ((e = launch_prep_tc(p, !RDNV, s)) != cudaSuccess) return e;
     } else {
       RDN_LAUNCH("chunk_prep", s, prep<<<(unsigned)p.nrec, kThreads, prep_smem<DK>(), s>>>(p));
@@ -558,10 +573,11 @@ FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   pl.NC = (a.T + C - 1) / C;
   pl.prep_bytes = sizeof(float) * (size_t)kRecFloats;
   const size_t nrec = (size_t)call_records(a);
-  // per-chunk records, the saved intermediates if asked for, the packed-
-  // sequence table, then a 256-byte tail
+  // per-chunk records, the saved intermediates if asked for, the normalised
+  // q, k (RDN_FLAG_QK_NORM), the packed-sequence table, then a 256-byte tail
   pl.total_bytes = pl.prep_bytes * nrec + seq_table_bytes(a) + 256;
   if (a.flags & RDN_FLAG_SAVE_FOR_BWD) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
+  pl.total_bytes += qk_norm_bytes(a);  // (after those: qk_norm_offset)
   return pl;
 }
 
@@ -593,6 +609,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
     p.sv_E2 = (uint8_t *)a.workspace + l.e2;
     p.sv_mask = (unsigned long long *)((char *)a.workspace + l.mask);
   }
+  if (p.qk_norm) set_qk_norm_copies(p, a, (char *)a.workspace + qk_norm_offset(a));
   return launch_fwd_parts(p, a.Dk, variant == 1, a.dtype == RDN_BF16, true, true, s);
 }
 

@@ -72,6 +72,9 @@ void end(cudaStream_t s);
 namespace rdn {
 cudaError_t launch_decode(const rdn_decode_args &a, cudaStream_t s);
 cudaError_t launch_prologue(const rdn_prologue_args &a, bool bwd, cudaStream_t s);
+// The prologue's backward with dy in fp32 whatever a.dtype (x in a.dtype; dx
+// in a.dtype, or fp32 when f32dx).
+cudaError_t launch_prologue_bwd_f32dy(const rdn_prologue_args &a, bool f32dx, cudaStream_t s);
 
 // Sequences and record slots of a call: B sequences of T tokens with B * H *
 // ceil(T/64) records, or num_seqs packed sequences whose sum over s of

@@ -171,7 +171,11 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H = p.H;
   const size_t nct = (size_t)total_records(p);
-  const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k;
+  // the rows loaded: the caller's q, k, or with RDN_FLAG_QK_NORM their raw x,
+  // normalised here (and the results stored to the copies p.q, p.k)
+  const bool qkn = p.qk_norm != 0;
+  const __nv_bfloat16 *q = (const __nv_bfloat16 *)(qkn ? p.qraw : p.q);
+  const __nv_bfloat16 *k = (const __nv_bfloat16 *)(qkn ? p.kraw : p.k);
   constexpr float kLog2e = 1.4426950408889634f;
   const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
   const bool plain = p.mods & RDN_FLAG_PLAIN_COMBINE;
@@ -218,6 +222,60 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
     }
     return x;
   };
+  // RDN_FLAG_QK_NORM: y = SiLU(x) / max(||SiLU(x)||, eps) for the 128 rows of
+  // the [K ; Q] tile in place (thread (row, half): 64 of a row's 128
+  // elements in registers, the pair's sums of squares combined by a
+  // shuffle; zero rows past the end stay zero).  The sigmoid is the prologue
+  // kernel's, so that both paths give the same y up to the order of the sum.
+  auto normalize_rows = [&]() {
+    const int r = tid >> 1, hh = tid & 1;  // row (K rows 0..63, Q rows 64..127), column half
+    uint8_t *blk = sm + KQ + hh * 16384;
+    float u[64];  // SiLU(x), this thread's half row
+    float ss = 0.f;
+#pragma unroll
+    for (int c8 = 0; c8 < 8; ++c8) {
+      const uint4 w = *reinterpret_cast<const uint4 *>(blk + sw128(r, 8 * c8));
+      const __nv_bfloat16 *b = reinterpret_cast<const __nv_bfloat16 *>(&w);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float x = __bfloat162float(b[e]);
+        u[8 * c8 + e] = x * __fdividef(1.f, 1.f + __expf(-x));
+        ss = fmaf(u[8 * c8 + e], u[8 * c8 + e], ss);
+      }
+    }
+    ss += __shfl_xor_sync(0xffffffffu, ss, 1);
+    const float inv = 1.f / fmaxf(sqrtf(ss), p.qk_eps);
+#pragma unroll
+    for (int c8 = 0; c8 < 8; ++c8) {
+      uint4 w;
+      uint32_t *wv = reinterpret_cast<uint32_t *>(&w);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 o2 =
+            __floats2bfloat162_rn(u[8 * c8 + 2 * e] * inv, u[8 * c8 + 2 * e + 1] * inv);
+        wv[e] = *reinterpret_cast<const uint32_t *>(&o2);
+      }
+      *reinterpret_cast<uint4 *>(blk + sw128(r, 8 * c8)) = w;
+    }
+  };
+  // ... and the valid rows of y from the tile to the normalised copies, 16
+  // bytes a thread, whole rows per half warp (after a barrier; while the Gram
+  // product reads the same tile)
+  auto store_rows = [&](size_t ck) {
+    int s_, h_, cc_;
+    rec_decode(p, (long long)ck, s_, h_, cc_);
+    const SeqSpan sp_ = seq_span(p, s_, h_);
+    const int t0_ = cc_ * C, n_ = min(C, sp_.len - t0_);
+    for (int e = tid; e < 128 * 16; e += NTH) {
+      const int r = e >> 4, chn = e & 15, t = r & 63;
+      if (t >= n_) continue;
+      const uint4 w = *reinterpret_cast<const uint4 *>(sm + KQ + (chn >> 3) * 16384 +
+                                                       sw128(r, (chn & 7) * 8));
+      __nv_bfloat16 *dst = (__nv_bfloat16 *)(r < 64 ? p.k : p.q) +
+                           ((size_t)(sp_.tok0 + t0_ + t) * H + h_) * D + chn * 8;
+      *reinterpret_cast<uint4 *>(dst) = w;
+    }
+  };
   Gates gt{0.f, 0.f, 0.f};
   if (blockIdx.x < nct) {
     fetch_kq(blockIdx.x);
@@ -238,6 +296,10 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
       gam[tid] = gt.m;
     }
     cp_async_wait_all();  // this chunk's K, Q
+    if (qkn) {
+      __syncthreads();  // (every thread's copies landed)
+      normalize_rows();
+    }
     fence_async_smem();
     fence_before_sync();
     __syncthreads();  // (also: every thread is done with the previous chunk)
@@ -246,6 +308,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
       mma_tile(tm, sb + KQ, 16384, sb + KQ, 16384, 8, idesc_bf16(128, 64), false);
       mma_commit(bar);
     }
+    if (qkn) store_rows(chunk);  // (while the product runs)
     if (warp == 0) {  // in-chunk cumulative log-decay, while the product runs
       float a = gg[lane], a2 = gg[32 + lane];
 #pragma unroll

@@ -117,7 +117,9 @@ struct ProP {
   void *o[2];  // y (forward) or dx (backward)
 };
 
-template <typename InT, int D, bool BWD>
+// GT, OT: the element types of dy and of dx (InT, or fp32 for gradients the
+// library keeps in fp32 before this step, and for fp32 results)
+template <typename InT, int D, bool BWD, typename GT = InT, typename OT = InT>
 __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
   // elements per lane: one 16-byte access (the backward, which holds x and
   // dy, one warp per row: D / 32 elements per lane, fewer registers)
@@ -126,24 +128,27 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
   constexpr int RPW = 32 / LPR;              // rows per warp access
   constexpr int ROWS = kRowsInFlight * RPW;  // rows a warp has in flight
   using V = Vec<InT, E>;
+  using VG = Vec<GT, E>;
+  using VO = Vec<OT, E>;
   const int lane = threadIdx.x & 31, sub = lane / LPR, li = lane % LPR;
   const long long warp = ((long long)blockIdx.x * kProThreads + threadIdx.x) >> 5;
   const long long nwarps = ((long long)gridDim.x * kProThreads) >> 5;
   const InT *X = reinterpret_cast<const InT *>(p.x[blockIdx.y]);
-  const InT *DY = reinterpret_cast<const InT *>(p.dy[blockIdx.y]);
-  InT *O = reinterpret_cast<InT *>(p.o[blockIdx.y]);
+  const GT *DY = reinterpret_cast<const GT *>(p.dy[blockIdx.y]);
+  OT *O = reinterpret_cast<OT *>(p.o[blockIdx.y]);
   for (long long base = warp * ROWS; base < p.rows; base += nwarps * ROWS) {
-    typename V::Raw xr[kRowsInFlight], gr[kRowsInFlight];  // packed until used
+    typename V::Raw xr[kRowsInFlight];  // packed until used
+    typename VG::Raw gr[kRowsInFlight];
     // the loads of all rows first
 #pragma unroll
     for (int u = 0; u < kRowsInFlight; ++u) {
       const long long r = base + u * RPW + sub;
       xr[u] = typename V::Raw{};
-      gr[u] = typename V::Raw{};
+      gr[u] = typename VG::Raw{};
       if (r < p.rows) {
         const size_t off = (size_t)r * D + li * E;
         xr[u] = V::ldr(X + off);
-        if (BWD) gr[u] = V::ldr(DY + off);
+        if (BWD) gr[u] = VG::ldr(DY + off);
       }
     }
 #pragma unroll
@@ -151,7 +156,7 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
       const long long r = base + u * RPW + sub;  // (rows past the end: computed, not stored)
       float x[E], g[E], s[E], uu[E], ss = 0.f;
       V::unpack(xr[u], x);
-      if (BWD) V::unpack(gr[u], g);
+      if (BWD) VG::unpack(gr[u], g);
 #pragma unroll
       for (int e = 0; e < E; ++e) {
         s[e] = __fdividef(1.f, 1.f + __expf(-x[e]));  // (2-ulp divide: issue-bound loop)
@@ -176,12 +181,12 @@ __global__ void __launch_bounds__(kProThreads) prologue_kernel(ProP p) {
           out[e] = du * s[e] * (1.f + x[e] * (1.f - s[e]));
         }
       }
-      if (r < p.rows) V::st(O + (size_t)r * D + li * E, out);
+      if (r < p.rows) VO::st(O + (size_t)r * D + li * E, out);
     }
   }
 }
 
-template <typename InT, int D>
+template <typename InT, int D, typename GT = InT, typename OT = InT>
 cudaError_t launch_t(const ProP &p, bool bwd, cudaStream_t s) {
   int dev = 0, nsm = 0;
   cudaError_t e;
@@ -193,13 +198,13 @@ cudaError_t launch_t(const ProP &p, bool bwd, cudaStream_t s) {
   const long long warps = (p.rows + rows_per_warp - 1) / rows_per_warp;
   const long long want = (warps + kProThreads / 32 - 1) / (kProThreads / 32);
   int occ = 0;  // a few waves of resident CTAs, grid-stride beyond
-  e = bwd ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, prologue_kernel<InT, D, true>, kProThreads, 0)
+  e = bwd ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, prologue_kernel<InT, D, true, GT, OT>, kProThreads, 0)
           : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, prologue_kernel<InT, D, false>, kProThreads, 0);
   if (e != cudaSuccess) return e;
   const long long cap = ((long long)nsm * (occ > 0 ? occ : 1) * kWaves + nt - 1) / nt;
   const dim3 grid((unsigned)(want < cap ? want : cap), nt);
   if (bwd)
-    RDN_LAUNCH("qk_prologue_bwd", s, prologue_kernel<InT, D, true><<<grid, kProThreads, 0, s>>>(p));
+    RDN_LAUNCH("qk_prologue_bwd", s, prologue_kernel<InT, D, true, GT, OT><<<grid, kProThreads, 0, s>>>(p));
   else
     RDN_LAUNCH("qk_prologue", s, prologue_kernel<InT, D, false><<<grid, kProThreads, 0, s>>>(p));
   return cudaGetLastError();
@@ -219,6 +224,25 @@ cudaError_t launch_prologue(const rdn_prologue_args &a, bool bwd, cudaStream_t s
   if (a.dtype == RDN_BF16)
     return a.D == 128 ? launch_t<__nv_bfloat16, 128>(p, bwd, s) : launch_t<__nv_bfloat16, 64>(p, bwd, s);
   return a.D == 128 ? launch_t<float, 128>(p, bwd, s) : launch_t<float, 64>(p, bwd, s);
+}
+
+cudaError_t launch_prologue_bwd_f32dy(const rdn_prologue_args &a, bool f32dx, cudaStream_t s) {
+  ProP p;
+  p.rows = a.rows;
+  p.eps = a.eps;
+  for (int i = 0; i < 2; ++i) {
+    p.x[i] = a.x[i];
+    p.dy[i] = a.dy[i];
+    p.o[i] = a.dx[i];
+  }
+  if (a.dtype == RDN_BF16) {
+    if (f32dx)
+      return a.D == 128 ? launch_t<__nv_bfloat16, 128, float, float>(p, true, s)
+                        : launch_t<__nv_bfloat16, 64, float, float>(p, true, s);
+    return a.D == 128 ? launch_t<__nv_bfloat16, 128, float>(p, true, s)
+                      : launch_t<__nv_bfloat16, 64, float>(p, true, s);
+  }
+  return a.D == 128 ? launch_t<float, 128>(p, true, s) : launch_t<float, 64>(p, true, s);
 }
 
 }  // namespace rdn

@@ -64,7 +64,14 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(dtype=7)) == 2
     assert _status(fn, _fwd_args(clip=-1.0)) == 1
     assert _status(fn, _fwd_args(clip=float("nan"))) == 1
-    assert _status(fn, _fwd_args(flags=0x80)) == 2
+    assert _status(fn, _fwd_args(flags=0x100)) == 2
+    # q, k normalisation: needs a positive finite floor; then the NULL check
+    QKN = _abi.RDN_FLAG_QK_NORM
+    assert _status(fn, _fwd_args(flags=QKN)) == 1
+    assert "qk_eps" in lib.rdn_last_error().decode()
+    assert _status(fn, _fwd_args(flags=QKN, qk_eps=float("inf"))) == 1
+    assert _status(fn, _fwd_args(flags=QKN, qk_eps=1e-12)) == 1
+    assert "q is NULL" in lib.rdn_last_error().decode()
     # fp32 results: bf16 inputs need the tensor-core path (Dk = 128, no tanh /
     # stateless variant); fp32 inputs take the flag as a no-op (then the call
     # gets as far as the NULL pointer check)
@@ -236,7 +243,7 @@ def test_binding_rejects_cpu_tensors():
 
 _STRUCTS = {
     "rdn_fwd_args": ("FwdArgs", ["B", "q", "clip", "S0", "scale", "flags", "workspace",
-                                 "workspace_bytes", "cu_seqlens", "num_seqs"]),
+                                 "workspace_bytes", "cu_seqlens", "num_seqs", "qk_eps"]),
     "rdn_bwd_args": ("BwdArgs", ["fwd", "dO", "dq", "dS0", "dR0", "workspace",
                                  "workspace_bytes"]),
     "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o", "flags"]),
@@ -270,7 +277,7 @@ def test_binding_flag_values_match_the_header():
     """Every RDN_FLAG_* of include/rdn.h has the same value in the binding."""
     src = open(os.path.join(ROOT, "include", "rdn.h")).read()
     flags = dict(re.findall(r"#define\s+(RDN_FLAG_\w+)\s+(0x[0-9a-fA-F]+)u", src))
-    assert len(flags) == 7, flags
+    assert len(flags) == 8, flags
     for name, val in flags.items():
         assert getattr(_abi, name) == int(val, 16), name
     variants = ("RDN_FLAG_DECAYED_RESIDUAL", "RDN_FLAG_PLAIN_COMBINE", "RDN_FLAG_TANH_RESIDUAL",
@@ -322,8 +329,17 @@ int main(void) {
   if (strstr(rdn_last_error(), "q is NULL") == NULL) return 4;
   a.flags = RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_TIED_GAMMA;
   if (rdn_fwd_workspace_size(&a, &ws) != RDN_OK) return 5;
-  a.flags = 0x80u;
+  a.flags = 0x100u;
   if (rdn_fwd_workspace_size(&a, &ws) != RDN_ERR_UNSUPPORTED) return 6;
+  {
+    size_t ws2 = 0;  /* the normalised q, k copies: 2 B T H Dk bf16 more */
+    a.flags = RDN_FLAG_QK_NORM;
+    a.qk_eps = 1e-12f;
+    if (rdn_fwd_workspace_size(&a, &ws2) != RDN_OK) return 7;
+    a.flags = 0;
+    if (rdn_fwd_workspace_size(&a, &ws) != RDN_OK || ws2 != ws + 2u * 2 * 300 * 4 * 128 * 2)
+      return 8;
+  }
   printf("%s\n", rdn_version());
   return 0;
 }
