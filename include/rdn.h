@@ -118,19 +118,22 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  * and, as a no-op, for RDN_F32; otherwise RDN_ERR_UNSUPPORTED. */
 #define RDN_FLAG_F32_OUT 0x40u
 
-/* RDN_FLAG_QK_NORM (rla_fwd / rdn_fwd, and in the backward's fwd.flags): q
- * and k are the raw projections x, and the library applies the activation and
- * normalisation of rdn_qk_prologue to them itself, per row of Dk elements
+/* RDN_FLAG_QK_NORM (rla_fwd / rdn_fwd, rdn_decode_step, and in the
+ * backward's fwd.flags): q and k are the raw projections x, and the library
+ * applies the activation and normalisation of rdn_qk_prologue to them itself,
+ * per row of Dk elements
  *     y = SiLU(x) / max(||SiLU(x)||_2, qk_eps),
- * before the recurrence; the backward returns dq and dk with respect to x
- * (the map's transposed Jacobian applied to the gradients w.r.t. y).  On the
- * tensor-core path (RDN_BF16, Dk = Dv = 128) the forward's per-chunk pass
- * normalises the rows it loads and keeps y (bf16) in the workspace for the
- * scan and the backward, and the backward's final kernel applies the
- * Jacobian as it writes dq and dk; elsewhere the rdn_qk_prologue kernels run
- * as passes of their own.  Needs qk_eps > 0 and finite (else
- * RDN_ERR_INVALID_ARG); *_fwd_workspace_size and *_bwd_workspace_size grow
- * by the normalised copies (2 B T H Dk elements of dtype). */
+ * before the recurrence, holding y in `dtype` (as a caller's own prologue
+ * pass would); the backward returns dq and dk with respect to x (the map's
+ * transposed Jacobian applied to the gradients w.r.t. y).  On the tensor-core
+ * path (RDN_BF16, Dk = Dv = 128) the forward's per-chunk pass normalises the
+ * rows as it loads them and keeps y in the workspace for the scan and the
+ * backward; elsewhere the prologue kernel writes y first.  The backward keeps
+ * the gradients w.r.t. y in fp32 (for bf16 inputs) and applies the Jacobian
+ * in one streaming pass.  Needs qk_eps > 0 and finite (else
+ * RDN_ERR_INVALID_ARG); *_fwd_workspace_size and *_bwd_workspace_size grow by
+ * the normalised copies (2 B T H Dk elements of dtype) and the fp32 gradients
+ * (2 B T H Dk floats, bf16 inputs). */
 #define RDN_FLAG_QK_NORM 0x80u
 
 /* Arguments of rla_fwd / rdn_fwd.
@@ -239,8 +242,10 @@ typedef struct {
  *   other argument).
  *   variant           0 = RLA, 1 = RDN.
  *   flags             0, or RDN_FLAG_TIED_GAMMA (gamma ignored, beta serves
- *                     as both rates) and / or the variant flags: the same
- *                     token step as the forward with those flags.        */
+ *                     as both rates), the variant flags and / or
+ *                     RDN_FLAG_QK_NORM (q, k raw x, normalised in the step
+ *                     with qk_eps and held in dtype, as the forward does):
+ *                     the same token step as the forward with those flags. */
 typedef struct {
   int N, H, Dk, Dv;
   int dtype;
@@ -252,6 +257,7 @@ typedef struct {
   float *S, *R;
   void *o;
   unsigned flags;
+  float qk_eps; /* the norm floor of RDN_FLAG_QK_NORM; ignored without it */
 } rdn_decode_args;
 
 /* Arguments of rdn_qk_prologue / rdn_qk_prologue_bwd: the activation and

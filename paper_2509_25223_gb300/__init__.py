@@ -305,10 +305,10 @@ def qk_prologue_bwd(q, k, dyq, dyk=None, eps=1e-12, out=None):
 
 
 def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant="rdn", out=None,
-                    tied_gamma=False, variant_flags=0):
+                    tied_gamma=False, variant_flags=0, qk_norm=False, qk_eps=1e-12):
     """One recurrent step for N sequences; S, R [N,H,Dk,Dv] fp32 are updated
     in place.  q, k [N,H,Dk]; v [N,H,Dv]; gates [N,H].  Returns o [N,H,Dv].
-    tied_gamma / variant_flags: as for the forward."""
+    tied_gamma / variant_flags / qk_norm, qk_eps: as for the forward."""
     lib = _abi.load()
     _check_variant_flags(variant_flags)
     N, H, Dk = q.shape
@@ -322,7 +322,9 @@ def rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, scale=1.0, variant=
     a.g, a.beta, a.gamma = _ptr(g), _ptr(beta), _ptr(gamma)
     a.clip, a.scale = float(clip), float(scale)
     a.S, a.R, a.o = _ptr(S), _ptr(R), _ptr(o)
-    a.flags = (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags
+    a.flags = (_abi.RDN_FLAG_TIED_GAMMA if tied_gamma else 0) | variant_flags \
+        | (_abi.RDN_FLAG_QK_NORM if qk_norm else 0)
+    a.qk_eps = float(qk_eps)
     _check("rdn_decode_step", lib.rdn_decode_step(ctypes.byref(a), _stream(q)))
     return o
 

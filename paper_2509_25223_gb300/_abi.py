@@ -57,7 +57,8 @@ class DecodeArgs(ctypes.Structure):
                 ("Dv", ctypes.c_int), ("dtype", ctypes.c_int), ("variant", ctypes.c_int),
                 ("q", P), ("k", P), ("v", P), ("g", P), ("beta", P), ("gamma", P),
                 ("clip", ctypes.c_float), ("scale", ctypes.c_float),
-                ("S", P), ("R", P), ("o", P), ("flags", ctypes.c_uint)]
+                ("S", P), ("R", P), ("o", P), ("flags", ctypes.c_uint),
+                ("qk_eps", ctypes.c_float)]
 
 
 class PrologueArgs(ctypes.Structure):

@@ -545,8 +545,11 @@ rdn_status_t rdn_decode_step(const rdn_decode_args *a, rdn_stream_t stream) {
   rdn_status_t st = check_clip(fn, a->clip);
   if (st != RDN_OK) return st;
   if (isnan(a->scale) || isinf(a->scale)) return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
-  if (a->flags & ~(RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS))
+  if (a->flags & ~(RDN_FLAG_TIED_GAMMA | RDN_FLAG_VARIANTS | RDN_FLAG_QK_NORM))
     return fail(RDN_ERR_UNSUPPORTED, "%s: flags 0x%x unsupported", fn, a->flags);
+  if ((a->flags & RDN_FLAG_QK_NORM) && !(a->qk_eps > 0.f && !isinf(a->qk_eps)))
+    return fail(RDN_ERR_INVALID_ARG, "%s: RDN_FLAG_QK_NORM needs qk_eps > 0 and finite (got %g)",
+                fn, a->qk_eps);
   REQUIRE_PTR(a->q);
   REQUIRE_PTR(a->k);
   REQUIRE_PTR(a->v);

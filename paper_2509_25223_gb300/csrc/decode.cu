@@ -16,6 +16,9 @@
 //     o  = a sq + gam (q^T R') = a sq + gam (a rq + gam (k.q) e2)
 // which is the right (RDN) / left (RLA) formulation of Section 3.4 with the
 // delta-rule product expanded: a S (I - b k k^T) + b k v^T = a S + b k (v - a S^T k)^T.
+// With RDN_FLAG_QK_NORM the rows of q and k are the raw x, turned into
+// y = SiLU(x) / max(||SiLU(x)||, eps) here (held in the input dtype, as the
+// forward holds them) before the step.
 // The variant flags change the step as in the chunk kernels: r = resid(v - a p)
 // (decayed residual), c tanh(x / c) (tanh residual), R' = k r^T without
 // reading R (stateless correction, o's correction term gam (k.q) r), and
@@ -34,13 +37,14 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
               const InT *__restrict__ v, const float *__restrict__ g,
               const float *__restrict__ beta, const float *__restrict__ gam,
               float clip, float scale, float *__restrict__ S, float *__restrict__ R,
-              InT *__restrict__ o, unsigned mods) {
+              InT *__restrict__ o, unsigned mods, bool qkn, float qk_eps) {
   constexpr int RPT = D / 16;             // rows per thread (16 row groups)
   constexpr int NSLICE = D / kSliceCols;  // column slices per (n,h)
   __shared__ float q_s[D], k_s[D];
   __shared__ float red[8][4][kSliceCols];  // per-warp partial read-outs
   __shared__ float tot[4][kSliceCols];
   __shared__ float kq_s;
+  __shared__ float nrm_s[2];
 
   const int nh = blockIdx.x / NSLICE;
   const int slice = blockIdx.x % NSLICE;
@@ -62,9 +66,29 @@ decode_kernel(int H, const InT *__restrict__ q, const InT *__restrict__ k,
     r_reg[i] = stl ? make_float4(0.f, 0.f, 0.f, 0.f)  // (the stateless R is not read)
                    : __ldcs(reinterpret_cast<const float4 *>(R + off));
   }
-  for (int i = tid; i < D; i += kDecThreads) {
-    q_s[i] = scale * to_f32(q[(size_t)nh * D + i]);
-    k_s[i] = to_f32(k[(size_t)nh * D + i]);
+  if (!qkn) {
+    for (int i = tid; i < D; i += kDecThreads) {
+      q_s[i] = scale * to_f32(q[(size_t)nh * D + i]);
+      k_s[i] = to_f32(k[(size_t)nh * D + i]);
+    }
+  } else {  // warp 0: q's row, warp 1: k's row
+    if (warp < 2) {
+      const InT *x = (warp == 0 ? q : k) + (size_t)nh * D;
+      float u[D / 32], ss = 0.f;
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) {
+        const float xi = to_f32(x[(tid & 31) + 32 * i]);
+        u[i] = xi * __fdividef(1.f, 1.f + __expf(-xi));
+        ss = fmaf(u[i], u[i], ss);
+      }
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+      const float inv = 1.f / fmaxf(sqrtf(ss), qk_eps);
+      float *dst = warp == 0 ? q_s : k_s;
+      const float f = warp == 0 ? scale : 1.f;
+#pragma unroll
+      for (int i = 0; i < D / 32; ++i) dst[(tid & 31) + 32 * i] = f * to_f32(from_f32<InT>(u[i] * inv));
+    }
   }
   __syncthreads();
   if (warp == 0) {
@@ -161,12 +185,14 @@ cudaError_t launch_decode_t(const rdn_decode_args &a, cudaStream_t s) {
     RDN_LAUNCH("decode", s,
                decode_kernel<D, true, InT><<<grid, kDecThreads, 0, s>>>(
                    a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
-                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS));
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS,
+                   (a.flags & RDN_FLAG_QK_NORM) != 0, a.qk_eps));
   else
     RDN_LAUNCH("decode", s,
                decode_kernel<D, false, InT><<<grid, kDecThreads, 0, s>>>(
                    a.H, (const InT *)a.q, (const InT *)a.k, (const InT *)a.v, a.g, a.beta,
-                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS));
+                   a.gamma, a.clip, a.scale, a.S, a.R, (InT *)a.o, a.flags & RDN_FLAG_VARIANTS,
+                   (a.flags & RDN_FLAG_QK_NORM) != 0, a.qk_eps));
   return cudaGetLastError();
 }
 

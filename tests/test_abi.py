@@ -246,7 +246,8 @@ _STRUCTS = {
                                  "workspace_bytes", "cu_seqlens", "num_seqs", "qk_eps"]),
     "rdn_bwd_args": ("BwdArgs", ["fwd", "dO", "dq", "dS0", "dR0", "workspace",
                                  "workspace_bytes"]),
-    "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o", "flags"]),
+    "rdn_decode_args": ("DecodeArgs", ["N", "variant", "q", "clip", "scale", "S", "o", "flags",
+                                       "qk_eps"]),
     "rdn_prologue_args": ("PrologueArgs", ["rows", "D", "dtype", "eps", "x", "y", "dy", "dx"]),
 }
 

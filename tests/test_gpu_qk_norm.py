@@ -225,3 +225,51 @@ def test_qk_norm_f32_out():
     ref = _ref_bwd(x, clip, oracle.RDN, None, None)
     for name in ("dq", "dk", "dv"):
         assert_close(d[name], ref[name], "bf16", name)
+
+
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
+@pytest.mark.parametrize("dtype,D", [("bf16", 128), ("f32", 64)])
+def test_qk_norm_decode_step(variant, dtype, D):
+    """rdn_decode_step with the flag: one token, normalised in the step."""
+    N, H = 3, 2
+    gen = torch.Generator(device="cpu").manual_seed(21)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    q = torch.randn(N, H, D, generator=gen).to(td).cuda()
+    k = torch.randn(N, H, D, generator=gen).to(td).cuda()
+    v = torch.randn(N, H, D, generator=gen).to(td).cuda()
+    g = -torch.rand(N, H, generator=gen).cuda()
+    beta = torch.rand(N, H, generator=gen).cuda()
+    gamma = torch.rand(N, H, generator=gen).cuda()
+    S = (0.1 * torch.randn(N, H, D, D, generator=gen)).cuda()
+    R = (0.1 * torch.randn(N, H, D, D, generator=gen)).cuda()
+    S0, R0 = S.clone(), R.clone()
+    o = rdn.rdn_decode_step(q, k, v, g, beta, gamma, S, R, clip=1.0, variant=variant,
+                            qk_norm=True, qk_eps=EPS)
+    torch.cuda.synchronize()
+    yq, yk = _oracle_y({"q": q, "k": k})
+    ov = oracle.RDN if variant == "rdn" else oracle.RLA
+    ro, rS, rR = oracle.decode_step(ov, yq, yk, as64(v), as64(g), as64(beta), as64(gamma), 1.0,
+                                    as64(S0), as64(R0))
+    assert_close(o, ro, dtype, "o")
+    assert_close(S, rS, dtype, "S")
+    assert_close(R, rR, dtype, "R")
+
+
+def test_qk_norm_decode_chain_equals_forward():
+    """T decode steps with the flag give the forward's o and final states."""
+    B, T, H, D = 2, 70, 2, 128
+    x = _inputs(B, T, H, D, "bf16", seed=8)
+    _condition(x, 1.0, "bf16", oracle.RDN)
+    o, ST, RT = rdn.rdn_fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                            qk_norm=True, qk_eps=EPS)
+    S, R = x["S0"].clone(), x["R0"].clone()
+    od = torch.empty_like(o)
+    for t in range(T):
+        od[:, t] = rdn.rdn_decode_step(*(x[n][:, t].contiguous() for n in NAMES), S, R,
+                                       clip=1.0, qk_norm=True, qk_eps=EPS)
+    torch.cuda.synchronize()
+    ro, rST, rRT = _ref_fwd(x, 1.0, oracle.RDN)
+    assert_close(od, ro, "bf16", "o (decode)")
+    assert_close(o, ro, "bf16", "o (forward)")
+    assert_close(S, rST, "bf16", "S (decode)")
+    assert_close(R, rRT, "bf16", "R (decode)")
