@@ -681,10 +681,14 @@ def run_ours(args):
     var = None
     if not args.no_variants:
         var = {"workload": w.name, "steps": 1, "flags": {},
-               "path": "tensor-core kernels for the decayed residual and the plain combine, "
-                       "fp32 chunk kernels for the tanh residual and the stateless correction"}
+               "path": "tensor-core kernels for the decayed residual, the plain combine and "
+                       "the tanh residual, fp32 chunk kernels for the stateless correction"}
         wsbv_ = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D,
-                                                variant_flags=rdn.DECAYED_RESIDUAL),
+                                                variant_flags=rdn.TANH_RESIDUAL),
+                            dtype=torch.uint8, device=dev)
+        # (the tanh residual saves a 16-bit derivative per element, not a mask bit)
+        wsfv_ = torch.empty(rdn.workspace_bytes("rdn_fwd", B, T, H, D, save_for_bwd=True,
+                                                variant_flags=rdn.TANH_RESIDUAL),
                             dtype=torch.uint8, device=dev)
         for fname, fl in (("decayed_residual", rdn.DECAYED_RESIDUAL),
                           ("plain_combine", rdn.PLAIN_COMBINE),
@@ -692,10 +696,10 @@ def run_ours(args):
                           ("stateless_aux", rdn.STATELESS_AUX)):
             def fstep(inp):  # (the RDN step's options: chunk states, saved intermediates)
                 _, _, _, Sc_, Rc_ = rdn.rdn_fwd(*(inp[n] for n in names), clip=w.clip,
-                                                return_chunk_states=True, out=o, workspace=wsf,
+                                                return_chunk_states=True, out=o, workspace=wsfv_,
                                                 save_for_bwd=True, variant_flags=fl)
                 rdn.rdn_bwd(*(inp[n] for n in names), inp["dO"], clip=w.clip, S_chunks=Sc_,
-                            R_chunks=Rc_, workspace=wsbv_, out=grads, fwd_workspace=wsf,
+                            R_chunks=Rc_, workspace=wsbv_, out=grads, fwd_workspace=wsfv_,
                             fwd_saved=True, variant_flags=fl)
             fstep(x)
             torch.cuda.synchronize()
@@ -707,7 +711,7 @@ def run_ours(args):
             barrier(dist)
             tf, fval = aggregate(dist, e0.elapsed_time(e1), tokens_per_step)
             var["flags"][fname] = {"value": fval, "unit": "tokens/s", "ms_per_step": tf}
-        del wsbv_
+        del wsbv_, wsfv_
 
     # ---- packed variable-length sequences: the same B*T tokens per head as
     # one packed row of seeded log-uniform lengths in [64, 8192] (the last one

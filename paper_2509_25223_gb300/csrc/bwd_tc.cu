@@ -377,6 +377,9 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     });
   }
   if (ok) {
+    // the clip mask, or with the tanh residual its derivative ([j][t], grad_q16)
+    const bool tnh = p.mods & RDN_FLAG_TANH_RESIDUAL;
+    uint16_t *drow = reinterpret_cast<uint16_t *>(P.mask) + (chunk * D + j) * 64;
     unsigned long long m = 0ull;
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
@@ -389,12 +392,13 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
         const int t = c0 + i;
         const float x = vval(t) - pp[i];
         if (fabsf(x) <= clip) m |= 1ull << t;
-        r[t] = clampf(x, clip);
+        r[t] = resid_map(x, clip, tnh);
+        if (tnh) drow[t] = (uint16_t)grad_q16(resid_grad(x, clip, true));
         x2[i] = r[t] - (P.rla ? 0.f : Gam[t] * kr[i]);
       }
       put16s(sm + XE, sm + XE_LO, j, c0, x2);
     }
-    P.mask[chunk * D + j] = m;
+    if (!tnh) P.mask[chunk * D + j] = m;
     ok = phase_run(K, tid, [&] {  // E2 = T_gamma X2
       if (!slot_wait(K.barA, K.phA)) return false;
       mma_s3_kk(tm + T_X, sb + XE, sb + XE_LO, sb + SLOTA, sb + SLOTA + 8192, idesc_bf16(128, 64),
@@ -570,7 +574,9 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
   struct Pre {
     float gam_, gprev, ws_, wr_, g_, gamc;
     unsigned m;
+    uint4 d0, d1;  // the tanh residual's derivative at this thread's 16 tokens (grad_q16)
   };
+  const bool tnh = kGeneric && (mods & RDN_FLAG_TANH_RESIDUAL);
   auto fetch_pre = [&](int c) {
     const size_t ck = (size_t)(sp.rbase + c);
     const int t0 = c * 64, n = min(64, T - t0);
@@ -587,7 +593,14 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     }
     x.gamc = rf[OFF_VEC + V_GAMC];
     // bits [g16, g16 + 16) of the column's 64-bit word (little-endian)
-    x.m = reinterpret_cast<const uint16_t *>(P.mask + ck * D + j)[g16 >> 4];
+    if (!tnh) {
+      x.m = reinterpret_cast<const uint16_t *>(P.mask + ck * D + j)[g16 >> 4];
+    } else {
+      const uint4 *dp_ = reinterpret_cast<const uint4 *>(
+          reinterpret_cast<const uint16_t *>(P.mask) + (ck * D + j) * 64 + g16);
+      x.d0 = dp_[0];
+      x.d1 = dp_[1];
+    }
     return x;
   };
   Pre pre{};
@@ -637,6 +650,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     }
     const float GamC = pre.gamc;
     const unsigned m = pre.m;  // bit i: clip inactive at t = g16 + i
+    const uint4 dd0 = pre.d0, dd1 = pre.d1;  // (tanh residual)
     cp_async_wait_all();  // this chunk's tiles (fetched during the previous one)
     if (tma && c < NC - 1) {  // (by tiled bulk copies)
       if (mbar_wait(K.barC, tma_ph & 1u))
@@ -727,7 +741,13 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
         for (int i = 0; i < 16; ++i) {
           const int t = c0 + i;
           stg[t * D + j] = x[i];
-          dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
+          if (tnh) {  // the derivative of c tanh(x / c) instead of the mask
+            const uint32_t w = (i < 8 ? reinterpret_cast<const uint32_t *>(&dd0)
+                                      : reinterpret_cast<const uint32_t *>(&dd1))[(i & 7) >> 1];
+            dp[i] = -grad_uq16((i & 1) ? w >> 16 : w & 0xffffu) * x[i];
+          } else {
+            dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
+          }
           dP[i] = dp[i];
           dkr[i] = rla ? 0.f : -dkr[i] * x[i];
         }
@@ -963,6 +983,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // residual against a_t S_{t-1} k_t; o = S_{t-1} q_t + R_t q_t
   const bool dec_res = kGeneric && (p.mods & RDN_FLAG_DECAYED_RESIDUAL);
   const bool plain = kGeneric && (p.mods & RDN_FLAG_PLAIN_COMBINE);
+  // the tanh residual: dP = -(1 - (r/c)^2) dX2 from the stored derivative
+  const bool tnh = kGeneric && (p.mods & RDN_FLAG_TANH_RESIDUAL);
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   Ctl K;
@@ -1081,7 +1103,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     return true;
   });
   // while P1 runs: this thread's dO, the gate vectors, dX2 and dX from their staging
-  const unsigned long long m = P.mask[chunk * D + j] >> tb;
+  const unsigned long long m = tnh ? 0ull : P.mask[chunk * D + j] >> tb;
+  const uint16_t *drow = reinterpret_cast<const uint16_t *>(P.mask) + (chunk * D + j) * 64 + tb;
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const int t = tb + i;
@@ -1105,7 +1128,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
   }
   ok = phase_wait(K);  // (its barrier also publishes the gate vectors)
-  auto dp_of = [&](int i) { return ((m >> i) & 1ull) ? -x2v[i] : 0.f; };
+  auto dp_of = [&](int i) {
+    if (tnh) return -grad_uq16(drow[i]) * x2v[i];
+    return ((m >> i) & 1ull) ? -x2v[i] : 0.f;
+  };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
     float rv[16];
     {
@@ -1538,7 +1564,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         const int t = tid >> 1;
         if (t < n_) prefetch_l1_line(dOp + ((size_t)(tok0_ + t0_ + t) * H + h_) * D + (tid & 1) * 64);
       } else if (tid < 136) {  // 128 mask words
-        prefetch_l1_line(P.mask + next * D + (tid - 128) * 16);
+        if (!tnh) prefetch_l1_line(P.mask + next * D + (tid - 128) * 16);
       } else if (tid < 148) {  // the record's 6 x 64 gate floats
         prefetch_l1_line(p.ws + next * kRecFloats + OFF_VEC + (tid - 136) * 32);
       } else if (tid < 180) {  // gamma, one line per two tokens
@@ -1589,10 +1615,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 
 size_t bwd_tc_acc_bytes(long long nrec) { return sizeof(float) * (size_t)nrec * A8::FLOATS; }
 
-size_t bwd_tc_extra_bytes(long long nrec) {
+size_t bwd_tc_extra_bytes(long long nrec, bool deriv) {
   const size_t nct = (size_t)nrec;
   return nct * (4 * 64 * D * sizeof(float) + 2 * (size_t)D * D * sizeof(float) +
-                D * sizeof(unsigned long long));
+                mask_bytes_per_chunk(D, deriv));
 }
 
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,

@@ -790,7 +790,7 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   l.states = need_states ? align256(sizeof(float) * nrec * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
   l.o = need_states ? align256(esz * (size_t)f.B * f.T * f.H * f.Dv) : 0;
-  l.tc = tc ? align256(bwd_tc_extra_bytes(nrec)) : 0;
+  l.tc = tc ? align256(bwd_tc_extra_bytes(nrec, f.flags & RDN_FLAG_TANH_RESIDUAL)) : 0;
   // normalised q, k (RDN_FLAG_QK_NORM), unless the forward's workspace has them
   l.qk = reuse_fwd_records(f, variant) ? 0 : align256(qk_norm_bytes(f));
   // and, with bf16 inputs, dq, dk (w.r.t. the normalised q, k) in fp32 for
@@ -874,7 +874,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
     set_qk_norm_copies(p.f, f, reuse ? (char *)f.workspace + qk_norm_offset(f)
                                      : ws + l.prep + l.acc + 2 * l.states + l.o + l.tc);
   if (reuse && (f.flags & RDN_FLAG_SAVE_FOR_BWD)) {  // E, E2 and the mask kept by the forward
-    const SavedLayout sl = saved_layout((size_t)p.f.nrec, f.Dv);
+    const SavedLayout sl = saved_layout((size_t)p.f.nrec, f.Dv, f.flags & RDN_FLAG_TANH_RESIDUAL);
     p.f.sv_E = (uint8_t *)f.workspace + sl.e;
     p.f.sv_E2 = (uint8_t *)f.workspace + sl.e2;
     p.f.sv_mask = (unsigned long long *)((char *)f.workspace + sl.mask);

@@ -185,15 +185,20 @@ __device__ __forceinline__ void rec_decode(const FwdParams &p, long long r, int 
 }
 
 // Where the forward keeps those intermediates: after the nrec record slots.
+// With the tanh residual (deriv) the clip mask's place holds the residual
+// map's derivative instead, [chunk][j][t] as 16-bit fixed point (grad_q16).
 struct SavedLayout {
   size_t e, e2, mask, bytes;  // byte offsets from the workspace base; region size
 };
-inline SavedLayout saved_layout(size_t nct, int Dv) {
+inline size_t mask_bytes_per_chunk(int Dv, bool deriv) {
+  return deriv ? (size_t)Dv * C * 2 : (size_t)Dv * sizeof(unsigned long long);
+}
+inline SavedLayout saved_layout(size_t nct, int Dv, bool deriv) {
   SavedLayout l;
   l.e = nct * sizeof(float) * (size_t)kRecFloats;
   l.e2 = l.e + nct * sizeof(float) * C * Dv;
   l.mask = l.e2 + nct * sizeof(float) * C * Dv;
-  l.bytes = l.mask + nct * sizeof(unsigned long long) * Dv - l.e;
+  l.bytes = l.mask + nct * mask_bytes_per_chunk(Dv, deriv) - l.e;
   return l;
 }
 
@@ -236,7 +241,8 @@ inline size_t qk_norm_bytes(const rdn_fwd_args &a) {
 inline size_t qk_norm_offset(const rdn_fwd_args &a) {
   const size_t nrec = (size_t)call_records(a);
   size_t off = sizeof(float) * (size_t)kRecFloats * nrec;
-  if (a.flags & RDN_FLAG_SAVE_FOR_BWD) off += saved_layout(nrec, a.Dv).bytes;
+  if (a.flags & RDN_FLAG_SAVE_FOR_BWD)
+    off += saved_layout(nrec, a.Dv, a.flags & RDN_FLAG_TANH_RESIDUAL).bytes;
   return off;
 }
 // Points p.q, p.k at the normalised copies starting at `base`.
@@ -247,8 +253,10 @@ inline void set_qk_norm_copies(FwdParams &p, const rdn_fwd_args &a, char *base) 
 }
 
 // The variant flags the tensor-core kernels implement (the others run on the
-// fp32 chunk kernels): the decayed residual and the plain combine.
-constexpr unsigned kTcVariants = RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE;
+// fp32 chunk kernels): the decayed residual, the plain combine and the tanh
+// residual.
+constexpr unsigned kTcVariants =
+    RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE | RDN_FLAG_TANH_RESIDUAL;
 // Whether the forward runs the tensor-core scan (and its records are
 // shared-memory images): bf16 inputs, d = 128, no variant flag outside
 // kTcVariants, for RDN and RLA alike.
@@ -265,7 +273,7 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
 
 // Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
 cudaError_t launch_prep_tc(const FwdParams &p, bool rla, cudaStream_t s);
-size_t bwd_tc_extra_bytes(long long nrec);  // per record slot
+size_t bwd_tc_extra_bytes(long long nrec, bool deriv);  // (deriv: the tanh residual's)
 size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,

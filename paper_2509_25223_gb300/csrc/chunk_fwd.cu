@@ -576,7 +576,8 @@ FwdPlan plan_fwd(const rdn_fwd_args &a, int variant) {
   // per-chunk records, the saved intermediates if asked for, the normalised
   // q, k (RDN_FLAG_QK_NORM), the packed-sequence table, then a 256-byte tail
   pl.total_bytes = pl.prep_bytes * nrec + seq_table_bytes(a) + 256;
-  if (a.flags & RDN_FLAG_SAVE_FOR_BWD) pl.total_bytes += saved_layout(nrec, a.Dv).bytes;
+  if (a.flags & RDN_FLAG_SAVE_FOR_BWD)
+    pl.total_bytes += saved_layout(nrec, a.Dv, a.flags & RDN_FLAG_TANH_RESIDUAL).bytes;
   pl.total_bytes += qk_norm_bytes(a);  // (after those: qk_norm_offset)
   return pl;
 }
@@ -604,7 +605,7 @@ cudaError_t launch_fwd(const rdn_fwd_args &a, int variant, cudaStream_t s) {
     p.seq = seq;
   }
   if (a.flags & RDN_FLAG_SAVE_FOR_BWD) {
-    const SavedLayout l = saved_layout((size_t)p.nrec, a.Dv);
+    const SavedLayout l = saved_layout((size_t)p.nrec, a.Dv, a.flags & RDN_FLAG_TANH_RESIDUAL);
     p.sv_E = (uint8_t *)a.workspace + l.e;
     p.sv_E2 = (uint8_t *)a.workspace + l.e2;
     p.sv_mask = (unsigned long long *)((char *)a.workspace + l.mask);

@@ -38,6 +38,12 @@ __device__ __forceinline__ float resid_map(float x, float c, bool tnh) {
   if (c == 0.f) return 0.f;
   return c * tanhf(x / c);
 }
+// The residual map's derivative (in [0, 1]) as 16-bit fixed point, d * 65535
+// rounded: an absolute error of at most 7.7e-6 over the whole range, where a
+// bf16 copy would be off by up to 2^-9 of d (the product d dX2 of the backward
+// can be large against the gradients it lands in).
+__device__ __forceinline__ uint32_t grad_q16(float d) { return __float2uint_rn(d * 65535.f); }
+__device__ __forceinline__ float grad_uq16(uint32_t q) { return (float)q * (1.f / 65535.f); }
 __device__ __forceinline__ float resid_grad(float x, float c, bool tnh) {
   if (!tnh) return fabsf(x) <= c ? 1.f : 0.f;
   if (isinf(c)) return 1.f;

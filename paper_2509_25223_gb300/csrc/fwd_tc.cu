@@ -162,6 +162,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   const float clip = p.clip;
   const bool dec_res = kGeneric && (p.mods & RDN_FLAG_DECAYED_RESIDUAL);
   const bool plain = kGeneric && (p.mods & RDN_FLAG_PLAIN_COMBINE);  // o = S_{t-1} q + R_t q
+  // the log-cosh residual r = c tanh(x / c); the backward then reads the
+  // derivative 1 - (r / c)^2 of each element (16-bit fixed point) where the
+  // clip mask goes
+  const bool tnh = kGeneric && (p.mods & RDN_FLAG_TANH_RESIDUAL);
   const size_t st_base = (size_t)bh * D * D;
 
   if (tid == 0) {
@@ -477,14 +481,32 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       unsigned msk = 0u;  // bit i: |x| <= c at t = c0 + i (the clip passes the gradient)
       float pp[16];
       tmem_ld16(tm + lane + T_D1 + c0, pp);
+      if (!tnh) {
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float x = vv[i] - pp[i];
-        if (fabsf(x) <= clip) msk |= 1u << i;
-        rres[i] = clampf(x, clip);
+        for (int i = 0; i < 16; ++i) {
+          const float x = vv[i] - pp[i];
+          if (fabsf(x) <= clip) msk |= 1u << i;
+          rres[i] = clampf(x, clip);
+        }
+        // bits [c0, c0 + 16) of the column's 64-bit mask word (little-endian)
+        if (p.sv_mask) reinterpret_cast<uint16_t *>(p.sv_mask + ci * D + j)[c0 >> 4] = (uint16_t)msk;
+      } else {
+        uint32_t dg[8];  // the derivative at t = c0 .. c0 + 15, pairs of 16-bit words
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          const float x0 = vv[i] - pp[i], x1 = vv[i + 1] - pp[i + 1];
+          rres[i] = resid_map(x0, clip, true);
+          rres[i + 1] = resid_map(x1, clip, true);
+          dg[i / 2] = grad_q16(resid_grad(x0, clip, true)) |
+                      (grad_q16(resid_grad(x1, clip, true)) << 16);
+        }
+        if (p.sv_mask) {
+          uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<uint16_t *>(p.sv_mask) +
+                                                 (ci * D + j) * 64 + c0);
+          dst[0] = make_uint4(dg[0], dg[1], dg[2], dg[3]);
+          dst[1] = make_uint4(dg[4], dg[5], dg[6], dg[7]);
+        }
       }
-      // bits [c0, c0 + 16) of the column's 64-bit mask word (little-endian)
-      if (p.sv_mask) reinterpret_cast<uint16_t *>(p.sv_mask + ci * D + j)[c0 >> 4] = (uint16_t)msk;
     }
     {
       float s0[16], s1[16];

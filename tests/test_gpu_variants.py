@@ -66,21 +66,24 @@ def test_variant_fwd(variant, dtype, D, flags):
 @pytest.mark.parametrize("variant", ["rdn", "rla"])
 @pytest.mark.parametrize("dtype,D", [("f32", 64), ("bf16", 128)])
 @pytest.mark.parametrize("flags", FLAGS)
-@pytest.mark.parametrize("reuse", [False, True])
+@pytest.mark.parametrize("reuse", [False, True, "saved"])
 def test_variant_bwd(variant, dtype, D, flags, reuse):
     ov = oracle.RDN if variant == "rdn" else oracle.RLA
     x = _inputs(dtype, D, seed=3)
     clip = 0.8
     _condition(x, clip, dtype, ov, _mods(flags))
     kw = {}
-    if reuse:  # the forward's chunk states and records
+    if reuse:  # the forward's chunk states and records (and its saved intermediates)
+        saved = reuse == "saved"
         nbytes = rdn.workspace_bytes(f"{variant}_fwd", *x["q"].shape[:3], D,
-                                     torch.bfloat16 if dtype == "bf16" else torch.float32)
+                                     torch.bfloat16 if dtype == "bf16" else torch.float32,
+                                     save_for_bwd=saved, variant_flags=flags)
         ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
         fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
         _, _, _, Sc, Rc = fwd(*(x[n] for n in NAMES), clip=clip, S0=x["S0"], R0=x["R0"],
-                              return_chunk_states=True, workspace=ws, variant_flags=flags)
-        kw = dict(S_chunks=Sc, R_chunks=Rc, fwd_workspace=ws)
+                              return_chunk_states=True, workspace=ws, variant_flags=flags,
+                              save_for_bwd=saved)
+        kw = dict(S_chunks=Sc, R_chunks=Rc, fwd_workspace=ws, fwd_saved=saved)
     fn = rdn.rdn_bwd if variant == "rdn" else rdn.rla_bwd
     d = fn(*(x[n] for n in NAMES), x["dO"], clip=clip, S0=x["S0"], R0=x["R0"], dST=x["dST"],
            dRT=x["dRT"], variant_flags=flags, **kw)
