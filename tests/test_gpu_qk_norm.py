@@ -76,8 +76,8 @@ def _fns(variant):
 
 
 # bf16 with D = 128 runs the tensor-core kernels (normalisation fused into the
-# per-chunk pass, the Jacobian into the last backward kernel); the others the
-# prologue kernels around the fp32 chunk kernels
+# per-chunk pass; the backward's gradients w.r.t. y kept in fp32 for one
+# Jacobian pass); the others the prologue kernels around the fp32 chunk kernels
 CASES = [("bf16", 128), ("bf16", 64), ("f32", 128), ("f32", 64)]
 
 
