@@ -681,8 +681,8 @@ def run_ours(args):
     var = None
     if not args.no_variants:
         var = {"workload": w.name, "steps": 1, "flags": {},
-               "path": "tensor-core kernels for the decayed residual, the plain combine and "
-                       "the tanh residual, fp32 chunk kernels for the stateless correction"}
+               "path": "tensor-core kernels for every flag (runtime modes of the generic "
+                       "kernel instances)"}
         wsbv_ = torch.empty(rdn.workspace_bytes("rdn_bwd", B, T, H, D,
                                                 variant_flags=rdn.TANH_RESIDUAL),
                             dtype=torch.uint8, device=dev)

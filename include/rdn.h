@@ -99,11 +99,10 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  *       fitting ablation (Section 4.3): R_t = r_t k_t^T replaces the
  *       recurrence for R, so R0 is ignored (dR0 = 0 unless T = 0) and RT =
  *       r_T k_T^T.
- * The decayed residual, the plain combine and the tanh residual also run on
- * the tensor-core kernels (bf16, Dk = 128; the tanh residual's backward reads
- * the map's derivative per element, bf16, where the clip mask goes); the
- * stateless correction runs on the fp32 chunk kernels, for every dtype and
- * head dimension. */
+ * Every variant runs on the tensor-core kernels for bf16 inputs with Dk = 128
+ * (the tanh residual's backward reads the map's derivative per element, 16-bit
+ * fixed point, where the clip mask goes) and on the fp32 chunk kernels for
+ * every other dtype and head dimension. */
 #define RDN_FLAG_DECAYED_RESIDUAL 0x4u
 #define RDN_FLAG_PLAIN_COMBINE 0x8u
 #define RDN_FLAG_TANH_RESIDUAL 0x10u
@@ -115,8 +114,7 @@ typedef enum { RDN_F32 = 0, RDN_BF16 = 1 } rdn_dtype_t;
  * either case; the flag only skips the final rounding to bf16, so a caller
  * can compare the computation itself against a reference without the bf16
  * storage rounding of the results (half a bf16 ulp, 2^-9 relative).
- * Supported where the tensor-core kernels run (RDN_BF16, Dk = Dv = 128, no
- * RDN_FLAG_STATELESS_AUX)
+ * Supported where the tensor-core kernels run (RDN_BF16, Dk = Dv = 128)
  * and, as a no-op, for RDN_F32; otherwise RDN_ERR_UNSUPPORTED. */
 #define RDN_FLAG_F32_OUT 0x40u
 

@@ -116,11 +116,9 @@ rdn_status_t check_fwd_shapes(const char *fn, const rdn_fwd_args *a) {
   if ((a->flags & RDN_FLAG_QK_NORM) && !(a->qk_eps > 0.f && !isinf(a->qk_eps)))
     return fail(RDN_ERR_INVALID_ARG, "%s: RDN_FLAG_QK_NORM needs qk_eps > 0 and finite (got %g)",
                 fn, a->qk_eps);
-  if ((a->flags & RDN_FLAG_F32_OUT) && a->dtype == RDN_BF16 &&
-      !(a->Dk == 128 && !(a->flags & RDN_FLAG_STATELESS_AUX)))
+  if ((a->flags & RDN_FLAG_F32_OUT) && a->dtype == RDN_BF16 && a->Dk != 128)
     return fail(RDN_ERR_UNSUPPORTED,
-                "%s: RDN_FLAG_F32_OUT with bf16 inputs needs Dk = 128 and the tensor-core "
-                "variants only", fn);
+                "%s: RDN_FLAG_F32_OUT with bf16 inputs needs Dk = 128 (the tensor-core path)", fn);
   if (isnan(a->scale) || isinf(a->scale))
     return fail(RDN_ERR_INVALID_ARG, "%s: scale must be finite", fn);
   return check_clip(fn, a->clip);

@@ -394,7 +394,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
         if (fabsf(x) <= clip) m |= 1ull << t;
         r[t] = resid_map(x, clip, tnh);
         if (tnh) drow[t] = (uint16_t)grad_q16(resid_grad(x, clip, true));
-        x2[i] = r[t] - (P.rla ? 0.f : Gam[t] * kr[i]);
+        x2[i] = r[t] - ((P.rla || (p.mods & RDN_FLAG_STATELESS_AUX)) ? 0.f : Gam[t] * kr[i]);
       }
       put16s(sm + XE, sm + XE_LO, j, c0, x2);
     }
@@ -577,6 +577,10 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     uint4 d0, d1;  // the tanh residual's derivative at this thread's 16 tokens (grad_q16)
   };
   const bool tnh = kGeneric && (mods & RDN_FLAG_TANH_RESIDUAL);
+  // the stateless correction: the chunk-end R is not carried into the next
+  // chunk nor read out there, so the gradient carried back to it is zero
+  // (dR_prev = 0; a chunk's own dR is the upstream dRT for the last chunk)
+  const bool stl = kGeneric && (mods & RDN_FLAG_STATELESS_AUX);
   auto fetch_pre = [&](int c) {
     const size_t ck = (size_t)(sp.rbase + c);
     const int t0 = c * 64, n = min(64, T - t0);
@@ -687,7 +691,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       bulk_wait_read();  // the tiles become scratch after this phase
       return true;
     }, [&] {
-      scale_grad(T_DR, GamC);
+      scale_grad(T_DR, stl ? 0.f : GamC);
       scale_grad(T_DS, GamC);
     });
     if (!ok) break;
@@ -713,7 +717,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       lds16(gamv + c0, w);
       const bool plain = mods & RDN_FLAG_PLAIN_COMBINE;  // (no gamma_t in the output)
 #pragma unroll
-      for (int i = 0; i < 16; ++i) x[i] = p.scale * x[i] * (plain ? 1.f : w[i]) * dO(c0 + i);  // dQR (Q unscaled)
+      for (int i = 0; i < 16; ++i)  // dQR (Q unscaled)
+        x[i] = stl ? 0.f : p.scale * x[i] * (plain ? 1.f : w[i]) * dO(c0 + i);
       put16s(sm + S1H, sm + S1L, j, c0, x);
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
@@ -749,7 +754,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
             dp[i] = ((m >> i) & 1u) ? -x[i] : 0.f;
           }
           dP[i] = dp[i];
-          dkr[i] = rla ? 0.f : -dkr[i] * x[i];
+          dkr[i] = (rla || stl) ? 0.f : -dkr[i] * x[i];
         }
         put16s(sm + S2H, sm + S2L, j, c0, dkr);
         put16s(sm + S3H, sm + S3L, j, c0, dp);
@@ -985,6 +990,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const bool plain = kGeneric && (p.mods & RDN_FLAG_PLAIN_COMBINE);
   // the tanh residual: dP = -(1 - (r/c)^2) dX2 from the stored derivative
   const bool tnh = kGeneric && (p.mods & RDN_FLAG_TANH_RESIDUAL);
+  // the stateless correction: R0 enters nothing (its read-outs, its P2 and
+  // <dR, R0> terms are zero), wR is a constant one-hot (no gate gradient
+  // through it) and M2 is diag(q_t . k_t) (no decay, no rate)
+  const bool stl = kGeneric && (p.mods & RDN_FLAG_STATELESS_AUX);
   const __nv_bfloat16 *q = (const __nv_bfloat16 *)p.q, *k = (const __nv_bfloat16 *)p.k,
                       *dOp = (const __nv_bfloat16 *)P.dO;
   Ctl K;
@@ -1137,6 +1146,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {
       float qs[16], qr[16];
       tmem_ld16x2(tm + tm_lane + T_KS + 64 + tb, qs, tm + tm_lane + T_KR + 64 + tb, qr);
+      if (stl) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) qr[i] = 0.f;
+      }
       // d gamma_t from the read-out: dO_t . (Gam_t Q R0)_t (the rest of Oa_t in P6)
       lds16(Gam + tb, rv);
 #pragma unroll
@@ -1153,6 +1166,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     {
       float ks[16], kr[16];
       tmem_ld16x2(tm + tm_lane + T_KS + tb, ks, tm + tm_lane + T_KR + tb, kr);
+      if (stl) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) kr[i] = 0.f;
+      }
       if (!rla) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) rv[i] -= x2v[i] * kr[i] + xv[i] * ks[i];
@@ -1179,8 +1196,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     lds16(gamv + tb, y);
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      y[i] = (plain ? 1.f : y[i]) * x[i] * dov[i];
-      x[i] = rla ? 0.f : -x[i] * x2v[i];
+      y[i] = stl ? 0.f : (plain ? 1.f : y[i]) * x[i] * dov[i];
+      x[i] = (rla || stl) ? 0.f : -x[i] * x2v[i];
     }
     put_tok(x, XH, XL);
     put_tok(y, YH, YL);
@@ -1227,7 +1244,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       return true;
     }, [&] {
       if (!mbar_wait(K.barB, it & 1u)) *K.flag = 1;  // dR's image
-      gdot = dot_state(R0, SB);
+      gdot = stl ? 0.f : dot_state(R0, SB);
     });
   }
   if (ok && tid == 0) {  // and dS's image into S0's; the E2^T, E^T images into the pair's
@@ -1301,7 +1318,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       image_row(w == 0 ? XH : YH, ev);
       tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb, rv);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) rv[i] *= ev[i];
+      for (int i = 0; i < 16; ++i) rv[i] = (w == 0 && stl) ? 0.f : rv[i] * ev[i];
       // parked in the record's slots (shared memory is full); read in the gate pass
       cta_row_sum512(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
     }
@@ -1362,7 +1379,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
             F[F_DAB + e] = rla ? 0.f : -g3[i];
             F[F_KK + e] = gr[i];
           } else {
-            F[F_DAG + e] = rla ? 0.f : -g1[i];
+            F[F_DAG + e] = (rla || stl) ? 0.f : -g1[i];  // (no T_gamma to differentiate)
             F[F_DAP + e] = g2[i];
             F[F_QK + e] = scale * gr[i];
           }
@@ -1412,7 +1429,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         if (i <= t) {
           const float dec = __expf(ct - cum[i]);
           const float kk = F[F_KK + e], qk = F[F_QK + e], bi = bet[i], gi = gam[i];
-          {  // M2: inclusive, gamma, Q K^T; G1 holds dO E2^T, dM2 = gamma_t dO E2^T
+          if (stl) {  // M2 = diag(Q K^T): the diagonal only, no decay, no rate
+            if (i == t) {
+              const float g1 = F[F_DM2 + e];
+              if (!plain) dgo += qk * g1;
+              dqk += plain ? g1 : gt * g1;
+            }
+          } else {  // M2: inclusive, gamma, Q K^T; G1 holds dO E2^T, dM2 = gamma_t dO E2^T
             const float g1 = F[F_DM2 + e];
             if (!plain) dgo += dec * gi * qk * g1;  // d gamma_t += (M2 E2)_t . dO_t
             const float dm = plain ? g1 : gt * g1;

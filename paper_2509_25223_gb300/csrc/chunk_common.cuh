@@ -252,11 +252,10 @@ inline void set_qk_norm_copies(FwdParams &p, const rdn_fwd_args &a, char *base) 
   p.k = base + half;
 }
 
-// The variant flags the tensor-core kernels implement (the others run on the
-// fp32 chunk kernels): the decayed residual, the plain combine and the tanh
-// residual.
-constexpr unsigned kTcVariants =
-    RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE | RDN_FLAG_TANH_RESIDUAL;
+// The variant flags the tensor-core kernels implement: all four (the decayed
+// residual, the plain combine, the tanh residual, the stateless correction).
+constexpr unsigned kTcVariants = RDN_FLAG_DECAYED_RESIDUAL | RDN_FLAG_PLAIN_COMBINE |
+                                 RDN_FLAG_TANH_RESIDUAL | RDN_FLAG_STATELESS_AUX;
 // Whether the forward runs the tensor-core scan (and its records are
 // shared-memory images): bf16 inputs, d = 128, no variant flag outside
 // kTcVariants, for RDN and RLA alike.

@@ -166,6 +166,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   // derivative 1 - (r / c)^2 of each element (16-bit fixed point) where the
   // clip mask goes
   const bool tnh = kGeneric && (p.mods & RDN_FLAG_TANH_RESIDUAL);
+  // the stateless correction R_t = r_t k_t^T: no read-out of the carried R
+  // (X2 = r, no gamma Gam Q R term in o), R not carried over a chunk (scaled
+  // by 0); the records hold the identity T_gamma, diag(gamma qk) and the
+  // one-hot wR that make the rest of the pass compute it
+  const bool stl = kGeneric && (p.mods & RDN_FLAG_STATELESS_AUX);
   const size_t st_base = (size_t)bh * D * D;
 
   if (tid == 0) {
@@ -390,7 +395,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       return true;
     }, [&] {
       scale_state(T_S, GamC);
-      scale_state(T_R, GamC);
+      scale_state(T_R, stl ? 0.f : GamC);
     });
     if (!alive) break;
     // Ob accumulates onto Gam * scale * QS
@@ -533,7 +538,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
         tmem_ld16(tm + lane + T_X + c0, x);
         lds16(Gam + c0, gm);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) x[i] = rres[i] - gm[i] * x[i];
+        for (int i = 0; i < 16; ++i) x[i] = stl ? rres[i] : rres[i] - gm[i] * x[i];
         st_row16_split(sm + SM_XE, sm + SM_XE_LO, j, c0, x);
       }
       alive = run_phase([&] {
@@ -601,7 +606,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       for (int i = 0; i < 16; ++i) {
         const int t = c0 + i;
         const float gg = plain ? 1.f : gv[i];
-        const float ov = fmaf(gg * gm[i] * p.scale, oa[i], ob[i]);
+        const float ov = stl ? ob[i] : fmaf(gg * gm[i] * p.scale, oa[i], ob[i]);
         if (p.f32out)
           ostg32[t * D + j] = ov;
         else

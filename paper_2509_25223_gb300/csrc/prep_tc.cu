@@ -179,6 +179,10 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
   constexpr float kLog2e = 1.4426950408889634f;
   const bool dec_res = p.mods & RDN_FLAG_DECAYED_RESIDUAL;
   const bool plain = p.mods & RDN_FLAG_PLAIN_COMBINE;
+  // the stateless correction R_t = r_t k_t^T: the auxiliary pass has no delta
+  // rule (identity T_gamma), its in-chunk product is diag(gamma_t q_t.k_t)
+  // (no decay), and the chunk-end R is the last valid token's k r^T (wR one-hot)
+  const bool stl = p.mods & RDN_FLAG_STATELESS_AUX;
 
   if (tid == 0) {
     mbar_init(bar, 1);
@@ -399,7 +403,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
             const float qk = p.scale * gv[c0 + u];
             const float dec = i <= t ? exp2f(ct2 - c2[u]) * qk : 0.f;
             mq[u] = i < t ? (plain ? exp2f(cq2 - c2[u]) * qk : dec) * bt[u] : 0.f;
-            m2[u] = gtt * dec * gm[u];
+            m2[u] = stl ? (i == t ? gtt * qk : 0.f) : gtt * dec * gm[u];
           }
           img_row16(img + IMG_APMQ, 16384, 64 + t, i0, mq);
           img_row16(img + IMG_M2, 8192, t, i0, m2);
@@ -426,7 +430,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
 #pragma unroll
       for (int c0 = 0; c0 < 32; c0 += 16) {
         float v[16];
-        if (rla) {
+        if (rla || (m && stl)) {
 #pragma unroll
           for (int u = 0; u < 16; ++u) v[u] = r == 32 * hf + c0 + u ? 1.f : 0.f;
         } else {
@@ -438,12 +442,15 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
     if (tid < C) {
       float *rec = p.ws + chunk * kRecFloats;
       const int t = tid;
+      int s_, h_, cc_;
+      rec_decode(p, (long long)chunk, s_, h_, cc_);
+      const int n_ = min(C, seq_span(p, s_, h_).len - cc_ * C);  // valid tokens
       const float cC = cum[C - 1];
       rec[OFF_VEC + V_GAM + t] = __expf(cum[t]);
       rec[OFF_VEC + V_GPREV + t] = __expf(cprev[t]);
       rec[OFF_VEC + V_ALPHA + t] = __expf(gg[t]);
       rec[OFF_VEC + V_WS + t] = bet[t] * __expf(cC - cum[t]);
-      rec[OFF_VEC + V_WR + t] = gam[t] * __expf(cC - cum[t]);
+      rec[OFF_VEC + V_WR + t] = stl ? (t == n_ - 1 ? 1.f : 0.f) : gam[t] * __expf(cC - cum[t]);
       if (t == 0) rec[OFF_VEC + V_GAMC] = __expf(cC);
     }
   }

@@ -72,13 +72,13 @@ def test_fwd_validation(fn):
     assert _status(fn, _fwd_args(flags=QKN, qk_eps=float("inf"))) == 1
     assert _status(fn, _fwd_args(flags=QKN, qk_eps=1e-12)) == 1
     assert "q is NULL" in lib.rdn_last_error().decode()
-    # fp32 results: bf16 inputs need the tensor-core path (Dk = 128, no
-    # stateless variant); fp32 inputs take the flag as a no-op (then the call
+    # fp32 results: bf16 inputs need the tensor-core path (Dk = 128); fp32
+    # inputs take the flag as a no-op (then the call
     # gets as far as the NULL pointer check)
     F32 = _abi.RDN_FLAG_F32_OUT
     assert _status(fn, _fwd_args(flags=F32, Dk=64, Dv=64)) == 2
     assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_TANH_RESIDUAL)) == 1
-    assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_STATELESS_AUX)) == 2
+    assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_STATELESS_AUX)) == 1
     assert _status(fn, _fwd_args(flags=F32)) == 1
     assert _status(fn, _fwd_args(flags=F32 | _abi.RDN_FLAG_DECAYED_RESIDUAL)) == 1
     assert _status(fn, _fwd_args(flags=F32, dtype=_abi.RDN_F32, Dk=64, Dv=64)) == 1
