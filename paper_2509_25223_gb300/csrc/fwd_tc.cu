@@ -72,8 +72,9 @@ constexpr uint32_t SM_XE_LO = 180224;  //   lo part
 constexpr uint32_t SM_W = 196608;      // (wS E)^T / (wR E2)^T, hi part
 constexpr uint32_t SM_W_LO = 212992;   //   lo part
 constexpr uint32_t SM_VEC = 229376;    // 7 x 64 fp32: Gam Gprev (unused) wS wR gamma, GamC
-constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;  // 4 mbarriers: MMA, slot A, slot B, drain
-constexpr uint32_t SM_SLOT = SM_BAR + 32;
+// 5 mbarriers: MMA, slot A, slot B, drain, tile copies
+constexpr uint32_t SM_BAR = SM_VEC + 7 * 64 * 4;
+constexpr uint32_t SM_SLOT = SM_BAR + 40;
 constexpr uint32_t SM_FLAG = SM_SLOT + 4;
 constexpr uint32_t SM_BYTES = SM_FLAG + 4;
 constexpr size_t kTcSmem = SM_BYTES;
@@ -130,8 +131,18 @@ __device__ __forceinline__ void mma_split3(uint32_t d, uint32_t a_hi, uint32_t a
 
 // kGeneric: the variant flags (FwdParams::mods) are read; the method's
 // instances have them folded away
+// Tensor maps (CUtensorMap, 64-byte aligned) over v, k, q as [tokens][H][D]
+// with a 64-token x 64-column box (make_tile_map); ok: they are valid.
+struct FwdMaps {
+  alignas(64) unsigned char v[128];
+  alignas(64) unsigned char k[128];
+  alignas(64) unsigned char q[128];
+  bool ok;
+};
+
 template <bool RDNV, bool kGeneric>
-__global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
+__global__ void __launch_bounds__(kTcThreads, 1)
+    fwd_tc_kernel(FwdParams p, const __grid_constant__ FwdMaps maps) {
   extern __shared__ __align__(1024) uint8_t sm[];
   const uint32_t sbase = smem_u32(sm);
   if (sbase & 1023u) {  // the swizzled tiles need a 1024-byte aligned base
@@ -144,6 +155,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + SM_BAR);
   uint64_t *barA = bar + 1, *barB = bar + 2;  // slot A / slot B bulk copies
   uint64_t *barD = bar + 3;  // the drain after a wait that gave up
+  uint64_t *barE = bar + 4;  // a whole chunk's V, K, Q tiles by tensor-map copies
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SM_SLOT);
   volatile int *flag = reinterpret_cast<volatile int *>(sm + SM_FLAG);
 
@@ -178,6 +190,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     mbar_init(barA, 1);
     mbar_init(barB, 1);
     mbar_init(barD, 1);
+    mbar_init(barE, 1);
     fence_mbar_init();
     *flag = 0;
   }
@@ -252,6 +265,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     fetch_v(0);
     fetch_kq(0);
   }
+  // Chunks between the first and the last are whole: with tensor maps thread 0
+  // brings their V (after step (e)) and K, Q (after step (g)) tiles by tiled
+  // bulk copies on one phase of barrier E, and no cp.async wait is needed for
+  // them.  The first chunk is fetched above and the last one, which may be
+  // ragged, by cp.async with zero fill.
+  const bool tma = maps.ok;
+  auto by_tma = [&](int cc) { return tma && cc > 0 && cc < NC - 1; };
+  uint32_t phE = 0;    // phases of barrier E waited for
+  bool pendE = false;  // (thread 0) a phase armed and not yet waited for
+  auto tma_v = [&](int cc) {  // (thread 0) arms barrier E for the chunk's three tiles
+    const int row = (int)(tok0 + (long long)cc * 64);
+    mbar_expect_tx(barE, 49152);
+    pendE = true;
+    for (int kb = 0; kb < 2; ++kb) tma_load_3d(sm + SM_V + kb * 8192, maps.v, 64 * kb, h, row, barE);
+  };
+  auto tma_kq = [&](int cc) {
+    const int row = (int)(tok0 + (long long)cc * 64);
+    for (int kb = 0; kb < 2; ++kb) {
+      tma_load_3d(sm + SM_KQ + kb * 16384, maps.k, 64 * kb, h, row, barE);
+      tma_load_3d(sm + SM_KQ + kb * 16384 + 8192, maps.q, 64 * kb, h, row, barE);
+    }
+  };
 
   // initial states -> TMEM (fp32) and bf16 A operands
   for (int c0 = g16; c0 < D; c0 += 64) {
@@ -360,8 +395,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     const int t0 = c * 64;
     const int n = min(64, T - t0);
     if (c + 1 < NC) prefetch_chunk(c + 1);
-    cp_async_wait_all();  // this chunk's V, K, Q tiles (fetched during the previous chunk)
-    __syncthreads();      // every thread is done with the previous chunk's tiles and vectors
+    // this chunk's V, K, Q tiles (fetched during the previous chunk)
+    if (by_tma(c)) {
+      if (!mbar_wait(barE, phE & 1u)) *flag = 1;
+      ++phE;
+      if (tid == 0) pendE = false;
+    } else {
+      cp_async_wait_all();
+    }
+    __syncthreads();  // every thread is done with the previous chunk's tiles and vectors
+    if (*flag) {
+      alive = false;
+      break;
+    }
 
     // ---- (a) chunk inputs -> shared memory (the chunk-start states for the
     // backward were stored by the previous chunk's updates)
@@ -528,7 +574,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }
     if (tid == 0 && p.sv_E) bulk_wait_read();  // the E^T tiles are rewritten next
     __syncthreads();
-    if (c + 1 < NC) fetch_v(c + 1);  // every thread is past its last read of V
+    if (c + 1 < NC) {  // every thread is past its last read of V
+      if (!by_tma(c + 1))
+        fetch_v(c + 1);
+      else if (tid == 0)
+        tma_v(c + 1);
+    }
 
     // ---- (f) X2 = r - Gam KR;  MMA6: E2^T = X2^T T_gamma^T (into D1[0,64))
     if (RDNV) {
@@ -588,7 +639,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
     }, nothing);
     if (!alive) break;
     if (tid == 0 && c + 1 < NC) load_slot(sm + SM_SLOTB, barB, rec_of(c + 1) + IMG_APMQ, 32768);
-    if (c + 1 < NC) fetch_kq(c + 1);  // K, Q are done with
+    if (c + 1 < NC) {  // K, Q are done with
+      if (!by_tma(c + 1))
+        fetch_kq(c + 1);
+      else if (tid == 0)
+        tma_kq(c + 1);
+    }
 
     // ---- (h) o = (Ob + diag(gamma) M2 E2) + gamma * Gam QR;  R (= Gam_C R + U2) -> RA
     // o is staged as a [t][j] tile in W's place (free after MMA8; bf16, or fp32
@@ -679,6 +735,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) fwd_tc_kernel(FwdParams p) {
       mbar_wait(barD, 0);
       if (pendA) mbar_wait(barA, phA);
       if (pendB) mbar_wait(barB, phB);
+      if (pendE) mbar_wait(barE, phE & 1u);
       bulk_wait_all();
     }
     cp_async_wait_all();
@@ -722,13 +779,17 @@ bool make_tile_map(void *map128, const void *base, int D, int H, long long rows)
 }
 
 cudaError_t launch_fwd_tc(const FwdParams &p, bool rdnv, cudaStream_t s) {
+  FwdMaps maps;
+  const long long rows = (long long)p.B * p.T;
+  maps.ok = make_tile_map(maps.v, p.v, D, p.H, rows) && make_tile_map(maps.k, p.k, D, p.H, rows) &&
+            make_tile_map(maps.q, p.q, D, p.H, rows);
   const bool generic = p.mods != 0;
   auto kern = rdnv ? (generic ? fwd_tc_kernel<true, true> : fwd_tc_kernel<true, false>)
                    : (generic ? fwd_tc_kernel<false, true> : fwd_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kTcSmem);
   if (e != cudaSuccess) return e;
-  RDN_LAUNCH("fwd_tc_scan", s, kern<<<p.nseq * p.H, kTcThreads, kTcSmem, s>>>(p));
+  RDN_LAUNCH("fwd_tc_scan", s, kern<<<p.nseq * p.H, kTcThreads, kTcSmem, s>>>(p, maps));
   return cudaGetLastError();
 }
 
