@@ -232,6 +232,60 @@ def qk_prologue_bwd(x, dy, eps=1e-12):
 QUANT = {"f64": 0, "f32": 1, "bf16": 2}
 
 
+def _bf16_tie_distance(y):
+    """|position of y between its two neighbouring bf16 values - 1/2|, in
+    units of that spacing (0 = exactly halfway, 1/2 = on a bf16 value)."""
+    a = np.abs(y)
+    e = np.floor(np.log2(np.maximum(a, np.finfo(np.float32).tiny)))
+    ulp = np.exp2(e - 7.0)  # 8 significant bits
+    f = a / ulp - np.floor(a / ulp)
+    return np.abs(f - 0.5)
+
+
+def qk_round_margin_condition(x, eps=1e-12, margin=2.0 ** -9, max_iter=64):
+    """Return (x_conditioned, n_moved): bf16 rows x [..., D] moved, one bf16
+    step at a time, so that every element of the fp64 prologue output y (as
+    qk_prologue computes it) is at least `margin` bf16 spacings away from a
+    rounding tie of bf16.  A library that holds y in bf16 after computing it
+    in fp32 (relative error well below 2^-17, i.e. 2^-9 of a bf16 spacing)
+    then rounds every y to the bf16 value that the fp64 y rounds to, so the
+    reference and the library see the same y.  In a row with an element too
+    close to a tie the element of largest SiLU(x) among those that are not
+    takes one bf16 step up (SiLU rises there with slope about 1, so the row's
+    norm, and with it every y of the row, moves by a fraction of a spacing;
+    stepping an element near a tie would move its own y by about one spacing
+    and keep it there); rows are revisited until none is left."""
+    x = _f64(x).copy()
+    D = x.shape[-1]
+    flat = x.reshape(-1, D)
+    moved = 0
+
+    def silu(rows):
+        return flat[rows] / (1.0 + np.exp(-flat[rows]))
+
+    def near(rows):
+        u = silu(rows)
+        n = np.sqrt((u * u).sum(-1, keepdims=True))
+        return _bf16_tie_distance(u / np.maximum(n, eps)) < margin
+
+    rows = np.arange(flat.shape[0])
+    rows = rows[near(rows).any(-1)]
+    for _ in range(max_iter):
+        if rows.size == 0:
+            break
+        j = np.where(near(rows), -np.inf, silu(rows)).argmax(-1)
+        v = flat[rows, j]
+        a = np.maximum(np.abs(v), np.finfo(np.float32).tiny)
+        # one bf16 step up: the spacing above v (below a power of two going
+        # down from a negative v it is half as large, a finer step, also fine)
+        flat[rows, j] = v + np.exp2(np.floor(np.log2(a)) - 7.0)
+        moved += rows.size
+        rows = rows[near(rows).any(-1)]
+    if rows.size:
+        raise RuntimeError(f"qk_round_margin_condition: {rows.size} rows left near a tie")
+    return flat.reshape(x.shape), moved
+
+
 def clip_margin_condition(variant, q, k, v, g, beta, gamma, c, S0=None, R0=None,
                           scale=1.0, margin=4e-3, quant="bf16", mods=0):
     """Return (v_conditioned, n_moved): v moved, in token order and in steps

@@ -103,3 +103,60 @@ def test_fwd_bwd_full_size_all_heads(variant):
         _check(test, name, d[name], ref[name], **extra)
     for name in ("dq", "dk", "dv"):
         _check(test, f"{name} (fp32 out)", d32[name], ref[name], **extra)
+
+
+@pytest.mark.parametrize("mode", ["tanh_residual", "stateless_aux", "qk_norm"])
+def test_fwd_bwd_full_size_modes(mode):
+    """The bench step (RDN, all 128 heads, the step's options) with one of
+    the tensor-core modes beyond the method: the tanh residual and the
+    stateless correction (variant flags, the oracle's mods bits), or the q, k
+    normalisation inside the library (q, k taken as raw x; the reference is
+    the oracle's prologue, rounded to bf16 as the library holds it, then its
+    recurrence, and dq, dk through the prologue's backward at x)."""
+    w = WORKLOADS["rdn_fwd_bwd_bf16_B8H16T4096D128"]
+    x = make_workload_inputs(w, device="cuda")
+    flags = {"tanh_residual": rdn.TANH_RESIDUAL, "stateless_aux": rdn.STATELESS_AUX}.get(mode, 0)
+    mods = {"tanh_residual": oracle.TANH, "stateless_aux": oracle.STATELESS}.get(mode, 0)
+    qkn = mode == "qk_norm"
+    if qkn:  # raw x moved off the bf16 rounding ties of y (tests/test_gpu_qk_norm.py)
+        for n in ("q", "k"):
+            xc, _ = oracle.qk_round_margin_condition(as64(x[n]), 1e-12)
+            x[n] = torch.from_numpy(xc).to(torch.bfloat16).cuda()
+    a = {n: as64(x[n]) for n in NAMES}
+    if qkn:
+        for n in ("q", "k"):
+            y = oracle.qk_prologue(a[n], 1e-12)
+            a[n] = as64(torch.from_numpy(y).to(torch.bfloat16))
+    v2, moved = oracle.clip_margin_condition(oracle.RDN, a["q"], a["k"], a["v"], a["g"],
+                                             a["beta"], a["gamma"], w.clip, None, None,
+                                             margin=MARGIN, quant="bf16", mods=mods)
+    x["v"] = torch.from_numpy(v2).to(torch.bfloat16).cuda()
+    a["v"] = as64(x["v"])
+    wsf = torch.empty(rdn.workspace_bytes("rdn_fwd", w.B, w.T, w.H, w.D, save_for_bwd=True,
+                                          variant_flags=flags, qk_norm=qkn),
+                      dtype=torch.uint8, device="cuda")
+    kw = dict(clip=w.clip, variant_flags=flags, qk_norm=qkn)
+    o, ST, RT, Sc, Rc = rdn.rdn_fwd(*(x[n] for n in NAMES), return_chunk_states=True,
+                                    workspace=wsf, save_for_bwd=True, **kw)
+    d = rdn.rdn_bwd(*(x[n] for n in NAMES), x["dO"], S_chunks=Sc, R_chunks=Rc,
+                    fwd_workspace=wsf, fwd_saved=True, **kw)
+    torch.cuda.synchronize()
+    assert rdn.device_status() == 0
+    oref, Sref, Rref = oracle.fwd(oracle.RDN, *(a[n] for n in NAMES), w.clip, None, None,
+                                  mods=mods)
+    ref = oracle.bwd(oracle.RDN, *(a[n] for n in NAMES), w.clip, None, None, as64(x["dO"]),
+                     mods=mods)
+    if qkn:
+        ref["dq"] = oracle.qk_prologue_bwd(as64(x["q"]), ref["dq"], 1e-12)
+        ref["dk"] = oracle.qk_prologue_bwd(as64(x["k"]), ref["dk"], 1e-12)
+    test = f"rdn fwd+bwd {w.name} {mode}"
+    extra = dict(conditioner_moved=moved, conditioner_margin=MARGIN)
+    _check(test, "o", o, oref, **extra)
+    _check(test, "ST", ST, Sref, **extra)
+    _check(test, "RT", RT, Rref, **extra)
+    for name in GRADS:
+        assert torch.isfinite(d[name].float()).all(), name
+        if mode == "stateless_aux" and name == "dR0":
+            assert float(d[name].abs().max()) == 0.0  # R0 enters nothing
+            continue
+        _check(test, name, d[name], ref[name], **extra)

@@ -6,9 +6,13 @@ q and k are raw projections x (normal draws, not normalised).  The library
 holds y in the input dtype (as a caller's own prologue pass would), so the
 reference rounds the oracle's fp64 y to that dtype before the recurrence,
 exactly as the other tests hand the oracle the bf16 q, k the kernels read;
-the backward's Jacobian is the oracle's, at the fp64 x.  The clip mask is
-made unique the usual way (v moved until every fp64 residual is a margin
-away from c), on the y the reference uses."""
+the backward's Jacobian is the oracle's, at the fp64 x.  The rounding of y
+to bf16 is a decision the two sides take in different precisions (fp32 in
+the library, fp64 in the oracle), so the raw rows are first conditioned
+(oracle.qk_round_margin_condition: x moved by bf16 steps) until every fp64 y
+is a margin away from a bf16 rounding tie; both then hold the same y.  The
+clip mask is made unique the usual way (v moved until every fp64 residual is
+a margin away from c), on the y the reference uses."""
 import numpy as np
 import pytest
 import torch
@@ -31,8 +35,11 @@ def _inputs(B, T, H, D, dtype, seed=0, zero_row=False):
                     device="cuda", state_std=0.1, seed=seed)
     gen = torch.Generator(device="cpu").manual_seed(seed + 100)
     td = x["q"].dtype
-    x["q"] = torch.randn(B, T, H, D, generator=gen).to(td).cuda()  # raw projections
-    x["k"] = torch.randn(B, T, H, D, generator=gen).to(td).cuda()
+    for n in ("q", "k"):  # raw projections, conditioned (bf16 y: see the module's text)
+        raw = torch.randn(B, T, H, D, generator=gen).to(td)
+        if td == torch.bfloat16:
+            raw = torch.from_numpy(oracle.qk_round_margin_condition(raw, EPS)[0]).to(td)
+        x[n] = raw.cuda()
     if zero_row:  # a row whose norm is below eps: y = u / eps = 0, du = dy / eps
         x["k"][0, 0, 0] = 0
         x["q"][0, T - 1, H - 1] = 0

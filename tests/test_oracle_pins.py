@@ -582,3 +582,31 @@ def test_tied_gate_gradient_matches_autograd(variant):
     d = oracle.bwd(variant, x["q"], x["k"], x["v"], x["g"], x["beta"], x["beta"], c, x["S0"],
                    x["R0"], x["dO"])
     np.testing.assert_allclose(d["dbeta"] + d["dgamma"], T_["beta"].grad.numpy(), atol=1e-11)
+
+
+def test_qk_round_margin_condition():
+    """The prologue-rounding conditioner: its rows are bf16 values, every fp64
+    y lands at least the margin away from a bf16 rounding tie, rows that were
+    clear are untouched, and y computed in fp32 (the library's precision,
+    with a plain sum of squares) then rounds to bf16 exactly like the fp64 y."""
+    import torch
+    rng = np.random.default_rng(3)
+    x = torch.from_numpy(rng.standard_normal((4096, 128))).to(torch.bfloat16).double().numpy()
+    x[7] = 0.0  # a row under the floor stays as it is (y = 0)
+    xc, moved = oracle.qk_round_margin_condition(x)
+    assert moved > 0
+    assert np.array_equal(torch.from_numpy(xc).to(torch.bfloat16).double().numpy(), xc)
+    y0 = oracle.qk_prologue(x)
+    clear = (oracle._bf16_tie_distance(y0) >= 2.0 ** -9).all(-1)
+    assert np.array_equal(xc[clear], x[clear]) and not clear.all()
+    y = oracle.qk_prologue(xc)
+    assert oracle._bf16_tie_distance(y).min() >= 2.0 ** -9
+    x32 = xc.astype(np.float32)
+    u32 = x32 / (np.float32(1.0) + np.exp(-x32))
+    y32 = u32 / np.maximum(np.sqrt((u32 * u32).sum(-1, keepdims=True, dtype=np.float32)),
+                           np.float32(1e-12))
+    assert torch.equal(torch.from_numpy(y).to(torch.bfloat16),
+                       torch.from_numpy(y32.astype(np.float64)).to(torch.bfloat16))
+    # the tie distance itself: a bf16 value is 1/2 from a tie, a midpoint 0
+    assert oracle._bf16_tie_distance(np.array([1.0, 1.0 + 2.0 ** -8, 3.0]))[[0, 2]].min() == 0.5
+    assert oracle._bf16_tie_distance(np.array([1.0 + 2.0 ** -8]))[0] == 0.0
