@@ -362,7 +362,8 @@ rdn_status_t rla_fwd_workspace_size(const rdn_fwd_args *args, size_t *bytes);
  * to "workspace" or "launch", the forward and backward entry points fail
  * with RDN_ERR_WORKSPACE or RDN_ERR_CUDA after validating their arguments,
  * before enqueueing anything; with "device_wait" the tensor-core forward
- * scan (bf16, Dk = 128) makes its first bounded wait give up, records
+ * scan (bf16, Dk = 128), and with "device_wait_bwd" the tensor-core
+ * backward chain, makes its first bounded wait give up, records
  * RDN_ERR_TIMEOUT here and drains its work in flight. */
 rdn_status_t rdn_device_status(rdn_stream_t stream, int *status);
 

@@ -283,6 +283,7 @@ int fault_injection() {
   if (!strcmp(e, "workspace")) return 1;
   if (!strcmp(e, "launch")) return 2;
   if (!strcmp(e, "device_wait")) return 3;
+  if (!strcmp(e, "device_wait_bwd")) return 4;
   return 0;
 }
 

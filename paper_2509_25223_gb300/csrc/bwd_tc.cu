@@ -136,11 +136,18 @@ __device__ __forceinline__ void mma_s3_kk(uint32_t d, uint32_t a_hi, uint32_t a_
   mma_tile(d, a_lo, 0, b_hi, 0, 4, idesc, true);
 }
 
-// Common per-CTA machinery: mbarriers (MMA, slot A, slot B), TMEM, phases.
+// Common per-CTA machinery: mbarriers (MMA, copies A, B, C, and D for the
+// drain), TMEM, phases.  Thread 0 counts the copy phases it arms on A, B, C
+// and the ones it has seen complete, so that a CTA whose bounded wait gave up
+// can wait (again with a limit) for every copy and MMA still in flight before
+// it releases its shared memory and TMEM (ctl_drain).
 struct Ctl {
-  uint64_t *bar, *barA, *barB, *barC;
+  uint64_t *bar, *barA, *barB, *barC, *barD;
   volatile int *flag;
   uint32_t phase, phA, phB;
+  uint32_t armA, armB, armC, seenA, seenB, seenC;  // (thread 0) copy phases on A, B, C
+  long long limit;             // the MMA waits' limit in cycles
+  bool skip;                   // (thread 0) the next phase skips its completion signal (tests)
 };
 
 __device__ __forceinline__ void ctl_init(Ctl &k, uint8_t *base, int tid) {
@@ -149,21 +156,67 @@ __device__ __forceinline__ void ctl_init(Ctl &k, uint8_t *base, int tid) {
   k.barB = k.bar + 2;
   k.barC = k.bar + 3;
   k.flag = reinterpret_cast<volatile int *>(base + 32);
+  k.barD = reinterpret_cast<uint64_t *>(base + 40);
   k.phase = k.phA = k.phB = 0;
+  k.armA = k.armB = k.armC = k.seenA = k.seenB = k.seenC = 0;
+  k.limit = 2000000000ll;
+  k.skip = false;
   if (tid == 0) {
     mbar_init(k.bar, 1);
     mbar_init(k.barA, 1);
     mbar_init(k.barB, 1);
     mbar_init(k.barC, 1);
+    mbar_init(k.barD, 1);
     fence_mbar_init();
     *k.flag = 0;
   }
 }
 
-__device__ __forceinline__ void load_slot(uint8_t *dst, uint64_t *bar, const void *src,
-                                          uint32_t bytes) {
-  mbar_expect_tx(bar, bytes);
-  bulk_g2s(dst, src, bytes, bar);
+// the barrier and counters of copy barrier W (0: A, 1: B, 2: C)
+template <int W>
+__device__ __forceinline__ uint64_t *ctl_bar(Ctl &k) {
+  return W == 0 ? k.barA : (W == 1 ? k.barB : k.barC);
+}
+template <int W>
+__device__ __forceinline__ uint32_t &ctl_armed(Ctl &k) {
+  return W == 0 ? k.armA : (W == 1 ? k.armB : k.armC);
+}
+template <int W>
+__device__ __forceinline__ uint32_t &ctl_seen(Ctl &k) {
+  return W == 0 ? k.seenA : (W == 1 ? k.seenB : k.seenC);
+}
+// (thread 0) arm a copy phase of barrier W for `bytes`
+template <int W>
+__device__ __forceinline__ void ctl_arm(Ctl &k, uint32_t bytes) {
+  mbar_expect_tx(ctl_bar<W>(k), bytes);
+  ++ctl_armed<W>(k);
+}
+// wait for a copy phase of barrier W (thread 0 counts it)
+template <int W>
+__device__ __forceinline__ bool ctl_wait(Ctl &k, uint32_t parity, int tid) {
+  const bool ok = mbar_wait(ctl_bar<W>(k), parity);
+  if (ok && tid == 0) ++ctl_seen<W>(k);
+  return ok;
+}
+template <int W>
+__device__ __forceinline__ void ctl_drain_copies(Ctl &k) {
+  for (; ctl_seen<W>(k) < ctl_armed<W>(k); ++ctl_seen<W>(k))
+    mbar_wait(ctl_bar<W>(k), ctl_seen<W>(k) & 1u);
+}
+// (thread 0, after a wait gave up) every MMA this thread issued (one commit
+// covers them) and every armed copy phase, with bounded waits
+__device__ __forceinline__ void ctl_drain(Ctl &k) {
+  mma_commit(k.barD);
+  mbar_wait(k.barD, 0);
+  ctl_drain_copies<0>(k);
+  ctl_drain_copies<1>(k);
+  ctl_drain_copies<2>(k);
+}
+
+template <int W>
+__device__ __forceinline__ void load_slot(Ctl &k, uint8_t *dst, const void *src, uint32_t bytes) {
+  ctl_arm<W>(k, bytes);
+  bulk_g2s(dst, src, bytes, ctl_bar<W>(k));
 }
 
 // One MMA phase: publish shared-memory writes, issue (thread 0), wait.
@@ -175,9 +228,10 @@ __device__ __forceinline__ bool phase_run(Ctl &k, int tid, F issue) {
   if (tid == 0) {
     fence_after_sync();
     if (!issue()) *k.flag = 1;
-    mma_commit(k.bar);
+    if (!k.skip) mma_commit(k.bar);
+    k.skip = false;
   }
-  const bool ok = mbar_wait(k.bar, k.phase);
+  const bool ok = mbar_wait(k.bar, k.phase, k.limit);
   k.phase ^= 1u;
   if (!ok) *k.flag = 1;
   __syncthreads();
@@ -195,10 +249,11 @@ __device__ __forceinline__ bool phase_run_with(Ctl &k, int tid, F issue, G durin
   if (tid == 0) {
     fence_after_sync();
     if (!issue()) *k.flag = 1;
-    mma_commit(k.bar);
+    if (!k.skip) mma_commit(k.bar);
+    k.skip = false;
   }
   during();
-  const bool ok = mbar_wait(k.bar, k.phase);
+  const bool ok = mbar_wait(k.bar, k.phase, k.limit);
   k.phase ^= 1u;
   if (!ok) *k.flag = 1;
   __syncthreads();
@@ -216,12 +271,13 @@ __device__ __forceinline__ void phase_issue(Ctl &k, int tid, F issue) {
   if (tid == 0) {
     fence_after_sync();
     if (!issue()) *k.flag = 1;
-    mma_commit(k.bar);
+    if (!k.skip) mma_commit(k.bar);
+    k.skip = false;
   }
 }
 // ... then wait for them (every thread).
 __device__ __forceinline__ bool phase_wait(Ctl &k) {
-  const bool ok = mbar_wait(k.bar, k.phase);
+  const bool ok = mbar_wait(k.bar, k.phase, k.limit);
   k.phase ^= 1u;
   if (!ok) *k.flag = 1;
   __syncthreads();
@@ -230,8 +286,9 @@ __device__ __forceinline__ bool phase_wait(Ctl &k) {
 }
 
 // thread 0: wait for a slot's bulk copy
-__device__ __forceinline__ bool slot_wait(uint64_t *bar, uint32_t &ph) {
-  const bool ok = mbar_wait(bar, ph);
+template <int W>
+__device__ __forceinline__ bool slot_wait(Ctl &k, uint32_t &ph) {
+  const bool ok = ctl_wait<W>(k, ph, 0);
   ph ^= 1u;
   return ok;
 }
@@ -283,8 +340,8 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
   ctl_init(K, sm + CTL, tid);
   if (warp == 0) tmem_alloc(slot, 512);
   if (tid == 0) {
-    load_slot(sm + SLOTA, K.barA, rec + IMG_TB, 16384);
-    load_slot(sm + SLOTB, K.barB, rec + IMG_APMQ, 32768);
+    load_slot<0>(K, sm + SLOTA, rec + IMG_TB, 16384);
+    load_slot<1>(K, sm + SLOTB, rec + IMG_APMQ, 32768);
   }
   if (tid < 64) {
     Gam[tid] = reinterpret_cast<const float *>(rec)[OFF_VEC + V_GAM + tid];
@@ -351,14 +408,14 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       put16s(sm + XE, sm + XE_LO, j, c0, x);
     }
     ok = phase_run(K, tid, [&] {
-      if (!slot_wait(K.barA, K.phA)) return false;
+      if (!slot_wait<0>(K, K.phA)) return false;
       mma_s3_kk(tm + T_X, sb + XE, sb + XE_LO, sb + SLOTA, sb + SLOTA + 8192, idesc_bf16(128, 64),
                  false);
       return true;
     });
   }
   if (ok) {
-    if (tid == 0) load_slot(sm + SLOTA, K.barA, rec + IMG_TG, 16384);
+    if (tid == 0) load_slot<0>(K, sm + SLOTA, rec + IMG_TG, 16384);
 #pragma unroll
     for (int c0 = 0; c0 < 64; c0 += 16) {
       float e[16];
@@ -366,7 +423,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       put16s(sm + XE, sm + XE_LO, j, c0, e);
     }
     ok = phase_run(K, tid, [&] {  // D1 += E Ap^T -> P (the Ap rows of the [Ap ; Mq] image)
-      if (!slot_wait(K.barB, K.phB)) return false;
+      if (!slot_wait<1>(K, K.phB)) return false;
       mma_s3_kk(tm + T_D1, sb + XE, sb + XE_LO, sb + SLOTB, sb + SLOTB + 16384,
                  idesc_bf16(128, 64), true);
       static_assert(XE_LO == XE + 16384, "contiguous");
@@ -400,7 +457,7 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
     }
     if (!tnh) P.mask[chunk * D + j] = m;
     ok = phase_run(K, tid, [&] {  // E2 = T_gamma X2
-      if (!slot_wait(K.barA, K.phA)) return false;
+      if (!slot_wait<0>(K, K.phA)) return false;
       mma_s3_kk(tm + T_X, sb + XE, sb + XE_LO, sb + SLOTA, sb + SLOTA + 8192, idesc_bf16(128, 64),
                  false);
       return true;
@@ -420,8 +477,9 @@ __global__ void __launch_bounds__(NT, 1) bwd_recompute_kernel(TcBwdParams P) {
       bulk_commit();
       bulk_wait_all();
     }
-  } else if (tid == 0 && p.err) {
-    atomicExch(p.err, RDN_ERR_TIMEOUT);
+  } else if (tid == 0) {
+    if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+    ctl_drain(K);  // no copy or MMA of this CTA outlives it
   }
   if (tid == 0) bulk_wait_all();
   fence_before_sync();
@@ -482,25 +540,29 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
 
   Ctl K;
   ctl_init(K, sm + CTL, tid);
+  if (p.inject == 2) {  // (a test: the first phase's signal is skipped, the wait gives up)
+    K.limit = 10000000ll;
+    K.skip = true;
+  }
   if (warp == 0) tmem_alloc(slot, 512);
   // slot loads: A holds diag(gamma) M2, then T_gamma, then T_beta; B holds
   // Mq (hi | lo), then Ap (hi | lo) -- each 8 KB half copied from the
   // [Ap ; Mq] image
   auto load_mq = [&](size_t ck) {
     const uint8_t *r = rec_bytes(p, ck);
-    mbar_expect_tx(K.barB, 16384);
+    ctl_arm<1>(K, 16384);
     bulk_g2s(sm + SLOTB, r + IMG_APMQ + 8192, 8192, K.barB);
     bulk_g2s(sm + SLOTB + 8192, r + IMG_APMQ + 16384 + 8192, 8192, K.barB);
   };
   auto load_ap = [&](size_t ck) {
     const uint8_t *r = rec_bytes(p, ck);
-    mbar_expect_tx(K.barB, 16384);
+    ctl_arm<1>(K, 16384);
     bulk_g2s(sm + SLOTB, r + IMG_APMQ, 8192, K.barB);
     bulk_g2s(sm + SLOTB + 8192, r + IMG_APMQ + 16384, 8192, K.barB);
   };
   if (tid == 0 && NC > 0) {  // (a packed sequence may be empty)
     const size_t last = (size_t)(sp.rbase + NC - 1);
-    load_slot(sm + SLOTA, K.barA, rec_bytes(p, last) + IMG_M2, 16384);
+    load_slot<0>(K, sm + SLOTA, rec_bytes(p, last) + IMG_M2, 16384);
     load_mq(last);
   }
   fence_before_sync();
@@ -679,8 +741,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     // dR, dS (TMEM) times Gam_C, onto which the products of phases B .. E accumulate
     // (the MMAs read their shared-memory tiles)
     ok = phase_run_with(K, tid, [&] {
-      if (!slot_wait(K.barA, K.phA)) return false;
-      if (!slot_wait(K.barB, K.phB)) return false;
+      if (!slot_wait<0>(K, K.phA)) return false;
+      if (!slot_wait<1>(K, K.phB)) return false;
       const uint32_t i64 = idesc_bf16(128, 64);
       mma_tile(tm + T_R1, sb + DRH, 16384, sb + KQ, 16384, 8, i64, false);
       mma_tile(tm + T_R1, sb + DRL, 16384, sb + KQ, 16384, 8, i64, true);
@@ -699,7 +761,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     });
     if (!ok) break;
     if (tid == 0) {
-      load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TG, 16384);
+      load_slot<0>(K, sm + SLOTA, rec_bytes(p, chunk) + IMG_TG, 16384);
       load_ap(chunk);
     }
     // dE2 = M2^T dOa + wR K dR ; dE (partial) = Mq^T dO + wS K dS ; dQR = Gam gamma dO
@@ -726,7 +788,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     }
     // ---- phase B: dX2 = T_gamma^T dE2 ; U_R = Q^T dQR
     ok = phase_run(K, tid, [&] {
-      if (!slot_wait(K.barA, K.phA)) return false;
+      if (!slot_wait<0>(K, K.phA)) return false;
       mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
                  idesc_bf16(128, 64), false);
       const uint32_t i128 = idesc_bf16(128, 128);
@@ -735,7 +797,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       return true;
     });
     if (!ok) break;
-    if (tid == 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk) + IMG_TB, 16384);
+    if (tid == 0) load_slot<0>(K, sm + SLOTA, rec_bytes(p, chunk) + IMG_TB, 16384);
     float dP[16];  // t in [g16, g16 + 16)
     {  // dX2 -> dP = -mask dX2, dKR = -Gam dX2; dX2 itself (fp32 [t][j]) for bwd_post,
        // staged in the free scratch tiles and bulk-copied
@@ -768,7 +830,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       static_assert(S0L == S0H + 16384, "contiguous");
       bulk_s2g(P.dX2buf + chunk * 64 * D, sm + S0H, 32768);  // (published by this barrier)
       bulk_commit();
-      if (!slot_wait(K.barB, K.phB)) return false;
+      if (!slot_wait<1>(K, K.phB)) return false;
       const uint32_t i128 = idesc_bf16(128, 128);
       mma_tile_kmn(tm + T_DR, sb + S2H, 0, sb + KQ, 16384, 4, i128, true);
       mma_tile_kmn(tm + T_DR, sb + S2L, 0, sb + KQ, 16384, 4, i128, true);
@@ -797,7 +859,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     }
     // ---- phase D: dX = T_beta^T dE ; U_S = Q^T dQS
     ok = phase_run(K, tid, [&] {
-      if (!slot_wait(K.barA, K.phA)) return false;
+      if (!slot_wait<0>(K, K.phA)) return false;
       mma_s3_kmn(tm + T_R3, sb + S0H, sb + S0L, sb + SLOTA, sb + SLOTA + 8192, 16384,
                  idesc_bf16(128, 64), false);
       const uint32_t i128 = idesc_bf16(128, 128);
@@ -806,7 +868,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       return true;
     });
     if (!ok) break;
-    if (tid == 0 && c > 0) load_slot(sm + SLOTA, K.barA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
+    if (tid == 0 && c > 0) load_slot<0>(K, sm + SLOTA, rec_bytes(p, chunk - 1) + IMG_M2, 16384);
     if (c > 0) {  // every thread is past its last read of this chunk's dO
       if (!tma)
         fetch_do(c - 1);
@@ -901,7 +963,8 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     }
   } else if (tid == 0) {
     if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
-    // no copy into this CTA's shared memory outlives it (bounded waits)
+    // no copy into this CTA's shared memory or MMA outlives it (bounded waits)
+    ctl_drain(K);
     for (; tma_seen < tma_arms; ++tma_seen) mbar_wait(K.barC, tma_seen & 1u);
   }
   cp_async_wait_all();
@@ -1012,14 +1075,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // until P2) and the K, Q tile.
   auto fetch_states = [&](size_t ck) {
     if (tid == 0) {
-      mbar_expect_tx(K.barA, 131072);
+      ctl_arm<0>(K, 131072);
       bulk_g2s(sm + SA, P.Sc + ck * D * D, 65536, K.barA);
       bulk_g2s(sm + SB, P.Rc + ck * D * D, 65536, K.barA);
     }
   };
   auto fetch_rest = [&](size_t ck) {
     if (tid == 0) {
-      mbar_expect_tx(K.barC, 65536);
+      ctl_arm<2>(K, 65536);
       bulk_g2s(sm + XH, P.dX2buf + ck * 64 * D, 32768, K.barC);
       bulk_g2s(sm + YH, P.dXbuf + ck * 64 * D, 32768, K.barC);
     }
@@ -1102,7 +1165,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const uint32_t i128 = idesc_bf16(128, 128), i64 = idesc_bf16(128, 64);
 
   cp_async_wait_all();  // K, Q tile (published by the barriers below)
-  if (!mbar_wait(K.barA, 0)) *K.flag = 1;  // phase_run below reports it to every thread
+  if (!ctl_wait<0>(K, 0, tid)) *K.flag = 1;  // phase_run below reports it to every thread
 #pragma unroll 1
   for (int s2 = 0; s2 < 2; ++s2) stage_to_image(s2 ? SB : SA);  // images of S0, R0
   // ---- P1: read-outs [K S0 | Q S0] and [K R0 | Q R0] (lanes j, columns t')
@@ -1129,7 +1192,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     wR[tid] = recf[OFF_VEC + V_WR + tid];
     gamv[tid] = tid < n ? p.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
   }
-  if (!mbar_wait(K.barC, 0)) *K.flag = 1;
+  if (!ctl_wait<2>(K, 0, tid)) *K.flag = 1;
   {
     const float *x2s = reinterpret_cast<const float *>(sm + XH);
     const float *xs = reinterpret_cast<const float *>(sm + YH);
@@ -1212,7 +1275,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     });
   }
   if (ok && tid == 0) {  // R0's image is done with: dR's image into its place
-    mbar_expect_tx(K.barB, 65536);
+    ctl_arm<1>(K, 65536);
     bulk_g2s(sm + SB, gimg + 32768, 32768, K.barB);
     bulk_g2s(sm + SB + 32768, gimg + 98304, 32768, K.barB);
   }
@@ -1246,15 +1309,15 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile_mnmn<true>(tm + T_DKQ, sb + SA + 32768, 16384, sb + XH, 32768, 8, i128, true);
       return true;
     }, [&] {
-      if (!mbar_wait(K.barB, it & 1u)) *K.flag = 1;  // dR's image
+      if (!ctl_wait<1>(K, it & 1u, tid)) *K.flag = 1;  // dR's image
       gdot = stl ? 0.f : dot_state(R0, SB);
     });
   }
   if (ok && tid == 0) {  // and dS's image into S0's; the E2^T, E^T images into the pair's
-    mbar_expect_tx(K.barA, 65536);
+    ctl_arm<0>(K, 65536);
     bulk_g2s(sm + SA, gimg, 32768, K.barA);
     bulk_g2s(sm + SA + 32768, gimg + 65536, 32768, K.barA);
-    mbar_expect_tx(K.barC, 65536);
+    ctl_arm<2>(K, 65536);
     bulk_g2s(sm + XH, P.E2buf + chunk * 32768, 32768, K.barC);  // hi at XH, lo at XL
     bulk_g2s(sm + YH, P.Ebuf + chunk * 32768, 32768, K.barC);   // hi at YH, lo at YL
   }
@@ -1274,8 +1337,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   };
   if (ok) {  // ---- P4: dR E2^T, dS E^T (scaled by wR, wS per token below); K dR, K dS read-outs;
              // meanwhile <dS, S0> and the dGamC reduction
-    if (!mbar_wait(K.barC, 1)) *K.flag = 1;  // the E images, for every thread
-    if (!mbar_wait(K.barA, 1)) *K.flag = 1;  // dS's image
+    if (!ctl_wait<2>(K, 1, tid)) *K.flag = 1;  // the E images, for every thread
+    if (!ctl_wait<0>(K, 1, tid)) *K.flag = 1;  // dS's image
     phase_issue(K, tid, [&] {
       mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XH, 16384, 8, i64, false);
       mma_tile_mnmn<true>(tm + T_U1, sb + SB, 16384, sb + XL, 16384, 8, i64, true);
@@ -1630,8 +1693,11 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
   }
   }  // chunks
-  if (!ok && tid == 0 && p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
-  cp_async_wait_all();  // no copy of this CTA outlives it (a fetch for a chunk not reached)
+  if (!ok && tid == 0) {
+    if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+    ctl_drain(K);  // no bulk copy or MMA of this CTA outlives it
+  }
+  cp_async_wait_all();  // (nor a cp.async of a chunk not reached)
   fence_before_sync();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, 512);

@@ -861,6 +861,7 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
   // a forward recomputed here keeps its o in fwd.dtype
   const bool grad_f32 = p.f.f32out != 0;
   p.f.f32out = 0;
+  p.f.inject = fault_injection() == 4 ? 2 : 0;
   const bool reuse = reuse_fwd_records(f, variant);
   p.f.ws = reuse ? (float *)f.workspace : (float *)ws;
   p.f.err = status_word();

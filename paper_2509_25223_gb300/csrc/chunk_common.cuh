@@ -126,7 +126,8 @@ struct FwdParams {
   long long nrec;  // record slots: B * H * NC, or a bound on H * (total chunks)
   unsigned mods;   // the variant flags (RDN_FLAG_VARIANTS bits of rdn_fwd_args.flags)
   int f32out;      // o stored in fp32 (RDN_FLAG_F32_OUT on the tensor-core forward)
-  int inject;      // 1: the tensor-core scan skips its first MMA completion signal (tests)
+  int inject;      // 1: the tensor-core scan, 2: the backward chain skips its first MMA
+                   // completion signal and waits ~5 ms for it (tests)
   // RDN_FLAG_QK_NORM: q and k above are then the normalised copies
   // SiLU(x) / max(||SiLU(x)||, qk_eps), written by the pass that makes the
   // chunk records (launch_t in chunk_fwd.cu), and qraw, kraw the caller's x

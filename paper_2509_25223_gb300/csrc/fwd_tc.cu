@@ -204,8 +204,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   bool pendA = false, pendB = false;      // (thread 0) a slot copy armed and not yet waited for
   // the waits on the MMAs: normally about a second; a test (p.inject) skips the
   // first phase's completion signal and waits about 5 ms for it instead
-  const long long mma_limit = p.inject ? 10000000ll : 2000000000ll;
-  bool skip_commit = p.inject != 0;
+  const long long mma_limit = p.inject == 1 ? 10000000ll : 2000000000ll;
+  bool skip_commit = p.inject == 1;
   // S - bf16(S) as a second bf16 image (rows j), so that the read-outs K S,
   // Q S use S to ~16 bits.  RLA's state is not contracted by a delta term and
   // its prediction S k is a large sum the residual v - S k cancels against;

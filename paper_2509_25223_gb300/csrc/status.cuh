@@ -16,7 +16,8 @@ int *status_word();
 // fail as a launch would, both after argument validation and before
 // anything is enqueued; "device_wait" (3) makes the tensor-core forward scan
 // skip one MMA completion signal, so that its bounded wait gives up
-// (RDN_ERR_TIMEOUT in the status word) and the kernel drains and exits.
+// (RDN_ERR_TIMEOUT in the status word) and the kernel drains and exits;
+// "device_wait_bwd" (4) does the same in the tensor-core backward chain.
 // 0 when unset or unrecognised.  Defined in api.cu.
 int fault_injection();
 }  // namespace rdn

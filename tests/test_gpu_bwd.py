@@ -289,3 +289,37 @@ def test_bwd_f32_out(variant, T):
             assert_close(d32[name], ref[name], "bf16", f"{name} (fp32 out)")
         else:
             assert torch.equal(d32[name], d[name]), name
+
+
+@pytest.mark.parametrize("variant", ["rdn", "rla"])
+@pytest.mark.parametrize("saved", [False, True])
+def test_bounded_wait_gives_up_cleanly_bwd(variant, saved, monkeypatch):
+    """A device wait of the backward that runs out: with
+    RDN_FAULT_INJECT=device_wait_bwd the backward chain skips its first MMA
+    completion signal, every thread's bounded wait on it gives up (~5 ms), and
+    the CTA records RDN_ERR_TIMEOUT, waits for its MMAs and copies still in
+    flight, frees its TMEM and returns (bwd_post then runs on what it has).
+    The context stays usable: the next backward matches the oracle and leaves
+    the status word at 0."""
+    x = make_inputs(2, 200, 2, 128, dtype="bf16", nonzero_state=True, with_grad_out=True,
+                    device="cuda", state_std=0.1)
+    ov = oracle.RDN if variant == "rdn" else oracle.RLA
+    _condition(x, 1.0, "bf16", variant=ov)
+    kw = {}
+    if saved:  # the forward's chunk states, records and saved intermediates
+        wsf = torch.empty(rdn.workspace_bytes(f"{variant}_fwd", 2, 200, 2, 128, save_for_bwd=True),
+                          dtype=torch.uint8, device="cuda")
+        fwd = rdn.rdn_fwd if variant == "rdn" else rdn.rla_fwd
+        _, _, _, Sc, Rc = fwd(*(x[n] for n in NAMES), clip=1.0, S0=x["S0"], R0=x["R0"],
+                              return_chunk_states=True, workspace=wsf, save_for_bwd=True)
+        kw = dict(S_chunks=Sc, R_chunks=Rc, fwd_workspace=wsf, fwd_saved=True)
+    rdn.device_status()  # whatever an earlier test left
+    monkeypatch.setenv("RDN_FAULT_INJECT", "device_wait_bwd")
+    _gpu(x, 1.0, variant=variant, **kw)
+    assert rdn.device_status() == 4  # RDN_ERR_TIMEOUT
+    monkeypatch.delenv("RDN_FAULT_INJECT")
+    d = _gpu(x, 1.0, variant=variant, **kw)
+    assert rdn.device_status() == 0
+    ref = _ref(x, 1.0, variant=ov)
+    for name in GRADS:
+        assert_close(d[name], ref[name], "bf16", name)
