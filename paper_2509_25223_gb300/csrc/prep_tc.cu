@@ -41,8 +41,8 @@ constexpr uint32_t WS = TG + 64 * LDT * 4;   // product scratch, 2 x [32][LDW]
 // cum, cprev, beta, gamma, g, and cum, cprev times log2(e) (7 x 64)
 constexpr uint32_t VEC = WS + 2 * 32 * LDW * 4;
 static_assert(TB % 16 == 0 && TG % 16 == 0 && WS % 16 == 0 && VEC % 16 == 0, "16-byte rows");
-constexpr uint32_t CTL = VEC + 7 * 64 * 4;   // mbarrier, flag
-constexpr uint32_t SLOT = CTL + 16;          // TMEM base
+constexpr uint32_t CTL = VEC + 7 * 64 * 4;   // mbarrier, flag, drain mbarrier
+constexpr uint32_t SLOT = CTL + 24;          // TMEM base
 constexpr size_t SMEM = SLOT + 16;
 static_assert(2 * (SMEM + 1024) <= 233472, "two CTAs per SM");
 }  // namespace pp
@@ -167,6 +167,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
   float *Wsc = reinterpret_cast<float *>(sm + WS);
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + CTL);
   volatile int *flag = reinterpret_cast<volatile int *>(sm + CTL + 8);
+  uint64_t *barD = reinterpret_cast<uint64_t *>(sm + CTL + 16);  // the drain after a wait gave up
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H = p.H;
@@ -186,6 +187,7 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
 
   if (tid == 0) {
     mbar_init(bar, 1);
+    mbar_init(barD, 1);
     fence_mbar_init();
     *flag = 0;
   }
@@ -454,7 +456,11 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
       if (t == 0) rec[OFF_VEC + V_GAMC] = __expf(cC);
     }
   }
-  if (!ok && tid == 0 && p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+  if (!ok && tid == 0) {
+    if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
+    mma_commit(barD);  // the Gram product still in flight, before TMEM is freed
+    mbar_wait(barD, 0);
+  }
   cp_async_wait_all();  // no copy of this CTA outlives it (a fetch for a chunk not reached)
   fence_before_sync();
   __syncthreads();
