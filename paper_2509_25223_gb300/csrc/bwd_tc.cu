@@ -1104,6 +1104,32 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     fetch_states(blockIdx.x);
     fetch_rest(blockIdx.x);
   }
+  // the previous chunk's dq, dk from TMEM to HBM (row = its first token row *
+  // H + h; n = its valid tokens, -1 = none pending)
+  long long dkq_row = 0;
+  int dkq_n = -1;
+  auto store_dkq = [&]() {
+    __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
+    const uint32_t tl = (uint32_t)((warp & 3) * 32) << 16;
+    float a[16], d2[16], qv[16];
+    tmem_ld16x2(tm + tl + T_DKQ + tb, a, tm + tl + T_D2 + tb, d2);
+    tmem_ld16(tm + tl + T_DKQ + 64 + tb, qv);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int t = tb + i;
+      if (t < dkq_n) {
+        const size_t off = (size_t)(dkq_row + (long long)t * H) * D + j;
+        if (P.f32qk) {
+          ((float *)P.dk)[off] = a[i] + scale * d2[i];
+          ((float *)P.dq)[off] = scale * qv[i];
+        } else {
+          dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
+          dq[off] = __float2bfloat16_rn(scale * qv[i]);
+        }
+      }
+    }
+    dkq_n = -1;
+  };
   bool ok = true;
   uint32_t it = 0;  // chunks done by this CTA: the parity of barrier B
   for (size_t chunk = blockIdx.x; chunk < nct && ok; chunk += gridDim.x, ++it) {
@@ -1177,7 +1203,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     mma_tile<true>(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
     return true;
   });
-  // while P1 runs: this thread's dO, the gate vectors, dX2 and dX from their staging
+  // while P1 runs: the previous chunk's dq, dk; this thread's dO, the gate
+  // vectors, dX2 and dX from their staging
+  if (dkq_n >= 0) store_dkq();
   const unsigned long long m = tnh ? 0ull : P.mask[chunk * D + j] >> tb;
   const uint16_t *drow = reinterpret_cast<const uint16_t *>(P.mask) + (chunk * D + j) * 64 + tb;
 #pragma unroll
@@ -1671,28 +1699,13 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       P.dbeta[off] = o_dbeta;
       P.dgamma[off] = o_dgamma;
     }
-    __nv_bfloat16 *dk = (__nv_bfloat16 *)P.dk, *dq = (__nv_bfloat16 *)P.dq;
-    {
-      float a[16], d2[16], qv[16];
-      tmem_ld16x2(tm + tm_lane + T_DKQ + tb, a, tm + tm_lane + T_D2 + tb, d2);
-      tmem_ld16(tm + tm_lane + T_DKQ + 64 + tb, qv);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int t = tb + i;
-        if (t < n) {
-          const size_t off = ((size_t)(tok0 + t0 + t) * H + h) * D + j;
-          if (P.f32qk) {
-            ((float *)P.dk)[off] = a[i] + scale * d2[i];
-            ((float *)P.dq)[off] = scale * qv[i];
-          } else {
-            dk[off] = __float2bfloat16_rn(a[i] + scale * d2[i]);
-            dq[off] = __float2bfloat16_rn(scale * qv[i]);
-          }
-        }
-      }
-    }
+    // dq, dk of this chunk: read out and stored during the next chunk's P1
+    // (T_DKQ, T_D2 keep them until its P2), or after the last chunk
+    dkq_row = (tok0 + t0) * H + h;
+    dkq_n = n;
   }
   }  // chunks
+  if (ok && dkq_n >= 0) store_dkq();
   if (!ok && tid == 0) {
     if (p.err) atomicExch(p.err, RDN_ERR_TIMEOUT);
     ctl_drain(K);  // no bulk copy or MMA of this CTA outlives it
