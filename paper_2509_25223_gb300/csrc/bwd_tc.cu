@@ -1419,13 +1419,20 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
   //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
-  //   and the Gram matrices [K ; Q] K^T
-  // images: E2 at XH (hi | lo), E at YH (hi | lo); dX at SB; the pairs at SA
-  // (X atom hi SA, lo SA + 16 KB; Y atom hi SA + 32 KB, lo SA + 48 KB)
+  //   and the Gram matrices [K ; Q] K^T, all in one phase
+  // images: E2 at XH (hi | lo), E at YH (hi | lo); dX at SB, dP at SB + 32 KB
+  // (dR's image is done with); the pair [dO ; dX2] at SA (dO atom hi SA, lo
+  // SA + 16 KB; dX2 atom hi SA + 32 KB, lo SA + 48 KB), and [dO ; dP] as the
+  // dO atom and the dP atom 96 KB after it
   if (ok) {
+    float y[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) y[i] = dp_of(i);
     put_tok(xv, SB, SB + 16384);
-    put_tok(dov, SA, SA + 16384);  // [dO ; dX2]: gamma_t enters in the element-wise pass
+    put_tok(y, SB + 32768, SB + 49152);
+    put_tok(dov, SA, SA + 16384);  // gamma_t enters in the element-wise pass
     put_tok(x2v, SA + 32768, SA + 49152);
+    static_assert(SB + 32768 - SA == 98304, "the [dO ; dP] atoms");
     ok = phase_run(K, tid, [&] {
       mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XH, 16384, 8, i64, false);
       mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XL, 16384, 8, i64, true);
@@ -1435,18 +1442,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile_mnmn<true>(tm + T_G3, sb + SB, 32768, sb + YL, 16384, 8, i64, true);
       mma_tile_mnmn<true>(tm + T_G3, sb + SB + 16384, 32768, sb + YH, 16384, 8, i64, true);
       mma_tile<true>(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
-      return true;
-    });
-  }
-  if (ok) {
-    float y[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) y[i] = dp_of(i);
-    put_tok(y, SA + 32768, SA + 49152);  // [dO ; dP]: the dO atom is still in place
-    ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 32768, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 32768, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA + 16384, 32768, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 98304, sb + YH, 16384, 8, i64, false);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 98304, sb + YL, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_G2, sb + SA + 16384, 98304, sb + YH, 16384, 8, i64, true);
       return true;
     });
   }
@@ -1516,7 +1514,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const float ct = cum[t], cpt = cprev[t];
       const float gt = gam[t];
       float rowc = 0.f, rowp = 0.f, dgo = 0.f;
-#pragma unroll 1
+#pragma unroll 2
       for (int ii = 0; ii < 8; ++ii) {
         const int i = 8 * q8 + ii, e = t * LDC + i;
         float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
