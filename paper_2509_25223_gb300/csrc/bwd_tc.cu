@@ -45,9 +45,8 @@ constexpr int D = 128;
 constexpr int NT = 128;   // threads per CTA of bwd_recompute
 constexpr int NTC = 512;  // threads per CTA of bwd_chain (4 warps per TMEM lane quadrant)
 
-// Per-chunk row-sum slots in the backward workspace (floats): read-out part of
-// d gamma, dwS, dwR (C each).  Used as scratch by bwd_post, whose shared
-// memory is full.
+// bwd_post's per-token sums kept in shared memory from where they are formed
+// to the gate pass (floats): the read-out part of d gamma, dwS, dwR (C each).
 struct A8 {
   static constexpr int V_DGAM_OUT = 0, V_DWS = C, V_DWR = 2 * C;
   static constexpr int FLOATS = 3 * C;
@@ -60,7 +59,6 @@ struct TcBwdParams {
   const float *Sc, *Rc;  // chunk-start states [B,H,NC,D,D]
   void *dv;
   float *dS0, *dR0;
-  float *acc;            // per-chunk records
   uint8_t *Ebuf, *E2buf; // [B*H*NC][32 KB]: images of E^T, E2^T (rows j, columns t; hi | lo)
   float *dX2buf, *dXbuf; // [B*H*NC][64][128]
   uint8_t *gimg;         // [B*H*NC][128 KB]: gradients w.r.t. each chunk's end states as
@@ -996,8 +994,9 @@ constexpr uint32_t SA = 0, SB = 65536;  // state images: hi 2 x 16 KB | lo 2 x 1
 constexpr uint32_t XH = 131072, XL = 147456, YH = 163840, YL = 180224;  // [j][t] atoms
 constexpr uint32_t KQ = 196608;         // K rows 0..63, Q rows 64..127, 2 x 16 KB
 constexpr uint32_t VEC = 229376;        // Gam Gprev wS wR gamma dGam dGprev (7 x 64), dGamC
-constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // 16 warps x 16 floats
-constexpr uint32_t CTL = RED + 16 * 16 * 4;
+constexpr uint32_t RED = VEC + 7 * 64 * 4 + 16;  // the 16 warps' <dS, S0> + <dR, R0> parts
+constexpr uint32_t PARK = RED + 16 * 4;           // per-token sums kept to the gate pass (A8)
+constexpr uint32_t CTL = PARK + A8::FLOATS * 4;
 constexpr uint32_t SLOT = CTL + 48;
 constexpr size_t SMEM = SLOT + 16;
 static_assert(SMEM <= 232448, "shared memory");
@@ -1013,21 +1012,20 @@ constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the re
 }  // namespace po
 
 // Sums over the 128 value columns: thread (j, qd) holds v[t - 16 qd] for the
-// tokens t of its quarter; out[t] for t in [0, 64).  Warp 4 qd + w covers
-// columns [32 w, 32 w + 32); after the warp's transposed reduction lane 2 i
-// holds its sum for token 16 qd + i.
-__device__ __forceinline__ void cta_row_sum512(const float (&v)[16], float *red, float *out,
-                                               int tid) {
+// tokens t of its quarter.  Warp 4 qd + w covers columns [32 w, 32 w + 32);
+// after the warp's transposed reduction lane 2 i holds its sum for token
+// 16 qd + i.  Each warp leaves its part (16 floats) at part[16 warp, +16), so
+// that several sums share the barriers ...
+__device__ __forceinline__ void warp_row_part(const float (&v)[16], float *part, int tid) {
   const float o = warp_transpose_reduce16(v);
   const int warp = tid >> 5, lane = tid & 31;
-  if (!(lane & 1)) red[warp * 16 + (lane >> 1)] = o;
-  __syncthreads();
-  if (tid < 64) {
-    const int g = tid >> 4, i = tid & 15;
-    out[tid] = red[(4 * g) * 16 + i] + red[(4 * g + 1) * 16 + i] + red[(4 * g + 2) * 16 + i] +
-               red[(4 * g + 3) * 16 + i];
-  }
-  __syncthreads();
+  if (!(lane & 1)) part[warp * 16 + (lane >> 1)] = o;
+}
+// ... and, after a barrier, token t's total is the sum of its four warps' parts.
+__device__ __forceinline__ float row_total(const float *part, int t) {
+  const int g = t >> 4, i = t & 15;
+  return part[(4 * g) * 16 + i] + part[(4 * g + 1) * 16 + i] + part[(4 * g + 2) * 16 + i] +
+         part[(4 * g + 3) * 16 + i];
 }
 
 template <bool kGeneric>  // (as bwd_chain_kernel's)
@@ -1044,6 +1042,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   float *Gam = vec, *Gprev = vec + 64, *wS = vec + 128, *wR = vec + 192, *gamv = vec + 256;
   float *dGamS = vec + 320, *dGprevS = vec + 384, *dGamC = vec + 448;
   float *red = reinterpret_cast<float *>(sm + RED);
+  float *park = reinterpret_cast<float *>(sm + PARK);
   uint32_t *slot = reinterpret_cast<uint32_t *>(sm + SLOT);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int j = tid & 127, qd = tid >> 7, tb = 16 * qd;
@@ -1140,7 +1139,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   const long long tok0 = sp.tok0;
   const int t0 = c * 64, n = min(64, sp.len - t0);
   const float *recf = p.ws + chunk * kRecFloats;
-  float *acc = P.acc + chunk * A8::FLOATS;
   const float *S0 = P.Sc + chunk * D * D, *R0 = P.Rc + chunk * D * D;
   const uint8_t *gimg = P.gimg + chunk * 131072;  // dS hi | dR hi | dS lo | dR lo
   // this thread's tokens of dX2, dX (from the staging) and dO: read after P1 is
@@ -1236,6 +1234,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     return ((m >> i) & 1ull) ? -x2v[i] : 0.f;
   };
   if (ok) {  // per-token gate terms: dGam, dGprev, and <dR,R0> + <dS,S0>
+    // the three sums' warp parts go where dX2 was staged (read into x2v above)
+    float *part = reinterpret_cast<float *>(sm + XH);
     float rv[16];
     {
       float qs[16], qr[16];
@@ -1248,10 +1248,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       lds16(Gam + tb, rv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = plain ? 0.f : scale * rv[i] * dov[i] * qr[i];
-      cta_row_sum512(rv, red, dGamS, tid);
-      // parked in the record's slot (shared memory is full); the same thread reads it back
-      if (tid < 64) acc[A8::V_DGAM_OUT + tid] = dGamS[tid];
-      __syncthreads();
+      warp_row_part(rv, part, tid);
       lds16(gamv + tb, rv);
 #pragma unroll
       for (int i = 0; i < 16; ++i)  // (plain combine: Gprev Q S0 and no gamma_t)
@@ -1273,7 +1270,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) rv[i] += dp_of(i) * ks[i];
       }
-      cta_row_sum512(rv, red, dGamS, tid);
+      warp_row_part(rv, part + 256, tid);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = dec_res ? 0.f : dp_of(i) * ks[i];
       if (plain) {  // the base read-out's gate is Gprev
@@ -1283,7 +1280,17 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
         for (int i = 0; i < 16; ++i) rv[i] += scale * dov[i] * qs[i];
       }
     }
-    cta_row_sum512(rv, red, dGprevS, tid);
+    warp_row_part(rv, part + 512, tid);
+    __syncthreads();
+    if (tid < 192) {
+      const int w = tid >> 6, t = tid & 63;
+      const float tot = row_total(part + 256 * w, t);
+      if (w == 0)
+        park[A8::V_DGAM_OUT + t] = tot;
+      else
+        (w == 1 ? dGamS : dGprevS)[t] = tot;
+    }
+    __syncthreads();  // (P2's operands go where the parts are)
     // ---- P2: dK, dQ += R0 [dKR ; dQR]^T, dKR = -Gam dX2, dQR = Gam gamma dO
     float x[16], y[16];
     lds16(Gam + tb, x);
@@ -1385,13 +1392,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 #pragma unroll
     for (int off = 16; off; off >>= 1) gdot += __shfl_xor_sync(0xffffffffu, gdot, off);
     if (lane == 0) red[warp] = gdot;
-    __syncthreads();
-    if (tid == 0) {
+    ok = phase_wait(K);  // (its barrier publishes the parts)
+    if (ok && tid == 0) {
       float s = 0.f;
       for (int w = 0; w < NTP / 32; ++w) s += red[w];
       *dGamC = s;
     }
-    ok = phase_wait(K);
   }
   if (ok) {
     // dK += diag(wR) E2 dR^T + diag(wS) E dS^T  (lanes i, columns t of this half)
@@ -1405,7 +1411,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       for (int i = 0; i < 16; ++i) a[i] = fmaf(wr[i], u1[i], fmaf(ws[i], u2[i], a[i]));
       tmem_st16(tm + tm_lane + T_DKQ + tb, a);
     }
-    // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]
+    // dwR_t = sum_j (K dR)[t,j] E2[t,j], dwS_t = sum_j (K dS)[t,j] E[t,j]; the
+    // warp parts where dS's image was
+    float *part = reinterpret_cast<float *>(sm + SA);
 #pragma unroll 1
     for (int w = 0; w < 2; ++w) {
       float ev[16], rv[16];
@@ -1413,9 +1421,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       tmem_ld16(tm + tm_lane + (w == 0 ? T_KDR : T_KDS) + tb, rv);
 #pragma unroll
       for (int i = 0; i < 16; ++i) rv[i] = (w == 0 && stl) ? 0.f : rv[i] * ev[i];
-      // parked in the record's slots (shared memory is full); read in the gate pass
-      cta_row_sum512(rv, red, acc + (w == 0 ? A8::V_DWR : A8::V_DWS), tid);
+      warp_row_part(rv, part + 256 * w, tid);
     }
+    __syncthreads();
+    if (tid < 128) {  // read in the gate pass
+      const int w = tid >> 6, t = tid & 63;
+      park[(w == 0 ? A8::V_DWR : A8::V_DWS) + t] = row_total(part + 256 * w, t);
+    }
+    __syncthreads();  // (P5's operands go where the parts are)
   }
   // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
   //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
@@ -1424,7 +1437,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
   // (dR's image is done with); the pair [dO ; dX2] at SA (dO atom hi SA, lo
   // SA + 16 KB; dX2 atom hi SA + 32 KB, lo SA + 48 KB), and [dO ; dP] as the
   // dO atom and the dP atom 96 KB after it
+  // token tid's g and beta for the element-wise pass, loaded while P5 runs
+  float g_t = 0.f, beta_t = 0.f;
   if (ok) {
+    if (tid < n) {
+      const size_t off = (size_t)(tok0 + t0 + tid) * H + h;
+      g_t = p.g[off];
+      beta_t = p.beta[off];
+    }
     float y[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) y[i] = dp_of(i);
@@ -1447,6 +1467,12 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       mma_tile_mnmn<true>(tm + T_G2, sb + SA + 16384, 98304, sb + YH, 16384, 8, i64, true);
       return true;
     });
+  }
+  // the next chunk's states into L2 while the element-wise pass and P7 run
+  // (their copies into shared memory start once P7's MMAs are done)
+  if (ok && tid == 0 && next < nct) {
+    prefetch_l2_bulk(P.Sc + next * D * D, 65536);
+    prefetch_l2_bulk(P.Rc + next * D * D, 65536);
   }
   // ---- element-wise pass over (t, i): the gradients of the chunk matrices'
   // entries turned into gradients of K K^T, Q K^T and of the gates
@@ -1479,16 +1505,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       }
     }
     if (tid < 64) {
-      const int t = tid;
-      float gv = 0.f, bv = 0.f;
-      if (t < n) {
-        const size_t off = (size_t)(tok0 + t0 + t) * H + h;
-        gv = p.g[off];
-        bv = p.beta[off];
-      }
-      gg[t] = gv;
-      bet[t] = bv;
-      gam[t] = gamv[t];
+      gg[tid] = g_t;
+      bet[tid] = beta_t;
+      gam[tid] = gamv[tid];
     }
     __syncthreads();
     if (warp == 0) {  // in-chunk cumulative log-decay
@@ -1514,7 +1533,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const float ct = cum[t], cpt = cprev[t];
       const float gt = gam[t];
       float rowc = 0.f, rowp = 0.f, dgo = 0.f;
-#pragma unroll 2
+#pragma unroll
       for (int ii = 0; ii < 8; ++ii) {
         const int i = 8 * q8 + ii, e = t * LDC + i;
         float dkk = 0.f, dqk = 0.f, cg = 0.f, cb = 0.f, cm = 0.f;
@@ -1606,9 +1625,9 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       }
       const float cC = cum[63];
       const float eC = __expf(cC - cum[i]);
-      const float dwS = acc[A8::V_DWS + i], dwR = acc[A8::V_DWR + i];
+      const float dwS = park[A8::V_DWS + i], dwR = park[A8::V_DWR + i];
       dbet[i] = s5[3] + dwS * eC;
-      dgam[i] = s5[4] + s5[5] + acc[A8::V_DGAM_OUT + i] + dwR * eC;
+      dgam[i] = s5[4] + s5[5] + park[A8::V_DGAM_OUT + i] + dwR * eC;
       dcum[i] = s5[0] - s5[2] - (dwS * bet[i] + dwR * gam[i]) * eC + dGamS[i] * __expf(cum[i]);
       dcprev[i] = s5[1] + dGprevS[i] * __expf(cprev[i]);
     }
@@ -1617,7 +1636,7 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const float cC = cum[63];
       float s = 0.f;
       for (int t = lane; t < 64; t += 32)
-        s += (acc[A8::V_DWS + t] * bet[t] + acc[A8::V_DWR + t] * gam[t]) *
+        s += (park[A8::V_DWS + t] * bet[t] + park[A8::V_DWR + t] * gam[t]) *
              __expf(cC - cum[t]);
 #pragma unroll
       for (int off = 16; off; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
@@ -1716,7 +1735,6 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
 
 }  // namespace
 
-size_t bwd_tc_acc_bytes(long long nrec) { return sizeof(float) * (size_t)nrec * A8::FLOATS; }
 
 size_t bwd_tc_extra_bytes(long long nrec, bool deriv) {
   const size_t nct = (size_t)nrec;
@@ -1726,8 +1744,8 @@ size_t bwd_tc_extra_bytes(long long nrec, bool deriv) {
 
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
-                          float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s) {
+                          float *dbeta, float *dgamma, float *dS0, float *dR0, char *extra,
+                          bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s) {
   TcBwdParams P;
   P.rla = rla;
   P.f32g = grad_f32;
@@ -1746,7 +1764,6 @@ cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, 
   P.dv = dv;
   P.dS0 = dS0;
   P.dR0 = dR0;
-  P.acc = acc;
   const size_t nct = (size_t)f.nrec;  // record slots (packed sequences: a bound)
   float *x = reinterpret_cast<float *>(extra);
   P.Ebuf = reinterpret_cast<uint8_t *>(x);

@@ -785,7 +785,8 @@ BwdLayout layout(const rdn_bwd_args &a, int variant) {
   BwdLayout l;
   // the forward's records are read from its workspace when it is passed
   l.prep = reuse_fwd_records(f, variant) ? 0 : align256(sizeof(float) * nrec * kRecFloats);
-  l.acc = tc ? align256(bwd_tc_acc_bytes(nrec)) : align256(sizeof(float) * nrec * accf);
+  // (the tensor-core kernels keep their per-chunk sums in shared memory)
+  l.acc = tc ? 0 : align256(sizeof(float) * nrec * accf);
   const bool need_states = f.S_chunks == nullptr;
   l.states = need_states ? align256(sizeof(float) * nrec * f.Dk * f.Dv) : 0;  // each of S, R
   const size_t esz = f.dtype == RDN_BF16 ? 2 : 4;
@@ -917,10 +918,9 @@ static cudaError_t launch_bwd_impl(const rdn_bwd_args &a, int variant, cudaStrea
     p.gq32 = (float *)(ws + l.prep + l.acc + 2 * l.states + l.o + l.tc + l.qk);
     p.gk32 = p.gq32 + (size_t)f.B * f.T * f.H * f.Dk;
   }
-  if (tc) {  // the accumulator words it reads are written by its own kernels
-    // (with the normalisation: dq, dk into the fp32 copies, as fp32 results)
+  if (tc) {  // (with the normalisation: dq, dk into the fp32 copies, as fp32 results)
     e = launch_bwd_tc(p.f, a.dO, a.dST, a.dRT, p.Sc, p.Rc, p.gq32 ? p.gq32 : a.dq,
-                      p.gk32 ? p.gk32 : a.dk, a.dv, a.dg, a.dbeta, a.dgamma, a.dS0, a.dR0, p.acc,
+                      p.gk32 ? p.gk32 : a.dk, a.dv, a.dg, a.dbeta, a.dgamma, a.dS0, a.dR0,
                       ws + l.prep + l.acc + 2 * l.states + l.o, !rdnv, grad_f32,
                       p.gq32 != nullptr, s);
   } else {

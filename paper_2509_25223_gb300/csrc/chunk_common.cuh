@@ -274,11 +274,10 @@ cudaError_t launch_prep(const FwdParams &p, int DK, bool rdnv, bool bf16, bool i
 // Tensor-core backward (bwd_tc.cu): recompute, chain and post kernels.
 cudaError_t launch_prep_tc(const FwdParams &p, bool rla, cudaStream_t s);
 size_t bwd_tc_extra_bytes(long long nrec, bool deriv);  // (deriv: the tanh residual's)
-size_t bwd_tc_acc_bytes(long long nrec);
 cudaError_t launch_bwd_tc(const FwdParams &f, const void *dO, const float *dST, const float *dRT,
                           const float *Sc, const float *Rc, void *dq, void *dk, void *dv, float *dg,
-                          float *dbeta, float *dgamma, float *dS0, float *dR0, float *acc,
-                          char *extra, bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s);
+                          float *dbeta, float *dgamma, float *dS0, float *dR0, char *extra,
+                          bool rla, bool grad_f32, bool dqk_f32, cudaStream_t s);
 
 // Launch the forward's prep kernel (per-chunk records into p.ws) and/or its
 // scan kernel (outputs, optional chunk-start states).
