@@ -700,9 +700,13 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
     const size_t chunk = (size_t)(sp.rbase + c);
     const int t0 = c * 64, n = min(64, T - t0);
     __syncthreads();
-    if (tid == 0) {  // gradients w.r.t. this chunk's end states, for bwd_post: the tile images
+    if (tid == 0) {  // gradients w.r.t. this chunk's end states, for bwd_post: the tile
+      // images, as two groups: the hi tiles (rewritten after phase A), then the
+      // lo tiles (rewritten after phase B)
       static_assert(DRH == DSH + 32768 && DSL == DRH + 32768 && DRL == DSL + 32768, "contiguous");
-      bulk_s2g(P.gimg + chunk * 131072, sm + DSH, 131072);
+      bulk_s2g(P.gimg + chunk * 131072, sm + DSH, 65536);
+      bulk_commit();
+      bulk_s2g(P.gimg + chunk * 131072 + 65536, sm + DSL, 65536);
       bulk_commit();
     }
     if (tid < 64) {
@@ -751,7 +755,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       mma_tile_mnmn(tm + T_R3, sb + DOT, 8192, sb + SLOTA + 8192, 16384, 4, i64, true);
       mma_tile_mnmn(tm + T_R4, sb + DOT, 8192, sb + SLOTB, 16384, 4, i64, false);
       mma_tile_mnmn(tm + T_R4, sb + DOT, 8192, sb + SLOTB + 8192, 16384, 4, i64, true);
-      bulk_wait_read();  // the tiles become scratch after this phase
+      bulk_wait_read_all_but_last();  // the hi tiles become scratch after this phase
       return true;
     }, [&] {
       scale_grad(T_DR, stl ? 0.f : GamC);
@@ -792,6 +796,7 @@ __global__ void __launch_bounds__(NTC, 1) bwd_chain_kernel(const __grid_constant
       const uint32_t i128 = idesc_bf16(128, 128);
       mma_tile_kmn(tm + T_DR, sb + S1H, 0, sb + KQ + 8192, 16384, 4, i128, true);
       mma_tile_kmn(tm + T_DR, sb + S1L, 0, sb + KQ + 8192, 16384, 4, i128, true);
+      bulk_wait_read();  // and the lo tiles after this one
       return true;
     });
     if (!ok) break;
