@@ -1013,7 +1013,9 @@ static_assert((F_VEC + 9 * 64 + 6 * 8 * 64) * 4 <= (int)XH, "finish scratch");
 // TMEM columns
 constexpr uint32_t T_KS = 0, T_KR = 128, T_DKQ = 256, T_D2 = 384;
 constexpr uint32_t T_KDR = 0, T_KDS = 64, T_U1 = 128, T_U2 = 192;  // P4, after the read-outs
-constexpr uint32_t T_G1 = 0, T_G2 = 64, T_G3 = 128, T_GR = 192;  // after the read-outs
+// P5 (after the read-outs and P4): two 128-column products and the Gram one
+// (past the dK, dQ accumulators)
+constexpr uint32_t T_P5A = 0, T_P5B = 128, T_GR = 448;
 }  // namespace po
 
 // Sums over the 128 value columns: thread (j, qd) holds v[t - 16 qd] for the
@@ -1206,22 +1208,34 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     mma_tile<true>(t_ + T_KR, sb + SB + 32768, 16384, sb + KQ, 16384, 8, i128, true);
     return true;
   });
-  // while P1 runs: the previous chunk's dq, dk; this thread's dO, the gate
-  // vectors, dX2 and dX from their staging
-  if (dkq_n >= 0) store_dkq();
+  // while P1 runs: this thread's dO and the gate vectors (loads first, their
+  // latency under the stores), the previous chunk's dq, dk, then dX2 and dX
+  // from their staging
   const unsigned long long m = tnh ? 0ull : P.mask[chunk * D + j] >> tb;
   const uint16_t *drow = reinterpret_cast<const uint16_t *>(P.mask) + (chunk * D + j) * 64 + tb;
+  __nv_bfloat16 dob[16];
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const int t = tb + i;
-    dov[i] = t < n ? __bfloat162float(dOp[((size_t)(tok0 + t0 + t) * H + h) * D + j]) : 0.f;
+    dob[i] = t < n ? dOp[((size_t)(tok0 + t0 + t) * H + h) * D + j] : __float2bfloat16(0.f);
   }
+  float gvv[5];
   if (tid < 64) {
-    Gam[tid] = recf[OFF_VEC + V_GAM + tid];
-    Gprev[tid] = recf[OFF_VEC + V_GPREV + tid];
-    wS[tid] = recf[OFF_VEC + V_WS + tid];
-    wR[tid] = recf[OFF_VEC + V_WR + tid];
-    gamv[tid] = tid < n ? p.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
+    gvv[0] = recf[OFF_VEC + V_GAM + tid];
+    gvv[1] = recf[OFF_VEC + V_GPREV + tid];
+    gvv[2] = recf[OFF_VEC + V_WS + tid];
+    gvv[3] = recf[OFF_VEC + V_WR + tid];
+    gvv[4] = tid < n ? p.gamma[(size_t)(tok0 + t0 + tid) * H + h] : 0.f;
+  }
+  if (dkq_n >= 0) store_dkq();
+#pragma unroll
+  for (int i = 0; i < 16; ++i) dov[i] = __bfloat162float(dob[i]);
+  if (tid < 64) {
+    Gam[tid] = gvv[0];
+    Gprev[tid] = gvv[1];
+    wS[tid] = gvv[2];
+    wR[tid] = gvv[3];
+    gamv[tid] = gvv[4];
   }
   if (!ctl_wait<2>(K, 0, tid)) *K.flag = 1;
   {
@@ -1435,13 +1449,14 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     }
     __syncthreads();  // (P5's operands go where the parts are)
   }
-  // ---- P5: C x C gradients (lanes t' of the stacked pair, columns s)
-  //   G1 = [dO ; dX2] E2^T   G3 = [dX ; -] E^T   G2 = [dO ; dP] E^T
-  //   and the Gram matrices [K ; Q] K^T, all in one phase
-  // images: E2 at XH (hi | lo), E at YH (hi | lo); dX at SB, dP at SB + 32 KB
-  // (dR's image is done with); the pair [dO ; dX2] at SA (dO atom hi SA, lo
-  // SA + 16 KB; dX2 atom hi SA + 32 KB, lo SA + 48 KB), and [dO ; dP] as the
-  // dO atom and the dP atom 96 KB after it
+  // ---- P5: C x C gradients (lanes t' of a stacked pair, columns s of [E2 ; E])
+  //   [dO ; dX2] [E2 ; E]^T -> dO E2^T | dO E^T ; dX2 E2^T | (unused)
+  //   [dX ; dP] [E2 ; E]^T  -> (unused) | dX E^T ; (unused) | dP E^T
+  //   and the Gram matrices [K ; Q] K^T, all in one phase: 128-column
+  //   products take about the issue time of 64-column ones
+  // images: E2 at XH (hi | lo), E at YH (hi | lo), 32 KB apart; the pair
+  // [dO ; dX2] at SA (dO atom hi SA, lo SA + 16 KB; dX2 atom hi SA + 32 KB, lo
+  // SA + 48 KB) and [dX ; dP] at SB the same way (dR's image is done with)
   // token tid's g and beta for the element-wise pass, loaded while P5 runs
   float g_t = 0.f, beta_t = 0.f;
   if (ok) {
@@ -1457,19 +1472,15 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     put_tok(y, SB + 32768, SB + 49152);
     put_tok(dov, SA, SA + 16384);  // gamma_t enters in the element-wise pass
     put_tok(x2v, SA + 32768, SA + 49152);
-    static_assert(SB + 32768 - SA == 98304, "the [dO ; dP] atoms");
+    static_assert(YH - XH == 32768 && YL - XL == 32768, "the [E2 ; E] atoms");
     ok = phase_run(K, tid, [&] {
-      mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XH, 16384, 8, i64, false);
-      mma_tile_mnmn<true>(tm + T_G1, sb + SA, 32768, sb + XL, 16384, 8, i64, true);
-      mma_tile_mnmn<true>(tm + T_G1, sb + SA + 16384, 32768, sb + XH, 16384, 8, i64, true);
-      // the second M atom of [dX ; -] is any valid tile: lanes 64..127 are unused
-      mma_tile_mnmn<true>(tm + T_G3, sb + SB, 32768, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn<true>(tm + T_G3, sb + SB, 32768, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn<true>(tm + T_G3, sb + SB + 16384, 32768, sb + YH, 16384, 8, i64, true);
+      mma_tile_mnmn<true>(tm + T_P5A, sb + SA, 32768, sb + XH, 32768, 8, i128, false);
+      mma_tile_mnmn<true>(tm + T_P5A, sb + SA, 32768, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_P5A, sb + SA + 16384, 32768, sb + XH, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_P5B, sb + SB, 32768, sb + XH, 32768, 8, i128, false);
+      mma_tile_mnmn<true>(tm + T_P5B, sb + SB, 32768, sb + XL, 32768, 8, i128, true);
+      mma_tile_mnmn<true>(tm + T_P5B, sb + SB + 16384, 32768, sb + XH, 32768, 8, i128, true);
       mma_tile<true>(tm + T_GR, sb + KQ, 16384, sb + KQ, 16384, 8, i64, false);
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 98304, sb + YH, 16384, 8, i64, false);
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA, 98304, sb + YL, 16384, 8, i64, true);
-      mma_tile_mnmn<true>(tm + T_G2, sb + SA + 16384, 98304, sb + YH, 16384, 8, i64, true);
       return true;
     });
   }
@@ -1491,8 +1502,10 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
       const int r = j & 63;
       {
         float g1[16], g2[16], g3[16], gr[16];
-        tmem_ld16x2(tm + tm_lane + T_G1 + tb, g1, tm + tm_lane + T_G2 + tb, g2);
-        tmem_ld16x2(tm + tm_lane + T_G3 + tb, g3, tm + tm_lane + T_GR + tb, gr);
+        // g1: dO E2^T (rows t < 64) | dX2 E2^T; g2: dO E^T | dP E^T; g3: dX E^T
+        tmem_ld16x2(tm + tm_lane + T_P5A + tb, g1,
+                    tm + tm_lane + (j < 64 ? T_P5A : T_P5B) + 64 + tb, g2);
+        tmem_ld16x2(tm + tm_lane + T_P5B + 64 + tb, g3, tm + tm_lane + T_GR + tb, gr);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int e = r * LDC + tb + i;
