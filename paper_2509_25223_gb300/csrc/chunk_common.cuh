@@ -167,6 +167,14 @@ __device__ __forceinline__ long long total_records(const FwdParams &p) {
 // record r -> (sequence s, head h, chunk c); r < total_records(p)
 __device__ __forceinline__ void rec_decode(const FwdParams &p, long long r, int &s, int &h, int &c) {
   if (!p.seq) {
+    if (r <= 0x7fffffffll) {  // (32-bit divisions: a 64-bit one is a long software routine)
+      const unsigned ru = (unsigned)r, nc = (unsigned)p.NC, hn = (unsigned)p.H;
+      const unsigned bh = ru / nc;
+      c = (int)(ru - bh * nc);
+      s = (int)(bh / hn);
+      h = (int)(bh - (unsigned)s * hn);
+      return;
+    }
     const long long bh = r / p.NC;
     c = (int)(r - bh * p.NC);
     s = (int)(bh / p.H);
@@ -180,8 +188,8 @@ __device__ __forceinline__ void rec_decode(const FwdParams &p, long long r, int 
   }
   s = lo;
   const int nc = (int)((p.seq[2 * s + 2] - p.seq[2 * s] + C - 1) / C);
-  const long long off = r - p.seq[2 * s + 1] * p.H;
-  h = (int)(off / nc);
+  const long long off = r - p.seq[2 * s + 1] * p.H;  // < H * nc
+  h = (int)((unsigned)off / (unsigned)nc);
   c = (int)(off - (long long)h * nc);
 }
 

@@ -67,27 +67,28 @@ __device__ __forceinline__ void img_row16(uint8_t *hi, uint32_t lo_off, int r, i
 // T = (I + A)^-1 for a strictly lower 64 x 64 A, by 128 threads (g = thread
 // index in the group); W is 32 x LDW scratch.  The caller synchronises the
 // block between the stages (0: diagonal blocks; 1, 2: the 16-row blocks; 3, 4:
-// the 32-row block), all groups of the block running the same stage.
+// the 32-row block), all groups of the block running the same stage.  The
+// 16 x 16 blocks above the diagonal are never written: the caller zeroes them
+// once.
 __device__ __forceinline__ void inv64_stage(int stage, const float *A, float *Tm, float *W, int g) {
   if (stage == 0) {
     // diagonal 16 x 16 blocks: thread (block, column) forward-substitutes its
-    // column; the blocks above the diagonal are zero
+    // column, x[r] = delta(r, col) - sum_{m < r} A[r][m] x[m], the terms added
+    // in the order of m; the updates of the rows below m are independent, so
+    // they are made as soon as x[m] is final (a 16-step chain instead of 120)
     if (g < 64) {
       const int b0 = (g >> 4) * 16, col = g & 15;
       float x[16];
 #pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        float s = (r == col) ? 1.f : 0.f;
+      for (int r = 0; r < 16; ++r) x[r] = (r == col) ? 1.f : 0.f;
 #pragma unroll
-        for (int m = 0; m < r; ++m) s = fmaf(-A[(b0 + r) * LDA + b0 + m], x[m], s);
-        x[r] = (r < col) ? 0.f : s;
+      for (int m = 0; m < 16; ++m) {
+        if (m < col) x[m] = 0.f;  // (above the diagonal)
+#pragma unroll
+        for (int r = m + 1; r < 16; ++r) x[r] = fmaf(-A[(b0 + r) * LDA + b0 + m], x[m], x[r]);
       }
 #pragma unroll
       for (int r = 0; r < 16; ++r) Tm[(b0 + r) * LDT + b0 + col] = x[r];
-    }
-    for (int e = g; e < 64 * 64; e += 128) {
-      const int r = e >> 6, c = e & 63;
-      if ((c >> 4) > (r >> 4)) Tm[r * LDT + c] = 0.f;
     }
   } else if (stage <= 2) {
     // 16-row blocks (i, j) = (1, 0) and (3, 2): W = A_ij T_jj, then
@@ -282,6 +283,11 @@ __global__ void __launch_bounds__(NTH, 2) prep_tc_kernel(FwdParams p, bool rla) 
       *reinterpret_cast<uint4 *>(dst) = w;
     }
   };
+  // the inverses' 16 x 16 blocks above the diagonal: zero throughout
+  for (int e = tid; e < 2 * 64 * 64; e += NTH) {
+    const int m = e >> 12, r = (e >> 6) & 63, c = e & 63;
+    if ((c >> 4) > (r >> 4)) (m ? Tg : Tb)[r * LDT + c] = 0.f;
+  }
   Gates gt{0.f, 0.f, 0.f};
   if (blockIdx.x < nct) {
     fetch_kq(blockIdx.x);
