@@ -678,17 +678,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       st_row16(sm + SM_RA, 16384, j, g16, r0);
       st_row16(sm + SM_RA, 16384, j, g16 + 64, r1);
     }
+    // the state's lo part below goes over the E2^T tiles: their bulk store to
+    // the saved E2 must have read them
+    if (p.sv_E2 && tid == 0) bulk_wait_read();
+    __syncthreads();  // the o tile, and the E2^T tiles
     {  // the updated state's lo part, for the next chunk's read-outs
-      if (p.sv_E2) {  // (over the E2^T tiles: their bulk store to the saved E2 must be done)
-        if (tid == 0) bulk_wait_read();
-        __syncthreads();
-      }
       float s0[16], s1[16];
       tmem_ld16x2(tm + lane + T_S + g16, s0, tm + lane + T_S + g16 + 64, s1);
       store_state_lo(g16, s0);
       store_state_lo(g16 + 64, s1);
     }
-    __syncthreads();  // the o tile
     if (p.f32out) {
       float *of = (float *)p.o;
       for (int e = tid; e < 64 * 32; e += kTcThreads) {
