@@ -1485,7 +1485,8 @@ __global__ void __launch_bounds__(po::NTP, 1) bwd_post_kernel(TcBwdParams P) {
     });
   }
   // the next chunk's states into L2 while the element-wise pass and P7 run
-  // (their copies into shared memory start once P7's MMAs are done)
+  // (their copies into shared memory start once the element-wise pass is done
+  // with the region, while P7 runs)
   if (ok && tid == 0 && next < nct) {
     prefetch_l2_bulk(P.Sc + next * D * D, 65536);
     prefetch_l2_bulk(P.Rc + next * D * D, 65536);
