@@ -84,17 +84,27 @@ def _peaks():
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
-    """nvidia-smi sampling of SM clock and throttle reasons during a region."""
+    """nvidia-smi sampling of SM clock and throttle reasons during a region:
+    samples every 50 ms with their timestamps; the summary keeps those that
+    fall inside the region marked by begin() / end() (host wall clock)."""
 
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    PERIOD_MS = 50
 
     def __init__(self, gpu_index, enabled=True):
         self.gpu = gpu_index
         self.enabled = enabled
         self.proc = None
         self.path = None
+        self.t0 = self.t1 = None
+
+    def begin(self):
+        self.t0 = time.time()
+
+    def end(self):
+        self.t1 = time.time()
 
     def __enter__(self):
         if not self.enabled:
@@ -104,7 +114,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.PERIOD_MS)],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
@@ -125,13 +135,10 @@ class ClockSampler:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["not sampled (--profile)"]}
         if self.proc is None or not self.path:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        rows = []
         with open(self.path) as f:
-            for ln in f:
-                parts = [p.strip() for p in ln.split(",")]
-                if len(parts) >= 9:
-                    rows.append(parts)
+            lines = f.readlines()
         os.unlink(self.path)
+        rows, where = clock_rows_in_region(lines, self.t0, self.t1)
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
         sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
@@ -144,9 +151,36 @@ class ClockSampler:
                     reasons.add(nm)
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
-                "samples": len(rows),
+                "samples": len(rows), "sampled": where,
+                "region_ms": (None if self.t0 is None or self.t1 is None
+                              else round(1e3 * (self.t1 - self.t0), 1)),
                 "power_w_max": max((float(r[3]) for r in rows
                                     if r[3].replace(".", "").isdigit()), default=None)}
+
+
+def clock_rows_in_region(lines, t0, t1):
+    """The nvidia-smi CSV rows (timestamp first) whose time falls in [t0, t1]
+    (host epoch seconds); if none does (a region shorter than the sampling
+    period), the first row after t0.  Returns (rows, "in region" | "first
+    after start" | "all")."""
+    import datetime
+    rows = []
+    for ln in lines:
+        parts = [p.strip() for p in ln.split(",")]
+        if len(parts) < 9:
+            continue
+        try:
+            ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            ts = None
+        rows.append((ts, parts))
+    if t0 is None or t1 is None or any(ts is None for ts, _ in rows):
+        return [r for _, r in rows], "all"
+    inside = [r for ts, r in rows if t0 <= ts <= t1]
+    if inside:
+        return inside, "in region"
+    after = [r for ts, r in rows if ts > t0]
+    return after[:1], "first after start"
 
 
 # ------------------------------------------------------------- distributed
@@ -477,11 +511,13 @@ def run_ours(args):
     with ClockSampler(local, enabled=not args.profile) as clk:
         with rdn.LaunchTimer() as lt:
             torch.cuda.synchronize()
+            clk.begin()
             e0.record(stream)
             for _ in range(args.steps):
                 step(x)
             e1.record(stream)
             torch.cuda.synchronize()
+            clk.end()
     barrier(dist)
     local_ms = e0.elapsed_time(e1)
     tokens_per_step = B * T
@@ -871,7 +907,9 @@ def run_ours(args):
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    # (default: 60 timed steps for this arm, ~0.2 s, so that the 50 ms clock
+    # samples fall inside the timed region; 10 oracle steps for the reference)
+    ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--decode-steps", type=int, default=1000)
@@ -890,6 +928,8 @@ def main(argv=None):
     ap.add_argument("--B", type=int, default=0, help="override B (profiling captures only)")
     ap.add_argument("--T", type=int, default=0, help="override T (profiling captures only)")
     args = ap.parse_args(argv)
+    if args.steps is None:
+        args.steps = 60 if args.impl == "ours" else 10
     if args.profile:
         args.no_decode = args.no_rla = args.no_prologue = args.no_varlen = True
         args.no_variants = args.no_forward = args.no_cpu_baseline = True
